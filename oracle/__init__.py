@@ -1,0 +1,207 @@
+"""fp64 CPU oracle of the GBLA layer-core forward.
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import this package.  It shares no code
+with the CUDA library in ``paper_2606_07317_gb300``; neither imports the other.
+
+The arithmetic lives in ``gbla_oracle.c`` (plain C, double precision), which
+follows Sec. 2 (bidirectional linear attention, Eq. bla) and Sec. 2.1 (GBLA:
+Conv1D, key gating, gated RMSNorm) of the paper.  This module only compiles
+it with gcc and marshals numpy arrays into it.
+
+Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
+against library routines, closed forms, the quadratic (L x L) form and
+invariants.  The paper's own unstated choices (phi, eps, conv tap order, the
+norm weight's shape) are readings, listed in the C file's header.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "gbla_oracle.c")
+_OUT_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_OUT_DIR, "liboracle.so")
+
+NO_CONV = 1  # identity Conv1D (ablation "W/o Conv1D")
+NO_GATE = 2  # uniform key gate (ablation "W/o Key gating")
+NO_NORM = 4  # no gated RMSNorm (ablation "W/o Gated RMSNorm")
+BLA = NO_CONV | NO_GATE | NO_NORM  # all add-ons off: Eq. bla
+
+RMS_EPS = 1e-6  # RMSNorm epsilon (the paper leaves it unstated; fixed reading)
+CONV_W = 4      # Conv1D kernel size used in the paper's experiments
+
+_lock = threading.Lock()
+_lib = None
+
+_dp = ctypes.POINTER(ctypes.c_double)
+
+
+def build(src: str = _SRC, out: str = _LIB_PATH, extra_flags=()) -> str:
+    """Compile the oracle into a shared library with gcc and return its path.
+
+    -ffp-contract=off keeps the double arithmetic identical on x86 and Arm.
+    """
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fPIC", "-shared",
+           *extra_flags, src, "-o", tmp, "-lm", "-lpthread"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
+def _declare(lib):
+    lib.oracle_phi.restype = ctypes.c_double
+    lib.oracle_phi.argtypes = [ctypes.c_double]
+    lib.oracle_silu.restype = ctypes.c_double
+    lib.oracle_silu.argtypes = [ctypes.c_double]
+    lib.oracle_conv1d.restype = None
+    lib.oracle_conv1d.argtypes = [_dp, ctypes.c_long, ctypes.c_int, ctypes.c_long,
+                                  _dp, ctypes.c_int, _dp]
+    lib.oracle_softmax.restype = None
+    lib.oracle_softmax.argtypes = [_dp, ctypes.c_long, ctypes.c_long, _dp]
+    lib.oracle_gated_rmsnorm_row.restype = None
+    lib.oracle_gated_rmsnorm_row.argtypes = [_dp, _dp, _dp, ctypes.c_int,
+                                             ctypes.c_double, _dp]
+    head_common = [_dp, _dp, _dp, _dp, _dp, ctypes.c_long, ctypes.c_long,
+                   ctypes.c_long, ctypes.c_int, _dp, _dp, _dp, ctypes.c_int, _dp,
+                   ctypes.c_double, ctypes.c_int, _dp]
+    lib.oracle_gbla_head.restype = ctypes.c_int
+    lib.oracle_gbla_head.argtypes = head_common + [_dp] * 7
+    lib.oracle_gbla_head_quadratic.restype = ctypes.c_int
+    lib.oracle_gbla_head_quadratic.argtypes = head_common + [_dp]
+    lib.oracle_gbla_forward.restype = ctypes.c_int
+    lib.oracle_gbla_forward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
+                                        ctypes.POINTER(ctypes.c_int32),
+                                        ctypes.c_long, ctypes.c_long, ctypes.c_long,
+                                        ctypes.c_int, ctypes.c_int, ctypes.c_double,
+                                        ctypes.c_int, ctypes.c_int, _dp]
+    return lib
+
+
+def load(path: str | None = None):
+    """Load (building first if needed) the oracle library."""
+    global _lib
+    with _lock:
+        if path is not None:
+            return _declare(ctypes.CDLL(path))
+        if _lib is None:
+            if (not os.path.exists(_LIB_PATH)
+                    or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC)):
+                build()
+            _lib = _declare(ctypes.CDLL(_LIB_PATH))
+        return _lib
+
+
+def _f64(x) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+
+
+def _ptr(a: np.ndarray | None):
+    if a is None:
+        return None
+    return a.ctypes.data_as(_dp)
+
+
+def phi(x: float, lib=None) -> float:
+    return (lib or load()).oracle_phi(float(x))
+
+
+def silu(x: float, lib=None) -> float:
+    return (lib or load()).oracle_silu(float(x))
+
+
+def conv1d(x, w, lib=None) -> np.ndarray:
+    """Causal depthwise Conv1D.  x: [L, C], w: [C, W] -> [L, C]."""
+    x = _f64(x); w = _f64(w)
+    L, C = x.shape
+    y = np.empty((L, C), np.float64)
+    (lib or load()).oracle_conv1d(_ptr(x), L, C, C, _ptr(w), w.shape[1], _ptr(y))
+    return y
+
+
+def softmax(a, lib=None) -> np.ndarray:
+    """Key-gate softmax over the sequence.  a: [L] -> [L]."""
+    a = _f64(a)
+    g = np.empty(a.shape[0], np.float64)
+    (lib or load()).oracle_softmax(_ptr(a), a.shape[0], 1, _ptr(g))
+    return g
+
+
+def gated_rmsnorm_row(O, og, w, eps=RMS_EPS, lib=None) -> np.ndarray:
+    O = _f64(O); og = _f64(og); w = _f64(w)
+    y = np.empty(O.shape[0], np.float64)
+    (lib or load()).oracle_gated_rmsnorm_row(_ptr(O), _ptr(og), _ptr(w), O.shape[0],
+                                             float(eps), _ptr(y))
+    return y
+
+
+def gbla_head(q, k, v, a, og, wq, wk, wv, norm_w, eps=RMS_EPS, flags=0,
+              intermediates=False, lib=None):
+    """One (batch, head): q, k, v, og [L, D]; a [L]; wq/wk/wv [D, W]; norm_w [D].
+
+    Returns y [L, D], or (y, dict of intermediates) when asked.
+    """
+    q, k, v, og = (_f64(t) for t in (q, k, v, og))
+    a = _f64(a); wq, wk, wv = (_f64(t) for t in (wq, wk, wv)); norm_w = _f64(norm_w)
+    L, D = q.shape
+    W = wq.shape[1]
+    y = np.empty((L, D), np.float64)
+    inter = None
+    if intermediates:
+        inter = dict(qt=np.empty((L, D)), kt=np.empty((L, D)), vt=np.empty((L, D)),
+                     g=np.empty(L), S=np.empty((D, D)), z=np.empty(D),
+                     O=np.empty((L, D)))
+    ptrs = ([_ptr(inter[n]) for n in ("qt", "kt", "vt", "g", "S", "z", "O")]
+            if inter else [None] * 7)
+    rc = (lib or load()).oracle_gbla_head(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(a), _ptr(og), D, 1, L, D,
+        _ptr(wq), _ptr(wk), _ptr(wv), W, _ptr(norm_w), float(eps), int(flags),
+        _ptr(y), *ptrs)
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_head rejected its arguments ({rc})")
+    return (y, inter) if intermediates else y
+
+
+def gbla_head_quadratic(q, k, v, a, og, wq, wk, wv, norm_w, eps=RMS_EPS, flags=0,
+                        lib=None):
+    """Same as gbla_head through the explicit L x L matrix; returns (y, O)."""
+    q, k, v, og = (_f64(t) for t in (q, k, v, og))
+    a = _f64(a); wq, wk, wv = (_f64(t) for t in (wq, wk, wv)); norm_w = _f64(norm_w)
+    L, D = q.shape
+    y = np.empty((L, D)); O = np.empty((L, D))
+    rc = (lib or load()).oracle_gbla_head_quadratic(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(a), _ptr(og), D, 1, L, D,
+        _ptr(wq), _ptr(wk), _ptr(wv), wq.shape[1], _ptr(norm_w), float(eps),
+        int(flags), _ptr(y), _ptr(O))
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_head_quadratic rejected its arguments ({rc})")
+    return y, O
+
+
+def gbla_forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None,
+                 eps=RMS_EPS, flags=0, n_threads=1, out=None, lib=None):
+    """Whole core over [B, N, H, D] arrays; rows t >= seq_lens[b] keep `out`'s values
+    (NaN when `out` is not given).  conv_w: [3, H, D, W]; norm_w: [H, D]."""
+    q, k, v, og = (_f64(t) for t in (q, k, v, out_gate))
+    gate = _f64(gate); conv_w = _f64(conv_w); norm_w = _f64(norm_w)
+    B, N, H, D = q.shape
+    W = conv_w.shape[-1]
+    y = np.full((B, N, H, D), np.nan) if out is None else out
+    assert y.dtype == np.float64 and y.flags.c_contiguous and y.shape == q.shape
+    sl = None
+    if seq_lens is not None:
+        sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    rc = (lib or load()).oracle_gbla_forward(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(og), _ptr(conv_w), _ptr(norm_w),
+        sl.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)) if sl is not None else None,
+        B, H, N, D, W, float(eps), int(flags), int(n_threads), _ptr(y))
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_forward rejected its arguments ({rc})")
+    return y

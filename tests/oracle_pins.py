@@ -1,0 +1,337 @@
+"""Checks that pin the fp64 oracle to something other than itself.
+
+Each check takes the loaded oracle library (so the same checks can be run
+against deliberately broken copies of the oracle) and raises AssertionError
+when the oracle disagrees with the paper or the mathematics.  The sources of
+truth are library routines (scipy, torch), closed forms, the quadratic form of
+Sec. 2.1 item 2 and invariants the equations imply.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import scipy.signal
+import scipy.special
+import torch
+
+import oracle
+
+W = oracle.CONV_W
+
+
+def _rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _head_inputs(rng, L, D, Wd=W):
+    q, k, v, og = (rng.standard_normal((L, D)) for _ in range(4))
+    a = rng.standard_normal(L)
+    wq, wk, wv = (0.5 * rng.standard_normal((D, Wd)) for _ in range(3))
+    nw = 1.0 + 0.02 * rng.standard_normal(D)
+    return q, k, v, a, og, wq, wk, wv, nw
+
+
+# --- element functions -------------------------------------------------------
+
+def pin_phi_closed_form(lib):
+    """phi = elu + 1 (Sec. 2): x+1 for x>0, e^x for x<=0; continuous, positive."""
+    for x, want in [(0.0, 1.0), (1.0, 2.0), (2.5, 3.5), (-1.0, math.exp(-1.0)),
+                    (-3.0, math.exp(-3.0)), (1e-9, 1.0 + 1e-9), (-40.0, math.exp(-40.0))]:
+        got = oracle.phi(x, lib)
+        assert abs(got - want) <= 1e-15 * max(1.0, abs(want)), (x, got, want)
+    xs = np.linspace(-30, 30, 601)
+    ys = np.array([oracle.phi(x, lib) for x in xs])
+    assert np.all(ys > 0)
+    # elu+1 by torch's library elu; elu(x)+1 cancels for very negative x, so the
+    # comparison is absolute there
+    ref = torch.nn.functional.elu(torch.tensor(xs, dtype=torch.float64)).numpy() + 1.0
+    np.testing.assert_allclose(ys, ref, rtol=1e-14, atol=1e-15)
+
+
+def pin_silu_library(lib):
+    """SiLU(x) = x * sigmoid(x) (gated RMSNorm, Sec. 2.1 item 3) vs torch and scipy."""
+    xs = np.linspace(-20, 20, 401)
+    got = np.array([oracle.silu(x, lib) for x in xs])
+    ref_t = torch.nn.functional.silu(torch.tensor(xs, dtype=torch.float64)).numpy()
+    ref_s = xs * scipy.special.expit(xs)
+    np.testing.assert_allclose(got, ref_t, rtol=1e-13, atol=1e-300)
+    np.testing.assert_allclose(got, ref_s, rtol=1e-13, atol=1e-300)
+
+
+def pin_conv1d_library(lib):
+    """Causal depthwise Conv1D (Sec. 2.1 item 1) equals a causal FIR filter
+    (scipy lfilter with reversed taps) and torch's conv1d with W-1 left zeros."""
+    rng = _rng(11)
+    L, C = 37, 6
+    x = rng.standard_normal((L, C))
+    w = rng.standard_normal((C, W))
+    y = oracle.conv1d(x, w, lib)
+    for c in range(C):
+        ref = scipy.signal.lfilter(w[c, ::-1], [1.0], x[:, c])
+        np.testing.assert_allclose(y[:, c], ref, rtol=1e-12, atol=1e-12)
+    xt = torch.tensor(x.T[None], dtype=torch.float64)          # [1, C, L]
+    xt = torch.nn.functional.pad(xt, (W - 1, 0))
+    ref = torch.nn.functional.conv1d(xt, torch.tensor(w[:, None, :]), groups=C)[0].T.numpy()
+    np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-12)
+
+
+def pin_conv1d_impulse(lib):
+    """An impulse at position s reaches only s..s+W-1 (causal), tap W-1 first."""
+    L, C, s = 12, 3, 5
+    rng = _rng(12)
+    w = rng.standard_normal((C, W))
+    x = np.zeros((L, C)); x[s, :] = 1.0
+    y = oracle.conv1d(x, w, lib)
+    for t in range(L):
+        for c in range(C):
+            want = w[c, W - 1 - (t - s)] if 0 <= t - s < W else 0.0
+            assert y[t, c] == want, (t, c, y[t, c], want)
+
+
+def pin_softmax_library(lib):
+    """Key gate g = softmax over the sequence (Sec. 2.1 item 2) vs scipy; stable
+    for logits near the exp overflow limit."""
+    rng = _rng(13)
+    for L in (1, 2, 7, 100):
+        a = 3.0 * rng.standard_normal(L)
+        np.testing.assert_allclose(oracle.softmax(a, lib), scipy.special.softmax(a),
+                                   rtol=1e-13, atol=1e-300)
+    a = np.array([1000.0, 999.0, 1001.0, -5.0])
+    g = oracle.softmax(a, lib)
+    assert np.all(np.isfinite(g))
+    np.testing.assert_allclose(g, scipy.special.softmax(a), rtol=1e-13, atol=1e-300)
+    assert abs(g.sum() - 1.0) < 1e-15
+
+
+def pin_rmsnorm_library(lib):
+    """Gated RMSNorm (Sec. 2.1 item 3) equals torch's rms_norm times SiLU(og)."""
+    rng = _rng(14)
+    for D in (1, 5, 64):
+        O = rng.standard_normal(D) * 0.01
+        og = rng.standard_normal(D)
+        w = 1.0 + 0.1 * rng.standard_normal(D)
+        y = oracle.gated_rmsnorm_row(O, og, w, 1e-6, lib)
+        Ot = torch.tensor(O[None])
+        ref = (torch.nn.functional.rms_norm(Ot, (D,), torch.tensor(w), eps=1e-6)[0]
+               * torch.nn.functional.silu(torch.tensor(og))).numpy()
+        np.testing.assert_allclose(y, ref, rtol=1e-12, atol=1e-15)
+
+
+def pin_rmsnorm_closed_form(lib):
+    """rms(y / (w * SiLU(og))) = sqrt(ms / (ms + eps)) with ms = mean O^2."""
+    rng = _rng(15)
+    D, eps = 16, 1e-3
+    O = 0.05 * rng.standard_normal(D)
+    og = np.abs(rng.standard_normal(D)) + 0.1
+    w = 1.0 + 0.1 * rng.standard_normal(D)
+    y = oracle.gated_rmsnorm_row(O, og, w, eps, lib)
+    u = y / (w * og * scipy.special.expit(og))
+    ms = np.mean(O ** 2)
+    assert abs(np.sqrt(np.mean(u ** 2)) - np.sqrt(ms / (ms + eps))) < 1e-13
+    np.testing.assert_allclose(u / O, 1.0 / np.sqrt(ms + eps) * np.ones(D), rtol=1e-12)
+
+
+# --- the layer ---------------------------------------------------------------
+
+def pin_linear_equals_quadratic(lib):
+    """The linear-time matrix form equals the explicit L x L form (Sec. 2.1
+    item 2: both displayed equations), for every ablation setting."""
+    for seed, L, D in [(21, 13, 5), (22, 1, 3), (23, 40, 8)]:
+        args = _head_inputs(_rng(seed), L, D)
+        for f in range(8):
+            y1 = oracle.gbla_head(*args, flags=f, lib=lib)
+            y2, _ = oracle.gbla_head_quadratic(*args, flags=f, lib=lib)
+            np.testing.assert_allclose(y1, y2, rtol=1e-11, atol=1e-13)
+
+
+def pin_bla_textbook(lib):
+    """With conv, gate and norm switched off GBLA is Eq. bla; O is also a
+    convex combination of the v rows (weights phi(q)^T phi(k_j), normalised)."""
+    rng = _rng(31)
+    L, D = 9, 4
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    y = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, flags=oracle.BLA, lib=lib)
+    pq = np.where(q > 0, q + 1, np.exp(np.minimum(q, 0)))
+    pk = np.where(k > 0, k + 1, np.exp(np.minimum(k, 0)))
+    sim = pq @ pk.T                        # L x L similarities
+    P = sim / sim.sum(axis=1, keepdims=True)
+    np.testing.assert_allclose(y, P @ v, rtol=1e-12, atol=1e-14)
+    # "W/o key gating" is the uniform gate softmax(0) = 1/L; z is then the mean
+    # of phi(k_j) over the sequence
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, flags=oracle.BLA,
+                                intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["g"], np.full(L, 1.0 / L), rtol=1e-15)
+    np.testing.assert_allclose(inter["z"], pk.mean(axis=0), rtol=1e-13)
+
+
+def pin_hand_worked_d1(lib):
+    """D=1, L=2, no conv: q cancels and O = sum g phi(k) v / sum g phi(k).
+    a = (0, ln 3) gives g = (1/4, 3/4); k = (0, 1) gives phi = (1, 2);
+    v = (2, -1) gives O = (1/2 - 3/2) / (1/4 + 3/2) = -4/7 for both rows."""
+    one = np.ones((1, W))
+    q = np.array([[0.3], [-2.0]]); k = np.array([[0.0], [1.0]])
+    v = np.array([[2.0], [-1.0]]); og = np.array([[1.0], [-0.5]])
+    a = np.array([0.0, math.log(3.0)])
+    nw = np.array([1.5])
+    _, inter = oracle.gbla_head(q, k, v, a, og, one, one, one, nw,
+                                flags=oracle.NO_CONV | oracle.NO_NORM,
+                                intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["g"], [0.25, 0.75], rtol=1e-15)
+    np.testing.assert_allclose(inter["z"], [0.25 + 1.5], rtol=1e-15)
+    np.testing.assert_allclose(inter["S"], [[0.5 - 1.5]], rtol=1e-15)
+    np.testing.assert_allclose(inter["O"][:, 0], [-4 / 7, -4 / 7], rtol=1e-14)
+    # Gated RMSNorm with D=1: y = O / sqrt(O^2 + eps) * w * silu(og)
+    eps = 1e-6
+    y = oracle.gbla_head(q, k, v, a, og, one, one, one, nw, eps=eps,
+                         flags=oracle.NO_CONV, lib=lib)
+    O = -4 / 7
+    for i, g_in in enumerate([1.0, -0.5]):
+        want = O / math.sqrt(O * O + eps) * 1.5 * g_in / (1 + math.exp(-g_in))
+        assert abs(y[i, 0] - want) < 1e-14, (y[i, 0], want)
+
+
+def pin_constant_values(lib):
+    """If every v~ row is the same vector c, every O row equals c (O is a
+    weighted mean of the v~ rows).  Identity taps on v keep v~ = v."""
+    rng = _rng(41)
+    L, D = 50, 6
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    c = rng.standard_normal(D)
+    v = np.tile(c, (L, 1))
+    wv = np.zeros((D, W)); wv[:, W - 1] = 1.0
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["O"], np.tile(c, (L, 1)), rtol=1e-12, atol=1e-14)
+
+
+def pin_state_ones(lib):
+    """With v~ = 1 the state rows equal the normaliser: S[d, e] = z[d] (both are
+    K^T applied to V and to 1)."""
+    rng = _rng(42)
+    L, D = 30, 5
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    v = np.ones((L, D))
+    wv = np.zeros((D, W)); wv[:, W - 1] = 1.0
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["S"], np.tile(inter["z"][:, None], (1, D)), rtol=1e-13)
+    assert np.all(inter["z"] > 0)
+    assert abs(inter["g"].sum() - 1.0) < 1e-14
+
+
+def pin_single_token(lib):
+    """L = 1: the softmax gate is 1, O = v~_0 = w_v[:, W-1] * v_0 (only the last
+    tap sees a real token), and the key side cancels."""
+    rng = _rng(43)
+    D = 7
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, 1, D)
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["O"][0], wv[:, W - 1] * v[0], rtol=1e-13)
+    np.testing.assert_allclose(inter["g"], [1.0], rtol=0, atol=0)
+
+
+def pin_permutation_equivariance(lib):
+    """Without the Conv1D the bidirectional core has no notion of order:
+    permuting positions permutes the outputs."""
+    rng = _rng(51)
+    L, D = 23, 4
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    p = rng.permutation(L)
+    y = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, flags=oracle.NO_CONV, lib=lib)
+    yp = oracle.gbla_head(q[p], k[p], v[p], a[p], og[p], wq, wk, wv, nw,
+                          flags=oracle.NO_CONV, lib=lib)
+    np.testing.assert_allclose(yp, y[p], rtol=1e-12, atol=1e-14)
+
+
+def pin_gate_shift_invariance(lib):
+    """softmax(a + c) = softmax(a): a shift of all gate logits changes nothing."""
+    rng = _rng(52)
+    L, D = 31, 4
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    y = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, lib=lib)
+    y2 = oracle.gbla_head(q, k, v, a + 7.25, og, wq, wk, wv, nw, lib=lib)
+    np.testing.assert_allclose(y2, y, rtol=1e-12, atol=1e-14)
+
+
+def pin_gate_weights_keys(lib):
+    """A dominant gate logit makes that key the only one: O_i -> v~_j for all i."""
+    rng = _rng(53)
+    L, D, j = 17, 4, 6
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    a = np.zeros(L); a[j] = 60.0
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, intermediates=True, lib=lib)
+    np.testing.assert_allclose(inter["O"], np.tile(inter["vt"][j], (L, 1)), rtol=1e-12, atol=1e-12)
+
+
+def _layer_inputs(rng, B, N, H, D):
+    q, k, v, og = (rng.standard_normal((B, N, H, D)) for _ in range(4))
+    gate = rng.standard_normal((B, N, H))
+    conv_w = 0.5 * rng.standard_normal((3, H, D, W))
+    norm_w = 1.0 + 0.02 * rng.standard_normal((H, D))
+    return q, k, v, gate, og, conv_w, norm_w
+
+
+def pin_layer_indexing(lib):
+    """The multi-head driver equals the single-head routine applied to each
+    (batch, head) slice with that head's own taps and norm weight (Sec. 2.1,
+    multi-head paragraph); threads do not change a bit."""
+    rng = _rng(61)
+    B, N, H, D = 2, 19, 3, 4
+    q, k, v, gate, og, conv_w, norm_w = _layer_inputs(rng, B, N, H, D)
+    sl = np.array([19, 11], np.int32)
+    y1 = oracle.gbla_forward(q, k, v, gate, og, conv_w, norm_w, sl, n_threads=1, lib=lib)
+    y4 = oracle.gbla_forward(q, k, v, gate, og, conv_w, norm_w, sl, n_threads=4, lib=lib)
+    assert np.array_equal(np.isnan(y1), np.isnan(y4))
+    assert np.array_equal(y1[~np.isnan(y1)], y4[~np.isnan(y4)])
+    for b in range(B):
+        Lb = sl[b]
+        assert np.all(np.isnan(y1[b, Lb:]))
+        for h in range(H):
+            ref = oracle.gbla_head(q[b, :Lb, h], k[b, :Lb, h], v[b, :Lb, h], gate[b, :Lb, h],
+                                   og[b, :Lb, h], conv_w[0, h], conv_w[1, h], conv_w[2, h],
+                                   norm_w[h], lib=lib)
+            np.testing.assert_array_equal(y1[b, :Lb, h], ref)
+
+
+def pin_padding_ignored(lib):
+    """Rows at t >= L_b (right padding) contribute nothing, whatever they hold:
+    a padded run equals the unpadded run on the valid rows."""
+    rng = _rng(62)
+    B, N, H, D = 2, 24, 2, 4
+    q, k, v, gate, og, conv_w, norm_w = _layer_inputs(rng, B, N, H, D)
+    sl = np.array([24, 9], np.int32)
+    y = oracle.gbla_forward(q, k, v, gate, og, conv_w, norm_w, sl, lib=lib)
+    for t in (q, k, v, og):
+        t[1, 9:] = np.nan
+    gate[1, 9:] = 1e30
+    y2 = oracle.gbla_forward(q, k, v, gate, og, conv_w, norm_w, sl, lib=lib)
+    np.testing.assert_array_equal(y2[1, :9], y[1, :9])
+    cut = [x[1:2, :9] for x in (q, k, v, gate, og)]
+    y3 = oracle.gbla_forward(*cut, conv_w, norm_w, None, lib=lib)
+    np.testing.assert_array_equal(y3[0], y[1, :9])
+
+
+def pin_heads_independent(lib):
+    """Permuting heads together with their taps and norm weights permutes the
+    outputs (heads share nothing)."""
+    rng = _rng(63)
+    B, N, H, D = 1, 15, 4, 3
+    q, k, v, gate, og, conv_w, norm_w = _layer_inputs(rng, B, N, H, D)
+    p = np.array([2, 0, 3, 1])
+    y = oracle.gbla_forward(q, k, v, gate, og, conv_w, norm_w, lib=lib)
+    yp = oracle.gbla_forward(q[:, :, p], k[:, :, p], v[:, :, p], gate[:, :, p], og[:, :, p],
+                             conv_w[:, p], norm_w[p], lib=lib)
+    np.testing.assert_array_equal(yp, y[:, :, p])
+
+
+def pin_denominator_positive(lib):
+    """phi > 0 and g > 0, so z > 0 and every readout denominator is positive."""
+    rng = _rng(64)
+    L, D = 40, 6
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    q *= 30; k *= 30
+    _, inter = oracle.gbla_head(q, k, v, a, og, wq, wk, wv, nw, intermediates=True, lib=lib)
+    assert np.all(inter["z"] > 0)
+    assert np.all(np.isfinite(inter["O"]))
+
+
+ALL_PINS = [v for k_, v in sorted(globals().items()) if k_.startswith("pin_")]

@@ -1,0 +1,66 @@
+"""Plausible mistakes planted in a copy of the oracle are each caught by at
+least one pin (CPU only; the planted copies are compiled into a temporary
+directory and never touch the real oracle)."""
+import os
+
+import pytest
+
+import oracle
+from oracle_pins import ALL_PINS
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "gbla_oracle.c")
+
+# (id, text in the oracle, replacement) -- each a one-token slip
+MUTANTS = [
+    ("phi_drops_plus_one", "return x > 0.0 ? x + 1.0 : exp(x);", "return x > 0.0 ? x : exp(x);"),
+    ("phi_wrong_branch", "return x > 0.0 ? x + 1.0 : exp(x);", "return x >= 1.0 ? x + 1.0 : exp(x);"),
+    ("silu_sign", "return x / (1.0 + exp(-x));", "return x / (1.0 + exp(x));"),
+    ("conv_taps_reversed", "acc += w[(long)c * W + i] * x[s * ldx + c];",
+     "acc += w[(long)c * W + (W - 1 - i)] * x[s * ldx + c];"),
+    ("conv_off_by_one", "long s = t - (W - 1) + i;", "long s = t - W + i;"),
+    ("conv_not_causal", "long s = t - (W - 1) + i;", "long s = t + i;"),
+    ("softmax_no_max", "g[j] = exp(a[j * lda] - m);", "g[j] = exp(a[j * lda]);"),
+    ("softmax_not_normalised", "for (long j = 0; j < L; ++j) g[j] /= s;",
+     "for (long j = 0; j < L; ++j) g[j] /= 1.0;"),
+    ("state_wrong_v_index", "S[d * D + e] += pk[d] * vt[j * D + e];",
+     "S[d * D + e] += pk[d] * vt[j * D + d];"),
+    ("z_ungated", "z[d] += pk[d];", "z[d] += oracle_phi(kt[j * D + d]);"),
+    ("state_gate_dropped",
+     "for (int d = 0; d < D; ++d) pk[d] = g[j] * oracle_phi(kt[j * D + d]);",
+     "for (int d = 0; d < D; ++d) pk[d] = oracle_phi(kt[j * D + d]);"),
+    ("readout_transposed", "num += pq[d] * S[d * D + e];", "num += pq[d] * S[e * D + d];"),
+    ("readout_no_phi_q", "pq[d] = oracle_phi(qt[i * D + d]);", "pq[d] = qt[i * D + d];"),
+    ("rms_sum_not_mean", "ms /= (double)D;", "ms /= 1.0;"),
+    ("rms_eps_outside", "double r = 1.0 / sqrt(ms + eps);", "double r = 1.0 / (sqrt(ms) + eps);"),
+    ("norm_weight_dropped", "y[d] = O[d] * r * w[d] * oracle_silu(og[d]);",
+     "y[d] = O[d] * r * oracle_silu(og[d]);"),
+    ("gate_not_silu", "y[d] = O[d] * r * w[d] * oracle_silu(og[d]);",
+     "y[d] = O[d] * r * w[d] * og[d];"),
+    ("uniform_gate_wrong", "g[j] = 1.0 / (double)L;", "g[j] = 1.0;"),
+    ("driver_conv_head_offset", "J->conv_w + ((1 * J->H + h) * D) * W",
+     "J->conv_w + ((1 * J->H + 0) * D) * W"),
+    ("driver_gate_stride", "J->gate + b * J->N * J->H + h, J->og + base, ld, J->H,",
+     "J->gate + b * J->N * J->H + h, J->og + base, ld, 1,"),
+    ("driver_norm_head", "J->norm_w + h * D", "J->norm_w"),
+    ("driver_len_unclamped", "if (L > J->N) L = J->N;", "if (L > J->N) L = J->N + 0; L = J->N;"),
+    ("quadratic_gate_on_query", "A[i * L + j] = g[j] * s;", "A[i * L + j] = g[i] * s;"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_mutant(name, old, new, tmp_path):
+    text = open(SRC).read()
+    assert text.count(old) >= 1, f"mutation target for {name} not found in the oracle"
+    src = tmp_path / "mutant.c"
+    src.write_text(text.replace(old, new, 1))
+    so = oracle.build(str(src), str(tmp_path / "libmutant.so"))
+    lib = oracle.load(so)
+    caught = []
+    for pin in ALL_PINS:
+        try:
+            pin(lib)
+        except AssertionError:
+            caught.append(pin.__name__)
+        except (ValueError, FloatingPointError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin caught the planted mistake {name}"
