@@ -1,0 +1,427 @@
+"""Benchmark of the GBLA layer-core forward on GB300 (one JSON line on rank 0).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+A step is one GBLA forward (Conv1D, phi, key gate, state reduction, readout,
+gated RMSNorm) over the paper's headline length: B=2, H=8, N=32768, D=64,
+bf16 inputs (synthetic, seeded).  `value` is whole-job tokens/s (valid tokens
+over all ranks, each token carrying all H heads) with the inputs resident in
+HBM; `e2e` is the same metric through the host-memory C-ABI entry point with
+the host<->device copies inside the timed region.  `roofline` reports the
+dominant kernel's algorithmic bytes per launch over its CUDA-event duration
+against the measured HBM copy bandwidth; `cpu_baseline` is the fp64 oracle
+timed on this machine's host cores.
+
+Under torchrun each rank runs its own copy of the workload (the (batch, head)
+pairs are independent, so the path shards with no collective): weak scaling.
+`--impl reference` times the fp64 oracle instead (on rank 0 only), a
+deliberately slow program; the GPU/CPU ratio says nothing about kernel quality.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2606_07317_gb300.workloads import HEADLINE, WORKLOADS, make_inputs  # noqa: E402
+
+METRIC = "GBLA fwd tokens/sec and % of GB300 HBM roofline at N=32768, 1 GPU"
+UNIT = "tokens/s"
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_HBM_GBS = 6800.0
+
+
+# --------------------------------------------------------------------------- helpers
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def init_dist(ws, backend):
+    if ws > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group(backend=backend)
+
+
+def barrier(ws):
+    if ws > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x: float, ws: int, device) -> float:
+    if ws == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def measured_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2606_07317_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on the
+    current kernel sources (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(kernel, {}).get(workload)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+            self.t0 = time.time()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.t1 = time.time()
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------- our arm
+
+def bench_ours(args, ws, rank, local):
+    from paper_2606_07317_gb300 import gbla
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(ws, "nccl")
+    lib = gbla.load()  # fails loudly if the CUDA library is missing
+    w = WORKLOADS[args.workload]
+    tokens = w.valid_tokens
+    inp0 = make_inputs(w, dev)
+    # Two input sets rotated between steps (each larger than L2 at the headline size).
+    sets = [inp0, {k: (v.clone() if v is not None else None) for k, v in inp0.items()}]
+    outs = [torch.empty_like(inp0["q"]) for _ in sets]
+    step_bytes = w.valid_tokens * w.H * w.bytes_per_token_head
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        s = sets[i % 2]
+        gbla.forward(s["q"], s["k"], s["v"], s["gate"], s["out_gate"], s["conv_w"],
+                     s["norm_w"], s["seq_lens"], out=outs[i % 2], algo=args.algo, stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize(dev)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.1)
+    n0 = gbla.launch_count()
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(ws)
+    launches = gbla.launch_count() - n0
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    ms = max_over_ranks(ms, ws, dev)
+    value = tokens * ws / (ms * 1e-3)
+
+    # Per-phase durations (state reduction vs readout) with CUDA events on the
+    # launching stream, over the same number of steps.
+    nph = min(args.steps, 500)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(nph)]
+    st_bufs = [torch.empty((w.B, w.H, w.D * w.D + w.D), dtype=torch.float32, device=dev)
+               for _ in sets]
+    torch.cuda.synchronize(dev)
+    for i in range(nph):
+        s = sets[i % 2]
+        evs[i][0].record(stream)
+        gbla.state(s["k"], s["v"], s["gate"], s["conv_w"], s["seq_lens"], out=st_bufs[i % 2],
+                   algo=args.algo, stream=stream)
+        evs[i][1].record(stream)
+        gbla.readout(s["q"], s["out_gate"], s["conv_w"], s["norm_w"], st_bufs[i % 2],
+                     s["seq_lens"], out=outs[i % 2], algo=args.algo, stream=stream)
+        evs[i][2].record(stream)
+    torch.cuda.synchronize(dev)
+    t_state = sum(e[0].elapsed_time(e[1]) for e in evs) / nph
+    t_read = sum(e[1].elapsed_time(e[2]) for e in evs) / nph
+    e_el = 2 if w.dtype == "bf16" else 4
+    per_th = w.valid_tokens * w.H
+    bytes_state = per_th * e_el * (2 * w.D + 1)   # k, v, gate
+    bytes_read = per_th * e_el * (3 * w.D)        # q, out_gate, o
+    if t_read >= t_state:
+        dom, dom_ms, dom_bytes = "readout", t_read, bytes_read
+    else:
+        dom, dom_ms, dom_bytes = "state", t_state, bytes_state
+    peak, peak_kind = measured_peaks()
+    achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                "unit": "GB/s", "frac": round(achieved / peak, 4),
+                "traffic": recorded_traffic(dom, w.name),
+                "kernel": dom, "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"
+                if peak_kind == "measured" else "fallback 6.8 TB/s",
+                "alg_bytes_per_launch": dom_bytes, "launch_ms": round(dom_ms, 5),
+                "phases_ms": {"state": round(t_state, 5), "readout": round(t_read, 5)},
+                "whole_step_frac": round(step_bytes / (ms * 1e-3) / 1e9 / peak, 4)}
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = bench_e2e(args, w, inp0, dev, gbla, tokens, ws)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, inp0)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic (seeded N(0,1) inputs of the workload's shape)",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "D": w.D,
+                       "conv_width": 4, "tokens_per_step": tokens,
+                       "alg_bytes_per_step": step_bytes,
+                       "l2": "inputs larger than L2 (%.0f MB per set vs 129 MB), two sets rotated"
+                             % (step_bytes / 1e6),
+                       "algo": {0: "auto", 1: "simt", 2: "tc"}[args.algo],
+                       "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"},
+            "roofline": roofline,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "clocks": clocks,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def bench_e2e(args, w, inp, dev, gbla, tokens, ws):
+    host = {k: (v.cpu().pin_memory() if v is not None else None) for k, v in inp.items()}
+    out = torch.empty_like(host["q"]).pin_memory()
+    n = max(3, min(args.steps, 30))
+
+    def call():
+        gbla.forward_host(host["q"], host["k"], host["v"], host["gate"], host["out_gate"],
+                          host["conv_w"], host["norm_w"], host["seq_lens"], out=out)
+
+    for _ in range(2):
+        call()
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    for _ in range(n):
+        call()
+    torch.cuda.synchronize(dev)
+    dt = (time.perf_counter() - t0) / n
+    dt = max_over_ranks(dt, ws, dev)
+    e_el = 2 if w.dtype == "bf16" else 4
+    th = w.valid_tokens * w.H
+    h2d = th * e_el * (4 * w.D + 1) + 4 * (3 * w.H * w.D * 4 + w.H * w.D)
+    if w.seq_lens is not None:
+        h2d += 4 * w.B
+    d2h = th * e_el * w.D
+    return {"value": round(tokens * ws / dt, 1), "unit": UNIT, "steps": n,
+            "ms_per_step": round(dt * 1e3, 4),
+            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "api": "gbla_forward_host (pinned host buffers)"}
+
+
+# --------------------------------------------------------------------------- oracle (CPU)
+
+def _oracle_inputs(inp, pairs, L):
+    """float64 per-(b, h) slices of the first L tokens, taken outside any timing."""
+    f64 = lambda t: t.detach().cpu().double().numpy()  # noqa: E731
+    q, k, v, og, gate = (f64(inp[n]) for n in ("q", "k", "v", "out_gate", "gate"))
+    cw, nw = f64(inp["conv_w"]), f64(inp["norm_w"])
+    out = []
+    for b, h in pairs:
+        out.append(dict(q=np.ascontiguousarray(q[b, :L, h]), k=np.ascontiguousarray(k[b, :L, h]),
+                        v=np.ascontiguousarray(v[b, :L, h]), a=np.ascontiguousarray(gate[b, :L, h]),
+                        og=np.ascontiguousarray(og[b, :L, h]), wq=cw[0, h], wk=cw[1, h],
+                        wv=cw[2, h], nw=nw[h]))
+    return out
+
+
+def _oracle_run(heads, n_threads):
+    import concurrent.futures as cf
+
+    import oracle
+    lib = oracle.load()
+
+    def one(x):
+        return oracle.gbla_head(x["q"], x["k"], x["v"], x["a"], x["og"], x["wq"], x["wk"],
+                                x["wv"], x["nw"], lib=lib)
+    if n_threads == 1:
+        for x in heads:
+            one(x)
+    else:  # ctypes releases the GIL, so threads run the C oracle in parallel
+        with cf.ThreadPoolExecutor(n_threads) as ex:
+            list(ex.map(one, heads))
+
+
+def cpu_baseline(w, inp, budget_s: float = 15.0):
+    """The oracle on all host cores over whole (batch, head) sequences of the
+    workload, as many as fit in about `budget_s` seconds."""
+    cores = os.cpu_count() or 1
+    pairs_all = [(b, h) for b in range(w.B) for h in range(w.H)]
+    L = w.lengths()[0]
+    # calibrate on one sequence
+    heads = _oracle_inputs(inp, pairs_all[:1], L)
+    t0 = time.perf_counter()
+    _oracle_run(heads, 1)
+    t1 = time.perf_counter() - t0
+    n_pairs = int(max(1, min(len(pairs_all), budget_s / max(t1, 1e-6) * cores * 0.8)))
+    n_pairs = max(1, (n_pairs // cores) * cores) if n_pairs >= cores else n_pairs
+    heads = _oracle_inputs(inp, pairs_all[:n_pairs], L)
+    threads = min(cores, n_pairs)
+    t0 = time.perf_counter()
+    _oracle_run(heads, threads)
+    dt = time.perf_counter() - t0
+    tok = n_pairs * L / w.H  # token-heads / heads = tokens
+    return {"value": round(tok / dt, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "seconds": round(dt, 3),
+            "sample": f"{n_pairs} of {len(pairs_all)} (batch, head) sequences of {L} tokens "
+                      f"({w.name}), fp64 C oracle, one thread per sequence; tokens = "
+                      f"token-heads / H"}
+
+
+def bench_reference(args, ws, rank):
+    """--impl reference: the fp64 oracle on the host cores (rank 0 only)."""
+    if rank != 0:
+        return
+    w = WORKLOADS[args.workload]
+    inp = make_inputs(w, "cpu")
+    cores = os.cpu_count() or 1
+    pairs = [(b, h) for b in range(w.B) for h in range(w.H)]
+    # calibrate the sample so that (warmup + steps) fit in ~120 s
+    probe_L = 1024
+    heads = _oracle_inputs(inp, pairs[:1], probe_L)
+    t0 = time.perf_counter()
+    _oracle_run(heads, 1)
+    per_tok = (time.perf_counter() - t0) / probe_L
+    n_pairs = min(len(pairs), cores)
+    step_budget = 120.0 / max(1, args.steps + args.warmup)
+    L = int(min(w.lengths()[0], max(64, step_budget / per_tok)))
+    heads = _oracle_inputs(inp, pairs[:n_pairs], L)
+    for _ in range(args.warmup):
+        _oracle_run(heads, n_pairs)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _oracle_run(heads, n_pairs)
+    dt = (time.perf_counter() - t0) / args.steps
+    tok = n_pairs * L / w.H
+    value = tok / dt
+    sample = (f"per step: {n_pairs} (batch, head) sequences x first {L} tokens of {w.name}, "
+              f"fp64 C oracle, one thread per sequence; tokens = token-heads / H")
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT,
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "D": w.D},
+            "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": n_pairs,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=HEADLINE, choices=sorted(WORKLOADS))
+    ap.add_argument("--algo", type=int, default=0, help="0 auto, 1 simt, 2 tc")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    ws, rank, local = dist_env()
+    if args.impl == "reference":
+        bench_reference(args, ws, rank)
+        return
+    bench_ours(args, ws, rank, local)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,166 @@
+/*
+ * gbla.h -- C ABI of the GB300 (sm_103a) GBLA layer-core forward.
+ *
+ * The layer is Gated Bidirectional Linear Attention, Sec. 2.1 of "Gated
+ * Bidirectional Linear Attention for Generative Retrieval".  For every batch
+ * row b, head h and valid position i < L_b it computes
+ *
+ *   q~, k~, v~ = Conv1D(q), Conv1D(k), Conv1D(v)        (Sec. 2.1 item 1)
+ *   g          = softmax_j(gate[b, j, h]), j < L_b     (Sec. 2.1 item 2)
+ *   K^         = g * phi(K~),  phi(x) = elu(x) + 1     (Sec. 2 / 2.1 item 2)
+ *   S = K^T V~ (D x D),  z = K^T 1 (D)                  (Sec. 2.1 item 2)
+ *   O_i        = phi(q~_i)^T S / phi(q~_i)^T z
+ *   o_i        = O_i / sqrt(mean(O_i^2) + eps) * norm_w[h] * SiLU(out_gate_i)
+ *                                                       (Sec. 2.1 item 3)
+ *
+ * Conv1D is causal and depthwise over the sequence, width GBLA_CONV_WIDTH, left
+ * zero padding, no bias: x~[t, c] = sum_i w[c, i] * x[t - (W-1) + i, c], so tap
+ * W-1 multiplies the current token.  The gate logits and the output-gate
+ * input are taken as given (already derived from the convolved sequence).
+ * eps is gbla_rms_eps().
+ *
+ * Layouts (all contiguous, row-major, no padding between rows):
+ *   q, k, v, out_gate, o : [B, N, H, D] of dtype
+ *   gate                 : [B, N, H]    of dtype (softmax logits)
+ *   conv_w               : [3, H, D, GBLA_CONV_WIDTH] fp32 (taps for q, k, v)
+ *   norm_w               : [H, D] fp32 (RMSNorm weight per head)
+ *   seq_lens             : [B] int32, or NULL meaning every row has length N;
+ *                          values are clamped to [0, N] on the device
+ *   state                : [B, H, D*D + D] fp32: S row-major (S[d][e]) then z
+ *
+ * Ownership: every pointer is a caller-owned DEVICE pointer on the current
+ * device, 16-byte aligned.  The library keeps no pointer after a call returns.
+ * Outputs must not overlap inputs.
+ *
+ * Asynchrony: every compute call only enqueues work on `stream` (NULL = the
+ * legacy default stream) and returns; it never synchronises.  Scratch memory
+ * is taken from the device's stream-ordered pool (cudaMallocAsync) and freed
+ * on the same stream, so concurrent calls on different streams are safe.
+ *
+ * Errors: arguments are validated on the host before anything is enqueued.
+ *   GBLA_ERR_INVALID_ARG  null pointer, negative size, misaligned pointer,
+ *                         overlapping output, or a size beyond the limits
+ *   GBLA_ERR_UNSUPPORTED  D not in {32, 64, 128}, unknown dtype or algo,
+ *                         or an algo that does not cover (dtype, D)
+ *   GBLA_ERR_ALLOC        the stream-ordered scratch allocation failed
+ *   GBLA_ERR_CUDA         a CUDA call or kernel launch failed
+ * A call with B, H or N equal to 0 has nothing to compute: it returns GBLA_OK
+ * without touching any pointer.  Rows t >= L_b of o are never written, and a
+ * sequence of length 0 writes nothing.
+ */
+#ifndef GBLA_H_
+#define GBLA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* cudaStream_t is `struct CUstream_st *` */
+typedef struct CUstream_st *gbla_stream_t;
+
+#define GBLA_CONV_WIDTH 4
+
+typedef enum gbla_status {
+  GBLA_OK = 0,
+  GBLA_ERR_INVALID_ARG = 1,
+  GBLA_ERR_UNSUPPORTED = 2,
+  GBLA_ERR_ALLOC = 3,
+  GBLA_ERR_CUDA = 4
+} gbla_status;
+
+typedef enum gbla_dtype {
+  GBLA_FP32 = 0, /* fp32 storage, exact fp32 arithmetic (CUDA-core FMA) */
+  GBLA_BF16 = 1  /* bf16 storage, fp32 accumulation                      */
+} gbla_dtype;
+
+typedef enum gbla_algo {
+  GBLA_ALGO_AUTO = 0, /* tensor-core kernels where they cover (dtype, D), else SIMT */
+  GBLA_ALGO_SIMT = 1, /* CUDA-core kernels, every (dtype, D)                        */
+  GBLA_ALGO_TC = 2    /* tcgen05/TMEM + TMA kernels: bf16 with D in {64, 128}      */
+} gbla_algo;
+
+/*
+ * gbla_forward -- the whole GBLA core, Sec. 2.1 (all three add-ons on).
+ * Writes o[b, t, h, :] for every b, h and t < L_b.  Equivalent to
+ * gbla_forward_ex(..., GBLA_ALGO_AUTO, stream).
+ */
+gbla_status gbla_forward(const void *q, const void *k, const void *v,
+                         const void *gate, const void *out_gate,
+                         const float *conv_w, const float *norm_w,
+                         const int32_t *seq_lens, void *o, int B, int H, int N,
+                         int D, gbla_dtype dtype, gbla_stream_t stream);
+
+/* gbla_forward with an explicit kernel family (see gbla_algo). */
+gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
+                            const void *gate, const void *out_gate,
+                            const float *conv_w, const float *norm_w,
+                            const int32_t *seq_lens, void *o, int B, int H,
+                            int N, int D, gbla_dtype dtype, gbla_algo algo,
+                            gbla_stream_t stream);
+
+/*
+ * gbla_state -- the sequence-global part of Sec. 2.1 item 2: Conv1D of k and
+ * v, phi, the softmax key gate, and per (b, h) the state S = K^T V~ and the
+ * normaliser z = K^T 1 with K^ = g * phi(K~), g the softmax over j < L_b.
+ * Writes state[b, h, :] (layout above; zeros when L_b = 0).  The sum over the
+ * sequence is split into chunks whose partial sums are combined in a fixed
+ * order, so the result is bitwise reproducible for a given (N, seq_lens).
+ */
+gbla_status gbla_state(const void *k, const void *v, const void *gate,
+                       const float *conv_w, const int32_t *seq_lens,
+                       float *state, int B, int H, int N, int D,
+                       gbla_dtype dtype, gbla_algo algo, gbla_stream_t stream);
+
+/*
+ * gbla_readout -- the per-token part: Conv1D of q, phi, O_i = phi(q~_i)^T S /
+ * phi(q~_i)^T z (Sec. 2.1 item 2) and the gated RMSNorm (Sec. 2.1 item 3),
+ * from a state laid out as gbla_state writes it.  Any positive common scale
+ * of S and z gives the same o.  Writes o rows t < L_b only.
+ */
+gbla_status gbla_readout(const void *q, const void *out_gate,
+                         const float *conv_w, const float *norm_w,
+                         const int32_t *seq_lens, const float *state, void *o,
+                         int B, int H, int N, int D, gbla_dtype dtype,
+                         gbla_algo algo, gbla_stream_t stream);
+
+/*
+ * gbla_forward_host -- gbla_forward for callers whose tensors live in HOST
+ * memory (pinned for full copy speed; pageable works).  Same layouts as
+ * above, all pointers host pointers.  Copies the inputs to device scratch,
+ * runs the forward and copies rows t < L_b of o back, all enqueued on
+ * `stream`; the call then waits for the stream, so o is ready on return.
+ */
+gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
+                              const void *gate, const void *out_gate,
+                              const float *conv_w, const float *norm_w,
+                              const int32_t *seq_lens, void *o, int B, int H,
+                              int N, int D, gbla_dtype dtype,
+                              gbla_stream_t stream);
+
+/* Number of floats per (b, h) in a state buffer: D*D + D. */
+size_t gbla_state_floats(int D);
+
+/* RMSNorm epsilon used by the readout (1e-6; the paper leaves it unstated). */
+float gbla_rms_eps(void);
+
+/* Static description of a status code; never NULL. */
+const char *gbla_status_string(gbla_status status);
+
+/* Library version, e.g. "0.1.0". */
+const char *gbla_version(void);
+
+/* Frees cached per-device resources (none are required between calls). */
+void gbla_release(void);
+
+/* Number of kernels this library has enqueued since it was loaded, over all
+ * devices and threads (a counter for benchmarks and tests). */
+uint64_t gbla_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GBLA_H_ */

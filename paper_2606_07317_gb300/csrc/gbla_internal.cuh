@@ -1,0 +1,53 @@
+// Internal declarations shared by the C-ABI front end and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "gbla.h"
+
+namespace gbla {
+
+constexpr int kConvW = GBLA_CONV_WIDTH;
+constexpr float kRmsEps = 1e-6f;
+
+struct Problem {
+  int B, H, N, D;
+  gbla_dtype dtype;
+  const int32_t *seq_lens;  // device [B] or nullptr
+};
+
+// Floats in one partial-state record of a sequence chunk: m (chunk max of the
+// gate logits), l (sum of exp(a - m) over the chunk), z[D], S[D*D].
+inline size_t partial_floats(int D) { return 2 + (size_t)D + (size_t)D * D; }
+inline size_t state_floats(int D) { return (size_t)D * D + D; }
+
+// Counts every kernel this library enqueues (read by gbla_launch_count).
+void count_launch(unsigned n = 1);
+
+// ---- CUDA-core (SIMT) family: every dtype and D ---------------------------
+struct SimtPlan {
+  int chunk_len;  // tokens per partial
+  int n_chunks;   // partials per (b, h)
+};
+SimtPlan simt_plan(const Problem &p);
+size_t simt_partials_bytes(const Problem &p, const SimtPlan &plan);
+cudaError_t simt_state(const Problem &p, const SimtPlan &plan, const void *k,
+                       const void *v, const void *gate, const float *conv_w,
+                       float *partials, float *state, cudaStream_t st);
+cudaError_t simt_readout(const Problem &p, const void *q, const void *og,
+                         const float *conv_w, const float *norm_w,
+                         const float *state, void *o, cudaStream_t st);
+
+// ---- tensor-core (tcgen05 + TMA) family: bf16, D in {64, 128} -------------
+bool tc_supports(const Problem &p);
+size_t tc_workspace_bytes(const Problem &p);
+cudaError_t tc_state(const Problem &p, const void *k, const void *v,
+                     const void *gate, const float *conv_w, void *workspace,
+                     float *state, cudaStream_t st);
+cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
+                       const float *conv_w, const float *norm_w,
+                       const float *state, void *o, cudaStream_t st);
+
+}  // namespace gbla

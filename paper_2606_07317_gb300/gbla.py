@@ -1,0 +1,197 @@
+"""Thin ctypes binding of libgbla (the C ABI declared in include/gbla.h).
+
+Argument marshalling only: every step of the GBLA core runs in the library's
+CUDA kernels.  Tensors are torch tensors; device calls take CUDA tensors and
+enqueue on the current torch stream (or the stream given).  There is no CPU
+fallback: if the library is missing or fails to load, calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+GBLA_OK, GBLA_ERR_INVALID_ARG, GBLA_ERR_UNSUPPORTED, GBLA_ERR_ALLOC, GBLA_ERR_CUDA = range(5)
+GBLA_FP32, GBLA_BF16 = 0, 1
+ALGO_AUTO, ALGO_SIMT, ALGO_TC = 0, 1, 2
+CONV_WIDTH = 4
+
+EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_state", "gbla_readout",
+            "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
+            "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count"]
+
+_lock = threading.Lock()
+_lib = None
+
+_vp = ctypes.c_void_p
+_i = ctypes.c_int
+
+
+class GblaError(RuntimeError):
+    def __init__(self, status: int, fn: str):
+        self.status = status
+        super().__init__(f"{fn}: {status_string(status)} (status {status})")
+
+
+def lib_path() -> str:
+    return _build.LIB_PATH
+
+
+def load(path: str | None = None):
+    """Load libgbla.so (it must have been built; see __graft_entry__.build())."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or lib_path()
+        if not os.path.exists(p):
+            raise RuntimeError(f"CUDA library not built: {p} is missing "
+                               "(run `python -c 'import __graft_entry__ as g; g.build()'`)")
+        lib = ctypes.CDLL(p)
+        fwd = [_vp] * 9 + [_i] * 5
+        lib.gbla_forward.argtypes = fwd + [_vp]
+        lib.gbla_forward.restype = _i
+        lib.gbla_forward_ex.argtypes = fwd + [_i, _vp]
+        lib.gbla_forward_ex.restype = _i
+        lib.gbla_forward_host.argtypes = fwd + [_vp]
+        lib.gbla_forward_host.restype = _i
+        lib.gbla_state.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
+        lib.gbla_state.restype = _i
+        lib.gbla_readout.argtypes = [_vp] * 7 + [_i] * 6 + [_vp]
+        lib.gbla_readout.restype = _i
+        lib.gbla_state_floats.argtypes = [_i]
+        lib.gbla_state_floats.restype = ctypes.c_size_t
+        lib.gbla_rms_eps.argtypes = []
+        lib.gbla_rms_eps.restype = ctypes.c_float
+        lib.gbla_status_string.argtypes = [_i]
+        lib.gbla_status_string.restype = ctypes.c_char_p
+        lib.gbla_version.argtypes = []
+        lib.gbla_version.restype = ctypes.c_char_p
+        lib.gbla_release.argtypes = []
+        lib.gbla_release.restype = None
+        lib.gbla_launch_count.argtypes = []
+        lib.gbla_launch_count.restype = ctypes.c_uint64
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    return load().gbla_status_string(int(status)).decode()
+
+
+def rms_eps() -> float:
+    return float(load().gbla_rms_eps())
+
+
+def version() -> str:
+    return load().gbla_version().decode()
+
+
+def launch_count() -> int:
+    """Kernels the library has enqueued so far (all devices, all threads)."""
+    return int(load().gbla_launch_count())
+
+
+def state_floats(D: int) -> int:
+    return int(load().gbla_state_floats(int(D)))
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return GBLA_FP32
+    if t.dtype == torch.bfloat16:
+        return GBLA_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return t.data_ptr() or None
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return _vp(stream.cuda_stream)
+
+
+def _check(status: int, fn: str):
+    if status != GBLA_OK:
+        raise GblaError(status, fn)
+
+
+def _bhnd(q: torch.Tensor):
+    if q.dim() != 4:
+        raise ValueError("q must be [B, N, H, D]")
+    B, N, H, D = q.shape
+    return B, H, N, D
+
+
+def forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
+            algo: int = ALGO_AUTO, stream=None) -> torch.Tensor:
+    """o = GBLA core forward; tensors on one CUDA device, layouts of include/gbla.h."""
+    B, H, N, D = _bhnd(q)
+    if out is None:
+        out = torch.empty_like(q)
+    st = load().gbla_forward_ex(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
+        _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),
+        _stream(stream))
+    _check(st, "gbla_forward_ex")
+    return out
+
+
+def forward_default(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, out, stream=None):
+    """Direct call of gbla_forward (the AUTO entry point)."""
+    B, H, N, D = _bhnd(q)
+    st = load().gbla_forward(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
+        _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q),
+        _stream(stream))
+    _check(st, "gbla_forward")
+    return out
+
+
+def state(k, v, gate, conv_w, seq_lens=None, out=None, algo: int = ALGO_AUTO,
+          stream=None) -> torch.Tensor:
+    """[B, H, D*D + D] fp32: S (row-major) then z per (batch, head)."""
+    B, H, N, D = _bhnd(k)
+    if out is None:
+        out = torch.empty((B, H, D * D + D), dtype=torch.float32, device=k.device)
+    st = load().gbla_state(_ptr(k), _ptr(v), _ptr(gate), _ptr(conv_w), _ptr(seq_lens),
+                           _ptr(out), B, H, N, D, _dtype_code(k), int(algo),
+                           _stream(stream))
+    _check(st, "gbla_state")
+    return out
+
+
+def readout(q, out_gate, conv_w, norm_w, state_t, seq_lens=None, out=None,
+            algo: int = ALGO_AUTO, stream=None) -> torch.Tensor:
+    B, H, N, D = _bhnd(q)
+    if out is None:
+        out = torch.empty_like(q)
+    st = load().gbla_readout(_ptr(q), _ptr(out_gate), _ptr(conv_w), _ptr(norm_w),
+                             _ptr(seq_lens), _ptr(state_t), _ptr(out), B, H, N, D,
+                             _dtype_code(q), int(algo), _stream(stream))
+    _check(st, "gbla_readout")
+    return out
+
+
+def forward_host(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
+                 stream=None) -> torch.Tensor:
+    """Host-memory entry point: CPU tensors (pinned for full copy speed) in and out."""
+    B, H, N, D = _bhnd(q)
+    if out is None:
+        out = torch.empty_like(q)
+    st = load().gbla_forward_host(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
+        _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q),
+        _stream(stream))
+    _check(st, "gbla_forward_host")
+    return out

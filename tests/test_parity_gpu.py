@@ -1,0 +1,183 @@
+"""GPU path vs the fp64 oracle on the same seeded inputs, through the C ABI.
+
+Tolerances (see parity_util): fp32 max |d| / max(|y|, 1) <= 1e-4; bf16
+|d| <= 2e-2 + half a bf16 ulp of the true value.  Rows past a sequence's end
+must keep the sentinel the output was filled with.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_07317_gb300 import gbla
+from paper_2606_07317_gb300.workloads import WORKLOADS, custom, make_inputs
+from parity_util import compare, oracle_full, oracle_head, to64, valid_mask
+
+pytestmark = pytest.mark.gpu
+
+SENTINEL = -777.0
+ALGOS = {"auto": gbla.ALGO_AUTO, "simt": gbla.ALGO_SIMT}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    gbla.load()
+    torch.cuda.init()
+
+
+def _run(inp, algo=gbla.ALGO_AUTO):
+    out = torch.full_like(inp["q"], SENTINEL)
+    gbla.forward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"],
+                 inp["conv_w"], inp["norm_w"], inp["seq_lens"], out=out, algo=algo)
+    torch.cuda.synchronize()
+    return out
+
+
+def _check_against(y_gpu_t, y_ref, inp, dtype):
+    B, N = inp["q"].shape[:2]
+    sl = inp["seq_lens"]
+    mask = valid_mask(B, N, None if sl is None else sl.cpu().numpy())
+    y_gpu = to64(y_gpu_t)
+    st = compare(y_gpu[mask], y_ref[mask], dtype)
+    assert st["ok"], st
+    pad = y_gpu[~mask]
+    assert np.all(pad == np.float64(torch.tensor(SENTINEL, dtype=y_gpu_t.dtype).item())), \
+        "rows past the sequence end were written"
+    return st
+
+
+@pytest.mark.parametrize("algo", list(ALGOS), ids=list(ALGOS))
+@pytest.mark.parametrize("name", ["tiny_fp32_b1_h2_n256_d32", "bf16_b8_h8_n2048_d64",
+                                  "bf16_b4_h8_n8192_d64"])
+def test_parity_workload(name, algo):
+    w = WORKLOADS[name]
+    inp = make_inputs(w, "cuda")
+    y = _run(inp, ALGOS[algo])
+    _check_against(y, oracle_full(inp), inp, w.dtype)
+
+
+def test_parity_headline_n32768():
+    w = WORKLOADS["bf16_b2_h8_n32768_d64"]
+    inp = make_inputs(w, "cuda")
+    y = _run(inp)
+    _check_against(y, oracle_full(inp), inp, w.dtype)
+
+
+def test_parity_ragged_d128_sampled():
+    """Full-size ragged workload; the oracle runs on a sample of (batch, head)
+    pairs: the longest, the shortest and a middle sequence."""
+    w = WORKLOADS["bf16_ragged_b32_h8_d128"]
+    inp = make_inputs(w, "cuda")
+    y = _run(inp)
+    lens = np.array(w.seq_lens)
+    order = np.argsort(lens)
+    picks = [(int(order[-1]), 0), (int(order[0]), 3), (int(order[len(order) // 2]), 7)]
+    yc = y.cpu()
+    for b, h in picks:
+        L = int(lens[b])
+        ref = oracle_head(inp, b, h)
+        st = compare(to64(yc[b, :L, h]), ref, "bf16")
+        assert st["ok"], (b, h, st)
+    # padded rows untouched everywhere
+    for b in range(w.B):
+        L = int(lens[b])
+        assert torch.all(yc[b, L:] == torch.tensor(SENTINEL, dtype=yc.dtype))
+
+
+@pytest.mark.parametrize("algo", list(ALGOS), ids=list(ALGOS))
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("D", [32, 64, 128])
+def test_edge_lengths_and_garbage_padding(D, dtype, algo):
+    """Lengths 0..3 (shorter than the conv), a ragged tail, a full row; the
+    padding holds NaN and huge logits, which must not leak into valid rows."""
+    lens = [0, 1, 2, 3, 129, 333]
+    w = custom(B=len(lens), H=2, N=333, D=D, dtype=dtype, seed=7, seq_lens=lens)
+    inp = make_inputs(w, "cuda")
+    for b, L in enumerate(lens):
+        for name in ("q", "k", "v", "out_gate"):
+            inp[name][b, L:] = float("nan")
+        inp["gate"][b, L:] = 1e30 if dtype == "fp32" else 1e30
+    y = _run(inp, ALGOS[algo])
+    _check_against(y, oracle_full(inp), inp, dtype)
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_state_matches_oracle(dtype):
+    """gbla_state writes S = K^T V~ and z = K^T 1 with the true softmax gate."""
+    w = custom(B=2, H=3, N=1000, D=64, dtype=dtype, seed=11, seq_lens=[1000, 517])
+    inp = make_inputs(w, "cuda")
+    st = gbla.state(inp["k"], inp["v"], inp["gate"], inp["conv_w"], inp["seq_lens"])
+    torch.cuda.synchronize()
+    st = st.cpu().double().numpy()
+    tol = 1e-5 if dtype == "fp32" else 1e-2
+    for b in range(2):
+        for h in range(3):
+            _, inter = oracle_head(inp, b, h, intermediates=True)
+            S = st[b, h, :64 * 64].reshape(64, 64)
+            z = st[b, h, 64 * 64:]
+            assert np.abs(S - inter["S"]).max() <= tol * np.abs(inter["S"]).max()
+            assert np.abs(z - inter["z"]).max() <= tol * np.abs(inter["z"]).max()
+
+
+def test_readout_scale_invariant():
+    """A positive common scale of S and z cancels in the readout."""
+    w = custom(B=1, H=2, N=700, D=64, dtype="bf16", seed=12)
+    inp = make_inputs(w, "cuda")
+    st = gbla.state(inp["k"], inp["v"], inp["gate"], inp["conv_w"])
+    o1 = gbla.readout(inp["q"], inp["out_gate"], inp["conv_w"], inp["norm_w"], st)
+    o2 = gbla.readout(inp["q"], inp["out_gate"], inp["conv_w"], inp["norm_w"], st * 4.0)
+    torch.cuda.synchronize()
+    assert torch.equal(o1, o2)
+
+
+@pytest.mark.parametrize("name", ["bf16_b8_h8_n2048_d64", "tiny_fp32_b1_h2_n256_d32"])
+def test_deterministic(name):
+    inp = make_inputs(WORKLOADS[name], "cuda")
+    assert torch.equal(_run(inp), _run(inp))
+
+
+def test_large_gate_logits():
+    """Logits near the fp32 exp overflow limit: the max-rescaled gate is stable."""
+    w = custom(B=2, H=2, N=600, D=64, dtype="bf16", seed=13)
+    inp = make_inputs(w, "cuda")
+    inp["gate"].mul_(30.0).add_(500.0)
+    y = _run(inp)
+    _check_against(y, oracle_full(inp), inp, "bf16")
+
+
+def test_host_entry_matches_device():
+    w = custom(B=3, H=2, N=500, D=64, dtype="bf16", seed=14, seq_lens=[500, 77, 0])
+    inp = make_inputs(w, "cuda")
+    y_dev = _run(inp)
+    host = {k_: (v_.cpu().pin_memory() if v_ is not None else None) for k_, v_ in inp.items()}
+    out = torch.full_like(host["q"], SENTINEL).pin_memory()
+    gbla.forward_host(host["q"], host["k"], host["v"], host["gate"], host["out_gate"],
+                      host["conv_w"], host["norm_w"], host["seq_lens"], out=out)
+    assert torch.equal(out, y_dev.cpu())
+
+
+def test_empty_inputs_are_noops():
+    for shape in [(0, 5, 2, 64), (2, 0, 2, 64), (2, 5, 0, 64)]:
+        q = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
+        g = torch.empty(shape[:3], dtype=torch.bfloat16, device="cuda")
+        cw = torch.empty((3, shape[2], 64, 4), device="cuda")
+        nw = torch.empty((shape[2], 64), device="cuda")
+        gbla.forward(q, q, q, g, q, cw, nw, None, out=torch.empty_like(q))
+    torch.cuda.synchronize()
+
+
+def test_invalid_arguments_rejected():
+    w = custom(B=1, H=2, N=64, D=64, dtype="bf16", seed=15)
+    inp = make_inputs(w, "cuda")
+    args = [inp[n] for n in ("q", "k", "v", "gate", "out_gate", "conv_w", "norm_w")]
+    with pytest.raises(gbla.GblaError) as e:   # output aliases q
+        gbla.forward(*args, None, out=inp["q"])
+    assert e.value.status == gbla.GBLA_ERR_INVALID_ARG
+    flat = torch.empty(inp["q"].numel() + 8, dtype=torch.bfloat16, device="cuda")
+    mis = flat[1:1 + inp["q"].numel()].view_as(inp["q"])   # 2-byte offset
+    with pytest.raises(gbla.GblaError) as e:
+        gbla.forward(mis, *args[1:], None)
+    assert e.value.status == gbla.GBLA_ERR_INVALID_ARG
+    q48 = torch.zeros((1, 64, 2, 48), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(gbla.GblaError) as e:
+        gbla.forward(q48, q48, q48, inp["gate"], q48, inp["conv_w"], inp["norm_w"], None)
+    assert e.value.status == gbla.GBLA_ERR_UNSUPPORTED
