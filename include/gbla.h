@@ -140,6 +140,36 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
                               int N, int D, gbla_dtype dtype,
                               gbla_stream_t stream);
 
+/*
+ * gbla_state_static_scratch -- gbla_state for callers that cannot allocate
+ * GPU memory.  The paper has no counterpart: this is a deployment variant.
+ *
+ * Same arguments, layouts and result as gbla_state with the CUDA-core kernel
+ * family, but the partial sums live in a fixed array of
+ * GBLA_STATIC_SCRATCH_BYTES compiled into the library, so the call allocates
+ * nothing (no cudaMalloc, no pool, no library allocator).  Meant for callers
+ * whose device memory is entirely owned by another allocator, or who cannot
+ * take the latency of an allocation call.
+ *
+ * Limits and rules:
+ *   - B * H * (D*D + D + 2) * 4 bytes must fit in GBLA_STATIC_SCRATCH_BYTES
+ *     (at most 2015 (batch, head) pairs at D = 64, 508 at D = 128); larger
+ *     problems return GBLA_ERR_INVALID_ARG before anything is enqueued.  Long
+ *     sequences are cut into fewer, longer chunks to fit.
+ *   - Each GPU that loads the library holds the array until the process exits.
+ *   - The first call on a device looks up the array's device address on that
+ *     device (once); make that first call before any stream capture starts.
+ *   - Every call shares the one array.  Calls that overlap on the GPU (other
+ *     streams or threads) race on it: serialise them.  Nothing carries over
+ *     between calls; each call writes all the scratch it later reads.
+ */
+#define GBLA_STATIC_SCRATCH_BYTES (32u << 20)
+gbla_status gbla_state_static_scratch(const void *k, const void *v,
+                                      const void *gate, const float *conv_w,
+                                      const int32_t *seq_lens, float *state,
+                                      int B, int H, int N, int D,
+                                      gbla_dtype dtype, gbla_stream_t stream);
+
 /* Number of floats per (b, h) in a state buffer: D*D + D. */
 size_t gbla_state_floats(int D);
 

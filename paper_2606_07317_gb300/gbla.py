@@ -22,7 +22,8 @@ CONV_WIDTH = 4
 
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_state", "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
-            "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count"]
+            "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
+            "gbla_state_static_scratch"]
 
 _lock = threading.Lock()
 _lib = None
@@ -63,6 +64,8 @@ def load(path: str | None = None):
         lib.gbla_state.restype = _i
         lib.gbla_readout.argtypes = [_vp] * 7 + [_i] * 6 + [_vp]
         lib.gbla_readout.restype = _i
+        lib.gbla_state_static_scratch.argtypes = [_vp] * 6 + [_i] * 5 + [_vp]
+        lib.gbla_state_static_scratch.restype = _i
         lib.gbla_state_floats.argtypes = [_i]
         lib.gbla_state_floats.restype = ctypes.c_size_t
         lib.gbla_rms_eps.argtypes = []
@@ -194,4 +197,20 @@ def forward_host(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=Non
         _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q),
         _stream(stream))
     _check(st, "gbla_forward_host")
+    return out
+
+
+def state_static_scratch(k, v, gate, conv_w, seq_lens=None, out=None,
+                         stream=None) -> torch.Tensor:
+    """gbla_state without any GPU allocation: for callers that cannot allocate
+    device memory (its partial sums live in a fixed array inside the library;
+    see include/gbla.h for the size limit and the rule against overlapping
+    calls)."""
+    B, H, N, D = _bhnd(k)
+    if out is None:
+        out = torch.empty((B, H, D * D + D), dtype=torch.float32, device=k.device)
+    st = load().gbla_state_static_scratch(_ptr(k), _ptr(v), _ptr(gate), _ptr(conv_w),
+                                          _ptr(seq_lens), _ptr(out), B, H, N, D,
+                                          _dtype_code(k), _stream(stream))
+    _check(st, "gbla_state_static_scratch")
     return out
