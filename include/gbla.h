@@ -189,6 +189,13 @@ void gbla_release(void);
  * devices and threads (a counter for benchmarks and tests). */
 uint64_t gbla_launch_count(void);
 
+/* Error bits recorded on the current device by a tensor-core kernel whose
+ * bounded wait (2 s per wait) ran out; 0 when none did.  Such a kernel stops
+ * early, leaves its outputs undefined and keeps the CUDA context usable.  The
+ * call synchronises with the device; reset != 0 clears the word afterwards.
+ * Returns 0xFFFFFFFF if the word could not be read. */
+uint32_t gbla_device_error(int reset);
+
 #ifdef __cplusplus
 }
 #endif

@@ -143,6 +143,8 @@ void gbla_release(void) {}
 
 uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+uint32_t gbla_device_error(int reset) { return tc_device_error(reset != 0); }
+
 gbla_status gbla_state(const void *k, const void *v, const void *gate,
                        const float *conv_w, const int32_t *seq_lens, float *state,
                        int B, int H, int N, int D, gbla_dtype dtype, gbla_algo algo,

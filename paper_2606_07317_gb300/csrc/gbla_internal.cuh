@@ -49,5 +49,8 @@ cudaError_t tc_state(const Problem &p, const void *k, const void *v,
 cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
                        const float *conv_w, const float *norm_w,
                        const float *state, void *o, cudaStream_t st);
+// Error bits set by tensor-core kernels whose bounded waits ran out (0 = none);
+// synchronous read of the current device, optionally clearing it.
+unsigned tc_device_error(bool reset);
 
 }  // namespace gbla

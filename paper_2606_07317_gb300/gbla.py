@@ -23,7 +23,7 @@ CONV_WIDTH = 4
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_state", "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
-            "gbla_state_static_scratch"]
+            "gbla_state_static_scratch", "gbla_device_error"]
 
 _lock = threading.Lock()
 _lib = None
@@ -76,6 +76,8 @@ def load(path: str | None = None):
         lib.gbla_version.restype = ctypes.c_char_p
         lib.gbla_release.argtypes = []
         lib.gbla_release.restype = None
+        lib.gbla_device_error.argtypes = [_i]
+        lib.gbla_device_error.restype = ctypes.c_uint32
         lib.gbla_launch_count.argtypes = []
         lib.gbla_launch_count.restype = ctypes.c_uint64
         if path is None:
@@ -98,6 +100,11 @@ def version() -> str:
 def launch_count() -> int:
     """Kernels the library has enqueued so far (all devices, all threads)."""
     return int(load().gbla_launch_count())
+
+
+def device_error(reset: bool = False) -> int:
+    """Error bits left by a tensor-core kernel whose bounded wait ran out (0 = none)."""
+    return int(load().gbla_device_error(1 if reset else 0))
 
 
 def state_floats(D: int) -> int:

@@ -181,3 +181,36 @@ def test_invalid_arguments_rejected():
     with pytest.raises(gbla.GblaError) as e:
         gbla.forward(q48, q48, q48, inp["gate"], q48, inp["conv_w"], inp["norm_w"], None)
     assert e.value.status == gbla.GBLA_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_tensor_core_path_matches_simt_and_oracle(D):
+    """The tcgen05 family against the CUDA-core family and the oracle on a
+    ragged batch spanning several chunks and tiles; no bounded wait ran out."""
+    lens = [1500, 129, 1, 700]
+    w = custom(B=4, H=4, N=1500, D=D, dtype="bf16", seed=21, seq_lens=lens)
+    inp = make_inputs(w, "cuda")
+    gbla.device_error(reset=True)
+    y_tc = _run(inp, gbla.ALGO_TC)
+    y_simt = _run(inp, gbla.ALGO_SIMT)
+    assert gbla.device_error() == 0
+    ref = oracle_full(inp)
+    _check_against(y_tc, ref, inp, "bf16")
+    _check_against(y_simt, ref, inp, "bf16")
+
+
+def test_tensor_core_state_matches_oracle():
+    w = custom(B=2, H=3, N=3000, D=64, dtype="bf16", seed=22, seq_lens=[3000, 1111])
+    inp = make_inputs(w, "cuda")
+    st = gbla.state(inp["k"], inp["v"], inp["gate"], inp["conv_w"], inp["seq_lens"],
+                    algo=gbla.ALGO_TC)
+    torch.cuda.synchronize()
+    assert gbla.device_error() == 0
+    st = st.cpu().double().numpy()
+    for b in range(2):
+        for h in range(3):
+            _, inter = oracle_head(inp, b, h, intermediates=True)
+            S = st[b, h, :64 * 64].reshape(64, 64)
+            z = st[b, h, 64 * 64:]
+            assert np.abs(S - inter["S"]).max() <= 1e-2 * np.abs(inter["S"]).max()
+            assert np.abs(z - inter["z"]).max() <= 1e-2 * np.abs(inter["z"]).max()
