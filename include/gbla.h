@@ -196,6 +196,10 @@ uint64_t gbla_launch_count(void);
  * Returns 0xFFFFFFFF if the word could not be read. */
 uint32_t gbla_device_error(int reset);
 
+/* Text of the CUDA error behind the calling thread's last GBLA_ERR_CUDA
+ * ("no error" if there was none); static storage, never NULL. */
+const char *gbla_last_cuda_error(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -69,7 +69,14 @@ bool use_tc(const Problem &p, gbla_algo algo, gbla_status *st) {
   }
 }
 
-gbla_status from_cuda(cudaError_t e) { return e == cudaSuccess ? GBLA_OK : GBLA_ERR_CUDA; }
+thread_local cudaError_t t_last_cuda_error = cudaSuccess;
+
+gbla_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return GBLA_OK;
+  t_last_cuda_error = e;
+  (void)cudaGetLastError();  // clear the non-sticky launch error
+  return GBLA_ERR_CUDA;
+}
 
 // Stream-ordered scratch: freed on the same stream after the kernels using it.
 struct Scratch {
@@ -144,6 +151,8 @@ void gbla_release(void) {}
 uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 uint32_t gbla_device_error(int reset) { return tc_device_error(reset != 0); }
+
+const char *gbla_last_cuda_error(void) { return cudaGetErrorString(t_last_cuda_error); }
 
 gbla_status gbla_state(const void *k, const void *v, const void *gate,
                        const float *conv_w, const int32_t *seq_lens, float *state,

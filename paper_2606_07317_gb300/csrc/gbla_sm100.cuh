@@ -49,16 +49,28 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Abort flag of a CTA, held in shared memory (0 = running).
+struct AbortFlag {
+  uint32_t saddr;
+  __device__ __forceinline__ bool raised() const {
+    int r;
+    asm volatile("ld.volatile.shared.s32 %0, [%1];" : "=r"(r) : "r"(saddr) : "memory");
+    return r != 0;
+  }
+  __device__ __forceinline__ void raise() const {
+    asm volatile("st.volatile.shared.s32 [%0], %1;" ::"r"(saddr), "r"(1) : "memory");
+  }
+};
+
 // Waits for the phase with the given parity to complete.  Gives up (returns
-// false) once kWaitLimitNs has passed, or at once when `abort` is non-null and
-// *abort is set; the caller records the error and sets the abort flag.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
-                                          const volatile int *abort) {
-  if (abort != nullptr && *abort) return false;
+// false) once kWaitLimitNs has passed, or at once when `ab` is given and
+// raised; the caller records the error and raises the flag.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, const AbortFlag *ab) {
   if (mbar_try_wait(bar, parity)) return true;
+  if (ab != nullptr && ab->raised()) return false;
   const uint64_t t0 = globaltimer();
   while (!mbar_try_wait(bar, parity)) {
-    if ((abort != nullptr && *abort) || globaltimer() - t0 > kWaitLimitNs) return false;
+    if ((ab != nullptr && ab->raised()) || globaltimer() - t0 > kWaitLimitNs) return false;
   }
   return true;
 }
@@ -93,6 +105,16 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
                : "memory");
 }
 
+// 32 lanes x 32-bit, 8 consecutive columns (see tmem_ld16).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
+  uint32_t r[8];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]),
+                 "=r"(r[6]), "=r"(r[7])
+               : "r"(taddr));
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
 // 32 lanes x 32-bit, 16 consecutive columns: thread i of the warp gets lane
 // (warp's lane quarter base + i), columns [col, col + 16).
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
@@ -109,6 +131,14 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
 }
 __device__ __forceinline__ void tmem_ld_wait() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// tcgen05.wait::ld that also pins the loaded registers, so no use of them can
+// be scheduled before the wait.
+template <int N>
+__device__ __forceinline__ void tmem_ld_wait_regs(float (&v)[N]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
 }
 
 // ---------------------------------------------------------------- MMA
@@ -185,6 +215,15 @@ template <int n>
 __device__ __forceinline__ void tma_store_wait_all() {
   asm volatile("cp.async.bulk.wait_group %0;" ::"n"(n) : "memory");
 }
+// Hint: pull one box of a tensor map into L2.
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap *m, int c0, int c1, int c2,
+                                                   int c3) {
+  asm volatile(
+      "cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+          reinterpret_cast<uint64_t>(m)),
+      "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
 // Hint: pull [p, p + bytes) into L2 (16-byte aligned, bytes a multiple of 16).
 __device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
@@ -211,6 +250,19 @@ __device__ __forceinline__ void sts_v4(uint32_t saddr, uint4 v) {
                "r"(v.z), "r"(v.w)
                : "memory");
 }
+__device__ __forceinline__ float lds_f32(uint32_t saddr) {
+  float r;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(r) : "r"(saddr) : "memory");
+  return r;
+}
+__device__ __forceinline__ void sts_f32(uint32_t saddr, float v) {
+  asm volatile("st.shared.f32 [%0], %1;" ::"r"(saddr), "f"(v) : "memory");
+}
+__device__ __forceinline__ int lds_volatile_s32(uint32_t saddr) {
+  int r;
+  asm volatile("ld.volatile.shared.s32 %0, [%1];" : "=r"(r) : "r"(saddr) : "memory");
+  return r;
+}
 __device__ __forceinline__ uint4 lds_v4(uint32_t saddr) {
   uint4 r;
   asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
@@ -222,6 +274,16 @@ __device__ __forceinline__ uint4 lds_v4(uint32_t saddr) {
 // bf16 pair (low half = element 0) -> two floats
 __device__ __forceinline__ float2 bf2_to_f2(uint32_t u) {
   return make_float2(__uint_as_float(u << 16), __uint_as_float(u & 0xFFFF0000u));
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 // two floats -> bf16 pair, round to nearest even (element 0 in the low half)
 __device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {

@@ -54,20 +54,22 @@ using namespace sm100;
 constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the state
 
 // ------------------------------------------------------------------ state
-constexpr int kSWarps = 8;                      // producer warps
-constexpr int kSThreads = (kSWarps + 1) * 32;   // + 1 MMA warp
-constexpr int kSProd = kSWarps * 32;
-constexpr int kSTok = 32;                       // tokens per pipeline stage
+// 13 warps: at most 4 per SM sub-partition, so each thread may hold 128 registers.
+constexpr int kSKWarps = 6;                       // warps producing K^ (A operand)
+constexpr int kSProdWarps = 2 * kSKWarps;         // + 6 warps producing V~ hi/lo (B)
+constexpr int kSThreads = (kSProdWarps + 1) * 32; // + 1 MMA warp
+constexpr int kSProd = kSProdWarps * 32;
+constexpr int kSSub = 2 * kSKWarps;               // sub-streams (half-warps of a k-warp)
+constexpr int kSTokPerSub = 4;
+constexpr int kSTok = kSSub * kSTokPerSub;        // 48 tokens per pipeline stage
 constexpr int kSStages = 4;
-constexpr int kSSub = 16;                       // sub-streams (half-warps)
-constexpr int kSTokPerSub = kSTok / kSSub;      // 2
-constexpr int kChunkMax = 2048;                 // longest chunk (tokens)
+constexpr int kChunkMax = 2048;                   // longest chunk (tokens)
 constexpr int kMaxChunksPerSeq = 4096;
-constexpr int kSBlock = kSTok * 128;            // 64-channel MN block: 32 rows x 128 B
-constexpr int kSOp = 2 * kSBlock;               // one 128-channel operand
-constexpr int kSStageBytes = 3 * kSOp;          // A, B_hi, B_lo
+constexpr int kSBlock = kSTok * 128;              // 64-channel MN block: 48 rows x 128 B
+constexpr int kSOp = 2 * kSBlock;                 // one 128-channel operand
+constexpr int kSStageBytes = 3 * kSOp;            // A, B_hi, B_lo
 constexpr uint32_t kSTmemCols = 128;
-constexpr int kSPrefetch = 12;                  // L2 prefetch distance (tokens)
+constexpr int kSPrefetch = 16;                    // L2 prefetch distance (tokens)
 
 constexpr int kMaxBatch = 2048;
 
@@ -75,47 +77,71 @@ constexpr int kMaxBatch = 2048;
 constexpr int kSOffStages = 0;
 constexpr int kSOffGate = kSStages * kSStageBytes;               // float [2][kChunkMax]
 constexpr int kSOffZred = kSOffGate + 2 * kChunkMax * 4;         // float [kSSub][128]
-constexpr int kSOffRed = kSOffZred + kSSub * kGroupCh * 4;       // float [96]
-constexpr int kSOffPre = kSOffRed + 96 * 4;                      // int [kMaxBatch + 1]
+constexpr int kSOffRed = kSOffZred + kSSub * kGroupCh * 4;       // float [160]
+constexpr int kSOffPre = kSOffRed + 160 * 4;                     // int [kMaxBatch + 1]
 constexpr int kSOffBar = kSOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
 constexpr int kSBarCount = 2 * kSStages + 2;                      // full, empty, done, final
 constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;              // tmem addr, abort flag
 constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                // + alignment slack
+static_assert(kSSmemBytes <= 227 * 1024, "state shared memory");
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 
 // ------------------------------------------------------------------ readout
+// 18 warps: 8 producer, 8 epilogue (two per TMEM lane quarter), MMA, TMA.
+// At most 5 warps per SM sub-partition, so each thread may hold 96 registers.
 constexpr int kRTok = 128;                      // tokens per tile (MMA M)
-constexpr int kRThreads = 10 * 32;              // 4 producer, 4 epilogue, MMA, TMA warps
+constexpr int kRProdWarps = 8;
+constexpr int kREpiWarps = 8;
+constexpr int kRMmaWarp = kRProdWarps + kREpiWarps;   // 16
+constexpr int kRTmaWarp = kRMmaWarp + 1;              // 17
+constexpr int kRThreads = (kRTmaWarp + 1) * 32;       // 576
+constexpr int kRProd = kRProdWarps * 32;
+constexpr int kREpi = kREpiWarps * 32;
 constexpr int kRAStages = 2;
 constexpr int kRAccBufs = 2;
+constexpr int kRQRows = kRTok + 3;              // q tile rows: 3-token conv halo + tile
 
 template <int D>
 struct ReadoutCfg {
+  static constexpr bool QT = D == 64;                     // q through TMA (else 128-bit loads)
   static constexpr int NR = D + 16;                       // MMA N: D columns of S, z, zeros
   static constexpr int KB = D / 64;                       // 64-element K blocks
+  static constexpr int TPR = D / 8;                       // producer threads per token row
+  static constexpr int STREAMS = kRProd / TPR;            // producer sub-streams per tile
+  static constexpr int TPS = kRTok / STREAMS;             // tokens per sub-stream
   static constexpr int kABytes = kRTok * D * 2;           // one A tile
   static constexpr int kBBytes = NR * D * 2;              // one of B_hi / B_lo
-  static constexpr int kOgStages = D == 128 ? 2 : 3;
+  static constexpr int kOgStages = D == 128 ? 2 : 4;
   static constexpr int kOgBytes = kRTok * D * 2;
+  static constexpr int kQStages = QT ? 3 : 0;
+  static constexpr int kQTileBytes = kRQRows * 128;                  // one 64-channel block
+  static constexpr int kQBytes = (kQTileBytes + 1023) / 1024 * 1024;  // 1024-aligned stride
   static constexpr int kOffA = 0;
   static constexpr int kOffBhi = kOffA + kRAStages * kABytes;
   static constexpr int kOffBlo = kOffBhi + kBBytes;
   static constexpr int kOffOg = kOffBlo + kBBytes;
-  static constexpr int kOffPre = kOffOg + kOgStages * kOgBytes;  // int [kMaxBatch + 1]
-  static constexpr int kOffBar = kOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
-  // a_full[2], a_empty[2], og_full[S], og_empty[S], acc_full[2], acc_empty[2],
-  // b_full, b_free, final
-  static constexpr int kBars = 2 * kRAStages + 2 * kOgStages + 2 * kRAccBufs + 3;
+  static constexpr int kOffQ = kOffOg + kOgStages * kOgBytes;
+  static constexpr int kOffPre = kOffQ + kQStages * kQBytes;      // int [kMaxBatch + 1]
+  static constexpr int kOffSs = kOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;  // float [256]
+  static constexpr int kOffBar = kOffSs + kREpi * 4;
+  // a_full[2], a_empty[2], og_full[S], og_empty[S], q_full[Q], q_empty[Q],
+  // acc_full[2], acc_empty[2], b_full, b_free, final
+  static constexpr int kBars =
+      2 * kRAStages + 2 * kOgStages + 2 * kQStages + 2 * kRAccBufs + 3;
   static constexpr int kOffMisc = kOffBar + kBars * 8;
   static constexpr int kSmem = kOffMisc + 16 + 1024;
   static constexpr uint32_t kAccStride = NR <= 128 ? 128 : 256;  // column offset of buffer 1
   static constexpr uint32_t kTmemCols = kAccStride + NR <= 256 ? 256 : 512;
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kRTok, NR, 0, 0);
   static_assert(kSmem <= 227 * 1024, "readout shared memory");
+  static_assert(TPS % 4 == 0, "producer sub-streams are processed 4 tokens at a time");
 };
 
-__device__ __forceinline__ void report_error(unsigned code, volatile int *abort_flag) {
+__device__ __forceinline__ void report_error(unsigned code, const AbortFlag &ab) {
   atomicOr(&g_tc_error, code);
-  *abort_flag = 1;
+  ab.raise();
 }
 
 __device__ __forceinline__ int clamp_len(const int32_t *seq_lens, int b, int N) {
@@ -125,7 +151,7 @@ __device__ __forceinline__ int clamp_len(const int32_t *seq_lens, int b, int N) 
 }
 
 // Exclusive prefix over b of count(b) into pre[0..B], computed by the `nthr`
-// threads with tid < nthr (a multiple of 32, at most 256).  Ends with a named
+// threads with tid < nthr (a multiple of 32, at most 1024).  Ends with a named
 // barrier over those threads.
 template <typename CountFn>
 __device__ void prefix_counts(int *pre, int B, int tid, int nthr, uint32_t bar_id,
@@ -164,11 +190,6 @@ __device__ __forceinline__ int find_batch(const int *pre, int B, int k) {
   return lo;
 }
 
-// phi(x) = elu(x) + 1 = exp(min(x, 0)) + max(x, 0)
-__device__ __forceinline__ float phi_fast(float x) {
-  return __expf(fminf(x, 0.f)) + fmaxf(x, 0.f);
-}
-
 __device__ __forceinline__ void unpack8(const uint4 &r, float (&x)[8]) {
   const uint32_t w[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
@@ -179,7 +200,7 @@ __device__ __forceinline__ void unpack8(const uint4 &r, float (&x)[8]) {
   }
 }
 
-// Causal Conv1D of two channels: taps 0..2 on x[t-3..t-1], tap 3 on x[t].
+// Causal Conv1D of channels i, i+1: taps 0..2 on x[t-3..t-1], tap 3 on x[t].
 __device__ __forceinline__ float2 conv2(const float (&w)[4][8], const float (&xm)[3][8],
                                         const float (&x)[8], int i) {
   float2 a = __fmul2_rn(make_float2(w[0][i], w[0][i + 1]), make_float2(xm[0][i], xm[0][i + 1]));
@@ -195,6 +216,103 @@ __device__ __forceinline__ void slide(float (&xm)[3][8], const float (&x)[8]) {
     xm[0][i] = xm[1][i];
     xm[1][i] = xm[2][i];
     xm[2][i] = x[i];
+  }
+}
+
+// phi(x) = elu(x) + 1 for two channels given xl = x * log2(e):
+// exp(min(x, 0)) + max(x, 0) = 2^min(xl, 0) + ln2 * max(xl, 0).
+__device__ __forceinline__ float2 phi2_log2(float2 xl) {
+  const float2 e = make_float2(ex2_approx(fminf(xl.x, 0.f)), ex2_approx(fminf(xl.y, 0.f)));
+  return __ffma2_rn(make_float2(kLn2, kLn2), make_float2(fmaxf(xl.x, 0.f), fmaxf(xl.y, 0.f)), e);
+}
+
+// One token of a state producer: conv of 8 channels, then K^ (IS_K) or V~ hi/lo
+// written to the stage at shared address sa.  al = a' = (gate - m) log2(e) of
+// this token's head (-inf past the sub-stream end, which makes K^ = 0).
+template <bool IS_K>
+__device__ __forceinline__ void state_token(const float (&w)[4][8], float (&xm)[3][8],
+                                            const uint4 &raw, float al, float2 (&z)[4],
+                                            uint32_t sa) {
+  float x[8];
+  unpack8(raw, x);
+  if constexpr (IS_K) {
+    // K^ = 2^a' phi(k~) = 2^min(x' + a', a') + (2^a' ln 2) max(x', 0),  x' = k~ log2(e)
+    const float wl = ex2_approx(al) * kLn2;
+    uint32_t pk[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 xl = conv2(w, xm, x, 2 * i);
+      const float2 ts = __fadd2_rn(xl, make_float2(al, al));
+      const float2 e = make_float2(ex2_approx(fminf(ts.x, al)), ex2_approx(fminf(ts.y, al)));
+      const float2 kh =
+          __ffma2_rn(make_float2(wl, wl), make_float2(fmaxf(xl.x, 0.f), fmaxf(xl.y, 0.f)), e);
+      pk[i] = f2_to_bf2(kh.x, kh.y);
+      z[i] = __fadd2_rn(z[i], kh);
+    }
+    sts_v4(sa, make_uint4(pk[0], pk[1], pk[2], pk[3]));
+  } else {
+    // V~ as hi + lo bf16 (16 significant bits)
+    uint32_t ph[4], pl[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 cv = conv2(w, xm, x, 2 * i);
+      ph[i] = f2_to_bf2(cv.x, cv.y);
+      const float2 lo = __ffma2_rn(bf2_to_f2(ph[i]), make_float2(-1.f, -1.f), cv);
+      pl[i] = f2_to_bf2(lo.x, lo.y);
+    }
+    sts_v4(sa + kSOp, make_uint4(ph[0], ph[1], ph[2], ph[3]));
+    sts_v4(sa + 2 * kSOp, make_uint4(pl[0], pl[1], pl[2], pl[3]));
+  }
+  slide(xm, x);
+}
+
+// What a state producer thread needs to stream one chunk's sub-stream.
+struct SubStream {
+  const __nv_bfloat16 *xp;   // this thread's 8 channels at token 0
+  const __nv_bfloat16 *grp;  // the head group's row at token 0 (L2 prefetch)
+  size_t rs;                 // token stride (elements)
+  int s0, s1, tlast, t0;     // sub-stream [s0, s1), last loadable token, chunk start
+  uint32_t grow_bytes;       // bytes of one group row
+  uint32_t gw_s;             // shared address of this head's a' values
+  int nst;                   // pipeline stages of this chunk
+};
+
+// All stages of one chunk for one producer thread (k or v role, fixed per warp).
+template <bool IS_K>
+__device__ __forceinline__ void state_stream(const SubStream &ss, const float (&w)[4][8],
+                                             float (&xm)[3][8], float2 (&z)[4], uint32_t &gs,
+                                             uint64_t *full, uint64_t *empty,
+                                             const AbortFlag &ab, uint32_t stages_s,
+                                             uint32_t rbase, uint32_t sw, int c, int lane) {
+  auto ld = [&](int t) { return ldg_nc_v4(ss.xp + (size_t)min(t, ss.tlast) * ss.rs); };
+  auto alpha = [&](int t) {
+    const float a = lds_f32(ss.gw_s + (uint32_t)max(min(t, ss.s1 - 1) - ss.t0, 0) * 4);
+    return t < ss.s1 ? a : -INFINITY;
+  };
+  uint4 ra0 = ld(ss.s0), ra1 = ld(ss.s0 + 1);
+  for (int it = 0; it < ss.nst; ++it, ++gs) {
+    const int s = gs % kSStages;
+    if (!mbar_wait(&empty[s], ((gs / kSStages) & 1) ^ 1, &ab) && !ab.raised())
+      report_error(1, ab);
+    const uint32_t stage = stages_s + s * kSStageBytes + rbase;
+    const int tb = ss.s0 + it * kSTokPerSub;
+    const uint4 rb0 = ld(tb + 2), rb1 = ld(tb + 3);
+    if (c < kSTokPerSub && tb + kSPrefetch + c < ss.s1)
+      prefetch_l2(ss.grp + (size_t)(tb + kSPrefetch + c) * ss.rs, ss.grow_bytes);
+    float al[4] = {0.f, 0.f, 0.f, 0.f};
+    if constexpr (IS_K) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) al[u] = alpha(tb + u);
+    }
+    state_token<IS_K>(w, xm, ra0, al[0], z, stage + 0 * 128 + ((sw ^ 0) << 4));
+    state_token<IS_K>(w, xm, ra1, al[1], z, stage + 1 * 128 + ((sw ^ 1) << 4));
+    ra0 = ld(tb + 4);
+    ra1 = ld(tb + 5);
+    state_token<IS_K>(w, xm, rb0, al[2], z, stage + 2 * 128 + ((sw ^ 2) << 4));
+    state_token<IS_K>(w, xm, rb1, al[3], z, stage + 3 * 128 + ((sw ^ 3) << 4));
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&full[s]);
   }
 }
 
@@ -214,26 +332,26 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
   constexpr int REC = D * D + D + 4;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float *gw = (float *)(smem + kSOffGate);           // [G][kChunkMax]
-  float *zred = (float *)(smem + kSOffZred);         // [kSSub][128]
-  float *red = (float *)(smem + kSOffRed);           // [0,32) max, [32,64) sum, 64+ m, 68+ l
+  float *gw = (float *)(smem + kSOffGate);   // [G][kChunkMax]: a' = (a - m) log2(e)
+  float *zred = (float *)(smem + kSOffZred); // [kSSub][128]
+  float *red = (float *)(smem + kSOffRed);   // [0,64) max, [64,128) sum, 128+ m, 136+ l
   int *pre = (int *)(smem + kSOffPre);
   uint64_t *bars = (uint64_t *)(smem + kSOffBar);
   uint64_t *full = bars, *empty = bars + kSStages, *done = bars + 2 * kSStages,
            *fin = bars + 2 * kSStages + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + kSOffMisc);
-  volatile int *abort_flag = (volatile int *)(smem + kSOffMisc + 4);
+  const AbortFlag ab{smem_u32(smem + kSOffMisc + 4)};
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, H = p.H, N = p.N, S = p.S, HG = p.HG;
 
   if (tid == 0) {
-    *abort_flag = 0;
-    for (int i = 0; i < kSBarCount; ++i) mbar_init(&bars[i], i < kSStages ? kSWarps : 1);
+    *(volatile int *)(smem + kSOffMisc + 4) = 0;
+    for (int i = 0; i < kSBarCount; ++i) mbar_init(&bars[i], i < kSStages ? kSProdWarps : 1);
     fence_mbar_init();
   }
   // Chunk prefix over the batch (producer threads), shared by all roles.
-  if (warp < kSWarps) {
+  if (warp < kSProdWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
       const int L = clamp_len(p.seq_lens, b, N);
       return HG * ((L + S - 1) / S);
@@ -248,19 +366,27 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
   grid_dep_launch();
   if (c0 >= c1) return;  // no chunks for this CTA
 
-  if (warp == kSWarps) tmem_alloc(tmem_slot, kSTmemCols);
+  if (warp == kSProdWarps) tmem_alloc(tmem_slot, kSTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp < kSWarps) {
+  if (warp < kSProdWarps) {
     // ------------------------------------------------------------ producers
-    const int half = lane >> 4, c = lane & 15;       // c: 8-channel chunk of the group
-    const int sub = warp * 2 + half;                 // sub-stream 0..15
-    const int hh = (8 * c) / D, d0 = 8 * c - D * hh; // head within group, first channel
-    const int blk = c >> 3, cc = c & 7;              // MN block, 16-byte chunk in block
-    uint32_t gs = 0;                                 // stage counter across chunks
+    const bool is_k = warp < kSKWarps;                // k-warps write A, v-warps write B
+    const int half = lane >> 4, c = lane & 15;        // c: 8-channel chunk of the group
+    const int sub = (warp % kSKWarps) * 2 + half;     // sub-stream 0..11
+    const int hh = (8 * c) / D, d0 = 8 * c - D * hh;  // head within group, first channel
+    const int blk = c >> 3, cc = c & 7;               // MN block, 16-byte chunk in block
+    const int tens = is_k ? 1 : 2;                    // conv_w stream: 1 = k, 2 = v
+    const __nv_bfloat16 *src = is_k ? p.k : p.v;
+    // stage-relative byte offset of this thread's 16 bytes in row sub*4 + u:
+    // rows of one sub-stream share an 8-row group; swizzle chunk = cc ^ (row & 7)
+    const uint32_t rbase = blk * kSBlock + (sub >> 1) * 1024 + (sub & 1) * 512;
+    const uint32_t sw = (uint32_t)(cc ^ ((sub & 1) * 4));
+    const uint32_t gw_s = smem_u32(gw) + hh * kChunkMax * 4;
+    uint32_t gs = 0;                                  // stage counter across chunks
     int nchunk = 0;
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
@@ -272,15 +398,15 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
       const int t0 = j * S, t1 = min(t0 + S, L), n = t1 - t0;
       const int hbase = hg * G;
 
-      // Gate pre-pass: chunk maximum and weights per head (thread's head = tid % G).
+      // Gate pre-pass: per-head chunk maximum m, a' = (a - m) log2(e), l = sum 2^a'.
       {
         const int myh = tid % G;
-        const int hglob = hbase + myh;
+        const bool hok = hbase + myh < H;
         float m = -INFINITY;
         for (int idx = tid; idx < n * G; idx += kSProd) {
           const int tt = idx / G;
           float a = -INFINITY;
-          if (hglob < H) a = __bfloat162float(p.gate[((size_t)b * N + t0 + tt) * H + hglob]);
+          if (hok) a = __bfloat162float(p.gate[((size_t)b * N + t0 + tt) * H + hbase + myh]);
           gw[myh * kChunkMax + tt] = a;
           m = fmaxf(m, a);
         }
@@ -289,156 +415,92 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
         if (lane < G) red[warp * 4 + lane] = m;
         named_barrier(1, kSProd);
         float M = red[myh];
-        for (int w = 1; w < kSWarps; ++w) M = fmaxf(M, red[w * 4 + myh]);
+        for (int w = 1; w < kSProdWarps; ++w) M = fmaxf(M, red[w * 4 + myh]);
         float l = 0.f;
         for (int idx = tid; idx < n * G; idx += kSProd) {
           const int tt = idx / G;
-          const float a = gw[myh * kChunkMax + tt];
-          const float w = (hglob < H) ? __expf(a - M) : 0.f;
-          gw[myh * kChunkMax + tt] = w;
-          l += w;
+          const float al = hok ? (gw[myh * kChunkMax + tt] - M) * kLog2e : -INFINITY;
+          gw[myh * kChunkMax + tt] = al;
+          l += ex2_approx(al);
         }
 #pragma unroll
         for (int o = 16; o >= G; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-        if (lane < G) red[32 + warp * 4 + lane] = l;
+        if (lane < G) red[64 + warp * 4 + lane] = l;
         named_barrier(1, kSProd);
         if (tid < G) {  // m and l of this chunk, per head, for the records
           float lt = 0.f;
-          for (int w = 0; w < kSWarps; ++w) lt += red[32 + w * 4 + tid];
-          red[64 + tid] = M;
-          red[68 + tid] = lt;
+          for (int w = 0; w < kSProdWarps; ++w) lt += red[64 + w * 4 + tid];
+          red[128 + tid] = M;
+          red[136 + tid] = lt;
         }
       }
 
-      // This thread's channels: group channels [8c, 8c+8) of k and v.
+      // This thread: channels [8c, 8c+8) of the group, of k or of v.
       const int h = hbase + hh;
       const bool hv = h < H;
-      const size_t rs = (size_t)H * D;  // token stride
-      const __nv_bfloat16 *kp = p.k + ((size_t)b * N * H + (hv ? h : 0)) * D + d0;
-      const __nv_bfloat16 *vp = p.v + ((size_t)b * N * H + (hv ? h : 0)) * D + d0;
-      float wk[4][8], wv[4][8];
+      const size_t rs = (size_t)H * D;  // token stride (elements)
+      const __nv_bfloat16 *xp = src + ((size_t)b * N * H + (hv ? h : 0)) * D + d0;
+      // taps; for k pre-scaled by log2(e) so the conv yields x * log2(e) directly
+      float w[4][8];
+      const float wsc = is_k ? kLog2e : 1.f;
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          wk[q][i] = hv ? p.conv_w[((size_t)(1 * H + h) * D + d0 + i) * 4 + q] : 0.f;
-          wv[q][i] = hv ? p.conv_w[((size_t)(2 * H + h) * D + d0 + i) * 4 + q] : 0.f;
-        }
+        for (int q = 0; q < 4; ++q)
+          w[q][i] = hv ? p.conv_w[((size_t)(tens * H + h) * D + d0 + i) * 4 + q] * wsc : 0.f;
       const int s0 = t0 + (int)((long long)n * sub / kSSub);
       const int s1 = t0 + (int)((long long)n * (sub + 1) / kSSub);
-      float km[3][8], vm[3][8];  // sliding windows x[t-3], x[t-2], x[t-1]
+      const int tlast = max(min(s1, L) - 1, 0);  // loads past the sub-stream repeat this row
+      float xm[3][8];  // sliding window x[t-3], x[t-2], x[t-1]
 #pragma unroll
       for (int q = 0; q < 3; ++q) {
         const int t = s0 - 3 + q;
-        uint4 rk = make_uint4(0, 0, 0, 0), rv = rk;
-        if (hv && t >= 0 && s0 < s1) {
-          rk = ldg_nc_v4(kp + (size_t)t * rs);
-          rv = ldg_nc_v4(vp + (size_t)t * rs);
-        }
-        float xk[8], xv[8];
-        unpack8(rk, xk);
-        unpack8(rv, xv);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          km[q][i] = xk[i];
-          vm[q][i] = xv[i];
-        }
+        uint4 rw = make_uint4(0, 0, 0, 0);
+        if (t >= 0 && s0 < s1) rw = ldg_nc_v4(xp + (size_t)t * rs);
+        unpack8(rw, xm[q]);
       }
-      float zacc[8];
+      float2 z[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) zacc[i] = 0.f;
-      const float *gwh = gw + hh * kChunkMax;
+      for (int i = 0; i < 4; ++i) z[i] = make_float2(0.f, 0.f);
       const int nst = ((n + kSSub - 1) / kSSub + kSTokPerSub - 1) / kSTokPerSub;
       const uint32_t grow_bytes = (uint32_t)(min(G, H - hbase) * D * 2);
-      const __nv_bfloat16 *kgrp = p.k + ((size_t)b * N * H + hbase) * D;
-      const __nv_bfloat16 *vgrp = p.v + ((size_t)b * N * H + hbase) * D;
+      const __nv_bfloat16 *grp = src + ((size_t)b * N * H + hbase) * D;
       if (c == 0)  // warm L2 with the first tokens of this sub-stream
-        for (int t = s0; t < min(s1, s0 + kSPrefetch); ++t) {
-          prefetch_l2(kgrp + (size_t)t * rs, grow_bytes);
-          prefetch_l2(vgrp + (size_t)t * rs, grow_bytes);
-        }
+        for (int t = s0; t < min(s1, s0 + kSPrefetch); ++t)
+          prefetch_l2(grp + (size_t)t * rs, grow_bytes);
+      const SubStream sst{xp, grp, rs, s0, s1, tlast, t0, grow_bytes, gw_s, nst};
+      const uint32_t stages_s = smem_u32(smem + kSOffStages);
+      if (is_k)
+        state_stream<true>(sst, w, xm, z, gs, full, empty, ab, stages_s, rbase, sw, c, lane);
+      else
+        state_stream<false>(sst, w, xm, z, gs, full, empty, ab, stages_s, rbase, sw, c, lane);
 
-      for (int it = 0; it < nst; ++it, ++gs) {
-        const int s = gs % kSStages;
-        if (!mbar_wait(&empty[s], ((gs / kSStages) & 1) ^ 1, abort_flag) && !*abort_flag)
-          report_error(1, abort_flag);
-        const uint32_t stage = smem_u32(smem + kSOffStages + s * kSStageBytes);
-        uint4 rk[kSTokPerSub], rv[kSTokPerSub];
+      // z of this chunk: the sub-streams summed in a fixed order.
+      if (is_k) {
 #pragma unroll
-        for (int u = 0; u < kSTokPerSub; ++u) {
-          const int t = s0 + it * kSTokPerSub + u;
-          rk[u] = make_uint4(0, 0, 0, 0);
-          rv[u] = rk[u];
-          if (hv && t < s1) {
-            rk[u] = ldg_nc_v4(kp + (size_t)t * rs);
-            rv[u] = ldg_nc_v4(vp + (size_t)t * rs);
-          }
-          const int tp = t + kSPrefetch;
-          if (c == 0 && tp < s1) {
-            prefetch_l2(kgrp + (size_t)tp * rs, grow_bytes);
-            prefetch_l2(vgrp + (size_t)tp * rs, grow_bytes);
-          }
+        for (int i = 0; i < 4; ++i) {
+          zred[sub * kGroupCh + 8 * c + 2 * i] = z[i].x;
+          zred[sub * kGroupCh + 8 * c + 2 * i + 1] = z[i].y;
         }
-#pragma unroll
-        for (int u = 0; u < kSTokPerSub; ++u) {
-          const int t = s0 + it * kSTokPerSub + u;
-          const bool valid = hv && t < s1;
-          float xk[8], xv[8];
-          unpack8(rk[u], xk);
-          unpack8(rv[u], xv);
-          const float wgt = valid ? gwh[t - t0] : 0.f;
-          uint32_t pk[4], ph[4], pl[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 ck = conv2(wk, km, xk, 2 * i);
-            const float2 cv = conv2(wv, vm, xv, 2 * i);
-            // K^ = w * phi(k~); rows past the sub-stream end are zero
-            const float k0 = valid ? wgt * phi_fast(ck.x) : 0.f;
-            const float k1 = valid ? wgt * phi_fast(ck.y) : 0.f;
-            pk[i] = f2_to_bf2(k0, k1);
-            const float2 kr = bf2_to_f2(pk[i]);  // z sums exactly what the MMA sees
-            zacc[2 * i] += kr.x;
-            zacc[2 * i + 1] += kr.y;
-            const float v0 = valid ? cv.x : 0.f, v1 = valid ? cv.y : 0.f;
-            ph[i] = f2_to_bf2(v0, v1);
-            const float2 vr = bf2_to_f2(ph[i]);
-            pl[i] = f2_to_bf2(v0 - vr.x, v1 - vr.y);
-          }
-          slide(km, xk);
-          slide(vm, xv);
-          // row of this token in the stage; MN-major, 128-byte swizzle
-          const int row = sub * kSTokPerSub + u;
-          const uint32_t sa = stage + blk * kSBlock + (row >> 3) * 1024 + (row & 7) * 128 +
-                              ((cc ^ (row & 7)) << 4);
-          sts_v4(sa, make_uint4(pk[0], pk[1], pk[2], pk[3]));
-          sts_v4(sa + kSOp, make_uint4(ph[0], ph[1], ph[2], ph[3]));
-          sts_v4(sa + 2 * kSOp, make_uint4(pl[0], pl[1], pl[2], pl[3]));
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&full[s]);
       }
-
-      // z of this chunk: the 16 sub-streams summed in a fixed order.
-#pragma unroll
-      for (int i = 0; i < 8; ++i) zred[sub * kGroupCh + 8 * c + i] = zacc[i];
       named_barrier(1, kSProd);
       float zsum = 0.f;
       if (tid < kGroupCh)
         for (int q = 0; q < kSSub; ++q) zsum += zred[q * kGroupCh + tid];
 
       // Wait for this chunk's accumulator, then write the partial records.
-      if (!mbar_wait(done, nchunk & 1, abort_flag) && !*abort_flag) report_error(2, abort_flag);
+      if (!mbar_wait(done, nchunk & 1, &ab) && !ab.raised()) report_error(2, ab);
       tc_fence_after();
-      {
-        const int q4 = warp & 3, colhalf = warp >> 2;
-        const int ch = 32 * q4 + lane;               // TMEM lane = group channel (row of S)
+      if (warp < 8) {  // two warps per TMEM lane quarter, half of the columns each
+        constexpr int CPW = D / 2;                    // columns per warp
+        const int q4 = warp & 3, part = warp >> 2;    // lane quarter, column half
+        const int ch = 32 * q4 + lane;                // TMEM lane = group channel (row of S)
         const int hh2 = ch / D, d = ch - D * hh2;
-        const int col0 = D * hh2 + colhalf * (D / 2);
+        const int col0 = D * hh2 + part * CPW;
         const bool ok2 = hbase + hh2 < H;
-        float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + colhalf * (D / 2);
+        float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + part * CPW;
 #pragma unroll
-        for (int cb = 0; cb < D / 2; cb += 16) {
+        for (int cb = 0; cb < CPW; cb += 16) {
           float vals[16];
           tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(col0 + cb), vals);
           tmem_ld_wait();
@@ -455,8 +517,8 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
             float *rz = p.records + ((size_t)k * G + hz) * REC;
             rz[D * D + dz] = zsum;
             if (dz == 0) {
-              rz[D * D + D] = red[64 + hz];
-              rz[D * D + D + 1] = red[68 + hz];
+              rz[D * D + D] = red[128 + hz];
+              rz[D * D + D + 1] = red[136 + hz];
             }
           }
         }
@@ -479,8 +541,8 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
       const int nst = ((n + kSSub - 1) / kSSub + kSTokPerSub - 1) / kSTokPerSub;
       for (int it = 0; it < nst; ++it, ++gs) {
         const int s = gs % kSStages;
-        if (!mbar_wait(&full[s], (gs / kSStages) & 1, abort_flag)) {
-          if (!*abort_flag) report_error(4, abort_flag);
+        if (!mbar_wait(&full[s], (gs / kSStages) & 1, &ab)) {
+          if (!ab.raised()) report_error(4, ab);
           ok = false;
           break;
         }
@@ -500,10 +562,10 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
       if (ok) mma_commit(done);
     }
     mma_commit(fin);  // every MMA issued above has completed once this arrives
-    if (!mbar_wait(fin, 0, nullptr)) report_error(8, abort_flag);
+    if (!mbar_wait(fin, 0, nullptr)) report_error(8, ab);
   }
   __syncthreads();
-  if (warp == kSWarps) {
+  if (warp == kSProdWarps) {
     tc_fence_after();
     tmem_dealloc(tmem, kSTmemCols);
   }
@@ -519,6 +581,7 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict_
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
+  constexpr int EPT = 4;  // elements per thread
   __shared__ float s_scale[kMaxChunksPerSeq];
   __shared__ float s_l;
   grid_dep_wait();
@@ -545,11 +608,22 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict_
     }
   }
   __syncthreads();
-  const int e = blockIdx.y * 256 + threadIdx.x;
-  if (e >= F) return;
-  float acc = 0.f;
-  for (int j = 0; j < nck; ++j) acc = fmaf(s_scale[j], rec0[j * rstride + e], acc);
-  state[(size_t)bh * F + e] = s_l > 0.f ? acc / s_l : 0.f;
+  const int e0 = (blockIdx.y * 256 + threadIdx.x) * EPT;
+  if (e0 >= F) return;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  const float *src = rec0 + e0;
+#pragma unroll 8
+  for (int j = 0; j < nck; ++j) {
+    const float4 v = __ldg((const float4 *)(src + j * rstride));
+    const float sc = s_scale[j];
+    acc.x = fmaf(sc, v.x, acc.x);
+    acc.y = fmaf(sc, v.y, acc.y);
+    acc.z = fmaf(sc, v.z, acc.z);
+    acc.w = fmaf(sc, v.w, acc.w);
+  }
+  const float inv = s_l > 0.f ? 1.f / s_l : 0.f;
+  float4 *dst = (float4 *)(state + (size_t)bh * F + e0);
+  *dst = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
 }
 
 // ===================================================================== readout
@@ -562,50 +636,81 @@ struct ReadoutParams {
   float eps;
 };
 
+// phi(conv(q)) for 4 consecutive rows of one producer sub-stream; xm holds the
+// window before the first row; rows are read by `row_raw(u)` (u = 0..3).
+template <typename RowFn>
+__device__ __forceinline__ void readout_rows4(const float (&wq)[4][8], float (&xm)[3][8],
+                                              RowFn row_raw, uint32_t abase, int row0, int kb,
+                                              int cc) {
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    float x[8];
+    unpack8(row_raw(u), x);
+    uint32_t pq[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 ph = phi2_log2(conv2(wq, xm, x, 2 * i));
+      pq[i] = f2_to_bf2(ph.x, ph.y);
+    }
+    slide(xm, x);
+    const int row = row0 + u;
+    const uint32_t off = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 +
+                         ((cc ^ (row & 7)) << 4);
+    sts_v4(abase + off, make_uint4(pq[0], pq[1], pq[2], pq[3]));
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kRThreads, 1)
     tc_readout_kernel(const ReadoutParams p, const __grid_constant__ CUtensorMap tm_og,
-                      const __grid_constant__ CUtensorMap tm_o) {
+                      const __grid_constant__ CUtensorMap tm_o,
+                      const __grid_constant__ CUtensorMap tm_q) {
   using C = ReadoutCfg<D>;
   constexpr int NR = C::NR;
   constexpr int OGS = C::kOgStages;
+  constexpr int QS = C::kQStages > 0 ? C::kQStages : 1;
   constexpr int F = D * D + D;
+  constexpr int CPE = D / 2;  // columns per epilogue warp
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   int *pre = (int *)(smem + C::kOffPre);
   uint64_t *bars = (uint64_t *)(smem + C::kOffBar);
   uint64_t *a_full = bars, *a_empty = bars + 2, *og_full = bars + 4, *og_empty = og_full + OGS,
-           *acc_full = og_empty + OGS, *acc_empty = acc_full + 2, *b_full = acc_empty + 2,
-           *b_free = b_full + 1, *fin = b_free + 1;
+           *q_full = og_empty + OGS, *q_empty = q_full + C::kQStages,
+           *acc_full = q_empty + C::kQStages, *acc_empty = acc_full + 2,
+           *b_full = acc_empty + 2, *b_free = b_full + 1, *fin = b_free + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + C::kOffMisc);
-  volatile int *abort_flag = (volatile int *)(smem + C::kOffMisc + 4);
+  const AbortFlag ab{smem_u32(smem + C::kOffMisc + 4)};
   __shared__ int s_tot[8];
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, H = p.H, N = p.N;
 
   if (tid == 0) {
-    *abort_flag = 0;
-    mbar_init(&a_full[0], 4);
-    mbar_init(&a_full[1], 4);
-    mbar_init(&a_empty[0], 1);
-    mbar_init(&a_empty[1], 1);
+    *(volatile int *)(smem + C::kOffMisc + 4) = 0;
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&a_full[i], kRProdWarps);
+      mbar_init(&a_empty[i], 1);
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kREpiWarps);
+    }
     for (int i = 0; i < OGS; ++i) {
       mbar_init(&og_full[i], 1);
       mbar_init(&og_empty[i], 1);
     }
-    mbar_init(&acc_full[0], 1);
-    mbar_init(&acc_full[1], 1);
-    mbar_init(&acc_empty[0], 4);
-    mbar_init(&acc_empty[1], 4);
-    mbar_init(b_full, 4);
+    for (int i = 0; i < C::kQStages; ++i) {
+      mbar_init(&q_full[i], 1);
+      mbar_init(&q_empty[i], kRProdWarps);
+    }
+    mbar_init(b_full, kRProdWarps);
     mbar_init(b_free, 1);
     mbar_init(fin, 1);
     fence_mbar_init();
   }
-  if (warp == 9 && lane == 0) {
+  if (warp == kRTmaWarp && lane == 0) {
     tma_prefetch_desc(&tm_og);
     tma_prefetch_desc(&tm_o);
+    tma_prefetch_desc(&tm_q);
   }
   // Everything below may read what earlier work on the stream wrote.
   grid_dep_wait();
@@ -620,7 +725,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
   const long long i0 = (long long)T * blockIdx.x / gridDim.x;
   const long long i1 = (long long)T * (blockIdx.x + 1) / gridDim.x;
   if (i0 >= i1) return;
-  if (warp == 8) tmem_alloc(tmem_slot, C::kTmemCols);
+  if (warp == kRMmaWarp) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -638,11 +743,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
     nrow = min(kRTok, L - r0);
   };
 
-  if (warp < 4) {
+  if (warp < kRProdWarps) {
     // ------------------------------------------------------------ producers: phi(conv(q))
-    constexpr int TPR = D / 8;            // threads per token row
-    constexpr int STREAMS = 128 / TPR;    // sub-streams per tile
-    constexpr int TPS = kRTok / STREAMS;  // tokens per sub-stream
+    constexpr int TPR = C::TPR, TPS = C::TPS;
     const int c = tid % TPR, stream = tid / TPR;
     const int kb = c >> 3, cc = c & 7;
     int cur_b = -1, cur_h = -1, nbh = 0;
@@ -654,10 +757,10 @@ __global__ void __launch_bounds__(kRThreads, 1)
       if (b != cur_b || h != cur_h) {
         // New (b, h): rebuild B = [S | z | 0] as bf16 hi/lo, K-major, 128B swizzle,
         // once the MMAs that read the previous one have completed.
-        if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, abort_flag) && !*abort_flag)
-          report_error(16, abort_flag);
+        if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, &ab) && !ab.raised())
+          report_error(16, ab);
         const float *st = p.state + ((size_t)b * H + h) * F;
-        for (int item = tid; item < NR * (D / 8); item += 128) {
+        for (int item = tid; item < NR * (D / 8); item += kRProd) {
           const int e = item % NR, ck = item / NR;  // row e of B, 8-element K chunk ck
           float vals[8];
 #pragma unroll
@@ -669,8 +772,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             hi[i] = f2_to_bf2(vals[2 * i], vals[2 * i + 1]);
-            const float2 hr = bf2_to_f2(hi[i]);
-            lo[i] = f2_to_bf2(vals[2 * i] - hr.x, vals[2 * i + 1] - hr.y);
+            const float2 r2 = __ffma2_rn(bf2_to_f2(hi[i]), make_float2(-1.f, -1.f),
+                                         make_float2(vals[2 * i], vals[2 * i + 1]));
+            lo[i] = f2_to_bf2(r2.x, r2.y);
           }
           const int kbk = ck >> 3, ckk = ck & 7;
           const uint32_t off = kbk * (NR * 128) + (e >> 3) * 1024 + (e & 7) * 128 +
@@ -681,152 +785,203 @@ __global__ void __launch_bounds__(kRThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(b_full);
+        // q taps, pre-scaled by log2(e) (phi2_log2 takes x log2(e))
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
           for (int q = 0; q < 4; ++q)
-            wq[q][i] = p.conv_w[((size_t)(0 * H + h) * D + 8 * c + i) * 4 + q];
+            wq[q][i] = p.conv_w[((size_t)(0 * H + h) * D + 8 * c + i) * 4 + q] * kLog2e;
         cur_b = b;
         cur_h = h;
         ++nbh;
       }
       const int sa = li & 1;
-      if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, abort_flag) && !*abort_flag)
-        report_error(32, abort_flag);
-      const size_t rs = (size_t)H * D;
-      const __nv_bfloat16 *qp = p.q + ((size_t)b * N * H + h) * D + 8 * c;
-      const int ts = r0 + stream * TPS;  // first token of this sub-stream
-      uint4 raw[TPS + 3];
-#pragma unroll
-      for (int u = 0; u < TPS + 3; ++u) {
-        const int t = ts - 3 + u;
-        raw[u] = make_uint4(0, 0, 0, 0);
-        if (t >= 0 && t < r0 + nrow) raw[u] = ldg_nc_v4(qp + (size_t)t * rs);
-      }
-      float xm[3][8];
-#pragma unroll
-      for (int u = 0; u < 3; ++u) {
-        float x[8];
-        unpack8(raw[u], x);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) xm[u][i] = x[i];
-      }
+      if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab) && !ab.raised())
+        report_error(32, ab);
       const uint32_t abase = smem_u32(smem + C::kOffA + sa * C::kABytes);
+      float xm[3][8];
+      const int row0 = stream * TPS;  // first tile row of this sub-stream
+      if constexpr (C::QT) {
+        // q tile from TMA: smem row j holds token r0 - 3 + j (128-byte swizzle)
+        const int sq = li % QS;
+        if (!mbar_wait(&q_full[sq], (li / QS) & 1, &ab) && !ab.raised()) report_error(32, ab);
+        const uint32_t qb = smem_u32(smem + C::kOffQ + sq * C::kQBytes);
+        auto qrow = [&](int j) {
+          return lds_v4(qb + (j >> 3) * 1024 + (j & 7) * 128 + ((cc ^ (j & 7)) << 4));
+        };
 #pragma unroll
-      for (int u = 0; u < TPS; ++u) {
-        const int row = stream * TPS + u;
-        const bool valid = row < nrow;
-        float x[8];
-        unpack8(raw[u + 3], x);
-        uint32_t pq[4];
+        for (int u = 0; u < 3; ++u) unpack8(qrow(row0 + u), xm[u]);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float2 a = conv2(wq, xm, x, 2 * i);
-          pq[i] = valid ? f2_to_bf2(phi_fast(a.x), phi_fast(a.y)) : 0u;
+        for (int g4 = 0; g4 < TPS; g4 += 4)
+          readout_rows4(wq, xm, [&](int u) { return qrow(row0 + g4 + u + 3); }, abase, row0 + g4,
+                        0, cc);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&q_empty[sq]);
+      } else {
+        const size_t rs = (size_t)H * D;
+        const __nv_bfloat16 *qp = p.q + ((size_t)b * N * H + h) * D + 8 * c;
+        const int ts = r0 + row0;        // first token of this sub-stream
+        const int tmax = r0 + nrow - 1;  // last valid token of the tile
+        auto ld = [&](int t) {
+          return t < 0 ? make_uint4(0, 0, 0, 0) : ldg_nc_v4(qp + (size_t)min(t, tmax) * rs);
+        };
+        uint4 raw[4];
+#pragma unroll
+        for (int u = 0; u < 3; ++u) raw[u] = ld(ts - 3 + u);
+#pragma unroll
+        for (int u = 0; u < 3; ++u) unpack8(raw[u], xm[u]);
+#pragma unroll
+        for (int g4 = 0; g4 < TPS; g4 += 4) {
+#pragma unroll
+          for (int u = 0; u < 4; ++u) raw[u] = ld(ts + g4 + u);
+          readout_rows4(wq, xm, [&](int u) { return raw[u]; }, abase, row0 + g4, kb, cc);
         }
-        slide(xm, x);
-        const uint32_t off = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 +
-                             ((cc ^ (row & 7)) << 4);
-        sts_v4(abase + off, make_uint4(pq[0], pq[1], pq[2], pq[3]));
       }
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&a_full[sa]);
     }
-  } else if (warp < 8) {
+  } else if (warp < kRMmaWarp) {
     // ------------------------------------------------------------ epilogue
-    const int q4 = warp & 3;
+    const int ew = warp - kRProdWarps;           // 0..7
+    const int q4 = ew & 3, part = ew >> 2;       // TMEM lane quarter, column half
     const int row = 32 * q4 + lane;
+    const uint32_t ss_s = smem_u32(smem + C::kOffSs);
+    constexpr int NH = CPE / 32;                 // 32-column pieces per warp
+    int pend = -1;  // og stage whose TMA store may still be reading it (leader only)
     for (long long ii = i0; ii < i1; ++ii) {
       int b, h, r0, nrow;
       tile_of(ii, b, h, r0, nrow);
       const int li = (int)(ii - i0);
-      const int ab = li & 1, so = li % OGS;
-      if (!mbar_wait(&acc_full[ab], (li >> 1) & 1, abort_flag) && !*abort_flag)
-        report_error(64, abort_flag);
-      if (!mbar_wait(&og_full[so], (li / OGS) & 1, abort_flag) && !*abort_flag)
-        report_error(64, abort_flag);
+      const int abuf = li & 1, so = li % OGS;
+      if (!mbar_wait(&acc_full[abuf], (li >> 1) & 1, &ab) && !ab.raised()) report_error(64, ab);
+      if (!mbar_wait(&og_full[so], (li / OGS) & 1, &ab) && !ab.raised()) report_error(64, ab);
       tc_fence_after();
-      const uint32_t tacc = tmem + ((uint32_t)(32 * q4) << 16) + ab * C::kAccStride;
-      float den[16];
-      tmem_ld16(tacc + D, den);
-      tmem_ld_wait();
-      const float inv = 1.f / den[0];
-      float ss = 0.f;
+      const uint32_t tacc = tmem + ((uint32_t)(32 * q4) << 16) + abuf * C::kAccStride;
+      const uint32_t tcol = tacc + part * CPE;
+      // pass 1: this warp's half-row sum of squares of the numerators
+      float den[8], va[16], vb[16];
+      float2 ss2 = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int cb = 0; cb < D; cb += 16) {
-        float v[16];
-        tmem_ld16(tacc + cb, v);
-        tmem_ld_wait();
+      for (int h2 = 0; h2 < NH; ++h2) {
+        if (h2 == 0) tmem_ld8(tacc + D, den);
+        tmem_ld16(tcol + 32 * h2, va);
+        tmem_ld16(tcol + 32 * h2 + 16, vb);
+        tmem_ld_wait_regs(va);
+        tmem_ld_wait_regs(vb);
+        if (h2 == 0) tmem_ld_wait_regs(den);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float O = v[i] * inv;
-          ss = fmaf(O, O, ss);
+        for (int i = 0; i < 16; i += 2) {
+          ss2 = __ffma2_rn(make_float2(va[i], va[i + 1]), make_float2(va[i], va[i + 1]), ss2);
+          ss2 = __ffma2_rn(make_float2(vb[i], vb[i + 1]), make_float2(vb[i], vb[i + 1]), ss2);
         }
       }
-      const float rr = rsqrtf(ss / (float)D + p.eps) * inv;  // y = acc * rr * w * silu(og)
-      const float *nwh = p.norm_w + (size_t)h * D;
-      uint8_t *ogt = smem + C::kOffOg + so * C::kOgBytes;
+      // the two warps of a lane quarter exchange their half-row sums of squares
+      sts_f32(ss_s + (uint32_t)(part * 128 + row) * 4, ss2.x + ss2.y);
+      named_barrier(3 + q4, 64);
+      const float ss = lds_f32(ss_s + (uint32_t)row * 4) + lds_f32(ss_s + (uint32_t)(128 + row) * 4);
+      // O = acc / den;  y = O / sqrt(mean O^2 + eps) * w * silu(og) = acc * rr * w * silu(og)
+      const float inv = rcp_approx(den[0]);
+      const float ms = ss * inv * inv * (1.f / (float)D);
+      const float rr = rsqrtf(ms + p.eps) * inv;
+      const float *nwh = p.norm_w + (size_t)h * D + part * CPE;
+      const uint32_t ogt = smem_u32(smem + C::kOffOg + so * C::kOgBytes);
+      auto og_addr = [&](int col) {  // col: channel offset within this warp's half
+        const int ch0 = part * CPE + col;
+        const int kbo = ch0 >> 6, cco = (ch0 & 63) >> 3;
+        return ogt + kbo * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 +
+               ((cco ^ (row & 7)) << 4);
+      };
 #pragma unroll
-      for (int cb = 0; cb < D; cb += 16) {
-        float v[16];
-        tmem_ld16(tacc + cb, v);
-        tmem_ld_wait();
+      for (int h2 = 0; h2 < NH; ++h2) {
+        if (NH > 1) {  // pass 1 kept only the last piece in registers
+          tmem_ld16(tcol + 32 * h2, va);
+          tmem_ld16(tcol + 32 * h2 + 16, vb);
+          tmem_ld_wait_regs(va);
+          tmem_ld_wait_regs(vb);
+        }
+        // four groups of 8 channels; out_gate and weights of the next group in flight
+        uint4 gcur = lds_v4(og_addr(32 * h2));
+        float4 wc0 = __ldg((const float4 *)(nwh + 32 * h2));
+        float4 wc1 = __ldg((const float4 *)(nwh + 32 * h2 + 4));
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          const int ch0 = cb + 8 * half;  // first channel of this 16-byte chunk
-          const int kbo = ch0 >> 6, cco = (ch0 & 63) >> 3;
-          const uint32_t sa = smem_u32(ogt) + kbo * (kRTok * 128) + (row >> 3) * 1024 +
-                              (row & 7) * 128 + ((cco ^ (row & 7)) << 4);
-          float g[8];
-          unpack8(lds_v4(sa), g);
-          const float4 w0 = __ldg((const float4 *)(nwh + ch0));
-          const float4 w1 = __ldg((const float4 *)(nwh + ch0 + 4));
-          const float wv8[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+        for (int g = 0; g < 4; ++g) {
+          uint4 gnext = gcur;
+          float4 wn0 = wc0, wn1 = wc1;
+          if (g < 3) {
+            gnext = lds_v4(og_addr(32 * h2 + 8 * (g + 1)));
+            wn0 = __ldg((const float4 *)(nwh + 32 * h2 + 8 * (g + 1)));
+            wn1 = __ldg((const float4 *)(nwh + 32 * h2 + 8 * (g + 1) + 4));
+          }
+          float gv[8];
+          unpack8(gcur, gv);
+          const float wv8[8] = {wc0.x, wc0.y, wc0.z, wc0.w, wc1.x, wc1.y, wc1.z, wc1.w};
+          const float *acc8 = g < 2 ? &va[8 * g] : &vb[8 * (g - 2)];
           uint32_t outw[4];
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            const float s0v = g[2 * i] / (1.f + __expf(-g[2 * i]));
-            const float s1v = g[2 * i + 1] / (1.f + __expf(-g[2 * i + 1]));
-            const float y0 = v[8 * half + 2 * i] * rr * wv8[2 * i] * s0v;
-            const float y1 = v[8 * half + 2 * i + 1] * rr * wv8[2 * i + 1] * s1v;
-            outw[i] = f2_to_bf2(y0, y1);
+            // silu(g) = g / (1 + 2^(-g log2 e))
+            const float2 gg = make_float2(gv[2 * i], gv[2 * i + 1]);
+            const float2 tl = __fmul2_rn(gg, make_float2(-kLog2e, -kLog2e));
+            const float2 d2 = __fadd2_rn(make_float2(ex2_approx(tl.x), ex2_approx(tl.y)),
+                                         make_float2(1.f, 1.f));
+            const float2 sg = __fmul2_rn(gg, make_float2(rcp_approx(d2.x), rcp_approx(d2.y)));
+            const float2 av = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
+                                         make_float2(wv8[2 * i], wv8[2 * i + 1]));
+            const float2 y = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
+            outw[i] = f2_to_bf2(y.x, y.y);
           }
-          sts_v4(sa, make_uint4(outw[0], outw[1], outw[2], outw[3]));
+          sts_v4(og_addr(32 * h2 + 8 * g), make_uint4(outw[0], outw[1], outw[2], outw[3]));
+          gcur = gnext;
+          wc0 = wn0;
+          wc1 = wn1;
         }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[ab]);
+      if (lane == 0) mbar_arrive(&acc_empty[abuf]);
       if (nrow == kRTok) {
         fence_proxy_async_smem();
-        named_barrier(2, 128);
-        if (warp == 4 && lane == 0) {
+        named_barrier(2, kREpi);
+        if (ew == 0 && lane == 0) {
 #pragma unroll
           for (int kbo = 0; kbo < C::KB; ++kbo)
-            tma_store_4d(&tm_o, ogt + kbo * (kRTok * 128), kbo * 64, h, r0, b);
+            tma_store_4d(&tm_o, smem + C::kOffOg + so * C::kOgBytes + kbo * (kRTok * 128),
+                         kbo * 64, h, r0, b);
           tma_store_commit();
-          tma_store_wait_read<0>();
-          mbar_arrive(&og_empty[so]);
+          if constexpr (OGS >= 3) {
+            // release the previous tile's buffer once its store has read it; this
+            // tile's buffer is released one tile later, so the store overlaps work
+            if (pend >= 0) {
+              tma_store_wait_read<1>();
+              mbar_arrive(&og_empty[pend]);
+            }
+            pend = so;
+          } else {
+            tma_store_wait_read<0>();
+            mbar_arrive(&og_empty[so]);
+          }
         }
       } else {
         // Ragged tail: rows past the sequence end must not be written.
         if (row < nrow) {
-          __nv_bfloat16 *orow = p.o + (((size_t)b * N + r0 + row) * H + h) * D;
+          __nv_bfloat16 *orow = p.o + (((size_t)b * N + r0 + row) * H + h) * D + part * CPE;
 #pragma unroll
-          for (int ch0 = 0; ch0 < D; ch0 += 8) {
-            const int kbo = ch0 >> 6, cco = (ch0 & 63) >> 3;
-            const uint32_t sa = smem_u32(ogt) + kbo * (kRTok * 128) + (row >> 3) * 1024 +
-                                (row & 7) * 128 + ((cco ^ (row & 7)) << 4);
-            *(uint4 *)(orow + ch0) = lds_v4(sa);
-          }
+          for (int cb = 0; cb < CPE; cb += 8) *(uint4 *)(orow + cb) = lds_v4(og_addr(cb));
         }
-        named_barrier(2, 128);
-        if (warp == 4 && lane == 0) mbar_arrive(&og_empty[so]);
+        named_barrier(2, kREpi);
+        if (ew == 0 && lane == 0) {
+          if (pend >= 0) {
+            tma_store_wait_read<0>();
+            mbar_arrive(&og_empty[pend]);
+            pend = -1;
+          }
+          mbar_arrive(&og_empty[so]);
+        }
       }
     }
-    if (warp == 4 && lane == 0) tma_store_wait_all<0>();
-  } else if (warp == 8) {
+    if (ew == 0 && lane == 0) tma_store_wait_all<0>();
+  } else if (warp == kRMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       int cur_b = -1, cur_h = -1, nbh = 0;
@@ -836,22 +991,22 @@ __global__ void __launch_bounds__(kRThreads, 1)
         const int li = (int)(ii - i0);
         bool ok = true;
         if (b != cur_b || h != cur_h) {
-          ok = mbar_wait(b_full, nbh & 1, abort_flag);
+          ok = mbar_wait(b_full, nbh & 1, &ab);
           cur_b = b;
           cur_h = h;
           ++nbh;
         }
-        const int sa = li & 1, ab = li & 1;
-        ok = ok && mbar_wait(&a_full[sa], (li >> 1) & 1, abort_flag) &&
-             mbar_wait(&acc_empty[ab], ((li >> 1) & 1) ^ 1, abort_flag);
+        const int sa = li & 1, abuf = li & 1;
+        ok = ok && mbar_wait(&a_full[sa], (li >> 1) & 1, &ab) &&
+             mbar_wait(&acc_empty[abuf], ((li >> 1) & 1) ^ 1, &ab);
         if (!ok) {
-          if (!*abort_flag) report_error(128, abort_flag);
+          if (!ab.raised()) report_error(128, ab);
           break;
         }
         tc_fence_after();
         const uint32_t abase = smem_u32(smem + C::kOffA + sa * C::kABytes);
         const uint32_t bhi = smem_u32(smem + C::kOffBhi), blo = smem_u32(smem + C::kOffBlo);
-        const uint32_t dacc = tmem + ab * C::kAccStride;
+        const uint32_t dacc = tmem + abuf * C::kAccStride;
 #pragma unroll
         for (int kbk = 0; kbk < C::KB; ++kbk)
 #pragma unroll
@@ -863,7 +1018,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
             mma_bf16(dacc, ad, sw128_desc(blo + bo, 16, 1024), C::kIdesc, 1);
           }
         mma_commit(&a_empty[sa]);
-        mma_commit(&acc_full[ab]);
+        mma_commit(&acc_full[abuf]);
         // last tile of this (b, h) in this CTA: release B for the next rebuild
         bool last = ii + 1 >= i1;
         if (!last) {
@@ -874,18 +1029,18 @@ __global__ void __launch_bounds__(kRThreads, 1)
         if (last) mma_commit(b_free);
       }
       mma_commit(fin);  // every MMA issued above has completed once this arrives
-      if (!mbar_wait(fin, 0, nullptr)) report_error(256, abort_flag);
+      if (!mbar_wait(fin, 0, nullptr)) report_error(256, ab);
     }
   } else {
-    // ------------------------------------------------------------ TMA loads of out_gate
+    // ------------------------------------------------------------ TMA: out_gate (lane 0), q (lane 1)
     if (lane == 0) {
       for (long long ii = i0; ii < i1; ++ii) {
         int b, h, r0, nrow;
         tile_of(ii, b, h, r0, nrow);
         const int li = (int)(ii - i0);
         const int so = li % OGS;
-        if (!mbar_wait(&og_empty[so], ((li / OGS) & 1) ^ 1, abort_flag)) {
-          if (!*abort_flag) report_error(512, abort_flag);
+        if (!mbar_wait(&og_empty[so], ((li / OGS) & 1) ^ 1, &ab)) {
+          if (!ab.raised()) report_error(512, ab);
           break;
         }
         uint8_t *dst = smem + C::kOffOg + so * C::kOgBytes;
@@ -893,11 +1048,33 @@ __global__ void __launch_bounds__(kRThreads, 1)
 #pragma unroll
         for (int kbo = 0; kbo < C::KB; ++kbo)
           tma_load_4d(dst + kbo * (kRTok * 128), &tm_og, &og_full[so], kbo * 64, h, r0, b);
+        if constexpr (!C::QT) {  // q is read with plain loads: warm L2 two tiles ahead
+          if (ii + 2 < i1) {
+            int b2, h2, r02, nrow2;
+            tile_of(ii + 2, b2, h2, r02, nrow2);
+#pragma unroll
+            for (int kbo = 0; kbo < C::KB; ++kbo)
+              tma_prefetch_l2_4d(&tm_q, kbo * 64, h2, r02, b2);
+          }
+        }
+      }
+    } else if (lane == 1 && C::QT) {
+      for (long long ii = i0; ii < i1; ++ii) {
+        int b, h, r0, nrow;
+        tile_of(ii, b, h, r0, nrow);
+        const int li = (int)(ii - i0);
+        const int sq = li % QS;
+        if (!mbar_wait(&q_empty[sq], ((li / QS) & 1) ^ 1, &ab)) {
+          if (!ab.raised()) report_error(1024, ab);
+          break;
+        }
+        mbar_arrive_expect_tx(&q_full[sq], C::kQTileBytes);
+        tma_load_4d(smem + C::kOffQ + sq * C::kQBytes, &tm_q, &q_full[sq], 0, h, r0 - 3, b);
       }
     }
   }
   __syncthreads();
-  if (warp == 8) {
+  if (warp == kRMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, C::kTmemCols);
   }
@@ -923,15 +1100,16 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 4-D map over a [B, N, H, D] bf16 tensor; box = 64 channels x 1 head x 128 tokens,
-// 128-byte swizzle (the layout the readout's thread-per-row epilogue reads).
-cudaError_t make_bnhd_map(CUtensorMap *m, const void *base, int B, int N, int H, int D) {
+// 4-D map over a [B, N, H, D] bf16 tensor; box = 64 channels x 1 head x `rows`
+// tokens, 128-byte swizzle (the layout the readout's producers and epilogue read).
+cudaError_t make_bnhd_map(CUtensorMap *m, const void *base, int B, int N, int H, int D,
+                          int rows) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return cudaErrorNotSupported;
   const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)N, (cuuint64_t)B};
   const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2,
                                  (cuuint64_t)N * H * D * 2};
-  const cuuint32_t box[4] = {64, 1, kRTok, 1};
+  const cuuint32_t box[4] = {64, 1, (cuuint32_t)rows, 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -939,12 +1117,29 @@ cudaError_t make_bnhd_map(CUtensorMap *m, const void *base, int B, int N, int H,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-int num_sms() {
-  int dev = 0, n = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-  return n > 0 ? n : 1;
+struct DeviceInfo {
+  int sms = 0;
+  bool sm103 = false;
+};
+constexpr int kMaxDevices = 128;
+DeviceInfo g_dev_info[kMaxDevices];
+std::once_flag g_dev_once[kMaxDevices];
+
+const DeviceInfo &device_info() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) dev = 0;
+  std::call_once(g_dev_once[dev], [dev] {
+    int n = 0, major = 0, minor = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    g_dev_info[dev].sms = n > 0 ? n : 1;
+    g_dev_info[dev].sm103 = (major == 10 && minor == 3);
+  });
+  return g_dev_info[dev];
 }
+
+int num_sms() { return device_info().sms; }
 
 // Chunk length: about one chunk per SM over the padded problem, 32-aligned,
 // within [256, kChunkMax], and at most kMaxChunksPerSeq chunks per sequence.
@@ -1000,7 +1195,7 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.gridDim = dim3(p.B * p.H, (F + 255) / 256);
+  cfg.gridDim = dim3(p.B * p.H, (F / 4 + 255) / 256);
   cfg.blockDim = dim3(256);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
@@ -1016,10 +1211,12 @@ template <int D>
 cudaError_t run_readout(const Problem &p, const void *q, const void *og, const float *conv_w,
                         const float *norm_w, const float *state, void *o, cudaStream_t st) {
   using C = ReadoutCfg<D>;
-  CUtensorMap tm_og, tm_o;
-  cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D);
+  CUtensorMap tm_og, tm_o, tm_q;
+  cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D, kRTok);
   if (e != cudaSuccess) return e;
-  if ((e = make_bnhd_map(&tm_o, o, p.B, p.N, p.H, D)) != cudaSuccess) return e;
+  if ((e = make_bnhd_map(&tm_o, o, p.B, p.N, p.H, D, kRTok)) != cudaSuccess) return e;
+  if ((e = make_bnhd_map(&tm_q, q, p.B, p.N, p.H, D, C::QT ? kRQRows : kRTok)) != cudaSuccess)
+    return e;
   ReadoutParams rp;
   rp.q = (const __nv_bfloat16 *)q;
   rp.conv_w = conv_w;
@@ -1045,7 +1242,7 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   cfg.stream = st;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, kern, rp, tm_og, tm_o);
+  e = cudaLaunchKernelEx(&cfg, kern, rp, tm_og, tm_o, tm_q);
   count_launch();
   return e;
 }
@@ -1058,11 +1255,7 @@ bool tc_supports(const Problem &p) {
   if (p.B > kMaxBatch) return false;
   if ((long long)p.N > (long long)kChunkMax * kMaxChunksPerSeq) return false;
   if ((long long)p.B * p.H > 2147483647ll / 4) return false;
-  int dev = 0, major = 0, minor = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
-  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
-  return major == 10 && minor == 3 && encode_fn() != nullptr;
+  return device_info().sm103 && encode_fn() != nullptr;
 }
 
 size_t tc_workspace_bytes(const Problem &p) {

@@ -23,7 +23,7 @@ CONV_WIDTH = 4
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_state", "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
-            "gbla_state_static_scratch", "gbla_device_error"]
+            "gbla_state_static_scratch", "gbla_device_error", "gbla_last_cuda_error"]
 
 _lock = threading.Lock()
 _lib = None
@@ -35,7 +35,10 @@ _i = ctypes.c_int
 class GblaError(RuntimeError):
     def __init__(self, status: int, fn: str):
         self.status = status
-        super().__init__(f"{fn}: {status_string(status)} (status {status})")
+        msg = f"{fn}: {status_string(status)} (status {status})"
+        if status == GBLA_ERR_CUDA:
+            msg += f": {load().gbla_last_cuda_error().decode()}"
+        super().__init__(msg)
 
 
 def lib_path() -> str:
@@ -76,6 +79,8 @@ def load(path: str | None = None):
         lib.gbla_version.restype = ctypes.c_char_p
         lib.gbla_release.argtypes = []
         lib.gbla_release.restype = None
+        lib.gbla_last_cuda_error.argtypes = []
+        lib.gbla_last_cuda_error.restype = ctypes.c_char_p
         lib.gbla_device_error.argtypes = [_i]
         lib.gbla_device_error.restype = ctypes.c_uint32
         lib.gbla_launch_count.argtypes = []
