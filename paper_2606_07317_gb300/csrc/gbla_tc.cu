@@ -6,14 +6,14 @@
 //      is cut into chunks of S tokens and every CTA takes a contiguous range of
 //      chunks, so work is balanced whatever the sequence lengths.  Per chunk:
 //      a pre-pass over the gate logits gives the chunk maximum m and the
-//      weights w_j = exp(a_j - m); eight producer warps then stream k and v
-//      from HBM with 128-bit loads, run the causal Conv1D (sliding window in
-//      registers, packed f32x2 FMAs), phi and the gate weight, and write
-//      K^ (bf16) and V~ as a bf16 hi/lo pair into 128B-swizzled MN-major
-//      tiles; one thread issues tcgen05.mma (M = N = 128, K = 16, fp32
-//      accumulation in TMEM): D += K^T V~_hi + K^T V~_lo.  The diagonal
-//      D x D blocks of the accumulator are the per-head partial states S_c;
-//      z_c, m_c and l_c = sum w_j complete each partial record.
+//      per-token weights 2^a' (a' = (a - m) log2 e); one warp streams raw k
+//      and v tiles (32 tokens + 3 rows of conv history) into a TMA ring;
+//      sixteen converter warps run the causal Conv1D, phi and the gate weight
+//      in fp32 and write K^ and V~ as fp32 into 128B-swizzled K-major tiles;
+//      one thread issues tcgen05.mma kind::tf32 (M = N = 128, K = 8, fp32
+//      accumulation in TMEM): D += K^T V~.  The diagonal D x D blocks of the
+//      accumulator are the per-head partial states S_c; z_c, m_c and
+//      l_c = sum 2^a' complete each partial record.
 //  tc_reduce_kernel  fixed-order, max-rescaled combination of the partial
 //      records into S = K^T V~ and z = K^T 1 with the softmax gate.
 //  tc_readout_kernel (Sec. 2.1 item 2 readout and item 3)
@@ -25,11 +25,12 @@
 //      SiLU(out_gate) (out_gate tile brought in by TMA) and write o in place
 //      of the out_gate tile, which TMA stores back.
 //
-// Why V~ is split into hi + lo: V~ = Conv1D(v) is not representable in bf16,
-// and its rounding error does not average out, because O is a heavily
+// Why V~ is not rounded to bf16: V~ = Conv1D(v) is not representable in
+// bf16, and its rounding error does not average out, because O is a heavily
 // cancelling weighted mean of the v rows (|O| shrinks like 1/sqrt(L) while the
-// rows stay O(1)); V~_hi + V~_lo carries 16 significant bits.  K^ only weights
-// the mean, so bf16 is enough there, and z sums the same rounded K^ the MMA sees.
+// rows stay O(1)).  The state kernel therefore contracts tf32 operands (V~
+// with 11 significant bits after the tf32 rounding inside the MMA, K^ alike),
+// and the readout multiplies by [S | z] as a bf16 hi + lo pair.
 //
 // Every mbarrier wait is bounded (2 s).  A wait that runs out sets a bit in
 // g_tc_error and the CTA's abort flag; the other waits then return at once,
@@ -54,49 +55,62 @@ using namespace sm100;
 constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the state
 
 // ------------------------------------------------------------------ state
-// 13 warps: at most 4 per SM sub-partition, so each thread may hold 128 registers.
-constexpr int kSKWarps = 6;                       // warps producing K^ (A operand)
-constexpr int kSProdWarps = 2 * kSKWarps;         // + 6 warps producing V~ hi/lo (B)
-constexpr int kSThreads = (kSProdWarps + 1) * 32; // + 1 MMA warp
+// 18 warps: 8 k-warps and 8 v-warps convert raw tiles into the MMA operands,
+// one warp issues the MMAs and one the TMA loads.  At most 5 warps per SM
+// sub-partition, so each thread may hold 96 registers.  K^ and V~ are written
+// as fp32 and contracted with kind::tf32 (K-major operands): no bf16 packing
+// and no hi/lo split of V~.
+constexpr int kSKWarps = 8;                          // warps producing K^ (A operand)
+constexpr int kSProdWarps = 2 * kSKWarps;            // + 8 warps producing V~ (B operand)
+constexpr int kSMmaWarp = kSProdWarps;               // 16
+constexpr int kSTmaWarp = kSProdWarps + 1;           // 17
+constexpr int kSThreads = (kSTmaWarp + 1) * 32;      // 576
 constexpr int kSProd = kSProdWarps * 32;
-constexpr int kSSub = 2 * kSKWarps;               // sub-streams (half-warps of a k-warp)
-constexpr int kSTokPerSub = 4;
-constexpr int kSTok = kSSub * kSTokPerSub;        // 48 tokens per pipeline stage
-constexpr int kSStages = 4;
-constexpr int kChunkMax = 2048;                   // longest chunk (tokens)
+constexpr int kSTok = 32;                            // tokens per stage: one 128-byte tf32 row
+constexpr int kSHalo = kConvW - 1;                   // conv history rows in front of a tile
+constexpr int kSRawRows = kSTok + kSHalo;            // 35
+constexpr int kSRawRow = kGroupCh * 2;               // bytes of one token's group row (bf16)
+constexpr int kSRawBytes = kSRawRows * kSRawRow;     // 8960: one raw tile of k or v
+constexpr int kSRawStages = 4;                       // raw ring (k and v tiles per stage)
+constexpr int kSOpStages = 3;                        // operand ring
+constexpr int kSOp = kGroupCh * kSTok * 4;           // one operand: 128 channel rows x 128 B
+constexpr int kSOpStageBytes = 2 * kSOp;             // A = K^T, B = V~^T
+constexpr int kChunkMax = 2048;                      // longest chunk (tokens)
 constexpr int kMaxChunksPerSeq = 4096;
-constexpr int kSBlock = kSTok * 128;              // 64-channel MN block: 48 rows x 128 B
-constexpr int kSOp = 2 * kSBlock;                 // one 128-channel operand
-constexpr int kSStageBytes = 3 * kSOp;            // A, B_hi, B_lo
+constexpr int kSGateStride = kChunkMax + kSTok;      // (a', 2^a' ln 2) entries per head
 constexpr uint32_t kSTmemCols = 128;
-constexpr int kSPrefetch = 16;                    // L2 prefetch distance (tokens)
 
 constexpr int kMaxBatch = 2048;
 
 // Shared-memory map of the state kernel (offsets from a 1024-aligned base).
-constexpr int kSOffStages = 0;
-constexpr int kSOffGate = kSStages * kSStageBytes;               // float [2][kChunkMax]
-constexpr int kSOffZred = kSOffGate + 2 * kChunkMax * 4;         // float [kSSub][128]
-constexpr int kSOffRed = kSOffZred + kSSub * kGroupCh * 4;       // float [160]
-constexpr int kSOffPre = kSOffRed + 160 * 4;                     // int [kMaxBatch + 1]
+constexpr int kSOffOp = 0;
+constexpr int kSOffRaw = kSOffOp + kSOpStages * kSOpStageBytes;
+constexpr int kSOffGate = kSOffRaw + kSRawStages * 2 * kSRawBytes;  // float2 [2][kSGateStride]
+constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 8;         // float [8][128]
+constexpr int kSOffRed = kSOffZred + 8 * kGroupCh * 4;              // float [256]
+constexpr int kSOffPre = kSOffRed + 256 * 4;                        // int [kMaxBatch + 1]
 constexpr int kSOffBar = kSOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
-constexpr int kSBarCount = 2 * kSStages + 2;                      // full, empty, done, final
-constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;              // tmem addr, abort flag
-constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                // + alignment slack
+// raw_full, raw_empty, op_full, op_empty, done, final
+constexpr int kSBarCount = 2 * kSRawStages + 2 * kSOpStages + 2;
+constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;                // tmem addr, abort flag
+constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                  // + alignment slack
 static_assert(kSSmemBytes <= 227 * 1024, "state shared memory");
+static_assert(kSRawBytes % 128 == 0, "raw tiles keep TMA destinations 128-byte aligned");
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
 // ------------------------------------------------------------------ readout
-// 18 warps: 8 producer, 8 epilogue (two per TMEM lane quarter), MMA, TMA.
-// At most 5 warps per SM sub-partition, so each thread may hold 96 registers.
+// 19 warps: 8 producer, 8 epilogue (two per TMEM lane quarter), MMA, and one
+// TMA warp each for out_gate and q.  At most 5 warps per SM sub-partition, so
+// each thread may hold 96 registers.
 constexpr int kRTok = 128;                      // tokens per tile (MMA M)
 constexpr int kRProdWarps = 8;
 constexpr int kREpiWarps = 8;
 constexpr int kRMmaWarp = kRProdWarps + kREpiWarps;   // 16
-constexpr int kRTmaWarp = kRMmaWarp + 1;              // 17
-constexpr int kRThreads = (kRTmaWarp + 1) * 32;       // 576
+constexpr int kRTmaWarp = kRMmaWarp + 1;              // 17: out_gate loads
+constexpr int kRQWarp = kRTmaWarp + 1;                // 18: q loads
+constexpr int kRThreads = (kRQWarp + 1) * 32;         // 608
 constexpr int kRProd = kRProdWarps * 32;
 constexpr int kREpi = kREpiWarps * 32;
 constexpr int kRAStages = 2;
@@ -199,10 +213,15 @@ __device__ __forceinline__ void unpack8(const uint4 &r, float (&x)[8]) {
     x[2 * i + 1] = f.y;
   }
 }
+__device__ __forceinline__ void unpack4(const uint2 &r, float (&x)[4]) {
+  const float2 a = bf2_to_f2(r.x), b = bf2_to_f2(r.y);
+  x[0] = a.x; x[1] = a.y; x[2] = b.x; x[3] = b.y;
+}
 
 // Causal Conv1D of channels i, i+1: taps 0..2 on x[t-3..t-1], tap 3 on x[t].
-__device__ __forceinline__ float2 conv2(const float (&w)[4][8], const float (&xm)[3][8],
-                                        const float (&x)[8], int i) {
+template <int NC>
+__device__ __forceinline__ float2 conv2(const float (&w)[4][NC], const float (&xm)[3][NC],
+                                        const float (&x)[NC], int i) {
   float2 a = __fmul2_rn(make_float2(w[0][i], w[0][i + 1]), make_float2(xm[0][i], xm[0][i + 1]));
   a = __ffma2_rn(make_float2(w[1][i], w[1][i + 1]), make_float2(xm[1][i], xm[1][i + 1]), a);
   a = __ffma2_rn(make_float2(w[2][i], w[2][i + 1]), make_float2(xm[2][i], xm[2][i + 1]), a);
@@ -210,9 +229,10 @@ __device__ __forceinline__ float2 conv2(const float (&w)[4][8], const float (&xm
   return a;
 }
 
-__device__ __forceinline__ void slide(float (&xm)[3][8], const float (&x)[8]) {
+template <int NC>
+__device__ __forceinline__ void slide(float (&xm)[3][NC], const float (&x)[NC]) {
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
+  for (int i = 0; i < NC; ++i) {
     xm[0][i] = xm[1][i];
     xm[1][i] = xm[2][i];
     xm[2][i] = x[i];
@@ -226,99 +246,101 @@ __device__ __forceinline__ float2 phi2_log2(float2 xl) {
   return __ffma2_rn(make_float2(kLn2, kLn2), make_float2(fmaxf(xl.x, 0.f), fmaxf(xl.y, 0.f)), e);
 }
 
-// One token of a state producer: conv of 8 channels, then K^ (IS_K) or V~ hi/lo
-// written to the stage at shared address sa.  al = a' = (gate - m) log2(e) of
-// this token's head (-inf past the sub-stream end, which makes K^ = 0).
-template <bool IS_K>
-__device__ __forceinline__ void state_token(const float (&w)[4][8], float (&xm)[3][8],
-                                            const uint4 &raw, float al, float2 (&z)[4],
-                                            uint32_t sa) {
-  float x[8];
-  unpack8(raw, x);
-  if constexpr (IS_K) {
-    // K^ = 2^a' phi(k~) = 2^min(x' + a', a') + (2^a' ln 2) max(x', 0),  x' = k~ log2(e)
-    const float wl = ex2_approx(al) * kLn2;
-    uint32_t pk[4];
+// Causal Conv1D of channels i, i+1 at token u of a thread's 4 tokens: taps
+// 0..3 on raw rows u..u+3 (row u + 3 is the token itself).
+__device__ __forceinline__ float2 conv_rows(const float (&w)[4][4], const float (&x)[7][4],
+                                            int u, int i) {
+  float2 a = __fmul2_rn(make_float2(w[0][i], w[0][i + 1]), make_float2(x[u][i], x[u][i + 1]));
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 xl = conv2(w, xm, x, 2 * i);
-      const float2 ts = __fadd2_rn(xl, make_float2(al, al));
-      const float2 e = make_float2(ex2_approx(fminf(ts.x, al)), ex2_approx(fminf(ts.y, al)));
-      const float2 kh =
-          __ffma2_rn(make_float2(wl, wl), make_float2(fmaxf(xl.x, 0.f), fmaxf(xl.y, 0.f)), e);
-      pk[i] = f2_to_bf2(kh.x, kh.y);
-      z[i] = __fadd2_rn(z[i], kh);
-    }
-    sts_v4(sa, make_uint4(pk[0], pk[1], pk[2], pk[3]));
-  } else {
-    // V~ as hi + lo bf16 (16 significant bits)
-    uint32_t ph[4], pl[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 cv = conv2(w, xm, x, 2 * i);
-      ph[i] = f2_to_bf2(cv.x, cv.y);
-      const float2 lo = __ffma2_rn(bf2_to_f2(ph[i]), make_float2(-1.f, -1.f), cv);
-      pl[i] = f2_to_bf2(lo.x, lo.y);
-    }
-    sts_v4(sa + kSOp, make_uint4(ph[0], ph[1], ph[2], ph[3]));
-    sts_v4(sa + 2 * kSOp, make_uint4(pl[0], pl[1], pl[2], pl[3]));
-  }
-  slide(xm, x);
+  for (int tau = 1; tau < 4; ++tau)
+    a = __ffma2_rn(make_float2(w[tau][i], w[tau][i + 1]),
+                   make_float2(x[u + tau][i], x[u + tau][i + 1]), a);
+  return a;
 }
 
-// What a state producer thread needs to stream one chunk's sub-stream.
-struct SubStream {
-  const __nv_bfloat16 *xp;   // this thread's 8 channels at token 0
-  const __nv_bfloat16 *grp;  // the head group's row at token 0 (L2 prefetch)
-  size_t rs;                 // token stride (elements)
-  int s0, s1, tlast, t0;     // sub-stream [s0, s1), last loadable token, chunk start
-  uint32_t grow_bytes;       // bytes of one group row
-  uint32_t gw_s;             // shared address of this head's a' values
-  int nst;                   // pipeline stages of this chunk
+// One stage of a converter thread: channels 4q..4q+3 of the head group at the
+// stage's tokens 4j..4j+3.  Reads the 7 raw rows it needs (3 of conv history)
+// from the TMA tile, convolves, and for K^ (IS_K) applies phi and the gate
+// weight: K^ = 2^a' phi(k~) = 2^min(x' + a', a') + (2^a' ln 2) max(x', 0), with
+// x' = k~ log2(e) (the taps carry the log2(e)) and a' = (a - m) log2(e).  Each
+// channel's 4 tokens are one 16-byte piece of its K-major row.  Tokens past
+// the sequence end (nvalid < 4, last stage only) are written as zeros.
+template <bool IS_K>
+__device__ __forceinline__ void state_convert(uint32_t raw, uint32_t op, uint32_t gws,
+                                              const float (&w)[4][4], float (&z)[4],
+                                              uint32_t sw, int nvalid) {
+  float x[7][4];
+#pragma unroll
+  for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRow), x[r]);
+  float y[4][4];  // [token][channel]
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const float2 c01 = conv_rows(w, x, u, 0), c23 = conv_rows(w, x, u, 2);
+    if constexpr (IS_K) {
+      const uint2 gr = lds_v2(gws + u * 8);
+      const float al = __uint_as_float(gr.x), wl = __uint_as_float(gr.y);
+      const float2 t01 = __fadd2_rn(c01, make_float2(al, al));
+      const float2 t23 = __fadd2_rn(c23, make_float2(al, al));
+      const float2 e01 = make_float2(ex2_approx(fminf(t01.x, al)), ex2_approx(fminf(t01.y, al)));
+      const float2 e23 = make_float2(ex2_approx(fminf(t23.x, al)), ex2_approx(fminf(t23.y, al)));
+      const float2 k01 = __ffma2_rn(make_float2(wl, wl),
+                                    make_float2(fmaxf(c01.x, 0.f), fmaxf(c01.y, 0.f)), e01);
+      const float2 k23 = __ffma2_rn(make_float2(wl, wl),
+                                    make_float2(fmaxf(c23.x, 0.f), fmaxf(c23.y, 0.f)), e23);
+      y[u][0] = k01.x; y[u][1] = k01.y; y[u][2] = k23.x; y[u][3] = k23.y;
+    } else {
+      y[u][0] = c01.x; y[u][1] = c01.y; y[u][2] = c23.x; y[u][3] = c23.y;
+    }
+  }
+  if (nvalid < 4) {  // rows past the sequence end may hold anything, NaN included
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) y[u][i] = u < nvalid ? y[u][i] : 0.f;
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if constexpr (IS_K) z[i] += (y[0][i] + y[1][i]) + (y[2][i] + y[3][i]);
+    sts_v4(op + i * 128 + ((sw ^ i) << 4),
+           make_uint4(__float_as_uint(y[0][i]), __float_as_uint(y[1][i]),
+                      __float_as_uint(y[2][i]), __float_as_uint(y[3][i])));
+  }
+}
+
+// Ring position of a pipeline: slot and phase parity.
+struct Ring {
+  uint32_t slot = 0, phase = 0;
+  __device__ __forceinline__ void next(uint32_t n) {
+    if (++slot == n) { slot = 0; phase ^= 1; }
+  }
 };
 
-// All stages of one chunk for one producer thread (k or v role, fixed per warp).
+// All stages of one chunk for one converter thread.
 template <bool IS_K>
-__device__ __forceinline__ void state_stream(const SubStream &ss, const float (&w)[4][8],
-                                             float (&xm)[3][8], float2 (&z)[4], uint32_t &gs,
-                                             uint64_t *full, uint64_t *empty,
-                                             const AbortFlag &ab, uint32_t stages_s,
-                                             uint32_t rbase, uint32_t sw, int c, int lane) {
-  auto ld = [&](int t) { return ldg_nc_v4(ss.xp + (size_t)min(t, ss.tlast) * ss.rs); };
-  auto alpha = [&](int t) {
-    const float a = lds_f32(ss.gw_s + (uint32_t)max(min(t, ss.s1 - 1) - ss.t0, 0) * 4);
-    return t < ss.s1 ? a : -INFINITY;
-  };
-  uint4 ra0 = ld(ss.s0), ra1 = ld(ss.s0 + 1);
-  for (int it = 0; it < ss.nst; ++it, ++gs) {
-    const int s = gs % kSStages;
-    if (!mbar_wait(&empty[s], ((gs / kSStages) & 1) ^ 1, &ab) && !ab.raised())
-      report_error(1, ab);
-    const uint32_t stage = stages_s + s * kSStageBytes + rbase;
-    const int tb = ss.s0 + it * kSTokPerSub;
-    const uint4 rb0 = ld(tb + 2), rb1 = ld(tb + 3);
-    if (c < kSTokPerSub && tb + kSPrefetch + c < ss.s1)
-      prefetch_l2(ss.grp + (size_t)(tb + kSPrefetch + c) * ss.rs, ss.grow_bytes);
-    float al[4] = {0.f, 0.f, 0.f, 0.f};
-    if constexpr (IS_K) {
-#pragma unroll
-      for (int u = 0; u < 4; ++u) al[u] = alpha(tb + u);
-    }
-    state_token<IS_K>(w, xm, ra0, al[0], z, stage + 0 * 128 + ((sw ^ 0) << 4));
-    state_token<IS_K>(w, xm, ra1, al[1], z, stage + 1 * 128 + ((sw ^ 1) << 4));
-    ra0 = ld(tb + 4);
-    ra1 = ld(tb + 5);
-    state_token<IS_K>(w, xm, rb0, al[2], z, stage + 2 * 128 + ((sw ^ 2) << 4));
-    state_token<IS_K>(w, xm, rb1, al[3], z, stage + 3 * 128 + ((sw ^ 3) << 4));
-    fence_proxy_async_smem();
+__device__ __forceinline__ void state_chunk_stages(
+    int nst, int t0, int L, int j, const float (&w)[4][4], float (&z)[4], Ring &rr, Ring &ro,
+    uint64_t *raw_full, uint64_t *raw_empty, uint64_t *op_full, uint64_t *op_empty,
+    const AbortFlag &ab, uint32_t raw_s, uint32_t op_s, uint32_t gws, uint32_t sw, int lane) {
+  for (int it = 0; it < nst; ++it) {
+    if (!mbar_wait(&raw_full[rr.slot], rr.phase, &ab) && !ab.raised()) report_error(1, ab);
+    if (!mbar_wait(&op_empty[ro.slot], ro.phase ^ 1, &ab) && !ab.raised()) report_error(1, ab);
+    const int nvalid = min(max(L - (t0 + it * kSTok + 4 * j), 0), 4);
+    state_convert<IS_K>(raw_s + rr.slot * (2 * kSRawBytes), op_s + ro.slot * kSOpStageBytes,
+                        gws + (uint32_t)(it * kSTok) * 8, w, z, sw, nvalid);
+    fence_proxy_async_smem();  // operand writes visible to the tensor cores
     __syncwarp();
-    if (lane == 0) mbar_arrive(&full[s]);
+    if (lane == 0) {
+      mbar_arrive(&op_full[ro.slot]);
+      mbar_arrive(&raw_empty[rr.slot]);
+    }
+    rr.next(kSRawStages);
+    ro.next(kSOpStages);
   }
 }
 
 // ===================================================================== state
 struct StateParams {
-  const __nv_bfloat16 *k, *v, *gate;
+  const __nv_bfloat16 *gate;
   const float *conv_w;
   const int32_t *seq_lens;
   float *records;        // [chunks][G][D*D + D + 4]: S, z, m, l, 2 pad
@@ -326,35 +348,65 @@ struct StateParams {
   int B, H, N, S, HG;
 };
 
+// Chunk k of the flattened (batch, head group, chunk) order.
+struct ChunkRef {
+  int b, L, hbase, t0, n, nst;
+};
+template <int G>
+__device__ __forceinline__ ChunkRef decode_chunk(const StateParams &p, const int *pre, int k) {
+  ChunkRef c;
+  c.b = find_batch(pre, p.B, k);
+  c.L = clamp_len(p.seq_lens, c.b, p.N);
+  const int nck = (c.L + p.S - 1) / p.S;
+  const int r = k - pre[c.b];
+  c.hbase = (r / nck) * G;
+  c.t0 = (r % nck) * p.S;
+  c.n = min(c.t0 + p.S, c.L) - c.t0;
+  c.nst = (c.n + kSTok - 1) / kSTok;
+  return c;
+}
+
 template <int D>
-__global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParams p) {
+__global__ void __launch_bounds__(kSThreads, 1)
+    tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
+                    const __grid_constant__ CUtensorMap tm_v) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float *gw = (float *)(smem + kSOffGate);   // [G][kChunkMax]: a' = (a - m) log2(e)
-  float *zred = (float *)(smem + kSOffZred); // [kSSub][128]
-  float *red = (float *)(smem + kSOffRed);   // [0,64) max, [64,128) sum, 128+ m, 136+ l
+  float2 *gw = (float2 *)(smem + kSOffGate);  // [G][kSGateStride]: (a', 2^a' ln 2)
+  float *zred = (float *)(smem + kSOffZred);  // [8][128]
+  float *red = (float *)(smem + kSOffRed);    // [0,64) max, [64,128) sum, 128+ m, 132+ l
   int *pre = (int *)(smem + kSOffPre);
   uint64_t *bars = (uint64_t *)(smem + kSOffBar);
-  uint64_t *full = bars, *empty = bars + kSStages, *done = bars + 2 * kSStages,
-           *fin = bars + 2 * kSStages + 1;
+  uint64_t *raw_full = bars, *raw_empty = bars + kSRawStages;
+  uint64_t *op_full = bars + 2 * kSRawStages, *op_empty = op_full + kSOpStages;
+  uint64_t *done = op_empty + kSOpStages, *fin = done + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + kSOffMisc);
   const AbortFlag ab{smem_u32(smem + kSOffMisc + 4)};
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int B = p.B, H = p.H, N = p.N, S = p.S, HG = p.HG;
+  const int B = p.B, H = p.H;
 
   if (tid == 0) {
     *(volatile int *)(smem + kSOffMisc + 4) = 0;
-    for (int i = 0; i < kSBarCount; ++i) mbar_init(&bars[i], i < kSStages ? kSProdWarps : 1);
+    for (int i = 0; i < kSRawStages; ++i) {
+      mbar_init(&raw_full[i], 1);
+      mbar_init(&raw_empty[i], kSProdWarps);
+    }
+    for (int i = 0; i < kSOpStages; ++i) {
+      mbar_init(&op_full[i], kSProdWarps);
+      mbar_init(&op_empty[i], 1);
+    }
+    mbar_init(done, 1);
+    mbar_init(fin, 1);
     fence_mbar_init();
   }
-  // Chunk prefix over the batch (producer threads), shared by all roles.
+  // Chunk prefix over the batch (converter threads), shared by all roles.
   if (warp < kSProdWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
-      const int L = clamp_len(p.seq_lens, b, N);
-      return HG * ((L + S - 1) / S);
+      const int L = clamp_len(p.seq_lens, b, p.N);
+      return p.HG * ((L + p.S - 1) / p.S);
     });
   }
   __syncthreads();
@@ -366,127 +418,122 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
   grid_dep_launch();
   if (c0 >= c1) return;  // no chunks for this CTA
 
-  if (warp == kSProdWarps) tmem_alloc(tmem_slot, kSTmemCols);
+  if (warp == kSMmaWarp) tmem_alloc(tmem_slot, kSTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
   if (warp < kSProdWarps) {
-    // ------------------------------------------------------------ producers
-    const bool is_k = warp < kSKWarps;                // k-warps write A, v-warps write B
-    const int half = lane >> 4, c = lane & 15;        // c: 8-channel chunk of the group
-    const int sub = (warp % kSKWarps) * 2 + half;     // sub-stream 0..11
-    const int hh = (8 * c) / D, d0 = 8 * c - D * hh;  // head within group, first channel
-    const int blk = c >> 3, cc = c & 7;               // MN block, 16-byte chunk in block
-    const int tens = is_k ? 1 : 2;                    // conv_w stream: 1 = k, 2 = v
-    const __nv_bfloat16 *src = is_k ? p.k : p.v;
-    // stage-relative byte offset of this thread's 16 bytes in row sub*4 + u:
-    // rows of one sub-stream share an 8-row group; swizzle chunk = cc ^ (row & 7)
-    const uint32_t rbase = blk * kSBlock + (sub >> 1) * 1024 + (sub & 1) * 512;
-    const uint32_t sw = (uint32_t)(cc ^ ((sub & 1) * 4));
-    const uint32_t gw_s = smem_u32(gw) + hh * kChunkMax * 4;
-    uint32_t gs = 0;                                  // stage counter across chunks
+    // ------------------------------------------------------------ converters
+    // Thread -> (channel quad q, token quad j) of each stage, chosen so that
+    // both the raw-tile reads (16 lanes, 16 distinct quads of one 256-byte
+    // row) and the swizzled operand writes (8 lanes, 8 distinct 16-byte
+    // chunks) are free of bank conflicts.
+    const bool is_k = warp < kSKWarps;
+    const int hw = 2 * (warp % kSKWarps) + (lane >> 4);          // half-warp 0..15
+    const int q = (lane & 15) + 16 * (hw & 1);                   // channel quad 0..31
+    const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
+    const int c0ch = 4 * q;
+    const int hh = c0ch / D, d0 = c0ch - D * hh;                 // head in group, channel
+    const int tens = is_k ? 1 : 2;                               // conv_w stream: 1 = k, 2 = v
+    // K-major tf32 rows (128 B = 32 tokens), 128-byte swizzle: channel row r at
+    // (r >> 3) * 1024 + (r & 7) * 128; this thread's 16 bytes are chunk j ^ (r & 7)
+    const uint32_t rbase = (q >> 1) * 1024 + (q & 1) * 512;
+    const uint32_t sw = (uint32_t)(j ^ ((q & 1) * 4));
+    const uint32_t op_s = smem_u32(smem + kSOffOp) + (is_k ? 0u : (uint32_t)kSOp) + rbase;
+    const uint32_t raw_s = smem_u32(smem + kSOffRaw) + (is_k ? 0u : (uint32_t)kSRawBytes) +
+                           (uint32_t)(4 * j * kSRawRow + q * 8);
+    const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kSGateStride + 4 * j) * 8;
+    Ring rr, ro;
     int nchunk = 0;
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
-      const int b = find_batch(pre, B, k);
-      const int L = clamp_len(p.seq_lens, b, N);
-      const int nck = (L + S - 1) / S;
-      const int r = k - pre[b];
-      const int hg = r / nck, j = r % nck;
-      const int t0 = j * S, t1 = min(t0 + S, L), n = t1 - t0;
-      const int hbase = hg * G;
+      const ChunkRef c = decode_chunk<G>(p, pre, k);
 
-      // Gate pre-pass: per-head chunk maximum m, a' = (a - m) log2(e), l = sum 2^a'.
-      {
-        const int myh = tid % G;
-        const bool hok = hbase + myh < H;
-        float m = -INFINITY;
-        for (int idx = tid; idx < n * G; idx += kSProd) {
-          const int tt = idx / G;
-          float a = -INFINITY;
-          if (hok) a = __bfloat162float(p.gate[((size_t)b * N + t0 + tt) * H + hbase + myh]);
-          gw[myh * kChunkMax + tt] = a;
-          m = fmaxf(m, a);
-        }
-#pragma unroll
-        for (int o = 16; o >= G; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        if (lane < G) red[warp * 4 + lane] = m;
-        named_barrier(1, kSProd);
-        float M = red[myh];
-        for (int w = 1; w < kSProdWarps; ++w) M = fmaxf(M, red[w * 4 + myh]);
-        float l = 0.f;
-        for (int idx = tid; idx < n * G; idx += kSProd) {
-          const int tt = idx / G;
-          const float al = hok ? (gw[myh * kChunkMax + tt] - M) * kLog2e : -INFINITY;
-          gw[myh * kChunkMax + tt] = al;
-          l += ex2_approx(al);
-        }
-#pragma unroll
-        for (int o = 16; o >= G; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-        if (lane < G) red[64 + warp * 4 + lane] = l;
-        named_barrier(1, kSProd);
-        if (tid < G) {  // m and l of this chunk, per head, for the records
-          float lt = 0.f;
-          for (int w = 0; w < kSProdWarps; ++w) lt += red[64 + w * 4 + tid];
-          red[128 + tid] = M;
-          red[136 + tid] = lt;
-        }
-      }
-
-      // This thread: channels [8c, 8c+8) of the group, of k or of v.
-      const int h = hbase + hh;
+      // taps of this thread's 4 channels; for k pre-scaled by log2(e)
+      const int h = c.hbase + hh;
       const bool hv = h < H;
-      const size_t rs = (size_t)H * D;  // token stride (elements)
-      const __nv_bfloat16 *xp = src + ((size_t)b * N * H + (hv ? h : 0)) * D + d0;
-      // taps; for k pre-scaled by log2(e) so the conv yields x * log2(e) directly
-      float w[4][8];
+      float w[4][4];
       const float wsc = is_k ? kLog2e : 1.f;
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
+      for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
-          w[q][i] = hv ? p.conv_w[((size_t)(tens * H + h) * D + d0 + i) * 4 + q] * wsc : 0.f;
-      const int s0 = t0 + (int)((long long)n * sub / kSSub);
-      const int s1 = t0 + (int)((long long)n * (sub + 1) / kSSub);
-      const int tlast = max(min(s1, L) - 1, 0);  // loads past the sub-stream repeat this row
-      float xm[3][8];  // sliding window x[t-3], x[t-2], x[t-1]
-#pragma unroll
-      for (int q = 0; q < 3; ++q) {
-        const int t = s0 - 3 + q;
-        uint4 rw = make_uint4(0, 0, 0, 0);
-        if (t >= 0 && s0 < s1) rw = ldg_nc_v4(xp + (size_t)t * rs);
-        unpack8(rw, xm[q]);
-      }
-      float2 z[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) z[i] = make_float2(0.f, 0.f);
-      const int nst = ((n + kSSub - 1) / kSSub + kSTokPerSub - 1) / kSTokPerSub;
-      const uint32_t grow_bytes = (uint32_t)(min(G, H - hbase) * D * 2);
-      const __nv_bfloat16 *grp = src + ((size_t)b * N * H + hbase) * D;
-      if (c == 0)  // warm L2 with the first tokens of this sub-stream
-        for (int t = s0; t < min(s1, s0 + kSPrefetch); ++t)
-          prefetch_l2(grp + (size_t)t * rs, grow_bytes);
-      const SubStream sst{xp, grp, rs, s0, s1, tlast, t0, grow_bytes, gw_s, nst};
-      const uint32_t stages_s = smem_u32(smem + kSOffStages);
-      if (is_k)
-        state_stream<true>(sst, w, xm, z, gs, full, empty, ab, stages_s, rbase, sw, c, lane);
-      else
-        state_stream<false>(sst, w, xm, z, gs, full, empty, ab, stages_s, rbase, sw, c, lane);
+        for (int tau = 0; tau < 4; ++tau)
+          w[tau][i] = hv ? p.conv_w[((size_t)(tens * H + h) * D + d0 + i) * 4 + tau] * wsc : 0.f;
 
-      // z of this chunk: the sub-streams summed in a fixed order.
+      // Gate pre-pass: per-head chunk maximum m; (a', 2^a' ln 2) per token with
+      // a' = (a - m) log2(e); l = sum 2^a'.  Entries past the chunk: (-inf, 0).
+      // Each thread holds the logits of tokens tid + 512 i in registers.
+      {
+        constexpr int kPer = kChunkMax / kSProd;
+        float a[kPer][G], m[G];
+#pragma unroll
+        for (int hh3 = 0; hh3 < G; ++hh3) m[hh3] = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+          const int tt = tid + i * kSProd;
+          const __nv_bfloat16 *gp = p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
+#pragma unroll
+          for (int hh3 = 0; hh3 < G; ++hh3) {
+            a[i][hh3] = (tt < c.n && c.hbase + hh3 < H) ? __bfloat162float(gp[hh3]) : -INFINITY;
+            m[hh3] = fmaxf(m[hh3], a[i][hh3]);
+          }
+        }
+#pragma unroll
+        for (int hh3 = 0; hh3 < G; ++hh3) {
+#pragma unroll
+          for (int o = 16; o >= 1; o >>= 1)
+            m[hh3] = fmaxf(m[hh3], __shfl_xor_sync(0xffffffffu, m[hh3], o));
+          if (lane == 0) red[warp * 4 + hh3] = m[hh3];
+        }
+        named_barrier(1, kSProd);
+        const int npad = c.nst * kSTok;
+        float l[G];
+#pragma unroll
+        for (int hh3 = 0; hh3 < G; ++hh3) {
+          float M = red[hh3];
+          for (int w2 = 1; w2 < kSProdWarps; ++w2) M = fmaxf(M, red[w2 * 4 + hh3]);
+          const bool hok = c.hbase + hh3 < H;
+          l[hh3] = 0.f;
+#pragma unroll
+          for (int i = 0; i < kPer; ++i) {
+            const int tt = tid + i * kSProd;
+            const float al = hok ? (a[i][hh3] - M) * kLog2e : -INFINITY;
+            const float ex = ex2_approx(al);
+            if (tt < npad) gw[hh3 * kSGateStride + tt] = make_float2(al, ex * kLn2);
+            l[hh3] += ex;
+          }
+#pragma unroll
+          for (int o = 16; o >= 1; o >>= 1) l[hh3] += __shfl_xor_sync(0xffffffffu, l[hh3], o);
+          if (lane == 0) red[64 + warp * 4 + hh3] = l[hh3];
+          if (tid == 0) red[128 + hh3] = M;
+        }
+        named_barrier(1, kSProd);
+        if (tid < G) {  // l of this chunk, per head, for the records
+          float lt = 0.f;
+          for (int w2 = 0; w2 < kSProdWarps; ++w2) lt += red[64 + w2 * 4 + tid];
+          red[132 + tid] = lt;
+        }
+      }
+
+      float z[4] = {0.f, 0.f, 0.f, 0.f};
+      if (is_k)
+        state_chunk_stages<true>(c.nst, c.t0, c.L, j, w, z, rr, ro, raw_full, raw_empty, op_full,
+                                 op_empty, ab, raw_s, op_s, gws, sw, lane);
+      else
+        state_chunk_stages<false>(c.nst, c.t0, c.L, j, w, z, rr, ro, raw_full, raw_empty,
+                                  op_full, op_empty, ab, raw_s, op_s, gws, sw, lane);
+
+      // z of this chunk: the token quads summed in a fixed order.
       if (is_k) {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          zred[sub * kGroupCh + 8 * c + 2 * i] = z[i].x;
-          zred[sub * kGroupCh + 8 * c + 2 * i + 1] = z[i].y;
-        }
+        for (int i = 0; i < 4; ++i) zred[j * kGroupCh + c0ch + i] = z[i];
       }
       named_barrier(1, kSProd);
       float zsum = 0.f;
       if (tid < kGroupCh)
-        for (int q = 0; q < kSSub; ++q) zsum += zred[q * kGroupCh + tid];
+        for (int jj = 0; jj < 8; ++jj) zsum += zred[jj * kGroupCh + tid];
 
       // Wait for this chunk's accumulator, then write the partial records.
       if (!mbar_wait(done, nchunk & 1, &ab) && !ab.raised()) report_error(2, ab);
@@ -497,13 +544,13 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
         const int ch = 32 * q4 + lane;                // TMEM lane = group channel (row of S)
         const int hh2 = ch / D, d = ch - D * hh2;
         const int col0 = D * hh2 + part * CPW;
-        const bool ok2 = hbase + hh2 < H;
+        const bool ok2 = c.hbase + hh2 < H;
         float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + part * CPW;
 #pragma unroll
         for (int cb = 0; cb < CPW; cb += 16) {
           float vals[16];
           tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(col0 + cb), vals);
-          tmem_ld_wait();
+          tmem_ld_wait_regs(vals);
           if (ok2) {
             float4 *dst = (float4 *)(srow + cb);
 #pragma unroll
@@ -513,12 +560,12 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
         }
         if (tid < kGroupCh) {
           const int hz = tid / D, dz = tid - D * hz;
-          if (hbase + hz < H) {
+          if (c.hbase + hz < H) {
             float *rz = p.records + ((size_t)k * G + hz) * REC;
             rz[D * D + dz] = zsum;
             if (dz == 0) {
               rz[D * D + D] = red[128 + hz];
-              rz[D * D + D + 1] = red[136 + hz];
+              rz[D * D + D + 1] = red[132 + hz];
             }
           }
         }
@@ -526,52 +573,78 @@ __global__ void __launch_bounds__(kSThreads, 1) tc_state_kernel(const StateParam
       tc_fence_before();
       named_barrier(1, kSProd);  // accumulator drained before the next chunk's MMAs
     }
+  } else if (warp == kSMmaWarp) {
+    if (lane == 0) {
+      // ---------------------------------------------------------- MMA issuer
+      constexpr uint32_t idesc = idesc_tf32_f32(128, 128);
+      const uint32_t op0 = smem_u32(smem + kSOffOp);
+      Ring ro;
+      bool ok = true;
+      for (long long kk = c0; kk < c1 && ok; ++kk) {
+        const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
+        for (int it = 0; it < c.nst; ++it) {
+          if (!mbar_wait(&op_full[ro.slot], ro.phase, &ab)) {
+            if (!ab.raised()) report_error(4, ab);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t base = op0 + ro.slot * kSOpStageBytes;
+#pragma unroll
+          for (int k8 = 0; k8 < kSTok / 8; ++k8) {  // K = 8 tf32 (32 bytes) per MMA
+            const uint64_t ad = sw128_desc(base + k8 * 32, 16, 1024);
+            const uint64_t bd = sw128_desc(base + kSOp + k8 * 32, 16, 1024);
+            mma_tf32(tmem, ad, bd, idesc, (it | k8) != 0);
+          }
+          mma_commit(&op_empty[ro.slot]);
+          ro.next(kSOpStages);
+        }
+        if (ok) mma_commit(done);
+      }
+      mma_commit(fin);  // every MMA issued above has completed once this arrives
+      if (!mbar_wait(fin, 0, nullptr)) report_error(8, ab);
+    }
   } else if (lane == 0) {
-    // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(128, 128, 1, 1);
-    uint32_t gs = 0;
-    bool ok = true;
-    for (long long kk = c0; kk < c1 && ok; ++kk) {
-      const int k = (int)kk;
-      const int b = find_batch(pre, B, k);
-      const int L = clamp_len(p.seq_lens, b, N);
-      const int nck = (L + S - 1) / S;
-      const int j = (k - pre[b]) % nck;
-      const int n = min(S, L - j * S);
-      const int nst = ((n + kSSub - 1) / kSSub + kSTokPerSub - 1) / kSTokPerSub;
-      for (int it = 0; it < nst; ++it, ++gs) {
-        const int s = gs % kSStages;
-        if (!mbar_wait(&full[s], (gs / kSStages) & 1, &ab)) {
-          if (!ab.raised()) report_error(4, ab);
-          ok = false;
+    // ------------------------------------------------------------ TMA loads
+    // Raw k and v tiles of 35 token rows (3 rows of conv history, zero-filled
+    // before the sequence start) x the group's 128 channels.
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    uint8_t *raw0 = smem + kSOffRaw;
+    uint32_t issued = 0;
+    for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
+      const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
+      for (int it = 0; it < c.nst; ++it) {
+        const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
+        if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
+          if (!ab.raised()) report_error(256, ab);
           break;
         }
-        tc_fence_after();
-        const uint32_t base = smem_u32(smem + kSOffStages + s * kSStageBytes);
-#pragma unroll
-        for (int k16 = 0; k16 < kSTok / 16; ++k16) {
-          const uint32_t o = k16 * 2048;
-          const uint64_t ad = sw128_desc(base + o, kSBlock, 1024);
-          const uint64_t bh = sw128_desc(base + kSOp + o, kSBlock, 1024);
-          const uint64_t bl = sw128_desc(base + 2 * kSOp + o, kSBlock, 1024);
-          mma_bf16(tmem, ad, bh, idesc, (it | k16) != 0);
-          mma_bf16(tmem, ad, bl, idesc, 1);
-        }
-        mma_commit(&empty[s]);
+        uint8_t *dst = raw0 + s * (2 * kSRawBytes);
+        const int tok = c.t0 + it * kSTok - kSHalo;
+        mbar_arrive_expect_tx(&raw_full[s], 2 * kSRawBytes);
+        tma_load_4d(dst, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b);
+        tma_load_4d(dst + kSRawBytes, &tm_v, &raw_full[s], 0, c.hbase, tok, c.b);
+        ++issued;
       }
-      if (ok) mma_commit(done);
     }
-    mma_commit(fin);  // every MMA issued above has completed once this arrives
-    if (!mbar_wait(fin, 0, nullptr)) report_error(8, ab);
+    // every issued copy has landed before the CTA can exit
+    for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
+      if (!mbar_wait(&raw_full[g % kSRawStages], (g / kSRawStages) & 1, nullptr))
+        report_error(512, ab);
   }
   __syncthreads();
-  if (warp == kSProdWarps) {
+  if (warp == kSMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kSTmemCols);
   }
 }
 
-// Fixed-order combination of the chunk records of one (b, h).
+// Fixed-order combination of the chunk records of one (b, h):
+//   M = max_j m_j,  S = sum_j e^{m_j - M} S_j / sum_j e^{m_j - M} l_j  (z likewise).
+// Each thread owns 4 consecutive state elements and walks the chunks in index
+// order, 16 at a time with every load of a batch in flight together; a batch
+// whose maximum exceeds the running one rescales what was summed so far.
 template <int D>
 __global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict__ records,
                                                          const int32_t *__restrict__ chunk_pre,
@@ -581,49 +654,62 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict_
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
-  constexpr int EPT = 4;  // elements per thread
-  __shared__ float s_scale[kMaxChunksPerSeq];
-  __shared__ float s_l;
+  constexpr int EPT = 4;   // elements per thread
+  constexpr int BATCH = 16;
   grid_dep_wait();
   grid_dep_launch();
   const int bh = blockIdx.x;
   const int b = bh / H, h = bh % H;
   const int hg = h / G, hh = h % G;
+  const int e0 = (blockIdx.y * 256 + threadIdx.x) * EPT;
+  if (e0 >= F) return;
   const int L = clamp_len(seq_lens, b, N);
   const int nck = (L + S - 1) / S;
   const int k0 = chunk_pre[b] + hg * nck;
   const float *rec0 = records + ((size_t)k0 * G + hh) * REC;
   const size_t rstride = (size_t)G * REC;
-  if (threadIdx.x < 32) {
-    float M = -INFINITY;
-    for (int j = threadIdx.x; j < nck; j += 32) M = fmaxf(M, rec0[j * rstride + F]);
+  float M = -INFINITY, l = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int j0 = 0; j0 < nck; j0 += BATCH) {
+    float4 v[BATCH];
+    float m[BATCH], lj[BATCH];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    for (int j = threadIdx.x; j < nck; j += 32) s_scale[j] = __expf(rec0[j * rstride + F] - M);
-    __syncwarp();
-    if (threadIdx.x == 0) {
-      float l = 0.f;
-      for (int j = 0; j < nck; ++j) l = fmaf(s_scale[j], rec0[j * rstride + F + 1], l);
-      s_l = l;
+    for (int j = 0; j < BATCH; ++j) {
+      if (j0 + j < nck) {
+        const float *r = rec0 + (size_t)(j0 + j) * rstride;
+        v[j] = __ldg((const float4 *)(r + e0));
+        m[j] = __ldg(r + F);
+        lj[j] = __ldg(r + F + 1);
+      } else {
+        v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+        m[j] = -INFINITY;
+        lj[j] = 0.f;
+      }
+    }
+    float Mb = M;
+#pragma unroll
+    for (int j = 0; j < BATCH; ++j) Mb = fmaxf(Mb, m[j]);
+    if (Mb > M) {  // rescale the running sums to the new maximum
+      const float r = (M == -INFINITY) ? 0.f : __expf(M - Mb);
+      acc.x *= r; acc.y *= r; acc.z *= r; acc.w *= r;
+      l *= r;
+      M = Mb;
+    }
+#pragma unroll
+    for (int j = 0; j < BATCH; ++j) {
+      if (j0 + j < nck) {
+        const float sc = __expf(m[j] - M);
+        acc.x = fmaf(sc, v[j].x, acc.x);
+        acc.y = fmaf(sc, v[j].y, acc.y);
+        acc.z = fmaf(sc, v[j].z, acc.z);
+        acc.w = fmaf(sc, v[j].w, acc.w);
+        l = fmaf(sc, lj[j], l);
+      }
     }
   }
-  __syncthreads();
-  const int e0 = (blockIdx.y * 256 + threadIdx.x) * EPT;
-  if (e0 >= F) return;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  const float *src = rec0 + e0;
-#pragma unroll 8
-  for (int j = 0; j < nck; ++j) {
-    const float4 v = __ldg((const float4 *)(src + j * rstride));
-    const float sc = s_scale[j];
-    acc.x = fmaf(sc, v.x, acc.x);
-    acc.y = fmaf(sc, v.y, acc.y);
-    acc.z = fmaf(sc, v.z, acc.z);
-    acc.w = fmaf(sc, v.w, acc.w);
-  }
-  const float inv = s_l > 0.f ? 1.f / s_l : 0.f;
-  float4 *dst = (float4 *)(state + (size_t)bh * F + e0);
-  *dst = make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  const float inv = l > 0.f ? 1.f / l : 0.f;
+  *(float4 *)(state + (size_t)bh * F + e0) =
+      make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
 }
 
 // ===================================================================== readout
@@ -920,12 +1006,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
           uint32_t outw[4];
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
-            // silu(g) = g / (1 + 2^(-g log2 e))
-            const float2 gg = make_float2(gv[2 * i], gv[2 * i + 1]);
-            const float2 tl = __fmul2_rn(gg, make_float2(-kLog2e, -kLog2e));
-            const float2 d2 = __fadd2_rn(make_float2(ex2_approx(tl.x), ex2_approx(tl.y)),
-                                         make_float2(1.f, 1.f));
-            const float2 sg = __fmul2_rn(gg, make_float2(rcp_approx(d2.x), rcp_approx(d2.y)));
+            // silu(g) = g sigmoid(g) = h + h tanh(h),  h = g / 2
+            const float2 hg = __fmul2_rn(make_float2(gv[2 * i], gv[2 * i + 1]),
+                                         make_float2(0.5f, 0.5f));
+            const float2 sg =
+                __ffma2_rn(hg, make_float2(tanh_approx(hg.x), tanh_approx(hg.y)), hg);
             const float2 av = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
                                          make_float2(wv8[2 * i], wv8[2 * i + 1]));
             const float2 y = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
@@ -962,6 +1047,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
             mbar_arrive(&og_empty[so]);
           }
         }
+        __syncwarp();
       } else {
         // Ragged tail: rows past the sequence end must not be written.
         if (row < nrow) {
@@ -978,6 +1064,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
           }
           mbar_arrive(&og_empty[so]);
         }
+        __syncwarp();
       }
     }
     if (ew == 0 && lane == 0) tma_store_wait_all<0>();
@@ -1031,8 +1118,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
       mma_commit(fin);  // every MMA issued above has completed once this arrives
       if (!mbar_wait(fin, 0, nullptr)) report_error(256, ab);
     }
-  } else {
-    // ------------------------------------------------------------ TMA: out_gate (lane 0), q (lane 1)
+  } else if (warp == kRTmaWarp) {
+    // ------------------------------------------------------------ TMA: out_gate
     if (lane == 0) {
       for (long long ii = i0; ii < i1; ++ii) {
         int b, h, r0, nrow;
@@ -1058,7 +1145,10 @@ __global__ void __launch_bounds__(kRThreads, 1)
           }
         }
       }
-    } else if (lane == 1 && C::QT) {
+    }
+  } else {
+    // ------------------------------------------------------------ TMA: q
+    if (lane == 0 && C::QT) {
       for (long long ii = i0; ii < i1; ++ii) {
         int b, h, r0, nrow;
         tile_of(ii, b, h, r0, nrow);
@@ -1117,6 +1207,23 @@ cudaError_t make_bnhd_map(CUtensorMap *m, const void *base, int B, int N, int H,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 4-D map over a [B, N, H, D] bf16 tensor for the state kernel's raw tiles:
+// box = one head group (128 channels) x kSRawRows tokens, no swizzle, so a
+// token's group row is 256 contiguous bytes in shared memory.
+cudaError_t make_group_map(CUtensorMap *m, const void *base, int B, int N, int H, int D) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)H, (cuuint64_t)N, (cuuint64_t)B};
+  const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)H * D * 2,
+                                 (cuuint64_t)N * H * D * 2};
+  const cuuint32_t box[4] = {(cuuint32_t)D, (cuuint32_t)(kGroupCh / D), (cuuint32_t)kSRawRows, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 struct DeviceInfo {
   int sms = 0;
   bool sm103 = false;
@@ -1170,8 +1277,6 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   const int S = chunk_len(p);
   const size_t rb = records_bytes(p, S);
   StateParams sp;
-  sp.k = (const __nv_bfloat16 *)k;
-  sp.v = (const __nv_bfloat16 *)v;
   sp.gate = (const __nv_bfloat16 *)gate;
   sp.conv_w = conv_w;
   sp.seq_lens = p.seq_lens;
@@ -1182,11 +1287,15 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   sp.N = p.N;
   sp.S = S;
   sp.HG = (p.H + G - 1) / G;
-  auto k1 = tc_state_kernel<D>;
-  cudaError_t e =
-      cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes);
+  CUtensorMap tm_k, tm_v;
+  cudaError_t e = make_group_map(&tm_k, k, p.B, p.N, p.H, D);
   if (e != cudaSuccess) return e;
-  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp);
+  if ((e = make_group_map(&tm_v, v, p.B, p.N, p.H, D)) != cudaSuccess) return e;
+  auto k1 = tc_state_kernel<D>;
+  if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
+      cudaSuccess)
+    return e;
+  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v);
   count_launch();
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
@@ -1255,6 +1364,7 @@ bool tc_supports(const Problem &p) {
   if (p.B > kMaxBatch) return false;
   if ((long long)p.N > (long long)kChunkMax * kMaxChunksPerSeq) return false;
   if ((long long)p.B * p.H > 2147483647ll / 4) return false;
+  if (p.H < kGroupCh / p.D) return false;  // the state tiles span a whole head group
   return device_info().sm103 && encode_fn() != nullptr;
 }
 
