@@ -153,6 +153,13 @@ __device__ __forceinline__ void tmem_ld_wait_regs(float (&v)[N]) {
 #pragma unroll
   for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
 }
+// Keeps reads of registers filled by an earlier tcgen05.ld after a preceding
+// tmem_ld_wait_regs (volatile asm statements keep their order).
+template <int N>
+__device__ __forceinline__ void tmem_pin(float (&v)[N]) {
+#pragma unroll
+  for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
+}
 
 // ---------------------------------------------------------------- MMA
 // Shared-memory matrix descriptor, 128-byte swizzle (sm_100 layout type 2),

@@ -55,47 +55,57 @@ using namespace sm100;
 constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the state
 
 // ------------------------------------------------------------------ state
-// 18 warps: 8 k-warps and 8 v-warps convert raw tiles into the MMA operands,
-// one warp issues the MMAs and one the TMA loads.  At most 5 warps per SM
-// sub-partition, so each thread may hold 96 registers.  K^ and V~ are written
-// as fp32 and contracted with kind::tf32 (K-major operands): no bf16 packing
-// and no hi/lo split of V~.
-constexpr int kSKWarps = 8;                          // warps producing K^ (A operand)
-constexpr int kSProdWarps = 2 * kSKWarps;            // + 8 warps producing V~ (B operand)
-constexpr int kSMmaWarp = kSProdWarps;               // 16
-constexpr int kSTmaWarp = kSProdWarps + 1;           // 17
+// 18 warps: two groups of 8 converter warps turn raw k tiles into K^ (bf16,
+// the A operand), the groups taking alternate stages; one warp issues the
+// MMAs and one the TMA loads.  At most 5 warps per SM sub-partition, so each
+// thread may hold 96 registers.  V~ is never formed: the Conv1D of v is
+// linear, so S = sum_tau w_tau (K^T v shifted by tau) with the taps applied
+// per column of the accumulators when they are drained, and the raw bf16 v
+// tiles that TMA brings in are the B operand as they stand.
+constexpr int kSGroupWarps = 8;                      // converter warps per group
+constexpr int kSCvtWarps = 2 * kSGroupWarps;         // 16
+constexpr int kSMmaWarp = kSCvtWarps;                // 16
+constexpr int kSTmaWarp = kSCvtWarps + 1;            // 17
 constexpr int kSThreads = (kSTmaWarp + 1) * 32;      // 576
-constexpr int kSProd = kSProdWarps * 32;
-constexpr int kSTok = 32;                            // tokens per stage: one 128-byte tf32 row
+constexpr int kSProd = kSCvtWarps * 32;              // converter threads
+constexpr int kSGroupThreads = kSGroupWarps * 32;
+constexpr int kSTok = 32;                            // tokens per stage
 constexpr int kSHalo = kConvW - 1;                   // conv history rows in front of a tile
 constexpr int kSRawRows = kSTok + kSHalo;            // 35
-constexpr int kSRawRow = kGroupCh * 2;               // bytes of one token's group row (bf16)
-constexpr int kSRawBytes = kSRawRows * kSRawRow;     // 8960: one raw tile of k or v
-constexpr int kSRawStages = 4;                       // raw ring (k and v tiles per stage)
-constexpr int kSOpStages = 3;                        // operand ring
-constexpr int kSOp = kGroupCh * kSTok * 4;           // one operand: 128 channel rows x 128 B
-constexpr int kSOpStageBytes = 2 * kSOp;             // A = K^T, B = V~^T
+// raw stage: v as two 64-channel MN blocks (128B swizzle, 40-row pitch) + k group rows
+constexpr int kSVBlock = 40 * 128;                   // 5120: v block pitch (1024-aligned)
+constexpr int kSVBoxBytes = kSRawRows * 128;         // 4480 written by one v box
+constexpr int kSRawRowK = kGroupCh * 2;              // bytes of one token's k group row
+constexpr int kSRawKBytes = kSRawRows * kSRawRowK;   // 8960
+constexpr int kSRawK = 2 * kSVBlock;                 // k tile offset within a raw stage
+constexpr int kSRawStage = 20 * 1024;                // 10240 + 8960, rounded to 1024
+constexpr int kSRawStages = 6;
+constexpr int kSABlock = kSTok * 128;                // 4096: one 64-channel MN block of K^
+constexpr int kSAStage = 2 * kSABlock;
+constexpr int kSAStages = 4;
 constexpr int kChunkMax = 2048;                      // longest chunk (tokens)
 constexpr int kMaxChunksPerSeq = 4096;
 constexpr int kSGateStride = kChunkMax + kSTok;      // (a', 2^a' ln 2) entries per head
-constexpr uint32_t kSTmemCols = 128;
+constexpr uint32_t kSTmemCols = 512;                 // per v block: 4 taps x 64 columns
 
 constexpr int kMaxBatch = 2048;
 
 // Shared-memory map of the state kernel (offsets from a 1024-aligned base).
-constexpr int kSOffOp = 0;
-constexpr int kSOffRaw = kSOffOp + kSOpStages * kSOpStageBytes;
-constexpr int kSOffGate = kSOffRaw + kSRawStages * 2 * kSRawBytes;  // float2 [2][kSGateStride]
-constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 8;         // float [8][128]
-constexpr int kSOffRed = kSOffZred + 8 * kGroupCh * 4;              // float [256]
+constexpr int kSOffRaw = 0;
+constexpr int kSOffA = kSOffRaw + kSRawStages * kSRawStage;
+constexpr int kSOffGate = kSOffA + kSAStages * kSAStage;            // float2 [2][kSGateStride]
+constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 8;         // float [16][128]
+constexpr int kSOffWv = kSOffZred + 16 * kGroupCh * 4;               // float4 [128]: v taps
+constexpr int kSOffRed = kSOffWv + kGroupCh * 16;                   // float [256]
 constexpr int kSOffPre = kSOffRed + 256 * 4;                        // int [kMaxBatch + 1]
 constexpr int kSOffBar = kSOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
-// raw_full, raw_empty, op_full, op_empty, done, final
-constexpr int kSBarCount = 2 * kSRawStages + 2 * kSOpStages + 2;
+// raw_full, raw_empty, a_full, a_empty, done, final
+constexpr int kSBarCount = 2 * kSRawStages + 2 * kSAStages + 2;
 constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;                // tmem addr, abort flag
 constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                  // + alignment slack
 static_assert(kSSmemBytes <= 227 * 1024, "state shared memory");
-static_assert(kSRawBytes % 128 == 0, "raw tiles keep TMA destinations 128-byte aligned");
+static_assert(kSRawK + kSRawKBytes <= kSRawStage, "raw stage");
+static_assert(kSRawStage % 1024 == 0 && kSVBlock % 1024 == 0, "swizzled v blocks");
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -258,83 +268,40 @@ __device__ __forceinline__ float2 conv_rows(const float (&w)[4][4], const float 
   return a;
 }
 
-// One stage of a converter thread: channels 4q..4q+3 of the head group at the
-// stage's tokens 4j..4j+3.  Reads the 7 raw rows it needs (3 of conv history)
-// from the TMA tile, convolves, and for K^ (IS_K) applies phi and the gate
-// weight: K^ = 2^a' phi(k~) = 2^min(x' + a', a') + (2^a' ln 2) max(x', 0), with
-// x' = k~ log2(e) (the taps carry the log2(e)) and a' = (a - m) log2(e).  Each
-// channel's 4 tokens are one 16-byte piece of its K-major row.  Tokens past
-// the sequence end (nvalid < 4, last stage only) are written as zeros.
-template <bool IS_K>
-__device__ __forceinline__ void state_convert(uint32_t raw, uint32_t op, uint32_t gws,
-                                              const float (&w)[4][4], float (&z)[4],
-                                              uint32_t sw, int nvalid) {
-  float x[7][4];
-#pragma unroll
-  for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRow), x[r]);
-  float y[4][4];  // [token][channel]
-#pragma unroll
-  for (int u = 0; u < 4; ++u) {
-    const float2 c01 = conv_rows(w, x, u, 0), c23 = conv_rows(w, x, u, 2);
-    if constexpr (IS_K) {
-      const uint2 gr = lds_v2(gws + u * 8);
-      const float al = __uint_as_float(gr.x), wl = __uint_as_float(gr.y);
-      const float2 t01 = __fadd2_rn(c01, make_float2(al, al));
-      const float2 t23 = __fadd2_rn(c23, make_float2(al, al));
-      const float2 e01 = make_float2(ex2_approx(fminf(t01.x, al)), ex2_approx(fminf(t01.y, al)));
-      const float2 e23 = make_float2(ex2_approx(fminf(t23.x, al)), ex2_approx(fminf(t23.y, al)));
-      const float2 k01 = __ffma2_rn(make_float2(wl, wl),
-                                    make_float2(fmaxf(c01.x, 0.f), fmaxf(c01.y, 0.f)), e01);
-      const float2 k23 = __ffma2_rn(make_float2(wl, wl),
-                                    make_float2(fmaxf(c23.x, 0.f), fmaxf(c23.y, 0.f)), e23);
-      y[u][0] = k01.x; y[u][1] = k01.y; y[u][2] = k23.x; y[u][3] = k23.y;
-    } else {
-      y[u][0] = c01.x; y[u][1] = c01.y; y[u][2] = c23.x; y[u][3] = c23.y;
-    }
-  }
-  if (nvalid < 4) {  // rows past the sequence end may hold anything, NaN included
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int i = 0; i < 4; ++i) y[u][i] = u < nvalid ? y[u][i] : 0.f;
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    if constexpr (IS_K) z[i] += (y[0][i] + y[1][i]) + (y[2][i] + y[3][i]);
-    sts_v4(op + i * 128 + ((sw ^ i) << 4),
-           make_uint4(__float_as_uint(y[0][i]), __float_as_uint(y[1][i]),
-                      __float_as_uint(y[2][i]), __float_as_uint(y[3][i])));
-  }
+// K^ of two channels from x' = k~ log2(e) and the token's (a', wl = 2^a' ln 2):
+// K^ = 2^a' phi(k~) = wl (x' - min(x', 0)) + 2^(min(x', 0) + a').
+__device__ __forceinline__ float2 khat2(float2 xl, float al, float wl) {
+  const float2 mn = make_float2(fminf(xl.x, 0.f), fminf(xl.y, 0.f));
+  const float2 d = __ffma2_rn(mn, make_float2(-1.f, -1.f), xl);
+  const float2 ea = __fadd2_rn(mn, make_float2(al, al));
+  const float2 e = make_float2(ex2_approx(ea.x), ex2_approx(ea.y));
+  return __ffma2_rn(make_float2(wl, wl), d, e);
 }
 
-// Ring position of a pipeline: slot and phase parity.
-struct Ring {
-  uint32_t slot = 0, phase = 0;
-  __device__ __forceinline__ void next(uint32_t n) {
-    if (++slot == n) { slot = 0; phase ^= 1; }
-  }
-};
-
-// All stages of one chunk for one converter thread.
-template <bool IS_K>
-__device__ __forceinline__ void state_chunk_stages(
-    int nst, int t0, int L, int j, const float (&w)[4][4], float (&z)[4], Ring &rr, Ring &ro,
-    uint64_t *raw_full, uint64_t *raw_empty, uint64_t *op_full, uint64_t *op_empty,
-    const AbortFlag &ab, uint32_t raw_s, uint32_t op_s, uint32_t gws, uint32_t sw, int lane) {
-  for (int it = 0; it < nst; ++it) {
-    if (!mbar_wait(&raw_full[rr.slot], rr.phase, &ab) && !ab.raised()) report_error(1, ab);
-    if (!mbar_wait(&op_empty[ro.slot], ro.phase ^ 1, &ab) && !ab.raised()) report_error(1, ab);
-    const int nvalid = min(max(L - (t0 + it * kSTok + 4 * j), 0), 4);
-    state_convert<IS_K>(raw_s + rr.slot * (2 * kSRawBytes), op_s + ro.slot * kSOpStageBytes,
-                        gws + (uint32_t)(it * kSTok) * 8, w, z, sw, nvalid);
-    fence_proxy_async_smem();  // operand writes visible to the tensor cores
-    __syncwarp();
-    if (lane == 0) {
-      mbar_arrive(&op_full[ro.slot]);
-      mbar_arrive(&raw_empty[rr.slot]);
+// One stage of a converter thread: channels 4q..4q+3 of the head group at the
+// stage's tokens 4j..4j+3.  Reads the 7 raw k rows it needs (3 of conv
+// history) from the TMA tile, convolves, applies phi and the gate weight, and
+// writes K^ as bf16 into the MN-major, 128B-swizzled A tile (one 8-byte piece
+// per token row).  Tokens past the sequence end (nvalid < 4) are zeros.
+__device__ __forceinline__ void state_convert(uint32_t raw, uint32_t arow, uint32_t cs,
+                                              uint32_t gws, const float (&w)[4][4],
+                                              float2 (&z)[2], int nvalid) {
+  float x[7][4];
+#pragma unroll
+  for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRowK), x[r]);
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const uint2 gr = lds_v2(gws + u * 8);
+    const float al = __uint_as_float(gr.x), wl = __uint_as_float(gr.y);
+    float2 k01 = khat2(conv_rows(w, x, u, 0), al, wl);
+    float2 k23 = khat2(conv_rows(w, x, u, 2), al, wl);
+    if (u >= nvalid) {  // rows past the sequence end may hold anything, NaN included
+      k01 = make_float2(0.f, 0.f);
+      k23 = make_float2(0.f, 0.f);
     }
-    rr.next(kSRawStages);
-    ro.next(kSOpStages);
+    z[0] = __fadd2_rn(z[0], k01);
+    z[1] = __fadd2_rn(z[1], k23);
+    sts_v2(arow + u * 128 + ((cs ^ u) << 4), f2_to_bf2(k01.x, k01.y), f2_to_bf2(k23.x, k23.y));
   }
 }
 
@@ -366,6 +333,39 @@ __device__ __forceinline__ ChunkRef decode_chunk(const StateParams &p, const int
   return c;
 }
 
+// Global inputs of one chunk for one converter thread, held in registers so
+// that all of them are in flight together: the k taps of its 4 channels, the
+// v taps of group channel tid (tid < 128), and the gate logits of tokens
+// tid + 256 i of the chunk (-inf past the chunk or for a missing head).
+template <int G>
+struct ChunkIn {
+  float4 wk[4];  // [channel]: taps 0..3
+  float4 wv;
+  float a[kChunkMax / kSProd][G];
+};
+template <int D, int G>
+__device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const ChunkRef &c,
+                                                  int tid, int hh, int d0, ChunkIn<G> &in) {
+  const int H = p.H, h = c.hbase + hh;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    in.wk[i] = h < H ? __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4))
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
+  in.wv = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (tid < kGroupCh) {
+    const int hz = c.hbase + tid / D, dz = tid % D;
+    if (hz < H) in.wv = __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
+  }
+#pragma unroll
+  for (int i = 0; i < kChunkMax / kSProd; ++i) {
+    const int tt = tid + i * kSProd;
+    const __nv_bfloat16 *gp = p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+      in.a[i][g] = (tt < c.n && c.hbase + g < H) ? __bfloat162float(gp[g]) : -INFINITY;
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
@@ -375,13 +375,14 @@ __global__ void __launch_bounds__(kSThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   float2 *gw = (float2 *)(smem + kSOffGate);  // [G][kSGateStride]: (a', 2^a' ln 2)
-  float *zred = (float *)(smem + kSOffZred);  // [8][128]
+  float *zred = (float *)(smem + kSOffZred);  // [16][128]
+  float4 *wv = (float4 *)(smem + kSOffWv);    // [128]: v taps of the group's channels
   float *red = (float *)(smem + kSOffRed);    // [0,64) max, [64,128) sum, 128+ m, 132+ l
   int *pre = (int *)(smem + kSOffPre);
   uint64_t *bars = (uint64_t *)(smem + kSOffBar);
   uint64_t *raw_full = bars, *raw_empty = bars + kSRawStages;
-  uint64_t *op_full = bars + 2 * kSRawStages, *op_empty = op_full + kSOpStages;
-  uint64_t *done = op_empty + kSOpStages, *fin = done + 1;
+  uint64_t *a_full = bars + 2 * kSRawStages, *a_empty = a_full + kSAStages;
+  uint64_t *done = a_empty + kSAStages, *fin = done + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + kSOffMisc);
   const AbortFlag ab{smem_u32(smem + kSOffMisc + 4)};
 
@@ -392,18 +393,18 @@ __global__ void __launch_bounds__(kSThreads, 1)
     *(volatile int *)(smem + kSOffMisc + 4) = 0;
     for (int i = 0; i < kSRawStages; ++i) {
       mbar_init(&raw_full[i], 1);
-      mbar_init(&raw_empty[i], kSProdWarps);
+      mbar_init(&raw_empty[i], kSGroupWarps + 1);  // one converter group reads k, the MMAs v
     }
-    for (int i = 0; i < kSOpStages; ++i) {
-      mbar_init(&op_full[i], kSProdWarps);
-      mbar_init(&op_empty[i], 1);
+    for (int i = 0; i < kSAStages; ++i) {
+      mbar_init(&a_full[i], kSGroupWarps);
+      mbar_init(&a_empty[i], 1);
     }
     mbar_init(done, 1);
     mbar_init(fin, 1);
     fence_mbar_init();
   }
   // Chunk prefix over the batch (converter threads), shared by all roles.
-  if (warp < kSProdWarps) {
+  if (warp < kSCvtWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
       const int L = clamp_len(p.seq_lens, b, p.N);
       return p.HG * ((L + p.S - 1) / p.S);
@@ -417,6 +418,60 @@ __global__ void __launch_bounds__(kSThreads, 1)
   const long long c1 = (long long)K * (blockIdx.x + 1) / gridDim.x;
   grid_dep_launch();
   if (c0 >= c1) return;  // no chunks for this CTA
+  const ChunkRef cfirst = decode_chunk<G>(p, pre, (int)c0);
+
+  // TMA producer state: the next (chunk, stage) to load.  Per stage: v as two
+  // 64-channel blocks of 35 token rows (128B swizzle) and the k group rows (no
+  // swizzle); 3 rows of conv history in front, zero-filled before the
+  // sequence start.
+  long long t_k = c0;
+  int t_it = 0;
+  ChunkRef t_c = cfirst;
+  uint32_t issued = 0;
+  auto tma_step = [&]() -> bool {
+    if (t_it == t_c.nst) {
+      if (++t_k >= c1) return false;
+      t_c = decode_chunk<G>(p, pre, (int)t_k);
+      t_it = 0;
+    }
+    const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
+    if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
+      if (!ab.raised()) report_error(256, ab);
+      return false;
+    }
+    uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
+    const int tok = t_c.t0 + t_it * kSTok - kSHalo;
+    const int nvb = D == 64 ? min(2, H - t_c.hbase) : 2;  // v blocks of existing heads
+    mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes + nvb * kSVBoxBytes);
+    tma_load_4d(dst + kSRawK, &tm_k, &raw_full[s], 0, t_c.hbase, tok, t_c.b);
+    for (int blk = 0; blk < nvb; ++blk)
+      tma_load_4d(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
+                  t_c.hbase + (blk * 64) / D, tok, t_c.b);
+    ++issued;
+    ++t_it;
+    return true;
+  };
+  // The first ring's worth of loads, and the first chunk's global reads of
+  // the converters, go out before the TMEM set-up.
+  if (warp == kSTmaWarp && lane == 0) {
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    for (int i = 0; i < kSRawStages && tma_step(); ++i) {
+    }
+  }
+  // Converter thread -> (group, channel quad q, token quad j): the groups take
+  // alternate stages; within a group the mapping makes both the raw-tile
+  // reads (16 lanes, 16 distinct quads of one 256-byte row) and the swizzled
+  // K^ writes (16 lanes, 16 distinct 8-byte slots of the 128-byte bank
+  // window) free of bank conflicts.
+  const int grp = warp / kSGroupWarps, gtid = tid % kSGroupThreads;
+  const int hw = 2 * (warp % kSGroupWarps) + (lane >> 4);              // half-warp 0..15
+  const int q = (lane & 15) + 16 * (hw & 1);                           // channel quad 0..31
+  const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
+  const int c0ch = 4 * q;
+  const int hh = c0ch / D, d0 = c0ch - D * hh;                         // head in group, channel
+  ChunkIn<G> cin;
+  if (warp < kSCvtWarps) load_chunk_inputs<D, G>(p, cfirst, tid, hh, d0, cin);
 
   if (warp == kSMmaWarp) tmem_alloc(tmem_slot, kSTmemCols);
   tc_fence_before();
@@ -424,138 +479,150 @@ __global__ void __launch_bounds__(kSThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp < kSProdWarps) {
+  if (warp < kSCvtWarps) {
     // ------------------------------------------------------------ converters
-    // Thread -> (channel quad q, token quad j) of each stage, chosen so that
-    // both the raw-tile reads (16 lanes, 16 distinct quads of one 256-byte
-    // row) and the swizzled operand writes (8 lanes, 8 distinct 16-byte
-    // chunks) are free of bank conflicts.
-    const bool is_k = warp < kSKWarps;
-    const int hw = 2 * (warp % kSKWarps) + (lane >> 4);          // half-warp 0..15
-    const int q = (lane & 15) + 16 * (hw & 1);                   // channel quad 0..31
-    const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
-    const int c0ch = 4 * q;
-    const int hh = c0ch / D, d0 = c0ch - D * hh;                 // head in group, channel
-    const int tens = is_k ? 1 : 2;                               // conv_w stream: 1 = k, 2 = v
-    // K-major tf32 rows (128 B = 32 tokens), 128-byte swizzle: channel row r at
-    // (r >> 3) * 1024 + (r & 7) * 128; this thread's 16 bytes are chunk j ^ (r & 7)
-    const uint32_t rbase = (q >> 1) * 1024 + (q & 1) * 512;
-    const uint32_t sw = (uint32_t)(j ^ ((q & 1) * 4));
-    const uint32_t op_s = smem_u32(smem + kSOffOp) + (is_k ? 0u : (uint32_t)kSOp) + rbase;
-    const uint32_t raw_s = smem_u32(smem + kSOffRaw) + (is_k ? 0u : (uint32_t)kSRawBytes) +
-                           (uint32_t)(4 * j * kSRawRow + q * 8);
+    // K^ rows: MN block q / 16, token row 4j + u, 16-byte chunk (q % 16) / 2
+    // swizzled by the row, 8-byte half q & 1
+    const uint32_t arow0 = smem_u32(smem + kSOffA) + (uint32_t)((q >> 4) * kSABlock +
+                                                                4 * j * 128 + (q & 1) * 8);
+    const uint32_t cs = (uint32_t)(((q & 15) >> 1) ^ (4 * (j & 1)));
+    const uint32_t raw0 = smem_u32(smem + kSOffRaw + kSRawK) + (uint32_t)(4 * j * kSRawRowK + q * 8);
     const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kSGateStride + 4 * j) * 8;
-    Ring rr, ro;
+    uint32_t gs0 = 0;  // first stage of the chunk in the CTA's stage sequence
     int nchunk = 0;
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
-      const ChunkRef c = decode_chunk<G>(p, pre, k);
+      const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, k);
+      if (kk != c0) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
 
-      // taps of this thread's 4 channels; for k pre-scaled by log2(e)
-      const int h = c.hbase + hh;
-      const bool hv = h < H;
+      // k taps of this thread's 4 channels, pre-scaled by log2(e); v taps of
+      // the group's channels for the drain
       float w[4][4];
-      const float wsc = is_k ? kLog2e : 1.f;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int tau = 0; tau < 4; ++tau)
-          w[tau][i] = hv ? p.conv_w[((size_t)(tens * H + h) * D + d0 + i) * 4 + tau] * wsc : 0.f;
+      for (int i = 0; i < 4; ++i) {
+        w[0][i] = cin.wk[i].x * kLog2e;
+        w[1][i] = cin.wk[i].y * kLog2e;
+        w[2][i] = cin.wk[i].z * kLog2e;
+        w[3][i] = cin.wk[i].w * kLog2e;
+      }
+      if (tid < kGroupCh) wv[tid] = cin.wv;
 
       // Gate pre-pass: per-head chunk maximum m; (a', 2^a' ln 2) per token with
       // a' = (a - m) log2(e); l = sum 2^a'.  Entries past the chunk: (-inf, 0).
-      // Each thread holds the logits of tokens tid + 512 i in registers.
       {
         constexpr int kPer = kChunkMax / kSProd;
-        float a[kPer][G], m[G];
+        float m[G];
 #pragma unroll
-        for (int hh3 = 0; hh3 < G; ++hh3) m[hh3] = -INFINITY;
+        for (int g = 0; g < G; ++g) {
+          m[g] = -INFINITY;
 #pragma unroll
-        for (int i = 0; i < kPer; ++i) {
-          const int tt = tid + i * kSProd;
-          const __nv_bfloat16 *gp = p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
+          for (int i = 0; i < kPer; ++i) m[g] = fmaxf(m[g], cin.a[i][g]);
 #pragma unroll
-          for (int hh3 = 0; hh3 < G; ++hh3) {
-            a[i][hh3] = (tt < c.n && c.hbase + hh3 < H) ? __bfloat162float(gp[hh3]) : -INFINITY;
-            m[hh3] = fmaxf(m[hh3], a[i][hh3]);
-          }
-        }
-#pragma unroll
-        for (int hh3 = 0; hh3 < G; ++hh3) {
-#pragma unroll
-          for (int o = 16; o >= 1; o >>= 1)
-            m[hh3] = fmaxf(m[hh3], __shfl_xor_sync(0xffffffffu, m[hh3], o));
-          if (lane == 0) red[warp * 4 + hh3] = m[hh3];
+          for (int o = 16; o >= 1; o >>= 1) m[g] = fmaxf(m[g], __shfl_xor_sync(0xffffffffu, m[g], o));
+          if (lane == 0) red[warp * 4 + g] = m[g];
         }
         named_barrier(1, kSProd);
         const int npad = c.nst * kSTok;
-        float l[G];
 #pragma unroll
-        for (int hh3 = 0; hh3 < G; ++hh3) {
-          float M = red[hh3];
-          for (int w2 = 1; w2 < kSProdWarps; ++w2) M = fmaxf(M, red[w2 * 4 + hh3]);
-          const bool hok = c.hbase + hh3 < H;
-          l[hh3] = 0.f;
+        for (int g = 0; g < G; ++g) {
+          float M = red[g];
+          for (int w2 = 1; w2 < kSCvtWarps; ++w2) M = fmaxf(M, red[w2 * 4 + g]);
+          const bool hok = c.hbase + g < H;
+          float l = 0.f;
 #pragma unroll
           for (int i = 0; i < kPer; ++i) {
             const int tt = tid + i * kSProd;
-            const float al = hok ? (a[i][hh3] - M) * kLog2e : -INFINITY;
+            const float al = hok ? (cin.a[i][g] - M) * kLog2e : -INFINITY;
             const float ex = ex2_approx(al);
-            if (tt < npad) gw[hh3 * kSGateStride + tt] = make_float2(al, ex * kLn2);
-            l[hh3] += ex;
+            if (tt < npad) gw[g * kSGateStride + tt] = make_float2(al, ex * kLn2);
+            l += ex;
           }
 #pragma unroll
-          for (int o = 16; o >= 1; o >>= 1) l[hh3] += __shfl_xor_sync(0xffffffffu, l[hh3], o);
-          if (lane == 0) red[64 + warp * 4 + hh3] = l[hh3];
-          if (tid == 0) red[128 + hh3] = M;
+          for (int o = 16; o >= 1; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+          if (lane == 0) red[64 + warp * 4 + g] = l;
+          if (tid == 0) red[128 + g] = M;
         }
         named_barrier(1, kSProd);
         if (tid < G) {  // l of this chunk, per head, for the records
           float lt = 0.f;
-          for (int w2 = 0; w2 < kSProdWarps; ++w2) lt += red[64 + w2 * 4 + tid];
+          for (int w2 = 0; w2 < kSCvtWarps; ++w2) lt += red[64 + w2 * 4 + tid];
           red[132 + tid] = lt;
         }
       }
 
-      float z[4] = {0.f, 0.f, 0.f, 0.f};
-      if (is_k)
-        state_chunk_stages<true>(c.nst, c.t0, c.L, j, w, z, rr, ro, raw_full, raw_empty, op_full,
-                                 op_empty, ab, raw_s, op_s, gws, sw, lane);
-      else
-        state_chunk_stages<false>(c.nst, c.t0, c.L, j, w, z, rr, ro, raw_full, raw_empty,
-                                  op_full, op_empty, ab, raw_s, op_s, gws, sw, lane);
-
-      // z of this chunk: the token quads summed in a fixed order.
-      if (is_k) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) zred[j * kGroupCh + c0ch + i] = z[i];
+      float2 z[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      for (int it = (int)((gs0 ^ grp) & 1); it < c.nst; it += 2) {  // this group's stages
+        const uint32_t gs = gs0 + it;
+        const uint32_t rs = gs % kSRawStages, rph = (gs / kSRawStages) & 1;
+        const uint32_t as = gs % kSAStages, aph = (gs / kSAStages) & 1;
+        if (!mbar_wait(&raw_full[rs], rph, &ab) && !ab.raised()) report_error(1, ab);
+        if (!mbar_wait(&a_empty[as], aph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
+        const int T = c.t0 + it * kSTok;
+        const int nvalid = min(max(c.L - (T + 4 * j), 0), 4);
+        state_convert(raw0 + rs * kSRawStage, arow0 + as * kSAStage, cs,
+                      gws + (uint32_t)(it * kSTok) * 8, w, z, nvalid);
+        if (T + kSTok > c.L) {
+          // v rows past the sequence end meet K^ = 0 in the MMA, but may hold
+          // NaN or inf: zero them (both 64-channel blocks)
+          const int r0 = max(c.L - (T - kSHalo), 0);
+          const uint32_t vb = smem_u32(smem + kSOffRaw) + rs * kSRawStage;
+          for (int e = gtid; e < (kSRawRows - r0) * 16; e += kSGroupThreads) {
+            const int r = r0 + e / 16, blk = (e / 8) & 1, ck = e & 7;
+            sts_v4(vb + blk * kSVBlock + r * 128 + ck * 16, make_uint4(0, 0, 0, 0));
+          }
+        }
+        fence_proxy_async_smem();  // K^ (and zeroed v rows) visible to the tensor cores
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&a_full[as]);
+          mbar_arrive(&raw_empty[rs]);
+        }
       }
+      gs0 += c.nst;
+
+      // z of this chunk: the token quads of both groups summed in a fixed order.
+      *(float4 *)&zred[(grp * 8 + j) * kGroupCh + c0ch] = make_float4(z[0].x, z[0].y, z[1].x, z[1].y);
       named_barrier(1, kSProd);
       float zsum = 0.f;
       if (tid < kGroupCh)
-        for (int jj = 0; jj < 8; ++jj) zsum += zred[jj * kGroupCh + tid];
+        for (int jj = 0; jj < 16; ++jj) zsum += zred[jj * kGroupCh + tid];
 
-      // Wait for this chunk's accumulator, then write the partial records.
+      // Wait for this chunk's accumulators, then write the partial records:
+      // S[a][c] = sum_tau w_tau[c] P_tau[a][c] on the diagonal D x D blocks.
+      // P_tau of v channel c = 64 blk + c' sits in TMEM column 256 blk + 64 tau + c'.
       if (!mbar_wait(done, nchunk & 1, &ab) && !ab.raised()) report_error(2, ab);
       tc_fence_after();
-      if (warp < 8) {  // two warps per TMEM lane quarter, half of the columns each
-        constexpr int CPW = D / 2;                    // columns per warp
-        const int q4 = warp & 3, part = warp >> 2;    // lane quarter, column half
+      {
+        constexpr int CPW = D / 4;                    // columns per warp
+        const int q4 = warp & 3, part = warp >> 2;    // lane quarter, column quarter
         const int ch = 32 * q4 + lane;                // TMEM lane = group channel (row of S)
         const int hh2 = ch / D, d = ch - D * hh2;
-        const int col0 = D * hh2 + part * CPW;
+        const int cv0 = D * hh2 + part * CPW;         // first v channel (of the group) of this warp
         const bool ok2 = c.hbase + hh2 < H;
         float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + part * CPW;
+        const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16) +
+                            (uint32_t)(256 * (cv0 / 64) + cv0 % 64);
+#pragma unroll 1
+        for (int cb = 0; cb < CPW; cb += 8) {
+          float v0[8], v1[8], v2[8], v3[8];
+          tmem_ld8(tl + cb, v0);
+          tmem_ld8(tl + 64 + cb, v1);
+          tmem_ld8(tl + 128 + cb, v2);
+          tmem_ld8(tl + 192 + cb, v3);
+          tmem_ld_wait_regs(v0);
+          tmem_pin(v1);
+          tmem_pin(v2);
+          tmem_pin(v3);
+          float o[8];
 #pragma unroll
-        for (int cb = 0; cb < CPW; cb += 16) {
-          float vals[16];
-          tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(col0 + cb), vals);
-          tmem_ld_wait_regs(vals);
+          for (int i = 0; i < 8; ++i) {
+            const float4 wt = wv[cv0 + cb + i];
+            o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
+          }
           if (ok2) {
             float4 *dst = (float4 *)(srow + cb);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              dst[i] = make_float4(vals[4 * i], vals[4 * i + 1], vals[4 * i + 2], vals[4 * i + 3]);
+            dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+            dst[1] = make_float4(o[4], o[5], o[6], o[7]);
           }
         }
         if (tid < kGroupCh) {
@@ -571,33 +638,42 @@ __global__ void __launch_bounds__(kSThreads, 1)
         }
       }
       tc_fence_before();
-      named_barrier(1, kSProd);  // accumulator drained before the next chunk's MMAs
+      named_barrier(1, kSProd);  // accumulators drained before the next chunk's MMAs
     }
   } else if (warp == kSMmaWarp) {
     if (lane == 0) {
       // ---------------------------------------------------------- MMA issuer
-      constexpr uint32_t idesc = idesc_tf32_f32(128, 128);
-      const uint32_t op0 = smem_u32(smem + kSOffOp);
-      Ring ro;
+      // P_tau += K^T v[t - 3 + tau] for tau = 0..3 in one N = 256 MMA per
+      // 64-channel v block: its four 64-column B blocks are the same raw tile
+      // with the start moved down 0..3 rows (LBO = one 128-byte row).  The
+      // 128-byte swizzle follows the absolute shared address, so the shifted
+      // views read the rows TMA wrote.
+      constexpr uint32_t idesc = idesc_bf16_f32(128, 256, 1, 1);
+      const uint32_t a0 = smem_u32(smem + kSOffA), v0 = smem_u32(smem + kSOffRaw);
+      uint32_t gs = 0;
       bool ok = true;
       for (long long kk = c0; kk < c1 && ok; ++kk) {
         const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
-        for (int it = 0; it < c.nst; ++it) {
-          if (!mbar_wait(&op_full[ro.slot], ro.phase, &ab)) {
+        for (int it = 0; it < c.nst; ++it, ++gs) {
+          const uint32_t rs = gs % kSRawStages, rph = (gs / kSRawStages) & 1;
+          const uint32_t as = gs % kSAStages, aph = (gs / kSAStages) & 1;
+          if (!mbar_wait(&a_full[as], aph, &ab) || !mbar_wait(&raw_full[rs], rph, &ab)) {
             if (!ab.raised()) report_error(4, ab);
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t base = op0 + ro.slot * kSOpStageBytes;
+          const uint32_t ab0 = a0 + as * kSAStage, vb0 = v0 + rs * kSRawStage;
 #pragma unroll
-          for (int k8 = 0; k8 < kSTok / 8; ++k8) {  // K = 8 tf32 (32 bytes) per MMA
-            const uint64_t ad = sw128_desc(base + k8 * 32, 16, 1024);
-            const uint64_t bd = sw128_desc(base + kSOp + k8 * 32, 16, 1024);
-            mma_tf32(tmem, ad, bd, idesc, (it | k8) != 0);
-          }
-          mma_commit(&op_empty[ro.slot]);
-          ro.next(kSOpStages);
+          for (int blk = 0; blk < 2; ++blk)
+#pragma unroll
+            for (int k16 = 0; k16 < kSTok / 16; ++k16) {
+              const uint64_t ad = sw128_desc(ab0 + k16 * 2048, kSABlock, 1024);
+              const uint64_t bd = sw128_desc(vb0 + blk * kSVBlock + 16 * k16 * 128, 128, 1024);
+              mma_bf16(tmem + 256 * blk, ad, bd, idesc, (it | k16) != 0);
+            }
+          mma_commit(&a_empty[as]);
+          mma_commit(&raw_empty[rs]);
         }
         if (ok) mma_commit(done);
       }
@@ -606,27 +682,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     }
   } else if (lane == 0) {
     // ------------------------------------------------------------ TMA loads
-    // Raw k and v tiles of 35 token rows (3 rows of conv history, zero-filled
-    // before the sequence start) x the group's 128 channels.
-    tma_prefetch_desc(&tm_k);
-    tma_prefetch_desc(&tm_v);
-    uint8_t *raw0 = smem + kSOffRaw;
-    uint32_t issued = 0;
-    for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
-      const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
-      for (int it = 0; it < c.nst; ++it) {
-        const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
-        if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
-          if (!ab.raised()) report_error(256, ab);
-          break;
-        }
-        uint8_t *dst = raw0 + s * (2 * kSRawBytes);
-        const int tok = c.t0 + it * kSTok - kSHalo;
-        mbar_arrive_expect_tx(&raw_full[s], 2 * kSRawBytes);
-        tma_load_4d(dst, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b);
-        tma_load_4d(dst + kSRawBytes, &tm_v, &raw_full[s], 0, c.hbase, tok, c.b);
-        ++issued;
-      }
+    while (!ab.raised() && tma_step()) {
     }
     // every issued copy has landed before the CTA can exit
     for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
@@ -1295,7 +1351,7 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   CUtensorMap tm_k, tm_v;
   cudaError_t e = make_group_map(&tm_k, k, p.B, p.N, p.H, D);
   if (e != cudaSuccess) return e;
-  if ((e = make_group_map(&tm_v, v, p.B, p.N, p.H, D)) != cudaSuccess) return e;
+  if ((e = make_bnhd_map(&tm_v, v, p.B, p.N, p.H, D, kSRawRows)) != cudaSuccess) return e;
   auto k1 = tc_state_kernel<D>;
   if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
       cudaSuccess)
