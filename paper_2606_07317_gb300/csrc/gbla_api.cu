@@ -118,10 +118,12 @@ gbla_status run_state(const Problem &p, bool tc, const void *k, const void *v,
   return from_cuda(simt_state(p, plan, k, v, gate, conv_w, (float *)ws.ptr, state, st));
 }
 
+// after_state: the kernel just before on the stream is this library's state
+// reduction, so only the readout's reads of `state` wait for it.
 gbla_status run_readout(const Problem &p, bool tc, const void *q, const void *og,
                         const float *conv_w, const float *norm_w, const float *state,
-                        void *o, cudaStream_t st) {
-  if (tc) return from_cuda(tc_readout(p, q, og, conv_w, norm_w, state, o, st));
+                        void *o, cudaStream_t st, bool after_state = false) {
+  if (tc) return from_cuda(tc_readout(p, q, og, conv_w, norm_w, state, o, st, after_state));
   return from_cuda(simt_readout(p, q, og, conv_w, norm_w, state, o, st));
 }
 
@@ -224,7 +226,8 @@ gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
   Scratch state;
   if ((s = state.alloc(sizeof(float) * state_floats(D) * B * H, st)) != GBLA_OK) return s;
   if ((s = run_state(p, tc, k, v, gate, conv_w, (float *)state.ptr, st)) != GBLA_OK) return s;
-  return run_readout(p, tc, q, out_gate, conv_w, norm_w, (const float *)state.ptr, o, st);
+  return run_readout(p, tc, q, out_gate, conv_w, norm_w, (const float *)state.ptr, o, st,
+                     true);
 }
 
 gbla_status gbla_forward(const void *q, const void *k, const void *v,

@@ -46,9 +46,13 @@ size_t tc_workspace_bytes(const Problem &p);
 cudaError_t tc_state(const Problem &p, const void *k, const void *v,
                      const void *gate, const float *conv_w, void *workspace,
                      float *state, cudaStream_t st);
+// after_state: launched right behind tc_state on the same stream; only the
+// reads of `state` then wait for the preceding kernel (the other inputs were
+// complete before tc_state started).
 cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
                        const float *conv_w, const float *norm_w,
-                       const float *state, void *o, cudaStream_t st);
+                       const float *state, void *o, cudaStream_t st,
+                       bool after_state = false);
 // Error bits set by tensor-core kernels whose bounded waits ran out (0 = none);
 // synchronous read of the current device, optionally clearing it.
 unsigned tc_device_error(bool reset);

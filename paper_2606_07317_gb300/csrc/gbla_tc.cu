@@ -366,6 +366,21 @@ __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const Ch
   }
 }
 
+// L2 prefetch of what load_chunk_inputs will read, holding no registers.
+template <int D, int G>
+__device__ __forceinline__ void prefetch_chunk_inputs(const StateParams &p, const ChunkRef &c,
+                                                      int tid, int hh, int d0) {
+  const int H = p.H, h = c.hbase + hh;
+  if (h < H) prefetch_l2_line(p.conv_w + ((size_t)(H + h) * D + d0) * 4);
+  if (tid < kGroupCh && c.hbase + tid / D < H)
+    prefetch_l2_line(p.conv_w + ((size_t)(2 * H + c.hbase + tid / D) * D + tid % D) * 4);
+#pragma unroll
+  for (int i = 0; i < kChunkMax / kSProd; ++i) {
+    const int tt = tid + i * kSProd;
+    if (tt < c.n) prefetch_l2_line(p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase);
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
@@ -420,45 +435,44 @@ __global__ void __launch_bounds__(kSThreads, 1)
   if (c0 >= c1) return;  // no chunks for this CTA
   const ChunkRef cfirst = decode_chunk<G>(p, pre, (int)c0);
 
-  // TMA producer state: the next (chunk, stage) to load.  Per stage: v as two
-  // 64-channel blocks of 35 token rows (128B swizzle) and the k group rows (no
-  // swizzle); 3 rows of conv history in front, zero-filled before the
-  // sequence start.
-  long long t_k = c0;
-  int t_it = 0;
-  ChunkRef t_c = cfirst;
-  uint32_t issued = 0;
-  auto tma_step = [&]() -> bool {
-    if (t_it == t_c.nst) {
-      if (++t_k >= c1) return false;
-      t_c = decode_chunk<G>(p, pre, (int)t_k);
-      t_it = 0;
+  if (warp == kSTmaWarp) {
+    // ------------------------------------------------------------ TMA loads
+    // Per stage: v as two 64-channel blocks of 35 token rows (128B swizzle)
+    // and the k group rows (no swizzle); 3 rows of conv history in front,
+    // zero-filled before the sequence start.  This warp takes no part in the
+    // TMEM hand-off, so its first loads go out at once.
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      uint32_t issued = 0;
+      for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
+        const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, (int)kk);
+        const int nvb = D == 64 ? min(2, H - c.hbase) : 2;  // v blocks of existing heads
+        for (int it = 0; it < c.nst; ++it) {
+          const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
+          if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
+            if (!ab.raised()) report_error(2048, ab);
+            break;
+          }
+          uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
+          const int tok = c.t0 + it * kSTok - kSHalo;
+          mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes + nvb * kSVBoxBytes);
+          tma_load_4d(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b);
+          for (int blk = 0; blk < nvb; ++blk)
+            tma_load_4d(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
+                        c.hbase + (blk * 64) / D, tok, c.b);
+          ++issued;
+        }
+      }
+      // every issued copy has landed before the CTA can exit
+      for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
+        if (!mbar_wait(&raw_full[g % kSRawStages], (g / kSRawStages) & 1, nullptr))
+          report_error(4096, ab);
     }
-    const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
-    if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
-      if (!ab.raised()) report_error(256, ab);
-      return false;
-    }
-    uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
-    const int tok = t_c.t0 + t_it * kSTok - kSHalo;
-    const int nvb = D == 64 ? min(2, H - t_c.hbase) : 2;  // v blocks of existing heads
-    mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes + nvb * kSVBoxBytes);
-    tma_load_4d(dst + kSRawK, &tm_k, &raw_full[s], 0, t_c.hbase, tok, t_c.b);
-    for (int blk = 0; blk < nvb; ++blk)
-      tma_load_4d(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
-                  t_c.hbase + (blk * 64) / D, tok, t_c.b);
-    ++issued;
-    ++t_it;
-    return true;
-  };
-  // The first ring's worth of loads, and the first chunk's global reads of
-  // the converters, go out before the TMEM set-up.
-  if (warp == kSTmaWarp && lane == 0) {
-    tma_prefetch_desc(&tm_k);
-    tma_prefetch_desc(&tm_v);
-    for (int i = 0; i < kSRawStages && tma_step(); ++i) {
-    }
+    __syncthreads();
+    return;
   }
+
   // Converter thread -> (group, channel quad q, token quad j): the groups take
   // alternate stages; within a group the mapping makes both the raw-tile
   // reads (16 lanes, 16 distinct quads of one 256-byte row) and the swizzled
@@ -470,12 +484,14 @@ __global__ void __launch_bounds__(kSThreads, 1)
   const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
   const int c0ch = 4 * q;
   const int hh = c0ch / D, d0 = c0ch - D * hh;                         // head in group, channel
+  // The first chunk's global reads are pulled into L2 during the TMEM hand-off
+  // (holding them in registers across it would spill).
+  if (warp < kSCvtWarps) prefetch_chunk_inputs<D, G>(p, cfirst, tid, hh, d0);
   ChunkIn<G> cin;
-  if (warp < kSCvtWarps) load_chunk_inputs<D, G>(p, cfirst, tid, hh, d0, cin);
 
   if (warp == kSMmaWarp) tmem_alloc(tmem_slot, kSTmemCols);
   tc_fence_before();
-  __syncthreads();
+  named_barrier(2, kSThreads - 32);  // converters and the MMA warp
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
@@ -493,7 +509,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
       const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, k);
-      if (kk != c0) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
+      load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
 
       // k taps of this thread's 4 channels, pre-scaled by log2(e); v taps of
       // the group's channels for the drain
@@ -680,14 +696,6 @@ __global__ void __launch_bounds__(kSThreads, 1)
       mma_commit(fin);  // every MMA issued above has completed once this arrives
       if (!mbar_wait(fin, 0, nullptr)) report_error(8, ab);
     }
-  } else if (lane == 0) {
-    // ------------------------------------------------------------ TMA loads
-    while (!ab.raised() && tma_step()) {
-    }
-    // every issued copy has landed before the CTA can exit
-    for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
-      if (!mbar_wait(&raw_full[g % kSRawStages], (g / kSRawStages) & 1, nullptr))
-        report_error(512, ab);
   }
   __syncthreads();
   if (warp == kSMmaWarp) {
@@ -699,10 +707,11 @@ __global__ void __launch_bounds__(kSThreads, 1)
 // Fixed-order combination of the chunk records of one (b, h):
 //   M = max_j m_j,  S = sum_j e^{m_j - M} S_j / sum_j e^{m_j - M} l_j  (z likewise).
 // Each thread owns 4 consecutive state elements and walks the chunks in index
-// order, 16 at a time with every load of a batch in flight together; a batch
+// order, 24 at a time with every load of a batch in flight together; a batch
 // whose maximum exceeds the running one rescales what was summed so far.
+constexpr int kReduceThreads = 128;
 template <int D>
-__global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict__ records,
+__global__ void __launch_bounds__(kReduceThreads) tc_reduce_kernel(const float *__restrict__ records,
                                                          const int32_t *__restrict__ chunk_pre,
                                                          const int32_t *__restrict__ seq_lens,
                                                          float *__restrict__ state, int B, int H,
@@ -711,13 +720,13 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const float *__restrict_
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
   constexpr int EPT = 4;   // elements per thread
-  constexpr int BATCH = 16;
+  constexpr int BATCH = 24;
   grid_dep_wait();
   grid_dep_launch();
   const int bh = blockIdx.x;
   const int b = bh / H, h = bh % H;
   const int hg = h / G, hh = h % G;
-  const int e0 = (blockIdx.y * 256 + threadIdx.x) * EPT;
+  const int e0 = (blockIdx.y * kReduceThreads + threadIdx.x) * EPT;
   if (e0 >= F) return;
   const int L = clamp_len(seq_lens, b, N);
   const int nck = (L + S - 1) / S;
@@ -776,6 +785,7 @@ struct ReadoutParams {
   __nv_bfloat16 *o;
   int B, H, N;
   float eps;
+  int wait_late;  // only the reads of `state` wait for the preceding kernel
 };
 
 // phi(conv(q)) for 4 consecutive rows of one producer sub-stream; xm holds the
@@ -854,8 +864,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
     tma_prefetch_desc(&tm_o);
     tma_prefetch_desc(&tm_q);
   }
-  // Everything below may read what earlier work on the stream wrote.
-  grid_dep_wait();
+  // Everything below may read what earlier work on the stream wrote, unless
+  // that work is the state reduction, which only `state` depends on.
+  if (!p.wait_late) grid_dep_wait();
   if (warp < 4) {
     prefix_counts(pre, B, tid, 128, 1, s_tot, [&](int b) {
       const int L = clamp_len(p.seq_lens, b, N);
@@ -901,38 +912,58 @@ __global__ void __launch_bounds__(kRThreads, 1)
         // once the MMAs that read the previous one have completed.
         if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, &ab) && !ab.raised())
           report_error(16, ab);
+        // q taps first (in flight during the rebuild), pre-scaled by log2(e)
+        // later (phi2_log2 takes x log2(e)): 32 consecutive floats per thread
+        float4 wq4[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          wq4[i] = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + 8 * c + i) * 4));
+        if (nbh == 0) grid_dep_wait();  // the state comes from the preceding kernel
         const float *st = p.state + ((size_t)b * H + h) * F;
-        for (int item = tid; item < NR * (D / 8); item += kRProd) {
-          const int e = item % NR, ck = item / NR;  // row e of B, 8-element K chunk ck
-          float vals[8];
+        constexpr int NI = NR * (D / 8);  // (row e of B, 8-element K chunk ck) items
+        for (int item0 = tid; item0 < NI; item0 += 2 * kRProd) {
+          float vals[2][8];  // both items' loads in flight together
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int d = 8 * ck + i;
-            vals[i] = e < D ? st[(size_t)d * D + e] : (e == D ? st[D * D + d] : 0.f);
-          }
-          uint32_t hi[4], lo[4];
+          for (int u = 0; u < 2; ++u) {
+            const int item = item0 + u * kRProd;
+            const int e = item % NR, ck = item / NR;
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            hi[i] = f2_to_bf2(vals[2 * i], vals[2 * i + 1]);
-            const float2 r2 = __ffma2_rn(bf2_to_f2(hi[i]), make_float2(-1.f, -1.f),
-                                         make_float2(vals[2 * i], vals[2 * i + 1]));
-            lo[i] = f2_to_bf2(r2.x, r2.y);
+            for (int i = 0; i < 8; ++i) {
+              const int d = 8 * ck + i;
+              vals[u][i] = item < NI && e < D ? st[(size_t)d * D + e]
+                                              : (item < NI && e == D ? st[D * D + d] : 0.f);
+            }
           }
-          const int kbk = ck >> 3, ckk = ck & 7;
-          const uint32_t off = kbk * (NR * 128) + (e >> 3) * 1024 + (e & 7) * 128 +
-                               ((ckk ^ (e & 7)) << 4);
-          sts_v4(smem_u32(smem + C::kOffBhi) + off, make_uint4(hi[0], hi[1], hi[2], hi[3]));
-          sts_v4(smem_u32(smem + C::kOffBlo) + off, make_uint4(lo[0], lo[1], lo[2], lo[3]));
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int item = item0 + u * kRProd;
+            if (item >= NI) break;
+            const int e = item % NR, ck = item / NR;
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              hi[i] = f2_to_bf2(vals[u][2 * i], vals[u][2 * i + 1]);
+              const float2 r2 = __ffma2_rn(bf2_to_f2(hi[i]), make_float2(-1.f, -1.f),
+                                           make_float2(vals[u][2 * i], vals[u][2 * i + 1]));
+              lo[i] = f2_to_bf2(r2.x, r2.y);
+            }
+            const int kbk = ck >> 3, ckk = ck & 7;
+            const uint32_t off = kbk * (NR * 128) + (e >> 3) * 1024 + (e & 7) * 128 +
+                                 ((ckk ^ (e & 7)) << 4);
+            sts_v4(smem_u32(smem + C::kOffBhi) + off, make_uint4(hi[0], hi[1], hi[2], hi[3]));
+            sts_v4(smem_u32(smem + C::kOffBlo) + off, make_uint4(lo[0], lo[1], lo[2], lo[3]));
+          }
         }
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(b_full);
-        // q taps, pre-scaled by log2(e) (phi2_log2 takes x log2(e))
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            wq[q][i] = p.conv_w[((size_t)(0 * H + h) * D + 8 * c + i) * 4 + q] * kLog2e;
+        for (int i = 0; i < 8; ++i) {
+          wq[0][i] = wq4[i].x * kLog2e;
+          wq[1][i] = wq4[i].y * kLog2e;
+          wq[2][i] = wq4[i].z * kLog2e;
+          wq[3][i] = wq4[i].w * kLog2e;
+        }
         cur_b = b;
         cur_h = h;
         ++nbh;
@@ -1365,8 +1396,8 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.gridDim = dim3(p.B * p.H, (F / 4 + 255) / 256);
-  cfg.blockDim = dim3(256);
+  cfg.gridDim = dim3(p.B * p.H, (F / 4 + kReduceThreads - 1) / kReduceThreads);
+  cfg.blockDim = dim3(kReduceThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
   cfg.attrs = attr;
@@ -1379,7 +1410,8 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
 
 template <int D>
 cudaError_t run_readout(const Problem &p, const void *q, const void *og, const float *conv_w,
-                        const float *norm_w, const float *state, void *o, cudaStream_t st) {
+                        const float *norm_w, const float *state, void *o, cudaStream_t st,
+                        bool after_state) {
   using C = ReadoutCfg<D>;
   CUtensorMap tm_og, tm_o, tm_q;
   cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D, kRTok);
@@ -1398,6 +1430,7 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   rp.H = p.H;
   rp.N = p.N;
   rp.eps = kRmsEps;
+  rp.wait_late = after_state ? 1 : 0;
   auto kern = tc_readout_kernel<D>;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem)) !=
       cudaSuccess)
@@ -1443,10 +1476,11 @@ cudaError_t tc_state(const Problem &p, const void *k, const void *v, const void 
 }
 
 cudaError_t tc_readout(const Problem &p, const void *q, const void *og, const float *conv_w,
-                       const float *norm_w, const float *state, void *o, cudaStream_t st) {
+                       const float *norm_w, const float *state, void *o, cudaStream_t st,
+                       bool after_state) {
   switch (p.D) {
-    case 64: return run_readout<64>(p, q, og, conv_w, norm_w, state, o, st);
-    case 128: return run_readout<128>(p, q, og, conv_w, norm_w, state, o, st);
+    case 64: return run_readout<64>(p, q, og, conv_w, norm_w, state, o, st, after_state);
+    case 128: return run_readout<128>(p, q, og, conv_w, norm_w, state, o, st, after_state);
   }
   return cudaErrorInvalidValue;
 }
