@@ -250,10 +250,12 @@ __device__ __forceinline__ void slide(float (&xm)[3][NC], const float (&x)[NC]) 
 }
 
 // phi(x) = elu(x) + 1 for two channels given xl = x * log2(e):
-// exp(min(x, 0)) + max(x, 0) = 2^min(xl, 0) + ln2 * max(xl, 0).
+// exp(min(x, 0)) + max(x, 0) = 2^mn + ln2 (xl - mn),  mn = min(xl, 0).
 __device__ __forceinline__ float2 phi2_log2(float2 xl) {
-  const float2 e = make_float2(ex2_approx(fminf(xl.x, 0.f)), ex2_approx(fminf(xl.y, 0.f)));
-  return __ffma2_rn(make_float2(kLn2, kLn2), make_float2(fmaxf(xl.x, 0.f), fmaxf(xl.y, 0.f)), e);
+  const float2 mn = make_float2(fminf(xl.x, 0.f), fminf(xl.y, 0.f));
+  const float2 e = make_float2(ex2_approx(mn.x), ex2_approx(mn.y));
+  const float2 d = __ffma2_rn(mn, make_float2(-1.f, -1.f), xl);
+  return __ffma2_rn(make_float2(kLn2, kLn2), d, e);
 }
 
 // Causal Conv1D of channels i, i+1 at token u of a thread's 4 tokens: taps
@@ -792,8 +794,8 @@ struct ReadoutParams {
 // window before the first row; rows are read by `row_raw(u)` (u = 0..3).
 template <typename RowFn>
 __device__ __forceinline__ void readout_rows4(const float (&wq)[4][8], float (&xm)[3][8],
-                                              RowFn row_raw, uint32_t abase, int row0, int kb,
-                                              int cc) {
+                                              RowFn row_raw, uint32_t abase,
+                                              const uint32_t *aoff) {
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     float x[8];
@@ -805,11 +807,41 @@ __device__ __forceinline__ void readout_rows4(const float (&wq)[4][8], float (&x
       pq[i] = f2_to_bf2(ph.x, ph.y);
     }
     slide(xm, x);
-    const int row = row0 + u;
-    const uint32_t off = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 +
-                         ((cc ^ (row & 7)) << 4);
-    sts_v4(abase + off, make_uint4(pq[0], pq[1], pq[2], pq[3]));
+    sts_v4(abase + aoff[u], make_uint4(pq[0], pq[1], pq[2], pq[3]));
   }
+}
+
+// Position in the flattened (batch, head, 128-token tile) order of the readout.
+struct TileCursor {
+  int b, h, r0, nrow, L;
+};
+__device__ __forceinline__ TileCursor tile_at(const int *pre, const int32_t *seq_lens, int B,
+                                              int N, int i) {
+  TileCursor t;
+  t.b = find_batch(pre, B, i);
+  t.L = clamp_len(seq_lens, t.b, N);
+  const int nt = (t.L + kRTok - 1) / kRTok;
+  const int r = i - pre[t.b];
+  t.h = r / nt;
+  t.r0 = (r % nt) * kRTok;
+  t.nrow = min(kRTok, t.L - t.r0);
+  return t;
+}
+// The next tile; only called while one remains.
+__device__ __forceinline__ void tile_next(TileCursor &t, const int32_t *seq_lens, int B, int H,
+                                          int N) {
+  t.r0 += kRTok;
+  if (t.r0 >= t.L) {
+    t.r0 = 0;
+    if (++t.h == H) {
+      t.h = 0;
+      do {
+        ++t.b;
+        t.L = t.b < B ? clamp_len(seq_lens, t.b, N) : 0;
+      } while (t.b < B && t.L == 0);
+    }
+  }
+  t.nrow = min(kRTok, t.L - t.r0);
 }
 
 template <int D>
@@ -884,16 +916,15 @@ __global__ void __launch_bounds__(kRThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  // Tile -> (b, h, first token, valid rows)
+  // Tile -> (b, h, first token, valid rows): decoded once, then stepped; each
+  // role calls tile_of for ii = i0, i0 + 1, ... in order.
+  TileCursor tc0 = tile_at(pre, p.seq_lens, B, N, (int)i0);
   auto tile_of = [&](long long ii, int &b, int &h, int &r0, int &nrow) {
-    const int i = (int)ii;
-    b = find_batch(pre, B, i);
-    const int L = clamp_len(p.seq_lens, b, N);
-    const int nt = (L + kRTok - 1) / kRTok;
-    const int r = i - pre[b];
-    h = r / nt;
-    r0 = (r % nt) * kRTok;
-    nrow = min(kRTok, L - r0);
+    if (ii != i0) tile_next(tc0, p.seq_lens, B, H, N);
+    b = tc0.b;
+    h = tc0.h;
+    r0 = tc0.r0;
+    nrow = tc0.nrow;
   };
 
   if (warp < kRProdWarps) {
@@ -901,6 +932,23 @@ __global__ void __launch_bounds__(kRThreads, 1)
     constexpr int TPR = C::TPR, TPS = C::TPS;
     const int c = tid % TPR, stream = tid / TPR;
     const int kb = c >> 3, cc = c & 7;
+    const int row0 = stream * TPS;  // first tile row of this sub-stream
+    // swizzled offsets of this thread's 16-byte pieces: A rows row0 + u and
+    // (TMA q tile) q rows row0 + j, j = 0..TPS+2 (row j holds token r0 - 3 + j)
+    uint32_t aoff[TPS];
+#pragma unroll
+    for (int u = 0; u < TPS; ++u) {
+      const int row = row0 + u;
+      aoff[u] = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
+    }
+    uint32_t qoff[C::QT ? TPS + 3 : 1];
+    if constexpr (C::QT) {
+#pragma unroll
+      for (int jj = 0; jj < TPS + 3; ++jj) {
+        const int row = row0 + jj;
+        qoff[jj] = (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
+      }
+    }
     int cur_b = -1, cur_h = -1, nbh = 0;
     float wq[4][8];
     for (long long ii = i0; ii < i1; ++ii) {
@@ -973,21 +1021,17 @@ __global__ void __launch_bounds__(kRThreads, 1)
         report_error(32, ab);
       const uint32_t abase = smem_u32(smem + C::kOffA + sa * C::kABytes);
       float xm[3][8];
-      const int row0 = stream * TPS;  // first tile row of this sub-stream
       if constexpr (C::QT) {
         // q tile from TMA: smem row j holds token r0 - 3 + j (128-byte swizzle)
         const int sq = li % QS;
         if (!mbar_wait(&q_full[sq], (li / QS) & 1, &ab) && !ab.raised()) report_error(32, ab);
         const uint32_t qb = smem_u32(smem + C::kOffQ + sq * C::kQBytes);
-        auto qrow = [&](int j) {
-          return lds_v4(qb + (j >> 3) * 1024 + (j & 7) * 128 + ((cc ^ (j & 7)) << 4));
-        };
 #pragma unroll
-        for (int u = 0; u < 3; ++u) unpack8(qrow(row0 + u), xm[u]);
+        for (int u = 0; u < 3; ++u) unpack8(lds_v4(qb + qoff[u]), xm[u]);
 #pragma unroll
         for (int g4 = 0; g4 < TPS; g4 += 4)
-          readout_rows4(wq, xm, [&](int u) { return qrow(row0 + g4 + u + 3); }, abase, row0 + g4,
-                        0, cc);
+          readout_rows4(wq, xm, [&](int u) { return lds_v4(qb + qoff[g4 + u + 3]); }, abase,
+                        aoff + g4);
         __syncwarp();
         if (lane == 0) mbar_arrive(&q_empty[sq]);
       } else {
@@ -1007,7 +1051,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         for (int g4 = 0; g4 < TPS; g4 += 4) {
 #pragma unroll
           for (int u = 0; u < 4; ++u) raw[u] = ld(ts + g4 + u);
-          readout_rows4(wq, xm, [&](int u) { return raw[u]; }, abase, row0 + g4, kb, cc);
+          readout_rows4(wq, xm, [&](int u) { return raw[u]; }, abase, aoff + g4);
         }
       }
       fence_proxy_async_smem();
@@ -1021,6 +1065,14 @@ __global__ void __launch_bounds__(kRThreads, 1)
     const int row = 32 * q4 + lane;
     const uint32_t ss_s = smem_u32(smem + C::kOffSs);
     constexpr int NH = CPE / 32;                 // 32-column pieces per warp
+    // swizzled offsets of this row's 8-channel pieces in an out_gate/o tile
+    uint32_t ogoff[CPE / 8];
+#pragma unroll
+    for (int g8 = 0; g8 < CPE / 8; ++g8) {
+      const int ch0 = part * CPE + 8 * g8;
+      const int kbo = ch0 >> 6, cco = (ch0 & 63) >> 3;
+      ogoff[g8] = kbo * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cco ^ (row & 7)) << 4);
+    }
     int pend = -1;  // og stage whose TMA store may still be reading it (leader only)
     for (long long ii = i0; ii < i1; ++ii) {
       int b, h, r0, nrow;
@@ -1060,10 +1112,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
       const float *nwh = p.norm_w + (size_t)h * D + part * CPE;
       const uint32_t ogt = smem_u32(smem + C::kOffOg + so * C::kOgBytes);
       auto og_addr = [&](int col) {  // col: channel offset within this warp's half
-        const int ch0 = part * CPE + col;
-        const int kbo = ch0 >> 6, cco = (ch0 & 63) >> 3;
-        return ogt + kbo * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 +
-               ((cco ^ (row & 7)) << 4);
+        return ogt + ogoff[col / 8];
       };
 #pragma unroll
       for (int h2 = 0; h2 < NH; ++h2) {
@@ -1196,9 +1245,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
         // last tile of this (b, h) in this CTA: release B for the next rebuild
         bool last = ii + 1 >= i1;
         if (!last) {
-          int b2, h2, r02, nrow2;
-          tile_of(ii + 1, b2, h2, r02, nrow2);
-          last = (b2 != b || h2 != h);
+          TileCursor nx = tc0;
+          tile_next(nx, p.seq_lens, B, H, N);
+          last = (nx.b != b || nx.h != h);
         }
         if (last) mma_commit(b_free);
       }
@@ -1224,11 +1273,12 @@ __global__ void __launch_bounds__(kRThreads, 1)
           tma_load_4d(dst + kbo * (kRTok * 128), &tm_og, &og_full[so], kbo * 64, h, r0, b);
         if constexpr (!C::QT) {  // q is read with plain loads: warm L2 two tiles ahead
           if (ii + 2 < i1) {
-            int b2, h2, r02, nrow2;
-            tile_of(ii + 2, b2, h2, r02, nrow2);
+            TileCursor nx = tc0;
+            tile_next(nx, p.seq_lens, B, H, N);
+            tile_next(nx, p.seq_lens, B, H, N);
 #pragma unroll
             for (int kbo = 0; kbo < C::KB; ++kbo)
-              tma_prefetch_l2_4d(&tm_q, kbo * 64, h2, r02, b2);
+              tma_prefetch_l2_4d(&tm_q, kbo * 64, nx.h, nx.r0, nx.b);
           }
         }
       }

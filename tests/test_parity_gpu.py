@@ -214,3 +214,15 @@ def test_tensor_core_state_matches_oracle():
             z = st[b, h, 64 * 64:]
             assert np.abs(S - inter["S"]).max() <= 1e-2 * np.abs(inter["S"]).max()
             assert np.abs(z - inter["z"]).max() <= 1e-2 * np.abs(inter["z"]).max()
+
+
+def test_many_tiles_per_cta_with_empty_sequences():
+    """Enough 128-token tiles that every persistent CTA walks several of them
+    across head and batch boundaries, with empty sequences in between."""
+    lens = [4096, 0, 1000, 0, 0, 2500, 129]
+    w = custom(B=len(lens), H=8, N=4096, D=64, dtype="bf16", seed=23, seq_lens=lens)
+    inp = make_inputs(w, "cuda")
+    gbla.device_error(reset=True)
+    y = _run(inp, gbla.ALGO_TC)
+    assert gbla.device_error() == 0
+    _check_against(y, oracle_full(inp), inp, "bf16")
