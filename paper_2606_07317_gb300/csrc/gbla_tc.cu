@@ -132,7 +132,8 @@ struct ReadoutCfg {
   static constexpr bool QT = D == 64;                     // q through TMA (else 128-bit loads)
   static constexpr int NR = D + 16;                       // MMA N: D columns of S, z, zeros
   static constexpr int KB = D / 64;                       // 64-element K blocks
-  static constexpr int TPR = D / 8;                       // producer threads per token row
+  static constexpr int NCH = QT ? 4 : 8;                  // channels per producer thread
+  static constexpr int TPR = D / NCH;                     // producer threads per token row
   static constexpr int STREAMS = kRProd / TPR;            // producer sub-streams per tile
   static constexpr int TPS = kRTok / STREAMS;             // tokens per sub-stream
   static constexpr int kABytes = kRTok * D * 2;           // one A tile
@@ -161,6 +162,7 @@ struct ReadoutCfg {
   static constexpr uint32_t kIdesc = idesc_bf16_f32(kRTok, NR, 0, 0);
   static_assert(kSmem <= 227 * 1024, "readout shared memory");
   static_assert(TPS % 4 == 0, "producer sub-streams are processed 4 tokens at a time");
+  static_assert(!QT || TPS == 8, "TMA q path: one 8-row swizzle atom per sub-stream");
 };
 
 __device__ __forceinline__ void report_error(unsigned code, const AbortFlag &ab) {
@@ -262,6 +264,19 @@ __device__ __forceinline__ float2 phi2_log2(float2 xl) {
 // 0..3 on raw rows u..u+3 (row u + 3 is the token itself).
 __device__ __forceinline__ float2 conv_rows(const float (&w)[4][4], const float (&x)[7][4],
                                             int u, int i) {
+  float2 a = __fmul2_rn(make_float2(w[0][i], w[0][i + 1]), make_float2(x[u][i], x[u][i + 1]));
+#pragma unroll
+  for (int tau = 1; tau < 4; ++tau)
+    a = __ffma2_rn(make_float2(w[tau][i], w[tau][i + 1]),
+                   make_float2(x[u + tau][i], x[u + tau][i + 1]), a);
+  return a;
+}
+
+// Causal Conv1D of channels i, i+1 at row u + 3 of a row array: taps 0..3 on
+// rows u..u+3.
+template <int R>
+__device__ __forceinline__ float2 conv_rows_n(const float (&w)[4][4], const float (&x)[R][4],
+                                              int u, int i) {
   float2 a = __fmul2_rn(make_float2(w[0][i], w[0][i + 1]), make_float2(x[u][i], x[u][i + 1]));
 #pragma unroll
   for (int tau = 1; tau < 4; ++tau)
@@ -929,28 +944,25 @@ __global__ void __launch_bounds__(kRThreads, 1)
 
   if (warp < kRProdWarps) {
     // ------------------------------------------------------------ producers: phi(conv(q))
-    constexpr int TPR = C::TPR, TPS = C::TPS;
+    constexpr int TPR = C::TPR, TPS = C::TPS, NCH = C::NCH;
     const int c = tid % TPR, stream = tid / TPR;
-    const int kb = c >> 3, cc = c & 7;
+    const int kb = (NCH * c) >> 6, cc = ((NCH * c) & 63) >> 3;  // 64-channel block, 16-byte chunk
     const int row0 = stream * TPS;  // first tile row of this sub-stream
-    // swizzled offsets of this thread's 16-byte pieces: A rows row0 + u and
-    // (TMA q tile) q rows row0 + j, j = 0..TPS+2 (row j holds token r0 - 3 + j)
-    uint32_t aoff[TPS];
+    // swizzled offsets of this thread's 16-byte pieces of A rows row0 + u
+    // (the TMA q path uses one 8-row atom per sub-stream and needs none)
+    uint32_t aoff[C::QT ? 1 : TPS];
+    if constexpr (!C::QT) {
 #pragma unroll
-    for (int u = 0; u < TPS; ++u) {
-      const int row = row0 + u;
-      aoff[u] = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
-    }
-    uint32_t qoff[C::QT ? TPS + 3 : 1];
-    if constexpr (C::QT) {
-#pragma unroll
-      for (int jj = 0; jj < TPS + 3; ++jj) {
-        const int row = row0 + jj;
-        qoff[jj] = (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
+      for (int u = 0; u < TPS; ++u) {
+        const int row = row0 + u;
+        aoff[u] = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
       }
     }
+    // TMA q path: q tile row j holds token r0 - 3 + j; this thread reads rows
+    // row0 + k (k = 0..10, 4 channels = 8 bytes) and writes A rows row0 + u
+    const uint32_t thr8 = (uint32_t)(stream * 1024 + (c & 1) * 8);
     int cur_b = -1, cur_h = -1, nbh = 0;
-    float wq[4][8];
+    float wq[4][NCH];
     for (long long ii = i0; ii < i1; ++ii) {
       int b, h, r0, nrow;
       tile_of(ii, b, h, r0, nrow);
@@ -961,11 +973,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
         if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, &ab) && !ab.raised())
           report_error(16, ab);
         // q taps first (in flight during the rebuild), pre-scaled by log2(e)
-        // later (phi2_log2 takes x log2(e)): 32 consecutive floats per thread
-        float4 wq4[8];
+        // later (phi2_log2 takes x log2(e)): 4 NCH consecutive floats per thread
+        float4 wq4[NCH];
 #pragma unroll
-        for (int i = 0; i < 8; ++i)
-          wq4[i] = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + 8 * c + i) * 4));
+        for (int i = 0; i < NCH; ++i)
+          wq4[i] = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + NCH * c + i) * 4));
         if (nbh == 0) grid_dep_wait();  // the state comes from the preceding kernel
         const float *st = p.state + ((size_t)b * H + h) * F;
         constexpr int NI = NR * (D / 8);  // (row e of B, 8-element K chunk ck) items
@@ -1006,7 +1018,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(b_full);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < NCH; ++i) {
           wq[0][i] = wq4[i].x * kLog2e;
           wq[1][i] = wq4[i].y * kLog2e;
           wq[2][i] = wq4[i].z * kLog2e;
@@ -1020,21 +1032,27 @@ __global__ void __launch_bounds__(kRThreads, 1)
       if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab) && !ab.raised())
         report_error(32, ab);
       const uint32_t abase = smem_u32(smem + C::kOffA + sa * C::kABytes);
-      float xm[3][8];
       if constexpr (C::QT) {
-        // q tile from TMA: smem row j holds token r0 - 3 + j (128-byte swizzle)
+        // q tile from TMA (128-byte swizzle); rows row0 .. row0 + 10 hold this
+        // sub-stream's 3 history tokens and its 8 tokens
         const int sq = li % QS;
         if (!mbar_wait(&q_full[sq], (li / QS) & 1, &ab) && !ab.raised()) report_error(32, ab);
-        const uint32_t qb = smem_u32(smem + C::kOffQ + sq * C::kQBytes);
+        const uint32_t qb = smem_u32(smem + C::kOffQ + sq * C::kQBytes) + thr8;
+        float x[TPS + 3][4];
 #pragma unroll
-        for (int u = 0; u < 3; ++u) unpack8(lds_v4(qb + qoff[u]), xm[u]);
-#pragma unroll
-        for (int g4 = 0; g4 < TPS; g4 += 4)
-          readout_rows4(wq, xm, [&](int u) { return lds_v4(qb + qoff[g4 + u + 3]); }, abase,
-                        aoff + g4);
+        for (int k = 0; k < TPS + 3; ++k)
+          unpack4(lds_v2(qb + (k >> 3) * 1024 + (k & 7) * 128 + ((cc ^ (k & 7)) << 4)), x[k]);
         __syncwarp();
         if (lane == 0) mbar_arrive(&q_empty[sq]);
+        const uint32_t at = abase + thr8;
+#pragma unroll
+        for (int u = 0; u < TPS; ++u) {
+          const float2 p01 = phi2_log2(conv_rows_n(wq, x, u, 0));
+          const float2 p23 = phi2_log2(conv_rows_n(wq, x, u, 2));
+          sts_v2(at + u * 128 + ((cc ^ u) << 4), f2_to_bf2(p01.x, p01.y), f2_to_bf2(p23.x, p23.y));
+        }
       } else {
+        float xm[3][8];
         const size_t rs = (size_t)H * D;
         const __nv_bfloat16 *qp = p.q + ((size_t)b * N * H + h) * D + 8 * c;
         const int ts = r0 + row0;        // first token of this sub-stream
