@@ -401,7 +401,8 @@ __device__ __forceinline__ void prefetch_chunk_inputs(const StateParams &p, cons
 template <int D>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v) {
+                    const __grid_constant__ CUtensorMap tm_v,
+                    const __grid_constant__ CUtensorMap tm_rec) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   extern __shared__ uint8_t smem_raw[];
@@ -652,10 +653,34 @@ __global__ void __launch_bounds__(kSThreads, 1)
             const float4 wt = wv[cv0 + cb + i];
             o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
           }
-          if (ok2) {
+          if constexpr (D == 64) {
+            // staged in the idle A ring as 32-column, 128B-swizzled tiles for
+            // one TMA store per tile: row d, 16-byte chunk (col % 32) / 4 ^ (d & 7)
+            const int col = part * CPW + cb, cbk = col >> 5, c4 = (col & 31) >> 2;
+            const uint32_t trow = smem_u32(smem + kSOffA) +
+                                  (uint32_t)((hh2 * 2 + cbk) * (64 * 128) + d * 128);
+            sts_v4(trow + ((c4 ^ (d & 7)) << 4),
+                   make_uint4(__float_as_uint(o[0]), __float_as_uint(o[1]),
+                              __float_as_uint(o[2]), __float_as_uint(o[3])));
+            sts_v4(trow + (((c4 + 1) ^ (d & 7)) << 4),
+                   make_uint4(__float_as_uint(o[4]), __float_as_uint(o[5]),
+                              __float_as_uint(o[6]), __float_as_uint(o[7])));
+          } else if (ok2) {
             float4 *dst = (float4 *)(srow + cb);
             dst[0] = make_float4(o[0], o[1], o[2], o[3]);
             dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+          }
+        }
+        if constexpr (D == 64) {
+          fence_proxy_async_smem();
+          named_barrier(1, kSProd);
+          if (tid == 0) {
+            for (int hz = 0; hz < G && c.hbase + hz < H; ++hz)
+              for (int cbk = 0; cbk < 2; ++cbk)
+                tma_store_4d(&tm_rec, smem + kSOffA + (hz * 2 + cbk) * (64 * 128), cbk * 32, 0,
+                             hz, k);
+            tma_store_commit();
+            tma_store_wait_read<0>();  // the A ring is written again by the next chunk
           }
         }
         if (tid < kGroupCh) {
@@ -981,10 +1006,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
         if (nbh == 0) grid_dep_wait();  // the state comes from the preceding kernel
         const float *st = p.state + ((size_t)b * H + h) * F;
         constexpr int NI = NR * (D / 8);  // (row e of B, 8-element K chunk ck) items
-        for (int item0 = tid; item0 < NI; item0 += 2 * kRProd) {
-          float vals[2][8];  // both items' loads in flight together
+        constexpr int BU = (NI + kRProd - 1) / kRProd < 3 ? (NI + kRProd - 1) / kRProd : 3;
+        for (int item0 = tid; item0 < NI; item0 += BU * kRProd) {
+          float vals[BU][8];  // all items' loads in flight together
 #pragma unroll
-          for (int u = 0; u < 2; ++u) {
+          for (int u = 0; u < BU; ++u) {
             const int item = item0 + u * kRProd;
             const int e = item % NR, ck = item / NR;
 #pragma unroll
@@ -995,7 +1021,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
             }
           }
 #pragma unroll
-          for (int u = 0; u < 2; ++u) {
+          for (int u = 0; u < BU; ++u) {
             const int item = item0 + u * kRProd;
             if (item >= NI) break;
             const int e = item % NR, ck = item / NR;
@@ -1384,6 +1410,25 @@ cudaError_t make_group_map(CUtensorMap *m, const void *base, int B, int N, int H
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 4-D map over the partial-state records [chunks][G][D*D + D + 4] fp32, viewed
+// as S blocks {D columns, D rows, G heads, chunks}; box = 32 columns x D rows,
+// 128-byte swizzle (the state kernel stages S that way before storing it).
+cudaError_t make_records_map(CUtensorMap *m, void *records, const Problem &p, int D, int S) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const int G = kGroupCh / D;
+  const size_t chunks = (size_t)p.B * ((p.H + G - 1) / G) * ((p.N + S - 1) / S);
+  const size_t rec = (size_t)D * D + D + 4;
+  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)D, (cuuint64_t)G, (cuuint64_t)chunks};
+  const cuuint64_t strides[3] = {(cuuint64_t)D * 4, (cuuint64_t)rec * 4, (cuuint64_t)G * rec * 4};
+  const cuuint32_t box[4] = {32, (cuuint32_t)D, 1, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, records, dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 struct DeviceInfo {
   int sms = 0;
   bool sm103 = false;
@@ -1447,15 +1492,16 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   sp.N = p.N;
   sp.S = S;
   sp.HG = (p.H + G - 1) / G;
-  CUtensorMap tm_k, tm_v;
+  CUtensorMap tm_k, tm_v, tm_rec;
   cudaError_t e = make_group_map(&tm_k, k, p.B, p.N, p.H, D);
   if (e != cudaSuccess) return e;
   if ((e = make_bnhd_map(&tm_v, v, p.B, p.N, p.H, D, kSRawRows)) != cudaSuccess) return e;
+  if ((e = make_records_map(&tm_rec, ws, p, D, S)) != cudaSuccess) return e;
   auto k1 = tc_state_kernel<D>;
   if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
       cudaSuccess)
     return e;
-  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v);
+  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v, tm_rec);
   count_launch();
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
