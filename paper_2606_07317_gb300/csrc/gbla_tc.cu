@@ -398,6 +398,21 @@ __device__ __forceinline__ void prefetch_chunk_inputs(const StateParams &p, cons
   }
 }
 
+// decode_chunk when every sequence has N tokens (the prefix is b * HG * nck).
+template <int G>
+__device__ __forceinline__ ChunkRef decode_chunk_uniform(const StateParams &p, int k) {
+  ChunkRef c;
+  const int nck = (p.N + p.S - 1) / p.S;
+  c.b = k / (p.HG * nck);
+  c.L = p.N;
+  const int r = k - c.b * p.HG * nck;
+  c.hbase = (r / nck) * G;
+  c.t0 = (r % nck) * p.S;
+  c.n = min(c.t0 + p.S, c.L) - c.t0;
+  c.nst = (c.n + kSTok - 1) / kSTok;
+  return c;
+}
+
 template <int D>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
@@ -422,12 +437,52 @@ __global__ void __launch_bounds__(kSThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, H = p.H;
 
-  if (tid == 0) {
-    *(volatile int *)(smem + kSOffMisc + 4) = 0;
+  // Converter thread -> (group, channel quad q, token quad j): the groups take
+  // alternate stages; within a group the mapping makes both the raw-tile
+  // reads (16 lanes, 16 distinct quads of one 256-byte row) and the swizzled
+  // K^ writes (16 lanes, 16 distinct 8-byte slots of the 128-byte bank
+  // window) free of bank conflicts.
+  const int grp = warp / kSGroupWarps, gtid = tid % kSGroupThreads;
+  const int hw = 2 * (warp % kSGroupWarps) + (lane >> 4);              // half-warp 0..15
+  const int q = (lane & 15) + 16 * (hw & 1);                           // channel quad 0..31
+  const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
+  const int c0ch = 4 * q;
+  const int hh = c0ch / D, d0 = c0ch - D * hh;                         // head in group, channel
+
+  // With no seq_lens every sequence has N tokens, chunk k maps to (batch,
+  // head group, chunk) by arithmetic alone, and the first loads go out before
+  // the prefix over the batch is built.
+  const bool uniform = p.seq_lens == nullptr;
+  const int Ku = B * p.HG * ((p.N + p.S - 1) / p.S);
+  const long long c0u = (long long)Ku * blockIdx.x / gridDim.x;
+  const long long c1u = (long long)Ku * (blockIdx.x + 1) / gridDim.x;
+  const int early = uniform && c0u < c1u;  // first stages issued before the prefix
+  if (warp == kSTmaWarp && lane == 0) {
+    // the raw ring's barriers are first used by this thread
     for (int i = 0; i < kSRawStages; ++i) {
       mbar_init(&raw_full[i], 1);
       mbar_init(&raw_empty[i], kSGroupWarps + 1);  // one converter group reads k, the MMAs v
     }
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+    const uint64_t pol = l2_policy_evict_first();
+    if (early) {
+      const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
+      const int nvb = D == 64 ? min(2, H - c.hbase) : 2;
+      for (int it = 0; it < min(c.nst, kSRawStages); ++it) {
+        uint8_t *dst = smem + kSOffRaw + it * kSRawStage;
+        const int tok = c.t0 + it * kSTok - kSHalo;
+        mbar_arrive_expect_tx(&raw_full[it], kSRawKBytes + nvb * kSVBoxBytes);
+        tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[it], 0, c.hbase, tok, c.b, pol);
+        for (int blk = 0; blk < nvb; ++blk)
+          tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[it], (blk * 64) % D,
+                           c.hbase + (blk * 64) / D, tok, c.b, pol);
+      }
+    }
+  }
+  if (tid == 0) {
+    *(volatile int *)(smem + kSOffMisc + 4) = 0;
     for (int i = 0; i < kSAStages; ++i) {
       mbar_init(&a_full[i], kSGroupWarps);
       mbar_init(&a_empty[i], 1);
@@ -436,6 +491,8 @@ __global__ void __launch_bounds__(kSThreads, 1)
     mbar_init(fin, 1);
     fence_mbar_init();
   }
+  if (early && warp < kSCvtWarps)
+    prefetch_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0);
   // Chunk prefix over the batch (converter threads), shared by all roles.
   if (warp < kSCvtWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
@@ -460,13 +517,14 @@ __global__ void __launch_bounds__(kSThreads, 1)
     // zero-filled before the sequence start.  This warp takes no part in the
     // TMEM hand-off, so its first loads go out at once.
     if (lane == 0) {
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      uint32_t issued = 0;
+      // stages of the first chunk already issued before the prefix
+      const int it0 = early ? min(cfirst.nst, kSRawStages) : 0;
+      const uint64_t pol = l2_policy_evict_first();
+      uint32_t issued = (uint32_t)it0;
       for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
         const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, (int)kk);
         const int nvb = D == 64 ? min(2, H - c.hbase) : 2;  // v blocks of existing heads
-        for (int it = 0; it < c.nst; ++it) {
+        for (int it = kk == c0 ? it0 : 0; it < c.nst; ++it) {
           const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
           if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
             if (!ab.raised()) report_error(2048, ab);
@@ -475,10 +533,10 @@ __global__ void __launch_bounds__(kSThreads, 1)
           uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
           const int tok = c.t0 + it * kSTok - kSHalo;
           mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes + nvb * kSVBoxBytes);
-          tma_load_4d(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b);
+          tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b, pol);
           for (int blk = 0; blk < nvb; ++blk)
-            tma_load_4d(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
-                        c.hbase + (blk * 64) / D, tok, c.b);
+            tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
+                             c.hbase + (blk * 64) / D, tok, c.b, pol);
           ++issued;
         }
       }
@@ -491,20 +549,9 @@ __global__ void __launch_bounds__(kSThreads, 1)
     return;
   }
 
-  // Converter thread -> (group, channel quad q, token quad j): the groups take
-  // alternate stages; within a group the mapping makes both the raw-tile
-  // reads (16 lanes, 16 distinct quads of one 256-byte row) and the swizzled
-  // K^ writes (16 lanes, 16 distinct 8-byte slots of the 128-byte bank
-  // window) free of bank conflicts.
-  const int grp = warp / kSGroupWarps, gtid = tid % kSGroupThreads;
-  const int hw = 2 * (warp % kSGroupWarps) + (lane >> 4);              // half-warp 0..15
-  const int q = (lane & 15) + 16 * (hw & 1);                           // channel quad 0..31
-  const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
-  const int c0ch = 4 * q;
-  const int hh = c0ch / D, d0 = c0ch - D * hh;                         // head in group, channel
   // The first chunk's global reads are pulled into L2 during the TMEM hand-off
   // (holding them in registers across it would spill).
-  if (warp < kSCvtWarps) prefetch_chunk_inputs<D, G>(p, cfirst, tid, hh, d0);
+  if (!early && warp < kSCvtWarps) prefetch_chunk_inputs<D, G>(p, cfirst, tid, hh, d0);
   ChunkIn<G> cin;
 
   if (warp == kSMmaWarp) tmem_alloc(tmem_slot, kSTmemCols);
@@ -636,39 +683,56 @@ __global__ void __launch_bounds__(kSThreads, 1)
         float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + part * CPW;
         const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16) +
                             (uint32_t)(256 * (cv0 / 64) + cv0 % 64);
+        if constexpr (D == 64) {
+          // staged in the idle A ring as 32-column, 128B-swizzled tiles for
+          // one TMA store per tile: row d, 16-byte chunk (col % 32) / 4 ^ (d & 7);
+          // 4 columns (one chunk) per step
+          const uint32_t stg = smem_u32(smem + kSOffA) + (uint32_t)(hh2 * 2 * (64 * 128) + d * 128);
 #pragma unroll 1
-        for (int cb = 0; cb < CPW; cb += 8) {
-          float v0[8], v1[8], v2[8], v3[8];
-          tmem_ld8(tl + cb, v0);
-          tmem_ld8(tl + 64 + cb, v1);
-          tmem_ld8(tl + 128 + cb, v2);
-          tmem_ld8(tl + 192 + cb, v3);
-          tmem_ld_wait_regs(v0);
-          tmem_pin(v1);
-          tmem_pin(v2);
-          tmem_pin(v3);
-          float o[8];
+          for (int cb = 0; cb < CPW; cb += 4) {
+            float v0[4], v1[4], v2[4], v3[4];
+            tmem_ld4(tl + cb, v0);
+            tmem_ld4(tl + 64 + cb, v1);
+            tmem_ld4(tl + 128 + cb, v2);
+            tmem_ld4(tl + 192 + cb, v3);
+            tmem_ld_wait_regs(v0);
+            tmem_pin(v1);
+            tmem_pin(v2);
+            tmem_pin(v3);
+            uint32_t o[4];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const float4 wt = wv[cv0 + cb + i];
-            o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
-          }
-          if constexpr (D == 64) {
-            // staged in the idle A ring as 32-column, 128B-swizzled tiles for
-            // one TMA store per tile: row d, 16-byte chunk (col % 32) / 4 ^ (d & 7)
+            for (int i = 0; i < 4; ++i) {
+              const float4 wt = wv[cv0 + cb + i];
+              o[i] = __float_as_uint(
+                  fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i]))));
+            }
             const int col = part * CPW + cb, cbk = col >> 5, c4 = (col & 31) >> 2;
-            const uint32_t trow = smem_u32(smem + kSOffA) +
-                                  (uint32_t)((hh2 * 2 + cbk) * (64 * 128) + d * 128);
-            sts_v4(trow + ((c4 ^ (d & 7)) << 4),
-                   make_uint4(__float_as_uint(o[0]), __float_as_uint(o[1]),
-                              __float_as_uint(o[2]), __float_as_uint(o[3])));
-            sts_v4(trow + (((c4 + 1) ^ (d & 7)) << 4),
-                   make_uint4(__float_as_uint(o[4]), __float_as_uint(o[5]),
-                              __float_as_uint(o[6]), __float_as_uint(o[7])));
-          } else if (ok2) {
-            float4 *dst = (float4 *)(srow + cb);
-            dst[0] = make_float4(o[0], o[1], o[2], o[3]);
-            dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+            sts_v4(stg + cbk * (64 * 128) + ((c4 ^ (d & 7)) << 4),
+                   make_uint4(o[0], o[1], o[2], o[3]));
+          }
+        } else {
+#pragma unroll 1
+          for (int cb = 0; cb < CPW; cb += 8) {
+            float v0[8], v1[8], v2[8], v3[8];
+            tmem_ld8(tl + cb, v0);
+            tmem_ld8(tl + 64 + cb, v1);
+            tmem_ld8(tl + 128 + cb, v2);
+            tmem_ld8(tl + 192 + cb, v3);
+            tmem_ld_wait_regs(v0);
+            tmem_pin(v1);
+            tmem_pin(v2);
+            tmem_pin(v3);
+            float o[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float4 wt = wv[cv0 + cb + i];
+              o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
+            }
+            if (ok2) {
+              float4 *dst = (float4 *)(srow + cb);
+              dst[0] = make_float4(o[0], o[1], o[2], o[3]);
+              dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+            }
           }
         }
         if constexpr (D == 64) {
@@ -1301,6 +1365,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
   } else if (warp == kRTmaWarp) {
     // ------------------------------------------------------------ TMA: out_gate
     if (lane == 0) {
+      const uint64_t pol = l2_policy_evict_first();  // read once
       for (long long ii = i0; ii < i1; ++ii) {
         int b, h, r0, nrow;
         tile_of(ii, b, h, r0, nrow);
@@ -1314,7 +1379,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
         mbar_arrive_expect_tx(&og_full[so], C::kOgBytes);
 #pragma unroll
         for (int kbo = 0; kbo < C::KB; ++kbo)
-          tma_load_4d(dst + kbo * (kRTok * 128), &tm_og, &og_full[so], kbo * 64, h, r0, b);
+          tma_load_4d_hint(dst + kbo * (kRTok * 128), &tm_og, &og_full[so], kbo * 64, h, r0, b,
+                           pol);
         if constexpr (!C::QT) {  // q is read with plain loads: warm L2 two tiles ahead
           if (ii + 2 < i1) {
             TileCursor nx = tc0;
@@ -1330,6 +1396,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
   } else {
     // ------------------------------------------------------------ TMA: q
     if (lane == 0 && C::QT) {
+      const uint64_t pol = l2_policy_evict_first();  // read once (3 halo rows aside)
       for (long long ii = i0; ii < i1; ++ii) {
         int b, h, r0, nrow;
         tile_of(ii, b, h, r0, nrow);
@@ -1340,7 +1407,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
           break;
         }
         mbar_arrive_expect_tx(&q_full[sq], C::kQTileBytes);
-        tma_load_4d(smem + C::kOffQ + sq * C::kQBytes, &tm_q, &q_full[sq], 0, h, r0 - 3, b);
+        tma_load_4d_hint(smem + C::kOffQ + sq * C::kQBytes, &tm_q, &q_full[sq], 0, h, r0 - 3, b,
+                         pol);
       }
     }
   }
