@@ -383,21 +383,6 @@ __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const Ch
   }
 }
 
-// L2 prefetch of what load_chunk_inputs will read, holding no registers.
-template <int D, int G>
-__device__ __forceinline__ void prefetch_chunk_inputs(const StateParams &p, const ChunkRef &c,
-                                                      int tid, int hh, int d0) {
-  const int H = p.H, h = c.hbase + hh;
-  if (h < H) prefetch_l2_line(p.conv_w + ((size_t)(H + h) * D + d0) * 4);
-  if (tid < kGroupCh && c.hbase + tid / D < H)
-    prefetch_l2_line(p.conv_w + ((size_t)(2 * H + c.hbase + tid / D) * D + tid % D) * 4);
-#pragma unroll
-  for (int i = 0; i < kChunkMax / kSProd; ++i) {
-    const int tt = tid + i * kSProd;
-    if (tt < c.n) prefetch_l2_line(p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase);
-  }
-}
-
 // decode_chunk when every sequence has N tokens (the prefix is b * HG * nck).
 template <int G>
 __device__ __forceinline__ ChunkRef decode_chunk_uniform(const StateParams &p, int k) {
@@ -466,6 +451,28 @@ __global__ void __launch_bounds__(kSThreads, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_k);
     tma_prefetch_desc(&tm_v);
+  }
+  if (tid == 0) {
+    *(volatile int *)(smem + kSOffMisc + 4) = 0;
+    for (int i = 0; i < kSAStages; ++i) {
+      mbar_init(&a_full[i], kSGroupWarps);
+      mbar_init(&a_empty[i], 1);
+    }
+    mbar_init(done, 1);
+    mbar_init(fin, 1);
+    fence_mbar_init();
+  }
+  // The first chunk's global reads (gate logits, taps) go out before the bulk
+  // k/v loads, which would otherwise queue ahead of them: the gate pre-pass is
+  // on the critical path.  The TMA warp waits on barrier 3 until they are out.
+  ChunkIn<G> cin;
+  if (warp < kSCvtWarps) {
+    if (early) load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin);
+    named_barrier_arrive(3, kSProd + 32);
+  } else if (warp == kSTmaWarp) {
+    named_barrier(3, kSProd + 32);
+  }
+  if (warp == kSTmaWarp && lane == 0) {
     const uint64_t pol = l2_policy_evict_first();
     if (early) {
       const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
@@ -481,18 +488,6 @@ __global__ void __launch_bounds__(kSThreads, 1)
       }
     }
   }
-  if (tid == 0) {
-    *(volatile int *)(smem + kSOffMisc + 4) = 0;
-    for (int i = 0; i < kSAStages; ++i) {
-      mbar_init(&a_full[i], kSGroupWarps);
-      mbar_init(&a_empty[i], 1);
-    }
-    mbar_init(done, 1);
-    mbar_init(fin, 1);
-    fence_mbar_init();
-  }
-  if (early && warp < kSCvtWarps)
-    prefetch_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0);
   // Chunk prefix over the batch (converter threads), shared by all roles.
   if (warp < kSCvtWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
@@ -549,16 +544,15 @@ __global__ void __launch_bounds__(kSThreads, 1)
     return;
   }
 
-  // The first chunk's global reads are pulled into L2 during the TMEM hand-off
-  // (holding them in registers across it would spill).
-  if (!early && warp < kSCvtWarps) prefetch_chunk_inputs<D, G>(p, cfirst, tid, hh, d0);
-  ChunkIn<G> cin;
-
-  if (warp == kSMmaWarp) tmem_alloc(tmem_slot, kSTmemCols);
-  tc_fence_before();
-  named_barrier(2, kSThreads - 32);  // converters and the MMA warp
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
+  // TMEM hand-off between the MMA warp and the converters (barrier 2); the
+  // converters join it after the first chunk's gate pre-pass.
+  uint32_t tmem = 0;
+  auto tmem_handoff = [&]() {
+    tc_fence_before();
+    named_barrier(2, kSProd + 32);
+    tc_fence_after();
+    tmem = *tmem_slot;
+  };
 
   if (warp < kSCvtWarps) {
     // ------------------------------------------------------------ converters
@@ -574,7 +568,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
       const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, k);
-      load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
+      if (!(kk == c0 && early)) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
 
       // k taps of this thread's 4 channels, pre-scaled by log2(e); v taps of
       // the group's channels for the drain
@@ -631,6 +625,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
         }
       }
 
+      if (kk == c0) tmem_handoff();
       float2 z[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       for (int it = (int)((gs0 ^ grp) & 1); it < c.nst; it += 2) {  // this group's stages
         const uint32_t gs = gs0 + it;
@@ -763,6 +758,8 @@ __global__ void __launch_bounds__(kSThreads, 1)
       named_barrier(1, kSProd);  // accumulators drained before the next chunk's MMAs
     }
   } else if (warp == kSMmaWarp) {
+    tmem_alloc(tmem_slot, kSTmemCols);
+    tmem_handoff();
     if (lane == 0) {
       // ---------------------------------------------------------- MMA issuer
       // P_tau += K^T v[t - 3 + tau] for tau = 0..3 in one N = 256 MMA per
