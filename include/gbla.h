@@ -182,7 +182,10 @@ const char *gbla_status_string(gbla_status status);
 /* Library version, e.g. "0.1.0". */
 const char *gbla_version(void);
 
-/* Frees cached per-device resources (none are required between calls). */
+/* Returns the unused memory of the library's per-device scratch pools to the
+ * driver.  Scratch freed at the end of a call otherwise stays mapped for the
+ * next call (up to the largest amount one call has used).  Safe at any time;
+ * allocations still in use are kept. */
 void gbla_release(void);
 
 /* Number of kernels this library has enqueued since it was loaded, over all

@@ -4,6 +4,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <mutex>
 
 #include "gbla_internal.cuh"
 
@@ -78,7 +79,37 @@ gbla_status from_cuda(cudaError_t e) {
   return GBLA_ERR_CUDA;
 }
 
-// Stream-ordered scratch: freed on the same stream after the kernels using it.
+// Library-owned stream-ordered memory pool per device.  Its release threshold
+// is unbounded, so memory freed at the end of a call stays mapped for the
+// next one instead of being returned to the driver (and mapped again);
+// gbla_release() trims it.
+constexpr int kMaxDevices = 64;
+std::mutex g_pool_mu;
+cudaMemPool_t g_pools[kMaxDevices] = {};
+
+cudaMemPool_t device_pool() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_pool_mu);
+  if (!g_pools[dev]) {
+    cudaMemPoolProps props = {};
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    cudaMemPool_t pool = nullptr;
+    if (cudaMemPoolCreate(&pool, &props) != cudaSuccess) {
+      (void)cudaGetLastError();
+      return nullptr;
+    }
+    uint64_t thr = UINT64_MAX;
+    cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &thr);
+    g_pools[dev] = pool;
+  }
+  return g_pools[dev];
+}
+
+// Stream-ordered scratch from the library pool: freed on the same stream after
+// the kernels using it.
 struct Scratch {
   void *ptr = nullptr;
   cudaStream_t st = nullptr;
@@ -90,7 +121,9 @@ struct Scratch {
   gbla_status alloc(size_t bytes, cudaStream_t s) {
     st = s;
     if (bytes == 0) return GBLA_OK;
-    cudaError_t e = cudaMallocAsync(&ptr, bytes, s);
+    cudaMemPool_t pool = device_pool();
+    cudaError_t e = pool ? cudaMallocFromPoolAsync(&ptr, bytes, pool, s)
+                         : cudaMallocAsync(&ptr, bytes, s);
     if (e != cudaSuccess) {
       (void)cudaGetLastError();
       ptr = nullptr;
@@ -148,7 +181,11 @@ const char *gbla_status_string(gbla_status s) {
   return "unknown status";
 }
 
-void gbla_release(void) {}
+void gbla_release(void) {
+  std::lock_guard<std::mutex> lock(g_pool_mu);
+  for (int d = 0; d < kMaxDevices; ++d)
+    if (g_pools[d]) cudaMemPoolTrimTo(g_pools[d], 0);
+}
 
 uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
@@ -256,7 +293,8 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
   const size_t tens = (size_t)B * N * row;      // one [B, N, H, D] tensor
   const size_t gbytes = (size_t)B * N * grow;
   const size_t cw = sizeof(float) * 3 * H * D * kConvW, nw = sizeof(float) * H * D;
-  // Layout of the device scratch: q k v og o | gate | conv_w | norm_w | seq_lens
+  const size_t F = state_floats(D);
+  // Layout of the device scratch: q k v og o | gate | conv_w | norm_w | seq_lens | state
   size_t off[10];
   size_t at = 0;
   for (int i = 0; i < 5; ++i) { off[i] = at; at = round_up(at + tens, 256); }
@@ -264,25 +302,29 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
   off[6] = at; at = round_up(at + cw, 256);
   off[7] = at; at = round_up(at + nw, 256);
   off[8] = at; at = round_up(at + sizeof(int32_t) * B, 256);
+  off[9] = at; at = round_up(at + sizeof(float) * F * B * H, 256);
+  Problem p{B, H, N, D, dtype, nullptr};
+  bool tc = use_tc(p, GBLA_ALGO_AUTO, &s);
+  if (s != GBLA_OK) return s;
   Scratch dev;
   if ((s = dev.alloc(at, st)) != GBLA_OK) return s;
   char *base = (char *)dev.ptr;
-  // Valid rows only: rows t >= L_b are never read by the kernels.
-  const void *src[5] = {q, k, v, out_gate, nullptr};
-  for (int b = 0; b < B; ++b) {
+  auto valid_rows = [&](int b) -> size_t {
     long L = seq_lens ? seq_lens[b] : N;
-    if (L < 0) L = 0;
-    if (L > N) L = N;
-    if (L == 0) continue;
-    for (int i = 0; i < 4; ++i) {
-      if (cudaMemcpyAsync(base + off[i] + (size_t)b * N * row, (const char *)src[i] + (size_t)b * N * row,
-                          L * row, cudaMemcpyHostToDevice, st) != cudaSuccess)
-        return GBLA_ERR_CUDA;
-    }
-    if (cudaMemcpyAsync(base + off[5] + (size_t)b * N * grow, (const char *)gate + (size_t)b * N * grow,
-                        L * grow, cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return (size_t)(L < 0 ? 0 : (L > N ? N : L));
+  };
+  auto h2d = [&](int i, const void *src, size_t stride, int b) {  // rows t < L_b of row b
+    const size_t n = valid_rows(b) * stride;
+    if (n == 0) return cudaSuccess;
+    return cudaMemcpyAsync(base + off[i] + (size_t)b * N * stride,
+                           (const char *)src + (size_t)b * N * stride, n,
+                           cudaMemcpyHostToDevice, st);
+  };
+  // 1. What the state needs (k, v, gate, weights, lengths), then the state.
+  for (int b = 0; b < B; ++b)
+    if (h2d(1, k, row, b) != cudaSuccess || h2d(2, v, row, b) != cudaSuccess ||
+        h2d(5, gate, grow, b) != cudaSuccess)
       return GBLA_ERR_CUDA;
-  }
   if (cudaMemcpyAsync(base + off[6], conv_w, cw, cudaMemcpyHostToDevice, st) != cudaSuccess ||
       cudaMemcpyAsync(base + off[7], norm_w, nw, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return GBLA_ERR_CUDA;
@@ -293,21 +335,59 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
       return GBLA_ERR_CUDA;
     dsl = (const int32_t *)(base + off[8]);
   }
-  s = gbla_forward(base + off[0], base + off[1], base + off[2], base + off[5], base + off[3],
-                   (const float *)(base + off[6]), (const float *)(base + off[7]), dsl,
-                   base + off[4], B, H, N, D, dtype, stream);
-  if (s != GBLA_OK) return s;
-  for (int b = 0; b < B; ++b) {
-    long L = seq_lens ? seq_lens[b] : N;
-    if (L < 0) L = 0;
-    if (L > N) L = N;
-    if (L == 0) continue;
-    if (cudaMemcpyAsync((char *)o + (size_t)b * N * row, base + off[4] + (size_t)b * N * row, L * row,
-                        cudaMemcpyDeviceToHost, st) != cudaSuccess)
-      return GBLA_ERR_CUDA;
+  p.seq_lens = dsl;
+  float *state = (float *)(base + off[9]);
+  const float *dcw = (const float *)(base + off[6]), *dnw = (const float *)(base + off[7]);
+  if ((s = run_state(p, tc, base + off[1], base + off[2], base + off[5], dcw, state, st)) !=
+      GBLA_OK)
+    return s;
+  // 2. The readout in up to 4 slices of batch rows: q and out_gate of a slice
+  // come in on `stream`, its o goes out on a second stream, so the copy-out of
+  // one slice runs while the next slice is copied in.
+  cudaStream_t out_st = nullptr;
+  cudaEvent_t ev = nullptr, ev_out = nullptr;
+  if (cudaStreamCreateWithFlags(&out_st, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming) != cudaSuccess) {
+    if (out_st) cudaStreamDestroy(out_st);
+    if (ev) cudaEventDestroy(ev);
+    return from_cuda(cudaGetLastError());
   }
+  const int nseg = B < 4 ? B : 4;
+  const int per = (B + nseg - 1) / nseg;
+  cudaError_t e = cudaSuccess;
+  for (int b0 = 0; b0 < B && e == cudaSuccess && s == GBLA_OK; b0 += per) {
+    const int b1 = b0 + per < B ? b0 + per : B;
+    for (int b = b0; b < b1 && e == cudaSuccess; ++b) {
+      if ((e = h2d(0, q, row, b)) == cudaSuccess) e = h2d(3, out_gate, row, b);
+    }
+    if (e != cudaSuccess) break;
+    Problem ps{b1 - b0, H, N, D, dtype, dsl ? dsl + b0 : nullptr};
+    const size_t tb = (size_t)b0 * N * row;
+    s = run_readout(ps, tc, base + off[0] + tb, base + off[3] + tb, dcw, dnw,
+                    state + (size_t)b0 * H * F, base + off[4] + tb, st);
+    if (s != GBLA_OK) break;
+    if ((e = cudaEventRecord(ev, st)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(out_st, ev, 0)) != cudaSuccess)
+      break;
+    for (int b = b0; b < b1 && e == cudaSuccess; ++b) {
+      const size_t n = valid_rows(b) * row;
+      if (n)
+        e = cudaMemcpyAsync((char *)o + (size_t)b * N * row, base + off[4] + (size_t)b * N * row,
+                            n, cudaMemcpyDeviceToHost, out_st);
+    }
+  }
+  // the scratch is freed on `stream` only after the copies out have finished
+  if (cudaEventRecord(ev_out, out_st) != cudaSuccess || cudaStreamWaitEvent(st, ev_out, 0) != cudaSuccess)
+    e = e == cudaSuccess ? cudaGetLastError() : e;
   dev.release();
-  return from_cuda(cudaStreamSynchronize(st));
+  const cudaError_t es2 = cudaStreamSynchronize(st);
+  cudaEventDestroy(ev);
+  cudaEventDestroy(ev_out);
+  cudaStreamDestroy(out_st);
+  if (s != GBLA_OK) return s;
+  if (e != cudaSuccess) return from_cuda(e);
+  return from_cuda(es2);
 }
 
 }  // extern "C"

@@ -8,29 +8,34 @@
 //      a pre-pass over the gate logits gives the chunk maximum m and the
 //      per-token weights 2^a' (a' = (a - m) log2 e); one warp streams raw k
 //      and v tiles (32 tokens + 3 rows of conv history) into a TMA ring;
-//      sixteen converter warps run the causal Conv1D, phi and the gate weight
-//      in fp32 and write K^ and V~ as fp32 into 128B-swizzled K-major tiles;
-//      one thread issues tcgen05.mma kind::tf32 (M = N = 128, K = 8, fp32
-//      accumulation in TMEM): D += K^T V~.  The diagonal D x D blocks of the
-//      accumulator are the per-head partial states S_c; z_c, m_c and
-//      l_c = sum 2^a' complete each partial record.
+//      sixteen converter warps run the causal Conv1D of k, phi and the gate
+//      weight in fp32 and write K^ as bf16 into a 128B-swizzled tile; one
+//      thread issues tcgen05.mma (bf16, fp32 accumulation in TMEM).  The
+//      Conv1D of v is linear, so it is folded into the contraction:
+//      S = sum_tau w_tau (K^T v shifted by tau), the four shifted views of the
+//      raw v tile forming one N = 256 operand, and the taps are applied per
+//      column when the accumulators are drained.  The diagonal D x D blocks
+//      are the per-head partial states S_c; z_c, m_c and l_c = sum 2^a'
+//      complete each partial record.
 //  tc_reduce_kernel  fixed-order, max-rescaled combination of the partial
 //      records into S = K^T V~ and z = K^T 1 with the softmax gate.
 //  tc_readout_kernel (Sec. 2.1 item 2 readout and item 3)
-//      Persistent; 128-token tiles of one (batch, head).  Four producer warps
-//      compute phi(Conv1D(q)) into a K-major bf16 tile; one thread issues
-//      tcgen05.mma against [S | z] (bf16 hi + lo, N = D + 16), giving
-//      phi(q~)^T S and phi(q~)^T z per token in TMEM; four epilogue warps
-//      (one token row per thread) divide, apply RMSNorm, the norm weight and
-//      SiLU(out_gate) (out_gate tile brought in by TMA) and write o in place
-//      of the out_gate tile, which TMA stores back.
+//      Persistent; 128-token tiles of one (batch, head).  Eight producer warps
+//      compute phi(Conv1D(q)) from a TMA q tile into a K-major bf16 tile; one
+//      thread issues tcgen05.mma against [S | z] (bf16 hi + lo, N = D + 16),
+//      giving phi(q~)^T S and phi(q~)^T z per token in TMEM; eight epilogue
+//      warps (two per TMEM lane quarter, one token row per thread) divide,
+//      apply RMSNorm, the norm weight and SiLU(out_gate) (out_gate tile
+//      brought in by TMA) and write o in place of the out_gate tile, which TMA
+//      stores back.
 //
-// Why V~ is not rounded to bf16: V~ = Conv1D(v) is not representable in
+// Why V~ is never rounded to bf16: V~ = Conv1D(v) is not representable in
 // bf16, and its rounding error does not average out, because O is a heavily
 // cancelling weighted mean of the v rows (|O| shrinks like 1/sqrt(L) while the
-// rows stay O(1)).  The state kernel therefore contracts tf32 operands (V~
-// with 11 significant bits after the tf32 rounding inside the MMA, K^ alike),
-// and the readout multiplies by [S | z] as a bf16 hi + lo pair.
+// rows stay O(1)).  The state kernel multiplies the raw bf16 v (exact) and
+// applies the fp32 taps to the fp32 accumulators; the readout multiplies by
+// [S | z] as a bf16 hi + lo pair.  K^ only weights the mean, so bf16 is
+// enough there.
 //
 // Every mbarrier wait is bounded (2 s).  A wait that runs out sets a bit in
 // g_tc_error and the CTA's abort flag; the other waits then return at once,
