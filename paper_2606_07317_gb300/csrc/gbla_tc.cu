@@ -992,7 +992,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
       mbar_init(&q_full[i], 1);
       mbar_init(&q_empty[i], kRProdWarps);
     }
-    mbar_init(b_full, kRProdWarps);
+    mbar_init(b_full, kREpiWarps);
     mbar_init(b_free, 1);
     mbar_init(fin, 1);
     fence_mbar_init();
@@ -1052,73 +1052,26 @@ __global__ void __launch_bounds__(kRThreads, 1)
     // TMA q path: q tile row j holds token r0 - 3 + j; this thread reads rows
     // row0 + k (k = 0..10, 4 channels = 8 bytes) and writes A rows row0 + u
     const uint32_t thr8 = (uint32_t)(stream * 1024 + (c & 1) * 8);
-    int cur_b = -1, cur_h = -1, nbh = 0;
+    int cur_b = -1, cur_h = -1;
     float wq[4][NCH];
     for (long long ii = i0; ii < i1; ++ii) {
       int b, h, r0, nrow;
       tile_of(ii, b, h, r0, nrow);
       const int li = (int)(ii - i0);
       if (b != cur_b || h != cur_h) {
-        // New (b, h): rebuild B = [S | z | 0] as bf16 hi/lo, K-major, 128B swizzle,
-        // once the MMAs that read the previous one have completed.
-        if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, &ab) && !ab.raised())
-          report_error(16, ab);
-        // q taps first (in flight during the rebuild), pre-scaled by log2(e)
-        // later (phi2_log2 takes x log2(e)): 4 NCH consecutive floats per thread
-        float4 wq4[NCH];
-#pragma unroll
-        for (int i = 0; i < NCH; ++i)
-          wq4[i] = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + NCH * c + i) * 4));
-        if (nbh == 0) grid_dep_wait();  // the state comes from the preceding kernel
-        const float *st = p.state + ((size_t)b * H + h) * F;
-        constexpr int NI = NR * (D / 8);  // (row e of B, 8-element K chunk ck) items
-        constexpr int BU = (NI + kRProd - 1) / kRProd < 3 ? (NI + kRProd - 1) / kRProd : 3;
-        for (int item0 = tid; item0 < NI; item0 += BU * kRProd) {
-          float vals[BU][8];  // all items' loads in flight together
-#pragma unroll
-          for (int u = 0; u < BU; ++u) {
-            const int item = item0 + u * kRProd;
-            const int e = item % NR, ck = item / NR;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int d = 8 * ck + i;
-              vals[u][i] = item < NI && e < D ? st[(size_t)d * D + e]
-                                              : (item < NI && e == D ? st[D * D + d] : 0.f);
-            }
-          }
-#pragma unroll
-          for (int u = 0; u < BU; ++u) {
-            const int item = item0 + u * kRProd;
-            if (item >= NI) break;
-            const int e = item % NR, ck = item / NR;
-            uint32_t hi[4], lo[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              hi[i] = f2_to_bf2(vals[u][2 * i], vals[u][2 * i + 1]);
-              const float2 r2 = __ffma2_rn(bf2_to_f2(hi[i]), make_float2(-1.f, -1.f),
-                                           make_float2(vals[u][2 * i], vals[u][2 * i + 1]));
-              lo[i] = f2_to_bf2(r2.x, r2.y);
-            }
-            const int kbk = ck >> 3, ckk = ck & 7;
-            const uint32_t off = kbk * (NR * 128) + (e >> 3) * 1024 + (e & 7) * 128 +
-                                 ((ckk ^ (e & 7)) << 4);
-            sts_v4(smem_u32(smem + C::kOffBhi) + off, make_uint4(hi[0], hi[1], hi[2], hi[3]));
-            sts_v4(smem_u32(smem + C::kOffBlo) + off, make_uint4(lo[0], lo[1], lo[2], lo[3]));
-          }
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_full);
+        // New (b, h): the q taps, pre-scaled by log2(e) (phi2_log2 takes
+        // x log2(e)); 4 NCH consecutive floats per thread.  B = [S | z] is
+        // rebuilt by the epilogue warps.
 #pragma unroll
         for (int i = 0; i < NCH; ++i) {
-          wq[0][i] = wq4[i].x * kLog2e;
-          wq[1][i] = wq4[i].y * kLog2e;
-          wq[2][i] = wq4[i].z * kLog2e;
-          wq[3][i] = wq4[i].w * kLog2e;
+          const float4 t4 = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + NCH * c + i) * 4));
+          wq[0][i] = t4.x * kLog2e;
+          wq[1][i] = t4.y * kLog2e;
+          wq[2][i] = t4.z * kLog2e;
+          wq[3][i] = t4.w * kLog2e;
         }
         cur_b = b;
         cur_h = h;
-        ++nbh;
       }
       const int sa = li & 1;
       if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab) && !ab.raised())
@@ -1184,6 +1137,56 @@ __global__ void __launch_bounds__(kRThreads, 1)
       ogoff[g8] = kbo * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cco ^ (row & 7)) << 4);
     }
     int pend = -1;  // og stage whose TMA store may still be reading it (leader only)
+    // B = [S | z | 0] of (b, h) as bf16 hi/lo, K-major, 128B swizzle, rebuilt
+    // for the first tile and before the first tile of every new (b, h), once
+    // the MMAs that read the previous one have completed (b_free).
+    int nbh = 0;
+    const int etid = tid - kRProd;
+    auto build_b = [&](int b, int h) {
+      if (nbh > 0 && !mbar_wait(b_free, (nbh - 1) & 1, &ab) && !ab.raised()) report_error(16, ab);
+      if (nbh == 0) grid_dep_wait();  // the state comes from the preceding kernel
+      const float *st = p.state + ((size_t)b * H + h) * F;
+      constexpr int NI = NR * (D / 8);  // (row e of B, 8-element K chunk ck) items
+      constexpr int BU = (NI + kREpi - 1) / kREpi < 3 ? (NI + kREpi - 1) / kREpi : 3;
+      for (int item0 = etid; item0 < NI; item0 += BU * kREpi) {
+        float vals[BU][8];  // all items' loads in flight together
+#pragma unroll
+        for (int u = 0; u < BU; ++u) {
+          const int item = item0 + u * kREpi;
+          const int e = item % NR, ck = item / NR;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int d = 8 * ck + i;
+            vals[u][i] = item < NI && e < D ? st[(size_t)d * D + e]
+                                            : (item < NI && e == D ? st[D * D + d] : 0.f);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < BU; ++u) {
+          const int item = item0 + u * kREpi;
+          if (item >= NI) break;
+          const int e = item % NR, ck = item / NR;
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            hi[i] = f2_to_bf2(vals[u][2 * i], vals[u][2 * i + 1]);
+            const float2 r2 = __ffma2_rn(bf2_to_f2(hi[i]), make_float2(-1.f, -1.f),
+                                         make_float2(vals[u][2 * i], vals[u][2 * i + 1]));
+            lo[i] = f2_to_bf2(r2.x, r2.y);
+          }
+          const int kbk = ck >> 3, ckk = ck & 7;
+          const uint32_t off = kbk * (NR * 128) + (e >> 3) * 1024 + (e & 7) * 128 +
+                               ((ckk ^ (e & 7)) << 4);
+          sts_v4(smem_u32(smem + C::kOffBhi) + off, make_uint4(hi[0], hi[1], hi[2], hi[3]));
+          sts_v4(smem_u32(smem + C::kOffBlo) + off, make_uint4(lo[0], lo[1], lo[2], lo[3]));
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_full);
+      ++nbh;
+    };
+    build_b(tc0.b, tc0.h);
     for (long long ii = i0; ii < i1; ++ii) {
       int b, h, r0, nrow;
       tile_of(ii, b, h, r0, nrow);
@@ -1311,6 +1314,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
           mbar_arrive(&og_empty[so]);
         }
         __syncwarp();
+      }
+      if (ii + 1 < i1) {  // the next tile starts a new (b, h): its B, once this one's MMAs are done
+        TileCursor nx = tc0;
+        tile_next(nx, p.seq_lens, B, H, N);
+        if (nx.b != b || nx.h != h) build_b(nx.b, nx.h);
       }
     }
     if (ew == 0 && lane == 0) tma_store_wait_all<0>();
