@@ -260,6 +260,20 @@ __device__ __forceinline__ void tma_load_4d_hint(void *dst, const CUtensorMap *m
       "l"(pol)
       : "memory");
 }
+// L2 policy for data read again soon: its lines are the last to be evicted.
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ void tma_store_4d_hint(const CUtensorMap *m, const void *src, int c0,
+                                                  int c1, int c2, int c3, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.global.shared::cta.bulk_group.L2::cache_hint"
+      " [%0, {%2, %3, %4, %5}], [%1], %6;" ::"l"(reinterpret_cast<uint64_t>(m)),
+      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "l"(pol)
+      : "memory");
+}
 __device__ __forceinline__ void tma_store_4d(const CUtensorMap *m, const void *src, int c0,
                                              int c1, int c2, int c3) {
   asm volatile(

@@ -739,10 +739,11 @@ __global__ void __launch_bounds__(kSThreads, 1)
           fence_proxy_async_smem();
           named_barrier(1, kSProd);
           if (tid == 0) {
+            const uint64_t pol = l2_policy_evict_last();  // read back by the reduction
             for (int hz = 0; hz < G && c.hbase + hz < H; ++hz)
               for (int cbk = 0; cbk < 2; ++cbk)
-                tma_store_4d(&tm_rec, smem + kSOffA + (hz * 2 + cbk) * (64 * 128), cbk * 32, 0,
-                             hz, k);
+                tma_store_4d_hint(&tm_rec, smem + kSOffA + (hz * 2 + cbk) * (64 * 128), cbk * 32,
+                                  0, hz, k, pol);
             tma_store_commit();
             tma_store_wait_read<0>();  // the A ring is written again by the next chunk
           }
@@ -986,7 +987,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
     }
     for (int i = 0; i < OGS; ++i) {
       mbar_init(&og_full[i], 1);
-      mbar_init(&og_empty[i], 1);
+      mbar_init(&og_empty[i], kREpiWarps / 2);  // one release per TMEM lane quarter
     }
     for (int i = 0; i < C::kQStages; ++i) {
       mbar_init(&q_full[i], 1);
@@ -1274,14 +1275,19 @@ __global__ void __launch_bounds__(kRThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[abuf]);
+      // Each lane quarter's 32 rows (both halves) go out on their own: the
+      // pair meets on its named barrier, then one thread stores them with TMA
+      // (full tiles) or releases the buffer after the direct stores (tail).
+      const bool leader = part == 0 && lane == 0;
       if (nrow == kRTok) {
         fence_proxy_async_smem();
-        named_barrier(2, kREpi);
-        if (ew == 0 && lane == 0) {
+        named_barrier(3 + q4, 64);
+        if (leader) {
 #pragma unroll
           for (int kbo = 0; kbo < C::KB; ++kbo)
-            tma_store_4d(&tm_o, smem + C::kOffOg + so * C::kOgBytes + kbo * (kRTok * 128),
-                         kbo * 64, h, r0, b);
+            tma_store_4d(&tm_o, smem + C::kOffOg + so * C::kOgBytes + kbo * (kRTok * 128) +
+                                    q4 * (32 * 128),
+                         kbo * 64, h, r0 + 32 * q4, b);
           tma_store_commit();
           if constexpr (OGS >= 3) {
             // release the previous tile's buffer once its store has read it; this
@@ -1304,8 +1310,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
 #pragma unroll
           for (int cb = 0; cb < CPE; cb += 8) *(uint4 *)(orow + cb) = lds_v4(og_addr(cb));
         }
-        named_barrier(2, kREpi);
-        if (ew == 0 && lane == 0) {
+        named_barrier(3 + q4, 64);
+        if (leader) {
           if (pend >= 0) {
             tma_store_wait_read<0>();
             mbar_arrive(&og_empty[pend]);
@@ -1321,7 +1327,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         if (nx.b != b || nx.h != h) build_b(nx.b, nx.h);
       }
     }
-    if (ew == 0 && lane == 0) tma_store_wait_all<0>();
+    if (part == 0 && lane == 0) tma_store_wait_all<0>();
   } else if (warp == kRMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -1608,7 +1614,7 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   CUtensorMap tm_og, tm_o, tm_q;
   cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D, kRTok);
   if (e != cudaSuccess) return e;
-  if ((e = make_bnhd_map(&tm_o, o, p.B, p.N, p.H, D, kRTok)) != cudaSuccess) return e;
+  if ((e = make_bnhd_map(&tm_o, o, p.B, p.N, p.H, D, 32)) != cudaSuccess) return e;  // a quarter
   if ((e = make_bnhd_map(&tm_q, q, p.B, p.N, p.H, D, C::QT ? kRQRows : kRTok)) != cudaSuccess)
     return e;
   ReadoutParams rp;
