@@ -83,6 +83,18 @@ typedef enum gbla_algo {
 } gbla_algo;
 
 /*
+ * Ablations of the GBLA core (Sec. 4, Table 4): each flag turns one of the
+ * three add-ons of Sec. 2.1 off; all three off is plain bidirectional linear
+ * attention, Eq. bla.  Inputs an ablation ignores must still be valid pointers.
+ */
+typedef enum gbla_flags {
+  GBLA_FLAG_NO_CONV = 1, /* identity Conv1D: q~ = q, k~ = k, v~ = v (conv_w unused)   */
+  GBLA_FLAG_NO_GATE = 2, /* uniform key gate: g_j = 1 / L_b (gate logits unused)      */
+  GBLA_FLAG_NO_NORM = 4, /* no gated RMSNorm: o = O (out_gate and norm_w unused)       */
+  GBLA_FLAG_BLA = 7      /* all three off                                            */
+} gbla_flags;
+
+/*
  * gbla_forward -- the whole GBLA core, Sec. 2.1 (all three add-ons on).
  * Writes o[b, t, h, :] for every b, h and t < L_b.  Equivalent to
  * gbla_forward_ex(..., GBLA_ALGO_AUTO, stream).
@@ -100,6 +112,18 @@ gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
                             const int32_t *seq_lens, void *o, int B, int H,
                             int N, int D, gbla_dtype dtype, gbla_algo algo,
                             gbla_stream_t stream);
+
+/*
+ * gbla_forward_variant -- gbla_forward_ex with ablation flags (gbla_flags,
+ * OR-ed; 0 is gbla_forward_ex).  Flags outside GBLA_FLAG_BLA return
+ * GBLA_ERR_INVALID_ARG before anything is enqueued.
+ */
+gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
+                                 const void *gate, const void *out_gate,
+                                 const float *conv_w, const float *norm_w,
+                                 const int32_t *seq_lens, void *o, int B, int H, int N,
+                                 int D, gbla_dtype dtype, gbla_algo algo, uint32_t flags,
+                                 gbla_stream_t stream);
 
 /*
  * gbla_state -- the sequence-global part of Sec. 2.1 item 2: Conv1D of k and

@@ -242,6 +242,17 @@ gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
                             const int32_t *seq_lens, void *o, int B, int H, int N,
                             int D, gbla_dtype dtype, gbla_algo algo,
                             gbla_stream_t stream) {
+  return gbla_forward_variant(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, o, B, H, N,
+                              D, dtype, algo, 0u, stream);
+}
+
+gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
+                                 const void *gate, const void *out_gate,
+                                 const float *conv_w, const float *norm_w,
+                                 const int32_t *seq_lens, void *o, int B, int H, int N,
+                                 int D, gbla_dtype dtype, gbla_algo algo, uint32_t flags,
+                                 gbla_stream_t stream) {
+  if (flags & ~(uint32_t)GBLA_FLAG_BLA) return GBLA_ERR_INVALID_ARG;
   bool empty = false;
   gbla_status s = check_dims(B, H, N, D, dtype, &empty);
   if (s != GBLA_OK || empty) return s;
@@ -256,7 +267,7 @@ gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
       overlap(out, range_of(norm_w, sizeof(float) * H * D)) ||
       (seq_lens && overlap(out, range_of(seq_lens, sizeof(int32_t) * B))))
     return GBLA_ERR_INVALID_ARG;
-  Problem p{B, H, N, D, dtype, seq_lens};
+  Problem p{B, H, N, D, dtype, seq_lens, flags};
   bool tc = use_tc(p, algo, &s);
   if (s != GBLA_OK) return s;
   cudaStream_t st = (cudaStream_t)stream;

@@ -16,6 +16,7 @@ struct Problem {
   int B, H, N, D;
   gbla_dtype dtype;
   const int32_t *seq_lens;  // device [B] or nullptr
+  uint32_t flags = 0;       // gbla_flags: ablations of Sec. 4, Table 4
 };
 
 // Floats in one partial-state record of a sequence chunk: m (chunk max of the

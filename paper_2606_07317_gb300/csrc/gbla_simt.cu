@@ -59,7 +59,7 @@ __global__ void __launch_bounds__(kThreads)
 simt_partials_kernel(const T *__restrict__ k, const T *__restrict__ v,
                      const T *__restrict__ gate, const float *__restrict__ conv_w,
                      const int32_t *__restrict__ seq_lens, float *__restrict__ part,
-                     int H, int N, int chunk_len, int n_chunks) {
+                     int H, int N, int chunk_len, int n_chunks, uint32_t flags) {
   constexpr int R = D / 16;  // each thread owns an R x R block of S_c
   constexpr int REC = 2 + D + D * D;
   const int c = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -79,15 +79,19 @@ simt_partials_kernel(const T *__restrict__ k, const T *__restrict__ v,
   __shared__ float s_wk[D][kConvW], s_wv[D][kConvW];
   __shared__ float s_red[kThreads / 32];
 
+  const bool no_conv = flags & GBLA_FLAG_NO_CONV, no_gate = flags & GBLA_FLAG_NO_GATE;
   for (int i = tid; i < D * kConvW; i += kThreads) {
-    s_wk[i / kConvW][i % kConvW] = conv_w[((size_t)(1 * H + h) * D) * kConvW + i];
-    s_wv[i / kConvW][i % kConvW] = conv_w[((size_t)(2 * H + h) * D) * kConvW + i];
+    const float id = (i % kConvW) == kConvW - 1 ? 1.f : 0.f;  // identity taps
+    s_wk[i / kConvW][i % kConvW] = no_conv ? id : conv_w[((size_t)(1 * H + h) * D) * kConvW + i];
+    s_wv[i / kConvW][i % kConvW] = no_conv ? id : conv_w[((size_t)(2 * H + h) * D) * kConvW + i];
   }
+  // uniform key gate: every logit 0
+  auto logit = [&](size_t i) { return no_gate ? 0.f : ldf(gate, i); };
 
   // Chunk maximum of the gate logits: exp(a - m_c) <= 1 never overflows.
   const size_t gbase = (size_t)b * N * H + h;
   float m = -INFINITY;
-  for (int t = t0 + tid; t < t1; t += kThreads) m = fmaxf(m, ldf(gate, gbase + (size_t)t * H));
+  for (int t = t0 + tid; t < t1; t += kThreads) m = fmaxf(m, logit(gbase + (size_t)t * H));
   m = warp_max(m);
   if ((tid & 31) == 0) s_red[tid >> 5] = m;
   __syncthreads();
@@ -120,7 +124,7 @@ simt_partials_kernel(const T *__restrict__ k, const T *__restrict__ v,
             xv = fmaf(s_wv[d][i], ldf(vb, (size_t)s * rs + d), xv);
           }
         }
-        const float w = expf(ldf(gate, gbase + (size_t)t * H) - m);
+        const float w = expf(logit(gbase + (size_t)t * H) - m);
         kh = w * phi(xk);
         vv = xv;
       }
@@ -129,7 +133,7 @@ simt_partials_kernel(const T *__restrict__ k, const T *__restrict__ v,
     }
     if (tid < kTokTile) {
       const int t = ts + tid;
-      s_w[tid] = t < t1 ? expf(ldf(gate, gbase + (size_t)t * H) - m) : 0.f;
+      s_w[tid] = t < t1 ? expf(logit(gbase + (size_t)t * H) - m) : 0.f;
     }
     __syncthreads();
 #pragma unroll 4
@@ -202,7 +206,7 @@ __global__ void __launch_bounds__(kThreads)
 simt_readout_kernel(const T *__restrict__ q, const T *__restrict__ og,
                     const float *__restrict__ conv_w, const float *__restrict__ norm_w,
                     const int32_t *__restrict__ seq_lens, const float *__restrict__ state,
-                    T *__restrict__ o, int H, int N, float eps) {
+                    T *__restrict__ o, int H, int N, float eps, uint32_t flags) {
   constexpr int J = D / 32;  // output columns per lane
   const int h = blockIdx.y, b = blockIdx.z;
   const int L = clamp_len(seq_lens, b, N);
@@ -217,7 +221,8 @@ simt_readout_kernel(const T *__restrict__ q, const T *__restrict__ og,
   const float *st = state + ((size_t)b * H + h) * (D * D + D);
   for (int i = tid; i < D * D + D; i += kThreads) sS[i] = st[i];
   for (int i = tid; i < D * kConvW; i += kThreads)
-    swq[i] = conv_w[((size_t)(0 * H + h) * D) * kConvW + i];
+    swq[i] = (flags & GBLA_FLAG_NO_CONV) ? ((i % kConvW) == kConvW - 1 ? 1.f : 0.f)
+                                          : conv_w[((size_t)(0 * H + h) * D) * kConvW + i];
   __syncthreads();
 
   const size_t rs = (size_t)H * D;
@@ -265,7 +270,9 @@ simt_readout_kernel(const T *__restrict__ q, const T *__restrict__ og,
 #pragma unroll
     for (int j = 0; j < J; ++j) {
       const int e = lane + 32 * j;
-      const float y = O[j] * r * norm_w[(size_t)h * D + e] * silu(ldf(og, row + e));
+      const float y = (flags & GBLA_FLAG_NO_NORM)
+                          ? O[j]
+                          : O[j] * r * norm_w[(size_t)h * D + e] * silu(ldf(og, row + e));
       stf(o, row + e, y);
     }
   }
@@ -278,7 +285,7 @@ cudaError_t launch_state(const Problem &p, const SimtPlan &plan, const void *k,
   dim3 g1(plan.n_chunks, p.H, p.B);
   simt_partials_kernel<T, D><<<g1, kThreads, 0, st>>>(
       (const T *)k, (const T *)v, (const T *)gate, conv_w, p.seq_lens, partials,
-      p.H, p.N, plan.chunk_len, plan.n_chunks);
+      p.H, p.N, plan.chunk_len, plan.n_chunks, p.flags);
   count_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -301,7 +308,7 @@ cudaError_t launch_readout(const Problem &p, const void *q, const void *og,
   if (e != cudaSuccess) return e;
   dim3 g((p.N + kTokTile - 1) / kTokTile, p.H, p.B);
   kern<<<g, kThreads, smem, st>>>((const T *)q, (const T *)og, conv_w, norm_w,
-                                  p.seq_lens, state, (T *)o, p.H, p.N, kRmsEps);
+                                  p.seq_lens, state, (T *)o, p.H, p.N, kRmsEps, p.flags);
   count_launch();
   return cudaGetLastError();
 }

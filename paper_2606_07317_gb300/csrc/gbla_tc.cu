@@ -335,6 +335,7 @@ struct StateParams {
   float *records;        // [chunks][G][D*D + D + 4]: S, z, m, l, 2 pad
   int32_t *chunk_pre;    // [B + 1] chunk prefix (written by CTA 0)
   int B, H, N, S, HG;
+  uint32_t flags;        // gbla_flags (NO_CONV, NO_GATE)
 };
 
 // Chunk k of the flattened (batch, head group, chunk) order.
@@ -367,16 +368,22 @@ struct ChunkIn {
 };
 template <int D, int G>
 __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const ChunkRef &c,
-                                                  int tid, int hh, int d0, ChunkIn<G> &in) {
+                                                  int tid, int hh, int d0, ChunkIn<G> &in,
+                                                  uint32_t flags) {
   const int H = p.H, h = c.hbase + hh;
+  const bool no_conv = flags & GBLA_FLAG_NO_CONV, no_gate = flags & GBLA_FLAG_NO_GATE;
+  const float4 ident = make_float4(0.f, 0.f, 0.f, 1.f);  // identity taps (ablation)
 #pragma unroll
   for (int i = 0; i < 4; ++i)
-    in.wk[i] = h < H ? __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4))
-                     : make_float4(0.f, 0.f, 0.f, 0.f);
+    in.wk[i] = h >= H   ? make_float4(0.f, 0.f, 0.f, 0.f)
+               : no_conv ? ident
+                         : __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4));
   in.wv = make_float4(0.f, 0.f, 0.f, 0.f);
   if (tid < kGroupCh) {
     const int hz = c.hbase + tid / D, dz = tid % D;
-    if (hz < H) in.wv = __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
+    if (hz < H)
+      in.wv = no_conv ? ident
+                      : __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
   }
 #pragma unroll
   for (int i = 0; i < kChunkMax / kSProd; ++i) {
@@ -384,7 +391,9 @@ __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const Ch
     const __nv_bfloat16 *gp = p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
 #pragma unroll
     for (int g = 0; g < G; ++g)
-      in.a[i][g] = (tt < c.n && c.hbase + g < H) ? __bfloat162float(gp[g]) : -INFINITY;
+      in.a[i][g] = (tt < c.n && c.hbase + g < H)
+                       ? (no_gate ? 0.f : __bfloat162float(gp[g]))  // uniform gate: logits 0
+                       : -INFINITY;
   }
 }
 
@@ -403,7 +412,9 @@ __device__ __forceinline__ ChunkRef decode_chunk_uniform(const StateParams &p, i
   return c;
 }
 
-template <int D>
+// ABL: the ablation instantiation, which reads p.flags; the default one
+// compiles the full core with no flag tests.
+template <int D, bool ABL>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v,
@@ -426,6 +437,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, H = p.H;
+  const uint32_t flags = ABL ? p.flags : 0u;
 
   // Converter thread -> (group, channel quad q, token quad j): the groups take
   // alternate stages; within a group the mapping makes both the raw-tile
@@ -472,7 +484,8 @@ __global__ void __launch_bounds__(kSThreads, 1)
   // on the critical path.  The TMA warp waits on barrier 3 until they are out.
   ChunkIn<G> cin;
   if (warp < kSCvtWarps) {
-    if (early) load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin);
+    if (early)
+      load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin, flags);
     named_barrier_arrive(3, kSProd + 32);
   } else if (warp == kSTmaWarp) {
     named_barrier(3, kSProd + 32);
@@ -573,7 +586,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
       const int k = (int)kk;
       const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, k);
-      if (!(kk == c0 && early)) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin);
+      if (!(kk == c0 && early)) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin, flags);
 
       // k taps of this thread's 4 channels, pre-scaled by log2(e); v taps of
       // the group's channels for the drain
@@ -894,7 +907,8 @@ struct ReadoutParams {
   __nv_bfloat16 *o;
   int B, H, N;
   float eps;
-  int wait_late;  // only the reads of `state` wait for the preceding kernel
+  int wait_late;   // only the reads of `state` wait for the preceding kernel
+  uint32_t flags;  // gbla_flags (NO_CONV, NO_NORM)
 };
 
 // phi(conv(q)) for 4 consecutive rows of one producer sub-stream; xm holds the
@@ -951,7 +965,7 @@ __device__ __forceinline__ void tile_next(TileCursor &t, const int32_t *seq_lens
   t.nrow = min(kRTok, t.L - t.r0);
 }
 
-template <int D>
+template <int D, bool ABL>
 __global__ void __launch_bounds__(kRThreads, 1)
     tc_readout_kernel(const ReadoutParams p, const __grid_constant__ CUtensorMap tm_og,
                       const __grid_constant__ CUtensorMap tm_o,
@@ -976,6 +990,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int B = p.B, H = p.H, N = p.N;
+  const uint32_t flags = ABL ? p.flags : 0u;  // ablations (see tc_state_kernel)
 
   if (tid == 0) {
     *(volatile int *)(smem + C::kOffMisc + 4) = 0;
@@ -1065,7 +1080,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
         // rebuilt by the epilogue warps.
 #pragma unroll
         for (int i = 0; i < NCH; ++i) {
-          const float4 t4 = __ldg((const float4 *)(p.conv_w + ((size_t)h * D + NCH * c + i) * 4));
+          const float4 t4 = (flags & GBLA_FLAG_NO_CONV)
+                                ? make_float4(0.f, 0.f, 0.f, 1.f)  // identity taps (ablation)
+                                : __ldg((const float4 *)(p.conv_w + ((size_t)h * D + NCH * c + i) * 4));
           wq[0][i] = t4.x * kLog2e;
           wq[1][i] = t4.y * kLog2e;
           wq[2][i] = t4.z * kLog2e;
@@ -1223,6 +1240,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
       const float inv = rcp_approx(den[0]);
       const float ms = ss * inv * inv * (1.f / (float)D);
       const float rr = rsqrtf(ms + p.eps) * inv;
+      const bool no_norm = flags & GBLA_FLAG_NO_NORM;
       const float *nwh = p.norm_w + (size_t)h * D + part * CPE;
       const uint32_t ogt = smem_u32(smem + C::kOffOg + so * C::kOgBytes);
       auto og_addr = [&](int col) {  // col: channel offset within this warp's half
@@ -1254,17 +1272,26 @@ __global__ void __launch_bounds__(kRThreads, 1)
           const float wv8[8] = {wc0.x, wc0.y, wc0.z, wc0.w, wc1.x, wc1.y, wc1.z, wc1.w};
           const float *acc8 = g < 2 ? &va[8 * g] : &vb[8 * (g - 2)];
           uint32_t outw[4];
+          if (no_norm) {  // ablation without the gated RMSNorm: o = O = acc / den
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            // silu(g) = g sigmoid(g) = h + h tanh(h),  h = g / 2
-            const float2 hg = __fmul2_rn(make_float2(gv[2 * i], gv[2 * i + 1]),
-                                         make_float2(0.5f, 0.5f));
-            const float2 sg =
-                __ffma2_rn(hg, make_float2(tanh_approx(hg.x), tanh_approx(hg.y)), hg);
-            const float2 av = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
-                                         make_float2(wv8[2 * i], wv8[2 * i + 1]));
-            const float2 y = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
-            outw[i] = f2_to_bf2(y.x, y.y);
+            for (int i = 0; i < 4; ++i) {
+              const float2 y = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
+                                          make_float2(inv, inv));
+              outw[i] = f2_to_bf2(y.x, y.y);
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              // silu(g) = g sigmoid(g) = h + h tanh(h),  h = g / 2
+              const float2 hg = __fmul2_rn(make_float2(gv[2 * i], gv[2 * i + 1]),
+                                           make_float2(0.5f, 0.5f));
+              const float2 sg =
+                  __ffma2_rn(hg, make_float2(tanh_approx(hg.x), tanh_approx(hg.y)), hg);
+              const float2 av = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
+                                           make_float2(wv8[2 * i], wv8[2 * i + 1]));
+              const float2 y = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
+              outw[i] = f2_to_bf2(y.x, y.y);
+            }
           }
           sts_v4(og_addr(32 * h2 + 8 * g), make_uint4(outw[0], outw[1], outw[2], outw[3]));
           gcur = gnext;
@@ -1575,13 +1602,14 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   sp.H = p.H;
   sp.N = p.N;
   sp.S = S;
+  sp.flags = p.flags;
   sp.HG = (p.H + G - 1) / G;
   CUtensorMap tm_k, tm_v, tm_rec;
   cudaError_t e = make_group_map(&tm_k, k, p.B, p.N, p.H, D);
   if (e != cudaSuccess) return e;
   if ((e = make_bnhd_map(&tm_v, v, p.B, p.N, p.H, D, kSRawRows)) != cudaSuccess) return e;
   if ((e = make_records_map(&tm_rec, ws, p, D, S)) != cudaSuccess) return e;
-  auto k1 = tc_state_kernel<D>;
+  auto k1 = p.flags ? tc_state_kernel<D, true> : tc_state_kernel<D, false>;
   if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
       cudaSuccess)
     return e;
@@ -1629,7 +1657,8 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   rp.N = p.N;
   rp.eps = kRmsEps;
   rp.wait_late = after_state ? 1 : 0;
-  auto kern = tc_readout_kernel<D>;
+  rp.flags = p.flags;
+  auto kern = p.flags ? tc_readout_kernel<D, true> : tc_readout_kernel<D, false>;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem)) !=
       cudaSuccess)
     return e;

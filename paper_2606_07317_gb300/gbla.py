@@ -18,9 +18,13 @@ from . import build as _build
 GBLA_OK, GBLA_ERR_INVALID_ARG, GBLA_ERR_UNSUPPORTED, GBLA_ERR_ALLOC, GBLA_ERR_CUDA = range(5)
 GBLA_FP32, GBLA_BF16 = 0, 1
 ALGO_AUTO, ALGO_SIMT, ALGO_TC = 0, 1, 2
+# ablation flags (gbla_flags): identity Conv1D, uniform key gate, no gated RMSNorm
+FLAG_NO_CONV, FLAG_NO_GATE, FLAG_NO_NORM = 1, 2, 4
+FLAG_BLA = FLAG_NO_CONV | FLAG_NO_GATE | FLAG_NO_NORM
 CONV_WIDTH = 4
 
-EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_state", "gbla_readout",
+EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_state",
+            "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
             "gbla_state_static_scratch", "gbla_device_error", "gbla_last_cuda_error"]
@@ -61,6 +65,8 @@ def load(path: str | None = None):
         lib.gbla_forward.restype = _i
         lib.gbla_forward_ex.argtypes = fwd + [_i, _vp]
         lib.gbla_forward_ex.restype = _i
+        lib.gbla_forward_variant.argtypes = fwd + [_i, ctypes.c_uint32, _vp]
+        lib.gbla_forward_variant.restype = _i
         lib.gbla_forward_host.argtypes = fwd + [_vp]
         lib.gbla_forward_host.restype = _i
         lib.gbla_state.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
@@ -149,11 +155,19 @@ def _bhnd(q: torch.Tensor):
 
 
 def forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
-            algo: int = ALGO_AUTO, stream=None) -> torch.Tensor:
-    """o = GBLA core forward; tensors on one CUDA device, layouts of include/gbla.h."""
+            algo: int = ALGO_AUTO, stream=None, flags: int = 0) -> torch.Tensor:
+    """o = GBLA core forward; tensors on one CUDA device, layouts of include/gbla.h.
+    `flags` (FLAG_*) selects an ablation (gbla_forward_variant); 0 is the full core."""
     B, H, N, D = _bhnd(q)
     if out is None:
         out = torch.empty_like(q)
+    if flags:
+        st = load().gbla_forward_variant(
+            _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
+            _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),
+            int(flags), _stream(stream))
+        _check(st, "gbla_forward_variant")
+        return out
     st = load().gbla_forward_ex(
         _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
         _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),

@@ -10,7 +10,7 @@ import torch
 
 from paper_2606_07317_gb300 import gbla
 from paper_2606_07317_gb300.workloads import WORKLOADS, custom, make_inputs
-from parity_util import compare, oracle_full, oracle_head, to64, valid_mask
+from parity_util import compare, compare_prenorm, oracle_full, oracle_head, to64, valid_mask
 
 pytestmark = pytest.mark.gpu
 
@@ -226,3 +226,35 @@ def test_many_tiles_per_cta_with_empty_sequences():
     y = _run(inp, gbla.ALGO_TC)
     assert gbla.device_error() == 0
     _check_against(y, oracle_full(inp), inp, "bf16")
+
+
+@pytest.mark.parametrize("flags", [1, 2, 4, 3, 5, 6, 7], ids=lambda f: f"flags{f}")
+@pytest.mark.parametrize("algo,dtype", [("tc", "bf16"), ("simt", "fp32"), ("simt", "bf16")])
+def test_ablation_variants(flags, algo, dtype):
+    """The ablations of Table 4 (identity Conv1D, uniform key gate, no gated
+    RMSNorm) and Eq. bla (all three) against the oracle with the same flags."""
+    lens = [1500, 777]
+    w = custom(B=2, H=4, N=1500, D=64, dtype=dtype, seed=40 + flags, seq_lens=lens)
+    inp = make_inputs(w, "cuda")
+    out = torch.full_like(inp["q"], SENTINEL)
+    gbla.device_error(reset=True)
+    gbla.forward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"], inp["conv_w"],
+                 inp["norm_w"], inp["seq_lens"], out=out,
+                 algo=gbla.ALGO_TC if algo == "tc" else gbla.ALGO_SIMT, flags=flags)
+    torch.cuda.synchronize()
+    assert gbla.device_error() == 0
+    ref = oracle_full(inp, flags=flags)
+    mask = valid_mask(2, 1500, np.array(lens))
+    y = to64(out)
+    st = (compare_prenorm if flags & gbla.FLAG_NO_NORM else compare)(y[mask], ref[mask], dtype)
+    assert st["ok"], st
+    assert np.all(y[~mask] == np.float64(torch.tensor(SENTINEL, dtype=out.dtype).item()))
+
+
+def test_ablation_flags_rejected():
+    w = custom(B=1, H=2, N=64, D=64, dtype="bf16", seed=15)
+    inp = make_inputs(w, "cuda")
+    with pytest.raises(gbla.GblaError) as e:
+        gbla.forward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"], inp["conv_w"],
+                     inp["norm_w"], None, flags=8)
+    assert e.value.status == gbla.GBLA_ERR_INVALID_ARG
