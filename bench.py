@@ -173,12 +173,17 @@ def bench_ours(args, ws, rank, local):
     sets = [inp0, {k: (v.clone() if v is not None else None) for k, v in inp0.items()}]
     outs = [torch.empty_like(inp0["q"]) for _ in sets]
     step_bytes = w.valid_tokens * w.H * w.bytes_per_token_head
+    if args.flags:  # an ablation does not need out_gate (no norm) or the gate logits
+        e_el = 2 if w.dtype == "bf16" else 4
+        step_bytes -= w.valid_tokens * w.H * e_el * (
+            (w.D if args.flags & 4 else 0) + (1 if args.flags & 2 else 0))
     stream = torch.cuda.current_stream(dev)
 
     def step(i):
         s = sets[i % 2]
         gbla.forward(s["q"], s["k"], s["v"], s["gate"], s["out_gate"], s["conv_w"],
-                     s["norm_w"], s["seq_lens"], out=outs[i % 2], algo=args.algo, stream=stream)
+                     s["norm_w"], s["seq_lens"], out=outs[i % 2], algo=args.algo, stream=stream,
+                     flags=args.flags)
 
     for i in range(args.warmup):
         step(i)
@@ -204,8 +209,9 @@ def bench_ours(args, ws, rank, local):
     value = tokens * ws / (ms * 1e-3)
 
     # Per-phase durations (state reduction vs readout) with CUDA events on the
-    # launching stream, over the same number of steps.
-    nph = min(args.steps, 500)
+    # launching stream, over the same number of steps (full core only; an
+    # ablation reports the whole step against its own algorithmic bytes).
+    nph = min(args.steps, 500) if not args.flags else 0
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(nph)]
     st_bufs = [torch.empty((w.B, w.H, w.D * w.D + w.D), dtype=torch.float32, device=dev)
                for _ in sets]
@@ -220,8 +226,8 @@ def bench_ours(args, ws, rank, local):
                      s["seq_lens"], out=outs[i % 2], algo=args.algo, stream=stream)
         evs[i][2].record(stream)
     torch.cuda.synchronize(dev)
-    t_state = sum(e[0].elapsed_time(e[1]) for e in evs) / nph
-    t_read = sum(e[1].elapsed_time(e[2]) for e in evs) / nph
+    t_state = sum(e[0].elapsed_time(e[1]) for e in evs) / nph if nph else 0.0
+    t_read = sum(e[1].elapsed_time(e[2]) for e in evs) / nph if nph else 0.0
     e_el = 2 if w.dtype == "bf16" else 4
     per_th = w.valid_tokens * w.H
     bytes_state = per_th * e_el * (2 * w.D + 1)   # k, v, gate
@@ -230,6 +236,8 @@ def bench_ours(args, ws, rank, local):
         dom, dom_ms, dom_bytes = "readout", t_read, bytes_read
     else:
         dom, dom_ms, dom_bytes = "state", t_state, bytes_state
+    if not nph:
+        dom, dom_ms, dom_bytes = "whole step (ablation)", ms, step_bytes
     peak, peak_kind = measured_peaks()
     achieved = dom_bytes / (dom_ms * 1e-3) / 1e9
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
@@ -242,7 +250,7 @@ def bench_ours(args, ws, rank, local):
                 "whole_step_frac": round(step_bytes / (ms * 1e-3) / 1e9 / peak, 4)}
 
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not args.flags:  # the host-buffer entry point runs the full core
         e2e = bench_e2e(args, w, inp0, dev, gbla, tokens, ws)
 
     cpu = None
@@ -261,6 +269,7 @@ def bench_ours(args, ws, rank, local):
                        "l2": "inputs larger than L2 (%.0f MB per set vs 129 MB), two sets rotated"
                              % (step_bytes / 1e6),
                        "algo": {0: "auto", 1: "simt", 2: "tc"}[args.algo],
+                       "flags": args.flags,
                        "parallelism": f"replicas x{ws}" if ws > 1 else "1 GPU"},
             "roofline": roofline,
             "e2e": e2e,
@@ -411,6 +420,9 @@ def main(argv=None):
     ap.add_argument("--algo", type=int, default=0, help="0 auto, 1 simt, 2 tc")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--flags", type=int, default=0,
+                    help="ablation (gbla_flags): 1 no Conv1D, 2 uniform gate, 4 no gated "
+                         "RMSNorm, 7 BLA; 0 (default) is the full core")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
