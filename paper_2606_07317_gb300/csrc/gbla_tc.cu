@@ -60,18 +60,23 @@ using namespace sm100;
 constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the state
 
 // ------------------------------------------------------------------ state
-// 18 warps: two groups of 8 converter warps turn raw k tiles into K^ (bf16,
+// 20 warps: two groups of 8 converter warps turn raw k tiles into K^ (bf16,
 // the A operand), the groups taking alternate stages; one warp issues the
-// MMAs and one the TMA loads.  At most 5 warps per SM sub-partition, so each
-// thread may hold 96 registers.  V~ is never formed: the Conv1D of v is
+// MMAs and three the TMA loads, one box of each stage apiece, with two lanes
+// of each taking alternate stages (a single issuing thread caps an SM's
+// bulk-copy rate at about one box per 0.5 us, well below its share of HBM
+// bandwidth for boxes this size; independent issuers overlap).  At most 5 warps per SM
+// sub-partition, so each thread may hold 96 registers.  V~ is never formed: the Conv1D of v is
 // linear, so S = sum_tau w_tau (K^T v shifted by tau) with the taps applied
 // per column of the accumulators when they are drained, and the raw bf16 v
 // tiles that TMA brings in are the B operand as they stand.
 constexpr int kSGroupWarps = 8;                      // converter warps per group
 constexpr int kSCvtWarps = 2 * kSGroupWarps;         // 16
 constexpr int kSMmaWarp = kSCvtWarps;                // 16
-constexpr int kSTmaWarp = kSCvtWarps + 1;            // 17
-constexpr int kSThreads = (kSTmaWarp + 1) * 32;      // 576
+constexpr int kSTmaWarp = kSCvtWarps + 1;            // 17: k box; 18, 19: v boxes
+constexpr int kSTmaWarps = 3;
+constexpr int kSTmaLanes = 2;  // issuing lanes per TMA warp, taking alternate stages
+constexpr int kSThreads = (kSTmaWarp + kSTmaWarps) * 32;  // 640
 constexpr int kSProd = kSCvtWarps * 32;              // converter threads
 constexpr int kSGroupThreads = kSGroupWarps * 32;
 constexpr int kSTok = 32;                            // tokens per stage
@@ -87,10 +92,10 @@ constexpr int kSRawStage = 20 * 1024;                // 10240 + 8960, rounded to
 constexpr int kSRawStages = 6;
 constexpr int kSABlock = kSTok * 128;                // 4096: one 64-channel MN block of K^
 constexpr int kSAStage = 2 * kSABlock;
-constexpr int kSAStages = 4;
+constexpr int kSAStages = 8;
 constexpr int kChunkMax = 2048;                      // longest chunk (tokens)
 constexpr int kMaxChunksPerSeq = 4096;
-constexpr int kSGateStride = kChunkMax + kSTok;      // (a', 2^a' ln 2) entries per head
+constexpr int kSGateStride = kChunkMax + kSTok;      // gate logits (bf16 bits) per head
 constexpr uint32_t kSTmemCols = 512;                 // per v block: 4 taps x 64 columns
 
 constexpr int kMaxBatch = 2048;
@@ -98,8 +103,8 @@ constexpr int kMaxBatch = 2048;
 // Shared-memory map of the state kernel (offsets from a 1024-aligned base).
 constexpr int kSOffRaw = 0;
 constexpr int kSOffA = kSOffRaw + kSRawStages * kSRawStage;
-constexpr int kSOffGate = kSOffA + kSAStages * kSAStage;            // float2 [2][kSGateStride]
-constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 8;         // float [16][128]
+constexpr int kSOffGate = kSOffA + kSAStages * kSAStage;            // u16 [2][kSGateStride]
+constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 2;         // float [16][128]
 constexpr int kSOffWv = kSOffZred + 16 * kGroupCh * 4;               // float4 [128]: v taps
 constexpr int kSOffRed = kSOffWv + kGroupCh * 16;                   // float [256]
 constexpr int kSOffPre = kSOffRed + 256 * 4;                        // int [kMaxBatch + 1]
@@ -290,8 +295,8 @@ __device__ __forceinline__ float2 conv_rows_n(const float (&w)[4][4], const floa
   return a;
 }
 
-// K^ of two channels from x' = k~ log2(e) and the token's (a', wl = 2^a' ln 2):
-// K^ = 2^a' phi(k~) = wl (x' - min(x', 0)) + 2^(min(x', 0) + a').
+// K^ of two channels from x' = k~ log2(e) and the token's a' = (a - m) log2(e),
+// wl = 2^a' ln 2:  K^ = 2^a' phi(k~) = wl (x' - min(x', 0)) + 2^(min(x', 0) + a').
 __device__ __forceinline__ float2 khat2(float2 xl, float al, float wl) {
   const float2 mn = make_float2(fminf(xl.x, 0.f), fminf(xl.y, 0.f));
   const float2 d = __ffma2_rn(mn, make_float2(-1.f, -1.f), xl);
@@ -300,21 +305,30 @@ __device__ __forceinline__ float2 khat2(float2 xl, float al, float wl) {
   return __ffma2_rn(make_float2(wl, wl), d, e);
 }
 
+// a' = (a - m) log2(e) of a gate logit given as bf16 bits, with mlog = m log2(e)
+// (0 when the head is missing: its logits are all -inf, and so is a').
+__device__ __forceinline__ float gate_log2(unsigned short a, float mlog) {
+  return fmaf(__uint_as_float((uint32_t)a << 16), kLog2e, -mlog);
+}
+
 // One stage of a converter thread: channels 4q..4q+3 of the head group at the
 // stage's tokens 4j..4j+3.  Reads the 7 raw k rows it needs (3 of conv
-// history) from the TMA tile, convolves, applies phi and the gate weight, and
-// writes K^ as bf16 into the MN-major, 128B-swizzled A tile (one 8-byte piece
-// per token row).  Tokens past the sequence end (nvalid < 4) are zeros.
+// history) from the TMA tile and the 4 tokens' gate logits, convolves, applies
+// phi and the gate weight, and writes K^ as bf16 into the MN-major,
+// 128B-swizzled A tile (one 8-byte piece per token row).  Tokens past the
+// sequence end (nvalid < 4) are zeros.
 __device__ __forceinline__ void state_convert(uint32_t raw, uint32_t arow, uint32_t cs,
-                                              uint32_t gws, const float (&w)[4][4],
+                                              uint32_t gws, float mlog, const float (&w)[4][4],
                                               float2 (&z)[2], int nvalid) {
   float x[7][4];
 #pragma unroll
   for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRowK), x[r]);
+  const uint2 g4 = lds_v2(gws);  // 4 bf16 logits
+  const unsigned short ga[4] = {(unsigned short)(g4.x & 0xffffu), (unsigned short)(g4.x >> 16),
+                                (unsigned short)(g4.y & 0xffffu), (unsigned short)(g4.y >> 16)};
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
-    const uint2 gr = lds_v2(gws + u * 8);
-    const float al = __uint_as_float(gr.x), wl = __uint_as_float(gr.y);
+    const float al = gate_log2(ga[u], mlog), wl = ex2_approx(al) * kLn2;
     float2 k01 = khat2(conv_rows(w, x, u, 0), al, wl);
     float2 k23 = khat2(conv_rows(w, x, u, 2), al, wl);
     if (u >= nvalid) {  // rows past the sequence end may hold anything, NaN included
@@ -359,13 +373,17 @@ __device__ __forceinline__ ChunkRef decode_chunk(const StateParams &p, const int
 // Global inputs of one chunk for one converter thread, held in registers so
 // that all of them are in flight together: the k taps of its 4 channels, the
 // v taps of group channel tid (tid < 128), and the gate logits of tokens
-// tid + 256 i of the chunk (-inf past the chunk or for a missing head).
+// tid + 512 i of the chunk as bf16 bits (-inf past the chunk or for a missing
+// head).  Nothing here uses a loaded value, so issuing them never waits.
 template <int G>
 struct ChunkIn {
   float4 wk[4];  // [channel]: taps 0..3
   float4 wv;
-  float a[kChunkMax / kSProd][G];
+  unsigned short a[kChunkMax / kSProd][G];
 };
+__device__ __forceinline__ float bf16_bits_to_f32(unsigned short r) {
+  return __uint_as_float((uint32_t)r << 16);
+}
 template <int D, int G>
 __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const ChunkRef &c,
                                                   int tid, int hh, int d0, ChunkIn<G> &in,
@@ -374,26 +392,30 @@ __device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const Ch
   const bool no_conv = flags & GBLA_FLAG_NO_CONV, no_gate = flags & GBLA_FLAG_NO_GATE;
   const float4 ident = make_float4(0.f, 0.f, 0.f, 1.f);  // identity taps (ablation)
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
-    in.wk[i] = h >= H   ? make_float4(0.f, 0.f, 0.f, 0.f)
-               : no_conv ? ident
-                         : __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4));
+  for (int i = 0; i < 4; ++i) {
+    in.wk[i] = h >= H ? make_float4(0.f, 0.f, 0.f, 0.f) : ident;
+    if (h < H && !no_conv)
+      in.wk[i] = __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4));
+  }
   in.wv = make_float4(0.f, 0.f, 0.f, 0.f);
   if (tid < kGroupCh) {
     const int hz = c.hbase + tid / D, dz = tid % D;
-    if (hz < H)
-      in.wv = no_conv ? ident
-                      : __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
+    if (hz < H) {
+      in.wv = ident;
+      if (!no_conv) in.wv = __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
+    }
   }
 #pragma unroll
   for (int i = 0; i < kChunkMax / kSProd; ++i) {
     const int tt = tid + i * kSProd;
-    const __nv_bfloat16 *gp = p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
+    const unsigned short *gp =
+        (const unsigned short *)p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
 #pragma unroll
-    for (int g = 0; g < G; ++g)
-      in.a[i][g] = (tt < c.n && c.hbase + g < H)
-                       ? (no_gate ? 0.f : __bfloat162float(gp[g]))  // uniform gate: logits 0
-                       : -INFINITY;
+    for (int g = 0; g < G; ++g) {
+      const bool ok = tt < c.n && c.hbase + g < H;
+      in.a[i][g] = ok ? 0u : 0xff80u;  // bf16 -inf: no token
+      if (ok && !no_gate) in.a[i][g] = __ldg(gp + g);  // uniform gate: logits 0
+    }
   }
 }
 
@@ -423,7 +445,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
   constexpr int REC = D * D + D + 4;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float2 *gw = (float2 *)(smem + kSOffGate);  // [G][kSGateStride]: (a', 2^a' ln 2)
+  unsigned short *gw = (unsigned short *)(smem + kSOffGate);  // [G][kSGateStride]: logits
   float *zred = (float *)(smem + kSOffZred);  // [16][128]
   float4 *wv = (float4 *)(smem + kSOffWv);    // [128]: v taps of the group's channels
   float *red = (float *)(smem + kSOffRed);    // [0,64) max, [64,128) sum, 128+ m, 132+ l
@@ -462,7 +484,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
   if (warp == kSTmaWarp && lane == 0) {
     // the raw ring's barriers are first used by this thread
     for (int i = 0; i < kSRawStages; ++i) {
-      mbar_init(&raw_full[i], 1);
+      mbar_init(&raw_full[i], kSTmaWarps);         // one box per TMA warp
       mbar_init(&raw_empty[i], kSGroupWarps + 1);  // one converter group reads k, the MMAs v
     }
     fence_mbar_init();
@@ -479,79 +501,94 @@ __global__ void __launch_bounds__(kSThreads, 1)
     mbar_init(fin, 1);
     fence_mbar_init();
   }
+  // One box of a raw stage per TMA warp: 0 the k group rows, 1 + blk the v
+  // block blk (absent for a missing head: a plain arrival).
+  const int tbox = warp - kSTmaWarp;
+  auto issue_box = [&](const ChunkRef &c, int it, uint32_t s, uint64_t pol) {
+    uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
+    const int tok = c.t0 + it * kSTok - kSHalo;
+    if (tbox == 0) {
+      mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes);
+      tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b, pol);
+    } else {
+      const int blk = tbox - 1;
+      if (D == 64 && c.hbase + blk >= H) {
+        mbar_arrive(&raw_full[s]);
+      } else {
+        mbar_arrive_expect_tx(&raw_full[s], kSVBoxBytes);
+        tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
+                         c.hbase + (blk * 64) / D, tok, c.b, pol);
+      }
+    }
+  };
   // The first chunk's global reads (gate logits, taps) go out before the bulk
   // k/v loads, which would otherwise queue ahead of them: the gate pre-pass is
-  // on the critical path.  The TMA warp waits on barrier 3 until they are out.
+  // on the critical path.  The TMA warps wait on barrier 3 until they are out.
   ChunkIn<G> cin;
   if (warp < kSCvtWarps) {
     if (early)
       load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin, flags);
-    named_barrier_arrive(3, kSProd + 32);
-  } else if (warp == kSTmaWarp) {
-    named_barrier(3, kSProd + 32);
+    named_barrier_arrive(3, kSProd + 32 * kSTmaWarps);
+  } else if (warp >= kSTmaWarp) {
+    named_barrier(3, kSProd + 32 * kSTmaWarps);
   }
-  if (warp == kSTmaWarp && lane == 0) {
+  if (warp >= kSTmaWarp && lane < kSTmaLanes && early) {
     const uint64_t pol = l2_policy_evict_first();
-    if (early) {
-      const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
-      const int nvb = D == 64 ? min(2, H - c.hbase) : 2;
-      for (int it = 0; it < min(c.nst, kSRawStages); ++it) {
-        uint8_t *dst = smem + kSOffRaw + it * kSRawStage;
-        const int tok = c.t0 + it * kSTok - kSHalo;
-        mbar_arrive_expect_tx(&raw_full[it], kSRawKBytes + nvb * kSVBoxBytes);
-        tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[it], 0, c.hbase, tok, c.b, pol);
-        for (int blk = 0; blk < nvb; ++blk)
-          tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[it], (blk * 64) % D,
-                           c.hbase + (blk * 64) / D, tok, c.b, pol);
-      }
-    }
+    const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
+    for (int it = lane; it < min(c.nst, kSRawStages); it += kSTmaLanes)
+      issue_box(c, it, (uint32_t)it, pol);
   }
-  // Chunk prefix over the batch (converter threads), shared by all roles.
+  // Chunk prefix over the batch (converter threads), shared by all roles.  A
+  // TMA issuing thread can have about one copy in flight, so the early burst
+  // above takes a while: the converters hand the prefix to the TMA warps
+  // (barrier 4) and to the MMA warp (barrier 5) without waiting for them.
   if (warp < kSCvtWarps) {
     prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
       const int L = clamp_len(p.seq_lens, b, p.N);
       return p.HG * ((L + p.S - 1) / p.S);
     });
+    if (blockIdx.x == 0)
+      for (int i = tid; i <= B; i += kSProd) p.chunk_pre[i] = pre[i];
+    named_barrier_arrive(4, kSProd + 32 * kSTmaWarps);
+    named_barrier_arrive(5, kSProd + 32);
+  } else if (warp == kSMmaWarp) {
+    named_barrier(5, kSProd + 32);
+  } else {
+    named_barrier(4, kSProd + 32 * kSTmaWarps);
   }
-  __syncthreads();
   const int K = pre[B];
-  if (blockIdx.x == 0)
-    for (int i = tid; i <= B; i += kSThreads) p.chunk_pre[i] = pre[i];
   const long long c0 = (long long)K * blockIdx.x / gridDim.x;
   const long long c1 = (long long)K * (blockIdx.x + 1) / gridDim.x;
   grid_dep_launch();
   if (c0 >= c1) return;  // no chunks for this CTA
   const ChunkRef cfirst = decode_chunk<G>(p, pre, (int)c0);
 
-  if (warp == kSTmaWarp) {
+  if (warp >= kSTmaWarp) {
     // ------------------------------------------------------------ TMA loads
     // Per stage: v as two 64-channel blocks of 35 token rows (128B swizzle)
     // and the k group rows (no swizzle); 3 rows of conv history in front,
-    // zero-filled before the sequence start.  This warp takes no part in the
-    // TMEM hand-off, so its first loads go out at once.
-    if (lane == 0) {
+    // zero-filled before the sequence start.  These warps take no part in the
+    // TMEM hand-off, so their first loads go out at once.  Lane l issues the
+    // stages whose index in the CTA's sequence is l modulo kSTmaLanes.
+    if (lane < kSTmaLanes) {
       // stages of the first chunk already issued before the prefix
       const int it0 = early ? min(cfirst.nst, kSRawStages) : 0;
       const uint64_t pol = l2_policy_evict_first();
       uint32_t issued = (uint32_t)it0;
       for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
         const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, (int)kk);
-        const int nvb = D == 64 ? min(2, H - c.hbase) : 2;  // v blocks of existing heads
-        for (int it = kk == c0 ? it0 : 0; it < c.nst; ++it) {
+        bool ok = true;
+        for (int it = kk == c0 ? it0 : 0; it < c.nst; ++it, ++issued) {
+          if (issued % kSTmaLanes != (uint32_t)lane) continue;
           const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
           if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
             if (!ab.raised()) report_error(2048, ab);
+            ok = false;
             break;
           }
-          uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
-          const int tok = c.t0 + it * kSTok - kSHalo;
-          mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes + nvb * kSVBoxBytes);
-          tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b, pol);
-          for (int blk = 0; blk < nvb; ++blk)
-            tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
-                             c.hbase + (blk * 64) / D, tok, c.b, pol);
-          ++issued;
+          issue_box(c, it, s, pol);
         }
+        if (!ok) break;
       }
       // every issued copy has landed before the CTA can exit
       for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
@@ -580,7 +617,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
                                                                 4 * j * 128 + (q & 1) * 8);
     const uint32_t cs = (uint32_t)(((q & 15) >> 1) ^ (4 * (j & 1)));
     const uint32_t raw0 = smem_u32(smem + kSOffRaw + kSRawK) + (uint32_t)(4 * j * kSRawRowK + q * 8);
-    const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kSGateStride + 4 * j) * 8;
+    const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kSGateStride + 4 * j) * 2;
     uint32_t gs0 = 0;  // first stage of the chunk in the CTA's stage sequence
     int nchunk = 0;
     for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
@@ -600,8 +637,11 @@ __global__ void __launch_bounds__(kSThreads, 1)
       }
       if (tid < kGroupCh) wv[tid] = cin.wv;
 
-      // Gate pre-pass: per-head chunk maximum m; (a', 2^a' ln 2) per token with
-      // a' = (a - m) log2(e); l = sum 2^a'.  Entries past the chunk: (-inf, 0).
+      // Gate pre-pass: per-head chunk maximum m and l = sum 2^a' with
+      // a' = (a - m) log2(e); the logits go to shared memory for the stages,
+      // which form a' and 2^a' per token themselves.  Entries past the chunk
+      // are -inf.
+      float mlog = 0.f;  // m log2(e) of this thread's head
       {
         constexpr int kPer = kChunkMax / kSProd;
         float m[G];
@@ -609,7 +649,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
         for (int g = 0; g < G; ++g) {
           m[g] = -INFINITY;
 #pragma unroll
-          for (int i = 0; i < kPer; ++i) m[g] = fmaxf(m[g], cin.a[i][g]);
+          for (int i = 0; i < kPer; ++i) m[g] = fmaxf(m[g], bf16_bits_to_f32(cin.a[i][g]));
 #pragma unroll
           for (int o = 16; o >= 1; o >>= 1) m[g] = fmaxf(m[g], __shfl_xor_sync(0xffffffffu, m[g], o));
           if (lane == 0) red[warp * 4 + g] = m[g];
@@ -620,14 +660,15 @@ __global__ void __launch_bounds__(kSThreads, 1)
         for (int g = 0; g < G; ++g) {
           float M = red[g];
           for (int w2 = 1; w2 < kSCvtWarps; ++w2) M = fmaxf(M, red[w2 * 4 + g]);
-          const bool hok = c.hbase + g < H;
+          // a missing head has only -inf logits: M = -inf, and a' = -inf with mlog 0
+          const float ml = M == -INFINITY ? 0.f : M * kLog2e;
+          if (g == hh) mlog = ml;
           float l = 0.f;
 #pragma unroll
           for (int i = 0; i < kPer; ++i) {
             const int tt = tid + i * kSProd;
-            const float al = hok ? (cin.a[i][g] - M) * kLog2e : -INFINITY;
-            const float ex = ex2_approx(al);
-            if (tt < npad) gw[g * kSGateStride + tt] = make_float2(al, ex * kLn2);
+            const float ex = ex2_approx(gate_log2(cin.a[i][g], ml));
+            if (tt < npad) gw[g * kSGateStride + tt] = cin.a[i][g];
             l += ex;
           }
 #pragma unroll
@@ -654,7 +695,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
         const int T = c.t0 + it * kSTok;
         const int nvalid = min(max(c.L - (T + 4 * j), 0), 4);
         state_convert(raw0 + rs * kSRawStage, arow0 + as * kSAStage, cs,
-                      gws + (uint32_t)(it * kSTok) * 8, w, z, nvalid);
+                      gws + (uint32_t)(it * kSTok) * 2, mlog, w, z, nvalid);
         if (T + kSTok > c.L) {
           // v rows past the sequence end meet K^ = 0 in the MMA, but may hold
           // NaN or inf: zero them (both 64-channel blocks)
@@ -786,32 +827,36 @@ __global__ void __launch_bounds__(kSThreads, 1)
       // with the start moved down 0..3 rows (LBO = one 128-byte row).  The
       // 128-byte swizzle follows the absolute shared address, so the shifted
       // views read the rows TMA wrote.
+      // This warp shares its SM sub-partition with busy converter warps, so
+      // the loop is kept short: descriptors of slot 0 advanced by the slot
+      // offsets (a descriptor's address field is the byte address >> 4, and
+      // shared addresses stay below 256 KB, so adding to it never carries),
+      // and ring positions stepped rather than divided.
       constexpr uint32_t idesc = idesc_bf16_f32(128, 256, 1, 1);
-      const uint32_t a0 = smem_u32(smem + kSOffA), v0 = smem_u32(smem + kSOffRaw);
-      uint32_t gs = 0;
+      const uint64_t ad0 = sw128_desc(smem_u32(smem + kSOffA), kSABlock, 1024);
+      const uint64_t bd0 = sw128_desc(smem_u32(smem + kSOffRaw), 128, 1024);
+      uint32_t rs = 0, rph = 0, as = 0, aph = 0;
       bool ok = true;
       for (long long kk = c0; kk < c1 && ok; ++kk) {
         const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
-        for (int it = 0; it < c.nst; ++it, ++gs) {
-          const uint32_t rs = gs % kSRawStages, rph = (gs / kSRawStages) & 1;
-          const uint32_t as = gs % kSAStages, aph = (gs / kSAStages) & 1;
+        for (int it = 0; it < c.nst; ++it) {
           if (!mbar_wait(&a_full[as], aph, &ab) || !mbar_wait(&raw_full[rs], rph, &ab)) {
             if (!ab.raised()) report_error(4, ab);
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t ab0 = a0 + as * kSAStage, vb0 = v0 + rs * kSRawStage;
+          const uint64_t ad = ad0 + (as * kSAStage >> 4), bd = bd0 + (rs * kSRawStage >> 4);
 #pragma unroll
           for (int blk = 0; blk < 2; ++blk)
 #pragma unroll
-            for (int k16 = 0; k16 < kSTok / 16; ++k16) {
-              const uint64_t ad = sw128_desc(ab0 + k16 * 2048, kSABlock, 1024);
-              const uint64_t bd = sw128_desc(vb0 + blk * kSVBlock + 16 * k16 * 128, 128, 1024);
-              mma_bf16(tmem + 256 * blk, ad, bd, idesc, (it | k16) != 0);
-            }
+            for (int k16 = 0; k16 < kSTok / 16; ++k16)
+              mma_bf16(tmem + 256 * blk, ad + (k16 * 2048 >> 4),
+                       bd + ((blk * kSVBlock + 16 * k16 * 128) >> 4), idesc, (it | k16) != 0);
           mma_commit(&a_empty[as]);
           mma_commit(&raw_empty[rs]);
+          if (++as == kSAStages) { as = 0; aph ^= 1; }
+          if (++rs == kSRawStages) { rs = 0; rph ^= 1; }
         }
         if (ok) mma_commit(done);
       }
