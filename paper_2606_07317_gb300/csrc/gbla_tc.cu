@@ -6,8 +6,8 @@
 //      is cut into chunks of S tokens and every CTA takes a contiguous range of
 //      chunks, so work is balanced whatever the sequence lengths.  Per chunk:
 //      a pre-pass over the gate logits gives the chunk maximum m and the
-//      per-token weights 2^a' (a' = (a - m) log2 e); one warp streams raw k
-//      and v tiles (32 tokens + 3 rows of conv history) into a TMA ring;
+//      per-token weights 2^a' (a' = (a - m) log2 e); three warps stream raw
+//      k and v tiles (64 tokens + 3 rows of conv history) into a TMA ring;
 //      sixteen converter warps run the causal Conv1D of k, phi and the gate
 //      weight in fp32 and write K^ as bf16 into a 128B-swizzled tile; one
 //      thread issues tcgen05.mma (bf16, fp32 accumulation in TMEM).  The
@@ -79,20 +79,20 @@ constexpr int kSTmaLanes = 2;  // issuing lanes per TMA warp, taking alternate s
 constexpr int kSThreads = (kSTmaWarp + kSTmaWarps) * 32;  // 640
 constexpr int kSProd = kSCvtWarps * 32;              // converter threads
 constexpr int kSGroupThreads = kSGroupWarps * 32;
-constexpr int kSTok = 32;                            // tokens per stage
+constexpr int kSTok = 64;                            // tokens per stage
 constexpr int kSHalo = kConvW - 1;                   // conv history rows in front of a tile
-constexpr int kSRawRows = kSTok + kSHalo;            // 35
-// raw stage: v as two 64-channel MN blocks (128B swizzle, 40-row pitch) + k group rows
-constexpr int kSVBlock = 40 * 128;                   // 5120: v block pitch (1024-aligned)
-constexpr int kSVBoxBytes = kSRawRows * 128;         // 4480 written by one v box
+constexpr int kSRawRows = kSTok + kSHalo;            // 67
+// raw stage: v as two 64-channel MN blocks (128B swizzle, 72-row pitch) + k group rows
+constexpr int kSVBlock = 72 * 128;                   // 9216: v block pitch (1024-aligned)
+constexpr int kSVBoxBytes = kSRawRows * 128;         // 8576 written by one v box
 constexpr int kSRawRowK = kGroupCh * 2;              // bytes of one token's k group row
-constexpr int kSRawKBytes = kSRawRows * kSRawRowK;   // 8960
+constexpr int kSRawKBytes = kSRawRows * kSRawRowK;   // 17152
 constexpr int kSRawK = 2 * kSVBlock;                 // k tile offset within a raw stage
-constexpr int kSRawStage = 20 * 1024;                // 10240 + 8960, rounded to 1024
-constexpr int kSRawStages = 6;
-constexpr int kSABlock = kSTok * 128;                // 4096: one 64-channel MN block of K^
+constexpr int kSRawStage = (kSRawK + kSRawKBytes + 1023) / 1024 * 1024;  // 35840
+constexpr int kSRawStages = 4;
+constexpr int kSABlock = kSTok * 128;                // 8192: one 64-channel MN block of K^
 constexpr int kSAStage = 2 * kSABlock;
-constexpr int kSAStages = 8;
+constexpr int kSAStages = 3;
 constexpr int kChunkMax = 2048;                      // longest chunk (tokens)
 constexpr int kMaxChunksPerSeq = 4096;
 constexpr int kSGateStride = kChunkMax + kSTok;      // gate logits (bf16 bits) per head
@@ -311,8 +311,8 @@ __device__ __forceinline__ float gate_log2(unsigned short a, float mlog) {
   return fmaf(__uint_as_float((uint32_t)a << 16), kLog2e, -mlog);
 }
 
-// One stage of a converter thread: channels 4q..4q+3 of the head group at the
-// stage's tokens 4j..4j+3.  Reads the 7 raw k rows it needs (3 of conv
+// One token quad of a converter thread: channels 4q..4q+3 of the head group
+// at tokens 4j..4j+3 of a 32-token half of the stage.  Reads the 7 raw k rows it needs (3 of conv
 // history) from the TMA tile and the 4 tokens' gate logits, convolves, applies
 // phi and the gate weight, and writes K^ as bf16 into the MN-major,
 // 128B-swizzled A tile (one 8-byte piece per token row).  Tokens past the
@@ -565,7 +565,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
 
   if (warp >= kSTmaWarp) {
     // ------------------------------------------------------------ TMA loads
-    // Per stage: v as two 64-channel blocks of 35 token rows (128B swizzle)
+    // Per stage: v as two 64-channel blocks of 67 token rows (128B swizzle)
     // and the k group rows (no swizzle); 3 rows of conv history in front,
     // zero-filled before the sequence start.  These warps take no part in the
     // TMEM hand-off, so their first loads go out at once.  Lane l issues the
@@ -693,9 +693,13 @@ __global__ void __launch_bounds__(kSThreads, 1)
         if (!mbar_wait(&raw_full[rs], rph, &ab) && !ab.raised()) report_error(1, ab);
         if (!mbar_wait(&a_empty[as], aph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
         const int T = c.t0 + it * kSTok;
-        const int nvalid = min(max(c.L - (T + 4 * j), 0), 4);
-        state_convert(raw0 + rs * kSRawStage, arow0 + as * kSAStage, cs,
-                      gws + (uint32_t)(it * kSTok) * 2, mlog, w, z, nvalid);
+#pragma unroll
+        for (int hq = 0; hq < kSTok / 32; ++hq) {  // token quads j + 8 hq (rows 32 hq on)
+          const int nvalid = min(max(c.L - (T + 32 * hq + 4 * j), 0), 4);
+          state_convert(raw0 + rs * kSRawStage + hq * 32 * kSRawRowK,
+                        arow0 + as * kSAStage + hq * 32 * 128, cs,
+                        gws + (uint32_t)(it * kSTok + 32 * hq) * 2, mlog, w, z, nvalid);
+        }
         if (T + kSTok > c.L) {
           // v rows past the sequence end meet K^ = 0 in the MMA, but may hold
           // NaN or inf: zero them (both 64-channel blocks)
