@@ -160,7 +160,8 @@ struct ReadoutCfg {
   static constexpr int kOffQ = kOffOg + kOgStages * kOgBytes;
   static constexpr int kOffPre = kOffQ + kQStages * kQBytes;      // int [kMaxBatch + 1]
   static constexpr int kOffSs = kOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;  // float [256]
-  static constexpr int kOffBar = kOffSs + kREpi * 4;
+  static constexpr int kOffW = kOffSs + kREpi * 4;  // float [D]: norm weights of the head
+  static constexpr int kOffBar = kOffW + D * 4;
   // a_full[2], a_empty[2], og_full[S], og_empty[S], q_full[Q], q_empty[Q],
   // acc_full[2], acc_empty[2], b_full, b_free, final
   static constexpr int kBars =
@@ -1248,8 +1249,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
           sts_v4(smem_u32(smem + C::kOffBlo) + off, make_uint4(lo[0], lo[1], lo[2], lo[3]));
         }
       }
+      // the head's norm weights for the epilogue, read back after barrier 7
+      if (etid < D / 4)
+        *(float4 *)(smem + C::kOffW + 16 * etid) = __ldg((const float4 *)(p.norm_w + (size_t)h * D) + etid);
       fence_proxy_async_smem();
-      __syncwarp();
+      named_barrier(7, kREpi);
       if (lane == 0) mbar_arrive(b_full);
       ++nbh;
     };
@@ -1290,7 +1294,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
       const float ms = ss * inv * inv * (1.f / (float)D);
       const float rr = rsqrtf(ms + p.eps) * inv;
       const bool no_norm = flags & GBLA_FLAG_NO_NORM;
-      const float *nwh = p.norm_w + (size_t)h * D + part * CPE;
+      const uint32_t nws = smem_u32(smem + C::kOffW) + (uint32_t)(part * CPE) * 4;
       const uint32_t ogt = smem_u32(smem + C::kOffOg + so * C::kOgBytes);
       auto og_addr = [&](int col) {  // col: channel offset within this warp's half
         return ogt + ogoff[col / 8];
@@ -1305,16 +1309,23 @@ __global__ void __launch_bounds__(kRThreads, 1)
         }
         // four groups of 8 channels; out_gate and weights of the next group in flight
         uint4 gcur = lds_v4(og_addr(32 * h2));
-        float4 wc0 = __ldg((const float4 *)(nwh + 32 * h2));
-        float4 wc1 = __ldg((const float4 *)(nwh + 32 * h2 + 4));
+        uint4 wr0 = lds_v4(nws + (32 * h2) * 4), wr1 = lds_v4(nws + (32 * h2 + 4) * 4);
+        float4 wc0 = make_float4(__uint_as_float(wr0.x), __uint_as_float(wr0.y),
+                                 __uint_as_float(wr0.z), __uint_as_float(wr0.w));
+        float4 wc1 = make_float4(__uint_as_float(wr1.x), __uint_as_float(wr1.y),
+                                 __uint_as_float(wr1.z), __uint_as_float(wr1.w));
 #pragma unroll
         for (int g = 0; g < 4; ++g) {
           uint4 gnext = gcur;
           float4 wn0 = wc0, wn1 = wc1;
           if (g < 3) {
             gnext = lds_v4(og_addr(32 * h2 + 8 * (g + 1)));
-            wn0 = __ldg((const float4 *)(nwh + 32 * h2 + 8 * (g + 1)));
-            wn1 = __ldg((const float4 *)(nwh + 32 * h2 + 8 * (g + 1) + 4));
+            const uint4 r0 = lds_v4(nws + (32 * h2 + 8 * (g + 1)) * 4);
+            const uint4 r1 = lds_v4(nws + (32 * h2 + 8 * (g + 1) + 4) * 4);
+            wn0 = make_float4(__uint_as_float(r0.x), __uint_as_float(r0.y), __uint_as_float(r0.z),
+                              __uint_as_float(r0.w));
+            wn1 = make_float4(__uint_as_float(r1.x), __uint_as_float(r1.y), __uint_as_float(r1.z),
+                              __uint_as_float(r1.w));
           }
           float gv[8];
           unpack8(gcur, gv);
