@@ -90,6 +90,10 @@ constexpr int kSRawKBytes = kSRawRows * kSRawRowK;   // 17152
 constexpr int kSRawK = 2 * kSVBlock;                 // k tile offset within a raw stage
 constexpr int kSRawStage = (kSRawK + kSRawKBytes + 1023) / 1024 * 1024;  // 35840
 constexpr int kSRawStages = 4;
+// Raw stages issued before the chunk prefix: one.  The first stage then
+// arrives ahead of the rest of every CTA's start-up burst (measured: 1.1 us
+// shorter step than issuing the whole ring up front).
+constexpr int kSEarlyStages = 1;
 constexpr int kSABlock = kSTok * 128;                // 8192: one 64-channel MN block of K^
 constexpr int kSAStage = 2 * kSABlock;
 constexpr int kSAStages = 3;
@@ -527,8 +531,17 @@ __global__ void __launch_bounds__(kSThreads, 1)
   // on the critical path.  The TMA warps wait on barrier 3 until they are out.
   ChunkIn<G> cin;
   if (warp < kSCvtWarps) {
-    if (early)
+    if (early) {
       load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin, flags);
+      // the logits have arrived before the bulk loads go out: they would
+      // otherwise queue behind the whole start-up burst of every CTA
+      uint32_t sink = 0;
+#pragma unroll
+      for (int i = 0; i < kChunkMax / kSProd; ++i)
+#pragma unroll
+        for (int g = 0; g < G; ++g) sink += cin.a[i][g];
+      asm volatile("" ::"r"(sink));
+    }
     named_barrier_arrive(3, kSProd + 32 * kSTmaWarps);
   } else if (warp >= kSTmaWarp) {
     named_barrier(3, kSProd + 32 * kSTmaWarps);
@@ -536,7 +549,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
   if (warp >= kSTmaWarp && lane < kSTmaLanes && early) {
     const uint64_t pol = l2_policy_evict_first();
     const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
-    for (int it = lane; it < min(c.nst, kSRawStages); it += kSTmaLanes)
+    for (int it = lane; it < min(c.nst, kSEarlyStages); it += kSTmaLanes)
       issue_box(c, it, (uint32_t)it, pol);
   }
   // Chunk prefix over the batch (converter threads), shared by all roles.  A
@@ -573,7 +586,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     // stages whose index in the CTA's sequence is l modulo kSTmaLanes.
     if (lane < kSTmaLanes) {
       // stages of the first chunk already issued before the prefix
-      const int it0 = early ? min(cfirst.nst, kSRawStages) : 0;
+      const int it0 = early ? min(cfirst.nst, kSEarlyStages) : 0;
       const uint64_t pol = l2_policy_evict_first();
       uint32_t issued = (uint32_t)it0;
       for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
@@ -902,7 +915,8 @@ __global__ void __launch_bounds__(kReduceThreads) tc_reduce_kernel(const float *
   if (e0 >= F) return;
   const int L = clamp_len(seq_lens, b, N);
   const int nck = (L + S - 1) / S;
-  const int k0 = chunk_pre[b] + hg * nck;
+  // with every sequence N tokens long the prefix is b HG nck: no dependent load
+  const int k0 = (seq_lens == nullptr ? b * ((H + G - 1) / G) * nck : chunk_pre[b]) + hg * nck;
   const float *rec0 = records + ((size_t)k0 * G + hh) * REC;
   const size_t rstride = (size_t)G * REC;
   float M = -INFINITY, l = 0.f;
