@@ -76,6 +76,16 @@ def _declare(lib):
     lib.oracle_gbla_head.argtypes = head_common + [_dp] * 7
     lib.oracle_gbla_head_quadratic.restype = ctypes.c_int
     lib.oracle_gbla_head_quadratic.argtypes = head_common + [_dp]
+    lib.oracle_gbla_head_backward.restype = ctypes.c_int
+    lib.oracle_gbla_head_backward.argtypes = (
+        [_dp, _dp, _dp, _dp, _dp, ctypes.c_long, ctypes.c_long, ctypes.c_long, ctypes.c_int,
+         _dp, _dp, _dp, ctypes.c_int, _dp, ctypes.c_double, ctypes.c_int, _dp] + [_dp] * 9)
+    lib.oracle_gbla_backward.restype = ctypes.c_int
+    lib.oracle_gbla_backward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
+                                         ctypes.POINTER(ctypes.c_int32),
+                                         ctypes.c_long, ctypes.c_long, ctypes.c_long,
+                                         ctypes.c_int, ctypes.c_int, ctypes.c_double,
+                                         ctypes.c_int, _dp] + [_dp] * 7
     lib.oracle_gbla_forward.restype = ctypes.c_int
     lib.oracle_gbla_forward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
                                         ctypes.POINTER(ctypes.c_int32),
@@ -205,3 +215,52 @@ def gbla_forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None,
     if rc != 0:
         raise ValueError(f"oracle_gbla_forward rejected its arguments ({rc})")
     return y
+
+
+def gbla_head_backward(q, k, v, a, og, wq, wk, wv, norm_w, dy, eps=RMS_EPS, flags=0,
+                       lib=None):
+    """Gradients of sum(dy * y) for one (batch, head) (chain rule through the six
+    forward steps of Sec. 2.1, reverse order).  Returns a dict with dq, dk, dv, dog
+    [L, D], da [L], dwq, dwk, dwv [D, W] and dnorm_w [D]."""
+    q, k, v, og, dy = (_f64(t) for t in (q, k, v, og, dy))
+    a = _f64(a); wq, wk, wv = (_f64(t) for t in (wq, wk, wv)); norm_w = _f64(norm_w)
+    L, D = q.shape
+    W = wq.shape[1]
+    out = dict(dq=np.zeros((L, D)), dk=np.zeros((L, D)), dv=np.zeros((L, D)),
+               da=np.zeros(L), dog=np.zeros((L, D)), dwq=np.zeros((D, W)),
+               dwk=np.zeros((D, W)), dwv=np.zeros((D, W)), dnorm_w=np.zeros(D))
+    rc = (lib or load()).oracle_gbla_head_backward(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(a), _ptr(og), D, 1, L, D, _ptr(wq), _ptr(wk),
+        _ptr(wv), W, _ptr(norm_w), float(eps), int(flags), _ptr(dy),
+        *[_ptr(out[n]) for n in ("dq", "dk", "dv", "da", "dog", "dwq", "dwk", "dwv",
+                                 "dnorm_w")])
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_head_backward rejected its arguments ({rc})")
+    return out
+
+
+def gbla_backward(q, k, v, gate, out_gate, conv_w, norm_w, dy, seq_lens=None,
+                  eps=RMS_EPS, flags=0, lib=None):
+    """Whole-core backward over [B, N, H, D] arrays: gradients of sum(dy * y).
+
+    Returns a dict: dq, dk, dv, dout_gate [B, N, H, D]; dgate [B, N, H]; dconv_w
+    [3, H, D, W]; dnorm_w [H, D].  Rows past seq_lens[b] are zero."""
+    q, k, v, og, dy = (_f64(t) for t in (q, k, v, out_gate, dy))
+    gate = _f64(gate); conv_w = _f64(conv_w); norm_w = _f64(norm_w)
+    B, N, H, D = q.shape
+    W = conv_w.shape[-1]
+    out = dict(dq=np.empty_like(q), dk=np.empty_like(q), dv=np.empty_like(q),
+               dgate=np.empty_like(gate), dout_gate=np.empty_like(q),
+               dconv_w=np.empty_like(conv_w), dnorm_w=np.empty_like(norm_w))
+    sl = None
+    if seq_lens is not None:
+        sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    rc = (lib or load()).oracle_gbla_backward(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(og), _ptr(conv_w), _ptr(norm_w),
+        sl.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)) if sl is not None else None,
+        B, H, N, D, W, float(eps), int(flags), _ptr(dy),
+        *[_ptr(out[n]) for n in ("dq", "dk", "dv", "dgate", "dout_gate", "dconv_w",
+                                 "dnorm_w")])
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_backward rejected its arguments ({rc})")
+    return out

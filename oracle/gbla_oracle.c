@@ -335,3 +335,239 @@ int oracle_gbla_forward(const double *q, const double *k, const double *v,
   pthread_mutex_destroy(&J.mu);
   return J.status;
 }
+
+/* ------------------------------------------------------------------------
+ * Backward of the layer core (training; the paper trains the model end to
+ * end, Sec. 3's training-speed table).  The paper states only the forward;
+ * the gradients below are the chain rule through the six forward steps,
+ * taken in reverse order, written out term by term:
+ *
+ *   6'. gated RMSNorm   y = O r w silu(og),  r = (mean_e O_e^2 + eps)^(-1/2)
+ *         dog_e = dy_e O_e r w_e silu'(og_e),  silu'(x) = s(x) (1 + x (1 - s(x)))
+ *         dw_e += dy_e O_e r silu(og_e)
+ *         u_e = dy_e w_e silu(og_e);  dO_e = r u_e - (r^3 / D) O_e sum_f u_f O_f
+ *   5'. readout         O = num / den,  num = S^T P,  den = P . z,  P = phi(q~)
+ *         dnum = dO / den;  dden = -(dO . O) / den
+ *         dP = S dnum + z dden;  dS += P dnum^T;  dz += P dden
+ *   4'. state           S = sum_j K^_j v~_j^T,  z = sum_j K^_j,  K^_j = g_j phi(k~_j)
+ *         dK^_j = dS v~_j + dz;  dv~_j = dS^T K^_j
+ *         dphi(k~_j) = g_j dK^_j;  dg_j = phi(k~_j) . dK^_j
+ *   3'. key gate        g = softmax(a):  da_j = g_j (dg_j - sum_i g_i dg_i)
+ *   2'. feature map     phi'(x) = 1 (x > 0), e^x (x <= 0)
+ *   1'. Conv1D          x~_t = sum_i w_i x_{t-(W-1)+i}:
+ *         dx_s = sum_i w_i dx~_{s+(W-1)-i} (terms with s+(W-1)-i < L),
+ *         dw_i += sum_t dx~_t x_{t-(W-1)+i}
+ * Ablation switches: identity conv (dx = dx~, no tap gradient), uniform gate
+ * (no logit gradient), no norm (dO = dy, no out_gate / weight gradient).
+ * ------------------------------------------------------------------------ */
+
+static double oracle_sigmoid(double x) { return 1.0 / (1.0 + exp(-x)); }
+
+/* Conv1D backward for one channel block: dx (stride ldx) from dxt [L][C]. */
+static void conv1d_backward(const double *x, const double *dxt, long L, int C,
+                            long ldx, const double *w, int W, double *dx,
+                            double *dw) {
+  for (long s = 0; s < L; ++s)
+    for (int c = 0; c < C; ++c) {
+      double acc = 0.0;
+      for (int i = 0; i < W; ++i) {
+        long t = s + (W - 1) - i;
+        if (t < L) acc += w[(long)c * W + i] * dxt[t * C + c];
+      }
+      dx[s * ldx + c] = acc;
+    }
+  for (int c = 0; c < C; ++c)
+    for (int i = 0; i < W; ++i) {
+      double acc = 0.0;
+      for (long t = 0; t < L; ++t) {
+        long s = t - (W - 1) + i;
+        if (s >= 0) acc += dxt[t * C + c] * x[s * ldx + c];
+      }
+      dw[(long)c * W + i] += acc;
+    }
+}
+
+static double phi_prime(double x) { return x > 0.0 ? 1.0 : exp(x); }
+
+/*
+ * One (batch, head): gradients of sum(dy * y) with respect to every input.
+ * Inputs as oracle_gbla_head plus dy (L rows at stride ld).  Outputs: dq, dk,
+ * dv, dog (L rows at stride ld), da (stride lda), and tap / norm-weight
+ * gradients ADDED to dwq, dwk, dwv [D][W] and dnw [D].  Returns 0 or -1.
+ */
+int oracle_gbla_head_backward(const double *q, const double *k, const double *v,
+                              const double *a, const double *og, long ld, long lda,
+                              long L, int D, const double *wq, const double *wk,
+                              const double *wv, int W, const double *norm_w,
+                              double eps, int flags, const double *dy, double *dq,
+                              double *dk, double *dv, double *da, double *dog,
+                              double *dwq, double *dwk, double *dwv, double *dnw) {
+  if (L < 0 || D <= 0 || W <= 0) return -1;
+  if (L == 0) return 0;
+  double *qt = xmalloc(sizeof(double) * L * D);
+  double *kt = xmalloc(sizeof(double) * L * D);
+  double *vt = xmalloc(sizeof(double) * L * D);
+  double *g = xmalloc(sizeof(double) * L);
+  double *S = xmalloc(sizeof(double) * D * D);
+  double *z = xmalloc(sizeof(double) * D);
+  double *O = xmalloc(sizeof(double) * L * D);
+  double *dO = xmalloc(sizeof(double) * L * D);
+  double *dS = xmalloc(sizeof(double) * D * D);
+  double *dz = xmalloc(sizeof(double) * D);
+  double *dqt = xmalloc(sizeof(double) * L * D);
+  double *dkt = xmalloc(sizeof(double) * L * D);
+  double *dvt = xmalloc(sizeof(double) * L * D);
+  double *dg = xmalloc(sizeof(double) * L);
+  double *P = xmalloc(sizeof(double) * D);
+  double *dnum = xmalloc(sizeof(double) * D);
+  double *Kh = xmalloc(sizeof(double) * D);
+  double *dKh = xmalloc(sizeof(double) * D);
+  double *den = xmalloc(sizeof(double) * L);
+
+  /* forward, steps 1-5 (Sec. 2.1 items 1 and 2) */
+  int rc = oracle_gbla_head(q, k, v, a, og, ld, lda, L, D, wq, wk, wv, W, norm_w,
+                            eps, flags, dO /* y, unused */, qt, kt, vt, g, S, z, O);
+  if (rc != 0) goto done;
+  for (long i = 0; i < L; ++i) {
+    double s = 0.0;
+    for (int d = 0; d < D; ++d) s += oracle_phi(qt[i * D + d]) * z[d];
+    den[i] = s;
+  }
+
+  /* 6'. gated RMSNorm */
+  for (long i = 0; i < L; ++i) {
+    const double *Oi = O + i * D, *dyi = dy + i * ld, *ogi = og + i * ld;
+    double *dOi = dO + i * D, *dogi = dog + i * ld;
+    if (flags & ORACLE_NO_NORM) {
+      for (int e = 0; e < D; ++e) {
+        dOi[e] = dyi[e];
+        dogi[e] = 0.0;
+      }
+      continue;
+    }
+    double ms = 0.0;
+    for (int e = 0; e < D; ++e) ms += Oi[e] * Oi[e];
+    ms /= (double)D;
+    const double r = 1.0 / sqrt(ms + eps);
+    double uo = 0.0;
+    for (int e = 0; e < D; ++e) {
+      const double sg = oracle_sigmoid(ogi[e]), si = ogi[e] * sg;
+      dogi[e] = dyi[e] * Oi[e] * r * norm_w[e] * sg * (1.0 + ogi[e] * (1.0 - sg));
+      dnw[e] += dyi[e] * Oi[e] * r * si;
+      uo += dyi[e] * norm_w[e] * si * Oi[e];
+    }
+    for (int e = 0; e < D; ++e) {
+      const double u = dyi[e] * norm_w[e] * oracle_silu(ogi[e]);
+      dOi[e] = r * u - (r * r * r / (double)D) * Oi[e] * uo;
+    }
+  }
+
+  /* 5'. readout */
+  memset(dS, 0, sizeof(double) * D * D);
+  memset(dz, 0, sizeof(double) * D);
+  for (long i = 0; i < L; ++i) {
+    const double *Oi = O + i * D, *dOi = dO + i * D;
+    for (int d = 0; d < D; ++d) P[d] = oracle_phi(qt[i * D + d]);
+    double dOO = 0.0;
+    for (int e = 0; e < D; ++e) {
+      dnum[e] = dOi[e] / den[i];
+      dOO += dOi[e] * Oi[e];
+    }
+    const double dden = -dOO / den[i];
+    for (int d = 0; d < D; ++d) {
+      double dP = z[d] * dden;
+      for (int e = 0; e < D; ++e) dP += S[d * D + e] * dnum[e];
+      dqt[i * D + d] = dP * phi_prime(qt[i * D + d]);
+      dz[d] += P[d] * dden;
+      for (int e = 0; e < D; ++e) dS[d * D + e] += P[d] * dnum[e];
+    }
+  }
+
+  /* 4'. state */
+  for (long j = 0; j < L; ++j) {
+    for (int d = 0; d < D; ++d) Kh[d] = g[j] * oracle_phi(kt[j * D + d]);
+    double dgj = 0.0;
+    for (int d = 0; d < D; ++d) {
+      double s = dz[d];
+      for (int e = 0; e < D; ++e) s += dS[d * D + e] * vt[j * D + e];
+      dKh[d] = s;
+      dkt[j * D + d] = g[j] * s * phi_prime(kt[j * D + d]);
+      dgj += oracle_phi(kt[j * D + d]) * s;
+    }
+    dg[j] = dgj;
+    for (int e = 0; e < D; ++e) {
+      double s = 0.0;
+      for (int d = 0; d < D; ++d) s += Kh[d] * dS[d * D + e];
+      dvt[j * D + e] = s;
+    }
+  }
+
+  /* 3'. key gate */
+  if (flags & ORACLE_NO_GATE) {
+    for (long j = 0; j < L; ++j) da[j * lda] = 0.0;
+  } else {
+    double gdg = 0.0;
+    for (long j = 0; j < L; ++j) gdg += g[j] * dg[j];
+    for (long j = 0; j < L; ++j) da[j * lda] = g[j] * (dg[j] - gdg);
+  }
+
+  /* 1'. Conv1D (step 2' was applied with dqt / dkt above) */
+  if (flags & ORACLE_NO_CONV) {
+    for (long t = 0; t < L; ++t)
+      for (int d = 0; d < D; ++d) {
+        dq[t * ld + d] = dqt[t * D + d];
+        dk[t * ld + d] = dkt[t * D + d];
+        dv[t * ld + d] = dvt[t * D + d];
+      }
+  } else {
+    conv1d_backward(q, dqt, L, D, ld, wq, W, dq, dwq);
+    conv1d_backward(k, dkt, L, D, ld, wk, W, dk, dwk);
+    conv1d_backward(v, dvt, L, D, ld, wv, W, dv, dwv);
+  }
+
+done:
+  free(qt); free(kt); free(vt); free(g); free(S); free(z); free(O); free(dO);
+  free(dS); free(dz); free(dqt); free(dkt); free(dvt); free(dg); free(P);
+  free(dnum); free(Kh); free(dKh); free(den);
+  return rc;
+}
+
+/*
+ * Whole-layer backward over [B, N, H, D] tensors (layout of
+ * oracle_gbla_forward).  Rows t >= seq_lens[b] of dq, dk, dv, dog and dgate
+ * are set to 0 (padding does not reach the outputs).  dconv_w [3][H][D][W]
+ * and dnorm_w [H][D] are overwritten with sums over the batch in batch order.
+ * (batch, head) pairs run one after another.
+ */
+int oracle_gbla_backward(const double *q, const double *k, const double *v,
+                         const double *gate, const double *og, const double *conv_w,
+                         const double *norm_w, const int32_t *seq_lens, long B, long H,
+                         long N, int D, int W, double eps, int flags, const double *dy,
+                         double *dq, double *dk, double *dv, double *dgate,
+                         double *dog, double *dconv_w, double *dnorm_w) {
+  if (B < 0 || H < 0 || N < 0 || D <= 0 || W <= 0) return -1;
+  const long ld = H * D;
+  memset(dq, 0, sizeof(double) * B * N * ld);
+  memset(dk, 0, sizeof(double) * B * N * ld);
+  memset(dv, 0, sizeof(double) * B * N * ld);
+  memset(dog, 0, sizeof(double) * B * N * ld);
+  memset(dgate, 0, sizeof(double) * B * N * H);
+  memset(dconv_w, 0, sizeof(double) * 3 * H * D * W);
+  memset(dnorm_w, 0, sizeof(double) * H * D);
+  for (long b = 0; b < B; ++b)
+    for (long h = 0; h < H; ++h) {
+      long L = seq_lens ? seq_lens[b] : N;
+      if (L < 0) L = 0;
+      if (L > N) L = N;
+      const long base = (b * N * H + h) * D, gbase = b * N * H + h;
+      int rc = oracle_gbla_head_backward(
+          q + base, k + base, v + base, gate + gbase, og + base, ld, H, L, D,
+          conv_w + ((0 * H + h) * D) * W, conv_w + ((1 * H + h) * D) * W,
+          conv_w + ((2 * H + h) * D) * W, W, norm_w + h * D, eps, flags, dy + base,
+          dq + base, dk + base, dv + base, dgate + gbase, dog + base,
+          dconv_w + ((0 * H + h) * D) * W, dconv_w + ((1 * H + h) * D) * W,
+          dconv_w + ((2 * H + h) * D) * W, dnorm_w + h * D);
+      if (rc != 0) return rc;
+    }
+  return 0;
+}
