@@ -126,6 +126,33 @@ gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
                                  gbla_stream_t stream);
 
 /*
+ * gbla_backward -- gradients of sum(dy * o) of the layer core (full core, no
+ * ablation) with respect to every input: the chain rule through the steps of
+ * Sec. 2.1 in reverse (gated RMSNorm, readout, state, key-gate softmax, phi,
+ * Conv1D).  Used to train the model end to end (the paper's training-speed
+ * comparison, Sec. 3).
+ *
+ * Inputs as gbla_forward (same layouts, dtype and validation), plus
+ *   dy        [B, N, H, D] dtype: gradient of the loss with respect to o.
+ * Outputs (caller-owned device buffers, 16-byte aligned, no aliasing with any
+ * input or with one another):
+ *   dq, dk, dv, dout_gate  [B, N, H, D] dtype;  dgate [B, N, H] dtype;
+ *   dconv_w [3, H, D, W] fp32 (q, k, v taps);   dnorm_w [H, D] fp32.
+ * Rows t >= L_b of dq, dk, dv, dout_gate and dgate are written as 0; dconv_w
+ * and dnorm_w are overwritten with sums over the batch.  The forward state is
+ * recomputed inside (nothing is kept from a forward call).  fp32 arithmetic;
+ * every sum runs in a fixed order (bitwise reproducible).  Asynchronous on
+ * `stream`; scratch comes from the library's stream-ordered pool
+ * (GBLA_ERR_ALLOC when it cannot).  Same error codes as gbla_forward.
+ */
+gbla_status gbla_backward(const void *q, const void *k, const void *v, const void *gate,
+                          const void *out_gate, const float *conv_w, const float *norm_w,
+                          const int32_t *seq_lens, const void *dy, void *dq, void *dk,
+                          void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                          float *dnorm_w, int B, int H, int N, int D, gbla_dtype dtype,
+                          gbla_stream_t stream);
+
+/*
  * gbla_state -- the sequence-global part of Sec. 2.1 item 2: Conv1D of k and
  * v, phi, the softmax key gate, and per (b, h) the state S = K^T V~ and the
  * normaliser z = K^T 1 with K^ = g * phi(K~), g the softmax over j < L_b.

@@ -287,6 +287,58 @@ gbla_status gbla_forward(const void *q, const void *k, const void *v,
                          N, D, dtype, GBLA_ALGO_AUTO, stream);
 }
 
+gbla_status gbla_backward(const void *q, const void *k, const void *v, const void *gate,
+                          const void *out_gate, const float *conv_w, const float *norm_w,
+                          const int32_t *seq_lens, const void *dy, void *dq, void *dk,
+                          void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                          float *dnorm_w, int B, int H, int N, int D, gbla_dtype dtype,
+                          gbla_stream_t stream) {
+  bool empty = false;
+  gbla_status s = check_dims(B, H, N, D, dtype, &empty);
+  if (s != GBLA_OK) return s;
+  if ((s = check_ptrs({q, k, v, gate, out_gate, conv_w, norm_w, dy, dq, dk, dv, dgate,
+                       dout_gate, dconv_w, dnorm_w})) != GBLA_OK)
+    return s;
+  if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
+  cudaStream_t st = (cudaStream_t)stream;
+  const size_t wbytes = sizeof(float) * 3 * H * D * kConvW, nbytes = sizeof(float) * H * D;
+  if (empty) {  // no tokens: the weight gradients are empty sums
+    if (H > 0 && (cudaMemsetAsync(dconv_w, 0, wbytes, st) != cudaSuccess ||
+                  cudaMemsetAsync(dnorm_w, 0, nbytes, st) != cudaSuccess))
+      return GBLA_ERR_CUDA;
+    return GBLA_OK;
+  }
+  const size_t bytes = (size_t)B * N * H * D * elem_bytes(dtype);
+  const size_t gbytes = (size_t)B * N * H * elem_bytes(dtype);
+  const Range outs[7] = {range_of(dq, bytes),     range_of(dk, bytes),
+                         range_of(dv, bytes),     range_of(dgate, gbytes),
+                         range_of(dout_gate, bytes), range_of(dconv_w, wbytes),
+                         range_of(dnorm_w, nbytes)};
+  const Range ins[9] = {range_of(q, bytes),      range_of(k, bytes),
+                        range_of(v, bytes),      range_of(out_gate, bytes),
+                        range_of(dy, bytes),     range_of(gate, gbytes),
+                        range_of(conv_w, wbytes), range_of(norm_w, nbytes),
+                        range_of(seq_lens, seq_lens ? sizeof(int32_t) * B : 0)};
+  for (int i = 0; i < 7; ++i) {
+    for (int j = 0; j < 9; ++j)
+      if (overlap(outs[i], ins[j])) return GBLA_ERR_INVALID_ARG;
+    for (int j = i + 1; j < 7; ++j)
+      if (overlap(outs[i], outs[j])) return GBLA_ERR_INVALID_ARG;
+  }
+  Problem p{B, H, N, D, dtype, seq_lens, 0u};
+  bool tc = use_tc(p, GBLA_ALGO_AUTO, &s);
+  if (s != GBLA_OK) return s;
+  const BwdLayout lay = bwd_layout(p);
+  Scratch scr;
+  if ((s = scr.alloc(sizeof(float) * lay.total, st)) != GBLA_OK) return s;
+  float *base = (float *)scr.ptr;
+  // the forward state S, z through the forward's own state path
+  if ((s = run_state(p, tc, k, v, gate, conv_w, base + lay.state, st)) != GBLA_OK) return s;
+  BwdArgs a{q, k, v, gate, out_gate, dy, conv_w, norm_w, dq, dk, dv, dgate, dout_gate,
+            dconv_w, dnorm_w};
+  return from_cuda(bwd_run(p, a, base, st));
+}
+
 gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
                               const void *gate, const void *out_gate,
                               const float *conv_w, const float *norm_w,

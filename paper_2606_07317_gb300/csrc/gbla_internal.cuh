@@ -54,6 +54,23 @@ cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
                        const float *conv_w, const float *norm_w,
                        const float *state, void *o, cudaStream_t st,
                        bool after_state = false);
+// ---- backward (CUDA cores, fp32 arithmetic; gbla_bwd.cu) ------------------
+struct BwdArgs {
+  const void *q, *k, *v, *gate, *out_gate, *dy;
+  const float *conv_w, *norm_w;
+  void *dq, *dk, *dv, *dgate, *dout_gate;
+  float *dconv_w, *dnorm_w;
+};
+// Scratch of the backward, in floats from one base: the forward state (filled
+// by the caller through the forward's state path), gate statistics, chunk
+// partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
+// gradient partials.
+struct BwdLayout {
+  size_t state, stats, qpart, red, dxt, wpart, total;
+};
+BwdLayout bwd_layout(const Problem &p);
+cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
+
 // Error bits set by tensor-core kernels whose bounded waits ran out (0 = none);
 // synchronous read of the current device, optionally clearing it.
 unsigned tc_device_error(bool reset);
