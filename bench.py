@@ -282,6 +282,73 @@ def bench_ours(args, ws, rank, local):
         torch.distributed.destroy_process_group()
 
 
+def bench_backward(args, ws, rank, local):
+    """--backward: gbla_backward (gradients of sum(dy * o) for every input) on the
+    workload; tokens/s and the whole-step roofline (bf16: q, k, v, out_gate, dy, gate
+    read and dq, dk, dv, dout_gate, dgate written, 18 D + 4 bytes per token-head)."""
+    from paper_2606_07317_gb300 import gbla
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(ws, "nccl")
+    gbla.load()
+    w = WORKLOADS[args.workload]
+    tokens = w.valid_tokens
+    inp0 = make_inputs(w, dev)
+    sets = [inp0, {k: (v.clone() if v is not None else None) for k, v in inp0.items()}]
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(w.seed + 1000)
+    dys = [torch.randn(inp0["q"].shape, generator=gen, device=dev).to(inp0["q"].dtype)
+           for _ in sets]
+    e_el = 2 if w.dtype == "bf16" else 4
+    step_bytes = w.valid_tokens * w.H * e_el * (9 * w.D + 2)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i):
+        s = sets[i % 2]
+        gbla.backward(s["q"], s["k"], s["v"], s["gate"], s["out_gate"], s["conv_w"],
+                      s["norm_w"], s["seq_lens"], dys[i % 2], stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize(dev)
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.1)
+    n0 = gbla.launch_count()
+    barrier(ws)
+    torch.cuda.synchronize(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(ws)
+    launches = gbla.launch_count() - n0
+    clocks = sampler.stop()
+    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, ws, dev)
+    peak, peak_kind = measured_peaks()
+    achieved = step_bytes / (ms * 1e-3) / 1e9
+    if rank == 0:
+        print(json.dumps({
+            "metric": "GBLA bwd tokens/sec (gradients of every input)", "value":
+            round(tokens * ws / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": w.dtype, "data": "synthetic (seeded N(0,1) inputs and dy)",
+            "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "D": w.D,
+                       "alg_bytes_per_step": step_bytes,
+                       "l2": "inputs larger than L2, two sets rotated"},
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                         "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                         "kernel": "whole backward step",
+                         "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"},
+            "gpu_launches": launches, "clocks": clocks}), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
 def bench_e2e(args, w, inp, dev, gbla, tokens, ws):
     host = {k: (v.cpu().pin_memory() if v is not None else None) for k, v in inp.items()}
     out = torch.empty_like(host["q"]).pin_memory()
@@ -423,12 +490,17 @@ def main(argv=None):
     ap.add_argument("--flags", type=int, default=0,
                     help="ablation (gbla_flags): 1 no Conv1D, 2 uniform gate, 4 no gated "
                          "RMSNorm, 7 BLA; 0 (default) is the full core")
+    ap.add_argument("--backward", action="store_true",
+                    help="time gbla_backward instead of the forward")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     ws, rank, local = dist_env()
     if args.impl == "reference":
         bench_reference(args, ws, rank)
+        return
+    if args.backward:
+        bench_backward(args, ws, rank, local)
         return
     bench_ours(args, ws, rank, local)
 
