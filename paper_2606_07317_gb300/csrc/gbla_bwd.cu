@@ -33,7 +33,7 @@
 namespace gbla {
 namespace {
 
-constexpr int kBG = 4;        // tokens in flight per block (one thread group each)
+constexpr int kNT = 256;      // threads per block of the token passes
 constexpr int kChunk = 256;   // tokens per block
 
 __device__ __forceinline__ float ldf(const float *p, size_t i) { return p[i]; }
@@ -62,20 +62,52 @@ __device__ __forceinline__ float warp_max(float x) {
   return x;
 }
 
-// Sum of x over the D threads of each token group (kBG groups side by side);
-// every thread of the block calls it.  red: kBG * (D / 32) floats of shared memory.
+// Thread layout of a token pass: thread (tq, c), c = tid % D the channel and
+// tokens tq * TPT .. tq * TPT + TPT - 1 of the batch.
 template <int D>
-__device__ __forceinline__ float group_sum(float x, float *red) {
-  constexpr int WPG = D / 32;
-  const int w = threadIdx.x >> 5, g = threadIdx.x / D;
-  x = warp_sum(x);
-  __syncthreads();  // red free from the previous use
-  if ((threadIdx.x & 31) == 0) red[w] = x;
-  __syncthreads();
-  float s = 0.f;
+struct Tok {
+  static constexpr int TB = 16;                  // tokens per batch
+  static constexpr int TQ = kNT / D;             // token quads per batch
+  static constexpr int TPT = TB / TQ;            // tokens per thread
+};
+
+// Sums over the D channels of each of this thread's TPT tokens (every thread
+// of the block calls it).  red: kNT / 32 * TPT floats of shared memory.
+template <int D, int TPT>
+__device__ __forceinline__ void chan_sum(float (&x)[TPT], float *red) {
+  constexpr int WPT = D / 32;  // warps per token quad (D >= 32)
+  const int w = threadIdx.x >> 5, tq = threadIdx.x / D;
 #pragma unroll
-  for (int i = 0; i < WPG; ++i) s += red[g * WPG + i];
-  return s;
+  for (int u = 0; u < TPT; ++u) x[u] = warp_sum(x[u]);
+  if (WPT == 1) return;
+  __syncthreads();  // red free from the previous use
+  if ((threadIdx.x & 31) == 0)
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) red[w * TPT + u] = x[u];
+  __syncthreads();
+#pragma unroll
+  for (int u = 0; u < TPT; ++u) {
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < WPT; ++i) s += red[(tq * WPT + i) * TPT + u];
+    x[u] = s;
+  }
+}
+
+// y[u] = sum_k X[k][t_u] M[k][c] for this thread's tokens t_u = tq * TPT + u:
+// X in shared memory as [D][TB] (k-major), M as [D][D] row-major.
+template <int D, int TPT>
+__device__ __forceinline__ void xm(const float *X, const float *M, int tq, int c,
+                                   float (&y)[TPT]) {
+#pragma unroll
+  for (int u = 0; u < TPT; ++u) y[u] = 0.f;
+#pragma unroll 4
+  for (int k = 0; k < D; ++k) {
+    const float m = M[k * D + c];
+    const float *xr = X + k * Tok<D>::TB + tq * TPT;
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) y[u] = fmaf(xr[u], m, y[u]);
+  }
 }
 
 // Causal Conv1D of one channel at token t: sum_i w[i] x[t - 3 + i], x[<0] = 0.
@@ -124,98 +156,147 @@ template <int D>
 constexpr int qrec() { return D * D + 2 * D; }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(kBG * D) bwd_query(
+__global__ void __launch_bounds__(kNT) bwd_query(
     const T *__restrict__ q, const T *__restrict__ og, const T *__restrict__ dy,
     const float *__restrict__ conv_w, const float *__restrict__ norm_w,
     const float *__restrict__ state, const int32_t *__restrict__ seq_lens, float eps,
     T *__restrict__ dog, float *__restrict__ dqt, float *__restrict__ part, int H, int N,
     int nck) {
-  constexpr int NT = kBG * D;
   constexpr int F = D * D + D;
-  constexpr int PE = D * D / NT;  // dS entries per thread
+  constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
+  constexpr int RB = D / 16;  // this thread's RB x RB block of dS (16 x 16 threads)
   extern __shared__ float sm[];
   float *S = sm, *St = S + D * D, *z = St + D * D;
-  float *sP = z + D, *sDn = sP + kBG * D, *sDd = sDn + kBG * D, *red = sDd + kBG;
+  float *Pk = z + D, *Pt = Pk + D * kTB, *Nk = Pt + kTB * D, *Nt = Nk + D * kTB;
+  float *sDd = Nt + kTB * D, *red = sDd + kTB;
   const int chunk = blockIdx.x, bh = blockIdx.y, b = bh / H, h = bh % H;
-  const int tid = threadIdx.x, g = tid / D, c = tid % D;
+  const int tid = threadIdx.x, tq = tid / D, c = tid % D;
   const int L = clamp_len(seq_lens, b, N);
-  const int t0 = chunk * kChunk, t1 = min(t0 + kChunk, N);
+  const int t0 = chunk * kChunk, t1 = min(t0 + kChunk, N), tv = min(t1, L);
   const float *st = state + (size_t)bh * F;
-  for (int i = tid; i < D * D; i += NT) {
+  for (int i = tid; i < D * D; i += kNT) {
     const float x = st[i];
     S[i] = x;
     St[(i % D) * D + i / D] = x;
   }
-  for (int i = tid; i < D; i += NT) z[i] = st[D * D + i];
+  for (int i = tid; i < D; i += kNT) z[i] = st[D * D + i];
   float wq[kConvW];
 #pragma unroll
   for (int i = 0; i < kConvW; ++i) wq[i] = conv_w[((size_t)h * D + c) * kConvW + i];
   const float nw = norm_w[(size_t)h * D + c];
   const size_t rs = (size_t)H * D;
   const T *qc = q + ((size_t)b * N * H + h) * D + c;
-  float dS[PE];
+  const int bi = tid / 16, bj = tid % 16;  // dS block rows bi * RB.., columns bj * RB..
+  float acc[RB][RB];
 #pragma unroll
-  for (int k = 0; k < PE; ++k) dS[k] = 0.f;
+  for (int i = 0; i < RB; ++i)
+#pragma unroll
+    for (int j = 0; j < RB; ++j) acc[i][j] = 0.f;
   float dz = 0.f, dnw = 0.f;
   __syncthreads();
-  for (int base = t0; base < t1; base += kBG) {
-    const int t = base + g;
-    const bool valid = t < min(t1, L);
-    const size_t row = (((size_t)b * N + t) * H + h) * D + c;
-    const float qt = valid ? conv_at(qc, rs, t, wq) : 0.f;
-    const float P = valid ? phi(qt) : 0.f;
-    sP[g * D + c] = P;
-    __syncthreads();
-    float num = 0.f, den = 0.f;
-#pragma unroll 8
-    for (int d = 0; d < D; ++d) {
-      const float pd = sP[g * D + d];
-      num = fmaf(pd, S[d * D + c], num);
-      den = fmaf(pd, z[d], den);
-    }
-    const float O = valid ? num / den : 0.f;
-    const float ogv = valid ? ldf(og, row) : 0.f, dyv = valid ? ldf(dy, row) : 0.f;
-    const float ms = group_sum<D>(O * O, red) / (float)D;
-    const float r = 1.f / sqrtf(ms + eps);
-    const float sg = 1.f / (1.f + expf(-ogv)), si = ogv * sg;
-    if (t < t1) stf(dog, row, valid ? dyv * O * r * nw * sg * (1.f + ogv * (1.f - sg)) : 0.f);
-    dnw = fmaf(dyv * O, r * si, dnw);
-    const float u = dyv * nw * si;
-    const float uo = group_sum<D>(u * O, red);
-    const float dO = r * u - (r * r * r / (float)D) * O * uo;
-    const float dnum = valid ? dO / den : 0.f;
-    const float dOO = group_sum<D>(dO * O, red);
-    const float dden = valid ? -dOO / den : 0.f;
-    sDn[g * D + c] = dnum;
-    if (c == 0) sDd[g] = dden;
-    __syncthreads();
-    float dP = z[c] * dden;
-#pragma unroll 8
-    for (int e = 0; e < D; ++e) dP = fmaf(St[e * D + c], sDn[g * D + e], dP);
-    if (t < t1) dqt[row] = valid ? dP * dphi(qt) : 0.f;
-    dz = fmaf(P, dden, dz);
+  for (int base = t0; base < t1; base += kTB) {
+    float qt[TPT], P[TPT], ogv[TPT], dyv[TPT], x[TPT];
 #pragma unroll
-    for (int k = 0; k < PE; ++k) {
-      const int ent = tid + k * NT, d = ent / D, e = ent % D;
-      float a = dS[k];
-#pragma unroll
-      for (int gg = 0; gg < kBG; ++gg) a = fmaf(sP[gg * D + d], sDn[gg * D + e], a);
-      dS[k] = a;
+    for (int u = 0; u < TPT; ++u) {
+      const int tl = tq * TPT + u, t = base + tl;
+      const bool valid = t < tv;
+      const size_t row = (((size_t)b * N + t) * H + h) * D + c;
+      qt[u] = valid ? conv_at(qc, rs, t, wq) : 0.f;
+      P[u] = valid ? phi(qt[u]) : 0.f;
+      ogv[u] = valid ? ldf(og, row) : 0.f;
+      dyv[u] = valid ? ldf(dy, row) : 0.f;
+      Pk[c * kTB + tl] = P[u];
+      Pt[tl * D + c] = P[u];
+      x[u] = P[u] * z[c];
     }
-    __syncthreads();  // sP, sDn reused by the next tokens
+    chan_sum<D, TPT>(x, red);  // den
+    float den[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) den[u] = x[u];
+    __syncthreads();  // Pk complete
+    float num[TPT];
+    xm<D, TPT>(Pk, S, tq, c, num);
+    float O[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      O[u] = base + tq * TPT + u < tv ? num[u] / den[u] : 0.f;
+      x[u] = O[u] * O[u];
+    }
+    chan_sum<D, TPT>(x, red);  // D * mean O^2
+    float r[TPT], uu[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int t = base + tq * TPT + u;
+      r[u] = 1.f / sqrtf(x[u] / (float)D + eps);
+      const float sg = 1.f / (1.f + expf(-ogv[u])), si = ogv[u] * sg;
+      if (t < t1) {
+        const size_t row = (((size_t)b * N + t) * H + h) * D + c;
+        stf(dog, row, dyv[u] * O[u] * r[u] * nw * sg * (1.f + ogv[u] * (1.f - sg)));
+      }
+      dnw = fmaf(dyv[u] * O[u], r[u] * si, dnw);
+      uu[u] = dyv[u] * nw * si;
+      x[u] = uu[u] * O[u];
+    }
+    chan_sum<D, TPT>(x, red);  // u . O
+    float dO[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      dO[u] = r[u] * uu[u] - (r[u] * r[u] * r[u] / (float)D) * O[u] * x[u];
+      x[u] = dO[u] * O[u];
+    }
+    chan_sum<D, TPT>(x, red);  // dO . O
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int tl = tq * TPT + u;
+      const bool valid = base + tl < tv;
+      const float dn = valid ? dO[u] / den[u] : 0.f;
+      Nk[c * kTB + tl] = dn;
+      Nt[tl * D + c] = dn;
+      if (c == 0) sDd[tl] = valid ? -x[u] / den[u] : 0.f;
+    }
+    __syncthreads();  // Nk, Nt, sDd complete
+    float dP[TPT];
+    xm<D, TPT>(Nk, St, tq, c, dP);  // dP_t[d] = sum_e dnum_t[e] S[d][e]
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int tl = tq * TPT + u, t = base + tl;
+      const float dd = sDd[tl];
+      if (t < t1) {
+        const size_t row = (((size_t)b * N + t) * H + h) * D + c;
+        dqt[row] = (dP[u] + z[c] * dd) * dphi(qt[u]) * (t < tv ? 1.f : 0.f);
+      }
+      dz = fmaf(P[u], dd, dz);
+    }
+    // dS += P^T dnum over the batch's tokens
+#pragma unroll 2
+    for (int tl = 0; tl < kTB; ++tl) {
+      float pv[RB], nv[RB];
+#pragma unroll
+      for (int i = 0; i < RB; ++i) {
+        pv[i] = Pt[tl * D + bi * RB + i];
+        nv[i] = Nt[tl * D + bj * RB + i];
+      }
+#pragma unroll
+      for (int i = 0; i < RB; ++i)
+#pragma unroll
+        for (int j = 0; j < RB; ++j) acc[i][j] = fmaf(pv[i], nv[j], acc[i][j]);
+    }
+    __syncthreads();  // the batch's shared arrays are rewritten next
   }
-  // partial record: dS by entry; dz and dnw summed over the token groups in order
   float *rec = part + ((size_t)bh * nck + chunk) * qrec<D>();
 #pragma unroll
-  for (int k = 0; k < PE; ++k) rec[tid + k * NT] = dS[k];
-  sP[g * D + c] = dz;
-  sDn[g * D + c] = dnw;
+  for (int i = 0; i < RB; ++i)
+#pragma unroll
+    for (int j = 0; j < RB; ++j) rec[(bi * RB + i) * D + bj * RB + j] = acc[i][j];
+  // dz and dnw: sum over the token quads in order
+  Pk[tq * D + c] = dz;
+  Nk[tq * D + c] = dnw;
   __syncthreads();
   if (tid < D) {
     float a = 0.f, w = 0.f;
-    for (int gg = 0; gg < kBG; ++gg) {
-      a += sP[gg * D + tid];
-      w += sDn[gg * D + tid];
+    for (int i = 0; i < Tok<D>::TQ; ++i) {
+      a += Pk[i * D + tid];
+      w += Nk[i * D + tid];
     }
     rec[D * D + tid] = a;
     rec[D * D + D + tid] = w;
@@ -223,55 +304,53 @@ __global__ void __launch_bounds__(kBG * D) bwd_query(
 }
 
 // ---------------------------------------------------------------- state reduction
-// red record per (b, h): dS [D][D], dz [D], c.
+// red record per (b, h): dS [D][D], dz [D] (chunk partials summed in chunk order).
 template <int D>
 __global__ void __launch_bounds__(256) bwd_reduce_state(const float *__restrict__ part,
-                                                        const float *__restrict__ state,
                                                         float *__restrict__ red, int nck) {
   constexpr int F = D * D + D;
-  const int bh = blockIdx.x;
-  __shared__ float wred[8];
-  float cs = 0.f;
-  for (int i = threadIdx.x; i < F; i += 256) {
-    float a = 0.f;
-    for (int ch = 0; ch < nck; ++ch) a += part[((size_t)bh * nck + ch) * qrec<D>() + i];
-    red[(size_t)bh * (F + 1) + i] = a;
-    cs = fmaf(a, state[(size_t)bh * F + i], cs);
-  }
-  cs = warp_sum(cs);
-  if ((threadIdx.x & 31) == 0) wred[threadIdx.x >> 5] = cs;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int i = 0; i < 8; ++i) s += wred[i];
-    red[(size_t)bh * (F + 1) + F] = s;
-  }
+  const int bh = blockIdx.y, i = blockIdx.x * 256 + threadIdx.x;
+  if (i >= F) return;
+  float a = 0.f;
+  for (int ch = 0; ch < nck; ++ch) a += part[((size_t)bh * nck + ch) * qrec<D>() + i];
+  red[(size_t)bh * F + i] = a;
 }
 
 // ---------------------------------------------------------------- key pass
 template <typename T, int D>
-__global__ void __launch_bounds__(kBG * D) bwd_key(
+__global__ void __launch_bounds__(kNT) bwd_key(
     const T *__restrict__ k, const T *__restrict__ v, const T *__restrict__ gate,
     const float *__restrict__ conv_w, const float2 *__restrict__ stats,
-    const float *__restrict__ red, const int32_t *__restrict__ seq_lens, T *__restrict__ dgate,
-    float *__restrict__ dkt, float *__restrict__ dvt, int H, int N) {
-  constexpr int NT = kBG * D;
+    const float *__restrict__ state, const float *__restrict__ red,
+    const int32_t *__restrict__ seq_lens, T *__restrict__ dgate, float *__restrict__ dkt,
+    float *__restrict__ dvt, int H, int N) {
   constexpr int F = D * D + D;
+  constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   extern __shared__ float sm[];
   float *dS = sm, *dSt = dS + D * D, *dz = dSt + D * D;
-  float *sK = dz + D, *sV = sK + kBG * D, *rd = sV + kBG * D;
+  float *Kk = dz + D, *Vk = Kk + D * kTB, *rd = Vk + D * kTB;
   const int chunk = blockIdx.x, bh = blockIdx.y, b = bh / H, h = bh % H;
-  const int tid = threadIdx.x, g = tid / D, c = tid % D;
+  const int tid = threadIdx.x, tq = tid / D, c = tid % D;
   const int L = clamp_len(seq_lens, b, N);
-  const int t0 = chunk * kChunk, t1 = min(t0 + kChunk, N);
-  const float *rr = red + (size_t)bh * (F + 1);
-  for (int i = tid; i < D * D; i += NT) {
+  const int t0 = chunk * kChunk, t1 = min(t0 + kChunk, N), tv = min(t1, L);
+  const float *rr = red + (size_t)bh * F;
+  const float *st = state + (size_t)bh * F;
+  float cs = 0.f;  // c = <dS, S> + <dz, z>, this thread's part
+  for (int i = tid; i < F; i += kNT) {
     const float x = rr[i];
-    dS[i] = x;
-    dSt[(i % D) * D + i / D] = x;
+    if (i < D * D) {
+      dS[i] = x;
+      dSt[(i % D) * D + i / D] = x;
+    } else {
+      dz[i - D * D] = x;
+    }
+    cs = fmaf(x, st[i], cs);
   }
-  for (int i = tid; i < D; i += NT) dz[i] = rr[D * D + i];
-  const float cval = rr[F];
+  cs = warp_sum(cs);
+  if ((tid & 31) == 0) rd[tid >> 5] = cs;
+  __syncthreads();
+  float cval = 0.f;
+  for (int i = 0; i < kNT / 32; ++i) cval += rd[i];
   const float2 gs = stats[bh];
   float wk[kConvW], wv[kConvW];
 #pragma unroll
@@ -282,48 +361,68 @@ __global__ void __launch_bounds__(kBG * D) bwd_key(
   const size_t rs = (size_t)H * D;
   const T *kc = k + ((size_t)b * N * H + h) * D + c;
   const T *vc = v + ((size_t)b * N * H + h) * D + c;
-  __syncthreads();
-  for (int base = t0; base < t1; base += kBG) {
-    const int t = base + g;
-    const bool valid = t < min(t1, L);
-    const size_t row = (((size_t)b * N + t) * H + h) * D + c;
-    const float kt = valid ? conv_at(kc, rs, t, wk) : 0.f;
-    const float vt = valid ? conv_at(vc, rs, t, wv) : 0.f;
-    const float gj = valid ? expf(ldf(gate, ((size_t)b * N + t) * H + h) - gs.x) / gs.y : 0.f;
-    const float pk = valid ? phi(kt) : 0.f;
-    sK[g * D + c] = gj * pk;
-    sV[g * D + c] = vt;
-    __syncthreads();
-    float dK = dz[c], dvv = 0.f;
-#pragma unroll 8
-    for (int e = 0; e < D; ++e) {
-      dK = fmaf(dSt[e * D + c], sV[g * D + e], dK);
-      dvv = fmaf(sK[g * D + e], dS[e * D + c], dvv);
+  __syncthreads();  // rd read before chan_sum reuses it
+  for (int base = t0; base < t1; base += kTB) {
+    float kt[TPT], pk[TPT], g[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int tl = tq * TPT + u, t = base + tl;
+      const bool valid = t < tv;
+      kt[u] = valid ? conv_at(kc, rs, t, wk) : 0.f;
+      const float vt = valid ? conv_at(vc, rs, t, wv) : 0.f;
+      g[u] = valid ? expf(ldf(gate, ((size_t)b * N + t) * H + h) - gs.x) / gs.y : 0.f;
+      pk[u] = valid ? phi(kt[u]) : 0.f;
+      Kk[c * kTB + tl] = g[u] * pk[u];
+      Vk[c * kTB + tl] = vt;
     }
-    if (t < t1) {
-      dkt[row] = valid ? gj * dK * dphi(kt) : 0.f;
-      dvt[row] = valid ? dvv : 0.f;
+    __syncthreads();  // Kk, Vk complete
+    float dK[TPT], dvv[TPT];
+    xm<D, TPT>(Vk, dSt, tq, c, dK);   // dK^_t[d] = sum_e dS[d][e] v~_t[e]
+    xm<D, TPT>(Kk, dS, tq, c, dvv);   // dv~_t[e] = sum_d K^_t[d] dS[d][e]
+    float x[TPT];
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int t = base + tq * TPT + u;
+      dK[u] += dz[c];
+      if (t < t1) {
+        const size_t row = (((size_t)b * N + t) * H + h) * D + c;
+        const bool valid = t < tv;
+        dkt[row] = valid ? g[u] * dK[u] * dphi(kt[u]) : 0.f;
+        dvt[row] = valid ? dvv[u] : 0.f;
+      }
+      x[u] = pk[u] * dK[u];
     }
-    const float dg = group_sum<D>(pk * dK, rd);
-    if (c == 0 && t < t1) stf(dgate, ((size_t)b * N + t) * H + h, valid ? gj * (dg - cval) : 0.f);
-    __syncthreads();  // sK, sV reused by the next tokens
+    chan_sum<D, TPT>(x, rd);  // dg_t
+#pragma unroll
+    for (int u = 0; u < TPT; ++u) {
+      const int t = base + tq * TPT + u;
+      if (c == 0 && t < t1)
+        stf(dgate, ((size_t)b * N + t) * H + h, t < tv ? g[u] * (x[u] - cval) : 0.f);
+    }
+    __syncthreads();  // Kk, Vk rewritten next
   }
 }
 
 // ---------------------------------------------------------------- Conv1D backward
-// Stream s (0 q, 1 k, 2 v): dx_t = sum_i w_i dx~_{t+3-i} (t + 3 - i < L), and the
-// chunk partials of dw_i = sum_t dx~_t x_{t-3+i} for the D channels of (b, h).
+// Stream s = blockIdx.z (0 q, 1 k, 2 v): dx_t = sum_i w_i dx~_{t+3-i} (t + 3 - i
+// < L) and the chunk partials of dw_i = sum_t dx~_t x_{t-3+i} for the D channels
+// of (b, h).  Thread (run, c) walks kChunk / (kNT / D) consecutive tokens of
+// channel c with sliding windows of dx~ and x.
 template <typename T, int D>
-__global__ void __launch_bounds__(kBG * D) bwd_conv(
-    const T *__restrict__ x, const float *__restrict__ dxt, const float *__restrict__ conv_w,
-    const int32_t *__restrict__ seq_lens, T *__restrict__ dx, float *__restrict__ wpart, int s,
-    int H, int N, int nck) {
-  constexpr int NT = kBG * D;
-  __shared__ float sw[kBG][D][kConvW];
-  const int chunk = blockIdx.x, bh = blockIdx.y, b = bh / H, h = bh % H;
-  const int tid = threadIdx.x, g = tid / D, c = tid % D;
+__global__ void __launch_bounds__(kNT) bwd_conv(
+    const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v,
+    const float *__restrict__ dxt, const float *__restrict__ conv_w,
+    const int32_t *__restrict__ seq_lens, T *__restrict__ dq, T *__restrict__ dk,
+    T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck) {
+  constexpr int RUNS = kNT / D, RL = kChunk / RUNS;
+  __shared__ float sw[RUNS][D][kConvW];
+  const int chunk = blockIdx.x, bh = blockIdx.y, s = blockIdx.z, b = bh / H, h = bh % H;
+  const int tid = threadIdx.x, run = tid / D, c = tid % D;
+  const T *x = s == 0 ? q : (s == 1 ? k : v);
+  T *dx = s == 0 ? dq : (s == 1 ? dk : dv);
+  const float *dxs = dxt + (size_t)s * ((size_t)gridDim.y / H) * N * H * D;
   const int L = clamp_len(seq_lens, b, N);
-  const int t0 = chunk * kChunk, t1 = min(t0 + kChunk, N);
+  const int ta = chunk * kChunk + run * RL, tb = min(ta + RL, N);
   float w[kConvW], dw[kConvW];
 #pragma unroll
   for (int i = 0; i < kConvW; ++i) {
@@ -332,33 +431,54 @@ __global__ void __launch_bounds__(kBG * D) bwd_conv(
   }
   const size_t rs = (size_t)H * D;
   const size_t col = ((size_t)b * N * H + h) * D + c;
-  for (int t = t0 + g; t < t1; t += kBG) {
-    float a = 0.f;
-    if (t < L) {
+  // windows: d[i] = dx~_{t+i}, xw[i] = x_{t-3+i} (i = 0..3); four tokens a step,
+  // the next four tokens' values loaded together
+  float d[kConvW], xw[kConvW];
 #pragma unroll
-      for (int i = 0; i < kConvW; ++i) {
-        const int u = t + (kConvW - 1) - i;
-        if (u < L) a = fmaf(w[i], dxt[col + (size_t)u * rs], a);
-      }
-      const float d = dxt[col + (size_t)t * rs];
+  for (int i = 0; i < kConvW; ++i) {
+    const int u = ta + i, s2 = ta - (kConvW - 1) + i;
+    d[i] = u < L ? dxs[col + (size_t)u * rs] : 0.f;
+    xw[i] = (s2 >= 0 && s2 < L) ? ldf(x, col + (size_t)s2 * rs) : 0.f;
+  }
+  for (int t = ta; t < tb; t += 4) {
+    float dd[8], xx[8];  // dx~_{t..t+7}, x_{t-3..t+4}
 #pragma unroll
-      for (int i = 0; i < kConvW; ++i) {
-        const int u = t - (kConvW - 1) + i;
-        if (u >= 0) dw[i] = fmaf(d, ldf(x, col + (size_t)u * rs), dw[i]);
+    for (int i = 0; i < 4; ++i) {
+      dd[i] = d[i];
+      xx[i] = xw[i];
+      const int un = t + 4 + i, sn = t + 1 + i;
+      dd[4 + i] = un < L ? dxs[col + (size_t)un * rs] : 0.f;
+      xx[4 + i] = sn < L ? ldf(x, col + (size_t)sn * rs) : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int tj = t + j;
+      if (tj < tb) {
+        float a = 0.f;
+        if (tj < L) {
+#pragma unroll
+          for (int i = 0; i < kConvW; ++i) a = fmaf(w[i], dd[j + kConvW - 1 - i], a);
+#pragma unroll
+          for (int i = 0; i < kConvW; ++i) dw[i] = fmaf(dd[j], xx[j + i], dw[i]);
+        }
+        stf(dx, col + (size_t)tj * rs, a);
       }
     }
-    stf(dx, col + (size_t)t * rs, a);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      d[i] = dd[4 + i];
+      xw[i] = xx[4 + i];
+    }
   }
 #pragma unroll
-  for (int i = 0; i < kConvW; ++i) sw[g][c][i] = dw[i];
+  for (int i = 0; i < kConvW; ++i) sw[run][c][i] = dw[i];
   __syncthreads();
-  if (tid < D * kConvW) {
-    const int cc = tid / kConvW, i = tid % kConvW;
+  for (int j = tid; j < D * kConvW; j += kNT) {
+    const int cc = j / kConvW, i = j % kConvW;
     float a = 0.f;
-    for (int gg = 0; gg < kBG; ++gg) a += sw[gg][cc][i];
-    wpart[(((size_t)s * gridDim.y + bh) * nck + chunk) * D * kConvW + tid] = a;
+    for (int r = 0; r < RUNS; ++r) a += sw[r][cc][i];
+    wpart[(((size_t)s * gridDim.y + bh) * nck + chunk) * D * kConvW + j] = a;
   }
-  (void)NT;
 }
 
 // ---------------------------------------------------------------- weight reductions
@@ -403,34 +523,32 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   cudaError_t e;
   bwd_gate_stats<T><<<BH, 256, 0, st>>>((const T *)a.gate, p.seq_lens, stats, H, N);
   count_launch();
-  const size_t smq = sizeof(float) * (2 * D * D + D + 2 * kBG * D + kBG + kBG * D / 32);
+  constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
+  const size_t smq = sizeof(float) * (2 * D * D + D + 4 * D * kTB + kTB + kNT / 32 * TPT);
   auto kq = bwd_query<T, D>;
   if ((e = cudaFuncSetAttribute(kq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smq)) !=
       cudaSuccess)
     return e;
-  kq<<<dim3(nck, BH), kBG * D, smq, st>>>((const T *)a.q, (const T *)a.out_gate,
-                                         (const T *)a.dy, a.conv_w, a.norm_w, state, p.seq_lens,
-                                         kRmsEps, (T *)a.dout_gate, dxt, qpart, H, N, nck);
+  kq<<<dim3(nck, BH), kNT, smq, st>>>((const T *)a.q, (const T *)a.out_gate, (const T *)a.dy,
+                                      a.conv_w, a.norm_w, state, p.seq_lens, kRmsEps,
+                                      (T *)a.dout_gate, dxt, qpart, H, N, nck);
   count_launch();
-  bwd_reduce_state<D><<<BH, 256, 0, st>>>(qpart, state, red, nck);
+  constexpr int F = D * D + D;
+  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(qpart, red, nck);
   count_launch();
-  const size_t smk = sizeof(float) * (2 * D * D + D + 2 * kBG * D + kBG * D / 32);
+  const size_t smk = sizeof(float) * (2 * D * D + D + 2 * D * kTB + kNT / 32 * TPT);
   auto kk = bwd_key<T, D>;
   if ((e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smk)) !=
       cudaSuccess)
     return e;
-  kk<<<dim3(nck, BH), kBG * D, smk, st>>>((const T *)a.k, (const T *)a.v, (const T *)a.gate,
-                                         a.conv_w, stats, red, p.seq_lens, (T *)a.dgate,
-                                         dxt + plane, dxt + 2 * plane, H, N);
+  kk<<<dim3(nck, BH), kNT, smk, st>>>((const T *)a.k, (const T *)a.v, (const T *)a.gate,
+                                      a.conv_w, stats, state, red, p.seq_lens, (T *)a.dgate,
+                                      dxt + plane, dxt + 2 * plane, H, N);
   count_launch();
-  const void *xs[3] = {a.q, a.k, a.v};
-  void *dxs[3] = {a.dq, a.dk, a.dv};
-  for (int s = 0; s < 3; ++s) {
-    bwd_conv<T, D><<<dim3(nck, BH), kBG * D, 0, st>>>((const T *)xs[s], dxt + s * plane,
-                                                      a.conv_w, p.seq_lens, (T *)dxs[s], wpart,
-                                                      s, H, N, nck);
-    count_launch();
-  }
+  bwd_conv<T, D><<<dim3(nck, BH, 3), kNT, 0, st>>>(
+      (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
+      (T *)a.dk, (T *)a.dv, wpart, H, N, nck);
+  count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
   bwd_reduce_w<D><<<(nw + 255) / 256, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
                                                      nck);
