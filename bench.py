@@ -81,12 +81,13 @@ def measured_peaks():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the sources of the forward's tensor-core kernels (the ones whose DRAM
+    traffic profiles/traffic.json records)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_07317_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + f.read())
+    for name in ("gbla_tc.cu", "gbla_sm100.cuh", "gbla_internal.cuh"):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
 
 
