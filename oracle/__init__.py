@@ -9,6 +9,11 @@ follows Sec. 2 (bidirectional linear attention, Eq. bla) and Sec. 2.1 (GBLA:
 Conv1D, key gating, gated RMSNorm) of the paper.  This module only compiles
 it with gcc and marshals numpy arrays into it.
 
+The layer front end (``gbla_project``: the X-space Conv1D and the stacked
+Q, K, V, R and w_g projections of Sec. 2.1 items 1-3) and the whole layer
+(``gbla_layer``: front end, then the core with its Conv1D off) are pinned by
+the ``pin_project_*`` and ``pin_layer_conv_commutes`` checks.
+
 Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
 against library routines, closed forms, the quadratic (L x L) form and
 invariants.  The paper's own unstated choices (phi, eps, conv tap order, the
@@ -86,6 +91,10 @@ def _declare(lib):
                                          ctypes.c_long, ctypes.c_long, ctypes.c_long,
                                          ctypes.c_int, ctypes.c_int, ctypes.c_double,
                                          ctypes.c_int, _dp] + [_dp] * 7
+    lib.oracle_gbla_project.restype = ctypes.c_int
+    lib.oracle_gbla_project.argtypes = [_dp, _dp, _dp, ctypes.POINTER(ctypes.c_int32),
+                                        ctypes.c_long, ctypes.c_long, ctypes.c_int,
+                                        ctypes.c_int, ctypes.c_long, ctypes.c_int] + [_dp] * 6
     lib.oracle_gbla_forward.restype = ctypes.c_int
     lib.oracle_gbla_forward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
                                         ctypes.POINTER(ctypes.c_int32),
@@ -264,3 +273,53 @@ def gbla_backward(q, k, v, gate, out_gate, conv_w, norm_w, dy, seq_lens=None,
     if rc != 0:
         raise ValueError(f"oracle_gbla_backward rejected its arguments ({rc})")
     return out
+
+
+def gbla_project(x, conv_x, w, H, D, seq_lens=None, absdot=False, lib=None):
+    """Layer front end (Sec. 2.1 items 1-3): X~ = Conv1D(X) over the d channels of
+    x [B, N, d] with taps conv_x [d, W], then the stacked projections w [F, d],
+    F = 4 H D + H (rows: W_Q, W_K, W_V, W_R per head and dim, then w_g per head).
+
+    Returns a dict: q, k, v, out_gate [B, N, H, D], gate [B, N, H] (rows past
+    seq_lens[b] are NaN) and, when asked, absdot [B, N, F] = sum_c |x~_c w_fc|.
+    """
+    x = _f64(x); conv_x = _f64(conv_x); w = _f64(w)
+    B, N, d = x.shape
+    F = 4 * H * D + H
+    if w.shape != (F, d) or conv_x.shape[0] != d:
+        raise ValueError("gbla_project: w must be [4*H*D + H, d] and conv_x [d, W]")
+    out = {n: np.full((B, N, H, D), np.nan) for n in ("q", "k", "v", "out_gate")}
+    out["gate"] = np.full((B, N, H), np.nan)
+    ad = np.full((B, N, F), np.nan) if absdot else None
+    sl = None
+    if seq_lens is not None:
+        sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    rc = (lib or load()).oracle_gbla_project(
+        _ptr(x), _ptr(conv_x), _ptr(w),
+        sl.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)) if sl is not None else None,
+        B, N, d, conv_x.shape[1], H, D,
+        *[_ptr(out[n]) for n in ("q", "k", "v", "out_gate", "gate")], _ptr(ad))
+    if rc != 0:
+        raise ValueError(f"oracle_gbla_project rejected its arguments ({rc})")
+    if absdot:
+        out["absdot"] = ad
+    return out
+
+
+def gbla_layer(x, conv_x, w, norm_w, H, D, seq_lens=None, store=None, eps=RMS_EPS,
+               lib=None):
+    """Whole GBLA layer of Sec. 2.1 from the embedded sequence x [B, N, d]: the
+    front end (gbla_project) followed by the core with its Conv1D off (the
+    Conv1D already ran on X).  `store`, when given, maps each intermediate
+    array to the values the layer keeps between the two halves (for example
+    rounding to the storage dtype); None keeps them in double precision.
+    Returns y [B, N, H, D] (rows past seq_lens[b] are NaN)."""
+    pr = gbla_project(x, conv_x, w, H, D, seq_lens=seq_lens, lib=lib)
+    if store is not None:
+        pr = {n: store(a) for n, a in pr.items()}
+    B, N = pr["q"].shape[:2]
+    zeros_conv = np.zeros((3, H, D, CONV_W))  # unused with NO_CONV
+    inter = {n: np.nan_to_num(pr[n], nan=0.0) for n in pr}
+    return gbla_forward(inter["q"], inter["k"], inter["v"], inter["gate"],
+                        inter["out_gate"], zeros_conv, norm_w, seq_lens=seq_lens,
+                        eps=eps, flags=NO_CONV, lib=lib)

@@ -37,6 +37,10 @@
  *   - RmsNorm(O)_d = O_d / sqrt(mean_d O_d^2 + eps) * w_d, weight per head.
  *   - SiLU(x) = x * sigmoid(x).
  *
+ * The layer front end (oracle_gbla_project, at the end of this file) takes
+ * the embedded sequence X instead: it runs the Conv1D on X, as Sec. 2.1 item 1
+ * states it, and then the per-head projections Q, K, V, W_R and w_g.
+ *
  * Ablation switches follow the paper's ablation table (W/o Conv1D, W/o key
  * gating, W/o gated RMSNorm; all three off gives plain BLA, Eq. bla).
  */
@@ -569,5 +573,66 @@ int oracle_gbla_backward(const double *q, const double *k, const double *v,
           dconv_w + ((2 * H + h) * D) * W, dnorm_w + h * D);
       if (rc != 0) return rc;
     }
+  return 0;
+}
+
+/* ------------------------------------------------------------------------
+ * Layer front end: the X-space Conv1D and the per-head projections.
+ *
+ *   X~ = Conv1D(X)                            (Sec. 2.1 item 1)
+ *   Q = X~ W_Q,  K = X~ W_K,  V = X~ W_V      (Sec. 2.1 item 1)
+ *   gate logits = X~ w_g                      (Sec. 2.1 item 2)
+ *   out-gate input = X~ W_R                   (Sec. 2.1 item 3)
+ * with one set of matrices per head (the multi-head paragraph of Sec. 2.1).
+ *
+ * Readings: the Conv1D on X is depthwise over the d channels, causal, with
+ * the tap order of oracle_conv1d (tap W-1 multiplies the current token), no
+ * bias and no activation.  The weights of all heads and projections are
+ * stacked into one matrix w [F][d], F = 4 H D + H, one row per output feature
+ * over the d input channels (row f gives output f = sum_c x~[c] w[f][c]):
+ * rows s*H*D + h*D + e for stream s = Q, K, V, R (W_R) and head h, dim e, then
+ * rows 4 H D + h for w_g of head h.
+ *
+ * x [B][N][d]; conv_x [d][W]; q, k, v, og [B][N][H][D]; gate [B][N][H].
+ * Rows t >= seq_lens[b] are not written (they are padding, and no valid row
+ * reads them: the Conv1D is causal).  absdot, when given, is [B][N][F] and
+ * receives sum_c |x~[c] w[f][c]| per output: the scale of any rounding error
+ * in computing the output (the error bound of a dot product is proportional
+ * to it).
+ * ------------------------------------------------------------------------ */
+int oracle_gbla_project(const double *x, const double *conv_x, const double *w,
+                        const int32_t *seq_lens, long B, long N, int d, int W, long H,
+                        int D, double *q, double *k, double *v, double *og, double *gate,
+                        double *absdot) {
+  if (B < 0 || N < 0 || d <= 0 || W <= 0 || H <= 0 || D <= 0) return -1;
+  const long HD = H * (long)D;
+  const long F = 4 * HD + H;
+  double *xt = (double *)xmalloc(sizeof(double) * (size_t)(N > 0 ? N : 1) * d);
+  double *streams[4] = {q, k, v, og};
+  for (long b = 0; b < B; ++b) {
+    long L = seq_lens ? seq_lens[b] : N;
+    if (L < 0) L = 0;
+    if (L > N) L = N;
+    oracle_conv1d(x + b * N * d, L, d, d, conv_x, W, xt);
+    for (long t = 0; t < L; ++t) {
+      const double *xr = xt + t * d;
+      for (long f = 0; f < F; ++f) {
+        const double *wr = w + f * d;
+        double acc = 0.0, mag = 0.0;
+        for (int c = 0; c < d; ++c) {
+          acc += xr[c] * wr[c];
+          mag += fabs(xr[c] * wr[c]);
+        }
+        if (f < 4 * HD) {
+          const long s = f / HD, col = f % HD;
+          streams[s][(b * N + t) * HD + col] = acc;
+        } else {
+          gate[(b * N + t) * H + (f - 4 * HD)] = acc;
+        }
+        if (absdot) absdot[(b * N + t) * F + f] = mag;
+      }
+    }
+  }
+  free(xt);
   return 0;
 }

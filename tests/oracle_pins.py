@@ -334,4 +334,131 @@ def pin_denominator_positive(lib):
     assert np.all(np.isfinite(inter["O"]))
 
 
+# --- layer front end: X-space Conv1D and stacked projections (Sec. 2.1) ----
+
+def _project_inputs(rng, B, N, d, H, D):
+    x = rng.standard_normal((B, N, d))
+    conv_x = 0.5 * rng.standard_normal((d, W))
+    w = rng.standard_normal((4 * H * D + H, d)) / np.sqrt(d)
+    return x, conv_x, w
+
+
+def _np_conv_x(x, conv_x):
+    """Causal depthwise Conv1D of every channel through numpy's convolution:
+    y[t] = sum_i w[i] x[t - (W-1) + i] is the full convolution with the
+    reversed taps, cut to the first N outputs."""
+    B, N, d = x.shape
+    y = np.empty_like(x)
+    for b in range(B):
+        for c in range(d):
+            y[b, :, c] = np.convolve(x[b, :, c], conv_x[c, ::-1])[:N]
+    return y
+
+
+def _split(y, H, D):
+    B, N, _ = y.shape
+    HD = H * D
+    parts = [y[..., s * HD:(s + 1) * HD].reshape(B, N, H, D) for s in range(4)]
+    return dict(q=parts[0], k=parts[1], v=parts[2], out_gate=parts[3], gate=y[..., 4 * HD:])
+
+
+def pin_project_library(lib):
+    """Front end = numpy convolution of each X channel, then one matrix product
+    with the stacked weights, split into Q, K, V, R (per head) and w_g."""
+    rng = _rng(70)
+    for (B, N, d, H, D) in [(2, 13, 8, 2, 3), (1, 5, 16, 3, 4), (3, 2, 4, 1, 2)]:
+        x, conv_x, w = _project_inputs(rng, B, N, d, H, D)
+        got = oracle.gbla_project(x, conv_x, w, H, D, lib=lib)
+        want = _split(_np_conv_x(x, conv_x) @ w.T, H, D)
+        for n in want:
+            np.testing.assert_allclose(got[n], want[n], rtol=0, atol=1e-12, err_msg=n)
+
+
+def pin_project_identity_taps(lib):
+    """Conv1D taps (0, ..., 0, 1) are the identity, leaving plain projections."""
+    rng = _rng(71)
+    B, N, d, H, D = 2, 7, 6, 2, 2
+    x, _, w = _project_inputs(rng, B, N, d, H, D)
+    taps = np.zeros((d, W)); taps[:, W - 1] = 1.0
+    got = oracle.gbla_project(x, taps, w, H, D, lib=lib)
+    want = _split(x @ w.T, H, D)
+    for n in want:
+        np.testing.assert_allclose(got[n], want[n], rtol=0, atol=1e-12, err_msg=n)
+
+
+def pin_project_causal_window(lib):
+    """A change of x at position t0 reaches exactly the outputs at t0 .. t0+W-1
+    (causal, width-W receptive field)."""
+    rng = _rng(72)
+    B, N, d, H, D = 1, 16, 5, 2, 3
+    x, conv_x, w = _project_inputs(rng, B, N, d, H, D)
+    a = oracle.gbla_project(x, conv_x, w, H, D, lib=lib)
+    t0 = 6
+    x2 = x.copy(); x2[0, t0] += rng.standard_normal(d)
+    b = oracle.gbla_project(x2, conv_x, w, H, D, lib=lib)
+    for n in a:
+        diff = np.abs(a[n] - b[n]).reshape(N, -1).max(axis=1)
+        assert np.all(diff[:t0] == 0) and np.all(diff[t0 + W:] == 0), n
+        assert np.all(diff[t0:t0 + W] > 0), n
+
+
+def pin_project_padding(lib):
+    """Rows past seq_lens[b] are not written, and the valid rows equal an
+    unpadded run of that length whatever the padding holds."""
+    rng = _rng(73)
+    B, N, d, H, D = 2, 12, 6, 2, 2
+    x, conv_x, w = _project_inputs(rng, B, N, d, H, D)
+    sl = np.array([12, 5], np.int32)
+    a = oracle.gbla_project(x, conv_x, w, H, D, seq_lens=sl, lib=lib)
+    x2 = x.copy(); x2[1, 5:] = 1e30
+    b = oracle.gbla_project(x2, conv_x, w, H, D, seq_lens=sl, lib=lib)
+    c = oracle.gbla_project(x[1:2, :5], conv_x, w, H, D, lib=lib)
+    for n in a:
+        assert np.all(np.isnan(a[n][1, 5:])), n
+        assert not np.any(np.isnan(a[n][1, :5])) and not np.any(np.isnan(a[n][0])), n
+        np.testing.assert_array_equal(b[n][1, :5], a[n][1, :5])
+        np.testing.assert_array_equal(c[n][0], a[n][1, :5])
+
+
+def pin_project_absdot(lib):
+    """absdot = |X~| |W|^T (the magnitude sum of every output's terms): equal
+    to the output itself when every term is nonnegative, never below |output|."""
+    rng = _rng(74)
+    B, N, d, H, D = 1, 9, 7, 2, 2
+    x, conv_x, w = _project_inputs(rng, B, N, d, H, D)
+    r = oracle.gbla_project(x, conv_x, w, H, D, absdot=True, lib=lib)
+    xt = _np_conv_x(x, conv_x)
+    np.testing.assert_allclose(r["absdot"], np.abs(xt) @ np.abs(w).T, rtol=1e-13, atol=0)
+    y = _split(xt @ w.T, H, D)
+    full = np.concatenate([y[n].reshape(B, N, -1) for n in ("q", "k", "v", "out_gate", "gate")],
+                          axis=-1)
+    assert np.all(r["absdot"] >= np.abs(full) - 1e-12)
+    xp, cp, wp = np.abs(x), np.abs(conv_x), np.abs(w)
+    rp = oracle.gbla_project(xp, cp, wp, H, D, absdot=True, lib=lib)
+    yp = np.concatenate([rp[n].reshape(B, N, -1) for n in ("q", "k", "v", "out_gate", "gate")],
+                        axis=-1)
+    np.testing.assert_allclose(rp["absdot"], yp, rtol=1e-13, atol=0)
+
+
+def pin_layer_conv_commutes(lib):
+    """With one Conv1D kernel shared by all channels, convolving X before the
+    projections (Sec. 2.1 item 1, the layer) equals convolving the projected
+    q, k, v inside the core: Conv1D(X) W = Conv1D(X W).  Gate and out-gate
+    inputs come from X~ in both."""
+    rng = _rng(75)
+    B, N, d, H, D = 2, 21, 6, 2, 3
+    x, _, w = _project_inputs(rng, B, N, d, H, D)
+    shared = 0.5 * rng.standard_normal(W)
+    conv_x = np.tile(shared, (d, 1))
+    norm_w = 1.0 + 0.02 * rng.standard_normal((H, D))
+    sl = np.array([21, 14], np.int32)
+    y_layer = oracle.gbla_layer(x, conv_x, w, norm_w, H, D, seq_lens=sl, lib=lib)
+    plain = _split(x @ w.T, H, D)                      # projections of the raw X
+    conved = _split(_np_conv_x(x, conv_x) @ w.T, H, D)  # gate / out-gate from X~
+    conv_w = np.tile(shared, (3, H, D, 1))
+    y_core = oracle.gbla_forward(plain["q"], plain["k"], plain["v"], conved["gate"],
+                                 conved["out_gate"], conv_w, norm_w, seq_lens=sl, lib=lib)
+    np.testing.assert_allclose(y_layer, y_core, rtol=0, atol=1e-10)
+
+
 ALL_PINS = [v for k_, v in sorted(globals().items()) if k_.startswith("pin_")]

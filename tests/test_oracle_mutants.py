@@ -44,6 +44,19 @@ MUTANTS = [
     ("driver_norm_head", "J->norm_w + h * D", "J->norm_w"),
     ("driver_len_unclamped", "if (L > J->N) L = J->N;", "if (L > J->N) L = J->N + 0; L = J->N;"),
     ("quadratic_gate_on_query", "A[i * L + j] = g[j] * s;", "A[i * L + j] = g[i] * s;"),
+    ("project_stream_interleaved", "const long s = f / HD, col = f % HD;",
+     "const long s = f % 4, col = f / 4;"),
+    ("project_gate_column", "gate[(b * N + t) * H + (f - 4 * HD)] = acc;",
+     "gate[(b * N + t) * H + (f - 4 * HD + 1) % H] = acc;"),
+    ("project_weight_transposed", "acc += xr[c] * wr[c];",
+     "acc += xr[c] * w[(long)c * F + f];"),
+    ("project_skips_conv", "const double *xr = xt + t * d;",
+     "const double *xr = x + (b * N + t) * d;"),
+    ("project_batch_offset", "oracle_conv1d(x + b * N * d, L, d, d, conv_x, W, xt);",
+     "oracle_conv1d(x, L, d, d, conv_x, W, xt);"),
+    ("project_writes_padding", "for (long t = 0; t < L; ++t) {\n      const double *xr",
+     "for (long t = 0; t < N; ++t) {\n      const double *xr"),
+    ("project_absdot_signed", "mag += fabs(xr[c] * wr[c]);", "mag += xr[c] * wr[c];"),
 ]
 
 
