@@ -36,7 +36,8 @@ if ROOT not in sys.path:
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-from paper_2606_07317_gb300.workloads import HEADLINE, WORKLOADS, make_inputs  # noqa: E402
+from paper_2606_07317_gb300.workloads import (HEADLINE, WORKLOADS, make_inputs,  # noqa: E402
+                                              make_layer_inputs)
 
 METRIC = "GBLA fwd tokens/sec and % of GB300 HBM roofline at N=32768, 1 GPU"
 UNIT = "tokens/s"
@@ -350,6 +351,106 @@ def bench_backward(args, ws, rank, local):
         torch.distributed.destroy_process_group()
 
 
+def measured_bf16_peak():
+    """Dense bf16 tensor peak (TFLOP/s): the burst figure of MEASURED_PEAKS.json for a
+    kernel timed on its own, else the fallback."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        if "bf16_tflops" in d:
+            return float(d["bf16_tflops"]), "measured"
+    return 1900.0, "fallback"
+
+
+def bench_layer(args, ws, rank, local):
+    """--layer: the whole GBLA layer from the embedded sequence X (gbla_layer_forward:
+    X-space Conv1D and the stacked projections on tensor cores, then the core with its
+    Conv1D off) on the workload's B, N, H, D with model width d = H D; tokens/s of the
+    layer, and the front-end kernel (gbla_project) against the bf16 tensor peak:
+    2 d (4 H D + H) flops per token."""
+    from paper_2606_07317_gb300 import gbla
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(ws, "nccl")
+    gbla.load()
+    w = WORKLOADS[args.workload]
+    d = args.model_dim or w.H * w.D
+    F = 4 * w.H * w.D + w.H
+    tokens = w.valid_tokens
+    sets = [make_layer_inputs(w.B, w.N, d, w.H, w.D, seed=w.seed + i, seq_lens=w.seq_lens,
+                              device=dev) for i in range(2)]
+    outs = [torch.empty((w.B, w.N, w.H, w.D), dtype=torch.bfloat16, device=dev) for _ in sets]
+    pouts = [{n: torch.empty((w.B, w.N, w.H, w.D), dtype=torch.bfloat16, device=dev)
+              for n in ("q", "k", "v", "out_gate")} for _ in sets]
+    for po in pouts:
+        po["gate"] = torch.empty((w.B, w.N, w.H), dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def layer_step(i):
+        s = sets[i % 2]
+        gbla.layer_forward(s["x"], s["conv_x"], s["w_proj"], s["norm_w"], w.H, w.D,
+                           seq_lens=s["seq_lens"], out=outs[i % 2], stream=stream)
+
+    def project_step(i):
+        s = sets[i % 2]
+        gbla.project(s["x"], s["conv_x"], s["w_proj"], w.H, w.D, seq_lens=s["seq_lens"],
+                     out=pouts[i % 2], stream=stream)
+
+    def timed(fn, steps):
+        for i in range(args.warmup):
+            fn(i)
+        torch.cuda.synchronize(dev)
+        barrier(ws)
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for i in range(steps):
+            fn(i)
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(ws)
+        return max_over_ranks(ev0.elapsed_time(ev1) / steps, ws, dev)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.1)
+    n0 = gbla.launch_count()
+    ms = timed(layer_step, args.steps)
+    launches = gbla.launch_count() - n0
+    ms_proj = timed(project_step, args.steps)
+    clocks = sampler.stop()
+    assert gbla.device_error() == 0
+    flops = 2.0 * d * F * tokens
+    tf_peak, tf_kind = measured_bf16_peak()
+    achieved = flops / (ms_proj * 1e-3) / 1e12
+    hbm_peak, _ = measured_peaks()
+    proj_bytes = tokens * 2 * (d + F)
+    if rank == 0:
+        print(json.dumps({
+            "metric": "GBLA layer fwd tokens/sec (X-space Conv1D + fused projections + core)",
+            "value": round(tokens * ws / (ms * 1e-3), 1), "unit": "tokens/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 6),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic (seeded N(0,1) x, N(0,1/d) weights)",
+            "config": {"workload": w.name + f"_layer_d{d}", "B": w.B, "H": w.H, "N": w.N,
+                       "D": w.D, "d": d, "F": F, "tokens_per_step": tokens,
+                       "l2": "two input sets rotated; each step writes 4 B N H D bf16 "
+                             "intermediates (%.0f MB, above L2)" % (8 * tokens * w.H * w.D / 1e6)},
+            "roofline": {"bound": "tensor", "achieved": round(achieved, 1), "peak": tf_peak,
+                         "unit": "TFLOP/s", "frac": round(achieved / tf_peak, 4),
+                         "traffic": None, "kernel": "tc_project_kernel",
+                         "peak_source": f"{tf_kind} (MEASURED_PEAKS.json bf16_tflops, burst)",
+                         "flops_per_launch": flops, "launch_ms": round(ms_proj, 5),
+                         "hbm_gbs": round(proj_bytes / (ms_proj * 1e-3) / 1e9, 1),
+                         "hbm_frac": round(proj_bytes / (ms_proj * 1e-3) / 1e9 / hbm_peak, 4),
+                         "phases_ms": {"project": round(ms_proj, 5),
+                                       "core": round(ms - ms_proj, 5)}},
+            "gpu_launches": launches, "clocks": clocks}), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
 def bench_e2e(args, w, inp, dev, gbla, tokens, ws):
     host = {k: (v.cpu().pin_memory() if v is not None else None) for k, v in inp.items()}
     out = torch.empty_like(host["q"]).pin_memory()
@@ -493,6 +594,10 @@ def main(argv=None):
                          "RMSNorm, 7 BLA; 0 (default) is the full core")
     ap.add_argument("--backward", action="store_true",
                     help="time gbla_backward instead of the forward")
+    ap.add_argument("--layer", action="store_true",
+                    help="time the whole layer from X (gbla_layer_forward) and its front end")
+    ap.add_argument("--model-dim", type=int, default=0,
+                    help="--layer: model width d (default H * D)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -502,6 +607,9 @@ def main(argv=None):
         return
     if args.backward:
         bench_backward(args, ws, rank, local)
+        return
+    if args.layer:
+        bench_layer(args, ws, rank, local)
         return
     bench_ours(args, ws, rank, local)
 

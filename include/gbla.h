@@ -153,6 +153,54 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
                           gbla_stream_t stream);
 
 /*
+ * gbla_project -- the layer front end: Sec. 2.1 item 1 (X~ = Conv1D(X), then
+ * Q = X~ W_Q, K = X~ W_K, V = X~ W_V), item 2 (gate logits X~ w_g) and item 3
+ * (output-gate input X~ W_R), with one set of matrices per head (the
+ * multi-head paragraph of Sec. 2.1), as one tensor-core contraction.
+ *
+ *   x        [B, N, d] dtype  the embedded sequence X (token-major).
+ *   conv_x   [d, W] fp32      depthwise causal Conv1D taps on X; tap W-1
+ *                             multiplies the current token, history before
+ *                             t = 0 is zero; no bias, no activation.
+ *   w_proj   [F, d] dtype     stacked projection weights, F = 4 H D + H, one
+ *                             row per output feature over the d inputs (the
+ *                             nn.Linear weight layout): rows s*H*D + h*D + e
+ *                             give dim e of head h of stream s = Q, K, V, R
+ *                             (W_R), rows 4*H*D + h give w_g of head h.
+ *   seq_lens device [B] int32 or NULL, as gbla_forward.
+ *   q, k, v, out_gate [B, N, H, D] dtype and gate [B, N, H] dtype: outputs,
+ *                             laid out as gbla_forward's inputs.  Rows t >= L_b
+ *                             are not written.
+ * bf16 only (GBLA_FP32 returns GBLA_ERR_UNSUPPORTED): X~ is computed in fp32
+ * and rounded once to bf16, the products are summed in fp32, each output is
+ * rounded once to bf16.  Limits: d a multiple of 64 in [64, 512], H * D a
+ * multiple of 64, H <= 256, D in {32, 64, 128}; otherwise
+ * GBLA_ERR_UNSUPPORTED.  All pointers 16-byte aligned device pointers
+ * (caller-owned); the outputs must not overlap any input or one another
+ * (GBLA_ERR_INVALID_ARG).  Needs an sm_103 GPU (GBLA_ERR_UNSUPPORTED
+ * otherwise).  Asynchronous on `stream`; allocates nothing.
+ */
+gbla_status gbla_project(const void *x, const float *conv_x, const void *w_proj,
+                         const int32_t *seq_lens, void *q, void *k, void *v,
+                         void *out_gate, void *gate, int B, int N, int d, int H,
+                         int D, gbla_dtype dtype, gbla_stream_t stream);
+
+/*
+ * gbla_layer_forward -- the whole GBLA layer of Sec. 2.1 from X: gbla_project,
+ * then the core (gbla_forward_variant with GBLA_FLAG_NO_CONV, since the
+ * Conv1D already ran on X) with its Conv1D off.  Arguments as gbla_project
+ * plus norm_w [H, D] fp32 and the output o [B, N, H, D] dtype (rows t < L_b
+ * written).  q, k, v, out_gate and gate live in scratch from the library's
+ * stream-ordered pool, stored in dtype between the two halves (GBLA_ERR_ALLOC
+ * when the pool cannot provide 8 B N H D + 2 B N H bytes).  o must not overlap
+ * an input.  Same limits and error codes as gbla_project.
+ */
+gbla_status gbla_layer_forward(const void *x, const float *conv_x, const void *w_proj,
+                               const float *norm_w, const int32_t *seq_lens, void *o,
+                               int B, int N, int d, int H, int D, gbla_dtype dtype,
+                               gbla_stream_t stream);
+
+/*
  * gbla_state -- the sequence-global part of Sec. 2.1 item 2: Conv1D of k and
  * v, phi, the softmax key gate, and per (b, h) the state S = K^T V~ and the
  * normaliser z = K^T 1 with K^ = g * phi(K~), g the softmax over j < L_b.

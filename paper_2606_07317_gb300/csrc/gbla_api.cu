@@ -189,7 +189,10 @@ void gbla_release(void) {
 
 uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
-uint32_t gbla_device_error(int reset) { return tc_device_error(reset != 0); }
+uint32_t gbla_device_error(int reset) {
+  const unsigned a = tc_device_error(reset != 0), b = project_device_error(reset != 0);
+  return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu) ? 0xFFFFFFFFu : (a | b);
+}
 
 const char *gbla_last_cuda_error(void) { return cudaGetErrorString(t_last_cuda_error); }
 
@@ -337,6 +340,87 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
   BwdArgs a{q, k, v, gate, out_gate, dy, conv_w, norm_w, dq, dk, dv, dgate, dout_gate,
             dconv_w, dnorm_w};
   return from_cuda(bwd_run(p, a, base, st));
+}
+
+// Validation shared by gbla_project and gbla_layer_forward.
+static gbla_status check_project(const void *x, const float *conv_x, const void *w,
+                                 const int32_t *seq_lens, int B, int N, int d, int H, int D,
+                                 gbla_dtype dtype, bool *empty) {
+  gbla_status s = check_dims(B, H, N, D, dtype, empty);
+  if (s != GBLA_OK) return s;
+  if (d < 0) return GBLA_ERR_INVALID_ARG;
+  if (dtype != GBLA_BF16) return GBLA_ERR_UNSUPPORTED;
+  if ((s = check_ptrs({x, conv_x, w})) != GBLA_OK) return s;
+  if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
+  if (*empty) return GBLA_OK;
+  ProjProblem pp{B, N, d, H, D, seq_lens};
+  if (!project_supports(pp)) return GBLA_ERR_UNSUPPORTED;
+  return GBLA_OK;
+}
+
+gbla_status gbla_project(const void *x, const float *conv_x, const void *w_proj,
+                         const int32_t *seq_lens, void *q, void *k, void *v,
+                         void *out_gate, void *gate, int B, int N, int d, int H,
+                         int D, gbla_dtype dtype, gbla_stream_t stream) {
+  bool empty = false;
+  gbla_status s = check_project(x, conv_x, w_proj, seq_lens, B, N, d, H, D, dtype, &empty);
+  if (s != GBLA_OK) return s;
+  if ((s = check_ptrs({q, k, v, out_gate, gate})) != GBLA_OK) return s;
+  if (empty) return GBLA_OK;
+  const size_t tok = (size_t)B * N;
+  const size_t sb = tok * H * D * 2, gb = tok * H * 2;
+  const Range outs[5] = {range_of(q, sb), range_of(k, sb), range_of(v, sb),
+                         range_of(out_gate, sb), range_of(gate, gb)};
+  const Range ins[4] = {range_of(x, tok * d * 2), range_of(conv_x, sizeof(float) * d * kConvW),
+                        range_of(w_proj, ((size_t)4 * H * D + H) * d * 2),
+                        range_of(seq_lens, seq_lens ? sizeof(int32_t) * B : 0)};
+  for (int i = 0; i < 5; ++i) {
+    for (int j = 0; j < 4; ++j)
+      if (overlap(outs[i], ins[j])) return GBLA_ERR_INVALID_ARG;
+    for (int j = i + 1; j < 5; ++j)
+      if (overlap(outs[i], outs[j])) return GBLA_ERR_INVALID_ARG;
+  }
+  ProjProblem pp{B, N, d, H, D, seq_lens};
+  return from_cuda(tc_project(pp, x, conv_x, w_proj, q, k, v, out_gate, gate,
+                              (cudaStream_t)stream));
+}
+
+gbla_status gbla_layer_forward(const void *x, const float *conv_x, const void *w_proj,
+                               const float *norm_w, const int32_t *seq_lens, void *o,
+                               int B, int N, int d, int H, int D, gbla_dtype dtype,
+                               gbla_stream_t stream) {
+  bool empty = false;
+  gbla_status s = check_project(x, conv_x, w_proj, seq_lens, B, N, d, H, D, dtype, &empty);
+  if (s != GBLA_OK) return s;
+  if ((s = check_ptrs({norm_w, o})) != GBLA_OK) return s;
+  if (empty) return GBLA_OK;
+  const size_t tok = (size_t)B * N;
+  const size_t sb = tok * H * D * 2, gb = tok * H * 2;
+  const Range out = range_of(o, sb);
+  if (overlap(out, range_of(x, tok * d * 2)) ||
+      overlap(out, range_of(conv_x, sizeof(float) * d * kConvW)) ||
+      overlap(out, range_of(w_proj, ((size_t)4 * H * D + H) * d * 2)) ||
+      overlap(out, range_of(norm_w, sizeof(float) * H * D)) ||
+      (seq_lens && overlap(out, range_of(seq_lens, sizeof(int32_t) * B))))
+    return GBLA_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  Problem p{B, H, N, D, dtype, seq_lens, (uint32_t)GBLA_FLAG_NO_CONV};
+  bool tc = use_tc(p, GBLA_ALGO_AUTO, &s);
+  if (s != GBLA_OK) return s;
+  // q, k, v, out_gate, gate, then the state, in one scratch block
+  const size_t off_g = 4 * sb, off_s = round_up(off_g + gb, 256);
+  const size_t st_bytes = sizeof(float) * state_floats(D) * B * H;
+  Scratch scr;
+  if ((s = scr.alloc(off_s + st_bytes, st)) != GBLA_OK) return s;
+  char *base = (char *)scr.ptr;
+  void *q = base, *k = base + sb, *v = base + 2 * sb, *og = base + 3 * sb, *gate = base + off_g;
+  float *state = (float *)(base + off_s);
+  ProjProblem pp{B, N, d, H, D, seq_lens};
+  if ((s = from_cuda(tc_project(pp, x, conv_x, w_proj, q, k, v, og, gate, st))) != GBLA_OK)
+    return s;
+  // the core with its Conv1D off (the taps are never read)
+  if ((s = run_state(p, tc, k, v, gate, nullptr, state, st)) != GBLA_OK) return s;
+  return run_readout(p, tc, q, og, nullptr, norm_w, state, o, st, true);
 }
 
 gbla_status gbla_forward_host(const void *q, const void *k, const void *v,

@@ -71,6 +71,18 @@ struct BwdLayout {
 BwdLayout bwd_layout(const Problem &p);
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
 
+// ---- layer front end (tcgen05; gbla_project.cu): bf16 ----------------------
+struct ProjProblem {
+  int B, N, d, H, D;
+  const int32_t *seq_lens;  // device [B] or nullptr
+};
+// d a multiple of 64 in [64, 512], H * D a multiple of 64, H <= 256, sm_103.
+bool project_supports(const ProjProblem &pp);
+cudaError_t tc_project(const ProjProblem &pp, const void *x, const float *conv_x,
+                       const void *w, void *q, void *k, void *v, void *og, void *gate,
+                       cudaStream_t st);
+unsigned project_device_error(bool reset);
+
 // Error bits set by tensor-core kernels whose bounded waits ran out (0 = none);
 // synchronous read of the current device, optionally clearing it.
 unsigned tc_device_error(bool reset);

@@ -28,7 +28,8 @@ EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_bac
             "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
-            "gbla_state_static_scratch", "gbla_device_error", "gbla_last_cuda_error"]
+            "gbla_state_static_scratch", "gbla_device_error", "gbla_last_cuda_error",
+            "gbla_project", "gbla_layer_forward"]
 
 _lock = threading.Lock()
 _lib = None
@@ -70,6 +71,10 @@ def load(path: str | None = None):
         lib.gbla_forward_variant.restype = _i
         lib.gbla_backward.argtypes = [_vp] * 16 + [_i] * 5 + [_vp]
         lib.gbla_backward.restype = _i
+        lib.gbla_project.argtypes = [_vp] * 9 + [_i] * 6 + [_vp]
+        lib.gbla_project.restype = _i
+        lib.gbla_layer_forward.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
+        lib.gbla_layer_forward.restype = _i
         lib.gbla_forward_host.argtypes = fwd + [_vp]
         lib.gbla_forward_host.restype = _i
         lib.gbla_state.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
@@ -194,6 +199,37 @@ def backward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, stream=None)
         B, H, N, D, _dtype_code(q), _stream(stream))
     _check(st, "gbla_backward")
     return g
+
+
+def project(x, conv_x, w_proj, H, D, seq_lens=None, out=None, stream=None) -> dict:
+    """Layer front end (gbla_project): X~ = Conv1D(x) over the d channels of x [B, N, d],
+    then the stacked projections w_proj [4 H D + H, d] (rows W_Q, W_K, W_V, W_R per head
+    and dim, then w_g per head).  Returns q, k, v, out_gate [B, N, H, D] and gate
+    [B, N, H] (rows past seq_lens are not written; `out` may supply the five tensors)."""
+    B, N, d = x.shape
+    if out is None:
+        out = {n: x.new_empty((B, N, H, D)) for n in ("q", "k", "v", "out_gate")}
+        out["gate"] = x.new_empty((B, N, H))
+    st = load().gbla_project(
+        _ptr(x), _ptr(conv_x), _ptr(w_proj), _ptr(seq_lens), _ptr(out["q"]), _ptr(out["k"]),
+        _ptr(out["v"]), _ptr(out["out_gate"]), _ptr(out["gate"]), B, N, d, H, D,
+        _dtype_code(x), _stream(stream))
+    _check(st, "gbla_project")
+    return out
+
+
+def layer_forward(x, conv_x, w_proj, norm_w, H, D, seq_lens=None, out=None,
+                  stream=None) -> torch.Tensor:
+    """Whole GBLA layer from x [B, N, d] (gbla_layer_forward): front end, then the core
+    with its Conv1D off.  Returns o [B, N, H, D]."""
+    B, N, d = x.shape
+    if out is None:
+        out = x.new_empty((B, N, H, D))
+    st = load().gbla_layer_forward(
+        _ptr(x), _ptr(conv_x), _ptr(w_proj), _ptr(norm_w), _ptr(seq_lens), _ptr(out),
+        B, N, d, H, D, _dtype_code(x), _stream(stream))
+    _check(st, "gbla_layer_forward")
+    return out
 
 
 def forward_default(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, out, stream=None):

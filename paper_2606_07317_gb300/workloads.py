@@ -111,3 +111,31 @@ def make_inputs(w: Workload, device="cpu") -> dict:
     out["seq_lens"] = (torch.tensor(w.seq_lens, dtype=torch.int32, device=dev)
                        if w.seq_lens is not None else None)
     return out
+
+
+# --- layer front end (X-space Conv1D and stacked projections) ---------------
+#
+# Recipe: a ``torch.Generator`` on the target device seeded with `seed` draws,
+# in this order, the embedded sequence x ``[B, N, d]`` from N(0, 1) (rounded to
+# nearest bf16), the Conv1D taps on X ``[d, 4]`` from N(0, 1/4) (fp32), the
+# stacked projection weights ``[4 H D + H, d]`` from N(0, 1/d) (rounded to
+# bf16; an output then has unit variance, as with a standard linear-layer
+# initialisation) and the RMSNorm weight ``[H, D]`` as 1 + N(0, 0.02^2).
+# The default model width is d = H * D (512 for the 8 x 64 headline core).
+
+def make_layer_inputs(B, N, d, H, D, seed=0, seq_lens=None, device="cpu") -> dict:
+    dev = torch.device(device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+
+    def normal(shape, std=1.0):
+        t = torch.randn(shape, generator=g, device=dev, dtype=torch.float32)
+        return t.mul_(std) if std != 1.0 else t
+
+    out = {"x": normal((B, N, d)).to(torch.bfloat16)}
+    out["conv_x"] = normal((d, CONV_WIDTH), std=0.5)
+    out["w_proj"] = normal((4 * H * D + H, d), std=1.0 / math.sqrt(d)).to(torch.bfloat16)
+    out["norm_w"] = normal((H, D), std=0.02).add_(1.0)
+    out["seq_lens"] = (torch.tensor(list(seq_lens), dtype=torch.int32, device=dev)
+                       if seq_lens is not None else None)
+    return out
