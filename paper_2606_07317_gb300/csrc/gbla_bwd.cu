@@ -94,19 +94,51 @@ __device__ __forceinline__ void chan_sum(float (&x)[TPT], float *red) {
   }
 }
 
+// Loads n consecutive floats of shared memory (n = 2, 4 or 8; p aligned to
+// min(n, 4) floats) with 8- or 16-byte loads.
+template <int n>
+__device__ __forceinline__ void ld_vec(const float *p, float (&v)[n]) {
+  if constexpr (n == 2) {
+    const float2 a = *reinterpret_cast<const float2 *>(p);
+    v[0] = a.x;
+    v[1] = a.y;
+  } else {
+#pragma unroll
+    for (int i = 0; i < n; i += 4) {
+      const float4 a = *reinterpret_cast<const float4 *>(p + i);
+      v[i] = a.x;
+      v[i + 1] = a.y;
+      v[i + 2] = a.z;
+      v[i + 3] = a.w;
+    }
+  }
+}
+
 // y[u] = sum_k X[k][t_u] M[k][c] for this thread's tokens t_u = tq * TPT + u:
-// X in shared memory as [D][TB] (k-major), M as [D][D] row-major.
+// X in shared memory as [D][TB] (k-major), M as [D][D] row-major.  The TPT
+// tokens of a thread are one vector load per k and the products go through
+// packed fp32 FMAs (two per instruction, each rounded as fmaf).
 template <int D, int TPT>
 __device__ __forceinline__ void xm(const float *X, const float *M, int tq, int c,
                                    float (&y)[TPT]) {
+  static_assert(TPT % 2 == 0, "token pairs");
+  float2 acc[TPT / 2];
 #pragma unroll
-  for (int u = 0; u < TPT; ++u) y[u] = 0.f;
-#pragma unroll 4
+  for (int i = 0; i < TPT / 2; ++i) acc[i] = make_float2(0.f, 0.f);
+  const float *xr = X + tq * TPT;
+#pragma unroll 8
   for (int k = 0; k < D; ++k) {
     const float m = M[k * D + c];
-    const float *xr = X + k * Tok<D>::TB + tq * TPT;
+    float xv[TPT];
+    ld_vec<TPT>(xr + k * Tok<D>::TB, xv);
 #pragma unroll
-    for (int u = 0; u < TPT; ++u) y[u] = fmaf(xr[u], m, y[u]);
+    for (int i = 0; i < TPT / 2; ++i)
+      acc[i] = __ffma2_rn(make_float2(xv[2 * i], xv[2 * i + 1]), make_float2(m, m), acc[i]);
+  }
+#pragma unroll
+  for (int i = 0; i < TPT / 2; ++i) {
+    y[2 * i] = acc[i].x;
+    y[2 * i + 1] = acc[i].y;
   }
 }
 
@@ -187,11 +219,11 @@ __global__ void __launch_bounds__(kNT) bwd_query(
   const size_t rs = (size_t)H * D;
   const T *qc = q + ((size_t)b * N * H + h) * D + c;
   const int bi = tid / 16, bj = tid % 16;  // dS block rows bi * RB.., columns bj * RB..
-  float acc[RB][RB];
+  float2 acc2[RB][RB / 2];
 #pragma unroll
   for (int i = 0; i < RB; ++i)
 #pragma unroll
-    for (int j = 0; j < RB; ++j) acc[i][j] = 0.f;
+    for (int j = 0; j < RB / 2; ++j) acc2[i][j] = make_float2(0.f, 0.f);
   float dz = 0.f, dnw = 0.f;
   __syncthreads();
   for (int base = t0; base < t1; base += kTB) {
@@ -267,19 +299,19 @@ __global__ void __launch_bounds__(kNT) bwd_query(
       }
       dz = fmaf(P[u], dd, dz);
     }
-    // dS += P^T dnum over the batch's tokens
+    // dS += P^T dnum over the batch's tokens (RB values of P and of dnum per
+    // token as vector loads; packed FMAs over pairs of columns)
 #pragma unroll 2
     for (int tl = 0; tl < kTB; ++tl) {
       float pv[RB], nv[RB];
-#pragma unroll
-      for (int i = 0; i < RB; ++i) {
-        pv[i] = Pt[tl * D + bi * RB + i];
-        nv[i] = Nt[tl * D + bj * RB + i];
-      }
+      ld_vec<RB>(Pt + tl * D + bi * RB, pv);
+      ld_vec<RB>(Nt + tl * D + bj * RB, nv);
 #pragma unroll
       for (int i = 0; i < RB; ++i)
 #pragma unroll
-        for (int j = 0; j < RB; ++j) acc[i][j] = fmaf(pv[i], nv[j], acc[i][j]);
+        for (int j = 0; j < RB / 2; ++j)
+          acc2[i][j] = __ffma2_rn(make_float2(pv[i], pv[i]),
+                                  make_float2(nv[2 * j], nv[2 * j + 1]), acc2[i][j]);
     }
     __syncthreads();  // the batch's shared arrays are rewritten next
   }
@@ -287,7 +319,8 @@ __global__ void __launch_bounds__(kNT) bwd_query(
 #pragma unroll
   for (int i = 0; i < RB; ++i)
 #pragma unroll
-    for (int j = 0; j < RB; ++j) rec[(bi * RB + i) * D + bj * RB + j] = acc[i][j];
+    for (int j = 0; j < RB / 2; ++j)
+      *reinterpret_cast<float2 *>(rec + (bi * RB + i) * D + bj * RB + 2 * j) = acc2[i][j];
   // dz and dnw: sum over the token quads in order
   Pk[tq * D + c] = dz;
   Nk[tq * D + c] = dnw;
