@@ -191,7 +191,8 @@ uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_rela
 
 uint32_t gbla_device_error(int reset) {
   const unsigned a = tc_device_error(reset != 0), b = project_device_error(reset != 0);
-  return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu) ? 0xFFFFFFFFu : (a | b);
+  const unsigned c = bwd_device_error(reset != 0);
+  return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu || c == 0xFFFFFFFFu) ? 0xFFFFFFFFu : (a | b | c);
 }
 
 const char *gbla_last_cuda_error(void) { return cudaGetErrorString(t_last_cuda_error); }

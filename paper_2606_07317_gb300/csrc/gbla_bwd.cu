@@ -569,6 +569,11 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   constexpr int F = D * D + D;
   bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(qpart, red, nck);
   count_launch();
+  if (bwd_tc_key_supported(p)) {
+    if ((e = bwd_tc_key(p, a, stats, state, red, scratch + lay.cval, dxt + plane,
+                        dxt + 2 * plane, st)) != cudaSuccess)
+      return e;
+  } else {
   const size_t smk = sizeof(float) * (2 * D * D + D + 2 * D * kTB + kNT / 32 * TPT);
   auto kk = bwd_key<T, D>;
   if ((e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smk)) !=
@@ -578,6 +583,7 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
                                       a.conv_w, stats, state, red, p.seq_lens, (T *)a.dgate,
                                       dxt + plane, dxt + 2 * plane, H, N);
   count_launch();
+  }
   bwd_conv<T, D><<<dim3(nck, BH, 3), kNT, 0, st>>>(
       (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
       (T *)a.dk, (T *)a.dv, wpart, H, N, nck);
@@ -601,7 +607,8 @@ BwdLayout bwd_layout(const Problem &p) {
   l.stats = up(l.state + BH * F);
   l.qpart = up(l.stats + 2 * BH);
   l.red = up(l.qpart + BH * nck * (D * D + 2 * D));
-  l.dxt = up(l.red + BH * (F + 1));
+  l.cval = up(l.red + BH * (F + 1));
+  l.dxt = up(l.cval + BH);
   l.wpart = up(l.dxt + 3 * BH * (size_t)p.N * D);
   l.total = up(l.wpart + 3 * BH * nck * D * kConvW);
   return l;

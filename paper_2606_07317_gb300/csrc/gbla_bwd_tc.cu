@@ -1,0 +1,555 @@
+// Key pass of the GBLA backward on tensor cores (bf16, D = 64): for every
+// valid token t of a (batch, head), with the reduced gradients dS, dz of the
+// state and c = <dS, S> + <dz, z> (the chain rule of Sec. 2.1 item 2 through
+// the state and the softmax key gate):
+//
+//   dK^_t = dS v~_t + dz            dk~_t = g_t dK^_t phi'(k~_t)
+//   dv~_t = dS^T K^_t               dgate_t = g_t (phi(k~_t) . dK^_t - c)
+//
+// with K^_t = g_t phi(k~_t), g the softmax gate and phi' = min(phi, 1) (elu + 1:
+// phi' = 1 where phi = x + 1 > 1, phi' = e^x = phi where x <= 0).
+//
+// tc_bwd_key_kernel: persistent, one CTA per SM, each taking a contiguous run
+// of 128-token tiles (so the (batch, head) changes rarely).  One TMA warp
+// brings the raw k and v rows of a tile (128 tokens + 3 rows of conv history,
+// 128B-swizzled) into a 2-deep ring; four producer warps (one token row per
+// thread) run both Conv1Ds, phi and the gate in fp32 and write V~ and K^ as
+// bf16 K-major A tiles, plus phi(k~) as bf16; one thread issues the MMAs
+// DK = V~ dS^T and DV = K^ dS (M = 128, N = 64, K = 64) against bf16 hi + lo
+// splits of dS, fp32 accumulation in TMEM (two buffers); four epilogue warps
+// (one token row per thread) form dk~, dv~ and dgate and write the fp32 dk~ /
+// dv~ rows through per-warp staging as whole 128-byte segments.  The epilogue
+// warps also build the dS tiles whenever the (batch, head) changes.
+//
+// Every mbarrier wait is bounded (2 s); a wait that runs out sets a bit in
+// g_bwd_error and the CTA's abort flag, every role leaves its loop, the TMA
+// lane waits (bounded) for its copies in flight and the MMA thread for its
+// MMAs before TMEM is freed.
+#include <math.h>
+
+#include <mutex>
+
+#include "gbla_internal.cuh"
+#include "gbla_sm100.cuh"
+
+namespace gbla {
+
+__device__ unsigned int g_bwd_error;
+
+namespace {
+
+using namespace sm100;
+
+constexpr int kD = 64;
+constexpr int kKTok = 128;                       // tokens per tile (MMA M)
+constexpr int kKRawRows = kKTok + kConvW - 1;    // 131
+constexpr int kKRawBox = kKRawRows * 128;        // 16768 bytes per raw box
+constexpr int kKRawHalf = (kKRawBox + 1023) / 1024 * 1024;  // 17408
+constexpr int kKRawStage = 2 * kKRawHalf;        // k box, v box
+constexpr int kKStages = 2;
+constexpr int kKTile = kKTok * 128;              // 16384: one 128 x 64 bf16 tile
+constexpr int kKAStage = 3 * kKTile;             // V~, K^, phi(k~)
+constexpr int kKBTile = kD * 128;                // 8192: one 64 x 64 bf16 tile
+constexpr int kKProdWarps = 4, kKEpiWarps = 4;
+constexpr int kKEpiWarp0 = kKProdWarps;          // 4
+constexpr int kKMmaWarp = kKEpiWarp0 + kKEpiWarps;  // 8
+constexpr int kKTmaWarp = kKMmaWarp + 1;         // 9
+constexpr int kKThreads = (kKTmaWarp + 1) * 32;  // 320
+constexpr int kKEpi = kKEpiWarps * 32;
+constexpr int kKStg = 32 * 128;                  // staging per epilogue warp: 32 rows x 32 fp32
+constexpr uint32_t kKTmemCols = 256;             // two buffers of [DK | DV]
+
+constexpr int kKOffRaw = 0;
+constexpr int kKOffA = kKOffRaw + kKStages * kKRawStage;     // 69632
+constexpr int kKOffB = kKOffA + kKStages * kKAStage;         // 167936: dS hi, lo, dS^T hi, lo
+constexpr int kKOffG = kKOffB + 4 * kKBTile;                 // 200704: float [2][128]
+constexpr int kKOffDz = kKOffG + kKStages * kKTok * 4;       // float [64]
+constexpr int kKOffStg = kKOffDz + kD * 4;
+constexpr int kKOffBar = kKOffStg + kKEpiWarps * kKStg;
+// raw_full[2], raw_empty[2], a_full[2], a_empty[2], phi_full[2], phi_empty[2],
+// acc_full[2], acc_empty[2], b_full, b_free, fin
+constexpr int kKBars = 8 * kKStages + 3;
+constexpr int kKOffMisc = kKOffBar + kKBars * 8;             // tmem address, abort flag, c
+constexpr int kKSmem = kKOffMisc + 16 + 1024;
+static_assert(kKSmem <= 227 * 1024, "key-pass shared memory");
+
+struct KeyParams {
+  const __nv_bfloat16 *gate;       // [B, N, H]
+  const float *conv_w;             // [3, H, D, 4]
+  const float2 *stats;             // [B*H]: gate max, sum of exp
+  const float *red;                // [B*H][D*D + D]: dS, dz
+  const float *cval;               // [B*H]: c
+  const int32_t *seq_lens;
+  float *dkt, *dvt;                // [B, N, H, D] fp32 planes
+  __nv_bfloat16 *dgate;            // [B, N, H]
+  int B, H, N, tps;
+};
+
+__device__ __forceinline__ void report(unsigned code, const AbortFlag &ab) {
+  atomicOr(&g_bwd_error, code);
+  ab.raise();
+}
+
+__device__ __forceinline__ int seq_len(const int32_t *seq_lens, int b, int N) {
+  if (seq_lens == nullptr) return N;
+  const int L = seq_lens[b];
+  return L < 0 ? 0 : (L > N ? N : L);
+}
+
+// Tile i of this CTA's contiguous run -> (b, h, t0, L); false for a tile that
+// lies wholly in the padding.
+struct KTile {
+  int bh, b, h, t0, L;
+};
+__device__ __forceinline__ bool key_tile(const KeyParams &p, long long i, KTile &t) {
+  t.bh = (int)(i / p.tps);
+  t.b = t.bh / p.H;
+  t.h = t.bh % p.H;
+  t.t0 = (int)(i % p.tps) * kKTok;
+  t.L = seq_len(p.seq_lens, t.b, p.N);
+  return t.t0 < t.L;
+}
+
+__device__ __forceinline__ void unpack8(uint4 r, float (&f)[8]) {
+  const float2 a = bf2_to_f2(r.x), b = bf2_to_f2(r.y), c = bf2_to_f2(r.z), d = bf2_to_f2(r.w);
+  f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
+  f[4] = c.x; f[5] = c.y; f[6] = d.x; f[7] = d.y;
+}
+__device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
+  return make_uint4(f2_to_bf2(f[0], f[1]), f2_to_bf2(f[2], f[3]), f2_to_bf2(f[4], f[5]),
+                    f2_to_bf2(f[6], f[7]));
+}
+// byte offset of 16-byte chunk c of row r in a 128B-swizzled K-major tile
+__device__ __forceinline__ uint32_t sw_off(int r, int c) {
+  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
+}
+__device__ __forceinline__ float phi_f(float x) { return x > 0.f ? x + 1.f : expf(x); }
+
+__global__ void __launch_bounds__(kKThreads, 1)
+    tc_bwd_key_kernel(const KeyParams p, const __grid_constant__ CUtensorMap tm_k,
+                      const __grid_constant__ CUtensorMap tm_v) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int H = p.H, N = p.N;
+
+  uint64_t *bars = (uint64_t *)(smem + kKOffBar);
+  uint64_t *raw_full = bars, *raw_empty = bars + 2, *a_full = bars + 4, *a_empty = bars + 6;
+  uint64_t *phi_full = bars + 8, *phi_empty = bars + 10, *acc_full = bars + 12;
+  uint64_t *acc_empty = bars + 14, *b_full = bars + 16, *b_free = bars + 17, *fin = bars + 18;
+  uint32_t *tmem_slot = (uint32_t *)(smem + kKOffMisc);
+  const AbortFlag ab{smem_u32(smem + kKOffMisc + 4)};
+  float *cslot = (float *)(smem + kKOffMisc + 8);
+
+  const long long T = (long long)p.B * H * p.tps;
+  const long long i0 = T * blockIdx.x / gridDim.x, i1 = T * (blockIdx.x + 1) / gridDim.x;
+  if (i0 >= i1) return;
+
+  if (tid == 0) {
+    for (int i = 0; i < kKStages; ++i) {
+      mbar_init(&raw_full[i], 1);
+      mbar_init(&raw_empty[i], kKProdWarps);
+      mbar_init(&a_full[i], kKProdWarps);
+      mbar_init(&a_empty[i], 1);
+      mbar_init(&phi_full[i], kKProdWarps);
+      mbar_init(&phi_empty[i], kKEpiWarps);
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kKEpiWarps);
+    }
+    mbar_init(b_full, 1);
+    mbar_init(b_free, 1);
+    mbar_init(fin, 1);
+    *(volatile int *)(smem + kKOffMisc + 4) = 0;
+    fence_mbar_init();
+  }
+  if (warp == kKTmaWarp && lane == 0) {
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+  }
+  if (warp == kKMmaWarp) tmem_alloc(tmem_slot, kKTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == kKTmaWarp) {
+    // ------------------------------------------------------------ TMA: raw k, v rows
+    if (lane == 0) {
+      int li = 0;
+      bool ok = true;
+      for (long long i = i0; i < i1 && ok; ++i) {
+        KTile t;
+        if (!key_tile(p, i, t)) continue;
+        const int s = li % kKStages;
+        if (!mbar_wait(&raw_empty[s], ((li / kKStages) & 1) ^ 1, &ab)) {
+          if (!ab.raised()) report(1, ab);
+          ok = false;
+          break;
+        }
+        uint8_t *dst = smem + kKOffRaw + s * kKRawStage;
+        mbar_arrive_expect_tx(&raw_full[s], 2 * kKRawBox);
+        // rows t0 - 3 .. t0 + 127; rows before the sequence start read as zeros
+        tma_load_4d(dst, &tm_k, &raw_full[s], 0, t.h, t.t0 - 3, t.b);
+        tma_load_4d(dst + kKRawHalf, &tm_v, &raw_full[s], 0, t.h, t.t0 - 3, t.b);
+        ++li;
+      }
+      for (int j = li - 1; j >= 0 && j >= li - kKStages; --j)
+        if (!mbar_wait(&raw_full[j % kKStages], (j / kKStages) & 1, nullptr)) report(2, ab);
+    }
+  } else if (warp < kKEpiWarp0) {
+    // ------------------------------------------------------------ producers
+    const int r = tid;  // tile row
+    int li = 0, cur_bh = -1;
+    float2 gs = make_float2(0.f, 1.f);
+    bool ok = true;
+    for (long long i = i0; i < i1 && ok; ++i) {
+      KTile t;
+      if (!key_tile(p, i, t)) continue;
+      const int s = li % kKStages;
+      if (t.bh != cur_bh) {
+        gs = p.stats[t.bh];
+        cur_bh = t.bh;
+      }
+      const int tok = t.t0 + r;
+      const bool valid = tok < t.L;
+      const float g =
+          valid ? expf(__bfloat162float(p.gate[((size_t)t.b * N + tok) * H + t.h]) - gs.x) / gs.y
+                : 0.f;
+      if (!mbar_wait(&raw_full[s], (li / kKStages) & 1, &ab) ||
+          !mbar_wait(&a_empty[s], ((li / kKStages) & 1) ^ 1, &ab) ||
+          !mbar_wait(&phi_empty[s], ((li / kKStages) & 1) ^ 1, &ab)) {
+        ok = false;
+        break;
+      }
+      const uint32_t rk = smem_u32(smem + kKOffRaw + s * kKRawStage);
+      const uint32_t rv = rk + kKRawHalf;
+      const uint32_t av = smem_u32(smem + kKOffA + s * kKAStage);
+      const uint32_t ak = av + kKTile, ap = av + 2 * kKTile;
+      const float *cwk = p.conv_w + ((size_t)(H + t.h) * kD) * kConvW;
+      const float *cwv = p.conv_w + ((size_t)(2 * H + t.h) * kD) * kConvW;
+#pragma unroll 2
+      for (int c = 0; c < kD / 8; ++c) {
+        float kx[kConvW][8], vx[kConvW][8];
+#pragma unroll
+        for (int j = 0; j < kConvW; ++j) {
+          unpack8(lds_v4(rk + sw_off(r + j, c)), kx[j]);
+          unpack8(lds_v4(rv + sw_off(r + j, c)), vx[j]);
+        }
+        float vt[8], kh[8], ph[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float4 tk = __ldg((const float4 *)(cwk + (8 * c + e) * kConvW));
+          const float4 tv = __ldg((const float4 *)(cwv + (8 * c + e) * kConvW));
+          const float kt = fmaf(tk.w, kx[3][e], fmaf(tk.z, kx[2][e], fmaf(tk.y, kx[1][e], tk.x * kx[0][e])));
+          const float v1 = fmaf(tv.w, vx[3][e], fmaf(tv.z, vx[2][e], fmaf(tv.y, vx[1][e], tv.x * vx[0][e])));
+          const float f = phi_f(kt);
+          vt[e] = valid ? v1 : 0.f;
+          kh[e] = g * f;  // 0 on padded rows (g = 0)
+          ph[e] = f;
+        }
+        const uint32_t o = sw_off(r, c);
+        sts_v4(av + o, pack8(vt));
+        sts_v4(ak + o, pack8(kh));
+        sts_v4(ap + o, pack8(ph));
+      }
+      sts_f32(smem_u32(smem + kKOffG) + (uint32_t)(s * kKTok + r) * 4, g);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&raw_empty[s]);
+        mbar_arrive(&a_full[s]);
+        mbar_arrive(&phi_full[s]);
+      }
+      ++li;
+    }
+    if (!ok && !ab.raised()) report(4, ab);
+  } else if (warp < kKMmaWarp) {
+    // ------------------------------------------------------------ epilogue
+    const int q4 = warp & 3, row = 32 * q4 + lane;
+    const int et = tid - kKEpiWarp0 * 32;  // 0..127
+    const uint32_t stg = smem_u32(smem + kKOffStg + (warp - kKEpiWarp0) * kKStg);
+    const uint32_t bb = smem_u32(smem + kKOffB);
+    const float *dzs = (const float *)(smem + kKOffDz);
+    // Every epilogue warp runs every iteration (a failed wait does not leave
+    // the loop), so the named barriers below always match.
+    int li = 0, cur_bh = -1, nbh = 0;
+    bool ok = true;
+    for (long long i = i0; i < i1; ++i) {
+      KTile t;
+      if (!key_tile(p, i, t)) continue;
+      const int s = li % kKStages, buf = li % 2;
+      if (t.bh != cur_bh) {
+        // dS of the new (b, h) as bf16 hi + lo: dS (rows d, K = e) for DK and
+        // dS^T (rows e, K = d) for DV, once the previous MMAs are done with them
+        if (nbh > 0) {
+          named_barrier(1, kKEpi);  // every epilogue warp is done with the previous tile
+          ok = mbar_wait(b_free, (nbh - 1) & 1, &ab) && ok;
+        }
+        const float *dS = p.red + (size_t)t.bh * (kD * kD + kD);
+        for (int u = et; u < kD * (kD / 8); u += kKEpi) {
+          const int rr = u >> 3, cc = u & 7;  // row rr, chunk cc
+          float hi[8], lo[8], hT[8], lT[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float x = dS[rr * kD + 8 * cc + e];           // dS[rr][8cc + e]
+            const float y = dS[(8 * cc + e) * kD + rr];         // dS^T[rr][8cc + e]
+            hi[e] = __bfloat162float(__float2bfloat16_rn(x));
+            lo[e] = x - hi[e];
+            hT[e] = __bfloat162float(__float2bfloat16_rn(y));
+            lT[e] = y - hT[e];
+          }
+          const uint32_t o = sw_off(rr, cc);
+          sts_v4(bb + o, pack8(hi));
+          sts_v4(bb + kKBTile + o, pack8(lo));
+          sts_v4(bb + 2 * kKBTile + o, pack8(hT));
+          sts_v4(bb + 3 * kKBTile + o, pack8(lT));
+        }
+        if (et < kD) ((float *)(smem + kKOffDz))[et] = dS[kD * kD + et];
+        if (et == 0) *cslot = p.cval[t.bh];
+        fence_proxy_async_smem();
+        named_barrier(1, kKEpi);
+        if (et == 0) mbar_arrive(b_full);
+        cur_bh = t.bh;
+        ++nbh;
+      }
+      ok = mbar_wait(&acc_full[buf], (li >> 1) & 1, &ab) && ok;
+      ok = mbar_wait(&phi_full[s], (li / kKStages) & 1, &ab) && ok;
+      tc_fence_after();
+      const uint32_t tacc = tmem + ((uint32_t)(32 * q4) << 16) + buf * 128;
+      const int tok = t.t0 + row;
+      const bool valid = tok < t.L;
+      const float g = lds_f32(smem_u32(smem + kKOffG) + (uint32_t)(s * kKTok + row) * 4);
+      const uint32_t ap = smem_u32(smem + kKOffA + s * kKAStage) + 2 * kKTile;
+      const size_t prow = (((size_t)t.b * N + t.t0) * H + t.h) * kD;  // plane row of tile row 0
+      const size_t prs = (size_t)H * kD;                               // plane row stride
+      float dg = 0.f;
+      // dk~ in two 32-column halves, then dv~: each half through the staging rows
+#pragma unroll 1
+      for (int part = 0; part < 4; ++part) {
+        float v[32];
+        tmem_ld16(tacc + 32 * part, *reinterpret_cast<float(*)[16]>(v));
+        tmem_ld16(tacc + 32 * part + 16, *reinterpret_cast<float(*)[16]>(v + 16));
+        tmem_ld_wait();
+        if (part == 3) {  // accumulators drained
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        }
+        if (part < 2) {
+#pragma unroll
+          for (int cq = 0; cq < 4; ++cq) {
+            float f[8];
+            unpack8(lds_v4(ap + sw_off(row, 4 * part + cq)), f);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              const int d = 32 * part + 8 * cq + e;
+              const float dk = v[8 * cq + e] + dzs[d];
+              dg = fmaf(f[e], dk, dg);
+              v[8 * cq + e] = g * dk * fminf(f[e], 1.f);
+            }
+          }
+          if (part == 1) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&phi_empty[s]);  // phi(k~) rows read
+          }
+        }
+        // this row's 32 values -> 8 swizzled 16-byte pieces of the staging row
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          sts_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4),
+                 make_uint4(__float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]),
+                            __float_as_uint(v[4 * j + 2]), __float_as_uint(v[4 * j + 3])));
+        __syncwarp();
+        float *plane = part < 2 ? p.dkt : p.dvt;
+        const int col = 32 * (part & 1);
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + (lane >> 3), ch = lane & 7;
+          const uint4 val = lds_v4(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
+          const int trow = 32 * q4 + rr;
+          if (t.t0 + trow < t.L)
+            *(uint4 *)(plane + prow + (size_t)trow * prs + col + ch * 4) = val;
+        }
+        __syncwarp();
+      }
+      if (valid)
+        p.dgate[((size_t)t.b * N + tok) * H + t.h] = __float2bfloat16_rn(g * (dg - *cslot));
+      ++li;
+    }
+    if (!ok && !ab.raised()) report(8, ab);
+  } else if (warp == kKMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(kKTok, kD, 0, 0);
+      const uint32_t bb = smem_u32(smem + kKOffB);
+      int li = 0, cur_bh = -1, nbh = 0;
+      bool ok = true;
+      for (long long i = i0; i < i1 && ok; ++i) {
+        KTile t;
+        if (!key_tile(p, i, t)) continue;
+        const int s = li % kKStages, buf = li % 2;
+        if (t.bh != cur_bh) {
+          if (!mbar_wait(b_full, nbh & 1, &ab)) {
+            ok = false;
+            break;
+          }
+          cur_bh = t.bh;
+          ++nbh;
+        }
+        if (!mbar_wait(&a_full[s], (li / kKStages) & 1, &ab) ||
+            !mbar_wait(&acc_empty[buf], ((li >> 1) & 1) ^ 1, &ab)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t av = smem_u32(smem + kKOffA + s * kKAStage), ak = av + kKTile;
+        const uint32_t dk = tmem + buf * 128, dv = dk + kD;
+#pragma unroll
+        for (int k16 = 0; k16 < 4; ++k16) {
+          const uint32_t ko = 32 * k16;
+          const uint64_t a1 = sw128_desc(av + ko, 16, 1024), a2 = sw128_desc(ak + ko, 16, 1024);
+          mma_bf16(dk, a1, sw128_desc(bb + ko, 16, 1024), idesc, k16 != 0);
+          mma_bf16(dk, a1, sw128_desc(bb + kKBTile + ko, 16, 1024), idesc, 1);
+          mma_bf16(dv, a2, sw128_desc(bb + 2 * kKBTile + ko, 16, 1024), idesc, k16 != 0);
+          mma_bf16(dv, a2, sw128_desc(bb + 3 * kKBTile + ko, 16, 1024), idesc, 1);
+        }
+        mma_commit(&a_empty[s]);
+        mma_commit(&acc_full[buf]);
+        // last tile of this (b, h) in this CTA: the dS tiles may be rebuilt
+        bool last = true;
+        for (long long j = i + 1; j < i1; ++j) {
+          KTile tn;
+          if (key_tile(p, j, tn)) {
+            last = tn.bh != t.bh;
+            break;
+          }
+        }
+        if (last) mma_commit(b_free);
+        ++li;
+      }
+      if (!ok && !ab.raised()) report(16, ab);
+      mma_commit(fin);
+      if (!mbar_wait(fin, 0, nullptr)) report(32, ab);
+    }
+  }
+  __syncthreads();
+  if (warp == kKMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kKTmemCols);
+  }
+}
+
+// c = <dS, S> + <dz, z> per (b, h), summed in a fixed order.
+__global__ void __launch_bounds__(256) bwd_state_dot(const float *__restrict__ red,
+                                                     const float *__restrict__ state,
+                                                     float *__restrict__ cval, int F) {
+  const int bh = blockIdx.x;
+  __shared__ float part[256];
+  float a = 0.f;
+  for (int i = threadIdx.x; i < F; i += 256)
+    a = fmaf(red[(size_t)bh * F + i], state[(size_t)bh * F + i], a);
+  part[threadIdx.x] = a;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) cval[bh] = part[0];
+}
+
+using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                              const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                              const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                              CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeFn encode() {
+  static EncodeFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (EncodeFn)f;
+  });
+  return fn;
+}
+
+// [B, N, H, 64] bf16 as {D, H, N, B}; box = 64 channels x 1 head x 131 tokens,
+// 128-byte swizzle; rows before 0 or past N read as zeros.
+cudaError_t make_rows_map(CUtensorMap *m, const void *base, int B, int N, int H) {
+  EncodeFn fn = encode();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)H, (cuuint64_t)N, (cuuint64_t)B};
+  const cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)H * kD * 2,
+                                 (cuuint64_t)N * H * kD * 2};
+  const cuuint32_t box[4] = {(cuuint32_t)kD, 1, (cuuint32_t)kKRawRows, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+bool bwd_tc_key_supported(const Problem &p) {
+  if (p.dtype != GBLA_BF16 || p.D != kD || p.flags != 0) return false;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  return major == 10 && minor == 3 && encode() != nullptr;
+}
+
+cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
+                       const float *state, const float *red, float *cval, float *dkt,
+                       float *dvt, cudaStream_t st) {
+  const int BH = p.B * p.H;
+  constexpr int F = kD * kD + kD;
+  bwd_state_dot<<<BH, 256, 0, st>>>(red, state, cval, F);
+  count_launch();
+  // rows past seq_lens[b] of dgate are zero; the kernel writes the valid rows
+  cudaError_t e = cudaMemsetAsync(a.dgate, 0, sizeof(__nv_bfloat16) * (size_t)BH * p.N, st);
+  if (e != cudaSuccess) return e;
+  CUtensorMap tm_k, tm_v;
+  if ((e = make_rows_map(&tm_k, a.k, p.B, p.N, p.H)) != cudaSuccess) return e;
+  if ((e = make_rows_map(&tm_v, a.v, p.B, p.N, p.H)) != cudaSuccess) return e;
+  KeyParams kp;
+  kp.gate = (const __nv_bfloat16 *)a.gate;
+  kp.conv_w = a.conv_w;
+  kp.stats = stats;
+  kp.red = red;
+  kp.cval = cval;
+  kp.seq_lens = p.seq_lens;
+  kp.dkt = dkt;
+  kp.dvt = dvt;
+  kp.dgate = (__nv_bfloat16 *)a.dgate;
+  kp.B = p.B;
+  kp.H = p.H;
+  kp.N = p.N;
+  kp.tps = (p.N + kKTok - 1) / kKTok;
+  if ((e = cudaFuncSetAttribute(tc_bwd_key_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kKSmem)) != cudaSuccess)
+    return e;
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long tiles = (long long)BH * kp.tps;
+  const int grid = (int)(tiles < sms ? tiles : sms);
+  tc_bwd_key_kernel<<<grid, kKThreads, kKSmem, st>>>(kp, tm_k, tm_v);
+  count_launch();
+  return cudaGetLastError();
+}
+
+unsigned bwd_device_error(bool reset) {
+  unsigned v = 0;
+  if (cudaMemcpyFromSymbol(&v, g_bwd_error, sizeof(v)) != cudaSuccess) return 0xFFFFFFFFu;
+  if (reset) {
+    const unsigned z = 0;
+    if (cudaMemcpyToSymbol(g_bwd_error, &z, sizeof(z)) != cudaSuccess) return 0xFFFFFFFFu;
+  }
+  return v;
+}
+
+}  // namespace gbla

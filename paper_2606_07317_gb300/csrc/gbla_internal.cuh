@@ -66,10 +66,17 @@ struct BwdArgs {
 // partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
 // gradient partials.
 struct BwdLayout {
-  size_t state, stats, qpart, red, dxt, wpart, total;
+  size_t state, stats, qpart, red, cval, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
+// Key pass on tensor cores (gbla_bwd_tc.cu): bf16, D = 64, sm_103.  Writes the
+// dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz.
+bool bwd_tc_key_supported(const Problem &p);
+cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
+                       const float *state, const float *red, float *cval, float *dkt,
+                       float *dvt, cudaStream_t st);
+unsigned bwd_device_error(bool reset);
 
 // ---- layer front end (tcgen05; gbla_project.cu): bf16 ----------------------
 struct ProjProblem {
