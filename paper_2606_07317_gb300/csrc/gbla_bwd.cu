@@ -515,13 +515,14 @@ __global__ void __launch_bounds__(kNT) bwd_conv(
 }
 
 // ---------------------------------------------------------------- weight reductions
-// dconv_w[s][h][c][i] = sum_b sum_chunk wpart;  dnorm_w[h][c] = sum_b sum_chunk qpart.dnw
+// dconv_w[s][h][c][i] = sum_b sum_chunk wpart (nck chunks);  dnorm_w[h][c] = sum_b
+// sum_chunk qpart.dnw (nckq query-pass records per (b, h))
 template <int D>
 __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wpart,
                                                     const float *__restrict__ qpart,
                                                     float *__restrict__ dconv_w,
                                                     float *__restrict__ dnorm_w, int B, int H,
-                                                    int nck) {
+                                                    int nck, int nckq) {
   const int total_w = 3 * H * D * kConvW;
   for (int idx = blockIdx.x * 256 + threadIdx.x; idx < total_w + H * D;
        idx += gridDim.x * 256) {
@@ -536,8 +537,8 @@ __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wp
     } else {
       const int j = idx - total_w, h = j / D, cc = j % D;
       for (int b = 0; b < B; ++b)
-        for (int ch = 0; ch < nck; ++ch)
-          a += qpart[(((size_t)b * H + h) * nck + ch) * qrec<D>() + D * D + D + cc];
+        for (int ch = 0; ch < nckq; ++ch)
+          a += qpart[(((size_t)b * H + h) * nckq + ch) * qrec<D>() + D * D + D + cc];
       dnorm_w[j] = a;
     }
   }
@@ -558,18 +559,25 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   count_launch();
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   const size_t smq = sizeof(float) * (2 * D * D + D + 4 * D * kTB + kTB + kNT / 32 * TPT);
-  auto kq = bwd_query<T, D>;
-  if ((e = cudaFuncSetAttribute(kq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smq)) !=
-      cudaSuccess)
-    return e;
-  kq<<<dim3(nck, BH), kNT, smq, st>>>((const T *)a.q, (const T *)a.out_gate, (const T *)a.dy,
-                                      a.conv_w, a.norm_w, state, p.seq_lens, kRmsEps,
-                                      (T *)a.dout_gate, dxt, qpart, H, N, nck);
-  count_launch();
+  const bool tc = bwd_tc_key_supported(p);  // bf16, D = 64, sm_103: both token passes on tcgen05
+  int nckq = nck;                           // partial records of the query pass per (b, h)
+  if (tc) {
+    nckq = bwd_tc_query_chunks(p);
+    if ((e = bwd_tc_query(p, a, state, qpart, dxt, st)) != cudaSuccess) return e;
+  } else {
+    auto kq = bwd_query<T, D>;
+    if ((e = cudaFuncSetAttribute(kq, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smq)) !=
+        cudaSuccess)
+      return e;
+    kq<<<dim3(nck, BH), kNT, smq, st>>>((const T *)a.q, (const T *)a.out_gate, (const T *)a.dy,
+                                        a.conv_w, a.norm_w, state, p.seq_lens, kRmsEps,
+                                        (T *)a.dout_gate, dxt, qpart, H, N, nck);
+    count_launch();
+  }
   constexpr int F = D * D + D;
-  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(qpart, red, nck);
+  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(qpart, red, nckq);
   count_launch();
-  if (bwd_tc_key_supported(p)) {
+  if (tc) {
     if ((e = bwd_tc_key(p, a, stats, state, red, scratch + lay.cval, dxt + plane,
                         dxt + 2 * plane, st)) != cudaSuccess)
       return e;
@@ -590,7 +598,7 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
   bwd_reduce_w<D><<<(nw + 255) / 256, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
-                                                     nck);
+                                                     nck, nckq);
   count_launch();
   return cudaGetLastError();
 }

@@ -215,9 +215,10 @@ __global__ void __launch_bounds__(kKThreads, 1)
       const float g =
           valid ? expf(__bfloat162float(p.gate[((size_t)t.b * N + tok) * H + t.h]) - gs.x) / gs.y
                 : 0.f;
-      if (!mbar_wait(&raw_full[s], (li / kKStages) & 1, &ab) ||
-          !mbar_wait(&a_empty[s], ((li / kKStages) & 1) ^ 1, &ab) ||
-          !mbar_wait(&phi_empty[s], ((li / kKStages) & 1) ^ 1, &ab)) {
+      const bool w = mbar_wait(&raw_full[s], (li / kKStages) & 1, &ab) &&
+                     mbar_wait(&a_empty[s], ((li / kKStages) & 1) ^ 1, &ab) &&
+                     mbar_wait(&phi_empty[s], ((li / kKStages) & 1) ^ 1, &ab);
+      if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
         ok = false;
         break;
       }
@@ -439,6 +440,499 @@ __global__ void __launch_bounds__(kKThreads, 1)
   }
 }
 
+// ===================================================================== query pass
+// Per (b, h, chunk of 1024 tokens), for every valid token t with P_t = phi(q~_t),
+// the forward's O_t = S^T P_t / (P_t . z) and the gated RMSNorm (Sec. 2.1
+// items 2 and 3), the chain rule in reverse:
+//
+//   dog_t = dy O r w silu'(og);  dnw += dy O r silu(og);  u = dy w silu(og)
+//   dO = r u - (r^3 / D) O (u . O);  dnum = dO / den;  dden = -(dO . O) / den
+//   dq~_t = (S dnum_t + z dden_t) phi'(q~_t);  dS += P_t dnum_t^T;  dz += P_t dden_t
+//
+// Four MMAs per 128-token tile: [num | den] = P [S | z] (S as bf16 hi + lo);
+// dP = dnum S^T (hi + lo); dS += P^T dnum (both operands read MN-major from the
+// same tiles, M = 128 with the two 64-row halves of A equal, accumulated in
+// TMEM over the chunk).  Roles: a TMA warp (raw q tile with 3 rows of history,
+// out_gate and dy tiles), four producer warps (P = phi(conv(q)) in fp32, bf16
+// A tile), one MMA thread, four warps for the gated-RMSNorm / readout
+// backward (one token row per thread; dog, dnum, dden, per-row dnw sums) and
+// four for dq~ and the per-row dz sums; the chunk's dS, dz and dnw go to a
+// partial record.
+constexpr int kQC = 1024;                          // tokens per CTA
+constexpr int kQTiles = kQC / kKTok;               // 8
+constexpr int kQInQ = kKRawHalf;                   // 17408: raw q box
+constexpr int kQIn = kQInQ + 2 * kKTile;           // + out_gate, dy tiles: 50176
+constexpr int kQSzT = 80 * 128;                    // [S^T | z] tile: 80 rows
+constexpr int kQProdWarps = 4, kQE1Warps = 4, kQE2Warps = 4;
+constexpr int kQE1Warp0 = kQProdWarps;             // 4
+constexpr int kQE2Warp0 = kQE1Warp0 + kQE1Warps;   // 8
+constexpr int kQMmaWarp = kQE2Warp0 + kQE2Warps;   // 12
+constexpr int kQTmaWarp = kQMmaWarp + 1;           // 13
+constexpr int kQThreads = (kQTmaWarp + 1) * 32;    // 448
+constexpr int kQOffIn = 0;
+constexpr int kQOffP = kQOffIn + kKStages * kQIn;          // 100352
+constexpr int kQOffDn = kQOffP + kKStages * kKTile;        // 133120
+constexpr int kQOffB = kQOffDn + kKStages * kKTile;        // 165888: SzT hi, lo, S hi, lo
+constexpr int kQOffZ = kQOffB + 2 * kQSzT + 2 * kKBTile;   // 202752: z [64], w [64]
+constexpr int kQOffDd = kQOffZ + 2 * kD * 4;               // float [2][128]: dden
+constexpr int kQOffStg = kQOffDd + kKStages * kKTok * 4;
+constexpr int kQOffBar = kQOffStg + kQE2Warps * kKStg;
+// in_full, in_empty, p_full, p_empty, a1_full, a1_empty, dn_full, dn_empty,
+// a2_full, a2_empty (2 each), b_full, a3_full, fin
+constexpr int kQBars = 10 * kKStages + 3;
+constexpr int kQOffMisc = kQOffBar + kQBars * 8;
+constexpr int kQSmem = kQOffMisc + 16 + 1024;
+static_assert(kQSmem <= 227 * 1024, "query-pass shared memory");
+static_assert(2 * kKTok * kD * 4 <= kKStages * kQIn, "end-of-chunk reduction space");
+constexpr uint32_t kQA1 = 0, kQA2 = 256, kQA3 = 384;     // TMEM columns
+constexpr int kQRec = kD * kD + 2 * kD;            // dS, dz, dnw
+
+struct QueryParams {
+  const float *conv_w, *norm_w, *state;  // state: [B*H][D*D + D]
+  const int32_t *seq_lens;
+  __nv_bfloat16 *dog;                    // [B, N, H, D]
+  float *dqt;                            // fp32 plane
+  float *part;                           // [B*H][nck][kQRec]
+  float eps;
+  int B, H, N, nck;
+};
+
+__device__ __forceinline__ float sigmoid_f(float x) { return 1.f / (1.f + expf(-x)); }
+
+__global__ void __launch_bounds__(kQThreads, 1)
+    tc_bwd_query_kernel(const QueryParams p, const __grid_constant__ CUtensorMap tm_q,
+                        const __grid_constant__ CUtensorMap tm_og,
+                        const __grid_constant__ CUtensorMap tm_dy) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int H = p.H, N = p.N;
+  const int chunk = blockIdx.x, bh = blockIdx.y, b = bh / H, h = bh % H;
+  const int L = seq_len(p.seq_lens, b, N);
+  const int c0 = chunk * kQC;
+  // valid tiles of this chunk: t0 = c0 + 128 j < min(L, N)
+  const int nt = L > c0 ? min(kQTiles, (L - c0 + kKTok - 1) / kKTok) : 0;
+
+  uint64_t *bars = (uint64_t *)(smem + kQOffBar);
+  uint64_t *in_full = bars, *in_empty = bars + 2, *p_full = bars + 4, *p_empty = bars + 6;
+  uint64_t *a1_full = bars + 8, *a1_empty = bars + 10, *dn_full = bars + 12;
+  uint64_t *dn_empty = bars + 14, *a2_full = bars + 16, *a2_empty = bars + 18;
+  uint64_t *b_full = bars + 20, *a3_full = bars + 21, *fin = bars + 22;
+  uint32_t *tmem_slot = (uint32_t *)(smem + kQOffMisc);
+  const AbortFlag ab{smem_u32(smem + kQOffMisc + 4)};
+  const float *zs = (const float *)(smem + kQOffZ), *ws = zs + kD;
+  float *dds = (float *)(smem + kQOffDd);
+
+  if (tid == 0) {
+    for (int i = 0; i < kKStages; ++i) {
+      mbar_init(&in_full[i], 1);
+      mbar_init(&in_empty[i], kQProdWarps + kQE1Warps);
+      mbar_init(&p_full[i], kQProdWarps);
+      mbar_init(&p_empty[i], 1 + kQE2Warps);
+      mbar_init(&a1_full[i], 1);
+      mbar_init(&a1_empty[i], kQE1Warps);
+      mbar_init(&dn_full[i], kQE1Warps);
+      mbar_init(&dn_empty[i], 1);
+      mbar_init(&a2_full[i], 1);
+      mbar_init(&a2_empty[i], kQE2Warps);
+    }
+    mbar_init(b_full, 1);
+    mbar_init(a3_full, 1);
+    mbar_init(fin, 1);
+    *(volatile int *)(smem + kQOffMisc + 4) = 0;
+    fence_mbar_init();
+  }
+  if (warp == kQTmaWarp && lane == 0) {
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_og);
+    tma_prefetch_desc(&tm_dy);
+  }
+  if (warp == kQMmaWarp) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const size_t prs = (size_t)H * kD;                         // plane row stride
+  const size_t prow0 = (((size_t)b * N + c0) * H + h) * kD;  // plane row of the chunk's token 0
+
+  if (warp == kQTmaWarp) {
+    // ------------------------------------------------------------ TMA: q, out_gate, dy
+    if (lane == 0) {
+      int li = 0;
+      for (; li < nt; ++li) {
+        const int s = li % kKStages, t0 = c0 + li * kKTok;
+        if (!mbar_wait(&in_empty[s], ((li / kKStages) & 1) ^ 1, &ab)) {
+          if (!ab.raised()) report(64, ab);
+          break;
+        }
+        uint8_t *dst = smem + kQOffIn + s * kQIn;
+        mbar_arrive_expect_tx(&in_full[s], kKRawBox + 2 * kKTile);
+        tma_load_4d(dst, &tm_q, &in_full[s], 0, h, t0 - 3, b);
+        tma_load_4d(dst + kQInQ, &tm_og, &in_full[s], 0, h, t0, b);
+        tma_load_4d(dst + kQInQ + kKTile, &tm_dy, &in_full[s], 0, h, t0, b);
+      }
+      for (int j = li - 1; j >= 0 && j >= li - kKStages; --j)
+        if (!mbar_wait(&in_full[j % kKStages], (j / kKStages) & 1, nullptr)) report(128, ab);
+    }
+  } else if (warp < kQE1Warp0) {
+    // ------------------------------------------------------------ producers: P = phi(conv(q))
+    const int r = tid;
+    const float *cwq = p.conv_w + ((size_t)h * kD) * kConvW;
+    bool ok = true;
+    for (int li = 0; li < nt && ok; ++li) {
+      const int s = li % kKStages, ph = (li / kKStages) & 1;
+      const bool valid = c0 + li * kKTok + r < L;
+      const bool w = mbar_wait(&in_full[s], ph, &ab) && mbar_wait(&p_empty[s], ph ^ 1, &ab);
+      if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
+        ok = false;
+        break;
+      }
+      const uint32_t rq = smem_u32(smem + kQOffIn + s * kQIn);
+      const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
+#pragma unroll 2
+      for (int c = 0; c < kD / 8; ++c) {
+        float qx[kConvW][8], pv[8];
+#pragma unroll
+        for (int j = 0; j < kConvW; ++j) unpack8(lds_v4(rq + sw_off(r + j, c)), qx[j]);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float4 tq = __ldg((const float4 *)(cwq + (8 * c + e) * kConvW));
+          const float qt = fmaf(tq.w, qx[3][e], fmaf(tq.z, qx[2][e], fmaf(tq.y, qx[1][e], tq.x * qx[0][e])));
+          pv[e] = valid ? phi_f(qt) : 0.f;
+        }
+        sts_v4(pt + sw_off(r, c), pack8(pv));
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&p_full[s]);
+        mbar_arrive(&in_empty[s]);
+      }
+    }
+    if (!ok && !ab.raised()) report(256, ab);
+  } else if (warp < kQE2Warp0) {
+    // ------------------------------------------------------------ gated RMSNorm / readout backward
+    const int q4 = warp & 3, row = 32 * q4 + lane;
+    float dnw[kD];
+#pragma unroll
+    for (int i = 0; i < kD; ++i) dnw[i] = 0.f;
+    bool ok = __all_sync(0xffffffffu, mbar_wait(b_full, 0, &ab));  // z and w in shared memory
+    for (int li = 0; li < nt && ok; ++li) {
+      const int s = li % kKStages, ph = (li / kKStages) & 1;
+      const int t = c0 + li * kKTok + row;
+      const bool valid = t < L;
+      const bool w = mbar_wait(&a1_full[s], ph, &ab) && mbar_wait(&in_full[s], ph, &ab) &&
+                     mbar_wait(&dn_empty[s], ph ^ 1, &ab);
+      if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t ta = tmem + ((uint32_t)(32 * q4) << 16) + kQA1 + 128 * s;
+      const uint32_t ogt = smem_u32(smem + kQOffIn + s * kQIn) + kQInQ, dyt = ogt + kKTile;
+      const uint32_t dnt = smem_u32(smem + kQOffDn + s * kKTile);
+      float den;
+      {
+        float v4[4];
+        tmem_ld4(ta + kD, v4);
+        tmem_ld_wait();
+        den = v4[0];
+      }
+      const float inv = valid ? 1.f / den : 0.f;
+      // pass 1: mean O^2
+      float ss = 0.f;
+#pragma unroll 1
+      for (int j = 0; j < 4; ++j) {
+        float v[16];
+        tmem_ld16(ta + 16 * j, v);
+        tmem_ld_wait_regs(v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float o = v[i] * inv;
+          ss = fmaf(o, o, ss);
+        }
+      }
+      const float rr = rsqrtf(ss * (1.f / kD) + p.eps);
+      // pass 2: dog, dnw, u . O
+      float uo = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float v[16], og[16], dy[16];
+        tmem_ld16(ta + 16 * j, v);
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(og));
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(og + 8));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
+        tmem_ld_wait_regs(v);
+        float gq[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int d = 16 * j + i;
+          const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
+          const float w = ws[d];
+          gq[i] = dy[i] * o * rr * w * sg * (1.f + og[i] * (1.f - sg));
+          dnw[d] = valid ? fmaf(dy[i] * o, rr * si, dnw[d]) : dnw[d];
+          uo = fmaf(dy[i] * w * si, o, uo);
+        }
+        if (valid) {
+          float a[8], c[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            a[i] = gq[i];
+            c[i] = gq[8 + i];
+          }
+          __nv_bfloat16 *dst = p.dog + prow0 + (size_t)(li * kKTok + row) * prs + 16 * j;
+          *(uint4 *)dst = pack8(a);
+          *(uint4 *)(dst + 8) = pack8(c);
+        }
+      }
+      // pass 3: dO, dnum (bf16 A / B tile), dO . O
+      const float r3 = rr * rr * rr * (1.f / kD);
+      float doo = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float v[16], og[16], dy[16];
+        tmem_ld16(ta + 16 * j, v);
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(og));
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(og + 8));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
+        tmem_ld_wait_regs(v);
+        float dn[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int d = 16 * j + i;
+          const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
+          const float u = dy[i] * ws[d] * si;
+          const float dO = rr * u - r3 * o * uo;
+          doo = fmaf(dO, o, doo);
+          dn[i] = valid ? dO * inv : 0.f;
+        }
+        float a[8], c[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          a[i] = dn[i];
+          c[i] = dn[8 + i];
+        }
+        sts_v4(dnt + sw_off(row, 2 * j), pack8(a));
+        sts_v4(dnt + sw_off(row, 2 * j + 1), pack8(c));
+      }
+      dds[s * kKTok + row] = valid ? -doo * inv : 0.f;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&a1_empty[s]);
+        mbar_arrive(&dn_full[s]);
+        mbar_arrive(&in_empty[s]);
+      }
+    }
+    if (!ok && !ab.raised()) report(512, ab);
+    // this thread's dnw row into the reduction space: the input ring is no
+    // longer read (the producers finished before the last tile's MMAs, and
+    // this role read the last out_gate / dy rows above)
+    float *red = (float *)(smem + kQOffIn);
+#pragma unroll
+    for (int i = 0; i < kD; ++i) red[row * kD + i] = dnw[i];
+  } else if (warp < kQMmaWarp) {
+    // ------------------------------------------------------------ dq~, dz; the B tiles
+    const int q4 = warp & 3, row = 32 * q4 + lane, et = tid - kQE2Warp0 * 32;
+    const uint32_t bb = smem_u32(smem + kQOffB);
+    const uint32_t stg = smem_u32(smem + kQOffStg + (warp - kQE2Warp0) * kKStg);
+    {
+      // [S^T | z] (80 rows: B[e][d] = S[d][e], B[64][d] = z[d], zero rows) and S
+      // (B[d][e] = S[d][e]) as bf16 hi + lo, K-major 128B-swizzled
+      const float *S = p.state + (size_t)bh * (kD * kD + kD);
+      for (int u = et; u < 80 * (kD / 8); u += 128) {
+        const int rr = u >> 3, cc = u & 7;
+        float hi[8], lo[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const int d = 8 * cc + e;
+          const float x = rr < kD ? S[d * kD + rr] : (rr == kD ? S[kD * kD + d] : 0.f);
+          hi[e] = __bfloat162float(__float2bfloat16_rn(x));
+          lo[e] = x - hi[e];
+        }
+        sts_v4(bb + sw_off(rr, cc), pack8(hi));
+        sts_v4(bb + kQSzT + sw_off(rr, cc), pack8(lo));
+      }
+      for (int u = et; u < kD * (kD / 8); u += 128) {
+        const int rr = u >> 3, cc = u & 7;
+        float hi[8], lo[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float x = S[rr * kD + 8 * cc + e];
+          hi[e] = __bfloat162float(__float2bfloat16_rn(x));
+          lo[e] = x - hi[e];
+        }
+        sts_v4(bb + 2 * kQSzT + sw_off(rr, cc), pack8(hi));
+        sts_v4(bb + 2 * kQSzT + kKBTile + sw_off(rr, cc), pack8(lo));
+      }
+      if (et < kD) {
+        ((float *)(smem + kQOffZ))[et] = S[kD * kD + et];
+        ((float *)(smem + kQOffZ))[kD + et] = p.norm_w[(size_t)h * kD + et];
+      }
+      fence_proxy_async_smem();
+      named_barrier(2, 128);
+      if (et == 0) mbar_arrive(b_full);
+    }
+    float dz[kD];
+#pragma unroll
+    for (int i = 0; i < kD; ++i) dz[i] = 0.f;
+    bool ok = true;
+    for (int li = 0; li < nt && ok; ++li) {
+      const int s = li % kKStages, ph = (li / kKStages) & 1;
+      const bool w = mbar_wait(&a2_full[s], ph, &ab) && mbar_wait(&dn_full[s], ph, &ab);
+      if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t ta = tmem + ((uint32_t)(32 * q4) << 16) + kQA2 + kD * s;
+      const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
+      const float dd = dds[s * kKTok + row];
+#pragma unroll 1
+      for (int part = 0; part < 2; ++part) {
+        float v[32];
+        tmem_ld16(ta + 32 * part, *reinterpret_cast<float(*)[16]>(v));
+        tmem_ld16(ta + 32 * part + 16, *reinterpret_cast<float(*)[16]>(v + 16));
+        tmem_ld_wait();
+        if (part == 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&a2_empty[s]);
+        }
+#pragma unroll
+        for (int cq = 0; cq < 4; ++cq) {
+          float f[8];
+          unpack8(lds_v4(pt + sw_off(row, 4 * part + cq)), f);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int d = 32 * part + 8 * cq + e;
+            dz[d] = fmaf(f[e], dd, dz[d]);
+            v[8 * cq + e] = (v[8 * cq + e] + zs[d] * dd) * fminf(f[e], 1.f);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          sts_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4),
+                 make_uint4(__float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]),
+                            __float_as_uint(v[4 * j + 2]), __float_as_uint(v[4 * j + 3])));
+        __syncwarp();
+#pragma unroll
+        for (int it = 0; it < 8; ++it) {
+          const int rr = it * 4 + (lane >> 3), ch = lane & 7;
+          const uint4 val = lds_v4(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
+          const int tl = li * kKTok + 32 * q4 + rr;
+          if (c0 + tl < L)
+            *(uint4 *)(p.dqt + prow0 + (size_t)tl * prs + 32 * part + ch * 4) = val;
+        }
+        __syncwarp();
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_empty[s]);  // P rows read
+    }
+    if (!ok && !ab.raised()) report(1024, ab);
+    // the last dnum tile followed the last out_gate / dy reads, so the input
+    // ring is free here too
+    float *red = (float *)(smem + kQOffIn) + kKTok * kD;
+#pragma unroll
+    for (int i = 0; i < kD; ++i) red[row * kD + i] = dz[i];
+  } else if (warp == kQMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t id1 = idesc_bf16_f32(kKTok, 80, 0, 0);
+      const uint32_t id2 = idesc_bf16_f32(kKTok, kD, 0, 0);
+      const uint32_t id3 = idesc_bf16_f32(kKTok, kD, 1, 1);
+      const uint32_t bb = smem_u32(smem + kQOffB);
+      bool ok = mbar_wait(b_full, 0, &ab);
+      auto mma1 = [&](int li) -> bool {
+        const int s = li % kKStages, ph = (li / kKStages) & 1;
+        if (!mbar_wait(&p_full[s], ph, &ab) || !mbar_wait(&a1_empty[s], ph ^ 1, &ab)) return false;
+        tc_fence_after();
+        const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
+#pragma unroll
+        for (int k16 = 0; k16 < 4; ++k16) {
+          const uint64_t a = sw128_desc(pt + 32 * k16, 16, 1024);
+          mma_bf16(tmem + kQA1 + 128 * s, a, sw128_desc(bb + 32 * k16, 16, 1024), id1, k16 != 0);
+          mma_bf16(tmem + kQA1 + 128 * s, a, sw128_desc(bb + kQSzT + 32 * k16, 16, 1024), id1, 1);
+        }
+        mma_commit(&a1_full[s]);
+        return true;
+      };
+      if (ok && nt > 0) ok = mma1(0);
+      for (int li = 0; li < nt && ok; ++li) {
+        const int s = li % kKStages, ph = (li / kKStages) & 1;
+        if (li + 1 < nt && !mma1(li + 1)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait(&dn_full[s], ph, &ab) || !mbar_wait(&a2_empty[s], ph ^ 1, &ab)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t dn = smem_u32(smem + kQOffDn + s * kKTile);
+        const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
+#pragma unroll
+        for (int k16 = 0; k16 < 4; ++k16) {  // dP = dnum S^T: K = e
+          const uint64_t a = sw128_desc(dn + 32 * k16, 16, 1024);
+          mma_bf16(tmem + kQA2 + kD * s, a, sw128_desc(bb + 2 * kQSzT + 32 * k16, 16, 1024),
+                   id2, k16 != 0);
+          mma_bf16(tmem + kQA2 + kD * s, a,
+                   sw128_desc(bb + 2 * kQSzT + kKBTile + 32 * k16, 16, 1024), id2, 1);
+        }
+#pragma unroll
+        for (int k16 = 0; k16 < kKTok / 16; ++k16)  // dS += P^T dnum: K = tokens
+          mma_bf16(tmem + kQA3, sw128_desc(pt + 2048 * k16, 0, 1024),
+                   sw128_desc(dn + 2048 * k16, 16, 1024), id3, (li | k16) != 0);
+        mma_commit(&a2_full[s]);
+        mma_commit(&dn_empty[s]);
+        mma_commit(&p_empty[s]);
+      }
+      if (!ok && !ab.raised()) report(2048, ab);
+      mma_commit(a3_full);
+      mma_commit(fin);
+      if (!mbar_wait(fin, 0, nullptr)) report(4096, ab);
+    }
+  }
+  // every role is done: the partial record of this chunk (fixed summation order)
+  __syncthreads();
+  float *rec = p.part + ((size_t)bh * p.nck + chunk) * kQRec;
+  const float *red = (const float *)(smem + kQOffIn);
+  if (tid < kD) {
+    float a = 0.f, w = 0.f;
+    for (int r = 0; r < kKTok; ++r) {
+      w += red[r * kD + tid];
+      a += red[kKTok * kD + r * kD + tid];
+    }
+    rec[kD * kD + tid] = a;
+    rec[kD * kD + kD + tid] = w;
+  }
+  if (warp >= kQE2Warp0 && warp < kQMmaWarp && (warp & 3) < 2) {
+    // dS rows d = 32 q4 + lane (q4 = 0, 1) from TMEM lanes 0..63
+    const int q4 = warp & 3, d = 32 * q4 + lane;
+    if (__all_sync(0xffffffffu, nt > 0 && mbar_wait(a3_full, 0, &ab))) {
+      tc_fence_after();
+      for (int j = 0; j < kD / 16; ++j) {
+        float v[16];
+        tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + kQA3 + 16 * j, v);
+        tmem_ld_wait_regs(v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) rec[d * kD + 16 * j + i] = v[i];
+      }
+    } else {
+      for (int i = 0; i < kD; ++i) rec[d * kD + i] = 0.f;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kQMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
 // c = <dS, S> + <dz, z> per (b, h), summed in a fixed order.
 __global__ void __launch_bounds__(256) bwd_state_dot(const float *__restrict__ red,
                                                      const float *__restrict__ state,
@@ -475,15 +969,16 @@ EncodeFn encode() {
   return fn;
 }
 
-// [B, N, H, 64] bf16 as {D, H, N, B}; box = 64 channels x 1 head x 131 tokens,
-// 128-byte swizzle; rows before 0 or past N read as zeros.
-cudaError_t make_rows_map(CUtensorMap *m, const void *base, int B, int N, int H) {
+// [B, N, H, 64] bf16 as {D, H, N, B}; box = 64 channels x 1 head x `rows`
+// tokens, 128-byte swizzle; rows before 0 or past N read as zeros.
+cudaError_t make_rows_map(CUtensorMap *m, const void *base, int B, int N, int H,
+                          int rows = kKRawRows) {
   EncodeFn fn = encode();
   if (!fn) return cudaErrorNotSupported;
   const cuuint64_t dims[4] = {(cuuint64_t)kD, (cuuint64_t)H, (cuuint64_t)N, (cuuint64_t)B};
   const cuuint64_t strides[3] = {(cuuint64_t)kD * 2, (cuuint64_t)H * kD * 2,
                                  (cuuint64_t)N * H * kD * 2};
-  const cuuint32_t box[4] = {(cuuint32_t)kD, 1, (cuuint32_t)kKRawRows, 1};
+  const cuuint32_t box[4] = {(cuuint32_t)kD, 1, (cuuint32_t)rows, 1};
   const cuuint32_t estr[4] = {1, 1, 1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -538,6 +1033,42 @@ cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
   const long long tiles = (long long)BH * kp.tps;
   const int grid = (int)(tiles < sms ? tiles : sms);
   tc_bwd_key_kernel<<<grid, kKThreads, kKSmem, st>>>(kp, tm_k, tm_v);
+  count_launch();
+  return cudaGetLastError();
+}
+
+int bwd_tc_query_chunks(const Problem &p) { return (p.N + kQC - 1) / kQC; }
+
+cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state, float *part,
+                         float *dqt, cudaStream_t st) {
+  const int BH = p.B * p.H;
+  cudaError_t e;
+  // rows past seq_lens[b] of dout_gate are zero; the kernel writes the valid rows
+  if (p.seq_lens != nullptr &&
+      (e = cudaMemsetAsync(a.dout_gate, 0, sizeof(__nv_bfloat16) * (size_t)BH * p.N * kD, st)) !=
+          cudaSuccess)
+    return e;
+  CUtensorMap tm_q, tm_og, tm_dy;
+  if ((e = make_rows_map(&tm_q, a.q, p.B, p.N, p.H)) != cudaSuccess) return e;
+  if ((e = make_rows_map(&tm_og, a.out_gate, p.B, p.N, p.H, kKTok)) != cudaSuccess) return e;
+  if ((e = make_rows_map(&tm_dy, a.dy, p.B, p.N, p.H, kKTok)) != cudaSuccess) return e;
+  QueryParams qp;
+  qp.conv_w = a.conv_w;
+  qp.norm_w = a.norm_w;
+  qp.state = state;
+  qp.seq_lens = p.seq_lens;
+  qp.dog = (__nv_bfloat16 *)a.dout_gate;
+  qp.dqt = dqt;
+  qp.part = part;
+  qp.eps = kRmsEps;
+  qp.B = p.B;
+  qp.H = p.H;
+  qp.N = p.N;
+  qp.nck = bwd_tc_query_chunks(p);
+  if ((e = cudaFuncSetAttribute(tc_bwd_query_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kQSmem)) != cudaSuccess)
+    return e;
+  tc_bwd_query_kernel<<<dim3(qp.nck, BH), kQThreads, kQSmem, st>>>(qp, tm_q, tm_og, tm_dy);
   count_launch();
   return cudaGetLastError();
 }

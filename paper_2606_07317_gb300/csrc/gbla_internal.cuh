@@ -76,6 +76,11 @@ bool bwd_tc_key_supported(const Problem &p);
 cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
                        const float *state, const float *red, float *cval, float *dkt,
                        float *dvt, cudaStream_t st);
+// Query pass on tensor cores (same conditions): dq~ plane, dout_gate, and one
+// partial record [dS, dz, dnorm_w] per (b, h, chunk of bwd_tc_query_chunks).
+int bwd_tc_query_chunks(const Problem &p);
+cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state, float *part,
+                         float *dqt, cudaStream_t st);
 unsigned bwd_device_error(bool reset);
 
 // ---- layer front end (tcgen05; gbla_project.cu): bf16 ----------------------
