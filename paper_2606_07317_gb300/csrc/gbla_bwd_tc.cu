@@ -90,6 +90,20 @@ __device__ __forceinline__ void report(unsigned code, const AbortFlag &ab) {
   ab.raise();
 }
 
+// As sm100::mbar_wait, but polling without the suspend hint: the roles of
+// these kernels hand work to each other every tile, and a suspended thread
+// can wake well after the phase completes.  Bounded by kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait_spin(uint64_t *bar, uint32_t parity,
+                                               const AbortFlag *ab) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((ab != nullptr && ab->raised()) || globaltimer() - t0 > kWaitLimitNs) return false;
+  }
+}
+#define mbar_wait mbar_wait_spin
+
 __device__ __forceinline__ int seq_len(const int32_t *seq_lens, int b, int N) {
   if (seq_lens == nullptr) return N;
   const int L = seq_lens[b];
@@ -474,7 +488,8 @@ constexpr int kQOffP = kQOffIn + kKStages * kQIn;          // 100352
 constexpr int kQOffDn = kQOffP + kKStages * kKTile;        // 133120
 constexpr int kQOffB = kQOffDn + kKStages * kKTile;        // 165888: SzT hi, lo, S hi, lo
 constexpr int kQOffZ = kQOffB + 2 * kQSzT + 2 * kKBTile;   // 202752: z [64], w [64]
-constexpr int kQOffDd = kQOffZ + 2 * kD * 4;               // float [2][128]: dden
+constexpr int kQOffTaps = kQOffZ + 2 * kD * 4;             // float4 [64]: q taps of the head
+constexpr int kQOffDd = kQOffTaps + kD * 16;               // float [2][128]: dden
 constexpr int kQOffStg = kQOffDd + kKStages * kKTok * 4;
 constexpr int kQOffBar = kQOffStg + kQE2Warps * kKStg;
 // in_full, in_empty, p_full, p_empty, a1_full, a1_empty, dn_full, dn_empty,
@@ -483,7 +498,7 @@ constexpr int kQBars = 10 * kKStages + 3;
 constexpr int kQOffMisc = kQOffBar + kQBars * 8;
 constexpr int kQSmem = kQOffMisc + 16 + 1024;
 static_assert(kQSmem <= 227 * 1024, "query-pass shared memory");
-static_assert(2 * kKTok * kD * 4 <= kKStages * kQIn, "end-of-chunk reduction space");
+static_assert(8 * kD * 4 <= kKStages * kQIn, "end-of-chunk reduction space");
 constexpr uint32_t kQA1 = 0, kQA2 = 256, kQA3 = 384;     // TMEM columns
 constexpr int kQRec = kD * kD + 2 * kD;            // dS, dz, dnw
 
@@ -497,7 +512,29 @@ struct QueryParams {
   int B, H, N, nck;
 };
 
-__device__ __forceinline__ float sigmoid_f(float x) { return 1.f / (1.f + expf(-x)); }
+// Fast-path sigmoid (a relative error near 1e-7, far inside the bf16 tolerance).
+__device__ __forceinline__ float sigmoid_f(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+
+// Column sums over the 32 rows of a warp (one row per lane) of n = 16 or 32
+// columns held one row per lane in x: recursive halving with shuffles, in a
+// fixed order.  n = 32: lane l returns the sum of column l; n = 16: lanes l
+// and l ^ 1 both return the sum of column l >> 1.  x is overwritten.
+template <int n>
+__device__ __forceinline__ float lane_colsum(float (&x)[n]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int o = 16, m = n; o > 0 && m > 1; o >>= 1, m >>= 1) {
+    const bool up = lane & o;
+#pragma unroll
+    for (int i = 0; i < m / 2; ++i) {
+      const float keep = up ? x[i + m / 2] : x[i];
+      const float send = up ? x[i] : x[i + m / 2];
+      x[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  if (n == 16) x[0] += __shfl_xor_sync(0xffffffffu, x[0], 1);
+  return x[0];
+}
 
 __global__ void __launch_bounds__(kQThreads, 1)
     tc_bwd_query_kernel(const QueryParams p, const __grid_constant__ CUtensorMap tm_q,
@@ -542,6 +579,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
     *(volatile int *)(smem + kQOffMisc + 4) = 0;
     fence_mbar_init();
   }
+  if (tid < kD)  // the head's q taps, read by the producers
+    *(float4 *)(smem + kQOffTaps + 16 * tid) =
+        __ldg((const float4 *)(p.conv_w + ((size_t)h * kD + tid) * kConvW));
   if (warp == kQTmaWarp && lane == 0) {
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_og);
@@ -577,7 +617,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
   } else if (warp < kQE1Warp0) {
     // ------------------------------------------------------------ producers: P = phi(conv(q))
     const int r = tid;
-    const float *cwq = p.conv_w + ((size_t)h * kD) * kConvW;
+    const uint32_t taps = smem_u32(smem + kQOffTaps);
     bool ok = true;
     for (int li = 0; li < nt && ok; ++li) {
       const int s = li % kKStages, ph = (li / kKStages) & 1;
@@ -596,7 +636,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
         for (int j = 0; j < kConvW; ++j) unpack8(lds_v4(rq + sw_off(r + j, c)), qx[j]);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float4 tq = __ldg((const float4 *)(cwq + (8 * c + e) * kConvW));
+          const uint4 tu = lds_v4(taps + 16 * (8 * c + e));
+          const float4 tq = make_float4(__uint_as_float(tu.x), __uint_as_float(tu.y),
+                                        __uint_as_float(tu.z), __uint_as_float(tu.w));
           const float qt = fmaf(tq.w, qx[3][e], fmaf(tq.z, qx[2][e], fmaf(tq.y, qx[1][e], tq.x * qx[0][e])));
           pv[e] = valid ? phi_f(qt) : 0.f;
         }
@@ -613,9 +655,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
   } else if (warp < kQE2Warp0) {
     // ------------------------------------------------------------ gated RMSNorm / readout backward
     const int q4 = warp & 3, row = 32 * q4 + lane;
-    float dnw[kD];
-#pragma unroll
-    for (int i = 0; i < kD; ++i) dnw[i] = 0.f;
+    float dnw4[4] = {0.f, 0.f, 0.f, 0.f};  // column 16 j + (lane >> 1) of the warp's rows
     bool ok = __all_sync(0xffffffffu, mbar_wait(b_full, 0, &ab));  // z and w in shared memory
     for (int li = 0; li < nt && ok; ++li) {
       const int s = li % kKStages, ph = (li / kKStages) & 1;
@@ -664,16 +704,17 @@ __global__ void __launch_bounds__(kQThreads, 1)
         unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
         unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
         tmem_ld_wait_regs(v);
-        float gq[16];
+        float gq[16], gw[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int d = 16 * j + i;
           const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
           const float w = ws[d];
           gq[i] = dy[i] * o * rr * w * sg * (1.f + og[i] * (1.f - sg));
-          dnw[d] = valid ? fmaf(dy[i] * o, rr * si, dnw[d]) : dnw[d];
+          gw[i] = valid ? dy[i] * o * (rr * si) : 0.f;
           uo = fmaf(dy[i] * w * si, o, uo);
         }
+        dnw4[j] += lane_colsum<16>(gw);
         if (valid) {
           float a[8], c[8];
 #pragma unroll
@@ -728,12 +769,13 @@ __global__ void __launch_bounds__(kQThreads, 1)
       }
     }
     if (!ok && !ab.raised()) report(512, ab);
-    // this thread's dnw row into the reduction space: the input ring is no
-    // longer read (the producers finished before the last tile's MMAs, and
+    // this warp's dnw column sums into the reduction space: the input ring is
+    // no longer read (the producers finished before the last tile's MMAs, and
     // this role read the last out_gate / dy rows above)
     float *red = (float *)(smem + kQOffIn);
+    if ((lane & 1) == 0)
 #pragma unroll
-    for (int i = 0; i < kD; ++i) red[row * kD + i] = dnw[i];
+      for (int j = 0; j < 4; ++j) red[q4 * kD + 16 * j + (lane >> 1)] = dnw4[j];
   } else if (warp < kQMmaWarp) {
     // ------------------------------------------------------------ dq~, dz; the B tiles
     const int q4 = warp & 3, row = 32 * q4 + lane, et = tid - kQE2Warp0 * 32;
@@ -776,9 +818,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
       named_barrier(2, 128);
       if (et == 0) mbar_arrive(b_full);
     }
-    float dz[kD];
-#pragma unroll
-    for (int i = 0; i < kD; ++i) dz[i] = 0.f;
+    float dz2[2] = {0.f, 0.f};  // column 32 part + lane of the warp's rows
     bool ok = true;
     for (int li = 0; li < nt && ok; ++li) {
       const int s = li % kKStages, ph = (li / kKStages) & 1;
@@ -802,6 +842,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&a2_empty[s]);
         }
+        float pz[32];
 #pragma unroll
         for (int cq = 0; cq < 4; ++cq) {
           float f[8];
@@ -809,10 +850,11 @@ __global__ void __launch_bounds__(kQThreads, 1)
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const int d = 32 * part + 8 * cq + e;
-            dz[d] = fmaf(f[e], dd, dz[d]);
+            pz[8 * cq + e] = f[e] * dd;
             v[8 * cq + e] = (v[8 * cq + e] + zs[d] * dd) * fminf(f[e], 1.f);
           }
         }
+        dz2[part] += lane_colsum<32>(pz);
 #pragma unroll
         for (int j = 0; j < 8; ++j)
           sts_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4),
@@ -835,9 +877,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
     if (!ok && !ab.raised()) report(1024, ab);
     // the last dnum tile followed the last out_gate / dy reads, so the input
     // ring is free here too
-    float *red = (float *)(smem + kQOffIn) + kKTok * kD;
-#pragma unroll
-    for (int i = 0; i < kD; ++i) red[row * kD + i] = dz[i];
+    float *red = (float *)(smem + kQOffIn) + 4 * kD;
+    red[q4 * kD + lane] = dz2[0];
+    red[q4 * kD + 32 + lane] = dz2[1];
   } else if (warp == kQMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -900,11 +942,11 @@ __global__ void __launch_bounds__(kQThreads, 1)
   __syncthreads();
   float *rec = p.part + ((size_t)bh * p.nck + chunk) * kQRec;
   const float *red = (const float *)(smem + kQOffIn);
-  if (tid < kD) {
+  if (tid < kD) {  // sums over the four lane quarters in order
     float a = 0.f, w = 0.f;
-    for (int r = 0; r < kKTok; ++r) {
-      w += red[r * kD + tid];
-      a += red[kKTok * kD + r * kD + tid];
+    for (int q = 0; q < 4; ++q) {
+      w += red[q * kD + tid];
+      a += red[4 * kD + q * kD + tid];
     }
     rec[kD * kD + tid] = a;
     rec[kD * kD + kD + tid] = w;
