@@ -137,7 +137,9 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
 __device__ __forceinline__ uint32_t sw_off(int r, int c) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
 }
-__device__ __forceinline__ float phi_f(float x) { return x > 0.f ? x + 1.f : expf(x); }
+// phi = elu + 1 with the fast exponential (its ~1e-7 relative error is far
+// below the bf16 rounding its uses apply).
+__device__ __forceinline__ float phi_f(float x) { return x > 0.f ? x + 1.f : __expf(x); }
 
 __global__ void __launch_bounds__(kKThreads, 1)
     tc_bwd_key_kernel(const KeyParams p, const __grid_constant__ CUtensorMap tm_k,
@@ -582,6 +584,53 @@ __global__ void __launch_bounds__(kQThreads, 1)
   if (tid < kD)  // the head's q taps, read by the producers
     *(float4 *)(smem + kQOffTaps + 16 * tid) =
         __ldg((const float4 *)(p.conv_w + ((size_t)h * kD + tid) * kConvW));
+  {
+    // B tiles from S (every thread; contiguous 32-byte reads of S rows, all in
+    // flight together): S as bf16 hi + lo with rows d, K = e (for dP), and its
+    // transpose [S^T | z] with rows e, K = d, row 64 = z, rows 65..79 zero (for
+    // [num | den]); K-major, 128B-swizzled.
+    const float *S = p.state + (size_t)bh * (kD * kD + kD);
+    const uint32_t bb = smem_u32(smem + kQOffB);
+    uint8_t *bsz = smem + kQOffB;
+    for (int u = tid; u < kD * (kD / 8); u += kQThreads) {
+      const int rr = u >> 3, cc = u & 7;  // S row rr, columns 8 cc ..
+      const float4 x0 = __ldg((const float4 *)(S + rr * kD + 8 * cc));
+      const float4 x1 = __ldg((const float4 *)(S + rr * kD + 8 * cc + 4));
+      const float x[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+      float hi[8], lo[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        hi[e] = __bfloat162float(__float2bfloat16_rn(x[e]));
+        lo[e] = x[e] - hi[e];
+      }
+      sts_v4(bb + 2 * kQSzT + sw_off(rr, cc), pack8(hi));
+      sts_v4(bb + 2 * kQSzT + kKBTile + sw_off(rr, cc), pack8(lo));
+      // transposed: element (row e = 8 cc + i, K = rr)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint32_t o = sw_off(8 * cc + i, rr >> 3) + (rr & 7) * 2;
+        *(__nv_bfloat16 *)(bsz + o) = __float2bfloat16_rn(hi[i]);
+        *(__nv_bfloat16 *)(bsz + kQSzT + o) = __float2bfloat16_rn(lo[i]);
+      }
+    }
+    for (int u = tid; u < 16 * (kD / 8); u += kQThreads) {  // rows 64 (z) .. 79
+      const int rr = kD + (u >> 3), cc = u & 7;
+      float hi[8], lo[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float x = rr == kD ? S[kD * kD + 8 * cc + e] : 0.f;
+        hi[e] = __bfloat162float(__float2bfloat16_rn(x));
+        lo[e] = x - hi[e];
+      }
+      sts_v4(bb + sw_off(rr, cc), pack8(hi));
+      sts_v4(bb + kQSzT + sw_off(rr, cc), pack8(lo));
+    }
+    if (tid < kD) {
+      ((float *)(smem + kQOffZ))[tid] = S[kD * kD + tid];
+      ((float *)(smem + kQOffZ))[kD + tid] = p.norm_w[(size_t)h * kD + tid];
+    }
+    fence_proxy_async_smem();
+  }
   if (warp == kQTmaWarp && lane == 0) {
     tma_prefetch_desc(&tm_q);
     tma_prefetch_desc(&tm_og);
@@ -656,7 +705,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
     // ------------------------------------------------------------ gated RMSNorm / readout backward
     const int q4 = warp & 3, row = 32 * q4 + lane;
     float dnw4[4] = {0.f, 0.f, 0.f, 0.f};  // column 16 j + (lane >> 1) of the warp's rows
-    bool ok = __all_sync(0xffffffffu, mbar_wait(b_full, 0, &ab));  // z and w in shared memory
+    bool ok = true;
     for (int li = 0; li < nt && ok; ++li) {
       const int s = li % kKStages, ph = (li / kKStages) & 1;
       const int t = c0 + li * kKTok + row;
@@ -704,7 +753,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
         unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
         unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
         tmem_ld_wait_regs(v);
-        float gq[16], gw[16];
+        float gq[16], gw[16], uu[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int d = 16 * j + i;
@@ -712,9 +761,20 @@ __global__ void __launch_bounds__(kQThreads, 1)
           const float w = ws[d];
           gq[i] = dy[i] * o * rr * w * sg * (1.f + og[i] * (1.f - sg));
           gw[i] = valid ? dy[i] * o * (rr * si) : 0.f;
-          uo = fmaf(dy[i] * w * si, o, uo);
+          uu[i] = dy[i] * w * si;
+          uo = fmaf(uu[i], o, uo);
         }
         dnw4[j] += lane_colsum<16>(gw);
+        {  // u replaces this row's out_gate values (read only by this thread from here on)
+          float a[8], c[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            a[i] = uu[i];
+            c[i] = uu[8 + i];
+          }
+          sts_v4(ogt + sw_off(row, 2 * j), pack8(a));
+          sts_v4(ogt + sw_off(row, 2 * j + 1), pack8(c));
+        }
         if (valid) {
           float a[8], c[8];
 #pragma unroll
@@ -732,20 +792,16 @@ __global__ void __launch_bounds__(kQThreads, 1)
       float doo = 0.f;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        float v[16], og[16], dy[16];
+        float v[16], uu[16];
         tmem_ld16(ta + 16 * j, v);
-        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(og));
-        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(og + 8));
-        unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
-        unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(uu));
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(uu + 8));
         tmem_ld_wait_regs(v);
         float dn[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const int d = 16 * j + i;
-          const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
-          const float u = dy[i] * ws[d] * si;
-          const float dO = rr * u - r3 * o * uo;
+          const float o = v[i] * inv;
+          const float dO = rr * uu[i] - r3 * o * uo;
           doo = fmaf(dO, o, doo);
           dn[i] = valid ? dO * inv : 0.f;
         }
@@ -778,46 +834,8 @@ __global__ void __launch_bounds__(kQThreads, 1)
       for (int j = 0; j < 4; ++j) red[q4 * kD + 16 * j + (lane >> 1)] = dnw4[j];
   } else if (warp < kQMmaWarp) {
     // ------------------------------------------------------------ dq~, dz; the B tiles
-    const int q4 = warp & 3, row = 32 * q4 + lane, et = tid - kQE2Warp0 * 32;
-    const uint32_t bb = smem_u32(smem + kQOffB);
+    const int q4 = warp & 3, row = 32 * q4 + lane;
     const uint32_t stg = smem_u32(smem + kQOffStg + (warp - kQE2Warp0) * kKStg);
-    {
-      // [S^T | z] (80 rows: B[e][d] = S[d][e], B[64][d] = z[d], zero rows) and S
-      // (B[d][e] = S[d][e]) as bf16 hi + lo, K-major 128B-swizzled
-      const float *S = p.state + (size_t)bh * (kD * kD + kD);
-      for (int u = et; u < 80 * (kD / 8); u += 128) {
-        const int rr = u >> 3, cc = u & 7;
-        float hi[8], lo[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int d = 8 * cc + e;
-          const float x = rr < kD ? S[d * kD + rr] : (rr == kD ? S[kD * kD + d] : 0.f);
-          hi[e] = __bfloat162float(__float2bfloat16_rn(x));
-          lo[e] = x - hi[e];
-        }
-        sts_v4(bb + sw_off(rr, cc), pack8(hi));
-        sts_v4(bb + kQSzT + sw_off(rr, cc), pack8(lo));
-      }
-      for (int u = et; u < kD * (kD / 8); u += 128) {
-        const int rr = u >> 3, cc = u & 7;
-        float hi[8], lo[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const float x = S[rr * kD + 8 * cc + e];
-          hi[e] = __bfloat162float(__float2bfloat16_rn(x));
-          lo[e] = x - hi[e];
-        }
-        sts_v4(bb + 2 * kQSzT + sw_off(rr, cc), pack8(hi));
-        sts_v4(bb + 2 * kQSzT + kKBTile + sw_off(rr, cc), pack8(lo));
-      }
-      if (et < kD) {
-        ((float *)(smem + kQOffZ))[et] = S[kD * kD + et];
-        ((float *)(smem + kQOffZ))[kD + et] = p.norm_w[(size_t)h * kD + et];
-      }
-      fence_proxy_async_smem();
-      named_barrier(2, 128);
-      if (et == 0) mbar_arrive(b_full);
-    }
     float dz2[2] = {0.f, 0.f};  // column 32 part + lane of the warp's rows
     bool ok = true;
     for (int li = 0; li < nt && ok; ++li) {
@@ -887,10 +905,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
       const uint32_t id2 = idesc_bf16_f32(kKTok, kD, 0, 0);
       const uint32_t id3 = idesc_bf16_f32(kKTok, kD, 1, 1);
       const uint32_t bb = smem_u32(smem + kQOffB);
-      bool ok = mbar_wait(b_full, 0, &ab);
+      bool ok = true;
       auto mma1 = [&](int li) -> bool {
-        const int s = li % kKStages, ph = (li / kKStages) & 1;
-        if (!mbar_wait(&p_full[s], ph, &ab) || !mbar_wait(&a1_empty[s], ph ^ 1, &ab)) return false;
+        const int s = li % kKStages;
         tc_fence_after();
         const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
 #pragma unroll
@@ -902,17 +919,11 @@ __global__ void __launch_bounds__(kQThreads, 1)
         mma_commit(&a1_full[s]);
         return true;
       };
-      if (ok && nt > 0) ok = mma1(0);
-      for (int li = 0; li < nt && ok; ++li) {
-        const int s = li % kKStages, ph = (li / kKStages) & 1;
-        if (li + 1 < nt && !mma1(li + 1)) {
-          ok = false;
-          break;
-        }
-        if (!mbar_wait(&dn_full[s], ph, &ab) || !mbar_wait(&a2_empty[s], ph ^ 1, &ab)) {
-          ok = false;
-          break;
-        }
+      // MMA1 of a tile needs its P tile and a free [num | den] buffer; MMA2 / MMA3
+      // need the tile's dnum.  Whichever is ready is issued, so neither waits
+      // behind the other.
+      auto mma23 = [&](int li) {
+        const int s = li % kKStages;
         tc_fence_after();
         const uint32_t dn = smem_u32(smem + kQOffDn + s * kKTile);
         const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
@@ -931,6 +942,32 @@ __global__ void __launch_bounds__(kQThreads, 1)
         mma_commit(&a2_full[s]);
         mma_commit(&dn_empty[s]);
         mma_commit(&p_empty[s]);
+      };
+      int n1 = 0, n2 = 0;
+      uint64_t tw = globaltimer();
+      while (ok && n2 < nt) {
+        bool moved = false;
+        if (n1 < nt) {
+          const int s = n1 % kKStages, ph = (n1 / kKStages) & 1;
+          if (mbar_try_wait(&p_full[s], ph) && mbar_try_wait(&a1_empty[s], ph ^ 1)) {
+            mma1(n1);
+            ++n1;
+            moved = true;
+          }
+        }
+        if (n2 < n1) {
+          const int s = n2 % kKStages, ph = (n2 / kKStages) & 1;
+          if (mbar_try_wait(&dn_full[s], ph) && mbar_try_wait(&a2_empty[s], ph ^ 1)) {
+            mma23(n2);
+            ++n2;
+            moved = true;
+          }
+        }
+        if (moved) {
+          tw = globaltimer();
+        } else if (ab.raised() || globaltimer() - tw > kWaitLimitNs) {
+          ok = false;
+        }
       }
       if (!ok && !ab.raised()) report(2048, ab);
       mma_commit(a3_full);
