@@ -849,7 +849,14 @@ __global__ void __launch_bounds__(kQThreads, 1)
       const uint32_t ta = tmem + ((uint32_t)(32 * q4) << 16) + kQA2 + kD * s;
       const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
       const float dd = dds[s * kKTok + row];
-#pragma unroll 1
+      // this row's P (packed bf16) into registers, so the P stage goes back to
+      // the producers before the row is processed
+      uint4 prow[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) prow[c] = lds_v4(pt + sw_off(row, c));
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_empty[s]);
+#pragma unroll
       for (int part = 0; part < 2; ++part) {
         float v[32];
         tmem_ld16(ta + 32 * part, *reinterpret_cast<float(*)[16]>(v));
@@ -864,7 +871,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
 #pragma unroll
         for (int cq = 0; cq < 4; ++cq) {
           float f[8];
-          unpack8(lds_v4(pt + sw_off(row, 4 * part + cq)), f);
+          unpack8(prow[4 * part + cq], f);
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
             const int d = 32 * part + 8 * cq + e;
@@ -889,8 +896,6 @@ __global__ void __launch_bounds__(kQThreads, 1)
         }
         __syncwarp();
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_empty[s]);  // P rows read
     }
     if (!ok && !ab.raised()) report(1024, ab);
     // the last dnum tile followed the last out_gate / dy reads, so the input
