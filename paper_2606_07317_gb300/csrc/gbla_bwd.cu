@@ -18,7 +18,8 @@
 // Launches (all on the caller's stream, after the forward state S, z has been
 // formed by the forward's own state path):
 //   bwd_gate_stats   per (b, h): M = max a, Ltot = sum e^{a - M} (g_j = e^{a_j-M}/Ltot)
-//   bwd_query        per (b, h, chunk): 5' and 6' per token; dq~ to scratch;
+//   bwd_query        per (b, h, chunk): 5' and 6' per token; dq~ to scratch
+//                    (the dq~, dk~, dv~ planes are stored in the I/O dtype);
 //                    chunk partials of dS, dz and the norm-weight gradient
 //   bwd_reduce_state per (b, h): fixed-order sums of the partials; c
 //   bwd_key          per (b, h, chunk): 4' and 3' per token; dk~, dv~ to scratch
@@ -39,6 +40,12 @@ constexpr int kChunk = 256;   // tokens per block
 __device__ __forceinline__ float ldf(const float *p, size_t i) { return p[i]; }
 __device__ __forceinline__ float ldf(const __nv_bfloat16 *p, size_t i) {
   return __bfloat162float(p[i]);
+}
+// Read-only loads (non-coherent path): the compiler may move them across
+// stores to buffers of the same element type.
+__device__ __forceinline__ float ldg_f(const float *p, size_t i) { return __ldg(p + i); }
+__device__ __forceinline__ float ldg_f(const __nv_bfloat16 *p, size_t i) {
+  return __bfloat162float(__ldg(p + i));
 }
 __device__ __forceinline__ void stf(float *p, size_t i, float x) { p[i] = x; }
 __device__ __forceinline__ void stf(__nv_bfloat16 *p, size_t i, float x) {
@@ -192,7 +199,7 @@ __global__ void __launch_bounds__(kNT) bwd_query(
     const T *__restrict__ q, const T *__restrict__ og, const T *__restrict__ dy,
     const float *__restrict__ conv_w, const float *__restrict__ norm_w,
     const float *__restrict__ state, const int32_t *__restrict__ seq_lens, float eps,
-    T *__restrict__ dog, float *__restrict__ dqt, float *__restrict__ part, int H, int N,
+    T *__restrict__ dog, T *__restrict__ dqt, float *__restrict__ part, int H, int N,
     int nck) {
   constexpr int F = D * D + D;
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
@@ -295,7 +302,7 @@ __global__ void __launch_bounds__(kNT) bwd_query(
       const float dd = sDd[tl];
       if (t < t1) {
         const size_t row = (((size_t)b * N + t) * H + h) * D + c;
-        dqt[row] = (dP[u] + z[c] * dd) * dphi(qt[u]) * (t < tv ? 1.f : 0.f);
+        stf(dqt, row, (dP[u] + z[c] * dd) * dphi(qt[u]) * (t < tv ? 1.f : 0.f));
       }
       dz = fmaf(P[u], dd, dz);
     }
@@ -355,8 +362,8 @@ __global__ void __launch_bounds__(kNT) bwd_key(
     const T *__restrict__ k, const T *__restrict__ v, const T *__restrict__ gate,
     const float *__restrict__ conv_w, const float2 *__restrict__ stats,
     const float *__restrict__ state, const float *__restrict__ red,
-    const int32_t *__restrict__ seq_lens, T *__restrict__ dgate, float *__restrict__ dkt,
-    float *__restrict__ dvt, int H, int N) {
+    const int32_t *__restrict__ seq_lens, T *__restrict__ dgate, T *__restrict__ dkt,
+    T *__restrict__ dvt, int H, int N) {
   constexpr int F = D * D + D;
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   extern __shared__ float sm[];
@@ -420,8 +427,8 @@ __global__ void __launch_bounds__(kNT) bwd_key(
       if (t < t1) {
         const size_t row = (((size_t)b * N + t) * H + h) * D + c;
         const bool valid = t < tv;
-        dkt[row] = valid ? g[u] * dK[u] * dphi(kt[u]) : 0.f;
-        dvt[row] = valid ? dvv[u] : 0.f;
+        stf(dkt, row, valid ? g[u] * dK[u] * dphi(kt[u]) : 0.f);
+        stf(dvt, row, valid ? dvv[u] : 0.f);
       }
       x[u] = pk[u] * dK[u];
     }
@@ -444,7 +451,7 @@ __global__ void __launch_bounds__(kNT) bwd_key(
 template <typename T, int D>
 __global__ void __launch_bounds__(kNT) bwd_conv(
     const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v,
-    const float *__restrict__ dxt, const float *__restrict__ conv_w,
+    const T *__restrict__ dxt, const float *__restrict__ conv_w,
     const int32_t *__restrict__ seq_lens, T *__restrict__ dq, T *__restrict__ dk,
     T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck) {
   constexpr int RUNS = kNT / D, RL = kChunk / RUNS;
@@ -453,7 +460,7 @@ __global__ void __launch_bounds__(kNT) bwd_conv(
   const int tid = threadIdx.x, run = tid / D, c = tid % D;
   const T *x = s == 0 ? q : (s == 1 ? k : v);
   T *dx = s == 0 ? dq : (s == 1 ? dk : dv);
-  const float *dxs = dxt + (size_t)s * ((size_t)gridDim.y / H) * N * H * D;
+  const T *dxs = dxt + (size_t)s * ((size_t)gridDim.y / H) * N * H * D;
   const int L = clamp_len(seq_lens, b, N);
   const int ta = chunk * kChunk + run * RL, tb = min(ta + RL, N);
   float w[kConvW], dw[kConvW];
@@ -470,8 +477,8 @@ __global__ void __launch_bounds__(kNT) bwd_conv(
 #pragma unroll
   for (int i = 0; i < kConvW; ++i) {
     const int u = ta + i, s2 = ta - (kConvW - 1) + i;
-    d[i] = u < L ? dxs[col + (size_t)u * rs] : 0.f;
-    xw[i] = (s2 >= 0 && s2 < L) ? ldf(x, col + (size_t)s2 * rs) : 0.f;
+    d[i] = u < L ? ldg_f(dxs, col + (size_t)u * rs) : 0.f;
+    xw[i] = (s2 >= 0 && s2 < L) ? ldg_f(x, col + (size_t)s2 * rs) : 0.f;
   }
   for (int t = ta; t < tb; t += 4) {
     float dd[8], xx[8];  // dx~_{t..t+7}, x_{t-3..t+4}
@@ -480,8 +487,8 @@ __global__ void __launch_bounds__(kNT) bwd_conv(
       dd[i] = d[i];
       xx[i] = xw[i];
       const int un = t + 4 + i, sn = t + 1 + i;
-      dd[4 + i] = un < L ? dxs[col + (size_t)un * rs] : 0.f;
-      xx[4 + i] = sn < L ? ldf(x, col + (size_t)sn * rs) : 0.f;
+      dd[4 + i] = un < L ? ldg_f(dxs, col + (size_t)un * rs) : 0.f;
+      xx[4 + i] = sn < L ? ldg_f(x, col + (size_t)sn * rs) : 0.f;
     }
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
@@ -550,7 +557,8 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   const int nck = (N + kChunk - 1) / kChunk;
   const BwdLayout lay = bwd_layout(p);
   float2 *stats = (float2 *)(scratch + lay.stats);
-  float *qpart = scratch + lay.qpart, *red = scratch + lay.red, *dxt = scratch + lay.dxt;
+  float *qpart = scratch + lay.qpart, *red = scratch + lay.red;
+  T *dxt = (T *)(scratch + lay.dxt);  // dq~, dk~, dv~ planes in the storage dtype
   float *wpart = scratch + lay.wpart;
   const float *state = scratch + lay.state;
   const size_t plane = (size_t)B * N * H * D;

@@ -71,16 +71,16 @@ struct BwdLayout {
 BwdLayout bwd_layout(const Problem &p);
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
 // Key pass on tensor cores (gbla_bwd_tc.cu): bf16, D = 64, sm_103.  Writes the
-// dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz.
+// bf16 dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz.
 bool bwd_tc_key_supported(const Problem &p);
 cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
-                       const float *state, const float *red, float *cval, float *dkt,
-                       float *dvt, cudaStream_t st);
+                       const float *state, const float *red, float *cval, void *dkt,
+                       void *dvt, cudaStream_t st);
 // Query pass on tensor cores (same conditions): dq~ plane, dout_gate, and one
 // partial record [dS, dz, dnorm_w] per (b, h, chunk of bwd_tc_query_chunks).
 int bwd_tc_query_chunks(const Problem &p);
 cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state, float *part,
-                         float *dqt, cudaStream_t st);
+                         void *dqt, cudaStream_t st);
 unsigned bwd_device_error(bool reset);
 
 // ---- layer front end (tcgen05; gbla_project.cu): bf16 ----------------------
