@@ -17,7 +17,8 @@
 //
 // Launches (all on the caller's stream, after the forward state S, z has been
 // formed by the forward's own state path):
-//   bwd_gate_stats   per (b, h): M = max a, Ltot = sum e^{a - M} (g_j = e^{a_j-M}/Ltot)
+//   bwd_gate_split / bwd_gate_join  per (b, h): M = max a, Ltot = sum e^{a - M}
+//                    (g_j = e^{a_j-M}/Ltot), over sequence splits, then combined
 //   bwd_query        per (b, h, chunk): 5' and 6' per token; dq~ to scratch
 //                    (the dq~, dk~, dv~ planes are stored in the I/O dtype);
 //                    chunk partials of dS, dz and the norm-weight gradient
@@ -162,31 +163,44 @@ __device__ __forceinline__ float conv_at(const T *x, size_t rs, int t, const flo
 }
 
 // ---------------------------------------------------------------- gate stats
+// Per (b, h): M = max_j a_j and Ltot = sum_j e^{a_j - M} over j < L_b, in two
+// steps.  bwd_gate_split: block (bh, split) walks its kGateSplitLen tokens once,
+// each thread keeping a running (max, sum) pair (the sum rescaled when the max
+// grows), and combines the 256 pairs in a fixed tree order.  bwd_gate_join:
+// the splits of one (b, h) in index order.
+constexpr int kGateSplits = 16;
+__device__ __forceinline__ float2 ms_join(float2 x, float2 y) {  // (max, sum) pairs
+  const float m = fmaxf(x.x, y.x);
+  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
+  return make_float2(m, x.y * expf(x.x - m) + y.y * expf(y.x - m));
+}
 template <typename T>
-__global__ void __launch_bounds__(256) bwd_gate_stats(const T *__restrict__ gate,
+__global__ void __launch_bounds__(256) bwd_gate_split(const T *__restrict__ gate,
                                                       const int32_t *__restrict__ seq_lens,
-                                                      float2 *__restrict__ stats, int H, int N) {
-  const int bh = blockIdx.x, b = bh / H, h = bh % H;
+                                                      float2 *__restrict__ part, int H, int N) {
+  const int bh = blockIdx.x, sp = blockIdx.y, b = bh / H, h = bh % H;
   const int L = clamp_len(seq_lens, b, N);
-  __shared__ float red[8];
-  float m = -INFINITY;
-  for (int t = threadIdx.x; t < L; t += 256) m = fmaxf(m, ldf(gate, ((size_t)b * N + t) * H + h));
-  m = warp_max(m);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+  const int len = (N + kGateSplits - 1) / kGateSplits;
+  const int ta = sp * len, tb = min(ta + len, L);
+  float2 acc = make_float2(-INFINITY, 0.f);
+  for (int t = ta + threadIdx.x; t < tb; t += 256)
+    acc = ms_join(acc, make_float2(ldf(gate, ((size_t)b * N + t) * H + h), 1.f));
+  __shared__ float2 red[256];
+  red[threadIdx.x] = acc;
   __syncthreads();
-  float M = red[0];
-  for (int i = 1; i < 8; ++i) M = fmaxf(M, red[i]);
-  __syncthreads();
-  float l = 0.f;
-  for (int t = threadIdx.x; t < L; t += 256) l += expf(ldf(gate, ((size_t)b * N + t) * H + h) - M);
-  l = warp_sum(l);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = l;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int i = 0; i < 8; ++i) s += red[i];
-    stats[bh] = make_float2(M, s);
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) red[threadIdx.x] = ms_join(red[threadIdx.x], red[threadIdx.x + w]);
+    __syncthreads();
   }
+  if (threadIdx.x == 0) part[(size_t)bh * kGateSplits + sp] = red[0];
+}
+__global__ void __launch_bounds__(256) bwd_gate_join(const float2 *__restrict__ part,
+                                                     float2 *__restrict__ stats, int BH) {
+  const int bh = blockIdx.x * 256 + threadIdx.x;
+  if (bh >= BH) return;
+  float2 acc = make_float2(-INFINITY, 0.f);
+  for (int sp = 0; sp < kGateSplits; ++sp) acc = ms_join(acc, part[(size_t)bh * kGateSplits + sp]);
+  stats[bh] = acc;
 }
 
 // ---------------------------------------------------------------- query pass
@@ -523,7 +537,10 @@ __global__ void __launch_bounds__(kNT) bwd_conv(
 
 // ---------------------------------------------------------------- weight reductions
 // dconv_w[s][h][c][i] = sum_b sum_chunk wpart (nck chunks);  dnorm_w[h][c] = sum_b
-// sum_chunk qpart.dnw (nckq query-pass records per (b, h))
+// sum_chunk qpart.dnw (nckq query-pass records per (b, h)).  A block takes 32
+// consecutive outputs (one per lane); its 8 warps take interleaved slices of
+// the (b, chunk) partials, read coalesced across the lanes, and the 8 warp
+// sums are added in warp order.
 template <int D>
 __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wpart,
                                                     const float *__restrict__ qpart,
@@ -531,23 +548,33 @@ __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wp
                                                     float *__restrict__ dnorm_w, int B, int H,
                                                     int nck, int nckq) {
   const int total_w = 3 * H * D * kConvW;
-  for (int idx = blockIdx.x * 256 + threadIdx.x; idx < total_w + H * D;
-       idx += gridDim.x * 256) {
-    float a = 0.f;
-    if (idx < total_w) {
-      const int s = idx / (H * D * kConvW), r = idx % (H * D * kConvW);
-      const int h = r / (D * kConvW), ci = r % (D * kConvW);
-      for (int b = 0; b < B; ++b)
-        for (int ch = 0; ch < nck; ++ch)
-          a += wpart[(((size_t)s * B * H + (size_t)b * H + h) * nck + ch) * D * kConvW + ci];
-      dconv_w[idx] = a;
-    } else {
-      const int j = idx - total_w, h = j / D, cc = j % D;
-      for (int b = 0; b < B; ++b)
-        for (int ch = 0; ch < nckq; ++ch)
-          a += qpart[(((size_t)b * H + h) * nckq + ch) * qrec<D>() + D * D + D + cc];
-      dnorm_w[j] = a;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int idx = blockIdx.x * 32 + lane;
+  __shared__ float part[8][32];
+  float a = 0.f;
+  if (idx < total_w) {
+    const int s = idx / (H * D * kConvW), r = idx % (H * D * kConvW);
+    const int h = r / (D * kConvW), ci = r % (D * kConvW);
+    const int n = B * nck;
+    for (int k = warp; k < n; k += 8) {
+      const int b = k / nck, ch = k % nck;
+      a += wpart[(((size_t)s * B * H + (size_t)b * H + h) * nck + ch) * D * kConvW + ci];
     }
+  } else if (idx < total_w + H * D) {
+    const int j = idx - total_w, h = j / D, cc = j % D;
+    const int n = B * nckq;
+    for (int k = warp; k < n; k += 8) {
+      const int b = k / nckq, ch = k % nckq;
+      a += qpart[(((size_t)b * H + h) * nckq + ch) * qrec<D>() + D * D + D + cc];
+    }
+  }
+  part[warp][lane] = a;
+  __syncthreads();
+  if (warp == 0) {
+    float t = 0.f;
+    for (int w = 0; w < 8; ++w) t += part[w][lane];
+    if (idx < total_w) dconv_w[idx] = t;
+    else if (idx < total_w + H * D) dnorm_w[idx - total_w] = t;
   }
 }
 
@@ -563,8 +590,11 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   const float *state = scratch + lay.state;
   const size_t plane = (size_t)B * N * H * D;
   cudaError_t e;
-  bwd_gate_stats<T><<<BH, 256, 0, st>>>((const T *)a.gate, p.seq_lens, stats, H, N);
-  count_launch();
+  float2 *gpart = (float2 *)(scratch + lay.gpart);
+  bwd_gate_split<T><<<dim3(BH, kGateSplits), 256, 0, st>>>((const T *)a.gate, p.seq_lens, gpart,
+                                                           H, N);
+  bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(gpart, stats, BH);
+  count_launch(2);
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   const size_t smq = sizeof(float) * (2 * D * D + D + 4 * D * kTB + kTB + kNT / 32 * TPT);
   const bool tc = bwd_tc_key_supported(p);  // bf16, D = 64, sm_103: both token passes on tcgen05
@@ -605,7 +635,7 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
       (T *)a.dk, (T *)a.dv, wpart, H, N, nck);
   count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
-  bwd_reduce_w<D><<<(nw + 255) / 256, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
+  bwd_reduce_w<D><<<(nw + 31) / 32, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
                                                      nck, nckq);
   count_launch();
   return cudaGetLastError();
@@ -621,7 +651,8 @@ BwdLayout bwd_layout(const Problem &p) {
   BwdLayout l;
   l.state = 0;
   l.stats = up(l.state + BH * F);
-  l.qpart = up(l.stats + 2 * BH);
+  l.gpart = up(l.stats + 2 * BH);
+  l.qpart = up(l.gpart + 2 * BH * kGateSplits);
   l.red = up(l.qpart + BH * nck * (D * D + 2 * D));
   l.cval = up(l.red + BH * (F + 1));
   l.dxt = up(l.cval + BH);

@@ -66,7 +66,7 @@ struct BwdArgs {
 // partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
 // gradient partials.
 struct BwdLayout {
-  size_t state, stats, qpart, red, cval, dxt, wpart, total;
+  size_t state, stats, gpart, qpart, red, cval, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
