@@ -458,79 +458,112 @@ __global__ void __launch_bounds__(kNT) bwd_key(
 }
 
 // ---------------------------------------------------------------- Conv1D backward
-// Stream s = blockIdx.z (0 q, 1 k, 2 v): dx_t = sum_i w_i dx~_{t+3-i} (t + 3 - i
-// < L) and the chunk partials of dw_i = sum_t dx~_t x_{t-3+i} for the D channels
-// of (b, h).  Thread (run, c) walks kChunk / (kNT / D) consecutive tokens of
-// channel c with sliding windows of dx~ and x.
+// Stream s = blockIdx.z (0 q, 1 k, 2 v) over a block of kConvChunk tokens of
+// one (b, h): dx_t = sum_i w_i dx~_{t+3-i} (terms with t + 3 - i >= L dropped;
+// dx_t = 0 for t >= L) and the block's partials of dw_i = sum_t dx~_t x_{t-3+i}.
+// Thread (run, g) walks kConvChunk / RUNS consecutive tokens of channels
+// 4g .. 4g+3 with sliding windows (x of the 3 tokens before, dx~ of the 3
+// after), every token's 4 channels one vector load; the runs' tap partials are
+// then added in run order.
+constexpr int kConvChunk = 1024;
+constexpr int kConvCh = 4;  // channels per thread
+__device__ __forceinline__ void ld4(const float *p, float (&f)[4]) {
+  const float4 a = __ldg((const float4 *)p);
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+}
+__device__ __forceinline__ void ld4(const __nv_bfloat16 *p, float (&f)[4]) {
+  const uint2 u = __ldg((const uint2 *)p);
+  f[0] = __uint_as_float(u.x << 16); f[1] = __uint_as_float(u.x & 0xFFFF0000u);
+  f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
+}
+__device__ __forceinline__ void st4(float *p, const float (&f)[4]) {
+  *(float4 *)p = make_float4(f[0], f[1], f[2], f[3]);
+}
+__device__ __forceinline__ void st4(__nv_bfloat16 *p, const float (&f)[4]) {
+  const __nv_bfloat162 a = __floats2bfloat162_rn(f[0], f[1]), b = __floats2bfloat162_rn(f[2], f[3]);
+  *(uint2 *)p = make_uint2(*reinterpret_cast<const uint32_t *>(&a),
+                           *reinterpret_cast<const uint32_t *>(&b));
+}
+
 template <typename T, int D>
-__global__ void __launch_bounds__(kNT) bwd_conv(
+__global__ void __launch_bounds__(kNT, 2) bwd_conv(
     const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v,
     const T *__restrict__ dxt, const float *__restrict__ conv_w,
     const int32_t *__restrict__ seq_lens, T *__restrict__ dq, T *__restrict__ dk,
     T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck) {
-  constexpr int RUNS = kNT / D, RL = kChunk / RUNS;
-  __shared__ float sw[RUNS][D][kConvW];
+  constexpr int G = D / kConvCh, RUNS = kNT / G, RL = kConvChunk / RUNS;
+  __shared__ float sw[RUNS][D * kConvW];
   const int chunk = blockIdx.x, bh = blockIdx.y, s = blockIdx.z, b = bh / H, h = bh % H;
-  const int tid = threadIdx.x, run = tid / D, c = tid % D;
+  const int tid = threadIdx.x, g = tid % G, run = tid / G;
   const T *x = s == 0 ? q : (s == 1 ? k : v);
   T *dx = s == 0 ? dq : (s == 1 ? dk : dv);
   const T *dxs = dxt + (size_t)s * ((size_t)gridDim.y / H) * N * H * D;
   const int L = clamp_len(seq_lens, b, N);
-  const int ta = chunk * kChunk + run * RL, tb = min(ta + RL, N);
-  float w[kConvW], dw[kConvW];
+  const int ta = chunk * kConvChunk + run * RL, tb = min(ta + RL, N);
+  float w[kConvCh][kConvW], dw[kConvCh][kConvW];
 #pragma unroll
-  for (int i = 0; i < kConvW; ++i) {
-    w[i] = conv_w[((size_t)(s * H + h) * D + c) * kConvW + i];
-    dw[i] = 0.f;
+  for (int c = 0; c < kConvCh; ++c) {
+    const float4 t4 =
+        __ldg((const float4 *)(conv_w + ((size_t)(s * H + h) * D + kConvCh * g + c) * kConvW));
+    w[c][0] = t4.x; w[c][1] = t4.y; w[c][2] = t4.z; w[c][3] = t4.w;
+#pragma unroll
+    for (int i = 0; i < kConvW; ++i) dw[c][i] = 0.f;
   }
   const size_t rs = (size_t)H * D;
-  const size_t col = ((size_t)b * N * H + h) * D + c;
-  // windows: d[i] = dx~_{t+i}, xw[i] = x_{t-3+i} (i = 0..3); four tokens a step,
-  // the next four tokens' values loaded together
-  float d[kConvW], xw[kConvW];
+  const size_t col = ((size_t)b * N * H + h) * D + kConvCh * g;
+  auto ldx = [&](int t, float (&f)[kConvCh]) {  // x_t, zero outside [0, L)
+    if (t >= 0 && t < L) ld4(x + col + (size_t)t * rs, f);
+    else
 #pragma unroll
-  for (int i = 0; i < kConvW; ++i) {
-    const int u = ta + i, s2 = ta - (kConvW - 1) + i;
-    d[i] = u < L ? ldg_f(dxs, col + (size_t)u * rs) : 0.f;
-    xw[i] = (s2 >= 0 && s2 < L) ? ldg_f(x, col + (size_t)s2 * rs) : 0.f;
+      for (int c = 0; c < kConvCh; ++c) f[c] = 0.f;
+  };
+  auto ldd = [&](int t, float (&f)[kConvCh]) {  // dx~_t, zero outside [0, L)
+    if (t >= 0 && t < L) ld4(dxs + col + (size_t)t * rs, f);
+    else
+#pragma unroll
+      for (int c = 0; c < kConvCh; ++c) f[c] = 0.f;
+  };
+  // xm[i] = x_{t-3+i} (i = 0..2), dm[i] = dx~_{t+i} (i = 0..2)
+  float xm[3][kConvCh], dm[3][kConvCh];
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    ldx(ta - 3 + i, xm[i]);
+    ldd(ta + i, dm[i]);
   }
-  for (int t = ta; t < tb; t += 4) {
-    float dd[8], xx[8];  // dx~_{t..t+7}, x_{t-3..t+4}
+#pragma unroll 4
+  for (int t = ta; t < tb; ++t) {
+    float xc[kConvCh], dn[kConvCh], o[kConvCh];
+    ldx(t, xc);      // x_t
+    ldd(t + 3, dn);  // dx~_{t+3}
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      dd[i] = d[i];
-      xx[i] = xw[i];
-      const int un = t + 4 + i, sn = t + 1 + i;
-      dd[4 + i] = un < L ? ldg_f(dxs, col + (size_t)un * rs) : 0.f;
-      xx[4 + i] = sn < L ? ldg_f(x, col + (size_t)sn * rs) : 0.f;
+    for (int c = 0; c < kConvCh; ++c) {
+      // dx_t = w0 dx~_{t+3} + w1 dx~_{t+2} + w2 dx~_{t+1} + w3 dx~_t
+      float a = w[c][0] * dn[c];
+      a = fmaf(w[c][1], dm[2][c], a);
+      a = fmaf(w[c][2], dm[1][c], a);
+      a = fmaf(w[c][3], dm[0][c], a);
+      o[c] = t < L ? a : 0.f;
+      // dw_i += dx~_t x_{t-3+i}  (dx~_t = 0 past L)
+      dw[c][0] = fmaf(dm[0][c], xm[0][c], dw[c][0]);
+      dw[c][1] = fmaf(dm[0][c], xm[1][c], dw[c][1]);
+      dw[c][2] = fmaf(dm[0][c], xm[2][c], dw[c][2]);
+      dw[c][3] = fmaf(dm[0][c], xc[c], dw[c][3]);
     }
+    st4(dx + col + (size_t)t * rs, o);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int tj = t + j;
-      if (tj < tb) {
-        float a = 0.f;
-        if (tj < L) {
-#pragma unroll
-          for (int i = 0; i < kConvW; ++i) a = fmaf(w[i], dd[j + kConvW - 1 - i], a);
-#pragma unroll
-          for (int i = 0; i < kConvW; ++i) dw[i] = fmaf(dd[j], xx[j + i], dw[i]);
-        }
-        stf(dx, col + (size_t)tj * rs, a);
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      d[i] = dd[4 + i];
-      xw[i] = xx[4 + i];
+    for (int c = 0; c < kConvCh; ++c) {
+      xm[0][c] = xm[1][c]; xm[1][c] = xm[2][c]; xm[2][c] = xc[c];
+      dm[0][c] = dm[1][c]; dm[1][c] = dm[2][c]; dm[2][c] = dn[c];
     }
   }
 #pragma unroll
-  for (int i = 0; i < kConvW; ++i) sw[run][c][i] = dw[i];
+  for (int c = 0; c < kConvCh; ++c)
+#pragma unroll
+    for (int i = 0; i < kConvW; ++i) sw[run][(kConvCh * g + c) * kConvW + i] = dw[c][i];
   __syncthreads();
   for (int j = tid; j < D * kConvW; j += kNT) {
-    const int cc = j / kConvW, i = j % kConvW;
     float a = 0.f;
-    for (int r = 0; r < RUNS; ++r) a += sw[r][cc][i];
+    for (int r = 0; r < RUNS; ++r) a += sw[r][j];
     wpart[(((size_t)s * gridDim.y + bh) * nck + chunk) * D * kConvW + j] = a;
   }
 }
@@ -630,13 +663,14 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
                                       dxt + plane, dxt + 2 * plane, H, N);
   count_launch();
   }
-  bwd_conv<T, D><<<dim3(nck, BH, 3), kNT, 0, st>>>(
+  const int nckc = (N + kConvChunk - 1) / kConvChunk;  // Conv1D backward blocks per (b, h)
+  bwd_conv<T, D><<<dim3(nckc, BH, 3), kNT, 0, st>>>(
       (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
-      (T *)a.dk, (T *)a.dv, wpart, H, N, nck);
+      (T *)a.dk, (T *)a.dv, wpart, H, N, nckc);
   count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
   bwd_reduce_w<D><<<(nw + 31) / 32, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
-                                                     nck, nckq);
+                                                     nckc, nckq);
   count_launch();
   return cudaGetLastError();
 }
