@@ -723,22 +723,11 @@ __global__ void __launch_bounds__(kQThreads, 1)
         den = v4[0];
       }
       const float inv = valid ? 1.f / den : 0.f;
-      // pass 1: mean O^2
-      float ss = 0.f;
-#pragma unroll 1
-      for (int j = 0; j < 4; ++j) {
-        float v[16];
-        tmem_ld16(ta + 16 * j, v);
-        tmem_ld_wait_regs(v);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float o = v[i] * inv;
-          ss = fmaf(o, o, ss);
-        }
-      }
-      const float rr = rsqrtf(ss * (1.f / kD) + p.eps);
-      // pass 2: dog, dnw, u . O
-      float uo = 0.f;
+      // pass 1 (nothing here needs r): sum O^2, u . O with u = dy w silu(og), and
+      // two per-element factors that replace this row's out_gate and dy values
+      // (read only by this thread from here on): A = dy w silu'(og) (dog = A O r)
+      // and Bv = dy silu(og) (dnorm_w term Bv O r, u = Bv w)
+      float ss = 0.f, uo = 0.f;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         float v[16], og[16], dy[16];
@@ -748,30 +737,60 @@ __global__ void __launch_bounds__(kQThreads, 1)
         unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(dy));
         unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(dy + 8));
         tmem_ld_wait_regs(v);
-        float gq[16], gw[16], uu[16];
+        float fa[16], fb[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int d = 16 * j + i;
           const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
           const float w = ws[d];
-          gq[i] = dy[i] * o * rr * w * sg * (1.f + og[i] * (1.f - sg));
-          gw[i] = valid ? dy[i] * o * (rr * si) : 0.f;
-          uu[i] = dy[i] * w * si;
-          uo = fmaf(uu[i], o, uo);
+          ss = fmaf(o, o, ss);
+          uo = fmaf(dy[i] * w * si, o, uo);
+          fa[i] = dy[i] * w * sg * (1.f + og[i] * (1.f - sg));
+          fb[i] = dy[i] * si;
+        }
+        float a[8], c[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          a[i] = fa[i];
+          c[i] = fa[8 + i];
+        }
+        sts_v4(ogt + sw_off(row, 2 * j), pack8(a));
+        sts_v4(ogt + sw_off(row, 2 * j + 1), pack8(c));
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          a[i] = fb[i];
+          c[i] = fb[8 + i];
+        }
+        sts_v4(dyt + sw_off(row, 2 * j), pack8(a));
+        sts_v4(dyt + sw_off(row, 2 * j + 1), pack8(c));
+      }
+      const float rr = rsqrtf(ss * (1.f / kD) + p.eps);
+      const float r3 = rr * rr * rr * (1.f / kD);
+      // pass 2: dog, dnorm_w, dnum (bf16 A / B tile); dO . O in closed form:
+      // sum_d (r u_d - r3 O_d (u . O)) O_d = r (u . O) - r3 (u . O) sum O^2
+      const float doo = rr * uo - r3 * uo * ss;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float v[16], fa[16], fb[16];
+        tmem_ld16(ta + 16 * j, v);
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(fa));
+        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(fa + 8));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(fb));
+        unpack8(lds_v4(dyt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(fb + 8));
+        tmem_ld_wait_regs(v);
+        float gq[16], gw[16], dn[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int d = 16 * j + i;
+          const float o = v[i] * inv, orr = o * rr;
+          gq[i] = fa[i] * orr;
+          gw[i] = valid ? fb[i] * orr : 0.f;
+          const float dO = rr * (fb[i] * ws[d]) - r3 * o * uo;
+          dn[i] = valid ? dO * inv : 0.f;
         }
         dnw4[j] += lane_colsum<16>(gw);
-        {  // u replaces this row's out_gate values (read only by this thread from here on)
-          float a[8], c[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            a[i] = uu[i];
-            c[i] = uu[8 + i];
-          }
-          sts_v4(ogt + sw_off(row, 2 * j), pack8(a));
-          sts_v4(ogt + sw_off(row, 2 * j + 1), pack8(c));
-        }
+        float a[8], c[8];
         if (valid) {
-          float a[8], c[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             a[i] = gq[i];
@@ -781,26 +800,6 @@ __global__ void __launch_bounds__(kQThreads, 1)
           *(uint4 *)dst = pack8(a);
           *(uint4 *)(dst + 8) = pack8(c);
         }
-      }
-      // pass 3: dO, dnum (bf16 A / B tile), dO . O
-      const float r3 = rr * rr * rr * (1.f / kD);
-      float doo = 0.f;
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float v[16], uu[16];
-        tmem_ld16(ta + 16 * j, v);
-        unpack8(lds_v4(ogt + sw_off(row, 2 * j)), *reinterpret_cast<float(*)[8]>(uu));
-        unpack8(lds_v4(ogt + sw_off(row, 2 * j + 1)), *reinterpret_cast<float(*)[8]>(uu + 8));
-        tmem_ld_wait_regs(v);
-        float dn[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float o = v[i] * inv;
-          const float dO = rr * uu[i] - r3 * o * uo;
-          doo = fmaf(dO, o, doo);
-          dn[i] = valid ? dO * inv : 0.f;
-        }
-        float a[8], c[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           a[i] = dn[i];
