@@ -140,8 +140,10 @@ gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
  *   dconv_w [3, H, D, W] fp32 (q, k, v taps);   dnorm_w [H, D] fp32.
  * Rows t >= L_b of dq, dk, dv, dout_gate and dgate are written as 0; dconv_w
  * and dnorm_w are overwritten with sums over the batch.  The forward state is
- * recomputed inside (nothing is kept from a forward call).  fp32 arithmetic;
- * every sum runs in a fixed order (bitwise reproducible).  Asynchronous on
+ * recomputed inside (nothing is kept from a forward call).  fp32 arithmetic
+ * (for bf16 with D = 64 the token contractions run on tensor cores with bf16
+ * operands, S and dS split into bf16 hi + lo, fp32 accumulation); every sum
+ * runs in a fixed order (bitwise reproducible).  Asynchronous on
  * `stream`; scratch comes from the library's stream-ordered pool
  * (GBLA_ERR_ALLOC when it cannot).  Same error codes as gbla_forward.
  */
