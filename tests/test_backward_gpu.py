@@ -88,6 +88,20 @@ def test_backward_padding_rows_zero_and_deterministic():
     _check(a, _oracle(inp, dy), "bf16")
 
 
+def test_backward_ragged_chunks_bf16():
+    """Sequences spanning several 1024-token chunks of the tensor-core query pass,
+    lengths that are not multiples of the 128-token tile, an empty sequence and
+    a chunk lying wholly in the padding; padded rows zero."""
+    w = custom(B=3, H=2, N=2500, D=64, dtype="bf16", seed=29, seq_lens=[2500, 1100, 0])
+    inp = make_inputs(w, "cuda")
+    dy = _dy(inp, 30)
+    got = _run(inp, dy)
+    for n in ("dq", "dk", "dv", "dout_gate"):
+        assert torch.all(got[n][1, 1100:] == 0) and torch.all(got[n][2] == 0), n
+    assert torch.all(got["dgate"][1, 1100:] == 0) and torch.all(got["dgate"][2] == 0)
+    _check(got, _oracle(inp, dy), "bf16")
+
+
 def test_backward_rejects_aliasing():
     w = custom(B=1, H=2, N=64, D=64, dtype="bf16", seed=27)
     inp = make_inputs(w, "cuda")
