@@ -86,7 +86,7 @@ def kernel_source_hash() -> str:
     traffic profiles/traffic.json records)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_07317_gb300", "csrc")
-    for name in ("gbla_tc.cu", "gbla_sm100.cuh", "gbla_internal.cuh"):
+    for name in ("gbla_tc.cu", "gbla_sm100.cuh"):
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
