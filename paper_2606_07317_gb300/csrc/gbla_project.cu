@@ -8,7 +8,8 @@
 // input), rows 4 H D + h the gate logits w_g of head h.
 //
 // tc_project_kernel: persistent, one CTA per SM, 128-token tiles of one
-// sequence taken round robin.  Roles:
+// sequence; each CTA takes an equal run of (tile, 256-column chunk) units.
+// Roles:
 //  - four converter warps compute X~ for all d channels of a tile in fp32
 //    (16-byte loads of the X rows plus 3 rows of history) and store it as
 //    bf16 into the K-major A operand: one 128B-swizzled 64-channel block per
@@ -111,28 +112,48 @@ __device__ __forceinline__ int seq_len(const int32_t *seq_lens, int b, int N) {
   return L < 0 ? 0 : (L > N ? N : L);
 }
 
-// Tiles of this CTA in order: i = blockIdx.x, + gridDim.x, ..., skipping tiles
-// that lie wholly in the padding (t0 >= L_b).
+// Work is split into units (tile, 256-column chunk of q, k, v, out_gate); the
+// gate chunk of a tile goes with the tile's last unit.  CTA c takes the
+// contiguous units [c U / G, (c + 1) U / G), U = tiles x chunks, so every CTA
+// gets the same number of chunks within one; a tile cut between two CTAs has
+// its X~ computed by both.  TileIt walks this CTA's tiles in order, skipping
+// tiles that lie wholly in the padding (t0 >= L_b), with the chunk range
+// nlo .. nend (nend = the gate chunk when the range reaches the last unit).
 struct TileIt {
-  int i, b, t0, L;
+  int i, b, t0, L, nlo, nend;
 };
+__device__ __forceinline__ void unit_range(const ProjParams &p, long long &u0, long long &u1) {
+  const long long U = (long long)p.B * p.tps * p.nmain;
+  u0 = U * blockIdx.x / gridDim.x;
+  u1 = U * (blockIdx.x + 1) / gridDim.x;
+}
 __device__ __forceinline__ bool tile_valid(const ProjParams &p, TileIt &t) {
-  const int T = p.B * p.tps;
-  while (t.i < T) {
+  long long u0, u1;
+  unit_range(p, u0, u1);
+  if (u0 >= u1) return false;
+  const long long ilast = (u1 - 1) / p.nmain;
+  while (t.i <= ilast) {
     t.b = t.i / p.tps;
     t.t0 = (t.i % p.tps) * kPTok;
     t.L = seq_len(p.seq_lens, t.b, p.N);
-    if (t.t0 < t.L) return true;
-    t.i += gridDim.x;
+    if (t.t0 < t.L) {
+      t.nlo = t.i == u0 / p.nmain ? (int)(u0 % p.nmain) : 0;
+      const int nhi = t.i == ilast ? (int)((u1 - 1) % p.nmain) : p.nmain - 1;
+      t.nend = nhi == p.nmain - 1 ? p.nmain : nhi;
+      return true;
+    }
+    ++t.i;
   }
   return false;
 }
 __device__ __forceinline__ bool tile_first(const ProjParams &p, TileIt &t) {
-  t.i = blockIdx.x;
+  long long u0, u1;
+  unit_range(p, u0, u1);
+  t.i = (int)(u0 / p.nmain);
   return tile_valid(p, t);
 }
 __device__ __forceinline__ bool tile_next(const ProjParams &p, TileIt &t) {
-  t.i += gridDim.x;
+  ++t.i;
   return tile_valid(p, t);
 }
 
@@ -156,7 +177,6 @@ __global__ void __launch_bounds__(kPThreads, 1)
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nkb = p.d / kPKB;
-  const int nch = p.nmain + 1;
 
   uint64_t *bars = (uint64_t *)(smem + kPOffBar);
   uint64_t *a_full = bars, *a_empty = bars + kPMaxKB;
@@ -201,7 +221,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       bool ok = true;
       TileIt t = t0;
       do {
-        for (int n = 0; n < nch && ok; ++n)
+        for (int n = t.nlo; n <= t.nend && ok; ++n)
           for (int kb = 0; kb < nkb && ok; ++kb)
             for (int half = 0; half < 2; ++half) {
               const int s = bs % kPBStages;
@@ -230,7 +250,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
       bool ok = true;
       TileIt t = t0;
       do {
-        for (int n = 0; n < nch && ok; ++n) {
+        for (int n = t.nlo; n <= t.nend && ok; ++n) {
           const int buf = cs & 1;
           if (!mbar_wait(&acc_empty[buf], ((cs >> 1) & 1) ^ 1, &ab)) {
             ok = false;
@@ -240,7 +260,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
           const uint32_t dacc = tmem + buf * kPChunk;
           const uint32_t idesc = n < p.nmain ? id_main : id_gate;
           for (int kb = 0; kb < nkb && ok; ++kb) {
-            if (n == 0 && !mbar_wait(&a_full[kb], tseq & 1, &ab)) {
+            if (n == t.nlo && !mbar_wait(&a_full[kb], tseq & 1, &ab)) {
               ok = false;
               break;
             }
@@ -261,7 +281,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
               mma_commit(&b_empty[s]);
               ++bs;
             }
-            if (ok && n == nch - 1) mma_commit(&a_empty[kb]);
+            if (ok && n == t.nend) mma_commit(&a_empty[kb]);
           }
           if (ok) mma_commit(&acc_full[buf]);
           ++cs;
@@ -366,7 +386,7 @@ __global__ void __launch_bounds__(kPThreads, 1)
     TileIt t = t0;
     do {
       const size_t tok0 = (size_t)t.b * p.N + t.t0;  // token index of tile row 0
-      for (int n = 0; n < nch; ++n, ++cs) {
+      for (int n = t.nlo; n <= t.nend; ++n, ++cs) {
         const int buf = cs & 1;
         if (!mbar_wait(&acc_full[buf], (cs >> 1) & 1, &ab)) {
           ok = false;
@@ -512,8 +532,8 @@ cudaError_t tc_project(const ProjProblem &pp, const void *x, const float *conv_x
   int dev = 0, sms = 1;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const long long tiles = (long long)pp.B * p.tps;
-  const int grid = (int)(tiles < sms ? tiles : sms);
+  const long long units = (long long)pp.B * p.tps * p.nmain;
+  const int grid = (int)(units < sms ? units : sms);
   tc_project_kernel<<<grid, kPThreads, kPSmemBytes, st>>>(p, tm_w);
   count_launch();
   return cudaGetLastError();
