@@ -245,8 +245,14 @@ __global__ void __launch_bounds__(kPThreads, 1)
     if (lane == 0) {
       const uint32_t id_main = idesc_bf16_f32(kPTok, kPChunk, 0, 0);
       const uint32_t id_gate = idesc_bf16_f32(kPTok, p.ngate, 0, 0);
-      const uint32_t abase = smem_u32(smem + kPOffA), bbase = smem_u32(smem + kPOffB);
-      int bs = 0, cs = 0, tseq = 0;
+      // The loop is kept short (this warp shares its sub-partition with busy
+      // converter and epilogue warps): descriptors of block 0 / stage 0 are
+      // advanced by byte offsets (the address field is the byte address >> 4
+      // and shared addresses stay below 256 KB, so adding never carries into
+      // the next field), and ring positions are stepped rather than divided.
+      const uint64_t ad0 = sw128_desc(smem_u32(smem + kPOffA), 16, 1024);
+      const uint64_t bd0 = sw64_desc(smem_u32(smem + kPOffB), 512);
+      int bstage = 0, bphase = 0, cs = 0, tseq = 0;
       bool ok = true;
       TileIt t = t0;
       do {
@@ -259,29 +265,30 @@ __global__ void __launch_bounds__(kPThreads, 1)
           tc_fence_after();
           const uint32_t dacc = tmem + buf * kPChunk;
           const uint32_t idesc = n < p.nmain ? id_main : id_gate;
+          const bool first = n == t.nlo, last = n == t.nend;
           for (int kb = 0; kb < nkb && ok; ++kb) {
-            if (n == t.nlo && !mbar_wait(&a_full[kb], tseq & 1, &ab)) {
+            if (first && !mbar_wait(&a_full[kb], tseq & 1, &ab)) {
               ok = false;
               break;
             }
+            const uint64_t adk = ad0 + (uint64_t)((kb * kPABlock) >> 4);
+#pragma unroll
             for (int half = 0; half < 2; ++half) {
-              const int s = bs % kPBStages;
-              if (!mbar_wait(&b_full[s], (bs / kPBStages) & 1, &ab)) {
+              if (!mbar_wait(&b_full[bstage], bphase, &ab)) {
                 ok = false;
                 break;
               }
               tc_fence_after();
-#pragma unroll
-              for (int k2 = 0; k2 < 2; ++k2) {
-                const uint64_t ad =
-                    sw128_desc(abase + kb * kPABlock + (half * 2 + k2) * 32, 16, 1024);
-                const uint64_t bd = sw64_desc(bbase + s * kPBStage + k2 * 32, 512);
-                mma_bf16(dacc, ad, bd, idesc, (kb | half | k2) != 0);
+              const uint64_t bds = bd0 + (uint64_t)((bstage * kPBStage) >> 4);
+              mma_bf16(dacc, adk + (uint64_t)((half * 64) >> 4), bds, idesc, (kb | half) != 0);
+              mma_bf16(dacc, adk + (uint64_t)((half * 64 + 32) >> 4), bds + 2, idesc, 1);
+              mma_commit(&b_empty[bstage]);
+              if (++bstage == kPBStages) {
+                bstage = 0;
+                bphase ^= 1;
               }
-              mma_commit(&b_empty[s]);
-              ++bs;
             }
-            if (ok && n == t.nend) mma_commit(&a_empty[kb]);
+            if (ok && last) mma_commit(&a_empty[kb]);
           }
           if (ok) mma_commit(&acc_full[buf]);
           ++cs;
