@@ -499,7 +499,7 @@ constexpr int kQBars = 10 * kKStages + 3;
 constexpr int kQOffMisc = kQOffBar + kQBars * 8;
 constexpr int kQSmem = kQOffMisc + 16 + 1024;
 static_assert(kQSmem <= 227 * 1024, "query-pass shared memory");
-static_assert(8 * kD * 4 <= kKStages * kQIn, "end-of-chunk reduction space");
+static_assert(16 * kD * 4 <= kKStages * kQIn, "end-of-chunk reduction space");
 constexpr uint32_t kQA1 = 0, kQA2 = 256, kQA3 = 384;     // TMEM columns
 constexpr int kQRec = kD * kD + 2 * kD;            // dS, dz, dnw
 
@@ -559,7 +559,6 @@ __global__ void __launch_bounds__(kQThreads, 1)
   uint32_t *tmem_slot = (uint32_t *)(smem + kQOffMisc);
   const AbortFlag ab{smem_u32(smem + kQOffMisc + 4)};
   const float *zs = (const float *)(smem + kQOffZ), *ws = zs + kD;
-  float *dds = (float *)(smem + kQOffDd);
 
   if (tid == 0) {
     for (int i = 0; i < kKStages; ++i) {
@@ -642,6 +641,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const size_t prs = (size_t)H * kD;                         // plane row stride
   const size_t prow0 = (((size_t)b * N + c0) * H + h) * kD;  // plane row of the chunk's token 0
+  // column sums of the epilogue groups (kept until every role is done):
+  // dnorm_w column 16 j + (lane >> 1) and dz column 32 part + lane of a warp's rows
+  float dnw4[4] = {0.f, 0.f, 0.f, 0.f};
+  float dz2[2] = {0.f, 0.f};
 
   if (warp == kQTmaWarp) {
     // ------------------------------------------------------------ TMA: q, out_gate, dy
@@ -700,12 +703,16 @@ __global__ void __launch_bounds__(kQThreads, 1)
       }
     }
     if (!ok && !ab.raised()) report(256, ab);
-  } else if (warp < kQE2Warp0) {
-    // ------------------------------------------------------------ gated RMSNorm / readout backward
+  } else if (warp < kQMmaWarp) {
+    // ------------------------------------------------------------ epilogue groups
+    // Two groups of four warps (one per TMEM lane quarter, one token row per
+    // thread) take the even and the odd tiles: for each, the gated-RMSNorm /
+    // readout backward (dog, dnum, dden, dnorm_w sums), then, once the dP / dS
+    // MMAs are done, dq~ and the dz sums.  The groups overlap one another.
+    const int grp = (warp - kQE1Warp0) >> 2;
     const int q4 = warp & 3, row = 32 * q4 + lane;
-    float dnw4[4] = {0.f, 0.f, 0.f, 0.f};  // column 16 j + (lane >> 1) of the warp's rows
     bool ok = true;
-    for (int li = 0; li < nt && ok; ++li) {
+    for (int li = grp; li < nt && ok; li += 2) {
       const int s = li % kKStages, ph = (li / kKStages) & 1;
       const int t = c0 + li * kKTok + row;
       const bool valid = t < L;
@@ -812,7 +819,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
         sts_v4(dnt + sw_off(row, 2 * j), pack8(a));
         sts_v4(dnt + sw_off(row, 2 * j + 1), pack8(c));
       }
-      dds[s * kKTok + row] = valid ? -doo * inv : 0.f;
+      const float dd = valid ? -doo * inv : 0.f;
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
@@ -821,32 +828,14 @@ __global__ void __launch_bounds__(kQThreads, 1)
         mbar_arrive(&dn_full[s]);
         mbar_arrive(&in_empty[s]);
       }
-    }
-    if (!ok && !ab.raised()) report(512, ab);
-    // this warp's dnw column sums into the reduction space: the input ring is
-    // no longer read (the producers finished before the last tile's MMAs, and
-    // this role read the last out_gate / dy rows above)
-    float *red = (float *)(smem + kQOffIn);
-    if ((lane & 1) == 0)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) red[q4 * kD + 16 * j + (lane >> 1)] = dnw4[j];
-  } else if (warp < kQMmaWarp) {
-    // ------------------------------------------------------------ dq~, dz; the B tiles
-    const int q4 = warp & 3, row = 32 * q4 + lane;
-    const uint32_t stg = smem_u32(smem + kQOffStg + (warp - kQE2Warp0) * kKStg);
-    float dz2[2] = {0.f, 0.f};  // column 32 part + lane of the warp's rows
-    bool ok = true;
-    for (int li = 0; li < nt && ok; ++li) {
-      const int s = li % kKStages, ph = (li / kKStages) & 1;
-      const bool w = mbar_wait(&a2_full[s], ph, &ab) && mbar_wait(&dn_full[s], ph, &ab);
-      if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
+      // ---- dq~ = (dP + z dden) phi'(q~) and dz, after the dP / dS MMAs
+      if (!__all_sync(0xffffffffu, mbar_wait(&a2_full[s], ph, &ab))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t ta = tmem + ((uint32_t)(32 * q4) << 16) + kQA2 + kD * s;
+      const uint32_t ta2 = tmem + ((uint32_t)(32 * q4) << 16) + kQA2 + kD * s;
       const uint32_t pt = smem_u32(smem + kQOffP + s * kKTile);
-      const float dd = dds[s * kKTok + row];
       // this row's P (packed bf16) into registers, so the P stage goes back to
       // the producers before the row is processed
       uint4 prow[8];
@@ -854,12 +843,12 @@ __global__ void __launch_bounds__(kQThreads, 1)
       for (int c = 0; c < 8; ++c) prow[c] = lds_v4(pt + sw_off(row, c));
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_empty[s]);
-      uint4 pk[8];
+      __nv_bfloat16 *dqrow = p.dqt + prow0 + (size_t)(li * kKTok + row) * prs;
 #pragma unroll
       for (int part = 0; part < 2; ++part) {
         float v[32];
-        tmem_ld16(ta + 32 * part, *reinterpret_cast<float(*)[16]>(v));
-        tmem_ld16(ta + 32 * part + 16, *reinterpret_cast<float(*)[16]>(v + 16));
+        tmem_ld16(ta2 + 32 * part, *reinterpret_cast<float(*)[16]>(v));
+        tmem_ld16(ta2 + 32 * part + 16, *reinterpret_cast<float(*)[16]>(v + 16));
         tmem_ld_wait();
         if (part == 1) {
           tc_fence_before();
@@ -880,29 +869,12 @@ __global__ void __launch_bounds__(kQThreads, 1)
           float a[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) a[e] = v[8 * cq + e];
-          pk[4 * part + cq] = pack8(a);
+          if (valid) *(uint4 *)(dqrow + 32 * part + 8 * cq) = pack8(a);
         }
         dz2[part] += lane_colsum<32>(pz);
       }
-      // the row's 64 bf16 values through the staging rows, 4 rows x 128 bytes a store
-#pragma unroll
-      for (int j = 0; j < 8; ++j) sts_v4(stg + lane * 128 + ((j ^ (lane & 7)) << 4), pk[j]);
-      __syncwarp();
-#pragma unroll
-      for (int it = 0; it < 8; ++it) {
-        const int rr = it * 4 + (lane >> 3), ch = lane & 7;
-        const uint4 val = lds_v4(stg + rr * 128 + ((ch ^ (rr & 7)) << 4));
-        const int tl = li * kKTok + 32 * q4 + rr;
-        if (c0 + tl < L) *(uint4 *)(p.dqt + prow0 + (size_t)tl * prs + ch * 8) = val;
-      }
-      __syncwarp();
     }
-    if (!ok && !ab.raised()) report(1024, ab);
-    // the last dnum tile followed the last out_gate / dy reads, so the input
-    // ring is free here too
-    float *red = (float *)(smem + kQOffIn) + 4 * kD;
-    red[q4 * kD + lane] = dz2[0];
-    red[q4 * kD + 32 + lane] = dz2[1];
+    if (!ok && !ab.raised()) report(512, ab);
   } else if (warp == kQMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -980,16 +952,28 @@ __global__ void __launch_bounds__(kQThreads, 1)
       if (!mbar_wait(fin, 0, nullptr)) report(4096, ab);
     }
   }
-  // every role is done: the partial record of this chunk (fixed summation order)
+  // every role is done: the input ring is free for the epilogue groups' column
+  // sums, then the partial record of this chunk (fixed summation order)
+  __syncthreads();
+  if (warp >= kQE1Warp0 && warp < kQMmaWarp) {
+    const int grp = (warp - kQE1Warp0) >> 2, q4 = warp & 3;
+    float *red = (float *)(smem + kQOffIn) + grp * 8 * kD;
+    if ((lane & 1) == 0)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) red[q4 * kD + 16 * j + (lane >> 1)] = dnw4[j];
+    red[4 * kD + q4 * kD + lane] = dz2[0];
+    red[4 * kD + q4 * kD + 32 + lane] = dz2[1];
+  }
   __syncthreads();
   float *rec = p.part + ((size_t)bh * p.nck + chunk) * kQRec;
   const float *red = (const float *)(smem + kQOffIn);
-  if (tid < kD) {  // sums over the four lane quarters in order
+  if (tid < kD) {  // sums over the two groups and four lane quarters in order
     float a = 0.f, w = 0.f;
-    for (int q = 0; q < 4; ++q) {
-      w += red[q * kD + tid];
-      a += red[4 * kD + q * kD + tid];
-    }
+    for (int g = 0; g < 2; ++g)
+      for (int q = 0; q < 4; ++q) {
+        w += red[g * 8 * kD + q * kD + tid];
+        a += red[g * 8 * kD + 4 * kD + q * kD + tid];
+      }
     rec[kD * kD + tid] = a;
     rec[kD * kD + kD + tid] = w;
   }
