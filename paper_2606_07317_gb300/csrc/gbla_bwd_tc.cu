@@ -65,7 +65,9 @@ constexpr int kKOffB = kKOffA + kKStages * kKAStage;         // 167936: dS hi, l
 constexpr int kKOffG = kKOffB + 4 * kKBTile;                 // 200704: float [2][128]
 constexpr int kKOffDz = kKOffG + kKStages * kKTok * 4;       // float [64]
 constexpr int kKOffStg = kKOffDz + kD * 4;
-constexpr int kKOffBar = kKOffStg + kKEpiWarps * kKStg;
+constexpr int kKOffTaps = kKOffStg + kKEpiWarps * kKStg;     // per producer warp: k, v taps
+constexpr int kKTapBytes = 2 * kD * 16;                      // float4 [2][64]
+constexpr int kKOffBar = kKOffTaps + kKProdWarps * kKTapBytes;
 // raw_full[2], raw_empty[2], a_full[2], a_empty[2], phi_full[2], phi_empty[2],
 // acc_full[2], acc_empty[2], b_full, b_free, fin
 constexpr int kKBars = 8 * kKStages + 3;
@@ -207,6 +209,9 @@ __global__ void __launch_bounds__(kKThreads, 1)
   } else if (warp < kKEpiWarp0) {
     // ------------------------------------------------------------ producers
     const int r = tid;  // tile row
+    // this warp's own copy of the head's k and v taps (rewritten when the
+    // (b, h) changes; a warp only reads the copy it wrote, so __syncwarp orders it)
+    const uint32_t taps = smem_u32(smem + kKOffTaps + warp * kKTapBytes);
     int li = 0, cur_bh = -1;
     float2 gs = make_float2(0.f, 1.f);
     bool ok = true;
@@ -217,6 +222,13 @@ __global__ void __launch_bounds__(kKThreads, 1)
       if (t.bh != cur_bh) {
         gs = p.stats[t.bh];
         cur_bh = t.bh;
+        __syncwarp();  // the previous head's taps are no longer read
+        for (int u = lane; u < 2 * kD; u += 32) {
+          const int str = 1 + u / kD, ch = u % kD;  // stream 1 (k) or 2 (v)
+          const float4 t4 = __ldg((const float4 *)(p.conv_w + ((size_t)(str * H + t.h) * kD + ch) * kConvW));
+          *(float4 *)(smem + kKOffTaps + warp * kKTapBytes + 16 * u) = t4;
+        }
+        __syncwarp();
       }
       const int tok = t.t0 + r;
       const bool valid = tok < t.L;
@@ -234,8 +246,6 @@ __global__ void __launch_bounds__(kKThreads, 1)
       const uint32_t rv = rk + kKRawHalf;
       const uint32_t av = smem_u32(smem + kKOffA + s * kKAStage);
       const uint32_t ak = av + kKTile, ap = av + 2 * kKTile;
-      const float *cwk = p.conv_w + ((size_t)(H + t.h) * kD) * kConvW;
-      const float *cwv = p.conv_w + ((size_t)(2 * H + t.h) * kD) * kConvW;
 #pragma unroll 2
       for (int c = 0; c < kD / 8; ++c) {
         float kx[kConvW][8], vx[kConvW][8];
@@ -247,8 +257,12 @@ __global__ void __launch_bounds__(kKThreads, 1)
         float vt[8], kh[8], ph[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
-          const float4 tk = __ldg((const float4 *)(cwk + (8 * c + e) * kConvW));
-          const float4 tv = __ldg((const float4 *)(cwv + (8 * c + e) * kConvW));
+          const uint4 uk = lds_v4(taps + 16 * (8 * c + e));
+          const uint4 uv = lds_v4(taps + 16 * (kD + 8 * c + e));
+          const float4 tk = make_float4(__uint_as_float(uk.x), __uint_as_float(uk.y),
+                                        __uint_as_float(uk.z), __uint_as_float(uk.w));
+          const float4 tv = make_float4(__uint_as_float(uv.x), __uint_as_float(uv.y),
+                                        __uint_as_float(uv.z), __uint_as_float(uv.w));
           const float kt = fmaf(tk.w, kx[3][e], fmaf(tk.z, kx[2][e], fmaf(tk.y, kx[1][e], tk.x * kx[0][e])));
           const float v1 = fmaf(tv.w, vx[3][e], fmaf(tv.z, vx[2][e], fmaf(tv.y, vx[1][e], tv.x * vx[0][e])));
           const float f = phi_f(kt);
