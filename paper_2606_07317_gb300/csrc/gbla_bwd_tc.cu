@@ -483,12 +483,12 @@ __global__ void __launch_bounds__(kKThreads, 1)
 // same tiles, M = 128 with the two 64-row halves of A equal, accumulated in
 // TMEM over the chunk).  Roles: a TMA warp (raw q tile with 3 rows of history,
 // out_gate and dy tiles), four producer warps (P = phi(conv(q)) in fp32, bf16
-// A tile), one MMA thread, four warps for the gated-RMSNorm / readout
-// backward (one token row per thread; dog, dnum, dden, per-row dnw sums) and
-// four for dq~ and the per-row dz sums; the chunk's dS, dz and dnw go to a
-// partial record.
-constexpr int kQC = 1024;                          // tokens per CTA
-constexpr int kQTiles = kQC / kKTok;               // 8
+// A tile), one MMA thread, and two groups of four warps taking the even and
+// the odd tiles (one token row per thread: the gated-RMSNorm / readout
+// backward, then dq~; per-warp dnw and dz sums); the chunk's dS, dz and dnw
+// go to a partial record.  One CTA per (b, h, chunk); the chunk length is
+// chosen on the host so that the chunks of all (b, h) fit one wave of CTAs
+// where they can (each CTA pays the pipeline fill once).
 constexpr int kQInQ = kKRawHalf;                   // 17408: raw q box
 constexpr int kQIn = kQInQ + 2 * kKTile;           // + out_gate, dy tiles: 50176
 constexpr int kQSzT = 80 * 128;                    // [S^T | z] tile: 80 rows
@@ -525,6 +525,7 @@ struct QueryParams {
   float *part;                           // [B*H][nck][kQRec]
   float eps;
   int B, H, N, nck;
+  int ctiles;  // 128-token tiles per chunk
 };
 
 // Fast-path sigmoid (a relative error near 1e-7, far inside the bf16 tolerance).
@@ -561,9 +562,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
   const int H = p.H, N = p.N;
   const int chunk = blockIdx.x, bh = blockIdx.y, b = bh / H, h = bh % H;
   const int L = seq_len(p.seq_lens, b, N);
-  const int c0 = chunk * kQC;
+  const int c0 = chunk * p.ctiles * kKTok;
   // valid tiles of this chunk: t0 = c0 + 128 j < min(L, N)
-  const int nt = L > c0 ? min(kQTiles, (L - c0 + kKTok - 1) / kKTok) : 0;
+  const int nt = L > c0 ? min(p.ctiles, (L - c0 + kKTok - 1) / kKTok) : 0;
 
   uint64_t *bars = (uint64_t *)(smem + kQOffBar);
   uint64_t *in_full = bars, *in_empty = bars + 2, *p_full = bars + 4, *p_empty = bars + 6;
@@ -1119,7 +1120,23 @@ cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
   return cudaGetLastError();
 }
 
-int bwd_tc_query_chunks(const Problem &p) { return (p.N + kQC - 1) / kQC; }
+// Tiles per query-pass chunk: as few chunks per (b, h) as keep all chunks in
+// one wave of one CTA per SM (at least 2 tiles, so the records never outnumber
+// the 256-token chunks the scratch layout provides for).
+static int bwd_tc_query_tiles(const Problem &p) {
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int tps = (p.N + kKTok - 1) / kKTok;
+  const int BH = p.B * p.H;
+  const int per = sms / BH > 1 ? sms / BH : 1;  // chunks per (b, h)
+  const int ct = (tps + per - 1) / per;
+  return ct < 2 ? 2 : ct;
+}
+int bwd_tc_query_chunks(const Problem &p) {
+  const int ct = bwd_tc_query_tiles(p), tps = (p.N + kKTok - 1) / kKTok;
+  return (tps + ct - 1) / ct;
+}
 
 cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state, float *part,
                          void *dqt, cudaStream_t st) {
@@ -1147,6 +1164,7 @@ cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state,
   qp.H = p.H;
   qp.N = p.N;
   qp.nck = bwd_tc_query_chunks(p);
+  qp.ctiles = bwd_tc_query_tiles(p);
   if ((e = cudaFuncSetAttribute(tc_bwd_query_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kQSmem)) != cudaSuccess)
     return e;
