@@ -42,12 +42,6 @@ __device__ __forceinline__ float ldf(const float *p, size_t i) { return p[i]; }
 __device__ __forceinline__ float ldf(const __nv_bfloat16 *p, size_t i) {
   return __bfloat162float(p[i]);
 }
-// Read-only loads (non-coherent path): the compiler may move them across
-// stores to buffers of the same element type.
-__device__ __forceinline__ float ldg_f(const float *p, size_t i) { return __ldg(p + i); }
-__device__ __forceinline__ float ldg_f(const __nv_bfloat16 *p, size_t i) {
-  return __bfloat162float(__ldg(p + i));
-}
 __device__ __forceinline__ void stf(float *p, size_t i, float x) { p[i] = x; }
 __device__ __forceinline__ void stf(__nv_bfloat16 *p, size_t i, float x) {
   p[i] = __float2bfloat16_rn(x);
@@ -64,12 +58,6 @@ __device__ __forceinline__ float warp_sum(float x) {
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
   return x;
 }
-__device__ __forceinline__ float warp_max(float x) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
-  return x;
-}
-
 // Thread layout of a token pass: thread (tq, c), c = tid % D the channel and
 // tokens tq * TPT .. tq * TPT + TPT - 1 of the batch.
 template <int D>
@@ -458,14 +446,13 @@ __global__ void __launch_bounds__(kNT) bwd_key(
 }
 
 // ---------------------------------------------------------------- Conv1D backward
-// Stream s = blockIdx.z (0 q, 1 k, 2 v) over a block of kConvChunk tokens of
+// Stream s = blockIdx.z (0 q, 1 k, 2 v) over a block of RUNS x rl tokens of
 // one (b, h): dx_t = sum_i w_i dx~_{t+3-i} (terms with t + 3 - i >= L dropped;
 // dx_t = 0 for t >= L) and the block's partials of dw_i = sum_t dx~_t x_{t-3+i}.
-// Thread (run, g) walks kConvChunk / RUNS consecutive tokens of channels
+// Thread (run, g) walks rl consecutive tokens of channels
 // 4g .. 4g+3 with sliding windows (x of the 3 tokens before, dx~ of the 3
 // after), every token's 4 channels one vector load; the runs' tap partials are
 // then added in run order.
-constexpr int kConvChunk = 1024;
 constexpr int kConvCh = 4;  // channels per thread
 __device__ __forceinline__ void ld4(const float *p, float (&f)[4]) {
   const float4 a = __ldg((const float4 *)p);
@@ -490,8 +477,8 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
     const T *__restrict__ q, const T *__restrict__ k, const T *__restrict__ v,
     const T *__restrict__ dxt, const float *__restrict__ conv_w,
     const int32_t *__restrict__ seq_lens, T *__restrict__ dq, T *__restrict__ dk,
-    T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck) {
-  constexpr int G = D / kConvCh, RUNS = kNT / G, RL = kConvChunk / RUNS;
+    T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck, int rl) {
+  constexpr int G = D / kConvCh, RUNS = kNT / G;
   __shared__ float sw[RUNS][D * kConvW];
   const int chunk = blockIdx.x, bh = blockIdx.y, s = blockIdx.z, b = bh / H, h = bh % H;
   const int tid = threadIdx.x, g = tid % G, run = tid / G;
@@ -499,7 +486,7 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
   T *dx = s == 0 ? dq : (s == 1 ? dk : dv);
   const T *dxs = dxt + (size_t)s * ((size_t)gridDim.y / H) * N * H * D;
   const int L = clamp_len(seq_lens, b, N);
-  const int ta = chunk * kConvChunk + run * RL, tb = min(ta + RL, N);
+  const int ta = (chunk * RUNS + run) * rl, tb = min(ta + rl, N);
   float w[kConvCh][kConvW], dw[kConvCh][kConvW];
 #pragma unroll
   for (int c = 0; c < kConvCh; ++c) {
@@ -663,10 +650,14 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
                                       dxt + plane, dxt + 2 * plane, H, N);
   count_launch();
   }
-  const int nckc = (N + kConvChunk - 1) / kConvChunk;  // Conv1D backward blocks per (b, h)
+  // Conv1D backward: 64 tokens a thread run (measured against 32..128-token
+  // runs chosen to fill whole waves: those were slower)
+  constexpr int kRuns = kNT / (D / kConvCh);
+  const int rl = 64;
+  const int nckc = (N + kRuns * rl - 1) / (kRuns * rl);  // Conv1D backward blocks per (b, h)
   bwd_conv<T, D><<<dim3(nckc, BH, 3), kNT, 0, st>>>(
       (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
-      (T *)a.dk, (T *)a.dv, wpart, H, N, nckc);
+      (T *)a.dk, (T *)a.dv, wpart, H, N, nckc, rl);
   count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
   bwd_reduce_w<D><<<(nw + 31) / 32, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
