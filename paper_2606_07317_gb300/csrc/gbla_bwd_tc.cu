@@ -105,11 +105,11 @@ __device__ __forceinline__ int seq_len(const int32_t *seq_lens, int b, int N) {
 struct KTile {
   int bh, b, h, t0, L;
 };
-__device__ __forceinline__ bool key_tile(const KeyParams &p, long long i, KTile &t) {
-  t.bh = (int)(i / p.tps);
+__device__ __forceinline__ bool key_tile(const KeyParams &p, int i, KTile &t) {
+  t.bh = i / p.tps;
   t.b = t.bh / p.H;
   t.h = t.bh % p.H;
-  t.t0 = (int)(i % p.tps) * kKTok;
+  t.t0 = (i - t.bh * p.tps) * kKTok;
   t.L = seq_len(p.seq_lens, t.b, p.N);
   return t.t0 < t.L;
 }
@@ -152,7 +152,8 @@ __global__ void __launch_bounds__(kKThreads, 1)
   float *cslot = (float *)(smem + kKOffMisc + 8);
 
   const long long T = (long long)p.B * H * p.tps;
-  const long long i0 = T * blockIdx.x / gridDim.x, i1 = T * (blockIdx.x + 1) / gridDim.x;
+  // tile indices fit an int (checked on the host)
+  const int i0 = (int)(T * blockIdx.x / gridDim.x), i1 = (int)(T * (blockIdx.x + 1) / gridDim.x);
   if (i0 >= i1) return;
 
   if (tid == 0) {
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
     if (lane == 0) {
       int li = 0;
       bool ok = true;
-      for (long long i = i0; i < i1 && ok; ++i) {
+      for (int i = i0; i < i1 && ok; ++i) {
         KTile t;
         if (!key_tile(p, i, t)) continue;
         const int s = li % kKStages;
@@ -212,15 +213,35 @@ __global__ void __launch_bounds__(kKThreads, 1)
     // this warp's own copy of the head's k and v taps (rewritten when the
     // (b, h) changes; a warp only reads the copy it wrote, so __syncwarp orders it)
     const uint32_t taps = smem_u32(smem + kKOffTaps + warp * kKTapBytes);
+    // The gate value and the head's softmax statistics of the NEXT tile are
+    // loaded one tile ahead, so their global-load latency hides behind this
+    // tile's Conv1D work (the producers are the slowest role of the pass).
+    auto next_tile = [&](int j, KTile &tn) {
+      for (; j < i1; ++j)
+        if (key_tile(p, j, tn)) return j;
+      return i1;
+    };
+    auto gate_raw = [&](const KTile &tn) {
+      const int tok = tn.t0 + r;
+      return tok < tn.L ? p.gate[((size_t)tn.b * N + tok) * H + tn.h] : __float2bfloat16_rn(0.f);
+    };
     int li = 0, cur_bh = -1;
-    float2 gs = make_float2(0.f, 1.f);
     bool ok = true;
-    for (long long i = i0; i < i1 && ok; ++i) {
-      KTile t;
-      if (!key_tile(p, i, t)) continue;
+    KTile t;
+    int i = next_tile(i0, t);
+    __nv_bfloat16 graw = i < i1 ? gate_raw(t) : __float2bfloat16_rn(0.f);
+    float2 gs = i < i1 ? p.stats[t.bh] : make_float2(0.f, 1.f);
+    while (i < i1 && ok) {
+      KTile tn;
+      const int inext = next_tile(i + 1, tn);
+      __nv_bfloat16 graw_n = __float2bfloat16_rn(0.f);
+      float2 gs_n = gs;
+      if (inext < i1) {
+        graw_n = gate_raw(tn);
+        if (tn.bh != t.bh) gs_n = p.stats[tn.bh];
+      }
       const int s = li % kKStages;
       if (t.bh != cur_bh) {
-        gs = p.stats[t.bh];
         cur_bh = t.bh;
         __syncwarp();  // the previous head's taps are no longer read
         for (int u = lane; u < 2 * kD; u += 32) {
@@ -232,9 +253,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
       }
       const int tok = t.t0 + r;
       const bool valid = tok < t.L;
-      const float g =
-          valid ? expf(__bfloat162float(p.gate[((size_t)t.b * N + tok) * H + t.h]) - gs.x) / gs.y
-                : 0.f;
+      const float g = valid ? expf(__bfloat162float(graw) - gs.x) / gs.y : 0.f;
       const bool w = mbar_wait(&raw_full[s], (li / kKStages) & 1, &ab) &&
                      mbar_wait(&a_empty[s], ((li / kKStages) & 1) ^ 1, &ab) &&
                      mbar_wait(&phi_empty[s], ((li / kKStages) & 1) ^ 1, &ab);
@@ -284,6 +303,10 @@ __global__ void __launch_bounds__(kKThreads, 1)
         mbar_arrive(&phi_full[s]);
       }
       ++li;
+      i = inext;
+      t = tn;
+      graw = graw_n;
+      gs = gs_n;
     }
     if (!ok && !ab.raised()) report(4, ab);
   } else if (warp < kKMmaWarp) {
@@ -297,7 +320,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
     // the loop), so the named barriers below always match.
     int li = 0, cur_bh = -1, nbh = 0;
     bool ok = true;
-    for (long long i = i0; i < i1; ++i) {
+    for (int i = i0; i < i1; ++i) {
       KTile t;
       if (!key_tile(p, i, t)) continue;
       const int s = li % kKStages, buf = li % 2;
@@ -414,7 +437,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
       const uint32_t bb = smem_u32(smem + kKOffB);
       int li = 0, cur_bh = -1, nbh = 0;
       bool ok = true;
-      for (long long i = i0; i < i1 && ok; ++i) {
+      for (int i = i0; i < i1 && ok; ++i) {
         KTile t;
         if (!key_tile(p, i, t)) continue;
         const int s = li % kKStages, buf = li % 2;
@@ -447,7 +470,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
         mma_commit(&acc_full[buf]);
         // last tile of this (b, h) in this CTA: the dS tiles may be rebuilt
         bool last = true;
-        for (long long j = i + 1; j < i1; ++j) {
+        for (int j = i + 1; j < i1; ++j) {
           KTile tn;
           if (key_tile(p, j, tn)) {
             last = tn.bh != t.bh;
@@ -1073,6 +1096,8 @@ cudaError_t make_rows_map(CUtensorMap *m, const void *base, int B, int N, int H,
 
 bool bwd_tc_key_supported(const Problem &p) {
   if (p.dtype != GBLA_BF16 || p.D != kD || p.flags != 0) return false;
+  // the key pass indexes its 128-token tiles with an int
+  if ((long long)p.B * p.H * ((p.N + kKTok - 1) / kKTok) > 0x7fffffffLL) return false;
   int dev = 0, major = 0, minor = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
   cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
