@@ -463,6 +463,22 @@ __device__ __forceinline__ void ld4(const __nv_bfloat16 *p, float (&f)[4]) {
   f[0] = __uint_as_float(u.x << 16); f[1] = __uint_as_float(u.x & 0xFFFF0000u);
   f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
 }
+// Four channels as loaded (raw), then widened to fp32: the Conv1D backward
+// issues a batch of raw loads before it converts any of them.
+template <typename T> struct Raw4;
+template <> struct Raw4<float> { using type = float4; };
+template <> struct Raw4<__nv_bfloat16> { using type = uint2; };
+__device__ __forceinline__ float4 ld4raw(const float *p) { return __ldg((const float4 *)p); }
+__device__ __forceinline__ uint2 ld4raw(const __nv_bfloat16 *p) { return __ldg((const uint2 *)p); }
+__device__ __forceinline__ void zero4raw(float4 &r) { r = make_float4(0.f, 0.f, 0.f, 0.f); }
+__device__ __forceinline__ void zero4raw(uint2 &r) { r = make_uint2(0u, 0u); }
+__device__ __forceinline__ void cvt4raw(const float4 &a, float (&f)[4]) {
+  f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
+}
+__device__ __forceinline__ void cvt4raw(const uint2 &u, float (&f)[4]) {
+  f[0] = __uint_as_float(u.x << 16); f[1] = __uint_as_float(u.x & 0xFFFF0000u);
+  f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
+}
 __device__ __forceinline__ void st4(float *p, const float (&f)[4]) {
   *(float4 *)p = make_float4(f[0], f[1], f[2], f[3]);
 }
@@ -517,11 +533,25 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
     ldx(ta - 3 + i, xm[i]);
     ldd(ta + i, dm[i]);
   }
-#pragma unroll 4
-  for (int t = ta; t < tb; ++t) {
+  // U steps at a time: their 2 U loads are issued together (zero outside
+  // [0, L)), then the steps run in order
+  using Raw = typename Raw4<T>::type;
+  constexpr int U = sizeof(T) == 2 ? 8 : 4;
+  for (int t0 = ta; t0 < tb; t0 += U) {
+    Raw xr[U], dr[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int tx = t0 + u, td = t0 + u + 3;
+      if (tx < L) xr[u] = ld4raw(x + col + (size_t)tx * rs); else zero4raw(xr[u]);
+      if (td < L) dr[u] = ld4raw(dxs + col + (size_t)td * rs); else zero4raw(dr[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+    const int t = t0 + u;
+    if (t >= tb) break;
     float xc[kConvCh], dn[kConvCh], o[kConvCh];
-    ldx(t, xc);      // x_t
-    ldd(t + 3, dn);  // dx~_{t+3}
+    cvt4raw(xr[u], xc);  // x_t
+    cvt4raw(dr[u], dn);  // dx~_{t+3}
 #pragma unroll
     for (int c = 0; c < kConvCh; ++c) {
       // dx_t = w0 dx~_{t+3} + w1 dx~_{t+2} + w2 dx~_{t+1} + w3 dx~_t
@@ -541,6 +571,7 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
     for (int c = 0; c < kConvCh; ++c) {
       xm[0][c] = xm[1][c]; xm[1][c] = xm[2][c]; xm[2][c] = xc[c];
       dm[0][c] = dm[1][c]; dm[1][c] = dm[2][c]; dm[2][c] = dn[c];
+    }
     }
   }
 #pragma unroll
