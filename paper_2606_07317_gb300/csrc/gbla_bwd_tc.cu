@@ -791,7 +791,8 @@ __global__ void __launch_bounds__(kQThreads, 1)
         den = v4[0];
       }
       const float inv = valid ? 1.f / den : 0.f;
-      // pass 1 (nothing here needs r): sum O^2, u . O with u = dy w silu(og), and
+      // pass 1 (nothing here needs r): sum O^2, u . O with u = dy w silu(og) (both
+      // summed over the accumulator num = O den and scaled once by 1/den), and
       // two per-element factors that replace this row's out_gate and dy values
       // (read only by this thread from here on): A = dy w silu'(og) (dog = A O r)
       // and Bv = dy silu(og) (dnorm_w term Bv O r, u = Bv w)
@@ -810,10 +811,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
         float fa[16], fb[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const float o = v[i] * inv, sg = sigmoid_f(og[i]), si = og[i] * sg;
+          const float sg = sigmoid_f(og[i]), si = og[i] * sg;
           const float w = wv[i];
-          ss = fmaf(o, o, ss);
-          uo = fmaf(dy[i] * w * si, o, uo);
+          ss = fmaf(v[i], v[i], ss);
+          uo = fmaf(dy[i] * w * si, v[i], uo);
           fa[i] = dy[i] * w * sg * (1.f + og[i] * (1.f - sg));
           fb[i] = dy[i] * si;
         }
@@ -833,11 +834,15 @@ __global__ void __launch_bounds__(kQThreads, 1)
         sts_v4(dyt + sw_off(row, 2 * j), pack8(a));
         sts_v4(dyt + sw_off(row, 2 * j + 1), pack8(c));
       }
+      ss *= inv * inv;
+      uo *= inv;
       const float rr = rsqrtf(ss * (1.f / kD) + p.eps);
       const float r3 = rr * rr * rr * (1.f / kD);
       // pass 2: dog, dnorm_w, dnum (bf16 A / B tile); dO . O in closed form:
       // sum_d (r u_d - r3 O_d (u . O)) O_d = r (u . O) - r3 (u . O) sum O^2
       const float doo = rr * uo - r3 * uo * ss;
+      // per element with v = num = O den:  O r = v ir,  dnum = dO / den = ir (Bv w) - bc v
+      const float ir = inv * rr, bc = r3 * uo * inv * inv;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         float v[16], fa[16], fb[16];
@@ -852,11 +857,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
         float gq[16], gw[16], dn[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-          const float o = v[i] * inv, orr = o * rr;
+          const float orr = v[i] * ir;
           gq[i] = fa[i] * orr;
           gw[i] = valid ? fb[i] * orr : 0.f;
-          const float dO = rr * (fb[i] * wv[i]) - r3 * o * uo;
-          dn[i] = valid ? dO * inv : 0.f;
+          dn[i] = valid ? fmaf(ir, fb[i] * wv[i], -bc * v[i]) : 0.f;
         }
         dnw4[j] += lane_colsum<16>(gw);
         float a[8], c[8];
