@@ -135,15 +135,16 @@ struct Scratch {
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// State (Conv1D of k, v, phi, gate, S and z) into `state`.
+// State (Conv1D of k, v, phi, gate, S and z) into `state`; with the tensor-core
+// family also the key gate's softmax statistics into gate_stats, if given.
 gbla_status run_state(const Problem &p, bool tc, const void *k, const void *v,
                       const void *gate, const float *conv_w, float *state,
-                      cudaStream_t st) {
+                      cudaStream_t st, float2 *gate_stats = nullptr) {
   Scratch ws;
   if (tc) {
     gbla_status s = ws.alloc(tc_workspace_bytes(p), st);
     if (s != GBLA_OK) return s;
-    return from_cuda(tc_state(p, k, v, gate, conv_w, ws.ptr, state, st));
+    return from_cuda(tc_state(p, k, v, gate, conv_w, ws.ptr, state, st, gate_stats));
   }
   SimtPlan plan = simt_plan(p);
   gbla_status s = ws.alloc(simt_partials_bytes(p, plan), st);
@@ -336,11 +337,14 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
   Scratch scr;
   if ((s = scr.alloc(sizeof(float) * lay.total, st)) != GBLA_OK) return s;
   float *base = (float *)scr.ptr;
-  // the forward state S, z through the forward's own state path
-  if ((s = run_state(p, tc, k, v, gate, conv_w, base + lay.state, st)) != GBLA_OK) return s;
+  // the forward state S, z through the forward's own state path, which on
+  // tensor cores also yields the gate statistics the backward needs
+  if ((s = run_state(p, tc, k, v, gate, conv_w, base + lay.state, st,
+                     tc ? (float2 *)(base + lay.stats) : nullptr)) != GBLA_OK)
+    return s;
   BwdArgs a{q, k, v, gate, out_gate, dy, conv_w, norm_w, dq, dk, dv, dgate, dout_gate,
             dconv_w, dnorm_w};
-  return from_cuda(bwd_run(p, a, base, st));
+  return from_cuda(bwd_run(p, a, base, tc, st));
 }
 
 // Validation shared by gbla_project and gbla_layer_forward.

@@ -18,7 +18,8 @@
 // Launches (all on the caller's stream, after the forward state S, z has been
 // formed by the forward's own state path):
 //   bwd_gate_split / bwd_gate_join  per (b, h): M = max a, Ltot = sum e^{a - M}
-//                    (g_j = e^{a_j-M}/Ltot), over sequence splits, then combined
+//                    (g_j = e^{a_j-M}/Ltot), over sequence splits, then combined;
+//                    skipped when the tensor-core state path already wrote them
 //   bwd_query        per (b, h, chunk): 5' and 6' per token; dq~ to scratch
 //                    (the dq~, dk~, dv~ planes are stored in the I/O dtype);
 //                    chunk partials of dS, dz and the norm-weight gradient
@@ -630,7 +631,8 @@ __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wp
 }
 
 template <typename T, int D>
-cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st) {
+cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,
+                    cudaStream_t st) {
   const int B = p.B, H = p.H, N = p.N, BH = B * H;
   const int nck = (N + kChunk - 1) / kChunk;
   const BwdLayout lay = bwd_layout(p);
@@ -642,10 +644,12 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, cudaStre
   const size_t plane = (size_t)B * N * H * D;
   cudaError_t e;
   float2 *gpart = (float2 *)(scratch + lay.gpart);
-  bwd_gate_split<T><<<dim3(BH, kGateSplits), 256, 0, st>>>((const T *)a.gate, p.seq_lens, gpart,
-                                                           H, N);
-  bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(gpart, stats, BH);
-  count_launch(2);
+  if (!stats_ready) {
+    bwd_gate_split<T><<<dim3(BH, kGateSplits), 256, 0, st>>>((const T *)a.gate, p.seq_lens,
+                                                             gpart, H, N);
+    bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(gpart, stats, BH);
+    count_launch(2);
+  }
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   const size_t smq = sizeof(float) * (2 * D * D + D + 4 * D * kTB + kTB + kNT / 32 * TPT);
   const bool tc = bwd_tc_key_supported(p);  // bf16, D = 64, sm_103: both token passes on tcgen05
@@ -717,18 +721,19 @@ BwdLayout bwd_layout(const Problem &p) {
   return l;
 }
 
-cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st) {
+cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,
+                    cudaStream_t st) {
   if (p.dtype == GBLA_BF16) {
     switch (p.D) {
-      case 32: return run_bwd<__nv_bfloat16, 32>(p, a, scratch, st);
-      case 64: return run_bwd<__nv_bfloat16, 64>(p, a, scratch, st);
-      case 128: return run_bwd<__nv_bfloat16, 128>(p, a, scratch, st);
+      case 32: return run_bwd<__nv_bfloat16, 32>(p, a, scratch, stats_ready, st);
+      case 64: return run_bwd<__nv_bfloat16, 64>(p, a, scratch, stats_ready, st);
+      case 128: return run_bwd<__nv_bfloat16, 128>(p, a, scratch, stats_ready, st);
     }
   } else {
     switch (p.D) {
-      case 32: return run_bwd<float, 32>(p, a, scratch, st);
-      case 64: return run_bwd<float, 64>(p, a, scratch, st);
-      case 128: return run_bwd<float, 128>(p, a, scratch, st);
+      case 32: return run_bwd<float, 32>(p, a, scratch, stats_ready, st);
+      case 64: return run_bwd<float, 64>(p, a, scratch, stats_ready, st);
+      case 128: return run_bwd<float, 128>(p, a, scratch, stats_ready, st);
     }
   }
   return cudaErrorInvalidValue;

@@ -44,9 +44,11 @@ cudaError_t simt_readout(const Problem &p, const void *q, const void *og,
 // ---- tensor-core (tcgen05 + TMA) family: bf16, D in {64, 128} -------------
 bool tc_supports(const Problem &p);
 size_t tc_workspace_bytes(const Problem &p);
+// gate_stats (optional, [B*H]): the key gate's softmax statistics (max of the
+// logits, sum of exp(logit - max)) over each sequence, as the state used them.
 cudaError_t tc_state(const Problem &p, const void *k, const void *v,
                      const void *gate, const float *conv_w, void *workspace,
-                     float *state, cudaStream_t st);
+                     float *state, cudaStream_t st, float2 *gate_stats = nullptr);
 // after_state: launched right behind tc_state on the same stream; only the
 // reads of `state` then wait for the preceding kernel (the other inputs were
 // complete before tc_state started).
@@ -62,14 +64,16 @@ struct BwdArgs {
   float *dconv_w, *dnorm_w;
 };
 // Scratch of the backward, in floats from one base: the forward state (filled
-// by the caller through the forward's state path), gate statistics, chunk
+// by the caller through the forward's state path), gate statistics (filled by
+// the caller too when stats_ready, else by the backward itself), chunk
 // partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
 // gradient partials.
 struct BwdLayout {
   size_t state, stats, gpart, qpart, red, cval, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
-cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, cudaStream_t st);
+cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,
+                    cudaStream_t st);
 // Key pass on tensor cores (gbla_bwd_tc.cu): bf16, D = 64, sm_103.  Writes the
 // bf16 dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz.
 bool bwd_tc_key_supported(const Problem &p);

@@ -899,8 +899,9 @@ template <int D>
 __global__ void __launch_bounds__(kReduceThreads) tc_reduce_kernel(const float *__restrict__ records,
                                                          const int32_t *__restrict__ chunk_pre,
                                                          const int32_t *__restrict__ seq_lens,
-                                                         float *__restrict__ state, int B, int H,
-                                                         int N, int S) {
+                                                         float *__restrict__ state,
+                                                         float2 *__restrict__ gate_stats, int B,
+                                                         int H, int N, int S) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
@@ -958,6 +959,8 @@ __global__ void __launch_bounds__(kReduceThreads) tc_reduce_kernel(const float *
       }
     }
   }
+  if (gate_stats != nullptr && blockIdx.y == 0 && threadIdx.x == 0)
+    gate_stats[bh] = make_float2(M, l);  // every thread of bh holds the same pair
   const float inv = l > 0.f ? 1.f / l : 0.f;
   *(float4 *)(state + (size_t)bh * F + e0) =
       make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
@@ -1662,7 +1665,8 @@ size_t records_bytes(const Problem &p, int S) {
 
 template <int D>
 cudaError_t run_state(const Problem &p, const void *k, const void *v, const void *gate,
-                      const float *conv_w, void *ws, float *state, cudaStream_t st) {
+                      const float *conv_w, void *ws, float *state, cudaStream_t st,
+                      float2 *gate_stats) {
   constexpr int G = kGroupCh / D;
   const int S = chunk_len(p);
   const size_t rb = records_bytes(p, S);
@@ -1703,7 +1707,8 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, tc_reduce_kernel<D>, (const float *)sp.records,
-                         (const int32_t *)sp.chunk_pre, p.seq_lens, state, p.B, p.H, p.N, S);
+                         (const int32_t *)sp.chunk_pre, p.seq_lens, state, gate_stats, p.B,
+                         p.H, p.N, S);
   count_launch();
   return e;
 }
@@ -1768,10 +1773,11 @@ size_t tc_workspace_bytes(const Problem &p) {
 }
 
 cudaError_t tc_state(const Problem &p, const void *k, const void *v, const void *gate,
-                     const float *conv_w, void *ws, float *state, cudaStream_t st) {
+                     const float *conv_w, void *ws, float *state, cudaStream_t st,
+                     float2 *gate_stats) {
   switch (p.D) {
-    case 64: return run_state<64>(p, k, v, gate, conv_w, ws, state, st);
-    case 128: return run_state<128>(p, k, v, gate, conv_w, ws, state, st);
+    case 64: return run_state<64>(p, k, v, gate, conv_w, ws, state, st, gate_stats);
+    case 128: return run_state<128>(p, k, v, gate, conv_w, ws, state, st, gate_stats);
   }
   return cudaErrorInvalidValue;
 }
