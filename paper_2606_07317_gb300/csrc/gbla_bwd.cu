@@ -349,14 +349,30 @@ __global__ void __launch_bounds__(kNT) bwd_query(
 // ---------------------------------------------------------------- state reduction
 // red record per (b, h): dS [D][D], dz [D] (chunk partials summed in chunk order).
 template <int D>
+// With state and dotpart given, block x of (b, h) also writes the partial dot
+// product of its slice of [dS | dz] with [S | z] (lanes, then warps in order):
+// c = <dS, S> + <dz, z> is the sum of the gridDim.x partials in order.
 __global__ void __launch_bounds__(256) bwd_reduce_state(const float *__restrict__ part,
-                                                        float *__restrict__ red, int nck) {
+                                                        float *__restrict__ red,
+                                                        const float *__restrict__ state,
+                                                        float *__restrict__ dotpart, int nck) {
   constexpr int F = D * D + D;
   const int bh = blockIdx.y, i = blockIdx.x * 256 + threadIdx.x;
-  if (i >= F) return;
   float a = 0.f;
-  for (int ch = 0; ch < nck; ++ch) a += part[((size_t)bh * nck + ch) * qrec<D>() + i];
-  red[(size_t)bh * F + i] = a;
+  if (i < F) {
+    for (int ch = 0; ch < nck; ++ch) a += part[((size_t)bh * nck + ch) * qrec<D>() + i];
+    red[(size_t)bh * F + i] = a;
+  }
+  if (dotpart == nullptr) return;
+  const float d = warp_sum(i < F ? a * state[(size_t)bh * F + i] : 0.f);
+  __shared__ float wsum[8];
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = d;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float c = 0.f;
+    for (int w = 0; w < 8; ++w) c += wsum[w];
+    dotpart[(size_t)bh * gridDim.x + blockIdx.x] = c;
+  }
 }
 
 // ---------------------------------------------------------------- key pass
@@ -668,10 +684,12 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
     count_launch();
   }
   constexpr int F = D * D + D;
-  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(qpart, red, nckq);
+  // on tensor cores the key pass forms c from the reduction's partial dot products
+  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(
+      qpart, red, tc ? state : nullptr, tc ? scratch + lay.cpart : nullptr, nckq);
   count_launch();
   if (tc) {
-    if ((e = bwd_tc_key(p, a, stats, state, red, scratch + lay.cval, dxt + plane,
+    if ((e = bwd_tc_key(p, a, stats, red, scratch + lay.cpart, (F + 255) / 256, dxt + plane,
                         dxt + 2 * plane, st)) != cudaSuccess)
       return e;
   } else {
@@ -714,8 +732,8 @@ BwdLayout bwd_layout(const Problem &p) {
   l.gpart = up(l.stats + 2 * BH);
   l.qpart = up(l.gpart + 2 * BH * kGateSplits);
   l.red = up(l.qpart + BH * nck * (D * D + 2 * D));
-  l.cval = up(l.red + BH * (F + 1));
-  l.dxt = up(l.cval + BH);
+  l.cpart = up(l.red + BH * (F + 1));
+  l.dxt = up(l.cpart + BH * ((F + 255) / 256));
   l.wpart = up(l.dxt + 3 * BH * (size_t)p.N * D);
   l.total = up(l.wpart + 3 * BH * nck * D * kConvW);
   return l;

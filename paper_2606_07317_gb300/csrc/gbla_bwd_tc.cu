@@ -80,7 +80,8 @@ struct KeyParams {
   const float *conv_w;             // [3, H, D, 4]
   const float2 *stats;             // [B*H]: gate max, sum of exp
   const float *red;                // [B*H][D*D + D]: dS, dz
-  const float *cval;               // [B*H]: c
+  const float *dotpart;            // [B*H][ndot]: partials of c = <dS, S> + <dz, z>
+  int ndot;
   const int32_t *seq_lens;
   __nv_bfloat16 *dkt, *dvt;        // [B, N, H, D] bf16 planes
   __nv_bfloat16 *dgate;            // [B, N, H]
@@ -364,7 +365,11 @@ __global__ void __launch_bounds__(kKThreads, 1)
           sts_v4(bb + 3 * kKBTile + o, pack8(lT));
         }
         if (et < kD) ((float *)(smem + kKOffDz))[et] = dS[kD * kD + et];
-        if (et == 0) *cslot = p.cval[t.bh];
+        if (et == 0) {  // c, the partials added in order
+          float c = 0.f;
+          for (int j = 0; j < p.ndot; ++j) c += p.dotpart[(size_t)t.bh * p.ndot + j];
+          *cslot = c;
+        }
         fence_proxy_async_smem();
         named_barrier(1, kKEpi);
         if (et == 0) mbar_arrive(b_full);
@@ -1064,24 +1069,6 @@ __global__ void __launch_bounds__(kQThreads, 1)
   }
 }
 
-// c = <dS, S> + <dz, z> per (b, h), summed in a fixed order.
-__global__ void __launch_bounds__(256) bwd_state_dot(const float *__restrict__ red,
-                                                     const float *__restrict__ state,
-                                                     float *__restrict__ cval, int F) {
-  const int bh = blockIdx.x;
-  __shared__ float part[256];
-  float a = 0.f;
-  for (int i = threadIdx.x; i < F; i += 256)
-    a = fmaf(red[(size_t)bh * F + i], state[(size_t)bh * F + i], a);
-  part[threadIdx.x] = a;
-  __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
-    if (threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) cval[bh] = part[0];
-}
-
 using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                               const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
                               const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
@@ -1131,15 +1118,15 @@ bool bwd_tc_key_supported(const Problem &p) {
 }
 
 cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
-                       const float *state, const float *red, float *cval, void *dkt,
+                       const float *red, const float *dotpart, int ndot, void *dkt,
                        void *dvt, cudaStream_t st) {
   const int BH = p.B * p.H;
-  constexpr int F = kD * kD + kD;
-  bwd_state_dot<<<BH, 256, 0, st>>>(red, state, cval, F);
-  count_launch();
+  cudaError_t e;
   // rows past seq_lens[b] of dgate are zero; the kernel writes the valid rows
-  cudaError_t e = cudaMemsetAsync(a.dgate, 0, sizeof(__nv_bfloat16) * (size_t)BH * p.N, st);
-  if (e != cudaSuccess) return e;
+  if (p.seq_lens != nullptr &&
+      (e = cudaMemsetAsync(a.dgate, 0, sizeof(__nv_bfloat16) * (size_t)BH * p.N, st)) !=
+          cudaSuccess)
+    return e;
   CUtensorMap tm_k, tm_v;
   if ((e = make_rows_map(&tm_k, a.k, p.B, p.N, p.H)) != cudaSuccess) return e;
   if ((e = make_rows_map(&tm_v, a.v, p.B, p.N, p.H)) != cudaSuccess) return e;
@@ -1148,7 +1135,8 @@ cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
   kp.conv_w = a.conv_w;
   kp.stats = stats;
   kp.red = red;
-  kp.cval = cval;
+  kp.dotpart = dotpart;
+  kp.ndot = ndot;
   kp.seq_lens = p.seq_lens;
   kp.dkt = (__nv_bfloat16 *)dkt;
   kp.dvt = (__nv_bfloat16 *)dvt;

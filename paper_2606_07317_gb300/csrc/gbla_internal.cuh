@@ -69,16 +69,17 @@ struct BwdArgs {
 // partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
 // gradient partials.
 struct BwdLayout {
-  size_t state, stats, gpart, qpart, red, cval, dxt, wpart, total;
+  size_t state, stats, gpart, qpart, red, cpart, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,
                     cudaStream_t st);
 // Key pass on tensor cores (gbla_bwd_tc.cu): bf16, D = 64, sm_103.  Writes the
-// bf16 dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz.
+// bf16 dk~ / dv~ planes and dgate (zero past seq_lens) from the reduced dS, dz
+// and the ndot partial sums per (b, h) of c = <dS, S> + <dz, z>.
 bool bwd_tc_key_supported(const Problem &p);
 cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
-                       const float *state, const float *red, float *cval, void *dkt,
+                       const float *red, const float *dotpart, int ndot, void *dkt,
                        void *dvt, cudaStream_t st);
 // Query pass on tensor cores (same conditions): dq~ plane, dout_gate, and one
 // partial record [dS, dz, dnorm_w] per (b, h, chunk of bwd_tc_query_chunks).
