@@ -23,8 +23,11 @@
 //   bwd_query        per (b, h, chunk): 5' and 6' per token; dq~ to scratch
 //                    (the dq~, dk~, dv~ planes are stored in the I/O dtype);
 //                    chunk partials of dS, dz and the norm-weight gradient
-//   bwd_reduce_state per (b, h): fixed-order sums of the partials; c
-//   bwd_key          per (b, h, chunk): 4' and 3' per token; dk~, dv~ to scratch
+//   bwd_reduce_state per (b, h): fixed-order sums of the partials (and, for the
+//                    tensor-core key pass, per-block partial sums of c)
+//   bwd_key          per (b, h, chunk): c, then 4' and 3' per token; dk~, dv~ to
+//                    scratch (tc_bwd_key_kernel and tc_bwd_query_kernel in
+//                    gbla_bwd_tc.cu replace bwd_key and bwd_query for bf16, D = 64)
 //   bwd_conv         per (stream, b, h, chunk): 1' (anti-causal taps) into dq,
 //                    dk, dv; chunk partials of the tap gradients
 //   bwd_reduce_w     fixed-order sums of the tap / norm-weight partials
