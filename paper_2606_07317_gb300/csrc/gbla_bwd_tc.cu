@@ -19,7 +19,8 @@
 // splits of dS, fp32 accumulation in TMEM (two buffers); four epilogue warps
 // (one token row per thread) form dk~, dv~ and dgate and write the bf16 dk~ /
 // dv~ rows through per-warp staging as whole 128-byte segments.  The epilogue
-// warps also build the dS tiles whenever the (batch, head) changes.
+// warps also build the dS tiles, and add up c from the dS reduction's partial
+// sums in order, whenever the (batch, head) changes.
 //
 // Every mbarrier wait is bounded (2 s); a wait that runs out sets a bit in
 // g_bwd_error and the CTA's abort flag, every role leaves its loop, the TMA
