@@ -14,7 +14,7 @@
 // brings the raw k and v rows of a tile (128 tokens + 3 rows of conv history,
 // 128B-swizzled) into a 2-deep ring; four producer warps (one token row per
 // thread) run both Conv1Ds, phi and the gate in fp32 and write V~ and K^ as
-// bf16 K-major A tiles, plus phi(k~) as bf16; one thread issues the MMAs
+// bf16 K-major A tiles; one thread issues the MMAs
 // DK = V~ dS^T and DV = K^ dS (M = 128, N = 64, K = 64) against bf16 hi + lo
 // splits of dS, fp32 accumulation in TMEM (two buffers); four epilogue warps
 // (one token row per thread) form dk~, dv~ and dgate and write the bf16 dk~ /
@@ -49,7 +49,7 @@ constexpr int kKRawHalf = (kKRawBox + 1023) / 1024 * 1024;  // 17408
 constexpr int kKRawStage = 2 * kKRawHalf;        // k box, v box
 constexpr int kKStages = 2;
 constexpr int kKTile = kKTok * 128;              // 16384: one 128 x 64 bf16 tile
-constexpr int kKAStage = 3 * kKTile;             // V~, K^, phi(k~)
+constexpr int kKAStage = 2 * kKTile;             // V~, K^
 constexpr int kKBTile = kD * 128;                // 8192: one 64 x 64 bf16 tile
 constexpr int kKProdWarps = 4, kKEpiWarps = 4;
 constexpr int kKEpiWarp0 = kKProdWarps;          // 4
@@ -62,14 +62,14 @@ constexpr uint32_t kKTmemCols = 256;             // two buffers of [DK | DV]
 
 constexpr int kKOffRaw = 0;
 constexpr int kKOffA = kKOffRaw + kKStages * kKRawStage;     // 69632
-constexpr int kKOffB = kKOffA + kKStages * kKAStage;         // 167936: dS hi, lo, dS^T hi, lo
-constexpr int kKOffG = kKOffB + 4 * kKBTile;                 // 200704: float [2][128]
+constexpr int kKOffB = kKOffA + kKStages * kKAStage;         // 135168: dS hi, lo, dS^T hi, lo
+constexpr int kKOffG = kKOffB + 4 * kKBTile;                 // 167936: float [2][128]
 constexpr int kKOffDz = kKOffG + kKStages * kKTok * 4;       // float [64]
 constexpr int kKOffStg = kKOffDz + kD * 4;
 constexpr int kKOffTaps = kKOffStg + kKEpiWarps * kKStg;     // per producer warp: k, v taps
 constexpr int kKTapBytes = 2 * kD * 16;                      // float4 [2][64]
 constexpr int kKOffBar = kKOffTaps + kKProdWarps * kKTapBytes;
-// raw_full[2], raw_empty[2], a_full[2], a_empty[2], phi_full[2], phi_empty[2],
+// raw_full[2], raw_empty[2], a_full[2], a_empty[2], kh_full[2], kh_empty[2],
 // acc_full[2], acc_empty[2], b_full, b_free, fin
 constexpr int kKBars = 8 * kKStages + 3;
 constexpr int kKOffMisc = kKOffBar + kKBars * 8;             // tmem address, abort flag, c
@@ -160,7 +160,8 @@ __global__ void __launch_bounds__(kKThreads, 1)
 
   uint64_t *bars = (uint64_t *)(smem + kKOffBar);
   uint64_t *raw_full = bars, *raw_empty = bars + 2, *a_full = bars + 4, *a_empty = bars + 6;
-  uint64_t *phi_full = bars + 8, *phi_empty = bars + 10, *acc_full = bars + 12;
+  // kh_full / kh_empty: the epilogue's reads of the K^ rows of an A stage
+  uint64_t *kh_full = bars + 8, *kh_empty = bars + 10, *acc_full = bars + 12;
   uint64_t *acc_empty = bars + 14, *b_full = bars + 16, *b_free = bars + 17, *fin = bars + 18;
   uint32_t *tmem_slot = (uint32_t *)(smem + kKOffMisc);
   const AbortFlag ab{smem_u32(smem + kKOffMisc + 4)};
@@ -177,8 +178,8 @@ __global__ void __launch_bounds__(kKThreads, 1)
       mbar_init(&raw_empty[i], kKProdWarps);
       mbar_init(&a_full[i], kKProdWarps);
       mbar_init(&a_empty[i], 1);
-      mbar_init(&phi_full[i], kKProdWarps);
-      mbar_init(&phi_empty[i], kKEpiWarps);
+      mbar_init(&kh_full[i], kKProdWarps);
+      mbar_init(&kh_empty[i], kKEpiWarps);
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kKEpiWarps);
     }
@@ -271,7 +272,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
       const float g = valid ? expf(__bfloat162float(graw) - gs.x) / gs.y : 0.f;
       const bool w = mbar_wait(&raw_full[s], (li / kKStages) & 1, &ab) &&
                      mbar_wait(&a_empty[s], ((li / kKStages) & 1) ^ 1, &ab) &&
-                     mbar_wait(&phi_empty[s], ((li / kKStages) & 1) ^ 1, &ab);
+                     mbar_wait(&kh_empty[s], ((li / kKStages) & 1) ^ 1, &ab);
       if (!__all_sync(0xffffffffu, w)) {  // the whole warp leaves together
         ok = false;
         break;
@@ -279,7 +280,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
       const uint32_t rk = smem_u32(smem + kKOffRaw + s * kKRawStage);
       const uint32_t rv = rk + kKRawHalf;
       const uint32_t av = smem_u32(smem + kKOffA + s * kKAStage);
-      const uint32_t ak = av + kKTile, ap = av + 2 * kKTile;
+      const uint32_t ak = av + kKTile;
 #pragma unroll 2
       for (int c = 0; c < kD / 8; ++c) {
         float kx[kConvW][8], vx[kConvW][8];
@@ -288,7 +289,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
           unpack8(lds_v4(rk + sw_off(r + j, c)), kx[j]);
           unpack8(lds_v4(rv + sw_off(r + j, c)), vx[j]);
         }
-        float vt[8], kh[8], ph[8];
+        float vt[8], kh[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
           const uint4 uk = lds_v4(taps + 16 * (8 * c + e));
@@ -299,15 +300,12 @@ __global__ void __launch_bounds__(kKThreads, 1)
                                         __uint_as_float(uv.z), __uint_as_float(uv.w));
           const float kt = fmaf(tk.w, kx[3][e], fmaf(tk.z, kx[2][e], fmaf(tk.y, kx[1][e], tk.x * kx[0][e])));
           const float v1 = fmaf(tv.w, vx[3][e], fmaf(tv.z, vx[2][e], fmaf(tv.y, vx[1][e], tv.x * vx[0][e])));
-          const float f = phi_f(kt);
           vt[e] = valid ? v1 : 0.f;
-          kh[e] = g * f;  // 0 on padded rows (g = 0)
-          ph[e] = f;
+          kh[e] = g * phi_f(kt);  // 0 on padded rows (g = 0)
         }
         const uint32_t o = sw_off(r, c);
         sts_v4(av + o, pack8(vt));
         sts_v4(ak + o, pack8(kh));
-        sts_v4(ap + o, pack8(ph));
       }
       sts_f32(smem_u32(smem + kKOffG) + (uint32_t)(s * kKTok + r) * 4, g);
       fence_proxy_async_smem();
@@ -315,7 +313,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
       if (lane == 0) {
         mbar_arrive(&raw_empty[s]);
         mbar_arrive(&a_full[s]);
-        mbar_arrive(&phi_full[s]);
+        mbar_arrive(&kh_full[s]);
       }
       ++li;
       i = inext;
@@ -378,16 +376,19 @@ __global__ void __launch_bounds__(kKThreads, 1)
         ++nbh;
       }
       ok = mbar_wait(&acc_full[buf], (li >> 1) & 1, &ab) && ok;
-      ok = mbar_wait(&phi_full[s], (li / kKStages) & 1, &ab) && ok;
+      ok = mbar_wait(&kh_full[s], (li / kKStages) & 1, &ab) && ok;
       tc_fence_after();
       const uint32_t tacc = tmem + ((uint32_t)(32 * q4) << 16) + buf * 128;
       const int tok = t.t0 + row;
       const bool valid = tok < t.L;
       const float g = lds_f32(smem_u32(smem + kKOffG) + (uint32_t)(s * kKTok + row) * 4);
-      const uint32_t ap = smem_u32(smem + kKOffA + s * kKAStage) + 2 * kKTile;
+      // K^ = g phi(k~) (the MMA's bf16 A tile) stands in for phi(k~):
+      //   dk~ = g dK^ min(phi, 1) = dK^ min(K^, g),
+      //   dgate = g (phi . dK^ - c) = K^ . dK^ - g c
+      const uint32_t ak = smem_u32(smem + kKOffA + s * kKAStage) + kKTile;
       const size_t prow = (((size_t)t.b * N + t.t0) * H + t.h) * kD;  // plane row of tile row 0
       const size_t prs = (size_t)H * kD;                               // plane row stride
-      float dg = 0.f;
+      float khdk = 0.f;
       // dk~ in two 32-column halves, then dv~; each row of 64 bf16 goes through
       // the staging rows as one 128-byte segment
 #pragma unroll 1
@@ -408,19 +409,19 @@ __global__ void __launch_bounds__(kKThreads, 1)
           if (mat == 0) {
 #pragma unroll
             for (int cq = 0; cq < 4; ++cq) {
-              float f[8], dz8[8];
-              unpack8(lds_v4(ap + sw_off(row, 4 * hp + cq)), f);
+              float kh[8], dz8[8];
+              unpack8(lds_v4(ak + sw_off(row, 4 * hp + cq)), kh);
               lds_f32n(dzs + 4 * (32 * hp + 8 * cq), dz8);
 #pragma unroll
               for (int e = 0; e < 8; ++e) {
                 const float dk = v[8 * cq + e] + dz8[e];
-                dg = fmaf(f[e], dk, dg);
-                v[8 * cq + e] = g * dk * fminf(f[e], 1.f);
+                khdk = fmaf(kh[e], dk, khdk);
+                v[8 * cq + e] = dk * fminf(kh[e], g);
               }
             }
             if (hp == 1) {
               __syncwarp();
-              if (lane == 0) mbar_arrive(&phi_empty[s]);  // phi(k~) rows read
+              if (lane == 0) mbar_arrive(&kh_empty[s]);  // K^ rows read
             }
           }
 #pragma unroll
@@ -445,7 +446,7 @@ __global__ void __launch_bounds__(kKThreads, 1)
         __syncwarp();
       }
       if (valid)
-        p.dgate[((size_t)t.b * N + tok) * H + t.h] = __float2bfloat16_rn(g * (dg - *cslot));
+        p.dgate[((size_t)t.b * N + tok) * H + t.h] = __float2bfloat16_rn(khdk - g * *cslot);
       ++li;
     }
     if (!ok && !ab.raised()) report(8, ab);
