@@ -547,9 +547,7 @@ constexpr int kQOffDn = kQOffP + kKStages * kKTile;        // 133120
 constexpr int kQOffB = kQOffDn + kKStages * kKTile;        // 165888: SzT hi, lo, S hi, lo
 constexpr int kQOffZ = kQOffB + 2 * kQSzT + 2 * kKBTile;   // 202752: z [64], w [64]
 constexpr int kQOffTaps = kQOffZ + 2 * kD * 4;             // float4 [64]: q taps of the head
-constexpr int kQOffDd = kQOffTaps + kD * 16;               // float [2][128]: dden
-constexpr int kQOffStg = kQOffDd + kKStages * kKTok * 4;
-constexpr int kQOffBar = kQOffStg + kQE2Warps * kKStg;
+constexpr int kQOffBar = kQOffTaps + kD * 16;
 // in_full, in_empty, p_full, p_empty, a1_full, a1_empty, dn_full, dn_empty,
 // a2_full, a2_empty (2 each), b_full, a3_full, fin
 constexpr int kQBars = 10 * kKStages + 3;
