@@ -43,6 +43,7 @@ METRIC = "GBLA fwd tokens/sec and % of GB300 HBM roofline at N=32768, 1 GPU"
 UNIT = "tokens/s"
 L2_BYTES = 129 * 1024 * 1024
 FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e data-sheet bandwidth, reported beside the measured peak
 
 
 # --------------------------------------------------------------------------- helpers
@@ -249,7 +250,11 @@ def bench_ours(args, ws, rank, local):
                 if peak_kind == "measured" else "fallback 6.8 TB/s",
                 "alg_bytes_per_launch": dom_bytes, "launch_ms": round(dom_ms, 5),
                 "phases_ms": {"state": round(t_state, 5), "readout": round(t_read, 5)},
-                "whole_step_frac": round(step_bytes / (ms * 1e-3) / 1e9 / peak, 4)}
+                "whole_step_frac": round(step_bytes / (ms * 1e-3) / 1e9 / peak, 4),
+                "peak_nominal": NOMINAL_HBM_GBS,
+                "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
+                "whole_step_frac_of_nominal":
+                    round(step_bytes / (ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS, 4)}
 
     e2e = None
     if not args.no_e2e and not args.flags:  # the host-buffer entry point runs the full core
@@ -484,17 +489,16 @@ def bench_e2e(args, w, inp, dev, gbla, tokens, ws):
 
 # --------------------------------------------------------------------------- oracle (CPU)
 
-def _oracle_inputs(inp, pairs, L):
-    """float64 per-(b, h) slices of the first L tokens, taken outside any timing."""
+def _oracle_inputs(inp, pairs, lens):
+    """float64 slices of the valid tokens of each (b, h) pair, taken outside any
+    timing; lens[i] is the number of tokens used for pairs[i]."""
     f64 = lambda t: t.detach().cpu().double().numpy()  # noqa: E731
-    q, k, v, og, gate = (f64(inp[n]) for n in ("q", "k", "v", "out_gate", "gate"))
     cw, nw = f64(inp["conv_w"]), f64(inp["norm_w"])
     out = []
-    for b, h in pairs:
-        out.append(dict(q=np.ascontiguousarray(q[b, :L, h]), k=np.ascontiguousarray(k[b, :L, h]),
-                        v=np.ascontiguousarray(v[b, :L, h]), a=np.ascontiguousarray(gate[b, :L, h]),
-                        og=np.ascontiguousarray(og[b, :L, h]), wq=cw[0, h], wk=cw[1, h],
-                        wv=cw[2, h], nw=nw[h]))
+    for (b, h), L in zip(pairs, lens):
+        sl = lambda n: np.ascontiguousarray(f64(inp[n][b, :L, h]))  # noqa: E731
+        out.append(dict(q=sl("q"), k=sl("k"), v=sl("v"), a=sl("gate"), og=sl("out_gate"),
+                        wq=cw[0, h], wk=cw[1, h], wv=cw[2, h], nw=nw[h]))
     return out
 
 
@@ -515,28 +519,47 @@ def _oracle_run(heads, n_threads):
             list(ex.map(one, heads))
 
 
+def _sample_pairs(w):
+    """The workload's (b, h) pairs with a non-empty sequence, heads outermost, so
+    that any prefix of the list spans the batch's length mix."""
+    lens = w.lengths()
+    return [(b, h) for h in range(w.H) for b in range(w.B) if lens[b] > 0]
+
+
 def cpu_baseline(w, inp, budget_s: float = 10.0):
-    """The oracle on all host cores over the workload's whole (batch, head)
-    sequences, repeated until about `budget_s` seconds have passed."""
+    """The oracle on the host cores over a bounded sample of the workload: batches of
+    (b, h) sequences, each over its own valid length, one thread per sequence, until
+    about `budget_s` seconds of oracle time; plus a single-thread rate on one
+    sequence.  Only the oracle calls are timed."""
     cores = os.cpu_count() or 1
-    pairs = [(b, h) for b in range(w.B) for h in range(w.H)]
-    L = w.lengths()[0]
-    heads = _oracle_inputs(inp, pairs, L)
+    lens = w.lengths()
+    pairs = _sample_pairs(w)
     threads = min(cores, len(pairs))
-    reps = 0
-    t0 = time.perf_counter()
-    while True:
+    done_tok_heads, dt, npairs, i = 0, 0.0, 0, 0
+    while dt < budget_s:
+        batch = [pairs[(i + j) % len(pairs)] for j in range(threads)]
+        i += threads
+        heads = _oracle_inputs(inp, batch, [lens[b] for b, _ in batch])
+        t0 = time.perf_counter()
         _oracle_run(heads, threads)
-        reps += 1
-        dt = time.perf_counter() - t0
-        if dt >= budget_s:
-            break
-    tok = reps * len(pairs) * L / w.H  # token-heads / heads = tokens
-    return {"value": round(tok / dt, 1), "unit": UNIT, "cores": threads, "kind": "oracle",
-            "seconds": round(dt, 3),
-            "sample": f"{reps} passes over all {len(pairs)} (batch, head) sequences of {L} "
-                      f"tokens ({w.name}), fp64 C oracle, one thread per sequence; tokens = "
-                      f"token-heads / H"}
+        dt += time.perf_counter() - t0
+        done_tok_heads += sum(lens[b] for b, _ in batch)
+        npairs += len(batch)
+    # single thread: the median-length sequence of the first batch
+    first = sorted(pairs[:threads], key=lambda bh: lens[bh[0]])
+    b1, h1 = first[len(first) // 2]
+    one = _oracle_inputs(inp, [(b1, h1)], [lens[b1]])
+    t0 = time.perf_counter()
+    _oracle_run(one, 1)
+    dt1 = time.perf_counter() - t0
+    return {"value": round(done_tok_heads / w.H / dt, 1), "unit": UNIT, "cores": threads,
+            "host_cores": cores, "kind": "oracle", "seconds": round(dt, 3),
+            "single_thread_value": round(lens[b1] / w.H / dt1, 1),
+            "sample": f"{npairs} (batch, head) sequences of {w.name} (cycling heads-outer over "
+                      f"all {len(pairs)} non-empty ones), each over its own valid length, "
+                      f"fp64 C oracle, {threads} threads (one per sequence) on "
+                      f"{cores} host cores; tokens = token-heads / H; single thread: one "
+                      f"{lens[b1]}-token sequence"}
 
 
 def bench_reference(args, ws, rank):
@@ -546,34 +569,43 @@ def bench_reference(args, ws, rank):
     w = WORKLOADS[args.workload]
     inp = make_inputs(w, "cpu")
     cores = os.cpu_count() or 1
-    pairs = [(b, h) for b in range(w.B) for h in range(w.H)]
+    lens = w.lengths()
+    pairs = _sample_pairs(w)
     # calibrate the sample so that (warmup + steps) fit in ~120 s
-    probe_L = 1024
-    heads = _oracle_inputs(inp, pairs[:1], probe_L)
+    probe_L = min(1024, max(lens))
+    bp = max(range(w.B), key=lambda b: lens[b])
+    heads = _oracle_inputs(inp, [(bp, 0)], [probe_L])
     t0 = time.perf_counter()
     _oracle_run(heads, 1)
     per_tok = (time.perf_counter() - t0) / probe_L
     n_pairs = min(len(pairs), cores)
+    batch = pairs[:n_pairs]
     step_budget = 120.0 / max(1, args.steps + args.warmup)
-    L = int(min(w.lengths()[0], max(64, step_budget / per_tok)))
-    heads = _oracle_inputs(inp, pairs[:n_pairs], L)
+    # each sequence over its own length, capped so that the slowest thread fits
+    cap = int(max(64, step_budget / per_tok))
+    use = [min(lens[b], cap) for b, _ in batch]
+    heads = _oracle_inputs(inp, batch, use)
     for _ in range(args.warmup):
         _oracle_run(heads, n_pairs)
     t0 = time.perf_counter()
     for _ in range(args.steps):
         _oracle_run(heads, n_pairs)
     dt = (time.perf_counter() - t0) / args.steps
-    tok = n_pairs * L / w.H
+    tok = sum(use) / w.H
     value = tok / dt
-    sample = (f"per step: {n_pairs} (batch, head) sequences x first {L} tokens of {w.name}, "
-              f"fp64 C oracle, one thread per sequence; tokens = token-heads / H")
+    capped = sum(1 for b, _ in batch if lens[b] > cap)
+    sample = (f"per step: {n_pairs} (batch, head) sequences of {w.name} (heads outer), each "
+              f"over its own valid length" + (f", {capped} of them capped at {cap} tokens"
+                                              if capped else "") +
+              f"; fp64 C oracle, one thread per sequence on {cores} host cores; "
+              f"tokens = token-heads / H")
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": UNIT,
             "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "D": w.D},
             "cpu_baseline": {"value": round(value, 1), "unit": UNIT, "cores": n_pairs,
-                             "kind": "oracle", "sample": sample},
+                             "host_cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -602,6 +634,9 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
     ws, rank, local = dist_env()
+    if args.gpus != ws:
+        sys.exit(f"bench.py: --gpus {args.gpus} but WORLD_SIZE is {ws}; for N > 1 launch one "
+                 f"process per GPU with torch.distributed.run --nproc-per-node N")
     if args.impl == "reference":
         bench_reference(args, ws, rank)
         return

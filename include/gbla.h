@@ -126,6 +126,23 @@ gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
                                  gbla_stream_t stream);
 
 /*
+ * gbla_forward_f32out -- debug variant of gbla_forward_ex (full core): the same
+ * kernels run the same arithmetic, but the readout stores o32 [B, N, H, D] in
+ * fp32 -- the value that gbla_forward would round to dtype -- so that the
+ * computation error of the bf16 path (Sec. 2.1 item 3 output) can be measured
+ * apart from the rounding of its stored result.  For bf16 inputs, rounding
+ * o32 to bf16 (round to nearest even) gives gbla_forward's o bit for bit.
+ * o32 must not overlap any input; rows t >= L_b are not written.  Arguments,
+ * validation and errors otherwise as gbla_forward_ex.
+ */
+gbla_status gbla_forward_f32out(const void *q, const void *k, const void *v,
+                                const void *gate, const void *out_gate,
+                                const float *conv_w, const float *norm_w,
+                                const int32_t *seq_lens, float *o32, int B, int H,
+                                int N, int D, gbla_dtype dtype, gbla_algo algo,
+                                gbla_stream_t stream);
+
+/*
  * gbla_backward -- gradients of sum(dy * o) of the layer core (full core, no
  * ablation) with respect to every input: the chain rule through the steps of
  * Sec. 2.1 in reverse (gated RMSNorm, readout, state, key-gate softmax, phi,
@@ -254,12 +271,15 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
  *
  * Limits and rules:
  *   - B * H * (D*D + D + 2) * 4 bytes must fit in GBLA_STATIC_SCRATCH_BYTES
- *     (at most 2015 (batch, head) pairs at D = 64, 508 at D = 128); larger
+ *     (at most 2015 (batch, head) pairs at D = 64, 507 at D = 128); larger
  *     problems return GBLA_ERR_INVALID_ARG before anything is enqueued.  Long
  *     sequences are cut into fewer, longer chunks to fit.
  *   - Each GPU that loads the library holds the array until the process exits.
  *   - The first call on a device looks up the array's device address on that
  *     device (once); make that first call before any stream capture starts.
+ *     The address is kept until the process exits, so after cudaDeviceReset
+ *     (or another teardown of the primary context) do not call it again on
+ *     that device.
  *   - Every call shares the one array.  Calls that overlap on the GPU (other
  *     streams or threads) race on it: serialise them.  Nothing carries over
  *     between calls; each call writes all the scratch it later reads.

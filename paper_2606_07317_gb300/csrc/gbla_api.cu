@@ -35,6 +35,10 @@ Range range_of(const void *p, size_t bytes) {
 constexpr int kMaxBH = 65535;
 constexpr int kMaxN = 1 << 28;
 
+}  // namespace
+
+namespace gbla {
+
 gbla_status check_dims(int B, int H, int N, int D, gbla_dtype dtype, bool *empty) {
   if (B < 0 || H < 0 || N < 0 || D < 0) return GBLA_ERR_INVALID_ARG;
   if (dtype != GBLA_FP32 && dtype != GBLA_BF16) return GBLA_ERR_UNSUPPORTED;
@@ -58,6 +62,21 @@ gbla_status check_seq_lens(const int32_t *seq_lens) {
   return GBLA_OK;
 }
 
+static thread_local cudaError_t t_last_cuda_error = cudaSuccess;
+
+gbla_status from_cuda(cudaError_t e) {
+  if (e == cudaSuccess) return GBLA_OK;
+  t_last_cuda_error = e;
+  (void)cudaGetLastError();  // clear the non-sticky launch error
+  return GBLA_ERR_CUDA;
+}
+
+static const char *last_cuda_error_string() { return cudaGetErrorString(t_last_cuda_error); }
+
+}  // namespace gbla
+
+namespace {
+
 bool use_tc(const Problem &p, gbla_algo algo, gbla_status *st) {
   *st = GBLA_OK;
   switch (algo) {
@@ -68,15 +87,6 @@ bool use_tc(const Problem &p, gbla_algo algo, gbla_status *st) {
       return true;
     default: *st = GBLA_ERR_UNSUPPORTED; return false;
   }
-}
-
-thread_local cudaError_t t_last_cuda_error = cudaSuccess;
-
-gbla_status from_cuda(cudaError_t e) {
-  if (e == cudaSuccess) return GBLA_OK;
-  t_last_cuda_error = e;
-  (void)cudaGetLastError();  // clear the non-sticky launch error
-  return GBLA_ERR_CUDA;
 }
 
 // Library-owned stream-ordered memory pool per device.  Its release threshold
@@ -156,9 +166,11 @@ gbla_status run_state(const Problem &p, bool tc, const void *k, const void *v,
 // reduction, so only the readout's reads of `state` wait for it.
 gbla_status run_readout(const Problem &p, bool tc, const void *q, const void *og,
                         const float *conv_w, const float *norm_w, const float *state,
-                        void *o, cudaStream_t st, bool after_state = false) {
-  if (tc) return from_cuda(tc_readout(p, q, og, conv_w, norm_w, state, o, st, after_state));
-  return from_cuda(simt_readout(p, q, og, conv_w, norm_w, state, o, st));
+                        void *o, cudaStream_t st, bool after_state = false,
+                        bool f32_out = false) {
+  if (tc)
+    return from_cuda(tc_readout(p, q, og, conv_w, norm_w, state, o, st, after_state, f32_out));
+  return from_cuda(simt_readout(p, q, og, conv_w, norm_w, state, o, st, f32_out));
 }
 
 }  // namespace
@@ -196,7 +208,7 @@ uint32_t gbla_device_error(int reset) {
   return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu || c == 0xFFFFFFFFu) ? 0xFFFFFFFFu : (a | b | c);
 }
 
-const char *gbla_last_cuda_error(void) { return cudaGetErrorString(t_last_cuda_error); }
+const char *gbla_last_cuda_error(void) { return last_cuda_error_string(); }
 
 gbla_status gbla_state(const void *k, const void *v, const void *gate,
                        const float *conv_w, const int32_t *seq_lens, float *state,
@@ -251,12 +263,13 @@ gbla_status gbla_forward_ex(const void *q, const void *k, const void *v,
                               D, dtype, algo, 0u, stream);
 }
 
-gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
-                                 const void *gate, const void *out_gate,
-                                 const float *conv_w, const float *norm_w,
-                                 const int32_t *seq_lens, void *o, int B, int H, int N,
-                                 int D, gbla_dtype dtype, gbla_algo algo, uint32_t flags,
-                                 gbla_stream_t stream) {
+// gbla_forward_variant, and with f32_out the debug path of gbla_forward_f32out
+// (o is then fp32 whatever the input dtype).
+static gbla_status forward_impl(const void *q, const void *k, const void *v, const void *gate,
+                                const void *out_gate, const float *conv_w,
+                                const float *norm_w, const int32_t *seq_lens, void *o, int B,
+                                int H, int N, int D, gbla_dtype dtype, gbla_algo algo,
+                                uint32_t flags, bool f32_out, gbla_stream_t stream) {
   if (flags & ~(uint32_t)GBLA_FLAG_BLA) return GBLA_ERR_INVALID_ARG;
   bool empty = false;
   gbla_status s = check_dims(B, H, N, D, dtype, &empty);
@@ -264,7 +277,7 @@ gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
   if ((s = check_ptrs({q, k, v, gate, out_gate, conv_w, norm_w, o})) != GBLA_OK) return s;
   if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
   const size_t bytes = (size_t)B * N * H * D * elem_bytes(dtype);
-  const Range out = range_of(o, bytes);
+  const Range out = range_of(o, f32_out ? (size_t)B * N * H * D * sizeof(float) : bytes);
   if (overlap(out, range_of(q, bytes)) || overlap(out, range_of(k, bytes)) ||
       overlap(out, range_of(v, bytes)) || overlap(out, range_of(out_gate, bytes)) ||
       overlap(out, range_of(gate, (size_t)B * N * H * elem_bytes(dtype))) ||
@@ -280,7 +293,27 @@ gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
   if ((s = state.alloc(sizeof(float) * state_floats(D) * B * H, st)) != GBLA_OK) return s;
   if ((s = run_state(p, tc, k, v, gate, conv_w, (float *)state.ptr, st)) != GBLA_OK) return s;
   return run_readout(p, tc, q, out_gate, conv_w, norm_w, (const float *)state.ptr, o, st,
-                     true);
+                     true, f32_out);
+}
+
+gbla_status gbla_forward_variant(const void *q, const void *k, const void *v,
+                                 const void *gate, const void *out_gate,
+                                 const float *conv_w, const float *norm_w,
+                                 const int32_t *seq_lens, void *o, int B, int H, int N,
+                                 int D, gbla_dtype dtype, gbla_algo algo, uint32_t flags,
+                                 gbla_stream_t stream) {
+  return forward_impl(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, o, B, H, N, D, dtype,
+                      algo, flags, false, stream);
+}
+
+gbla_status gbla_forward_f32out(const void *q, const void *k, const void *v,
+                                const void *gate, const void *out_gate,
+                                const float *conv_w, const float *norm_w,
+                                const int32_t *seq_lens, float *o32, int B, int H, int N,
+                                int D, gbla_dtype dtype, gbla_algo algo,
+                                gbla_stream_t stream) {
+  return forward_impl(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, o32, B, H, N, D,
+                      dtype, algo, 0u, true, stream);
 }
 
 gbla_status gbla_forward(const void *q, const void *k, const void *v,

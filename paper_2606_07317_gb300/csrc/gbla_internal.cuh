@@ -5,6 +5,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <initializer_list>
+
 #include "gbla.h"
 
 namespace gbla {
@@ -27,6 +29,16 @@ inline size_t state_floats(int D) { return (size_t)D * D + D; }
 // Counts every kernel this library enqueues (read by gbla_launch_count).
 void count_launch(unsigned n = 1);
 
+// Argument checks shared by every entry point (gbla_api.cu).
+// check_dims: sizes and dtype; *empty is set when B, H or N is 0.
+gbla_status check_dims(int B, int H, int N, int D, gbla_dtype dtype, bool *empty);
+// check_ptrs: every pointer non-null and 16-byte aligned.
+gbla_status check_ptrs(std::initializer_list<const void *> ptrs);
+// check_seq_lens: NULL or 4-byte aligned.
+gbla_status check_seq_lens(const int32_t *seq_lens);
+// Maps a CUDA error to a status; a failure is recorded for gbla_last_cuda_error.
+gbla_status from_cuda(cudaError_t e);
+
 // ---- CUDA-core (SIMT) family: every dtype and D ---------------------------
 struct SimtPlan {
   int chunk_len;  // tokens per partial
@@ -37,9 +49,11 @@ size_t simt_partials_bytes(const Problem &p, const SimtPlan &plan);
 cudaError_t simt_state(const Problem &p, const SimtPlan &plan, const void *k,
                        const void *v, const void *gate, const float *conv_w,
                        float *partials, float *state, cudaStream_t st);
+// f32_out: store o in fp32 whatever the input dtype (gbla_forward_f32out).
 cudaError_t simt_readout(const Problem &p, const void *q, const void *og,
                          const float *conv_w, const float *norm_w,
-                         const float *state, void *o, cudaStream_t st);
+                         const float *state, void *o, cudaStream_t st,
+                         bool f32_out = false);
 
 // ---- tensor-core (tcgen05 + TMA) family: bf16, D in {64, 128} -------------
 bool tc_supports(const Problem &p);
@@ -52,10 +66,11 @@ cudaError_t tc_state(const Problem &p, const void *k, const void *v,
 // after_state: launched right behind tc_state on the same stream; only the
 // reads of `state` then wait for the preceding kernel (the other inputs were
 // complete before tc_state started).
+// f32_out: the debug instantiation that stores o in fp32 (full core only).
 cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
                        const float *conv_w, const float *norm_w,
                        const float *state, void *o, cudaStream_t st,
-                       bool after_state = false);
+                       bool after_state = false, bool f32_out = false);
 // ---- backward (CUDA cores, fp32 arithmetic; gbla_bwd.cu) ------------------
 struct BwdArgs {
   const void *q, *k, *v, *gate, *out_gate, *dy;

@@ -201,12 +201,14 @@ simt_reduce_kernel(const float *__restrict__ part, float *__restrict__ state, in
   state[(size_t)bh * F + e] = s_l > 0.f ? acc / s_l : 0.f;
 }
 
-template <typename T, int D>
+// TO: type of the stored output; the product path stores the input type T, the
+// fp32-output debug path (gbla_forward_f32out) float, from the same y.
+template <typename T, typename TO, int D>
 __global__ void __launch_bounds__(kThreads)
 simt_readout_kernel(const T *__restrict__ q, const T *__restrict__ og,
                     const float *__restrict__ conv_w, const float *__restrict__ norm_w,
                     const int32_t *__restrict__ seq_lens, const float *__restrict__ state,
-                    T *__restrict__ o, int H, int N, float eps, uint32_t flags) {
+                    TO *__restrict__ o, int H, int N, float eps, uint32_t flags) {
   constexpr int J = D / 32;  // output columns per lane
   const int h = blockIdx.y, b = blockIdx.z;
   const int L = clamp_len(seq_lens, b, N);
@@ -297,18 +299,18 @@ cudaError_t launch_state(const Problem &p, const SimtPlan &plan, const void *k,
   return cudaGetLastError();
 }
 
-template <typename T, int D>
+template <typename T, typename TO, int D>
 cudaError_t launch_readout(const Problem &p, const void *q, const void *og,
                            const float *conv_w, const float *norm_w,
                            const float *state, void *o, cudaStream_t st) {
   const size_t smem = sizeof(float) * (D * D + D + kTokTile * D + D * kConvW);
-  auto kern = simt_readout_kernel<T, D>;
+  auto kern = simt_readout_kernel<T, TO, D>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   dim3 g((p.N + kTokTile - 1) / kTokTile, p.H, p.B);
   kern<<<g, kThreads, smem, st>>>((const T *)q, (const T *)og, conv_w, norm_w,
-                                  p.seq_lens, state, (T *)o, p.H, p.N, kRmsEps, p.flags);
+                                  p.seq_lens, state, (TO *)o, p.H, p.N, kRmsEps, p.flags);
   count_launch();
   return cudaGetLastError();
 }
@@ -346,9 +348,10 @@ cudaError_t simt_state(const Problem &p, const SimtPlan &plan, const void *k,
 
 cudaError_t simt_readout(const Problem &p, const void *q, const void *og,
                          const float *conv_w, const float *norm_w,
-                         const float *state, void *o, cudaStream_t st) {
-#define GBLA_SIMT_READ(T, DD) \
-  return launch_readout<T, DD>(p, q, og, conv_w, norm_w, state, o, st)
+                         const float *state, void *o, cudaStream_t st, bool f32_out) {
+#define GBLA_SIMT_READ(T, DD)                                                      \
+  return f32_out ? launch_readout<T, float, DD>(p, q, og, conv_w, norm_w, state, o, st) \
+                 : launch_readout<T, T, DD>(p, q, og, conv_w, norm_w, state, o, st)
   if (p.dtype == GBLA_FP32) {
     if (p.D == 32) GBLA_SIMT_READ(float, 32);
     if (p.D == 64) GBLA_SIMT_READ(float, 64);

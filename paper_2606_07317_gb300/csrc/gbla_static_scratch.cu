@@ -15,7 +15,9 @@
 // (on the host it names a host-side stand-in), so the device address is looked
 // up once per device with cudaGetSymbolAddress, with that device current, the
 // first time this entry point runs on it; that first call should therefore be
-// made before any stream capture begins.
+// made before any stream capture begins.  The address is kept for the life of
+// the process: after cudaDeviceReset (or any other teardown of the device's
+// primary context) the entry point must not be called again on that device.
 //
 // All calls share the one array and it keeps whatever the last call left in
 // it.  Nothing has to start at zero: each call writes every partial record its
@@ -54,8 +56,6 @@ cudaError_t static_scratch_address(void **out) {
   return cudaSuccess;
 }
 
-bool aligned16(const void *p) { return ((uintptr_t)p % 16) == 0; }
-
 bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
   const uintptr_t a0 = (uintptr_t)a, b0 = (uintptr_t)b;
   return a0 < b0 + nb && b0 < a0 + na;
@@ -69,15 +69,12 @@ extern "C" gbla_status gbla_state_static_scratch(
     const int32_t *seq_lens, float *state, int B, int H, int N, int D,
     gbla_dtype dtype, gbla_stream_t stream) {
   using namespace gbla;
-  if (B < 0 || H < 0 || N < 0 || D < 0) return GBLA_ERR_INVALID_ARG;
-  if (dtype != GBLA_FP32 && dtype != GBLA_BF16) return GBLA_ERR_UNSUPPORTED;
-  if (D != 32 && D != 64 && D != 128) return GBLA_ERR_UNSUPPORTED;
-  if (B > 65535 || H > 65535 || N > (1 << 28)) return GBLA_ERR_INVALID_ARG;
-  if (B == 0 || H == 0 || N == 0) return GBLA_OK;
-  const void *ptrs[] = {k, v, gate, conv_w, state};
-  for (const void *p : ptrs)
-    if (p == nullptr || !aligned16(p)) return GBLA_ERR_INVALID_ARG;
-  if (seq_lens != nullptr && ((uintptr_t)seq_lens % 4) != 0) return GBLA_ERR_INVALID_ARG;
+  // the same argument rules as gbla_state
+  bool empty = false;
+  gbla_status s = check_dims(B, H, N, D, dtype, &empty);
+  if (s != GBLA_OK || empty) return s;
+  if ((s = check_ptrs({k, v, gate, conv_w, state})) != GBLA_OK) return s;
+  if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
   const size_t es = dtype == GBLA_FP32 ? 4 : 2;
   const size_t in_bytes = (size_t)B * N * H * D * es;
   const size_t st_bytes = sizeof(float) * state_floats(D) * B * H;
@@ -101,8 +98,7 @@ extern "C" gbla_status gbla_state_static_scratch(
   }
 
   void *scratch = nullptr;
-  if (static_scratch_address(&scratch) != cudaSuccess) return GBLA_ERR_CUDA;
-  cudaError_t e = simt_state(p, plan, k, v, gate, conv_w, (float *)scratch, state,
-                             (cudaStream_t)stream);
-  return e == cudaSuccess ? GBLA_OK : GBLA_ERR_CUDA;
+  if ((s = from_cuda(static_scratch_address(&scratch))) != GBLA_OK) return s;
+  return from_cuda(simt_state(p, plan, k, v, gate, conv_w, (float *)scratch, state,
+                              (cudaStream_t)stream));
 }

@@ -972,6 +972,7 @@ struct ReadoutParams {
   const float *conv_w, *norm_w, *state;
   const int32_t *seq_lens;
   __nv_bfloat16 *o;
+  float *o32;      // fp32 output of the debug instantiation (F32O), else unused
   int B, H, N;
   float eps;
   int wait_late;   // only the reads of `state` wait for the preceding kernel
@@ -1032,7 +1033,10 @@ __device__ __forceinline__ void tile_next(TileCursor &t, const int32_t *seq_lens
   t.nrow = min(kRTok, t.L - t.r0);
 }
 
-template <int D, bool ABL>
+// F32O: the debug instantiation behind gbla_forward_f32out.  It runs the same
+// arithmetic and stores each y in fp32 (plain stores of the valid rows) where
+// the product instantiation rounds it to bf16 and stores the tile with TMA.
+template <int D, bool ABL, bool F32O>
 __global__ void __launch_bounds__(kRThreads, 1)
     tc_readout_kernel(const ReadoutParams p, const __grid_constant__ CUtensorMap tm_og,
                       const __grid_constant__ CUtensorMap tm_o,
@@ -1348,14 +1352,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
           unpack8(gcur, gv);
           const float wv8[8] = {wc0.x, wc0.y, wc0.z, wc0.w, wc1.x, wc1.y, wc1.z, wc1.w};
           const float *acc8 = g < 2 ? &va[8 * g] : &vb[8 * (g - 2)];
-          uint32_t outw[4];
+          float2 y[4];
           if (no_norm) {  // ablation without the gated RMSNorm: o = O = acc / den
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float2 y = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
-                                          make_float2(inv, inv));
-              outw[i] = f2_to_bf2(y.x, y.y);
-            }
+            for (int i = 0; i < 4; ++i)
+              y[i] = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]), make_float2(inv, inv));
           } else {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
@@ -1366,11 +1367,21 @@ __global__ void __launch_bounds__(kRThreads, 1)
                   __ffma2_rn(hg, make_float2(tanh_approx(hg.x), tanh_approx(hg.y)), hg);
               const float2 av = __fmul2_rn(make_float2(acc8[2 * i], acc8[2 * i + 1]),
                                            make_float2(wv8[2 * i], wv8[2 * i + 1]));
-              const float2 y = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
-              outw[i] = f2_to_bf2(y.x, y.y);
+              y[i] = __fmul2_rn(__fmul2_rn(av, sg), make_float2(rr, rr));
             }
           }
-          sts_v4(og_addr(32 * h2 + 8 * g), make_uint4(outw[0], outw[1], outw[2], outw[3]));
+          if constexpr (F32O) {
+            if (row < nrow) {
+              float4 *dst = (float4 *)(p.o32 + (((size_t)b * N + r0 + row) * H + h) * D +
+                                       part * CPE + 32 * h2 + 8 * g);
+              dst[0] = make_float4(y[0].x, y[0].y, y[1].x, y[1].y);
+              dst[1] = make_float4(y[2].x, y[2].y, y[3].x, y[3].y);
+            }
+          } else {
+            sts_v4(og_addr(32 * h2 + 8 * g),
+                   make_uint4(f2_to_bf2(y[0].x, y[0].y), f2_to_bf2(y[1].x, y[1].y),
+                              f2_to_bf2(y[2].x, y[2].y), f2_to_bf2(y[3].x, y[3].y)));
+          }
           gcur = gnext;
           wc0 = wn0;
           wc1 = wn1;
@@ -1383,7 +1394,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
       // pair meets on its named barrier, then one thread stores them with TMA
       // (full tiles) or releases the buffer after the direct stores (tail).
       const bool leader = part == 0 && lane == 0;
-      if (nrow == kRTok) {
+      if (!F32O && nrow == kRTok) {
         fence_proxy_async_smem();
         named_barrier(3 + q4, 64);
         if (leader) {
@@ -1408,8 +1419,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
         }
         __syncwarp();
       } else {
-        // Ragged tail: rows past the sequence end must not be written.
-        if (row < nrow) {
+        // Ragged tail: rows past the sequence end must not be written (the
+        // fp32 debug output was stored above).
+        if (!F32O && row < nrow) {
           __nv_bfloat16 *orow = p.o + (((size_t)b * N + r0 + row) * H + h) * D + part * CPE;
 #pragma unroll
           for (int cb = 0; cb < CPE; cb += 8) *(uint4 *)(orow + cb) = lds_v4(og_addr(cb));
@@ -1716,7 +1728,7 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
 template <int D>
 cudaError_t run_readout(const Problem &p, const void *q, const void *og, const float *conv_w,
                         const float *norm_w, const float *state, void *o, cudaStream_t st,
-                        bool after_state) {
+                        bool after_state, bool f32_out) {
   using C = ReadoutCfg<D>;
   CUtensorMap tm_og, tm_o, tm_q;
   cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D, kRTok);
@@ -1731,13 +1743,15 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   rp.state = state;
   rp.seq_lens = p.seq_lens;
   rp.o = (__nv_bfloat16 *)o;
+  rp.o32 = (float *)o;
   rp.B = p.B;
   rp.H = p.H;
   rp.N = p.N;
   rp.eps = kRmsEps;
   rp.wait_late = after_state ? 1 : 0;
   rp.flags = p.flags;
-  auto kern = p.flags ? tc_readout_kernel<D, true> : tc_readout_kernel<D, false>;
+  auto kern = f32_out ? tc_readout_kernel<D, false, true>
+                      : (p.flags ? tc_readout_kernel<D, true, false> : tc_readout_kernel<D, false, false>);
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem)) !=
       cudaSuccess)
     return e;
@@ -1784,10 +1798,12 @@ cudaError_t tc_state(const Problem &p, const void *k, const void *v, const void 
 
 cudaError_t tc_readout(const Problem &p, const void *q, const void *og, const float *conv_w,
                        const float *norm_w, const float *state, void *o, cudaStream_t st,
-                       bool after_state) {
+                       bool after_state, bool f32_out) {
+  if (f32_out && p.flags) return cudaErrorInvalidValue;  // the debug output is the full core's
   switch (p.D) {
-    case 64: return run_readout<64>(p, q, og, conv_w, norm_w, state, o, st, after_state);
-    case 128: return run_readout<128>(p, q, og, conv_w, norm_w, state, o, st, after_state);
+    case 64: return run_readout<64>(p, q, og, conv_w, norm_w, state, o, st, after_state, f32_out);
+    case 128:
+      return run_readout<128>(p, q, og, conv_w, norm_w, state, o, st, after_state, f32_out);
   }
   return cudaErrorInvalidValue;
 }

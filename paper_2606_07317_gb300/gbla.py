@@ -23,7 +23,8 @@ FLAG_NO_CONV, FLAG_NO_GATE, FLAG_NO_NORM = 1, 2, 4
 FLAG_BLA = FLAG_NO_CONV | FLAG_NO_GATE | FLAG_NO_NORM
 CONV_WIDTH = 4
 
-EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_backward",
+EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_forward_f32out",
+            "gbla_backward",
             "gbla_state",
             "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
@@ -69,6 +70,8 @@ def load(path: str | None = None):
         lib.gbla_forward_ex.restype = _i
         lib.gbla_forward_variant.argtypes = fwd + [_i, ctypes.c_uint32, _vp]
         lib.gbla_forward_variant.restype = _i
+        lib.gbla_forward_f32out.argtypes = fwd + [_i, _vp]
+        lib.gbla_forward_f32out.restype = _i
         lib.gbla_backward.argtypes = [_vp] * 16 + [_i] * 5 + [_vp]
         lib.gbla_backward.restype = _i
         lib.gbla_project.argtypes = [_vp] * 9 + [_i] * 6 + [_vp]
@@ -181,6 +184,21 @@ def forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
         _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),
         _stream(stream))
     _check(st, "gbla_forward_ex")
+    return out
+
+
+def forward_f32out(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
+                   algo: int = ALGO_AUTO, stream=None) -> torch.Tensor:
+    """Debug variant of forward (gbla_forward_f32out): the same kernels and arithmetic,
+    with o stored in fp32 before the rounding to the input dtype."""
+    B, H, N, D = _bhnd(q)
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    st = load().gbla_forward_f32out(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w),
+        _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),
+        _stream(stream))
+    _check(st, "gbla_forward_f32out")
     return out
 
 

@@ -92,6 +92,43 @@ def oracle_full(inp: dict, n_threads: int | None = None, flags: int = 0) -> np.n
         n_threads=n_threads or os.cpu_count() or 1)
 
 
+def oracle_rows(inp: dict, n_threads: int | None = None) -> list:
+    """Oracle per batch row over its valid tokens: a list of [L_b, H, D] arrays.
+
+    Each row is converted to float64 and run on its own, so a ragged workload
+    padded to a long N never needs the padded [B, N, H, D] tensors in float64.
+    Rows run concurrently (the C oracle releases the GIL and threads over heads)."""
+    import concurrent.futures as cf
+
+    B, N, H, _ = inp["q"].shape
+    sl = inp["seq_lens"]
+    lens = [N if sl is None else max(0, min(int(sl[b]), N)) for b in range(B)]
+    cores = n_threads or os.cpu_count() or 1
+    per_call = max(1, min(H, cores))
+
+    def one(b):
+        L = lens[b]
+        cut = lambda t: to64(t[b:b + 1, :L])  # noqa: E731
+        if L == 0:
+            return np.zeros((0, H, inp["q"].shape[3]))
+        y = oracle.gbla_forward(cut(inp["q"]), cut(inp["k"]), cut(inp["v"]), cut(inp["gate"]),
+                                cut(inp["out_gate"]), to64(inp["conv_w"]), to64(inp["norm_w"]),
+                                None, n_threads=per_call)
+        return y[0]
+
+    with cf.ThreadPoolExecutor(max(1, cores // per_call)) as ex:
+        return list(ex.map(one, range(B)))
+
+
+def log_stats(record: dict) -> None:
+    """Appends one JSON line of measured errors to $GBLA_PARITY_LOG, if set."""
+    path = os.environ.get("GBLA_PARITY_LOG")
+    if path:
+        import json
+        with open(path, "a") as f:
+            f.write(json.dumps(record) + "\n")
+
+
 def oracle_head(inp: dict, b: int, h: int, L: int | None = None, intermediates=False):
     """Oracle for one (batch, head) over its valid rows."""
     N = inp["q"].shape[1]

@@ -10,12 +10,42 @@ import torch
 
 from paper_2606_07317_gb300 import gbla
 from paper_2606_07317_gb300.workloads import WORKLOADS, custom, make_inputs
-from parity_util import compare, compare_prenorm, oracle_full, oracle_head, to64, valid_mask
+from parity_util import (compare, compare_prenorm, log_stats, oracle_full, oracle_head,
+                         oracle_rows, to64, valid_mask)
 
 pytestmark = pytest.mark.gpu
 
 SENTINEL = -777.0
 ALGOS = {"auto": gbla.ALGO_AUTO, "simt": gbla.ALGO_SIMT}
+# The benchmark spec's bound on the bf16 path's computation error after the gated
+# RMSNorm, applied literally to the fp32 output of gbla_forward_f32out.
+LITERAL_ABS_TOL = 2e-2
+
+_INPUTS, _REFS = {}, {}
+
+
+def _named(name):
+    """Seeded inputs (on the GPU) and the oracle per batch row, computed once per
+    workload for the whole module."""
+    if name not in _INPUTS:
+        inp = make_inputs(WORKLOADS[name], "cuda")
+        _INPUTS[name] = inp
+        _REFS[name] = oracle_rows(inp)
+    return _INPUTS[name], _REFS[name]
+
+
+def _rows_vs_ref(y_t, refs, lens):
+    """(gpu valid rows, oracle valid rows) as flat float64 arrays, plus a check that
+    every padded row still holds the sentinel."""
+    yc = y_t.cpu()
+    ys, rs = [], []
+    for b, L in enumerate(lens):
+        ys.append(to64(yc[b, :L]).ravel())
+        rs.append(refs[b].ravel())
+        if L < yc.shape[1]:
+            assert torch.all(yc[b, L:] == torch.tensor(SENTINEL, dtype=yc.dtype)), \
+                f"rows past the end of sequence {b} were written"
+    return np.concatenate(ys), np.concatenate(rs)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -50,37 +80,64 @@ def _check_against(y_gpu_t, y_ref, inp, dtype):
                                   "bf16_b4_h8_n8192_d64"])
 def test_parity_workload(name, algo):
     w = WORKLOADS[name]
-    inp = make_inputs(w, "cuda")
+    inp, refs = _named(name)
     y = _run(inp, ALGOS[algo])
-    _check_against(y, oracle_full(inp), inp, w.dtype)
+    st = compare(*_rows_vs_ref(y, refs, w.lengths()), w.dtype)
+    log_stats({"test": "parity", "workload": name, "algo": algo, **st})
+    assert st["ok"], st
 
 
 def test_parity_headline_n32768():
-    w = WORKLOADS["bf16_b2_h8_n32768_d64"]
-    inp = make_inputs(w, "cuda")
+    name = "bf16_b2_h8_n32768_d64"
+    w = WORKLOADS[name]
+    inp, refs = _named(name)
     y = _run(inp)
-    _check_against(y, oracle_full(inp), inp, w.dtype)
+    st = compare(*_rows_vs_ref(y, refs, w.lengths()), w.dtype)
+    log_stats({"test": "parity", "workload": name, "algo": "auto", **st})
+    assert st["ok"], st
 
 
-def test_parity_ragged_d128_sampled():
-    """Full-size ragged workload; the oracle runs on a sample of (batch, head)
-    pairs: the longest, the shortest and a middle sequence."""
-    w = WORKLOADS["bf16_ragged_b32_h8_d128"]
-    inp = make_inputs(w, "cuda")
+def test_parity_ragged_d128():
+    """Full-size ragged workload (32 rows, log-normal lengths up to 32768, D = 128):
+    every one of the 32 x 8 (batch, head) sequences against the oracle, element by
+    element, and every padded row left untouched."""
+    name = "bf16_ragged_b32_h8_d128"
+    w = WORKLOADS[name]
+    inp, refs = _named(name)
     y = _run(inp)
-    lens = np.array(w.seq_lens)
-    order = np.argsort(lens)
-    picks = [(int(order[-1]), 0), (int(order[0]), 3), (int(order[len(order) // 2]), 7)]
-    yc = y.cpu()
-    for b, h in picks:
-        L = int(lens[b])
-        ref = oracle_head(inp, b, h)
-        st = compare(to64(yc[b, :L, h]), ref, "bf16")
-        assert st["ok"], (b, h, st)
-    # padded rows untouched everywhere
-    for b in range(w.B):
-        L = int(lens[b])
-        assert torch.all(yc[b, L:] == torch.tensor(SENTINEL, dtype=yc.dtype))
+    st = compare(*_rows_vs_ref(y, refs, w.lengths()), "bf16")
+    log_stats({"test": "parity", "workload": name, "algo": "auto", **st})
+    assert st["ok"], st
+
+
+@pytest.mark.parametrize("algo", list(ALGOS), ids=list(ALGOS))
+@pytest.mark.parametrize("name", ["bf16_b8_h8_n2048_d64", "bf16_b4_h8_n8192_d64",
+                                  "bf16_b2_h8_n32768_d64", "bf16_ragged_b32_h8_d128"])
+def test_literal_budget_before_output_rounding(name, algo):
+    """The bf16 path's own arithmetic error, apart from the rounding of its stored
+    output: gbla_forward_f32out runs the same kernels and stores y in fp32.  Its
+    max |y - y_ref| must be <= 2e-2 literally (Sec. 2.1 item 3 output), and rounding
+    it to bf16 must give gbla_forward's output bit for bit (same arithmetic)."""
+    w = WORKLOADS[name]
+    inp, refs = _named(name)
+    y16 = _run(inp, ALGOS[algo])
+    y32 = torch.full(inp["q"].shape, SENTINEL, dtype=torch.float32, device="cuda")
+    gbla.forward_f32out(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"],
+                        inp["conv_w"], inp["norm_w"], inp["seq_lens"], out=y32,
+                        algo=ALGOS[algo])
+    torch.cuda.synchronize()
+    g32, r = _rows_vs_ref(y32, refs, w.lengths())
+    g16, _ = _rows_vs_ref(y16, refs, w.lengths())
+    assert torch.equal(y32.to(torch.bfloat16), y16), "f32 output rounds to a different o"
+    d32, d16 = np.abs(g32 - r), np.abs(g16 - r)
+    rec = {"test": "literal", "workload": name, "algo": algo,
+           "max_abs_before_rounding": float(d32.max()),
+           "max_abs_after_rounding": float(d16.max()),
+           "rms_err_before_rounding": float(np.sqrt(np.mean(d32 ** 2))),
+           "max_abs_ref": float(np.abs(r).max()), "elements": int(r.size)}
+    log_stats(rec)
+    assert np.all(np.isfinite(g32)), rec
+    assert rec["max_abs_before_rounding"] <= LITERAL_ABS_TOL, rec
 
 
 @pytest.mark.parametrize("algo", list(ALGOS), ids=list(ALGOS))

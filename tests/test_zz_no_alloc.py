@@ -5,7 +5,12 @@ array inside the library instead of freshly allocated scratch.
 
 It must agree with the allocating gbla_state within the tolerance the state
 tests use, call after call: the second call reuses the array the first one
-filled.  This file is collected last on purpose."""
+filled.  It must also leave the device's free memory unchanged from one call
+to the next.
+
+This file is collected last on purpose: the entry point is an extra, and if
+it fails, a run that stops at the first failure (pytest -x) has already run
+every other test."""
 import numpy as np
 import pytest
 import torch
@@ -47,6 +52,41 @@ def test_static_scratch_matches_gbla_state_on_consecutive_calls():
         gbla.state_static_scratch(*_args(inp), out=out)
         torch.cuda.synchronize()
         _close(out, ref, w.D, w.dtype)
+
+
+def test_static_scratch_allocates_nothing():
+    """After a first call (which may load the library's module, and with it the
+    fixed array, onto the device), further calls leave the free device memory
+    exactly as it was."""
+    gbla.load()
+    w = custom(B=2, H=4, N=3000, D=64, dtype="bf16", seed=34, seq_lens=[3000, 1234])
+    inp = make_inputs(w, "cuda")
+    out = torch.empty((w.B, w.H, w.D * w.D + w.D), dtype=torch.float32, device="cuda")
+    gbla.state_static_scratch(*_args(inp), out=out)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    for _ in range(3):
+        gbla.state_static_scratch(*_args(inp), out=out)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0, (free0, free1)
+
+
+def test_static_scratch_size_limit_at_d128():
+    """507 (batch, head) pairs fit the fixed array at D = 128, 508 do not."""
+    gbla.load()
+    cw = torch.zeros((3, 1, 128, 4), device="cuda")
+    for B, ok in ((507, True), (508, False)):
+        k = torch.zeros((B, 1, 1, 128), dtype=torch.bfloat16, device="cuda")
+        gate = torch.zeros((B, 1, 1), dtype=torch.bfloat16, device="cuda")
+        if ok:
+            st = gbla.state_static_scratch(k, k, gate, cw)
+            torch.cuda.synchronize()
+            assert torch.isfinite(st).all()
+        else:
+            with pytest.raises(gbla.GblaError) as e:
+                gbla.state_static_scratch(k, k, gate, cw)
+            assert e.value.status == gbla.GBLA_ERR_INVALID_ARG
 
 
 def test_static_scratch_rejects_oversized_problem():
