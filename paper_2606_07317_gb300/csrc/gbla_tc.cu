@@ -2,23 +2,24 @@
 // D in {64, 128}.  Three kernels, launched back to back on one stream:
 //
 //  tc_state_kernel   (Sec. 2.1 item 1 and item 2, k/v side)
-//      Persistent; one CTA per SM.  Each (batch, group of 128/D heads) sequence
-//      is cut into chunks of S tokens and every CTA takes a contiguous range of
-//      chunks, so work is balanced whatever the sequence lengths.  Per chunk:
-//      a pre-pass over the gate logits gives the chunk maximum m and the
-//      per-token weights 2^a' (a' = (a - m) log2 e); three warps stream raw
-//      k and v tiles (64 tokens + 3 rows of conv history) into a TMA ring;
-//      sixteen converter warps run the causal Conv1D of k, phi and the gate
-//      weight in fp32 and write K^ as bf16 into a 128B-swizzled tile; one
+//      Persistent; one CTA per SM.  The 64-token stages of all
+//      (batch, group of 128/D heads) sequences are cut into balanced ranges of
+//      consecutive stages (ranges may span sequences), so work is even whatever
+//      the lengths.  Per range: a pre-pass over its gate logits gives the
+//      maximum m over each segment (its part in one sequence); warp 17 streams
+//      k tiles (64 tokens + 3 rows of conv history) into a k ring, warp 18 the
+//      v tiles into the operand ring; sixteen converter warps run the causal
+//      Conv1D of k, phi and the gate weight 2^a' (a' = (a - m) log2 e) in fp32
+//      and write K^ as bf16 into a 128B-swizzled tile beside the v tile; one
 //      thread issues tcgen05.mma (bf16, fp32 accumulation in TMEM).  The
 //      Conv1D of v is linear, so it is folded into the contraction:
 //      S = sum_tau w_tau (K^T v shifted by tau), the four shifted views of the
 //      raw v tile forming one N = 256 operand, and the taps are applied per
 //      column when the accumulators are drained.  The diagonal D x D blocks
-//      are the per-head partial states S_c; z_c, m_c and l_c = sum 2^a'
-//      complete each partial record.
-//  tc_reduce_kernel  fixed-order, max-rescaled combination of the partial
-//      records into S = K^T V~ and z = K^T 1 with the softmax gate.
+//      are the segment's partial state; z, m and l = sum 2^a' complete its
+//      record.
+//  tc_reduce_kernel  fixed-order, max-rescaled combination of the records
+//      into S = K^T V~ and z = K^T 1 with the softmax gate.
 //  tc_readout_kernel (Sec. 2.1 item 2 readout and item 3)
 //      Persistent; 128-token tiles of one (batch, head).  Eight producer warps
 //      compute phi(Conv1D(q)) from a TMA q tile into a K-major bf16 tile; one
@@ -60,66 +61,71 @@ using namespace sm100;
 constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the state
 
 // ------------------------------------------------------------------ state
-// 20 warps: two groups of 8 converter warps turn raw k tiles into K^ (bf16,
-// the A operand), the groups taking alternate stages; one warp issues the
-// MMAs and three the TMA loads, one box of each stage apiece, with two lanes
-// of each taking alternate stages (a single issuing thread caps an SM's
-// bulk-copy rate at about one box per 0.5 us, well below its share of HBM
-// bandwidth for boxes this size; independent issuers overlap).  At most 5 warps per SM
-// sub-partition, so each thread may hold 96 registers.  V~ is never formed: the Conv1D of v is
-// linear, so S = sum_tau w_tau (K^T v shifted by tau) with the taps applied
-// per column of the accumulators when they are drained, and the raw bf16 v
-// tiles that TMA brings in are the B operand as they stand.
+// 19 warps: two groups of 8 converter warps, each group converting one
+// 32-token half of every 64-token stage; one warp issues the MMAs; warp 17
+// loads the k tiles (one issuing lane per k ring slot) and warp 18 the v tiles
+// (two issuing lanes, lane l filling the operand slots l and l + 2: a single
+// issuing thread caps an SM's bulk-copy rate at about one box per 0.5 us,
+// below its share of HBM bandwidth).  Every waiter on a ring barrier waits for
+// each of its phases in turn (a parity wait can only tell the current phase
+// from the one before it).
+//
+// The k tile of a stage (one head group, 64 tokens + 3 rows of conv history)
+// lands in the k ring and is free again as soon as the converters have turned
+// it into K^ = g phi(Conv1D(k)) (bf16, the A operand).  The v tile (two
+// 64-channel blocks, 128B-swizzled) lands next to K^ in the operand ring and
+// is the B operand as it stands: the Conv1D of v is linear, so
+// S = sum_tau w_tau (K^T v shifted by tau), the four shifted views of the v
+// tile forming one N = 256 operand per block, with the taps applied per column
+// when the accumulators are drained.  V~ is never formed or rounded.
 constexpr int kSGroupWarps = 8;                      // converter warps per group
 constexpr int kSCvtWarps = 2 * kSGroupWarps;         // 16
 constexpr int kSMmaWarp = kSCvtWarps;                // 16
-constexpr int kSTmaWarp = kSCvtWarps + 1;            // 17: k box; 18, 19: v boxes
-constexpr int kSTmaWarps = 3;
-constexpr int kSTmaLanes = 2;  // issuing lanes per TMA warp, taking alternate stages
-constexpr int kSThreads = (kSTmaWarp + kSTmaWarps) * 32;  // 640
+constexpr int kSKWarp = kSCvtWarps + 1;              // 17: k tiles
+constexpr int kSVWarp = kSCvtWarps + 2;              // 18: v tiles
+constexpr int kSThreads = (kSVWarp + 1) * 32;        // 608
 constexpr int kSProd = kSCvtWarps * 32;              // converter threads
-constexpr int kSGroupThreads = kSGroupWarps * 32;
 constexpr int kSTok = 64;                            // tokens per stage
 constexpr int kSHalo = kConvW - 1;                   // conv history rows in front of a tile
 constexpr int kSRawRows = kSTok + kSHalo;            // 67
-// raw stage: v as two 64-channel MN blocks (128B swizzle, 72-row pitch) + k group rows
+constexpr int kSRawRowB = kGroupCh * 2;              // bytes of one token's k group row
+constexpr int kSKBox = kSRawRows * kSRawRowB;        // 17152: one k tile
+constexpr int kSKStages = 3;                         // k ring: one issuing lane per slot
 constexpr int kSVBlock = 72 * 128;                   // 9216: v block pitch (1024-aligned)
 constexpr int kSVBoxBytes = kSRawRows * 128;         // 8576 written by one v box
-constexpr int kSRawRowK = kGroupCh * 2;              // bytes of one token's k group row
-constexpr int kSRawKBytes = kSRawRows * kSRawRowK;   // 17152
-constexpr int kSRawK = 2 * kSVBlock;                 // k tile offset within a raw stage
-constexpr int kSRawStage = (kSRawK + kSRawKBytes + 1023) / 1024 * 1024;  // 35840
-constexpr int kSRawStages = 4;
-// Raw stages issued before the chunk prefix: one.  The first stage then
-// arrives ahead of the rest of every CTA's start-up burst (measured: 1.1 us
-// shorter step than issuing the whole ring up front).
-constexpr int kSEarlyStages = 1;
-constexpr int kSABlock = kSTok * 128;                // 8192: one 64-channel MN block of K^
-constexpr int kSAStage = 2 * kSABlock;
-constexpr int kSAStages = 3;
-constexpr int kChunkMax = 2048;                      // longest chunk (tokens)
-constexpr int kMaxChunksPerSeq = 4096;
-constexpr int kSGateStride = kChunkMax + kSTok;      // gate logits (bf16 bits) per head
+constexpr int kSMnBlock = kSTok * 128;               // 8192: one 64-channel MN block of K^
+constexpr int kSOpV = 2 * kSMnBlock;                 // v blocks after K^ in an operand slot
+constexpr int kSOpStage = kSOpV + 2 * kSVBlock;      // 34816
+constexpr int kSOpStages = 4;                        // operand ring: v lane l fills l, l + 2
+constexpr int kSVLanes = 2;
+constexpr int kRangeStages = 32;                     // longest range (stages)
+constexpr int kRangeTok = kRangeStages * kSTok;      // 2048
 constexpr uint32_t kSTmemCols = 512;                 // per v block: 4 taps x 64 columns
 
 constexpr int kMaxBatch = 2048;
 
 // Shared-memory map of the state kernel (offsets from a 1024-aligned base).
-constexpr int kSOffRaw = 0;
-constexpr int kSOffA = kSOffRaw + kSRawStages * kSRawStage;
-constexpr int kSOffGate = kSOffA + kSAStages * kSAStage;            // u16 [2][kSGateStride]
-constexpr int kSOffZred = kSOffGate + 2 * kSGateStride * 2;         // float [16][128]
-constexpr int kSOffWv = kSOffZred + 16 * kGroupCh * 4;               // float4 [128]: v taps
-constexpr int kSOffRed = kSOffWv + kGroupCh * 16;                   // float [256]
-constexpr int kSOffPre = kSOffRed + 256 * 4;                        // int [kMaxBatch + 1]
+constexpr int kSOffOp = 0;
+constexpr int kSOffK = kSOffOp + kSOpStages * kSOpStage;
+constexpr int kSOffGate = kSOffK + kSKStages * kSKBox;              // u16 [2][kRangeTok]
+constexpr int kSOffHmax = kSOffGate + 2 * kRangeTok * 2;            // float [2][64]: half-stage max
+constexpr int kSOffSegm = kSOffHmax + 2 * 64 * 4;                   // float [2][32]: segment max
+constexpr int kSOffZred = kSOffSegm + 2 * kRangeStages * 4;         // float [16][128]
+constexpr int kSOffLred = kSOffZred + 16 * kGroupCh * 4;            // float [16][2]
+constexpr int kSOffWv = kSOffLred + 16 * 2 * 4;                     // float4 [128]: v taps
+constexpr int kSOffRed = kSOffWv + kGroupCh * 16;                   // int [32]: scan scratch
+constexpr int kSOffPre = kSOffRed + 32 * 4;                         // int [kMaxBatch + 1]
 constexpr int kSOffBar = kSOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
-// raw_full, raw_empty, a_full, a_empty, done, final
-constexpr int kSBarCount = 2 * kSRawStages + 2 * kSAStages + 2;
+// k_full, k_empty, op_full (K^ written), v_full (v landed), op_empty, done, final,
+// logits_in (the first range's gate logits are in shared memory)
+constexpr int kSBarCount = 2 * kSKStages + 3 * kSOpStages + 3;
 constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;                // tmem addr, abort flag
 constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                  // + alignment slack
 static_assert(kSSmemBytes <= 227 * 1024, "state shared memory");
-static_assert(kSRawK + kSRawKBytes <= kSRawStage, "raw stage");
-static_assert(kSRawStage % 1024 == 0 && kSVBlock % 1024 == 0, "swizzled v blocks");
+static_assert(kSOpStage % 1024 == 0 && kSVBlock % 1024 == 0 && kSOffK % 128 == 0 &&
+                  kSKBox % 128 == 0,
+              "TMA and swizzled operand alignment");
+static_assert(kSOpStages % kSVLanes == 0, "each operand slot has one issuing lane");
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -310,30 +316,37 @@ __device__ __forceinline__ float2 khat2(float2 xl, float al, float wl) {
   return __ffma2_rn(make_float2(wl, wl), d, e);
 }
 
+__device__ __forceinline__ float bf16_bits_to_f32(unsigned short r) {
+  return __uint_as_float((uint32_t)r << 16);
+}
+
 // a' = (a - m) log2(e) of a gate logit given as bf16 bits, with mlog = m log2(e)
 // (0 when the head is missing: its logits are all -inf, and so is a').
 __device__ __forceinline__ float gate_log2(unsigned short a, float mlog) {
   return fmaf(__uint_as_float((uint32_t)a << 16), kLog2e, -mlog);
 }
 
-// One token quad of a converter thread: channels 4q..4q+3 of the head group
-// at tokens 4j..4j+3 of a 32-token half of the stage.  Reads the 7 raw k rows it needs (3 of conv
-// history) from the TMA tile and the 4 tokens' gate logits, convolves, applies
-// phi and the gate weight, and writes K^ as bf16 into the MN-major,
-// 128B-swizzled A tile (one 8-byte piece per token row).  Tokens past the
-// sequence end (nvalid < 4) are zeros.
-__device__ __forceinline__ void state_convert(uint32_t raw, uint32_t arow, uint32_t cs,
-                                              uint32_t gws, float mlog, const float (&w)[4][4],
-                                              float2 (&z)[2], int nvalid) {
+// One token quad of a converter thread, k side: channels 4q..4q+3 of the head
+// group at 4 consecutive tokens of the stage.  Reads the 7 raw k rows it needs
+// (3 of conv history) from the TMA tile and the 4 tokens' gate logits,
+// convolves, applies phi and the gate weight, and writes K^ as bf16 into the
+// MN-major, 128B-swizzled A tile (one 8-byte piece per token row).  Tokens past
+// the sequence end (nvalid < 4) are zeros.  Returns the sum of 2^a' ln 2 over
+// the 4 tokens (0 for tokens past the end, whose logits are -inf).
+__device__ __forceinline__ float state_convert_k(uint32_t raw, uint32_t arow, uint32_t cs,
+                                                 uint32_t gws, float mlog, const float (&w)[4][4],
+                                                 float2 (&z)[2], int nvalid) {
   float x[7][4];
 #pragma unroll
-  for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRowK), x[r]);
+  for (int r = 0; r < 7; ++r) unpack4(lds_v2(raw + r * kSRawRowB), x[r]);
   const uint2 g4 = lds_v2(gws);  // 4 bf16 logits
   const unsigned short ga[4] = {(unsigned short)(g4.x & 0xffffu), (unsigned short)(g4.x >> 16),
                                 (unsigned short)(g4.y & 0xffffu), (unsigned short)(g4.y >> 16)};
+  float lsum = 0.f;
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     const float al = gate_log2(ga[u], mlog), wl = ex2_approx(al) * kLn2;
+    lsum += wl;
     float2 k01 = khat2(conv_rows(w, x, u, 0), al, wl);
     float2 k23 = khat2(conv_rows(w, x, u, 2), al, wl);
     if (u >= nvalid) {  // rows past the sequence end may hold anything, NaN included
@@ -344,6 +357,7 @@ __device__ __forceinline__ void state_convert(uint32_t raw, uint32_t arow, uint3
     z[1] = __fadd2_rn(z[1], k23);
     sts_v2(arow + u * 128 + ((cs ^ u) << 4), f2_to_bf2(k01.x, k01.y), f2_to_bf2(k23.x, k23.y));
   }
+  return lsum;
 }
 
 // ===================================================================== state
@@ -351,92 +365,68 @@ struct StateParams {
   const __nv_bfloat16 *gate;
   const float *conv_w;
   const int32_t *seq_lens;
-  float *records;        // [chunks][G][D*D + D + 4]: S, z, m, l, 2 pad
-  int32_t *chunk_pre;    // [B + 1] chunk prefix (written by CTA 0)
-  int B, H, N, S, HG;
+  float *records;        // [ranges + sequences][G][D*D + D + 4]: S, z, m, l, 2 pad
+  int32_t *stage_pre;    // [B + 1] stage prefix (written by CTA 0 when seq_lens is given)
+  int B, H, N, HG;
   uint32_t flags;        // gbla_flags (NO_CONV, NO_GATE)
 };
 
-// Chunk k of the flattened (batch, head group, chunk) order.
-struct ChunkRef {
-  int b, L, hbase, t0, n, nst;
-};
-template <int G>
-__device__ __forceinline__ ChunkRef decode_chunk(const StateParams &p, const int *pre, int k) {
-  ChunkRef c;
-  c.b = find_batch(pre, p.B, k);
-  c.L = clamp_len(p.seq_lens, c.b, p.N);
-  const int nck = (c.L + p.S - 1) / p.S;
-  const int r = k - pre[c.b];
-  c.hbase = (r / nck) * G;
-  c.t0 = (r % nck) * p.S;
-  c.n = min(c.t0 + p.S, c.L) - c.t0;
-  c.nst = (c.n + kSTok - 1) / kSTok;
-  return c;
+// Work split.  The state step's work is the list of 64-token stages of all
+// (batch, head group) sequences in (batch, head group, token) order, NS
+// stages in all.  It is cut into R balanced ranges of consecutive stages, R a
+// multiple of the grid size P chosen so that no range is longer than
+// kRangeStages; CTA x takes ranges x, x + P, ...  A range may span several
+// sequences; its part in one sequence is a segment, and each segment leaves one
+// partial record (S, z and the gate's m, l over the segment).  Sequence q and
+// range r meet in at most one segment, stored as record q + r: for q < q' every
+// range meeting q comes no later than every range meeting q', so the index is
+// unique, and below R + Q (Q sequences).
+__host__ __device__ __forceinline__ long long num_ranges(long long NS, long long P) {
+  return NS <= 0 ? 0 : P * ((NS + kRangeStages * P - 1) / (kRangeStages * P));
+}
+__device__ __forceinline__ long long range_begin(long long NS, long long R, long long r) {
+  return NS * r / R;
+}
+// The range holding stage s, the largest r with range_begin(r) <= s, i.e.
+// floor(((s + 1) R - 1) / NS), without a 64-bit division: a double-precision
+// estimate corrected by exact integer products.
+__device__ __forceinline__ long long range_of(long long NS, long long R, long long s) {
+  const long long x = (s + 1) * R - 1;
+  long long r = (long long)((double)x / (double)NS);
+  while (r > 0 && r * NS > x) --r;
+  while ((r + 1) * NS <= x) ++r;
+  return r;
 }
 
-// Global inputs of one chunk for one converter thread, held in registers so
-// that all of them are in flight together: the k taps of its 4 channels, the
-// v taps of group channel tid (tid < 128), and the gate logits of tokens
-// tid + 512 i of the chunk as bf16 bits (-inf past the chunk or for a missing
-// head).  Nothing here uses a loaded value, so issuing them never waits.
-template <int G>
-struct ChunkIn {
-  float4 wk[4];  // [channel]: taps 0..3
-  float4 wv;
-  unsigned short a[kChunkMax / kSProd][G];
+// The sequence of stage s: batch b, head group hg, stage st of its nst stages
+// (L tokens); s0 is the sequence's first stage in the flattened list.
+struct StageRef {
+  int b, hg, st, nst, L;
+  long long s0;
 };
-__device__ __forceinline__ float bf16_bits_to_f32(unsigned short r) {
-  return __uint_as_float((uint32_t)r << 16);
-}
-template <int D, int G>
-__device__ __forceinline__ void load_chunk_inputs(const StateParams &p, const ChunkRef &c,
-                                                  int tid, int hh, int d0, ChunkIn<G> &in,
-                                                  uint32_t flags) {
-  const int H = p.H, h = c.hbase + hh;
-  const bool no_conv = flags & GBLA_FLAG_NO_CONV, no_gate = flags & GBLA_FLAG_NO_GATE;
-  const float4 ident = make_float4(0.f, 0.f, 0.f, 1.f);  // identity taps (ablation)
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    in.wk[i] = h >= H ? make_float4(0.f, 0.f, 0.f, 0.f) : ident;
-    if (h < H && !no_conv)
-      in.wk[i] = __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4));
+// Stage indices fit in 32 bits (at most 2^30 stages, checked on the host).
+__device__ __forceinline__ StageRef decode_stage(const StateParams &p, const int *pre,
+                                                 long long s64) {
+  StageRef r;
+  const int s = (int)s64;
+  if (p.seq_lens == nullptr) {  // every sequence has N tokens: arithmetic only
+    r.L = p.N;
+    r.nst = (p.N + kSTok - 1) / kSTok;
+    const int per_b = p.HG * r.nst;
+    r.b = s / per_b;
+    const int rem = s - r.b * per_b;
+    r.hg = rem / r.nst;
+    r.st = rem - r.hg * r.nst;
+  } else {
+    r.b = find_batch(pre, p.B, s);
+    r.L = clamp_len(p.seq_lens, r.b, p.N);
+    r.nst = (r.L + kSTok - 1) / kSTok;
+    const int rem = s - pre[r.b];
+    r.hg = rem / r.nst;
+    r.st = rem - r.hg * r.nst;
   }
-  in.wv = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (tid < kGroupCh) {
-    const int hz = c.hbase + tid / D, dz = tid % D;
-    if (hz < H) {
-      in.wv = ident;
-      if (!no_conv) in.wv = __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
-    }
-  }
-#pragma unroll
-  for (int i = 0; i < kChunkMax / kSProd; ++i) {
-    const int tt = tid + i * kSProd;
-    const unsigned short *gp =
-        (const unsigned short *)p.gate + ((size_t)c.b * p.N + c.t0 + tt) * H + c.hbase;
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const bool ok = tt < c.n && c.hbase + g < H;
-      in.a[i][g] = ok ? 0u : 0xff80u;  // bf16 -inf: no token
-      if (ok && !no_gate) in.a[i][g] = __ldg(gp + g);  // uniform gate: logits 0
-    }
-  }
-}
-
-// decode_chunk when every sequence has N tokens (the prefix is b * HG * nck).
-template <int G>
-__device__ __forceinline__ ChunkRef decode_chunk_uniform(const StateParams &p, int k) {
-  ChunkRef c;
-  const int nck = (p.N + p.S - 1) / p.S;
-  c.b = k / (p.HG * nck);
-  c.L = p.N;
-  const int r = k - c.b * p.HG * nck;
-  c.hbase = (r / nck) * G;
-  c.t0 = (r % nck) * p.S;
-  c.n = min(c.t0 + p.S, c.L) - c.t0;
-  c.nst = (c.n + kSTok - 1) / kSTok;
-  return c;
+  r.s0 = s64 - r.st;
+  return r;
 }
 
 // ABL: the ablation instantiation, which reads p.flags; the default one
@@ -444,21 +434,23 @@ __device__ __forceinline__ ChunkRef decode_chunk_uniform(const StateParams &p, i
 template <int D, bool ABL>
 __global__ void __launch_bounds__(kSThreads, 1)
     tc_state_kernel(const StateParams p, const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v,
-                    const __grid_constant__ CUtensorMap tm_rec) {
+                    const __grid_constant__ CUtensorMap tm_v) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  unsigned short *gw = (unsigned short *)(smem + kSOffGate);  // [G][kSGateStride]: logits
+  unsigned short *gw = (unsigned short *)(smem + kSOffGate);  // [2][kRangeTok]: logits
+  float *hmax = (float *)(smem + kSOffHmax);  // [2][64]: half-stage maxima of the range
+  float *segm = (float *)(smem + kSOffSegm);  // [2][32]: max over each stage's segment
   float *zred = (float *)(smem + kSOffZred);  // [16][128]
-  float4 *wv = (float4 *)(smem + kSOffWv);    // [128]: v taps of the group's channels
-  float *red = (float *)(smem + kSOffRed);    // [0,64) max, [64,128) sum, 128+ m, 132+ l
+  float *lred = (float *)(smem + kSOffLred);  // [16][2]
+  float4 *wvs = (float4 *)(smem + kSOffWv);   // [128]: v taps of the group's channels
   int *pre = (int *)(smem + kSOffPre);
   uint64_t *bars = (uint64_t *)(smem + kSOffBar);
-  uint64_t *raw_full = bars, *raw_empty = bars + kSRawStages;
-  uint64_t *a_full = bars + 2 * kSRawStages, *a_empty = a_full + kSAStages;
-  uint64_t *done = a_empty + kSAStages, *fin = done + 1;
+  uint64_t *k_full = bars, *k_empty = bars + kSKStages;
+  uint64_t *op_full = bars + 2 * kSKStages, *v_full = op_full + kSOpStages;
+  uint64_t *op_empty = v_full + kSOpStages;
+  uint64_t *done = op_empty + kSOpStages, *fin = done + 1, *logits_in = fin + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + kSOffMisc);
   const AbortFlag ab{smem_u32(smem + kSOffMisc + 4)};
 
@@ -466,155 +458,132 @@ __global__ void __launch_bounds__(kSThreads, 1)
   const int B = p.B, H = p.H;
   const uint32_t flags = ABL ? p.flags : 0u;
 
-  // Converter thread -> (group, channel quad q, token quad j): the groups take
-  // alternate stages; within a group the mapping makes both the raw-tile
-  // reads (16 lanes, 16 distinct quads of one 256-byte row) and the swizzled
-  // K^ writes (16 lanes, 16 distinct 8-byte slots of the 128-byte bank
-  // window) free of bank conflicts.
-  const int grp = warp / kSGroupWarps, gtid = tid % kSGroupThreads;
+  // Converter thread -> (group, channel quad q, token quad j): group grp takes
+  // token rows 32 grp .. 32 grp + 31 of every stage; within a group the mapping
+  // makes both the raw-tile reads (16 lanes, 16 distinct quads of one 256-byte
+  // row) and the swizzled K^ writes (16 lanes, 16 distinct 8-byte slots of the
+  // 128-byte bank window) free of bank conflicts.
+  const int grp = warp / kSGroupWarps;
   const int hw = 2 * (warp % kSGroupWarps) + (lane >> 4);              // half-warp 0..15
   const int q = (lane & 15) + 16 * (hw & 1);                           // channel quad 0..31
   const int j = (((lane >> 1) & 3) ^ (hw >> 2)) + 4 * ((hw >> 1) & 1);  // token quad 0..7
   const int c0ch = 4 * q;
   const int hh = c0ch / D, d0 = c0ch - D * hh;                         // head in group, channel
 
-  // With no seq_lens every sequence has N tokens, chunk k maps to (batch,
-  // head group, chunk) by arithmetic alone, and the first loads go out before
-  // the prefix over the batch is built.
-  const bool uniform = p.seq_lens == nullptr;
-  const int Ku = B * p.HG * ((p.N + p.S - 1) / p.S);
-  const long long c0u = (long long)Ku * blockIdx.x / gridDim.x;
-  const long long c1u = (long long)Ku * (blockIdx.x + 1) / gridDim.x;
-  const int early = uniform && c0u < c1u;  // first stages issued before the prefix
-  if (warp == kSTmaWarp && lane == 0) {
-    // the raw ring's barriers are first used by this thread
-    for (int i = 0; i < kSRawStages; ++i) {
-      mbar_init(&raw_full[i], kSTmaWarps);         // one box per TMA warp
-      mbar_init(&raw_empty[i], kSGroupWarps + 1);  // one converter group reads k, the MMAs v
-    }
-    fence_mbar_init();
-    tma_prefetch_desc(&tm_k);
-    tma_prefetch_desc(&tm_v);
-  }
   if (tid == 0) {
     *(volatile int *)(smem + kSOffMisc + 4) = 0;
-    for (int i = 0; i < kSAStages; ++i) {
-      mbar_init(&a_full[i], kSGroupWarps);
-      mbar_init(&a_empty[i], 1);
+    for (int i = 0; i < kSKStages; ++i) {
+      mbar_init(&k_full[i], 1);            // the k box (expect_tx)
+      mbar_init(&k_empty[i], kSCvtWarps);  // released by both converter groups
+    }
+    for (int i = 0; i < kSOpStages; ++i) {
+      mbar_init(&op_full[i], kSCvtWarps);  // K^ written (and v rows past the end zeroed)
+      mbar_init(&v_full[i], 1);            // the v boxes (expect_tx)
+      mbar_init(&op_empty[i], 1);          // the stage's MMAs completed
     }
     mbar_init(done, 1);
     mbar_init(fin, 1);
+    mbar_init(logits_in, kSCvtWarps);
     fence_mbar_init();
   }
-  // One box of a raw stage per TMA warp: 0 the k group rows, 1 + blk the v
-  // block blk (absent for a missing head: a plain arrival).
-  const int tbox = warp - kSTmaWarp;
-  auto issue_box = [&](const ChunkRef &c, int it, uint32_t s, uint64_t pol) {
-    uint8_t *dst = smem + kSOffRaw + s * kSRawStage;
-    const int tok = c.t0 + it * kSTok - kSHalo;
-    if (tbox == 0) {
-      mbar_arrive_expect_tx(&raw_full[s], kSRawKBytes);
-      tma_load_4d_hint(dst + kSRawK, &tm_k, &raw_full[s], 0, c.hbase, tok, c.b, pol);
-    } else {
-      const int blk = tbox - 1;
-      if (D == 64 && c.hbase + blk >= H) {
-        mbar_arrive(&raw_full[s]);
-      } else {
-        mbar_arrive_expect_tx(&raw_full[s], kSVBoxBytes);
-        tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &raw_full[s], (blk * 64) % D,
-                         c.hbase + (blk * 64) / D, tok, c.b, pol);
-      }
-    }
-  };
-  // The first chunk's global reads (gate logits, taps) go out before the bulk
-  // k/v loads, which would otherwise queue ahead of them: the gate pre-pass is
-  // on the critical path.  The TMA warps wait on barrier 3 until they are out.
-  ChunkIn<G> cin;
-  if (warp < kSCvtWarps) {
-    if (early) {
-      load_chunk_inputs<D, G>(p, decode_chunk_uniform<G>(p, (int)c0u), tid, hh, d0, cin, flags);
-      // the logits have arrived before the bulk loads go out: they would
-      // otherwise queue behind the whole start-up burst of every CTA
-      uint32_t sink = 0;
-#pragma unroll
-      for (int i = 0; i < kChunkMax / kSProd; ++i)
-#pragma unroll
-        for (int g = 0; g < G; ++g) sink += cin.a[i][g];
-      asm volatile("" ::"r"(sink));
-    }
-    named_barrier_arrive(3, kSProd + 32 * kSTmaWarps);
-  } else if (warp >= kSTmaWarp) {
-    named_barrier(3, kSProd + 32 * kSTmaWarps);
+  if (warp == kSKWarp && lane == 0) {
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
   }
-  if (warp >= kSTmaWarp && lane < kSTmaLanes && early) {
-    const uint64_t pol = l2_policy_evict_first();
-    const ChunkRef c = decode_chunk_uniform<G>(p, (int)c0u);
-    for (int it = lane; it < min(c.nst, kSEarlyStages); it += kSTmaLanes)
-      issue_box(c, it, (uint32_t)it, pol);
-  }
-  // Chunk prefix over the batch (converter threads), shared by all roles.  A
-  // TMA issuing thread can have about one copy in flight, so the early burst
-  // above takes a while: the converters hand the prefix to the TMA warps
-  // (barrier 4) and to the MMA warp (barrier 5) without waiting for them.
-  if (warp < kSCvtWarps) {
-    prefix_counts(pre, B, tid, kSProd, 1, (int *)red, [&](int b) {
-      const int L = clamp_len(p.seq_lens, b, p.N);
-      return p.HG * ((L + p.S - 1) / p.S);
-    });
-    if (blockIdx.x == 0)
-      for (int i = tid; i <= B; i += kSProd) p.chunk_pre[i] = pre[i];
-    named_barrier_arrive(4, kSProd + 32 * kSTmaWarps);
-    named_barrier_arrive(5, kSProd + 32);
-  } else if (warp == kSMmaWarp) {
-    named_barrier(5, kSProd + 32);
-  } else {
-    named_barrier(4, kSProd + 32 * kSTmaWarps);
-  }
-  const int K = pre[B];
-  const long long c0 = (long long)K * blockIdx.x / gridDim.x;
-  const long long c1 = (long long)K * (blockIdx.x + 1) / gridDim.x;
-  grid_dep_launch();
-  if (c0 >= c1) return;  // no chunks for this CTA
-  const ChunkRef cfirst = decode_chunk<G>(p, pre, (int)c0);
+  __syncthreads();
 
-  if (warp >= kSTmaWarp) {
+  // Stage prefix over the batch (ragged lengths only; uniform lengths decode
+  // by arithmetic, so the first loads go out at once).
+  long long NS;
+  if (p.seq_lens == nullptr) {
+    NS = (long long)B * p.HG * ((p.N + kSTok - 1) / kSTok);
+  } else {
+    if (warp < kSCvtWarps)
+      prefix_counts(pre, B, tid, kSProd, 1, (int *)(smem + kSOffRed), [&](int b) {
+        const int L = clamp_len(p.seq_lens, b, p.N);
+        return p.HG * ((L + kSTok - 1) / kSTok);
+      });
+    __syncthreads();
+    NS = pre[B];
+    if (blockIdx.x == 0)
+      for (int i = tid; i <= B; i += kSThreads) p.stage_pre[i] = pre[i];
+  }
+  const long long R = num_ranges(NS, gridDim.x);
+  grid_dep_launch();
+  if ((long long)blockIdx.x >= R) return;  // no work for this CTA
+
+  if (warp >= kSKWarp) {
     // ------------------------------------------------------------ TMA loads
-    // Per stage: v as two 64-channel blocks of 67 token rows (128B swizzle)
-    // and the k group rows (no swizzle); 3 rows of conv history in front,
-    // zero-filled before the sequence start.  These warps take no part in the
-    // TMEM hand-off, so their first loads go out at once.  Lane l issues the
-    // stages whose index in the CTA's sequence is l modulo kSTmaLanes.
-    if (lane < kSTmaLanes) {
-      // stages of the first chunk already issued before the prefix
-      const int it0 = early ? min(cfirst.nst, kSEarlyStages) : 0;
-      const uint64_t pol = l2_policy_evict_first();
-      uint32_t issued = (uint32_t)it0;
-      for (long long kk = c0; kk < c1 && !ab.raised(); ++kk) {
-        const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, (int)kk);
-        bool ok = true;
-        for (int it = kk == c0 ? it0 : 0; it < c.nst; ++it, ++issued) {
-          if (issued % kSTmaLanes != (uint32_t)lane) continue;
-          const uint32_t s = issued % kSRawStages, ph = (issued / kSRawStages) & 1;
-          if (!mbar_wait(&raw_empty[s], ph ^ 1, &ab)) {
-            if (!ab.raised()) report_error(2048, ab);
+    // Warp 17: the k tile of each stage (one head group x 67 token rows, no
+    // swizzle; lane l issues the stages whose index in the CTA's stage
+    // sequence is l mod 3, all into k slot l).  Warp 18: the v tile (two
+    // 64-channel blocks x 67 rows, 128B swizzle) into the stage's operand slot
+    // (lane l issues the stages with index l mod 2, operand slots l and l + 2).
+    // 3 rows of conv history in front, zero-filled before the sequence start.
+    // Only the CTA's first stage goes out before the converters' gate logits of
+    // its first range are in shared memory (mbarrier logits_in): the logits
+    // would otherwise queue behind the start-up burst of every CTA's copies.
+    const bool kw = warp == kSKWarp;
+    const int nl = kw ? kSKStages : kSVLanes;
+    const uint64_t pol = l2_policy_evict_first();
+    auto issue = [&](long long s, uint32_t gs) -> bool {
+      const StageRef st = decode_stage(p, pre, s);
+      const int tok = st.st * kSTok - kSHalo;
+      if (kw) {
+        const uint32_t ks = gs % kSKStages, ph = (gs / kSKStages) & 1;
+        if (!mbar_wait(&k_empty[ks], ph ^ 1, &ab)) return false;
+        mbar_arrive_expect_tx(&k_full[ks], kSKBox);
+        tma_load_4d_hint(smem + kSOffK + ks * kSKBox, &tm_k, &k_full[ks], 0, st.hg * G, tok, st.b,
+                         pol);
+      } else {
+        const uint32_t os = gs % kSOpStages, ph = (gs / kSOpStages) & 1;
+        if (!mbar_wait(&op_empty[os], ph ^ 1, &ab)) return false;
+        uint8_t *dst = smem + kSOffOp + os * kSOpStage + kSOpV;
+        // the second block is absent for a missing head (D = 64, odd H)
+        const bool two = !(D == 64 && st.hg * G + 1 >= H);
+        mbar_arrive_expect_tx(&v_full[os], (two ? 2 : 1) * kSVBoxBytes);
+        for (int blk = 0; blk < (two ? 2 : 1); ++blk)
+          tma_load_4d_hint(dst + blk * kSVBlock, &tm_v, &v_full[os], (blk * 64) % D,
+                           st.hg * G + (blk * 64) / D, tok, st.b, pol);
+      }
+      return true;
+    };
+    uint32_t last = 0xffffffffu;
+    bool ok = true;
+    const long long s_first = range_begin(NS, R, blockIdx.x);
+    if (lane == 0 && s_first < range_begin(NS, R, blockIdx.x + 1)) {  // a non-empty first range
+      ok = issue(s_first, 0);
+      if (ok) last = 0;
+    }
+    if (lane < nl) {
+      if (!mbar_wait(logits_in, 0, &ab)) ok = false;
+      uint32_t gs = 0;
+      for (long long r = blockIdx.x; r < R && ok; r += gridDim.x) {
+        const long long se = range_begin(NS, R, r + 1);
+        for (long long s = range_begin(NS, R, r); s < se; ++s, ++gs) {
+          if (gs == 0 || gs % nl != (uint32_t)lane) continue;  // stage 0 went out above
+          if (!issue(s, gs)) {
             ok = false;
             break;
           }
-          issue_box(c, it, s, pol);
+          last = gs;
         }
-        if (!ok) break;
       }
-      // every issued copy has landed before the CTA can exit
-      for (uint32_t g = issued > (uint32_t)kSRawStages ? issued - kSRawStages : 0; g < issued; ++g)
-        if (!mbar_wait(&raw_full[g % kSRawStages], (g / kSRawStages) & 1, nullptr))
-          report_error(4096, ab);
+      if (!ok && !ab.raised()) report_error(2048, ab);
+      // every copy this lane issued has landed before the CTA can exit (the
+      // phases of its slot complete in order: waiting for the last suffices)
+      if (last != 0xffffffffu) {
+        const bool okw = kw ? mbar_wait(&k_full[last % kSKStages], (last / kSKStages) & 1, nullptr)
+                            : mbar_wait(&v_full[last % kSOpStages], (last / kSOpStages) & 1, nullptr);
+        if (!okw) report_error(4096, ab);
+      }
     }
     __syncthreads();
     return;
   }
 
   // TMEM hand-off between the MMA warp and the converters (barrier 2); the
-  // converters join it after the first chunk's gate pre-pass.
+  // converters join it after the first range's gate pre-pass.
   uint32_t tmem = 0;
   auto tmem_handoff = [&]() {
     tc_fence_before();
@@ -627,163 +596,156 @@ __global__ void __launch_bounds__(kSThreads, 1)
     // ------------------------------------------------------------ converters
     // K^ rows: MN block q / 16, token row 4j + u, 16-byte chunk (q % 16) / 2
     // swizzled by the row, 8-byte half q & 1
-    const uint32_t arow0 = smem_u32(smem + kSOffA) + (uint32_t)((q >> 4) * kSABlock +
-                                                                4 * j * 128 + (q & 1) * 8);
+    const uint32_t arow0 = smem_u32(smem + kSOffOp) +
+                           (uint32_t)((q >> 4) * kSMnBlock + 4 * j * 128 + (q & 1) * 8);
     const uint32_t cs = (uint32_t)(((q & 15) >> 1) ^ (4 * (j & 1)));
-    const uint32_t raw0 = smem_u32(smem + kSOffRaw + kSRawK) + (uint32_t)(4 * j * kSRawRowK + q * 8);
-    const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kSGateStride + 4 * j) * 2;
-    uint32_t gs0 = 0;  // first stage of the chunk in the CTA's stage sequence
-    int nchunk = 0;
-    for (long long kk = c0; kk < c1; ++kk, ++nchunk) {
-      const int k = (int)kk;
-      const ChunkRef c = kk == c0 ? cfirst : decode_chunk<G>(p, pre, k);
-      if (!(kk == c0 && early)) load_chunk_inputs<D, G>(p, c, tid, hh, d0, cin, flags);
-
-      // k taps of this thread's 4 channels, pre-scaled by log2(e); v taps of
-      // the group's channels for the drain
-      float w[4][4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        w[0][i] = cin.wk[i].x * kLog2e;
-        w[1][i] = cin.wk[i].y * kLog2e;
-        w[2][i] = cin.wk[i].z * kLog2e;
-        w[3][i] = cin.wk[i].w * kLog2e;
-      }
-      if (tid < kGroupCh) wv[tid] = cin.wv;
-
-      // Gate pre-pass: per-head chunk maximum m and l = sum 2^a' with
-      // a' = (a - m) log2(e); the logits go to shared memory for the stages,
-      // which form a' and 2^a' per token themselves.  Entries past the chunk
-      // are -inf.
-      float mlog = 0.f;  // m log2(e) of this thread's head
+    const uint32_t raw0 = smem_u32(smem + kSOffK) + (uint32_t)(4 * j * kSRawRowB + q * 8);
+    const uint32_t gws = smem_u32(gw) + (uint32_t)(hh * kRangeTok + 4 * j) * 2;
+    const bool no_conv = flags & GBLA_FLAG_NO_CONV, no_gate = flags & GBLA_FLAG_NO_GATE;
+    uint32_t gs0 = 0;  // first stage of the segment in the CTA's stage sequence
+    int nseg = 0, cur_hg = -1;
+    float wk[4][4];    // k taps of this thread's channels, times log2 e
+    bool first = true;
+    for (long long r = blockIdx.x; r < R; r += gridDim.x) {
+      const long long sb = range_begin(NS, R, r), se = range_begin(NS, R, r + 1);
+      const int nsr = (int)(se - sb);
+      // ---- range pre-pass: the range's gate logits into shared memory (-inf
+      // past a sequence end or for a missing head), half-stage maxima, then
+      // for every stage the maximum over its segment.
       {
-        constexpr int kPer = kChunkMax / kSProd;
-        float m[G];
+        unsigned short a[kRangeTok / kSProd][G];
 #pragma unroll
-        for (int g = 0; g < G; ++g) {
-          m[g] = -INFINITY;
+        for (int i = 0; i < kRangeTok / kSProd; ++i) {
+          const int slot = tid + i * kSProd;
 #pragma unroll
-          for (int i = 0; i < kPer; ++i) m[g] = fmaxf(m[g], bf16_bits_to_f32(cin.a[i][g]));
+          for (int g = 0; g < G; ++g) a[i][g] = 0xff80u;  // bf16 -inf
+          if (slot < nsr * kSTok) {
+            const StageRef st = decode_stage(p, pre, sb + slot / kSTok);
+            const int t = st.st * kSTok + slot % kSTok;
+            if (t < st.L) {
+              const unsigned short *gp = (const unsigned short *)p.gate +
+                                         ((size_t)st.b * p.N + t) * H + st.hg * G;
 #pragma unroll
-          for (int o = 16; o >= 1; o >>= 1) m[g] = fmaxf(m[g], __shfl_xor_sync(0xffffffffu, m[g], o));
-          if (lane == 0) red[warp * 4 + g] = m[g];
-        }
-        named_barrier(1, kSProd);
-        const int npad = c.nst * kSTok;
-#pragma unroll
-        for (int g = 0; g < G; ++g) {
-          float M = red[g];
-          for (int w2 = 1; w2 < kSCvtWarps; ++w2) M = fmaxf(M, red[w2 * 4 + g]);
-          // a missing head has only -inf logits: M = -inf, and a' = -inf with mlog 0
-          const float ml = M == -INFINITY ? 0.f : M * kLog2e;
-          if (g == hh) mlog = ml;
-          float l = 0.f;
-#pragma unroll
-          for (int i = 0; i < kPer; ++i) {
-            const int tt = tid + i * kSProd;
-            const float ex = ex2_approx(gate_log2(cin.a[i][g], ml));
-            if (tt < npad) gw[g * kSGateStride + tt] = cin.a[i][g];
-            l += ex;
-          }
-#pragma unroll
-          for (int o = 16; o >= 1; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
-          if (lane == 0) red[64 + warp * 4 + g] = l;
-          if (tid == 0) red[128 + g] = M;
-        }
-        named_barrier(1, kSProd);
-        if (tid < G) {  // l of this chunk, per head, for the records
-          float lt = 0.f;
-          for (int w2 = 0; w2 < kSCvtWarps; ++w2) lt += red[64 + w2 * 4 + tid];
-          red[132 + tid] = lt;
-        }
-      }
-
-      if (kk == c0) tmem_handoff();
-      float2 z[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      for (int it = (int)((gs0 ^ grp) & 1); it < c.nst; it += 2) {  // this group's stages
-        const uint32_t gs = gs0 + it;
-        const uint32_t rs = gs % kSRawStages, rph = (gs / kSRawStages) & 1;
-        const uint32_t as = gs % kSAStages, aph = (gs / kSAStages) & 1;
-        if (!mbar_wait(&raw_full[rs], rph, &ab) && !ab.raised()) report_error(1, ab);
-        if (!mbar_wait(&a_empty[as], aph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
-        const int T = c.t0 + it * kSTok;
-#pragma unroll
-        for (int hq = 0; hq < kSTok / 32; ++hq) {  // token quads j + 8 hq (rows 32 hq on)
-          const int nvalid = min(max(c.L - (T + 32 * hq + 4 * j), 0), 4);
-          state_convert(raw0 + rs * kSRawStage + hq * 32 * kSRawRowK,
-                        arow0 + as * kSAStage + hq * 32 * 128, cs,
-                        gws + (uint32_t)(it * kSTok + 32 * hq) * 2, mlog, w, z, nvalid);
-        }
-        if (T + kSTok > c.L) {
-          // v rows past the sequence end meet K^ = 0 in the MMA, but may hold
-          // NaN or inf: zero them (both 64-channel blocks)
-          const int r0 = max(c.L - (T - kSHalo), 0);
-          const uint32_t vb = smem_u32(smem + kSOffRaw) + rs * kSRawStage;
-          for (int e = gtid; e < (kSRawRows - r0) * 16; e += kSGroupThreads) {
-            const int r = r0 + e / 16, blk = (e / 8) & 1, ck = e & 7;
-            sts_v4(vb + blk * kSVBlock + r * 128 + ck * 16, make_uint4(0, 0, 0, 0));
-          }
-        }
-        fence_proxy_async_smem();  // K^ (and zeroed v rows) visible to the tensor cores
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&a_full[as]);
-          mbar_arrive(&raw_empty[rs]);
-        }
-      }
-      gs0 += c.nst;
-
-      // z of this chunk: the token quads of both groups summed in a fixed order.
-      *(float4 *)&zred[(grp * 8 + j) * kGroupCh + c0ch] = make_float4(z[0].x, z[0].y, z[1].x, z[1].y);
-      named_barrier(1, kSProd);
-      float zsum = 0.f;
-      if (tid < kGroupCh)
-        for (int jj = 0; jj < 16; ++jj) zsum += zred[jj * kGroupCh + tid];
-
-      // Wait for this chunk's accumulators, then write the partial records:
-      // S[a][c] = sum_tau w_tau[c] P_tau[a][c] on the diagonal D x D blocks.
-      // P_tau of v channel c = 64 blk + c' sits in TMEM column 256 blk + 64 tau + c'.
-      if (!mbar_wait(done, nchunk & 1, &ab) && !ab.raised()) report_error(2, ab);
-      tc_fence_after();
-      {
-        constexpr int CPW = D / 4;                    // columns per warp
-        const int q4 = warp & 3, part = warp >> 2;    // lane quarter, column quarter
-        const int ch = 32 * q4 + lane;                // TMEM lane = group channel (row of S)
-        const int hh2 = ch / D, d = ch - D * hh2;
-        const int cv0 = D * hh2 + part * CPW;         // first v channel (of the group) of this warp
-        const bool ok2 = c.hbase + hh2 < H;
-        float *srow = p.records + ((size_t)k * G + hh2) * REC + (size_t)d * D + part * CPW;
-        const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16) +
-                            (uint32_t)(256 * (cv0 / 64) + cv0 % 64);
-        if constexpr (D == 64) {
-          // staged in the idle A ring as 32-column, 128B-swizzled tiles for
-          // one TMA store per tile: row d, 16-byte chunk (col % 32) / 4 ^ (d & 7);
-          // 4 columns (one chunk) per step
-          const uint32_t stg = smem_u32(smem + kSOffA) + (uint32_t)(hh2 * 2 * (64 * 128) + d * 128);
-#pragma unroll 1
-          for (int cb = 0; cb < CPW; cb += 4) {
-            float v0[4], v1[4], v2[4], v3[4];
-            tmem_ld4(tl + cb, v0);
-            tmem_ld4(tl + 64 + cb, v1);
-            tmem_ld4(tl + 128 + cb, v2);
-            tmem_ld4(tl + 192 + cb, v3);
-            tmem_ld_wait_regs(v0);
-            tmem_pin(v1);
-            tmem_pin(v2);
-            tmem_pin(v3);
-            uint32_t o[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float4 wt = wv[cv0 + cb + i];
-              o[i] = __float_as_uint(
-                  fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i]))));
+              for (int g = 0; g < G; ++g)
+                if (st.hg * G + g < H) a[i][g] = no_gate ? (unsigned short)0 : __ldg(gp + g);
             }
-            const int col = part * CPW + cb, cbk = col >> 5, c4 = (col & 31) >> 2;
-            sts_v4(stg + cbk * (64 * 128) + ((c4 ^ (d & 7)) << 4),
-                   make_uint4(o[0], o[1], o[2], o[3]));
           }
-        } else {
-#pragma unroll 1
+        }
+#pragma unroll
+        for (int i = 0; i < kRangeTok / kSProd; ++i) {
+          const int slot = tid + i * kSProd;
+#pragma unroll
+          for (int g = 0; g < G; ++g) {
+            gw[g * kRangeTok + slot] = a[i][g];
+            float m = bf16_bits_to_f32(a[i][g]);
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+            if (lane == 0) hmax[g * 64 + slot / 32] = m;
+          }
+        }
+        if (first) {  // logits in: the TMA warps go on
+          __syncwarp();
+          if (lane == 0) mbar_arrive(logits_in);
+        }
+        named_barrier(1, kSProd);
+        if (tid < G * 32) {
+          const int g = tid / 32, k = tid % 32;
+          if (k < nsr) {
+            const StageRef st = decode_stage(p, pre, sb + k);
+            const int k0 = (int)(max(sb, st.s0) - sb), k1 = (int)(min(se, st.s0 + st.nst) - sb);
+            float m = -INFINITY;
+            for (int i = k0; i < k1; ++i)
+              m = fmaxf(m, fmaxf(hmax[g * 64 + 2 * i], hmax[g * 64 + 2 * i + 1]));
+            segm[g * kRangeStages + k] = m;
+          }
+        }
+        named_barrier(1, kSProd);
+      }
+      if (first) tmem_handoff();
+      first = false;
+
+      for (long long s = sb; s < se;) {
+        const StageRef st = decode_stage(p, pre, s);
+        const long long seg_end = min(se, st.s0 + st.nst);
+        const int nst = (int)(seg_end - s), lst0 = (int)(s - sb);
+        if (st.hg != cur_hg) {  // taps of this thread's 4 channels (identity: ablation)
+          const int h = st.hg * G + hh;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            float4 tk = make_float4(0.f, 0.f, 0.f, h < H ? 1.f : 0.f);
+            if (h < H && !no_conv)
+              tk = __ldg((const float4 *)(p.conv_w + ((size_t)(H + h) * D + d0 + i) * 4));
+            wk[0][i] = tk.x * kLog2e;
+            wk[1][i] = tk.y * kLog2e;
+            wk[2][i] = tk.z * kLog2e;
+            wk[3][i] = tk.w * kLog2e;
+          }
+          if (tid < kGroupCh) {  // v taps of group channel tid, applied at the drain
+            const int hz = st.hg * G + tid / D, dz = tid % D;
+            float4 tv = make_float4(0.f, 0.f, 0.f, hz < H ? 1.f : 0.f);
+            if (hz < H && !no_conv)
+              tv = __ldg((const float4 *)(p.conv_w + ((size_t)(2 * H + hz) * D + dz) * 4));
+            wvs[tid] = tv;
+          }
+          cur_hg = st.hg;
+        }
+        // a missing head has only -inf logits: M = -inf, and a' = -inf with mlog 0
+        const float M = segm[hh * kRangeStages + lst0];
+        const float mlog = M == -INFINITY ? 0.f : M * kLog2e;
+        float2 z[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        float lacc = 0.f;
+        for (int it = 0; it < nst; ++it) {  // this group converts token rows 32 grp .. 32 grp + 31
+          const uint32_t gs = gs0 + it;
+          const uint32_t ks = gs % kSKStages, kph = (gs / kSKStages) & 1;
+          const uint32_t os = gs % kSOpStages, oph = (gs / kSOpStages) & 1;
+          if (!mbar_wait(&k_full[ks], kph, &ab) && !ab.raised()) report_error(1, ab);
+          if (!mbar_wait(&op_empty[os], oph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
+          const int T = (st.st + it) * kSTok;
+          const int nvalid = min(max(st.L - (T + 32 * grp + 4 * j), 0), 4);
+          const float ls = state_convert_k(
+              raw0 + ks * kSKBox + grp * 32 * kSRawRowB, arow0 + os * kSOpStage + grp * 32 * 128, cs,
+              gws + (uint32_t)((lst0 + it) * kSTok + 32 * grp) * 2, mlog, wk, z, nvalid);
+          if (d0 == 0) lacc += ls;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&k_empty[ks]);  // the k tile is consumed
+          if (T + kSTok > st.L) {
+            // v rows past the sequence end meet K^ = 0 in the MMA, but may hold
+            // NaN or inf: zero them (both 64-channel blocks) once they have landed
+            if (!mbar_wait(&v_full[os], oph, &ab) && !ab.raised()) report_error(1, ab);
+            const int r0 = max(st.L - (T - kSHalo), 0);
+            const uint32_t vb = smem_u32(smem + kSOffOp) + os * kSOpStage + kSOpV;
+            for (int e = tid; e < (kSRawRows - r0) * 16; e += kSProd) {
+              const int rr = r0 + e / 16, blk = (e / 8) & 1, ck = e & 7;
+              sts_v4(vb + blk * kSVBlock + rr * 128 + ck * 16, make_uint4(0, 0, 0, 0));
+            }
+          }
+          fence_proxy_async_smem();  // K^ (and zeroed v rows) visible to the tensor cores
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&op_full[os]);
+        }
+        gs0 += nst;
+
+        // ---- segment end: z and l (token quads of both groups summed in a
+        // fixed order); S[a][c] = sum_tau w_tau[c] P_tau[a][c] on the diagonal
+        // D x D blocks, P_tau of v channel c = 64 blk + c' in TMEM column
+        // 256 blk + 64 tau + c'.
+        *(float4 *)&zred[(grp * 8 + j) * kGroupCh + c0ch] = make_float4(z[0].x, z[0].y, z[1].x, z[1].y);
+        if (d0 == 0) lred[(grp * 8 + j) * 2 + hh] = lacc;
+        named_barrier(1, kSProd);
+        if (!mbar_wait(done, nseg & 1, &ab) && !ab.raised()) report_error(2, ab);
+        tc_fence_after();
+        const long long rec = (long long)(st.b * p.HG + st.hg) + r;
+        {
+          constexpr int CPW = D / 4;                    // columns per warp
+          const int q4 = warp & 3, part = warp >> 2;    // lane quarter, column quarter
+          const int ch = 32 * q4 + lane;                // TMEM lane = group channel (row of S)
+          const int ha = ch / D, d = ch - D * ha;
+          const bool ok2 = st.hg * G + ha < H;
+          const int cv0 = D * ha + part * CPW;          // first v channel (of the group)
+          const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16) +
+                              (uint32_t)(256 * (cv0 / 64) + cv0 % 64);
+          float *dst = p.records + ((size_t)rec * G + ha) * REC + (size_t)d * D + part * CPW;
+#pragma unroll
           for (int cb = 0; cb < CPW; cb += 8) {
             float v0[8], v1[8], v2[8], v3[8];
             tmem_ld8(tl + cb, v0);
@@ -797,43 +759,36 @@ __global__ void __launch_bounds__(kSThreads, 1)
             float o[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-              const float4 wt = wv[cv0 + cb + i];
+              const float4 wt = wvs[cv0 + cb + i];
               o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
             }
             if (ok2) {
-              float4 *dst = (float4 *)(srow + cb);
-              dst[0] = make_float4(o[0], o[1], o[2], o[3]);
-              dst[1] = make_float4(o[4], o[5], o[6], o[7]);
+              float4 *dq = (float4 *)(dst + cb);
+              dq[0] = make_float4(o[0], o[1], o[2], o[3]);
+              dq[1] = make_float4(o[4], o[5], o[6], o[7]);
             }
-          }
-        }
-        if constexpr (D == 64) {
-          fence_proxy_async_smem();
-          named_barrier(1, kSProd);
-          if (tid == 0) {
-            const uint64_t pol = l2_policy_evict_last();  // read back by the reduction
-            for (int hz = 0; hz < G && c.hbase + hz < H; ++hz)
-              for (int cbk = 0; cbk < 2; ++cbk)
-                tma_store_4d_hint(&tm_rec, smem + kSOffA + (hz * 2 + cbk) * (64 * 128), cbk * 32,
-                                  0, hz, k, pol);
-            tma_store_commit();
-            tma_store_wait_read<0>();  // the A ring is written again by the next chunk
           }
         }
         if (tid < kGroupCh) {
           const int hz = tid / D, dz = tid - D * hz;
-          if (c.hbase + hz < H) {
-            float *rz = p.records + ((size_t)k * G + hz) * REC;
+          if (st.hg * G + hz < H) {
+            float zsum = 0.f;
+            for (int jj = 0; jj < 16; ++jj) zsum += zred[jj * kGroupCh + tid];
+            float *rz = p.records + ((size_t)rec * G + hz) * REC;
             rz[D * D + dz] = zsum;
             if (dz == 0) {
-              rz[D * D + D] = red[128 + hz];
-              rz[D * D + D + 1] = red[132 + hz];
+              float lt = 0.f;
+              for (int jj = 0; jj < 16; ++jj) lt += lred[jj * 2 + hz];
+              rz[D * D + D] = segm[hz * kRangeStages + lst0];
+              rz[D * D + D + 1] = lt * (1.f / kLn2);
             }
           }
         }
+        tc_fence_before();
+        named_barrier(1, kSProd);  // drained before the next segment's MMAs, taps and z/l sums
+        ++nseg;
+        s = seg_end;
       }
-      tc_fence_before();
-      named_barrier(1, kSProd);  // accumulators drained before the next chunk's MMAs
     }
   } else if (warp == kSMmaWarp) {
     tmem_alloc(tmem_slot, kSTmemCols);
@@ -841,42 +796,44 @@ __global__ void __launch_bounds__(kSThreads, 1)
     if (lane == 0) {
       // ---------------------------------------------------------- MMA issuer
       // P_tau += K^T v[t - 3 + tau] for tau = 0..3 in one N = 256 MMA per
-      // 64-channel v block: its four 64-column B blocks are the same raw tile
+      // 64-channel v block: its four 64-column B blocks are the same v tile
       // with the start moved down 0..3 rows (LBO = one 128-byte row).  The
       // 128-byte swizzle follows the absolute shared address, so the shifted
-      // views read the rows TMA wrote.
-      // This warp shares its SM sub-partition with busy converter warps, so
-      // the loop is kept short: descriptors of slot 0 advanced by the slot
-      // offsets (a descriptor's address field is the byte address >> 4, and
-      // shared addresses stay below 256 KB, so adding to it never carries),
-      // and ring positions stepped rather than divided.
+      // views read the rows TMA wrote.  Descriptors of slot 0 are advanced by
+      // the slot offsets (a descriptor's address field is the byte address
+      // >> 4, and shared addresses stay below 256 KB, so adding never carries).
       constexpr uint32_t idesc = idesc_bf16_f32(128, 256, 1, 1);
-      const uint64_t ad0 = sw128_desc(smem_u32(smem + kSOffA), kSABlock, 1024);
-      const uint64_t bd0 = sw128_desc(smem_u32(smem + kSOffRaw), 128, 1024);
-      uint32_t rs = 0, rph = 0, as = 0, aph = 0;
+      const uint64_t ad0 = sw128_desc(smem_u32(smem + kSOffOp), kSMnBlock, 1024);
+      const uint64_t bd0 = sw128_desc(smem_u32(smem + kSOffOp + kSOpV), 128, 1024);
+      uint32_t os = 0, oph = 0;
       bool ok = true;
-      for (long long kk = c0; kk < c1 && ok; ++kk) {
-        const ChunkRef c = decode_chunk<G>(p, pre, (int)kk);
-        for (int it = 0; it < c.nst; ++it) {
-          if (!mbar_wait(&a_full[as], aph, &ab) || !mbar_wait(&raw_full[rs], rph, &ab)) {
-            if (!ab.raised()) report_error(4, ab);
-            ok = false;
-            break;
+      for (long long r = blockIdx.x; r < R && ok; r += gridDim.x) {
+        const long long se = range_begin(NS, R, r + 1);
+        for (long long s = range_begin(NS, R, r); s < se && ok;) {
+          const StageRef st = decode_stage(p, pre, s);
+          const long long seg_end = min(se, st.s0 + st.nst);
+          const int nst = (int)(seg_end - s);
+          for (int it = 0; it < nst; ++it) {
+            if (!mbar_wait(&op_full[os], oph, &ab) || !mbar_wait(&v_full[os], oph, &ab)) {
+              if (!ab.raised()) report_error(4, ab);
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint64_t off = (uint64_t)(os * kSOpStage) >> 4;
+#pragma unroll
+            for (int blk = 0; blk < 2; ++blk)
+#pragma unroll
+              for (int k16 = 0; k16 < kSTok / 16; ++k16)
+                mma_bf16(tmem + 256 * blk, ad0 + off + (k16 * 2048 >> 4),
+                         bd0 + off + ((blk * kSVBlock + 16 * k16 * 128) >> 4), idesc,
+                         (it | k16) != 0);
+            mma_commit(&op_empty[os]);
+            if (++os == kSOpStages) { os = 0; oph ^= 1; }
           }
-          tc_fence_after();
-          const uint64_t ad = ad0 + (as * kSAStage >> 4), bd = bd0 + (rs * kSRawStage >> 4);
-#pragma unroll
-          for (int blk = 0; blk < 2; ++blk)
-#pragma unroll
-            for (int k16 = 0; k16 < kSTok / 16; ++k16)
-              mma_bf16(tmem + 256 * blk, ad + (k16 * 2048 >> 4),
-                       bd + ((blk * kSVBlock + 16 * k16 * 128) >> 4), idesc, (it | k16) != 0);
-          mma_commit(&a_empty[as]);
-          mma_commit(&raw_empty[rs]);
-          if (++as == kSAStages) { as = 0; aph ^= 1; }
-          if (++rs == kSRawStages) { rs = 0; rph ^= 1; }
+          if (ok) mma_commit(done);
+          s = seg_end;
         }
-        if (ok) mma_commit(done);
       }
       mma_commit(fin);  // every MMA issued above has completed once this arrives
       if (!mbar_wait(fin, 0, nullptr)) report_error(8, ab);
@@ -889,78 +846,108 @@ __global__ void __launch_bounds__(kSThreads, 1)
   }
 }
 
-// Fixed-order combination of the chunk records of one (b, h):
+// Fixed-order combination of the partial records of one (b, h): the records
+// q + r of the ranges r0..r1 meeting its sequence q, in range order,
 //   M = max_j m_j,  S = sum_j e^{m_j - M} S_j / sum_j e^{m_j - M} l_j  (z likewise).
-// Each thread owns 4 consecutive state elements and walks the chunks in index
-// order, 24 at a time with every load of a batch in flight together; a batch
-// whose maximum exceeds the running one rescales what was summed so far.
+// Records go 32 at a time: lane j of every warp fetches record j's (m, l),
+// the warp forms the batch maximum and the sum of l with shuffles (a fixed
+// butterfly order), and each thread then accumulates its 4 state elements
+// over the batch in record order, 16 loads in flight at a time, with the
+// scale factors broadcast from the lanes that computed them.
 constexpr int kReduceThreads = 128;
 template <int D>
-__global__ void __launch_bounds__(kReduceThreads) tc_reduce_kernel(const float *__restrict__ records,
-                                                         const int32_t *__restrict__ chunk_pre,
+__global__ void __launch_bounds__(kReduceThreads, 1) tc_reduce_kernel(const float *__restrict__ records,
+                                                         const int32_t *__restrict__ stage_pre,
                                                          const int32_t *__restrict__ seq_lens,
                                                          float *__restrict__ state,
                                                          float2 *__restrict__ gate_stats, int B,
-                                                         int H, int N, int S) {
+                                                         int H, int N, int P) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
-  constexpr int EPT = 4;   // elements per thread
-  constexpr int BATCH = 24;
+  constexpr int CH = 16;   // record loads in flight per thread
   grid_dep_wait();
   grid_dep_launch();
+  const int lane = threadIdx.x & 31;
   const int bh = blockIdx.x;
   const int b = bh / H, h = bh % H;
-  const int hg = h / G, hh = h % G;
-  const int e0 = (blockIdx.y * kReduceThreads + threadIdx.x) * EPT;
-  if (e0 >= F) return;
+  const int hg = h / G, hh = h % G, HG = (H + G - 1) / G;
+  const int e0 = (blockIdx.y * kReduceThreads + threadIdx.x) * 4;
+  const bool act = e0 < F;  // every thread takes part in the shuffles
   const int L = clamp_len(seq_lens, b, N);
-  const int nck = (L + S - 1) / S;
-  // with every sequence N tokens long the prefix is b HG nck: no dependent load
-  const int k0 = (seq_lens == nullptr ? b * ((H + G - 1) / G) * nck : chunk_pre[b]) + hg * nck;
-  const float *rec0 = records + ((size_t)k0 * G + hh) * REC;
-  const size_t rstride = (size_t)G * REC;
+  const int nst = (L + kSTok - 1) / kSTok;
   float M = -INFINITY, l = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int j0 = 0; j0 < nck; j0 += BATCH) {
-    float4 v[BATCH];
-    float m[BATCH], lj[BATCH];
+  if (nst > 0) {
+    // with every sequence N tokens long the prefix is b HG nst: no dependent load
+    int NS, pre_b;
+    if (seq_lens == nullptr) {
+      NS = B * HG * nst;
+      pre_b = b * HG * nst;
+    } else {
+      NS = stage_pre[B];
+      pre_b = stage_pre[b];
+    }
+    const int R = (NS + kRangeStages * P - 1) / (kRangeStages * P) * P;  // num_ranges
+    const int s0 = pre_b + hg * nst;
+    const long long r0 = range_of(NS, R, s0), r1 = range_of(NS, R, s0 + nst - 1);
+    const int nrec = (int)(r1 - r0 + 1);
+    const bool may_be_empty = NS < R;  // otherwise every range holds a stage
+    const float *rec0 = records + ((size_t)((long long)b * HG + hg + r0) * G + hh) * REC;
+    const size_t rstride = (size_t)G * REC;
+    for (int j0 = 0; j0 < nrec; j0 += 32) {
+      const int j = j0 + lane;
+      bool has = j < nrec;
+      if (has && may_be_empty)  // with fewer stages than ranges some left no record
+        has = range_begin(NS, R, r0 + j) < range_begin(NS, R, r0 + j + 1);
+      const float *rj = rec0 + (size_t)j * rstride;
+      const float mj = has ? __ldg(rj + F) : -INFINITY;
+      const float lj = has ? __ldg(rj + F + 1) : 0.f;
+      float Mb = mj;
 #pragma unroll
-    for (int j = 0; j < BATCH; ++j) {
-      if (j0 + j < nck) {
-        const float *r = rec0 + (size_t)(j0 + j) * rstride;
-        v[j] = __ldg((const float4 *)(r + e0));
-        m[j] = __ldg(r + F);
-        lj[j] = __ldg(r + F + 1);
-      } else {
-        v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-        m[j] = -INFINITY;
-        lj[j] = 0.f;
+      for (int o = 16; o >= 1; o >>= 1) Mb = fmaxf(Mb, __shfl_xor_sync(0xffffffffu, Mb, o));
+      if (Mb > M) {  // rescale the running sums to the new maximum
+        const float rsc = (M == -INFINITY) ? 0.f : __expf(M - Mb);
+        acc.x *= rsc; acc.y *= rsc; acc.z *= rsc; acc.w *= rsc;
+        l *= rsc;
+        M = Mb;
       }
-    }
-    float Mb = M;
+      const float sc = has ? __expf(mj - M) : 0.f;
+      float ls = sc * lj;
 #pragma unroll
-    for (int j = 0; j < BATCH; ++j) Mb = fmaxf(Mb, m[j]);
-    if (Mb > M) {  // rescale the running sums to the new maximum
-      const float r = (M == -INFINITY) ? 0.f : __expf(M - Mb);
-      acc.x *= r; acc.y *= r; acc.z *= r; acc.w *= r;
-      l *= r;
-      M = Mb;
-    }
+      for (int o = 16; o >= 1; o >>= 1) ls += __shfl_xor_sync(0xffffffffu, ls, o);
+      l += ls;
+      const int nb = min(32, nrec - j0);
+      for (int k0 = 0; k0 < nb; k0 += CH) {
+        float skk[CH];  // the chunk's scale factors, from the lanes that hold them
 #pragma unroll
-    for (int j = 0; j < BATCH; ++j) {
-      if (j0 + j < nck) {
-        const float sc = __expf(m[j] - M);
-        acc.x = fmaf(sc, v[j].x, acc.x);
-        acc.y = fmaf(sc, v[j].y, acc.y);
-        acc.z = fmaf(sc, v[j].z, acc.z);
-        acc.w = fmaf(sc, v[j].w, acc.w);
-        l = fmaf(sc, lj[j], l);
+        for (int k = 0; k < CH; ++k) skk[k] = __shfl_sync(0xffffffffu, sc, (k0 + k) & 31);
+        // every load of the chunk in flight together: past the batch (or the
+        // state) the index is clamped to a record and element that exist
+        float4 v[CH];
+        const int ec = act ? e0 : 0;
+#pragma unroll
+        for (int k = 0; k < CH; ++k) {
+          const int kk = k0 + k < nb ? j0 + k0 + k : j0;
+          v[k] = __ldg((const float4 *)(rec0 + (size_t)kk * rstride + ec));
+        }
+#pragma unroll
+        for (int k = 0; k < CH; ++k) {
+          // a zero factor marks a record that does not exist (an empty range,
+          // whose slot holds whatever was there) or that underflowed: skip it
+          if (k0 + k < nb && skk[k] != 0.f) {
+            acc.x = fmaf(skk[k], v[k].x, acc.x);
+            acc.y = fmaf(skk[k], v[k].y, acc.y);
+            acc.z = fmaf(skk[k], v[k].z, acc.z);
+            acc.w = fmaf(skk[k], v[k].w, acc.w);
+          }
+        }
       }
     }
   }
   if (gate_stats != nullptr && blockIdx.y == 0 && threadIdx.x == 0)
     gate_stats[bh] = make_float2(M, l);  // every thread of bh holds the same pair
+  if (!act) return;
   const float inv = l > 0.f ? 1.f / l : 0.f;
   *(float4 *)(state + (size_t)bh * F + e0) =
       make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
@@ -1610,25 +1597,6 @@ cudaError_t make_group_map(CUtensorMap *m, const void *base, int B, int N, int H
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-// 4-D map over the partial-state records [chunks][G][D*D + D + 4] fp32, viewed
-// as S blocks {D columns, D rows, G heads, chunks}; box = 32 columns x D rows,
-// 128-byte swizzle (the state kernel stages S that way before storing it).
-cudaError_t make_records_map(CUtensorMap *m, void *records, const Problem &p, int D, int S) {
-  EncodeTiledFn fn = encode_fn();
-  if (!fn) return cudaErrorNotSupported;
-  const int G = kGroupCh / D;
-  const size_t chunks = (size_t)p.B * ((p.H + G - 1) / G) * ((p.N + S - 1) / S);
-  const size_t rec = (size_t)D * D + D + 4;
-  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)D, (cuuint64_t)G, (cuuint64_t)chunks};
-  const cuuint64_t strides[3] = {(cuuint64_t)D * 4, (cuuint64_t)rec * 4, (cuuint64_t)G * rec * 4};
-  const cuuint32_t box[4] = {32, (cuuint32_t)D, 1, 1};
-  const cuuint32_t estr[4] = {1, 1, 1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, records, dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
-}
-
 struct DeviceInfo {
   int sms = 0;
   bool sm103 = false;
@@ -1653,26 +1621,17 @@ const DeviceInfo &device_info() {
 
 int num_sms() { return device_info().sms; }
 
-// Chunk length: about one chunk per SM over the padded problem, 32-aligned,
-// within [256, kChunkMax], and at most kMaxChunksPerSeq chunks per sequence.
-int chunk_len(const Problem &p) {
+// Partial records the state step may write: one per (sequence, range) meeting,
+// at most R + Q - 1 with R bounded by the stage count of full-length sequences.
+size_t record_slots(const Problem &p) {
   const int G = kGroupCh / p.D;
-  const int HG = (p.H + G - 1) / G;
-  const long long work = (long long)p.B * HG * p.N;
-  const int sms = num_sms();
-  long long S = (work + sms - 1) / sms;
-  S = (S + 31) / 32 * 32;
-  S = S < 256 ? 256 : (S > kChunkMax ? kChunkMax : S);
-  const long long Smin = ((long long)p.N + kMaxChunksPerSeq - 1) / kMaxChunksPerSeq;
-  if (S < Smin) S = (Smin + 31) / 32 * 32;
-  return (int)S;
+  const long long Q = (long long)p.B * ((p.H + G - 1) / G);
+  const long long ns_max = Q * ((p.N + kSTok - 1) / kSTok);
+  return (size_t)(num_ranges(ns_max, num_sms()) + Q);
 }
-
-size_t records_bytes(const Problem &p, int S) {
+size_t records_bytes(const Problem &p) {
   const int G = kGroupCh / p.D;
-  const int HG = (p.H + G - 1) / G;
-  const size_t chunks = (size_t)p.B * HG * ((p.N + S - 1) / S);
-  return chunks * G * ((size_t)p.D * p.D + p.D + 4) * sizeof(float);
+  return record_slots(p) * G * ((size_t)p.D * p.D + p.D + 4) * sizeof(float);
 }
 
 template <int D>
@@ -1680,30 +1639,27 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
                       const float *conv_w, void *ws, float *state, cudaStream_t st,
                       float2 *gate_stats) {
   constexpr int G = kGroupCh / D;
-  const int S = chunk_len(p);
-  const size_t rb = records_bytes(p, S);
+  const size_t rb = records_bytes(p);
   StateParams sp;
   sp.gate = (const __nv_bfloat16 *)gate;
   sp.conv_w = conv_w;
   sp.seq_lens = p.seq_lens;
   sp.records = (float *)ws;
-  sp.chunk_pre = (int32_t *)((char *)ws + rb);
+  sp.stage_pre = (int32_t *)((char *)ws + rb);
   sp.B = p.B;
   sp.H = p.H;
   sp.N = p.N;
-  sp.S = S;
   sp.flags = p.flags;
   sp.HG = (p.H + G - 1) / G;
-  CUtensorMap tm_k, tm_v, tm_rec;
+  CUtensorMap tm_k, tm_v;
   cudaError_t e = make_group_map(&tm_k, k, p.B, p.N, p.H, D);
   if (e != cudaSuccess) return e;
   if ((e = make_bnhd_map(&tm_v, v, p.B, p.N, p.H, D, kSRawRows)) != cudaSuccess) return e;
-  if ((e = make_records_map(&tm_rec, ws, p, D, S)) != cudaSuccess) return e;
   auto k1 = p.flags ? tc_state_kernel<D, true> : tc_state_kernel<D, false>;
   if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
       cudaSuccess)
     return e;
-  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v, tm_rec);
+  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v);
   count_launch();
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
@@ -1719,8 +1675,8 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, tc_reduce_kernel<D>, (const float *)sp.records,
-                         (const int32_t *)sp.chunk_pre, p.seq_lens, state, gate_stats, p.B,
-                         p.H, p.N, S);
+                         (const int32_t *)sp.stage_pre, p.seq_lens, state, gate_stats, p.B,
+                         p.H, p.N, num_sms());
   count_launch();
   return e;
 }
@@ -1776,14 +1732,20 @@ bool tc_supports(const Problem &p) {
   if (p.dtype != GBLA_BF16) return false;
   if (p.D != 64 && p.D != 128) return false;
   if (p.B > kMaxBatch) return false;
-  if ((long long)p.N > (long long)kChunkMax * kMaxChunksPerSeq) return false;
+  // sequences of at most 2^23 tokens (the combination's scale factors of one
+  // sequence fit in shared memory)
+  if (p.N > (1 << 23)) return false;
+  // stage indices are ints: B * HG * ceil(N / 64) stages at most
+  if ((long long)p.B * ((p.H + kGroupCh / p.D - 1) / (kGroupCh / p.D)) *
+          (((long long)p.N + kSTok - 1) / kSTok) > (1ll << 30))
+    return false;
   if ((long long)p.B * p.H > 2147483647ll / 4) return false;
   if (p.H < kGroupCh / p.D) return false;  // the state tiles span a whole head group
   return device_info().sm103 && encode_fn() != nullptr;
 }
 
 size_t tc_workspace_bytes(const Problem &p) {
-  return records_bytes(p, chunk_len(p)) + sizeof(int32_t) * (p.B + 1) + 256;
+  return records_bytes(p) + sizeof(int32_t) * (p.B + 1) + 256;
 }
 
 cudaError_t tc_state(const Problem &p, const void *k, const void *v, const void *gate,
