@@ -9,6 +9,11 @@ follows Sec. 2 (bidirectional linear attention, Eq. bla) and Sec. 2.1 (GBLA:
 Conv1D, key gating, gated RMSNorm) of the paper.  This module only compiles
 it with gcc and marshals numpy arrays into it.
 
+The bidirectional softmax attention of Sec. 2 (``softmax_attention``), the SA
+layer of the paper's hybrid [SA, LA, LA] encoder, is pinned by the
+``pin_sa_*`` checks (library softmax and matrix products, torch's own
+attention, invariants).
+
 The layer front end (``gbla_project``: the X-space Conv1D and the stacked
 Q, K, V, R and w_g projections of Sec. 2.1 items 1-3) and the whole layer
 (``gbla_layer``: front end, then the core with its Conv1D off) are pinned by
@@ -95,6 +100,10 @@ def _declare(lib):
     lib.oracle_gbla_project.argtypes = [_dp, _dp, _dp, ctypes.POINTER(ctypes.c_int32),
                                         ctypes.c_long, ctypes.c_long, ctypes.c_int,
                                         ctypes.c_int, ctypes.c_long, ctypes.c_int] + [_dp] * 6
+    lib.oracle_softmax_attention.restype = ctypes.c_int
+    lib.oracle_softmax_attention.argtypes = [_dp, _dp, _dp, ctypes.POINTER(ctypes.c_int32),
+                                             ctypes.c_long, ctypes.c_long, ctypes.c_long,
+                                             ctypes.c_int, ctypes.c_int, _dp]
     lib.oracle_gbla_forward.restype = ctypes.c_int
     lib.oracle_gbla_forward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
                                         ctypes.POINTER(ctypes.c_int32),
@@ -223,6 +232,27 @@ def gbla_forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None,
         B, H, N, D, W, float(eps), int(flags), int(n_threads), _ptr(y))
     if rc != 0:
         raise ValueError(f"oracle_gbla_forward rejected its arguments ({rc})")
+    return y
+
+
+def softmax_attention(q, k, v, seq_lens=None, n_threads=1, out=None, lib=None):
+    """Bidirectional softmax attention of Sec. 2 over [B, N, H, D] arrays: for
+    every valid query i < L_b, sum_j exp(q_i . k_j / sqrt(D)) v_j / sum_j exp(...)
+    over the valid keys j < L_b.  Rows t >= L_b keep `out`'s values (NaN when
+    `out` is not given)."""
+    q, k, v = (_f64(t) for t in (q, k, v))
+    B, N, H, D = q.shape
+    y = np.full((B, N, H, D), np.nan) if out is None else out
+    assert y.dtype == np.float64 and y.flags.c_contiguous and y.shape == q.shape
+    sl = None
+    if seq_lens is not None:
+        sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    rc = (lib or load()).oracle_softmax_attention(
+        _ptr(q), _ptr(k), _ptr(v),
+        sl.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)) if sl is not None else None,
+        B, N, H, D, int(n_threads), _ptr(y))
+    if rc != 0:
+        raise ValueError(f"oracle_softmax_attention rejected its arguments ({rc})")
     return y
 
 

@@ -636,3 +636,89 @@ int oracle_gbla_project(const double *x, const double *conv_x, const double *w,
   free(xt);
   return 0;
 }
+
+/* ------------------------------------------------------------------------
+ * Bidirectional softmax attention (Sec. 2, "Bidirectional softmax
+ * attention"), the SA layer of the hybrid [SA, LA, LA] encoder (Sec. 3):
+ *   Attn(q_i, K, V) = sum_j exp(q_i . k_j / sqrt(d_h)) v_j / sum_j exp(q_i . k_j / sqrt(d_h)),
+ * over the valid keys j < L of one (batch, head), for each valid query i < L.
+ * Arrays are [B, N, H, D] (token-major, heads interleaved); rows t >= L of
+ * out are left as they are.  The maximum score of each row is subtracted
+ * before exponentiating (the quotient does not change; it keeps exp finite).
+ * Rows are independent, so (batch, head) pairs run on n_threads threads.
+ * ------------------------------------------------------------------------ */
+typedef struct {
+  const double *q, *k, *v;
+  const int32_t *seq_lens;
+  long B, N, H;
+  int D;
+  double *out;
+  long next;
+  pthread_mutex_t mu;
+} oracle_sa_job;
+
+static void sa_pair(oracle_sa_job *J, long p) {
+  const long b = p / J->H, h = p % J->H, N = J->N, H = J->H;
+  const int D = J->D;
+  long L = J->seq_lens ? J->seq_lens[b] : N;
+  if (L < 0) L = 0;
+  if (L > N) L = N;
+  const double scale = 1.0 / sqrt((double)D);
+  double *s = (double *)xmalloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+  for (long i = 0; i < L; ++i) {
+    const double *qi = J->q + ((b * N + i) * H + h) * D;
+    double m = -INFINITY;
+    for (long j = 0; j < L; ++j) {
+      const double *kj = J->k + ((b * N + j) * H + h) * D;
+      double dot = 0.0;
+      for (int d = 0; d < D; ++d) dot += qi[d] * kj[d];
+      s[j] = dot * scale;
+      if (s[j] > m) m = s[j];
+    }
+    double den = 0.0;
+    for (long j = 0; j < L; ++j) {
+      s[j] = exp(s[j] - m);
+      den += s[j];
+    }
+    double *oi = J->out + ((b * N + i) * H + h) * D;
+    for (int d = 0; d < D; ++d) oi[d] = 0.0;
+    for (long j = 0; j < L; ++j) {
+      const double *vj = J->v + ((b * N + j) * H + h) * D;
+      for (int d = 0; d < D; ++d) oi[d] += s[j] * vj[d];
+    }
+    for (int d = 0; d < D; ++d) oi[d] /= den;
+  }
+  free(s);
+}
+
+static void *sa_worker(void *arg) {
+  oracle_sa_job *J = (oracle_sa_job *)arg;
+  for (;;) {
+    pthread_mutex_lock(&J->mu);
+    const long p = J->next++;
+    pthread_mutex_unlock(&J->mu);
+    if (p >= J->B * J->H) break;
+    sa_pair(J, p);
+  }
+  return NULL;
+}
+
+int oracle_softmax_attention(const double *q, const double *k, const double *v,
+                             const int32_t *seq_lens, long B, long N, long H, int D,
+                             int n_threads, double *out) {
+  if (B < 0 || N < 0 || H < 0 || D <= 0) return -1;
+  oracle_sa_job J;
+  J.q = q; J.k = k; J.v = v; J.seq_lens = seq_lens;
+  J.B = B; J.N = N; J.H = H; J.D = D; J.out = out; J.next = 0;
+  pthread_mutex_init(&J.mu, NULL);
+  if (n_threads < 1) n_threads = 1;
+  if (n_threads > 256) n_threads = 256;
+  pthread_t th[256];
+  int started = 0;
+  for (int i = 1; i < n_threads; ++i)
+    if (pthread_create(&th[started], NULL, sa_worker, &J) == 0) ++started;
+  sa_worker(&J);
+  for (int i = 0; i < started; ++i) pthread_join(th[i], NULL);
+  pthread_mutex_destroy(&J.mu);
+  return 0;
+}

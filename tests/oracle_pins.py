@@ -461,4 +461,84 @@ def pin_layer_conv_commutes(lib):
     np.testing.assert_allclose(y_layer, y_core, rtol=0, atol=1e-10)
 
 
+# --- bidirectional softmax attention (Sec. 2), the SA layer of the hybrid ------
+
+def _sa_inputs(rng, B=2, N=9, H=3, D=5):
+    return tuple(rng.standard_normal((B, N, H, D)) for _ in range(3))
+
+
+def pin_sa_library(lib):
+    """Attn(q_i) = softmax_j(q_i . k_j / sqrt(D)) V over the valid keys, by numpy
+    matrix products and scipy's softmax, per (batch, head)."""
+    rng = _rng(80)
+    q, k, v = _sa_inputs(rng)
+    sl = np.array([9, 4], np.int32)
+    y = oracle.softmax_attention(q, k, v, seq_lens=sl, lib=lib)
+    D = q.shape[3]
+    for b in range(2):
+        L = sl[b]
+        for h in range(3):
+            s = q[b, :L, h] @ k[b, :L, h].T / math.sqrt(D)
+            ref = scipy.special.softmax(s, axis=1) @ v[b, :L, h]
+            np.testing.assert_allclose(y[b, :L, h], ref, rtol=1e-12, atol=1e-14)
+        assert np.all(np.isnan(y[b, L:])), "rows past the sequence end were written"
+
+
+def pin_sa_torch(lib):
+    """torch's own attention (fp64, keys past the end masked) gives the same rows."""
+    rng = _rng(81)
+    q, k, v = _sa_inputs(rng, B=2, N=11, H=2, D=8)
+    sl = np.array([11, 6], np.int32)
+    y = oracle.softmax_attention(q, k, v, seq_lens=sl, lib=lib)
+    t = lambda a: torch.tensor(a).permute(0, 2, 1, 3)  # noqa: E731  [B, H, N, D]
+    mask = torch.zeros(2, 1, 11, 11, dtype=torch.bool)
+    for b in range(2):
+        mask[b, :, :, :sl[b]] = True
+    ref = torch.nn.functional.scaled_dot_product_attention(t(q), t(k), t(v), attn_mask=mask)
+    ref = ref.permute(0, 2, 1, 3).numpy()
+    for b in range(2):
+        np.testing.assert_allclose(y[b, :sl[b]], ref[b, :sl[b]], rtol=1e-12, atol=1e-14)
+
+
+def pin_sa_closed_forms(lib):
+    """A single key gives its own value; q = 0 gives the mean of the valid values;
+    equal value rows give that row back; a dominant score picks its key's value
+    without overflow (the row maximum is subtracted)."""
+    rng = _rng(82)
+    q, k, v = _sa_inputs(rng, B=1, N=7, H=2, D=4)
+    y1 = oracle.softmax_attention(q, k, v, seq_lens=np.array([1], np.int32), lib=lib)
+    np.testing.assert_allclose(y1[0, 0], v[0, 0], rtol=0, atol=1e-15)
+    y0 = oracle.softmax_attention(np.zeros_like(q), k, v, seq_lens=np.array([5], np.int32),
+                                  lib=lib)
+    np.testing.assert_allclose(y0[0, :5], np.broadcast_to(v[0, :5].mean(axis=0), (5, 2, 4)),
+                               rtol=1e-13, atol=1e-15)
+    vc = np.broadcast_to(v[:, :1], v.shape).copy()
+    yc = oracle.softmax_attention(q, k, vc, lib=lib)
+    np.testing.assert_allclose(yc, np.broadcast_to(vc[:, :1], vc.shape), rtol=1e-13, atol=1e-15)
+    kb = k.copy()
+    # key 3 dominates query 2 with a score of 1000 in both heads (exp would
+    # overflow without the row maximum subtracted)
+    for h in range(2):
+        kb[0, 3, h] = 1000.0 * math.sqrt(4) * q[0, 2, h] / (q[0, 2, h] @ q[0, 2, h])
+    yb = oracle.softmax_attention(q * 1.0, kb, v, lib=lib)
+    assert np.all(np.isfinite(yb))
+    np.testing.assert_allclose(yb[0, 2], v[0, 3], rtol=0, atol=1e-9)
+
+
+def pin_sa_permutations(lib):
+    """Permuting the valid keys together with their values changes nothing;
+    permuting the queries permutes the rows; heads are independent."""
+    rng = _rng(83)
+    q, k, v = _sa_inputs(rng, B=1, N=8, H=3, D=4)
+    y = oracle.softmax_attention(q, k, v, lib=lib)
+    perm = rng.permutation(8)
+    yk = oracle.softmax_attention(q, k[:, perm], v[:, perm], lib=lib)
+    np.testing.assert_allclose(yk, y, rtol=1e-12, atol=1e-14)
+    yq = oracle.softmax_attention(q[:, perm], k, v, lib=lib)
+    np.testing.assert_allclose(yq, y[:, perm], rtol=1e-12, atol=1e-14)
+    hp = [2, 0, 1]
+    yh = oracle.softmax_attention(q[:, :, hp], k[:, :, hp], v[:, :, hp], lib=lib)
+    np.testing.assert_allclose(yh, y[:, :, hp], rtol=1e-12, atol=1e-14)
+
+
 ALL_PINS = [v for k_, v in sorted(globals().items()) if k_.startswith("pin_")]

@@ -57,6 +57,15 @@ MUTANTS = [
     ("project_writes_padding", "for (long t = 0; t < L; ++t) {\n      const double *xr",
      "for (long t = 0; t < N; ++t) {\n      const double *xr"),
     ("project_absdot_signed", "mag += fabs(xr[c] * wr[c]);", "mag += xr[c] * wr[c];"),
+    ("sa_no_scale", "s[j] = dot * scale;", "s[j] = dot;"),
+    ("sa_no_max", "s[j] = exp(s[j] - m);", "s[j] = exp(s[j]);"),
+    ("sa_keys_from_tail", "const double *kj = J->k + ((b * N + j) * H + h) * D;",
+     "const double *kj = J->k + ((b * N + j + (N - L)) * H + h) * D;"),
+    ("sa_key_head", "const double *kj = J->k + ((b * N + j) * H + h) * D;",
+     "const double *kj = J->k + ((b * N + j) * H + 0) * D;"),
+    ("sa_not_normalised", "for (int d = 0; d < D; ++d) oi[d] /= den;",
+     "for (int d = 0; d < D; ++d) oi[d] /= 1.0;"),
+    ("sa_value_index", "oi[d] += s[j] * vj[d];", "oi[d] += s[j] * vj[0];"),
 ]
 
 
