@@ -1,6 +1,7 @@
 """Benchmark of the GBLA layer-core forward on GB300 (one JSON line on rank 0).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME] [--backward | --layer | --hybrid]
 
 A step is one GBLA forward (Conv1D, phi, key gate, state reduction, readout,
 gated RMSNorm) over the paper's headline length: B=2, H=8, N=32768, D=64,
@@ -456,6 +457,97 @@ def bench_layer(args, ws, rank, local):
         torch.distributed.destroy_process_group()
 
 
+def bench_hybrid(args, ws, rank, local):
+    """--hybrid: the paper's hybrid encoder block [SA, LA, LA] (Sec. 3) against an
+    all-softmax block [SA, SA, SA], core only (the mixing of given q, k, v, and for
+    GBLA the gate and out-gate inputs): batch 8, 16 heads of 64 (Table 5), L from
+    2048 to 32768.  Each stack is its three calls back to back on one stream;
+    per-layer latencies of both layers and the SA / GBLA ratio (Table 5's
+    columns) are printed per L.  SA is this library's tcgen05 kernel
+    (gbla_attention_forward), timed against the bf16 tensor peak."""
+    from paper_2606_07317_gb300 import gbla
+    from paper_2606_07317_gb300.workloads import custom
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    init_dist(ws, "nccl")
+    gbla.load()
+    B, H, D = 8, 16, 64
+    stream = torch.cuda.current_stream(dev)
+    tf_peak, tf_kind = measured_bf16_peak()
+    rows = []
+    sampler = ClockSampler(local)
+    sampler.start()
+    n0 = gbla.launch_count()
+    for L in args.hybrid_lengths:
+        inp = make_inputs(custom(B=B, H=H, N=L, D=D, dtype="bf16", seed=L), dev)
+        o_sa = torch.empty_like(inp["q"])
+        o_la = torch.empty_like(inp["q"])
+
+        def sa():
+            gbla.attention(inp["q"], inp["k"], inp["v"], None, out=o_sa, stream=stream)
+
+        def la():
+            gbla.forward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"],
+                         inp["conv_w"], inp["norm_w"], None, out=o_la, stream=stream)
+
+        def timed(fn, budget_s=4.0):
+            for _ in range(args.warmup):
+                fn()
+            torch.cuda.synchronize(dev)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            one = e0.elapsed_time(e1)
+            n = max(1, min(args.steps, int(budget_s * 1e3 / max(one, 1e-3))))
+            barrier(ws)
+            e0.record(stream)
+            for _ in range(n):
+                fn()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            return max_over_ranks(e0.elapsed_time(e1) / n, ws, dev), n
+
+        t_sa, n_sa = timed(sa)
+        t_la, n_la = timed(la)
+        t_hyb, _ = timed(lambda: (sa(), la(), la()))
+        t_all, _ = timed(lambda: (sa(), sa(), sa()))
+        flops = 4.0 * B * H * L * L * D
+        rows.append({"L": L, "sa_ms": round(t_sa, 4), "gbla_ms": round(t_la, 4),
+                     "sa_over_gbla": round(t_sa / t_la, 2),
+                     "block_sa_la_la_ms": round(t_hyb, 4), "block_sa_sa_sa_ms": round(t_all, 4),
+                     "block_speedup": round(t_all / t_hyb, 2),
+                     "sa_tflops": round(flops / (t_sa * 1e-3) / 1e12, 1),
+                     "sa_frac_of_bf16_peak": round(flops / (t_sa * 1e-3) / 1e12 / tf_peak, 4),
+                     "gbla_tokens_per_s": round(B * L / (t_la * 1e-3), 1),
+                     "timed_calls": {"sa": n_sa, "gbla": n_la}})
+        del inp, o_sa, o_la
+        torch.cuda.empty_cache()
+    clocks = sampler.stop()
+    assert gbla.device_error() == 0
+    if rank == 0:
+        last = rows[-1]
+        print(json.dumps({
+            "metric": "hybrid encoder block [SA, LA, LA] vs [SA, SA, SA]: per-layer latency "
+                      "(core), batch 8, 16 heads of 64",
+            "value": last["block_speedup"], "unit": "x (block [SA,SA,SA] / [SA,LA,LA] time) "
+                                                     "at the longest L",
+            "n_gpus": ws, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic (seeded N(0,1) inputs)",
+            "config": {"workload": "hybrid_block_b8_h16_d64", "B": B, "H": H, "D": D,
+                       "lengths": args.hybrid_lengths,
+                       "note": "core only: SA = softmax mixing of q, k, v; LA = the GBLA core "
+                               "(Conv1D, key gate, state, readout, gated RMSNorm); no "
+                               "projections in either"},
+            "per_length": rows,
+            "sa_peak": {"bf16_tflops": tf_peak, "source": tf_kind},
+            "gpu_launches": gbla.launch_count() - n0, "clocks": clocks}), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
 def bench_e2e(args, w, inp, dev, gbla, tokens, ws):
     host = {k: (v.cpu().pin_memory() if v is not None else None) for k, v in inp.items()}
     out = torch.empty_like(host["q"]).pin_memory()
@@ -630,6 +722,11 @@ def main(argv=None):
                     help="time the whole layer from X (gbla_layer_forward) and its front end")
     ap.add_argument("--model-dim", type=int, default=0,
                     help="--layer: model width d (default H * D)")
+    ap.add_argument("--hybrid", action="store_true",
+                    help="time the hybrid block [SA, LA, LA] against [SA, SA, SA] (Table 5's "
+                         "shapes: batch 8, 16 heads of 64) over --hybrid-lengths")
+    ap.add_argument("--hybrid-lengths", type=int, nargs="+",
+                    default=[2048, 4096, 8192, 16384, 32768])
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -645,6 +742,9 @@ def main(argv=None):
         return
     if args.layer:
         bench_layer(args, ws, rank, local)
+        return
+    if args.hybrid:
+        bench_hybrid(args, ws, rank, local)
         return
     bench_ours(args, ws, rank, local)
 

@@ -220,6 +220,25 @@ gbla_status gbla_layer_forward(const void *x, const float *conv_x, const void *w
                                gbla_stream_t stream);
 
 /*
+ * gbla_attention_forward -- bidirectional softmax attention, Sec. 2
+ * ("Bidirectional softmax attention"): the SA layer of the hybrid [SA, LA, LA]
+ * encoder of Sec. 3, whose latency the GBLA layer is compared with (Sec. 4,
+ * Table 5).  For every batch row b, head h and valid query i < L_b,
+ *   o_i = sum_j exp(q_i . k_j / sqrt(D)) v_j / sum_j exp(q_i . k_j / sqrt(D)),
+ * over the valid keys j < L_b (no causal mask).
+ *   q, k, v, o [B, N, H, D] dtype, token-major as gbla_forward's inputs;
+ *   seq_lens   device [B] int32 or NULL (= all N), clamped to [0, N].
+ * Rows t >= L_b of o are not written.  bf16 with D = 64 on an sm_103 GPU only
+ * (tcgen05 tensor cores: bf16 operands, fp32 accumulation, probabilities
+ * rounded to bf16 for the second product); anything else returns
+ * GBLA_ERR_UNSUPPORTED.  o must not overlap an input.  Asynchronous on
+ * `stream`; allocates nothing.
+ */
+gbla_status gbla_attention_forward(const void *q, const void *k, const void *v,
+                                   const int32_t *seq_lens, void *o, int B, int H, int N,
+                                   int D, gbla_dtype dtype, gbla_stream_t stream);
+
+/*
  * gbla_state -- the sequence-global part of Sec. 2.1 item 2: Conv1D of k and
  * v, phi, the softmax key gate, and per (b, h) the state S = K^T V~ and the
  * normaliser z = K^T 1 with K^ = g * phi(K~), g the softmax over j < L_b.

@@ -103,7 +103,10 @@ def _declare(lib):
     lib.oracle_softmax_attention.restype = ctypes.c_int
     lib.oracle_softmax_attention.argtypes = [_dp, _dp, _dp, ctypes.POINTER(ctypes.c_int32),
                                              ctypes.c_long, ctypes.c_long, ctypes.c_long,
-                                             ctypes.c_int, ctypes.c_int, _dp]
+                                             ctypes.c_int, ctypes.c_int, _dp, _dp]
+    lib.oracle_softmax_attention_rows.restype = ctypes.c_int
+    lib.oracle_softmax_attention_rows.argtypes = [_dp, ctypes.c_long, _dp, _dp, ctypes.c_long,
+                                                  ctypes.c_int, _dp, _dp]
     lib.oracle_gbla_forward.restype = ctypes.c_int
     lib.oracle_gbla_forward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
                                         ctypes.POINTER(ctypes.c_int32),
@@ -235,25 +238,43 @@ def gbla_forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None,
     return y
 
 
-def softmax_attention(q, k, v, seq_lens=None, n_threads=1, out=None, lib=None):
+def softmax_attention(q, k, v, seq_lens=None, n_threads=1, out=None, absout=False, lib=None):
     """Bidirectional softmax attention of Sec. 2 over [B, N, H, D] arrays: for
     every valid query i < L_b, sum_j exp(q_i . k_j / sqrt(D)) v_j / sum_j exp(...)
     over the valid keys j < L_b.  Rows t >= L_b keep `out`'s values (NaN when
-    `out` is not given)."""
+    `out` is not given).  With absout=True also returns sum_j p_j |v_j| / sum_j p_j
+    per output (the scale of the error a relative rounding of the probabilities
+    p_j makes)."""
     q, k, v = (_f64(t) for t in (q, k, v))
     B, N, H, D = q.shape
     y = np.full((B, N, H, D), np.nan) if out is None else out
     assert y.dtype == np.float64 and y.flags.c_contiguous and y.shape == q.shape
+    a = np.full((B, N, H, D), np.nan) if absout else None
     sl = None
     if seq_lens is not None:
         sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
     rc = (lib or load()).oracle_softmax_attention(
         _ptr(q), _ptr(k), _ptr(v),
         sl.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)) if sl is not None else None,
-        B, N, H, D, int(n_threads), _ptr(y))
+        B, N, H, D, int(n_threads), _ptr(y), _ptr(a))
     if rc != 0:
         raise ValueError(f"oracle_softmax_attention rejected its arguments ({rc})")
-    return y
+    return (y, a) if absout else y
+
+
+def softmax_attention_rows(q_rows, k, v, lib=None):
+    """Selected query rows q_rows [R, D] of one (batch, head) against its valid
+    keys and values k, v [L, D]; returns (out, absout), each [R, D]."""
+    q_rows, k, v = (_f64(t) for t in (q_rows, k, v))
+    R, D = q_rows.shape
+    L = k.shape[0]
+    y = np.empty((R, D))
+    a = np.empty((R, D))
+    rc = (lib or load()).oracle_softmax_attention_rows(_ptr(q_rows), R, _ptr(k), _ptr(v), L, D,
+                                                       _ptr(y), _ptr(a))
+    if rc != 0:
+        raise ValueError(f"oracle_softmax_attention_rows rejected its arguments ({rc})")
+    return y, a
 
 
 def gbla_head_backward(q, k, v, a, og, wq, wk, wv, norm_w, dy, eps=RMS_EPS, flags=0,

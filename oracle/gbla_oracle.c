@@ -652,10 +652,47 @@ typedef struct {
   const int32_t *seq_lens;
   long B, N, H;
   int D;
-  double *out;
+  double *out, *absout;
   long next;
   pthread_mutex_t mu;
 } oracle_sa_job;
+
+/* One query row against the L keys and values of one (batch, head), strided
+ * by ld between tokens: out[d] = the attention output, absout[d] (optional) =
+ * sum_j p_j |v_j[d]| / sum_j p_j, the scale of the error a relative rounding
+ * of the probabilities p_j makes.  s is scratch of L doubles. */
+static void sa_row(const double *qi, const double *k, const double *v, long L, long ld, int D,
+                   double *s, double *out, double *absout) {
+  const double scale = 1.0 / sqrt((double)D);
+  double m = -INFINITY;
+  for (long j = 0; j < L; ++j) {
+    const double *kj = k + j * ld;
+    double dot = 0.0;
+    for (int d = 0; d < D; ++d) dot += qi[d] * kj[d];
+    s[j] = dot * scale;
+    if (s[j] > m) m = s[j];
+  }
+  double den = 0.0;
+  for (long j = 0; j < L; ++j) {
+    s[j] = exp(s[j] - m);
+    den += s[j];
+  }
+  for (int d = 0; d < D; ++d) {
+    out[d] = 0.0;
+    if (absout) absout[d] = 0.0;
+  }
+  for (long j = 0; j < L; ++j) {
+    const double *vj = v + j * ld;
+    for (int d = 0; d < D; ++d) {
+      out[d] += s[j] * vj[d];
+      if (absout) absout[d] += s[j] * fabs(vj[d]);
+    }
+  }
+  for (int d = 0; d < D; ++d) {
+    out[d] /= den;
+    if (absout) absout[d] /= den;
+  }
+}
 
 static void sa_pair(oracle_sa_job *J, long p) {
   const long b = p / J->H, h = p % J->H, N = J->N, H = J->H;
@@ -663,31 +700,11 @@ static void sa_pair(oracle_sa_job *J, long p) {
   long L = J->seq_lens ? J->seq_lens[b] : N;
   if (L < 0) L = 0;
   if (L > N) L = N;
-  const double scale = 1.0 / sqrt((double)D);
+  const long ld = H * D, base = (b * N * H + h) * D;
   double *s = (double *)xmalloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
-  for (long i = 0; i < L; ++i) {
-    const double *qi = J->q + ((b * N + i) * H + h) * D;
-    double m = -INFINITY;
-    for (long j = 0; j < L; ++j) {
-      const double *kj = J->k + ((b * N + j) * H + h) * D;
-      double dot = 0.0;
-      for (int d = 0; d < D; ++d) dot += qi[d] * kj[d];
-      s[j] = dot * scale;
-      if (s[j] > m) m = s[j];
-    }
-    double den = 0.0;
-    for (long j = 0; j < L; ++j) {
-      s[j] = exp(s[j] - m);
-      den += s[j];
-    }
-    double *oi = J->out + ((b * N + i) * H + h) * D;
-    for (int d = 0; d < D; ++d) oi[d] = 0.0;
-    for (long j = 0; j < L; ++j) {
-      const double *vj = J->v + ((b * N + j) * H + h) * D;
-      for (int d = 0; d < D; ++d) oi[d] += s[j] * vj[d];
-    }
-    for (int d = 0; d < D; ++d) oi[d] /= den;
-  }
+  for (long i = 0; i < L; ++i)
+    sa_row(J->q + base + i * ld, J->k + base, J->v + base, L, ld, D, s, J->out + base + i * ld,
+           J->absout ? J->absout + base + i * ld : NULL);
   free(s);
 }
 
@@ -705,11 +722,11 @@ static void *sa_worker(void *arg) {
 
 int oracle_softmax_attention(const double *q, const double *k, const double *v,
                              const int32_t *seq_lens, long B, long N, long H, int D,
-                             int n_threads, double *out) {
+                             int n_threads, double *out, double *absout) {
   if (B < 0 || N < 0 || H < 0 || D <= 0) return -1;
   oracle_sa_job J;
   J.q = q; J.k = k; J.v = v; J.seq_lens = seq_lens;
-  J.B = B; J.N = N; J.H = H; J.D = D; J.out = out; J.next = 0;
+  J.B = B; J.N = N; J.H = H; J.D = D; J.out = out; J.absout = absout; J.next = 0;
   pthread_mutex_init(&J.mu, NULL);
   if (n_threads < 1) n_threads = 1;
   if (n_threads > 256) n_threads = 256;
@@ -720,5 +737,18 @@ int oracle_softmax_attention(const double *q, const double *k, const double *v,
   sa_worker(&J);
   for (int i = 0; i < started; ++i) pthread_join(th[i], NULL);
   pthread_mutex_destroy(&J.mu);
+  return 0;
+}
+
+/* Selected query rows of one (batch, head): q_rows [R][D] against keys and
+ * values k, v [L][D] (contiguous), giving out and absout [R][D] (see sa_row). */
+int oracle_softmax_attention_rows(const double *q_rows, long R, const double *k,
+                                  const double *v, long L, int D, double *out,
+                                  double *absout) {
+  if (R < 0 || L < 1 || D <= 0) return -1;
+  double *s = (double *)xmalloc(sizeof(double) * (size_t)L);
+  for (long r = 0; r < R; ++r)
+    sa_row(q_rows + r * D, k, v, L, D, D, s, out + r * D, absout ? absout + r * D : NULL);
+  free(s);
   return 0;
 }

@@ -204,8 +204,10 @@ uint64_t gbla_launch_count(void) { return g_launches.load(std::memory_order_rela
 
 uint32_t gbla_device_error(int reset) {
   const unsigned a = tc_device_error(reset != 0), b = project_device_error(reset != 0);
-  const unsigned c = bwd_device_error(reset != 0);
-  return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu || c == 0xFFFFFFFFu) ? 0xFFFFFFFFu : (a | b | c);
+  const unsigned c = bwd_device_error(reset != 0), d = sa_device_error(reset != 0);
+  return (a == 0xFFFFFFFFu || b == 0xFFFFFFFFu || c == 0xFFFFFFFFu || d == 0xFFFFFFFFu)
+             ? 0xFFFFFFFFu
+             : (a | b | c | d);
 }
 
 const char *gbla_last_cuda_error(void) { return last_cuda_error_string(); }
@@ -459,6 +461,24 @@ gbla_status gbla_layer_forward(const void *x, const float *conv_x, const void *w
   // the core with its Conv1D off (the taps are never read)
   if ((s = run_state(p, tc, k, v, gate, nullptr, state, st)) != GBLA_OK) return s;
   return run_readout(p, tc, q, og, nullptr, norm_w, state, o, st, true);
+}
+
+gbla_status gbla_attention_forward(const void *q, const void *k, const void *v,
+                                   const int32_t *seq_lens, void *o, int B, int H, int N,
+                                   int D, gbla_dtype dtype, gbla_stream_t stream) {
+  bool empty = false;
+  gbla_status s = check_dims(B, H, N, D, dtype, &empty);
+  if (s != GBLA_OK || empty) return s;
+  if ((s = check_ptrs({q, k, v, o})) != GBLA_OK) return s;
+  if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
+  if (!sa_supports(D, dtype)) return GBLA_ERR_UNSUPPORTED;
+  const size_t bytes = (size_t)B * N * H * D * elem_bytes(dtype);
+  const Range out = range_of(o, bytes);
+  if (overlap(out, range_of(q, bytes)) || overlap(out, range_of(k, bytes)) ||
+      overlap(out, range_of(v, bytes)) ||
+      (seq_lens && overlap(out, range_of(seq_lens, sizeof(int32_t) * B))))
+    return GBLA_ERR_INVALID_ARG;
+  return from_cuda(sa_forward(q, k, v, seq_lens, o, B, H, N, (cudaStream_t)stream));
 }
 
 gbla_status gbla_forward_host(const void *q, const void *k, const void *v,

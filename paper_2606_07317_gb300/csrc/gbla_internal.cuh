@@ -115,6 +115,12 @@ cudaError_t tc_project(const ProjProblem &pp, const void *x, const float *conv_x
                        cudaStream_t st);
 unsigned project_device_error(bool reset);
 
+// ---- bidirectional softmax attention (tcgen05; gbla_sa.cu): bf16, D = 64 --
+bool sa_supports(int D, gbla_dtype dtype);
+cudaError_t sa_forward(const void *q, const void *k, const void *v, const int32_t *seq_lens,
+                       void *o, int B, int H, int N, cudaStream_t st);
+unsigned sa_device_error(bool reset);
+
 // Error bits set by tensor-core kernels whose bounded waits ran out (0 = none);
 // synchronous read of the current device, optionally clearing it.
 unsigned tc_device_error(bool reset);

@@ -30,7 +30,7 @@ EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_for
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
             "gbla_state_static_scratch", "gbla_device_error", "gbla_last_cuda_error",
-            "gbla_project", "gbla_layer_forward"]
+            "gbla_project", "gbla_layer_forward", "gbla_attention_forward"]
 
 _lock = threading.Lock()
 _lib = None
@@ -78,6 +78,8 @@ def load(path: str | None = None):
         lib.gbla_project.restype = _i
         lib.gbla_layer_forward.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
         lib.gbla_layer_forward.restype = _i
+        lib.gbla_attention_forward.argtypes = [_vp] * 5 + [_i] * 5 + [_vp]
+        lib.gbla_attention_forward.restype = _i
         lib.gbla_forward_host.argtypes = fwd + [_vp]
         lib.gbla_forward_host.restype = _i
         lib.gbla_state.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
@@ -184,6 +186,18 @@ def forward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=None,
         _ptr(norm_w), _ptr(seq_lens), _ptr(out), B, H, N, D, _dtype_code(q), int(algo),
         _stream(stream))
     _check(st, "gbla_forward_ex")
+    return out
+
+
+def attention(q, k, v, seq_lens=None, out=None, stream=None) -> torch.Tensor:
+    """Bidirectional softmax attention of Sec. 2 (gbla_attention_forward): q, k, v,
+    out [B, N, H, D] bf16 (D = 64); rows past seq_lens are not written."""
+    B, H, N, D = _bhnd(q)
+    if out is None:
+        out = torch.empty_like(q)
+    st = load().gbla_attention_forward(_ptr(q), _ptr(k), _ptr(v), _ptr(seq_lens), _ptr(out),
+                                       B, H, N, D, _dtype_code(q), _stream(stream))
+    _check(st, "gbla_attention_forward")
     return out
 
 

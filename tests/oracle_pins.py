@@ -525,6 +525,22 @@ def pin_sa_closed_forms(lib):
     np.testing.assert_allclose(yb[0, 2], v[0, 3], rtol=0, atol=1e-9)
 
 
+def pin_sa_rows_and_abs_scale(lib):
+    """The one-row entry gives the full oracle's rows; the error scale
+    sum_j p_j |v_j| / sum_j p_j is at least |o| and equals it for v >= 0."""
+    rng = _rng(84)
+    q, k, v = _sa_inputs(rng, B=1, N=10, H=2, D=6)
+    y, a = oracle.softmax_attention(q, k, v, seq_lens=np.array([8], np.int32), absout=True,
+                                    lib=lib)
+    for h in range(2):
+        yr, ar = oracle.softmax_attention_rows(q[0, [1, 7], h], k[0, :8, h], v[0, :8, h], lib=lib)
+        np.testing.assert_allclose(yr, y[0, [1, 7], h], rtol=1e-14, atol=1e-15)
+        np.testing.assert_allclose(ar, a[0, [1, 7], h], rtol=1e-14, atol=1e-15)
+    assert np.all(a[0, :8] >= np.abs(y[0, :8]) - 1e-15)
+    yp, ap = oracle.softmax_attention(q, k, np.abs(v), absout=True, lib=lib)
+    np.testing.assert_allclose(ap, yp, rtol=1e-14, atol=0)
+
+
 def pin_sa_permutations(lib):
     """Permuting the valid keys together with their values changes nothing;
     permuting the queries permutes the rows; heads are independent."""

@@ -59,13 +59,13 @@ MUTANTS = [
     ("project_absdot_signed", "mag += fabs(xr[c] * wr[c]);", "mag += xr[c] * wr[c];"),
     ("sa_no_scale", "s[j] = dot * scale;", "s[j] = dot;"),
     ("sa_no_max", "s[j] = exp(s[j] - m);", "s[j] = exp(s[j]);"),
-    ("sa_keys_from_tail", "const double *kj = J->k + ((b * N + j) * H + h) * D;",
-     "const double *kj = J->k + ((b * N + j + (N - L)) * H + h) * D;"),
-    ("sa_key_head", "const double *kj = J->k + ((b * N + j) * H + h) * D;",
-     "const double *kj = J->k + ((b * N + j) * H + 0) * D;"),
-    ("sa_not_normalised", "for (int d = 0; d < D; ++d) oi[d] /= den;",
-     "for (int d = 0; d < D; ++d) oi[d] /= 1.0;"),
-    ("sa_value_index", "oi[d] += s[j] * vj[d];", "oi[d] += s[j] * vj[0];"),
+    ("sa_keys_from_tail", "sa_row(J->q + base + i * ld, J->k + base, J->v + base, L,",
+     "sa_row(J->q + base + i * ld, J->k + base + (N - L) * ld, J->v + base, L,"),
+    ("sa_key_head", "sa_row(J->q + base + i * ld, J->k + base, J->v + base",
+     "sa_row(J->q + base + i * ld, J->k + b * N * H * D, J->v + base"),
+    ("sa_not_normalised", "out[d] /= den;", "out[d] /= 1.0;"),
+    ("sa_value_index", "out[d] += s[j] * vj[d];", "out[d] += s[j] * vj[0];"),
+    ("sa_abs_unsigned", "absout[d] += s[j] * fabs(vj[d]);", "absout[d] += s[j] * vj[d];"),
 ]
 
 
