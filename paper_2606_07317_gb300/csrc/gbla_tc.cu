@@ -854,18 +854,22 @@ __global__ void __launch_bounds__(kSThreads, 1)
 // butterfly order), and each thread then accumulates its 4 state elements
 // over the batch in record order, 16 loads in flight at a time, with the
 // scale factors broadcast from the lanes that computed them.
+//
+// LEAN (the grid has at most one block per SM): 32 registers a thread and 4
+// loads in flight.  The state kernel's 19 warps leave exactly one 32-register
+// warp per SM sub-partition free, so a lean block is made resident beside the
+// state CTA as soon as the state grid signals its dependents, and waits there
+// for the state grid to complete instead of being scheduled after it.
 constexpr int kReduceThreads = 128;
-template <int D>
-__global__ void __launch_bounds__(kReduceThreads, 1) tc_reduce_kernel(const float *__restrict__ records,
-                                                         const int32_t *__restrict__ stage_pre,
-                                                         const int32_t *__restrict__ seq_lens,
-                                                         float *__restrict__ state,
-                                                         float2 *__restrict__ gate_stats, int B,
-                                                         int H, int N, int P) {
+template <int D, bool LEAN>
+__global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
+    tc_reduce_kernel(const float *__restrict__ records, const int32_t *__restrict__ stage_pre,
+                     const int32_t *__restrict__ seq_lens, float *__restrict__ state,
+                     float2 *__restrict__ gate_stats, int B, int H, int N, int P) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
-  constexpr int CH = 16;   // record loads in flight per thread
+  constexpr int CH = LEAN ? 4 : 16;   // record loads in flight per thread
   grid_dep_wait();
   grid_dep_launch();
   const int lane = threadIdx.x & 31;
@@ -1669,14 +1673,15 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(p.B * p.H, (F / 4 + kReduceThreads - 1) / kReduceThreads);
+  const bool lean = (long long)cfg.gridDim.x * cfg.gridDim.y <= num_sms();
   cfg.blockDim = dim3(kReduceThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, tc_reduce_kernel<D>, (const float *)sp.records,
-                         (const int32_t *)sp.stage_pre, p.seq_lens, state, gate_stats, p.B,
-                         p.H, p.N, num_sms());
+  e = cudaLaunchKernelEx(&cfg, lean ? tc_reduce_kernel<D, true> : tc_reduce_kernel<D, false>,
+                         (const float *)sp.records, (const int32_t *)sp.stage_pre, p.seq_lens,
+                         state, gate_stats, p.B, p.H, p.N, num_sms());
   count_launch();
   return e;
 }
