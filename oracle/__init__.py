@@ -89,7 +89,7 @@ def _declare(lib):
     lib.oracle_gbla_head_backward.restype = ctypes.c_int
     lib.oracle_gbla_head_backward.argtypes = (
         [_dp, _dp, _dp, _dp, _dp, ctypes.c_long, ctypes.c_long, ctypes.c_long, ctypes.c_int,
-         _dp, _dp, _dp, ctypes.c_int, _dp, ctypes.c_double, ctypes.c_int, _dp] + [_dp] * 9)
+         _dp, _dp, _dp, ctypes.c_int, _dp, ctypes.c_double, ctypes.c_int, _dp] + [_dp] * 18)
     lib.oracle_gbla_backward.restype = ctypes.c_int
     lib.oracle_gbla_backward.argtypes = [_dp, _dp, _dp, _dp, _dp, _dp, _dp,
                                          ctypes.POINTER(ctypes.c_int32),
@@ -278,10 +278,12 @@ def softmax_attention_rows(q_rows, k, v, lib=None):
 
 
 def gbla_head_backward(q, k, v, a, og, wq, wk, wv, norm_w, dy, eps=RMS_EPS, flags=0,
-                       lib=None):
+                       scales=False, lib=None):
     """Gradients of sum(dy * y) for one (batch, head) (chain rule through the six
     forward steps of Sec. 2.1, reverse order).  Returns a dict with dq, dk, dv, dog
-    [L, D], da [L], dwq, dwk, dwv [D, W] and dnorm_w [D]."""
+    [L, D], da [L], dwq, dwk, dwv [D, W] and dnorm_w [D]; with ``scales`` also the
+    error scales mdq, mdk, mdv, mdog [L, D], mda [L], mdwq, mdwk, mdwv [D, W] and
+    mdnorm_w [D] (see oracle_gbla_head_backward in the C file)."""
     q, k, v, og, dy = (_f64(t) for t in (q, k, v, og, dy))
     a = _f64(a); wq, wk, wv = (_f64(t) for t in (wq, wk, wv)); norm_w = _f64(norm_w)
     L, D = q.shape
@@ -289,22 +291,93 @@ def gbla_head_backward(q, k, v, a, og, wq, wk, wv, norm_w, dy, eps=RMS_EPS, flag
     out = dict(dq=np.zeros((L, D)), dk=np.zeros((L, D)), dv=np.zeros((L, D)),
                da=np.zeros(L), dog=np.zeros((L, D)), dwq=np.zeros((D, W)),
                dwk=np.zeros((D, W)), dwv=np.zeros((D, W)), dnorm_w=np.zeros(D))
+    mags = [None] * 9
+    if scales:
+        out.update(mdq=np.zeros((L, D)), mdk=np.zeros((L, D)), mdv=np.zeros((L, D)),
+                   mda=np.zeros(L), mdog=np.zeros((L, D)), mdwq=np.zeros((D, W)),
+                   mdwk=np.zeros((D, W)), mdwv=np.zeros((D, W)), mdnorm_w=np.zeros(D))
+        mags = [_ptr(out[n]) for n in ("mdq", "mdk", "mdv", "mda", "mdog", "mdwq", "mdwk",
+                                       "mdwv", "mdnorm_w")]
     rc = (lib or load()).oracle_gbla_head_backward(
         _ptr(q), _ptr(k), _ptr(v), _ptr(a), _ptr(og), D, 1, L, D, _ptr(wq), _ptr(wk),
         _ptr(wv), W, _ptr(norm_w), float(eps), int(flags), _ptr(dy),
         *[_ptr(out[n]) for n in ("dq", "dk", "dv", "da", "dog", "dwq", "dwk", "dwv",
-                                 "dnorm_w")])
+                                 "dnorm_w")], *mags)
     if rc != 0:
         raise ValueError(f"oracle_gbla_head_backward rejected its arguments ({rc})")
     return out
 
 
+def _at(arr, offset):
+    """Pointer to element `offset` of a C-contiguous float64 array."""
+    return ctypes.cast(arr.ctypes.data + 8 * int(offset), _dp)
+
+
 def gbla_backward(q, k, v, gate, out_gate, conv_w, norm_w, dy, seq_lens=None,
-                  eps=RMS_EPS, flags=0, lib=None):
+                  eps=RMS_EPS, flags=0, scales=False, n_threads=1, lib=None):
     """Whole-core backward over [B, N, H, D] arrays: gradients of sum(dy * y).
 
     Returns a dict: dq, dk, dv, dout_gate [B, N, H, D]; dgate [B, N, H]; dconv_w
-    [3, H, D, W]; dnorm_w [H, D].  Rows past seq_lens[b] are zero."""
+    [3, H, D, W]; dnorm_w [H, D].  Rows past seq_lens[b] are zero.  With
+    ``scales``, also the error scales mdq, mdk, mdv, mdout_gate [B, N, H, D],
+    mdgate [B, N, H] (zero past seq_lens[b]), mdconv_w [3, H, D, W] and
+    mdnorm_w [H, D].
+
+    One call of oracle_gbla_head_backward per (batch, head).  With n_threads > 1
+    the heads run on that many threads, each head taking its batches in batch
+    order, so the tap and norm-weight sums over the batch are added in the same
+    order as by oracle_gbla_backward (the serial loop in C) and equal its
+    results exactly."""
+    q, k, v, og, dy = (_f64(t) for t in (q, k, v, out_gate, dy))
+    gate = _f64(gate); conv_w = _f64(conv_w); norm_w = _f64(norm_w)
+    B, N, H, D = q.shape
+    W = conv_w.shape[-1]
+    names = ["dq", "dk", "dv", "dgate", "dout_gate", "dconv_w", "dnorm_w"]
+    out = dict(dq=np.zeros_like(q), dk=np.zeros_like(q), dv=np.zeros_like(q),
+               dgate=np.zeros_like(gate), dout_gate=np.zeros_like(q),
+               dconv_w=np.zeros_like(conv_w), dnorm_w=np.zeros_like(norm_w))
+    if scales:
+        for n in names:
+            out["m" + n] = np.zeros_like(out[n])
+    sl = None if seq_lens is None else np.asarray(seq_lens, dtype=np.int64)
+    lb = lib or load()
+    ld = H * D
+
+    def head(h):
+        for b in range(B):
+            L = N if sl is None else int(min(max(sl[b], 0), N))
+            base, gbase = (b * N * H + h) * D, b * N * H + h
+            grads = [_at(out[n], gbase if n == "dgate" else base)
+                     for n in ("dq", "dk", "dv", "dgate", "dout_gate")]
+            taps = [_at(out["dconv_w"], ((i * H + h) * D) * W) for i in range(3)]
+            mags = [None] * 9
+            if scales:
+                mags = [_at(out["m" + n], gbase if n == "dgate" else base)
+                        for n in ("dq", "dk", "dv", "dgate", "dout_gate")]
+                mags += [_at(out["mdconv_w"], ((i * H + h) * D) * W) for i in range(3)]
+                mags += [_at(out["mdnorm_w"], h * D)]
+            rc = lb.oracle_gbla_head_backward(
+                _at(q, base), _at(k, base), _at(v, base), _at(gate, gbase), _at(og, base),
+                ld, H, L, D, *[_at(conv_w, ((i * H + h) * D) * W) for i in range(3)], W,
+                _at(norm_w, h * D), float(eps), int(flags), _at(dy, base),
+                *grads, *taps, _at(out["dnorm_w"], h * D), *mags)
+            if rc != 0:
+                raise ValueError(f"oracle_gbla_head_backward rejected its arguments ({rc})")
+
+    if n_threads > 1 and H > 1:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=min(n_threads, H)) as ex:
+            list(ex.map(head, range(H)))
+    else:
+        for h in range(H):
+            head(h)
+    return out
+
+
+def gbla_backward_serial(q, k, v, gate, out_gate, conv_w, norm_w, dy, seq_lens=None,
+                         eps=RMS_EPS, flags=0, lib=None):
+    """The same gradients through oracle_gbla_backward, the serial (batch, head)
+    loop written in C (pins the Python loop of gbla_backward)."""
     q, k, v, og, dy = (_f64(t) for t in (q, k, v, out_gate, dy))
     gate = _f64(gate); conv_w = _f64(conv_w); norm_w = _f64(norm_w)
     B, N, H, D = q.shape

@@ -393,11 +393,175 @@ static void conv1d_backward(const double *x, const double *dxt, long L, int C,
 
 static double phi_prime(double x) { return x > 0.0 ? 1.0 : exp(x); }
 
+/* Error scales of the gradients (see oracle_gbla_head_backward): the
+ * backward steps 6' to 1' on magnitudes, from the inputs q, k, v, the forward
+ * intermediates qt, kt, vt, g, O, den and the exact dO.  Per-token scales are
+ * written; tap and norm-weight scales are ADDED (sums over the batch). */
+static void backward_scales(const double *q, const double *k, const double *v, long L, int D,
+                            long ld, long lda, int W, const double *wq, const double *wk,
+                            const double *wv, const double *norm_w, double eps, int flags,
+                            const double *dy, const double *og, const double *qt,
+                            const double *kt, const double *vt, const double *g,
+                            const double *O, const double *dO, const double *den,
+                            double *mdq, double *mdk, double *mdv, double *mda,
+                            double *mdog, double *mdwq, double *mdwk, double *mdwv,
+                            double *mdnw) {
+  double *Sa = xmalloc(sizeof(double) * D * D);
+  double *Oa = xmalloc(sizeof(double) * L * D);
+  double *dOa = xmalloc(sizeof(double) * L * D);
+  double *dSa = xmalloc(sizeof(double) * D * D);
+  double *dza = xmalloc(sizeof(double) * D);
+  double *dqta = xmalloc(sizeof(double) * L * D);
+  double *dkta = xmalloc(sizeof(double) * L * D);
+  double *dvta = xmalloc(sizeof(double) * L * D);
+  double *dga = xmalloc(sizeof(double) * L);
+  double *dKa = xmalloc(sizeof(double) * D);
+  double *za = xmalloc(sizeof(double) * D);  /* z = sum_j K^_j > 0: its own magnitude */
+
+  /* forward on magnitudes: Sa = sum_j K^_j |v~_j|^T, Oa_i = P_i^T Sa / den_i */
+  memset(Sa, 0, sizeof(double) * D * D);
+  memset(za, 0, sizeof(double) * D);
+  for (long j = 0; j < L; ++j)
+    for (int d = 0; d < D; ++d) {
+      const double kh = g[j] * oracle_phi(kt[j * D + d]);
+      za[d] += kh;
+      for (int e = 0; e < D; ++e) Sa[d * D + e] += kh * fabs(vt[j * D + e]);
+    }
+  for (long i = 0; i < L; ++i)
+    for (int e = 0; e < D; ++e) {
+      double s = 0.0;
+      for (int d = 0; d < D; ++d) s += oracle_phi(qt[i * D + d]) * Sa[d * D + e];
+      Oa[i * D + e] = s / den[i];
+    }
+
+  /* 6'. gated RMSNorm: dO = r u - (r^3 / D) O (u . O) */
+  for (long i = 0; i < L; ++i) {
+    const double *Oi = O + i * D, *Oai = Oa + i * D, *dyi = dy + i * ld, *ogi = og + i * ld;
+    double *dOai = dOa + i * D, *mdogi = mdog + i * ld;
+    if (flags & ORACLE_NO_NORM) {
+      for (int e = 0; e < D; ++e) {
+        dOai[e] = fabs(dyi[e]);
+        mdogi[e] = 0.0;
+      }
+      continue;
+    }
+    double ms = 0.0;
+    for (int e = 0; e < D; ++e) ms += Oi[e] * Oi[e];
+    ms /= (double)D;
+    const double r = 1.0 / sqrt(ms + eps);
+    double uo = 0.0, uoa = 0.0;
+    for (int e = 0; e < D; ++e) {
+      const double u = dyi[e] * norm_w[e] * oracle_silu(ogi[e]);
+      uo += u * Oi[e];
+      uoa += fabs(u) * Oai[e];
+    }
+    for (int e = 0; e < D; ++e) {
+      const double sg = oracle_sigmoid(ogi[e]);
+      const double u = dyi[e] * norm_w[e] * oracle_silu(ogi[e]);
+      dOai[e] = r * fabs(u) + (r * r * r / (double)D) * (Oai[e] * fabs(uo) + fabs(Oi[e]) * uoa);
+      mdogi[e] = fabs(dyi[e]) * Oai[e] * r * fabs(norm_w[e]) *
+                 fabs(sg * (1.0 + ogi[e] * (1.0 - sg)));
+      mdnw[e] += fabs(dyi[e]) * Oai[e] * r * fabs(oracle_silu(ogi[e]));
+    }
+  }
+
+  /* 5'. readout: dnum = dO / den, dden = -(dO . O) / den, dP = S dnum + z dden */
+  memset(dSa, 0, sizeof(double) * D * D);
+  memset(dza, 0, sizeof(double) * D);
+  for (long i = 0; i < L; ++i) {
+    const double *Oi = O + i * D, *Oai = Oa + i * D, *dOi = dO + i * D, *dOai = dOa + i * D;
+    double ddena = 0.0;
+    for (int e = 0; e < D; ++e) ddena += dOai[e] * fabs(Oi[e]) + fabs(dOi[e]) * Oai[e];
+    ddena /= den[i];
+    for (int d = 0; d < D; ++d) {
+      const double P = oracle_phi(qt[i * D + d]);
+      double s = za[d] * ddena;
+      for (int e = 0; e < D; ++e) s += Sa[d * D + e] * dOai[e] / den[i];
+      dqta[i * D + d] = phi_prime(qt[i * D + d]) * s;
+      dza[d] += P * ddena;
+      for (int e = 0; e < D; ++e) dSa[d * D + e] += P * dOai[e] / den[i];
+    }
+  }
+
+  /* 4'. state: dK^_j = dS v~_j + dz, dv~_j = dS^T K^_j, dg_j = phi(k~_j) . dK^_j */
+  double gdga = 0.0;
+  for (long j = 0; j < L; ++j) {
+    double dg = 0.0;
+    for (int d = 0; d < D; ++d) {
+      double s = dza[d];
+      for (int e = 0; e < D; ++e) s += dSa[d * D + e] * fabs(vt[j * D + e]);
+      dKa[d] = s;
+      dkta[j * D + d] = g[j] * phi_prime(kt[j * D + d]) * s;
+      dg += oracle_phi(kt[j * D + d]) * s;
+    }
+    dga[j] = dg;
+    gdga += g[j] * dg;
+    for (int e = 0; e < D; ++e) {
+      double s = 0.0;
+      for (int d = 0; d < D; ++d) s += g[j] * oracle_phi(kt[j * D + d]) * dSa[d * D + e];
+      dvta[j * D + e] = s;
+    }
+  }
+
+  /* 3'. key gate: da_j = g_j (dg_j - sum_i g_i dg_i) */
+  for (long j = 0; j < L; ++j)
+    mda[j * lda] = (flags & ORACLE_NO_GATE) ? 0.0 : g[j] * (dga[j] + gdga);
+
+  /* 1'. Conv1D: dx_s = sum_i w_i dx~_{s+(W-1)-i} on magnitudes */
+  const double *taps[3] = {wq, wk, wv};
+  const double *src[3] = {dqta, dkta, dvta};
+  const double *xin[3] = {q, k, v};
+  double *dst[3] = {mdq, mdk, mdv};
+  double *dwa[3] = {mdwq, mdwk, mdwv};
+  for (int m = 0; m < 3; ++m)
+    for (long s0 = 0; s0 < L; ++s0)
+      for (int c = 0; c < D; ++c) {
+        double acc = 0.0;
+        if (flags & ORACLE_NO_CONV) {
+          acc = src[m][s0 * D + c];
+        } else {
+          for (int i = 0; i < W; ++i) {
+            const long t = s0 + (W - 1) - i;
+            if (t < L) acc += fabs(taps[m][(long)c * W + i]) * src[m][t * D + c];
+          }
+        }
+        dst[m][s0 * ld + c] = acc;
+      }
+  /*     dw_i += sum_t dx~_t x_{t-(W-1)+i} on magnitudes */
+  if (!(flags & ORACLE_NO_CONV))
+    for (int m = 0; m < 3; ++m)
+      for (int c = 0; c < D; ++c)
+        for (int i = 0; i < W; ++i) {
+          double acc = 0.0;
+          for (long t = 0; t < L; ++t) {
+            const long s0 = t - (W - 1) + i;
+            if (s0 >= 0) acc += src[m][t * D + c] * fabs(xin[m][s0 * ld + c]);
+          }
+          dwa[m][(long)c * W + i] += acc;
+        }
+
+  free(Sa); free(Oa); free(dOa); free(dSa); free(dza); free(dqta); free(dkta);
+  free(dvta); free(dga); free(dKa); free(za);
+}
+
 /*
  * One (batch, head): gradients of sum(dy * y) with respect to every input.
  * Inputs as oracle_gbla_head plus dy (L rows at stride ld).  Outputs: dq, dk,
  * dv, dog (L rows at stride ld), da (stride lda), and tap / norm-weight
- * gradients ADDED to dwq, dwk, dwv [D][W] and dnw [D].  Returns 0 or -1.
+ * gradients ADDED to dwq, dwk, dwv [D][W] and dnw [D].
+ *
+ * Optional error scales (all NULL, or all given; same layouts as dq, dk, dv,
+ * da, dog, dwq, dwk, dwv, dnw, the last four ADDED to): for every gradient,
+ * the first-order magnitude of what a relative perturbation of size 1 in each
+ * rounded intermediate can move it by.
+ * They are the same chain rule evaluated on magnitudes: every product and sum
+ * on absolute values, and in place of the state and its gradient (both sums
+ * over the whole sequence, which cancel) their absolute sums
+ *   Sa = sum_j K^_j |v~_j|^T,  dSa = sum_i P_i dnuma_i^T,  dza = sum_i P_i ddena_i,
+ * so a computation whose every rounded quantity x carries an error of at most
+ * eps |x| (or eps times its own scale) stays within a small multiple of
+ * eps times these scales.  Each scale is at least |gradient|.
+ * Returns 0 or -1.
  */
 int oracle_gbla_head_backward(const double *q, const double *k, const double *v,
                               const double *a, const double *og, long ld, long lda,
@@ -405,7 +569,10 @@ int oracle_gbla_head_backward(const double *q, const double *k, const double *v,
                               const double *wv, int W, const double *norm_w,
                               double eps, int flags, const double *dy, double *dq,
                               double *dk, double *dv, double *da, double *dog,
-                              double *dwq, double *dwk, double *dwv, double *dnw) {
+                              double *dwq, double *dwk, double *dwv, double *dnw,
+                              double *mdq, double *mdk, double *mdv, double *mda,
+                              double *mdog, double *mdwq, double *mdwk, double *mdwv,
+                              double *mdnw) {
   if (L < 0 || D <= 0 || W <= 0) return -1;
   if (L == 0) return 0;
   double *qt = xmalloc(sizeof(double) * L * D);
@@ -529,6 +696,10 @@ int oracle_gbla_head_backward(const double *q, const double *k, const double *v,
     conv1d_backward(v, dvt, L, D, ld, wv, W, dv, dwv);
   }
 
+  if (mdq) backward_scales(q, k, v, L, D, ld, lda, W, wq, wk, wv, norm_w, eps, flags, dy, og,
+                           qt, kt, vt, g, O, dO, den, mdq, mdk, mdv, mda, mdog, mdwq, mdwk,
+                           mdwv, mdnw);
+
 done:
   free(qt); free(kt); free(vt); free(g); free(S); free(z); free(O); free(dO);
   free(dS); free(dz); free(dqt); free(dkt); free(dvt); free(dg); free(P);
@@ -570,7 +741,8 @@ int oracle_gbla_backward(const double *q, const double *k, const double *v,
           conv_w + ((2 * H + h) * D) * W, W, norm_w + h * D, eps, flags, dy + base,
           dq + base, dk + base, dv + base, dgate + gbase, dog + base,
           dconv_w + ((0 * H + h) * D) * W, dconv_w + ((1 * H + h) * D) * W,
-          dconv_w + ((2 * H + h) * D) * W, dnorm_w + h * D);
+          dconv_w + ((2 * H + h) * D) * W, dnorm_w + h * D, NULL, NULL, NULL, NULL, NULL,
+          NULL, NULL, NULL, NULL);
       if (rc != 0) return rc;
     }
   return 0;

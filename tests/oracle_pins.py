@@ -557,4 +557,117 @@ def pin_sa_permutations(lib):
     np.testing.assert_allclose(yh, y[:, :, hp], rtol=1e-12, atol=1e-14)
 
 
+# --- backward (chain rule through Sec. 2.1's steps) and its error scales ------
+
+_BWD = dict(q="dq", k="dk", v="dv", a="da", og="dog", wq="dwq", wk="dwk", wv="dwv",
+            norm_w="dnorm_w")
+_SCALED = (("dq", "mdq"), ("dk", "mdk"), ("dv", "mdv"), ("da", "mda"), ("dog", "mdog"),
+           ("dwq", "mdwq"), ("dwk", "mdwk"), ("dwv", "mdwv"), ("dnorm_w", "mdnorm_w"))
+
+
+def _bwd_inputs(rng, L, D):
+    q, k, v, a, og, wq, wk, wv, nw = _head_inputs(rng, L, D)
+    return dict(q=q, k=k, v=v, a=a, og=og, wq=wq, wk=wk, wv=wv, norm_w=nw)
+
+
+def pin_backward_finite_differences(lib):
+    """Every gradient equals the central difference of sum(dy * y) of the
+    oracle's forward (full core and Eq. bla's plain form)."""
+    rng = _rng(90)
+    x = _bwd_inputs(rng, 6, 3)
+    dy = rng.standard_normal((6, 3))
+    for flags in (0, oracle.BLA):
+        g = oracle.gbla_head_backward(**x, dy=dy, eps=1e-3, flags=flags, lib=lib)
+        h = 1e-5
+        for name, gname in _BWD.items():
+            num = np.empty_like(x[name])
+            for idx in np.ndindex(x[name].shape):
+                xp = {kk: vv.copy() for kk, vv in x.items()}
+                xm = {kk: vv.copy() for kk, vv in x.items()}
+                xp[name][idx] += h
+                xm[name][idx] -= h
+                lp = np.sum(dy * oracle.gbla_head(**xp, eps=1e-3, flags=flags, lib=lib))
+                lm = np.sum(dy * oracle.gbla_head(**xm, eps=1e-3, flags=flags, lib=lib))
+                num[idx] = (lp - lm) / (2 * h)
+            np.testing.assert_allclose(g[gname], num, rtol=1e-6, atol=1e-8,
+                                       err_msg=f"{gname} flags={flags}")
+
+
+def pin_backward_threaded_equals_serial(lib):
+    """The per-head Python loop (threads over heads) gives exactly the serial
+    (batch, head) loop written in C, padding rows zero."""
+    rng = _rng(91)
+    B, N, H, D = 2, 11, 3, 4
+    arrs = dict(q=rng.standard_normal((B, N, H, D)), k=rng.standard_normal((B, N, H, D)),
+                v=rng.standard_normal((B, N, H, D)), gate=rng.standard_normal((B, N, H)),
+                out_gate=rng.standard_normal((B, N, H, D)),
+                conv_w=0.5 * rng.standard_normal((3, H, D, W)),
+                norm_w=1.0 + 0.1 * rng.standard_normal((H, D)))
+    dy = rng.standard_normal((B, N, H, D))
+    a = oracle.gbla_backward(**arrs, dy=dy, seq_lens=[11, 4], n_threads=3, lib=lib)
+    b = oracle.gbla_backward_serial(**arrs, dy=dy, seq_lens=[11, 4], lib=lib)
+    for n in b:
+        assert np.array_equal(a[n], b[n]), n
+    assert np.all(a["dq"][1, 4:] == 0) and np.all(a["dgate"][1, 4:] == 0)
+
+
+def _scaled_case(seed, flags, L=40, D=6):
+    rng = _rng(seed)
+    x = _bwd_inputs(rng, L, D)
+    dy = rng.standard_normal((L, D))
+    return x, dy
+
+
+def pin_backward_scales_dominate(lib):
+    """Each error scale is at least the magnitude of its gradient (it is the
+    same chain rule on magnitudes, with the absolute state sums)."""
+    for flags in (0, oracle.NO_CONV, oracle.NO_GATE, oracle.NO_NORM, oracle.BLA):
+        x, dy = _scaled_case(92, flags)
+        g = oracle.gbla_head_backward(**x, dy=dy, flags=flags, scales=True, lib=lib)
+        for n, m in _SCALED:
+            assert np.all(g[m] >= np.abs(g[n]) * (1 - 1e-12)), (n, flags)
+
+
+def pin_backward_scales_bound_dy_perturbation(lib):
+    """The gradients are linear in dy and the scales depend on |dy| only, so a
+    perturbation dy -> dy (1 + e r), |r| <= 1, moves every gradient by at most
+    e times its scale."""
+    x, dy = _scaled_case(93, 0)
+    g0 = oracle.gbla_head_backward(**x, dy=dy, scales=True, lib=lib)
+    e = 1e-6
+    r = _rng(94).uniform(-1, 1, dy.shape)
+    g1 = oracle.gbla_head_backward(**x, dy=dy * (1 + e * r), lib=lib)
+    for n, m in _SCALED:
+        assert np.all(np.abs(g1[n] - g0[n]) <= e * g0[m] * (1 + 1e-6) + 1e-300), n
+    g2 = oracle.gbla_head_backward(**x, dy=-3.0 * dy, scales=True, lib=lib)
+    for n, m in _SCALED:
+        np.testing.assert_allclose(g2[m], 3.0 * g0[m], rtol=1e-12, atol=0, err_msg=m)
+
+
+def pin_backward_scales_bound_input_perturbation(lib):
+    """Relative perturbations e of q, k or v (which reach the rounded
+    intermediates phi(q~), K^ and V~ through the Conv1D) move every
+    per-token gradient by less than e times its scale."""
+    for flags in (0, oracle.NO_CONV):
+        x, dy = _scaled_case(95, flags, L=60)
+        g0 = oracle.gbla_head_backward(**x, dy=dy, flags=flags, scales=True, lib=lib)
+        e = 1e-7
+        for name in ("q", "k", "v"):
+            r = _rng(96).uniform(-1, 1, x[name].shape)
+            x1 = dict(x)
+            x1[name] = x[name] * (1 + e * r)
+            g1 = oracle.gbla_head_backward(**x1, dy=dy, flags=flags, lib=lib)
+            for n, m in _SCALED[:5]:
+                assert np.all(np.abs(g1[n] - g0[n]) <= e * g0[m]), (name, n, flags)
+
+
+def pin_backward_scales_exact_without_cancellation(lib):
+    """With nothing that can cancel (Eq. bla's plain form, v >= 0, dy >= 0) the
+    value gradient's scale equals the gradient: dv~ = dS^T K^ with dS >= 0."""
+    x, dy = _scaled_case(97, oracle.BLA)
+    x["v"] = np.abs(x["v"])
+    g = oracle.gbla_head_backward(**x, dy=np.abs(dy), flags=oracle.BLA, scales=True, lib=lib)
+    np.testing.assert_allclose(g["mdv"], g["dv"], rtol=1e-12, atol=0)
+
+
 ALL_PINS = [v for k_, v in sorted(globals().items()) if k_.startswith("pin_")]

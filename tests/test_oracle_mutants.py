@@ -66,6 +66,18 @@ MUTANTS = [
     ("sa_not_normalised", "out[d] /= den;", "out[d] /= 1.0;"),
     ("sa_value_index", "out[d] += s[j] * vj[d];", "out[d] += s[j] * vj[0];"),
     ("sa_abs_unsigned", "absout[d] += s[j] * fabs(vj[d]);", "absout[d] += s[j] * vj[d];"),
+    ("bwd_dden_sign", "const double dden = -dOO / den[i];", "const double dden = dOO / den[i];"),
+    ("bwd_dS_transposed", "for (int e = 0; e < D; ++e) dS[d * D + e] += P[d] * dnum[e];",
+     "for (int e = 0; e < D; ++e) dS[e * D + d] += P[d] * dnum[e];"),
+    ("bwd_phi_prime_branch", "return x > 0.0 ? 1.0 : exp(x);", "return x > 0.0 ? 1.0 : 1.0;"),
+    ("bwd_conv_transpose_causal", "long t = s + (W - 1) - i;", "long t = s - (W - 1) + i;"),
+    ("bwd_norm_cube", "dOi[e] = r * u - (r * r * r / (double)D) * Oi[e] * uo;",
+     "dOi[e] = r * u - (r * r / (double)D) * Oi[e] * uo;"),
+    ("scale_state_signed", "Sa[d * D + e] += kh * fabs(vt[j * D + e]);",
+     "Sa[d * D + e] += kh * vt[j * D + e];"),
+    ("scale_conv_signed",
+     "if (t < L) acc += fabs(taps[m][(long)c * W + i]) * src[m][t * D + c];",
+     "if (t < L) acc += taps[m][(long)c * W + i] * src[m][t * D + c];"),
 ]
 
 
