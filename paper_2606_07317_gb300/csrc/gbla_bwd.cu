@@ -466,7 +466,7 @@ __global__ void __launch_bounds__(kNT) bwd_key(
 }
 
 // ---------------------------------------------------------------- Conv1D backward
-// Stream s = blockIdx.z (0 q, 1 k, 2 v) over a block of RUNS x rl tokens of
+// Stream s = 2 - blockIdx.z (0 q, 1 k, 2 v) over a block of RUNS x rl tokens of
 // one (b, h): dx_t = sum_i w_i dx~_{t+3-i} (terms with t + 3 - i >= L dropped;
 // dx_t = 0 for t >= L) and the block's partials of dw_i = sum_t dx~_t x_{t-3+i}.
 // Thread (run, g) walks rl consecutive tokens of channels
@@ -516,7 +516,9 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
     T *__restrict__ dv, float *__restrict__ wpart, int H, int N, int nck, int rl) {
   constexpr int G = D / kConvCh, RUNS = kNT / G;
   __shared__ float sw[RUNS][D * kConvW];
-  const int chunk = blockIdx.x, bh = blockIdx.y, s = blockIdx.z, b = bh / H, h = bh % H;
+  // v first: its dv~ plane is the one most recently written (by the key pass)
+  // and the most likely still to sit in L2 when the first blocks run
+  const int chunk = blockIdx.x, bh = blockIdx.y, s = 2 - (int)blockIdx.z, b = bh / H, h = bh % H;
   const int tid = threadIdx.x, g = tid % G, run = tid / G;
   const T *x = s == 0 ? q : (s == 1 ? k : v);
   T *dx = s == 0 ? dq : (s == 1 ? dk : dv);

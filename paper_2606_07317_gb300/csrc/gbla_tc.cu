@@ -366,7 +366,6 @@ struct StateParams {
   const float *conv_w;
   const int32_t *seq_lens;
   float *records;        // [ranges + sequences][G][D*D + D + 4]: S, z, m, l, 2 pad
-  int32_t *stage_pre;    // [B + 1] stage prefix (written by CTA 0 when seq_lens is given)
   int B, H, N, HG;
   uint32_t flags;        // gbla_flags (NO_CONV, NO_GATE)
 };
@@ -505,8 +504,6 @@ __global__ void __launch_bounds__(kSThreads, 1)
       });
     __syncthreads();
     NS = pre[B];
-    if (blockIdx.x == 0)
-      for (int i = tid; i <= B; i += kSThreads) p.stage_pre[i] = pre[i];
   }
   const long long R = num_ranges(NS, gridDim.x);
   grid_dep_launch();
@@ -855,24 +852,32 @@ __global__ void __launch_bounds__(kSThreads, 1)
 // over the batch in record order, 16 loads in flight at a time, with the
 // scale factors broadcast from the lanes that computed them.
 //
-// LEAN (the grid has at most one block per SM): 32 registers a thread and 4
-// loads in flight.  The state kernel's 19 warps leave exactly one 32-register
-// warp per SM sub-partition free, so a lean block is made resident beside the
-// state CTA as soon as the state grid signals its dependents, and waits there
-// for the state grid to complete instead of being scheduled after it.
+// LEAN (the grid has at most one block per SM): 32 registers a thread, 4
+// loads in flight in registers and 5 more staged through shared memory by
+// cp.async (10 KB).  The state kernel's 19 warps leave exactly one 32-register
+// warp per SM sub-partition free, and its shared memory leaves room for the
+// staging buffer, so a lean block is made resident beside the state CTA as
+// soon as the state grid signals its dependents, and waits there for the
+// state grid to complete instead of being scheduled after it.
 constexpr int kReduceThreads = 128;
 template <int D, bool LEAN>
 __global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
-    tc_reduce_kernel(const float *__restrict__ records, const int32_t *__restrict__ stage_pre,
-                     const int32_t *__restrict__ seq_lens, float *__restrict__ state,
-                     float2 *__restrict__ gate_stats, int B, int H, int N, int P) {
+    tc_reduce_kernel(const float *__restrict__ records, const int32_t *__restrict__ seq_lens,
+                     float *__restrict__ state, float2 *__restrict__ gate_stats, int B, int H,
+                     int N, int P) {
   constexpr int G = kGroupCh / D;
   constexpr int REC = D * D + D + 4;
   constexpr int F = D * D + D;
-  constexpr int CH = LEAN ? 4 : 16;   // record loads in flight per thread
-  grid_dep_wait();
-  grid_dep_launch();
-  const int lane = threadIdx.x & 31;
+  constexpr int CH = LEAN ? 4 : 16;   // record loads in flight per thread (registers)
+  constexpr int SMR = LEAN ? 5 : 0;   // and staged through shared memory
+  constexpr int CHT = CH + SMR;       // records per round trip
+  __shared__ float4 stg[SMR > 0 ? SMR : 1][kReduceThreads];
+  __shared__ int red[2][kReduceThreads / 32];
+  // A lean block is resident while the state grid still runs: it lets the
+  // readout launch only once the state is complete (below).  Other blocks
+  // start after the state grid: the readout may be scheduled at once.
+  if constexpr (!LEAN) grid_dep_launch();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int bh = blockIdx.x;
   const int b = bh / H, h = bh % H;
   const int hg = h / G, hh = h % G, HG = (H + G - 1) / G;
@@ -880,26 +885,81 @@ __global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
   const bool act = e0 < F;  // every thread takes part in the shuffles
   const int L = clamp_len(seq_lens, b, N);
   const int nst = (L + kSTok - 1) / kSTok;
+  // The record indices first: they depend only on the lengths (an input,
+  // complete before the state kernel started), so this part runs while the
+  // state kernel does.  NS stages in all, pre_b before batch row b (the state
+  // kernel's stage prefix, formed here by the block).
+  int NS, pre_b;
+  if (seq_lens == nullptr) {
+    NS = B * HG * nst;
+    pre_b = b * HG * nst;
+  } else {
+    int sa = 0, sp = 0;
+    for (int i = threadIdx.x; i < B; i += kReduceThreads) {
+      const int c = HG * ((clamp_len(seq_lens, i, N) + kSTok - 1) / kSTok);
+      sa += c;
+      if (i < b) sp += c;
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+      sa += __shfl_xor_sync(0xffffffffu, sa, o);
+      sp += __shfl_xor_sync(0xffffffffu, sp, o);
+    }
+    if (lane == 0) {
+      red[0][warp] = sa;
+      red[1][warp] = sp;
+    }
+    __syncthreads();
+    NS = pre_b = 0;
+#pragma unroll
+    for (int w = 0; w < kReduceThreads / 32; ++w) {
+      NS += red[0][w];
+      pre_b += red[1][w];
+    }
+  }
+  long long r0 = 0;
+  int nrec = 0, R = 1;
+  if (nst > 0) {
+    R = (NS + kRangeStages * P - 1) / (kRangeStages * P) * P;  // num_ranges
+    const int s0 = pre_b + hg * nst;
+    r0 = range_of(NS, R, s0);
+    nrec = (int)(range_of(NS, R, s0 + nst - 1) - r0 + 1);
+  }
+  const bool may_be_empty = NS < R;  // otherwise every range holds a stage
+  const float *rec0 = records + ((size_t)((long long)b * HG + hg + r0) * G + hh) * REC;
+  const size_t rstride = (size_t)G * REC;
+  const int ec = act ? e0 : 0;
+  grid_dep_wait();  // the records come from the state kernel
+  if constexpr (LEAN) grid_dep_launch();
   float M = -INFINITY, l = 0.f;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   if (nst > 0) {
-    // with every sequence N tokens long the prefix is b HG nst: no dependent load
-    int NS, pre_b;
-    if (seq_lens == nullptr) {
-      NS = B * HG * nst;
-      pre_b = b * HG * nst;
-    } else {
-      NS = stage_pre[B];
-      pre_b = stage_pre[b];
-    }
-    const int R = (NS + kRangeStages * P - 1) / (kRangeStages * P) * P;  // num_ranges
-    const int s0 = pre_b + hg * nst;
-    const long long r0 = range_of(NS, R, s0), r1 = range_of(NS, R, s0 + nst - 1);
-    const int nrec = (int)(r1 - r0 + 1);
-    const bool may_be_empty = NS < R;  // otherwise every range holds a stage
-    const float *rec0 = records + ((size_t)((long long)b * HG + hg + r0) * G + hh) * REC;
-    const size_t rstride = (size_t)G * REC;
+    const uint32_t stg0 = smem_u32(&stg[0][threadIdx.x]);
     for (int j0 = 0; j0 < nrec; j0 += 32) {
+      const int nb = min(32, nrec - j0);
+      // one round trip's loads (records k0 .. k0 + CHT - 1 of the batch; past
+      // the batch the index is clamped to a record that exists): the first
+      // SMR into this thread's shared-memory slots, the next CH into v
+      float4 v[CH];
+      auto issue = [&](int k0) {
+        if constexpr (SMR > 0) {
+#pragma unroll
+          for (int k = 0; k < SMR; ++k) {
+            const int kk = k0 + k < nb ? j0 + k0 + k : j0;
+            cp_async_16(stg0 + (uint32_t)(k * kReduceThreads * 16),
+                        rec0 + (size_t)kk * rstride + ec);
+          }
+          cp_async_commit();
+        }
+#pragma unroll
+        for (int k = 0; k < CH; ++k) {
+          const int kk = k0 + SMR + k < nb ? j0 + k0 + SMR + k : j0;
+          v[k] = __ldg((const float4 *)(rec0 + (size_t)kk * rstride + ec));
+        }
+      };
+      // the first loads go out with the (m, l) loads: they do not depend on
+      // the scale factors
+      issue(0);
       const int j = j0 + lane;
       bool has = j < nrec;
       if (has && may_be_empty)  // with fewer stages than ranges some left no record
@@ -921,30 +981,29 @@ __global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
 #pragma unroll
       for (int o = 16; o >= 1; o >>= 1) ls += __shfl_xor_sync(0xffffffffu, ls, o);
       l += ls;
-      const int nb = min(32, nrec - j0);
-      for (int k0 = 0; k0 < nb; k0 += CH) {
-        float skk[CH];  // the chunk's scale factors, from the lanes that hold them
+      auto fma4 = [&](float s4, const float4 &x) {
+        acc.x = fmaf(s4, x.x, acc.x);
+        acc.y = fmaf(s4, x.y, acc.y);
+        acc.z = fmaf(s4, x.z, acc.z);
+        acc.w = fmaf(s4, x.w, acc.w);
+      };
+      for (int k0 = 0; k0 < nb; k0 += CHT) {
+        if (k0 > 0) issue(k0);
+        // in record order; a zero factor marks a record that does not exist
+        // (an empty range, whose slot holds whatever was there) or that
+        // underflowed: skip it
+        if constexpr (SMR > 0) {
+          cp_async_wait_all();  // this thread's own copies: no barrier needed
 #pragma unroll
-        for (int k = 0; k < CH; ++k) skk[k] = __shfl_sync(0xffffffffu, sc, (k0 + k) & 31);
-        // every load of the chunk in flight together: past the batch (or the
-        // state) the index is clamped to a record and element that exist
-        float4 v[CH];
-        const int ec = act ? e0 : 0;
-#pragma unroll
-        for (int k = 0; k < CH; ++k) {
-          const int kk = k0 + k < nb ? j0 + k0 + k : j0;
-          v[k] = __ldg((const float4 *)(rec0 + (size_t)kk * rstride + ec));
+          for (int k = 0; k < SMR; ++k) {
+            const float skk = __shfl_sync(0xffffffffu, sc, (k0 + k) & 31);
+            if (k0 + k < nb && skk != 0.f) fma4(skk, stg[k][threadIdx.x]);
+          }
         }
 #pragma unroll
         for (int k = 0; k < CH; ++k) {
-          // a zero factor marks a record that does not exist (an empty range,
-          // whose slot holds whatever was there) or that underflowed: skip it
-          if (k0 + k < nb && skk[k] != 0.f) {
-            acc.x = fmaf(skk[k], v[k].x, acc.x);
-            acc.y = fmaf(skk[k], v[k].y, acc.y);
-            acc.z = fmaf(skk[k], v[k].z, acc.z);
-            acc.w = fmaf(skk[k], v[k].w, acc.w);
-          }
+          const float skk = __shfl_sync(0xffffffffu, sc, (k0 + SMR + k) & 31);
+          if (k0 + SMR + k < nb && skk != 0.f) fma4(skk, v[k]);
         }
       }
     }
@@ -1643,13 +1702,11 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
                       const float *conv_w, void *ws, float *state, cudaStream_t st,
                       float2 *gate_stats) {
   constexpr int G = kGroupCh / D;
-  const size_t rb = records_bytes(p);
   StateParams sp;
   sp.gate = (const __nv_bfloat16 *)gate;
   sp.conv_w = conv_w;
   sp.seq_lens = p.seq_lens;
   sp.records = (float *)ws;
-  sp.stage_pre = (int32_t *)((char *)ws + rb);
   sp.B = p.B;
   sp.H = p.H;
   sp.N = p.N;
@@ -1674,14 +1731,23 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(p.B * p.H, (F / 4 + kReduceThreads - 1) / kReduceThreads);
   const bool lean = (long long)cfg.gridDim.x * cfg.gridDim.y <= num_sms();
+  if (lean) {  // the SMs keep the state kernel's shared-memory split for the lean blocks
+    static std::once_flag carve;
+    std::call_once(carve, [] {  // a hint: if it is refused, the launch goes on without it
+      if (cudaFuncSetAttribute(tc_reduce_kernel<D, true>,
+                               cudaFuncAttributePreferredSharedMemoryCarveout,
+                               (int)cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+        (void)cudaGetLastError();
+    });
+  }
   cfg.blockDim = dim3(kReduceThreads);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   e = cudaLaunchKernelEx(&cfg, lean ? tc_reduce_kernel<D, true> : tc_reduce_kernel<D, false>,
-                         (const float *)sp.records, (const int32_t *)sp.stage_pre, p.seq_lens,
-                         state, gate_stats, p.B, p.H, p.N, num_sms());
+                         (const float *)sp.records, p.seq_lens, state, gate_stats, p.B, p.H,
+                         p.N, num_sms());
   count_launch();
   return e;
 }
@@ -1749,9 +1815,7 @@ bool tc_supports(const Problem &p) {
   return device_info().sm103 && encode_fn() != nullptr;
 }
 
-size_t tc_workspace_bytes(const Problem &p) {
-  return records_bytes(p) + sizeof(int32_t) * (p.B + 1) + 256;
-}
+size_t tc_workspace_bytes(const Problem &p) { return records_bytes(p) + 256; }
 
 cudaError_t tc_state(const Problem &p, const void *k, const void *v, const void *gate,
                      const float *conv_w, void *ws, float *state, cudaStream_t st,

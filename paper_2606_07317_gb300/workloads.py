@@ -80,6 +80,9 @@ WORKLOADS = {
         Workload("bf16_b4_h8_n8192_d64", 4, 8, 8192, 64, "bf16", 2),
         Workload("bf16_b2_h8_n32768_d64", 2, 8, 32768, 64, "bf16", 3),
         _ragged("bf16_ragged_b32_h8_d128", 32, 8, 128, 4),
+        # a smaller ragged D = 128 batch of the same length distribution, for
+        # profiler captures that must stay within a few GB of device memory
+        _ragged("bf16_ragged_b8_h8_d128", 8, 8, 128, 11),
     ]
 }
 
