@@ -365,7 +365,7 @@ struct StateParams {
   const __nv_bfloat16 *gate;
   const float *conv_w;
   const int32_t *seq_lens;
-  float *records;        // [ranges + sequences][G][D*D + D + 4]: S, z, m, l, 2 pad
+  float *records;        // [ranges + sequences][G][D*D + D + 4]: S as [c / 8][a][c % 8], z, m, l, 2 pad
   int B, H, N, HG;
   uint32_t flags;        // gbla_flags (NO_CONV, NO_GATE)
 };
@@ -741,7 +741,10 @@ __global__ void __launch_bounds__(kSThreads, 1)
           const int cv0 = D * ha + part * CPW;          // first v channel (of the group)
           const uint32_t tl = tmem + ((uint32_t)(32 * q4) << 16) +
                               (uint32_t)(256 * (cv0 / 64) + cv0 % 64);
-          float *dst = p.records + ((size_t)rec * G + ha) * REC + (size_t)d * D + part * CPW;
+          // record layout of S: [c / 8][a][c % 8], so that a warp's stores of
+          // 32 rows x 8 columns are one contiguous kilobyte
+          float *dst = p.records + ((size_t)rec * G + ha) * REC + (size_t)(part * CPW / 8) * (D * 8) +
+                       (size_t)d * 8;
 #pragma unroll
           for (int cb = 0; cb < CPW; cb += 8) {
             float v0[8], v1[8], v2[8], v3[8];
@@ -760,7 +763,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
               o[i] = fmaf(wt.w, v3[i], fmaf(wt.z, v2[i], fmaf(wt.y, v1[i], wt.x * v0[i])));
             }
             if (ok2) {
-              float4 *dq = (float4 *)(dst + cb);
+              float4 *dq = (float4 *)(dst + (size_t)(cb / 8) * (D * 8));
               dq[0] = make_float4(o[0], o[1], o[2], o[3]);
               dq[1] = make_float4(o[4], o[5], o[6], o[7]);
             }
@@ -1012,7 +1015,9 @@ __global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
     gate_stats[bh] = make_float2(M, l);  // every thread of bh holds the same pair
   if (!act) return;
   const float inv = l > 0.f ? 1.f / l : 0.f;
-  *(float4 *)(state + (size_t)bh * F + e0) =
+  // record position e0 of S ([c / 8][a][c % 8]) -> state element a D + c
+  const int se = e0 < D * D ? (e0 % (D * 8)) / 8 * D + e0 / (D * 8) * 8 + e0 % 8 : e0;
+  *(float4 *)(state + (size_t)bh * F + se) =
       make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
 }
 
