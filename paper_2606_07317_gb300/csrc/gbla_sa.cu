@@ -64,6 +64,30 @@ constexpr uint32_t kTmemCols = 512;  // S0 [0,128), S1 [128,256), O [256,320)
 constexpr uint32_t kOCol = 256;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLazy = 8.f;  // rescale only when the maximum grows by more than 2^8
+constexpr int kPolyEvery = 4;  // every fourth pair of exponentials on the FMA pipe
+
+// 2^x for two values on the FMA and integer pipes (no special-function op):
+// x = n + f with n = round(x) (the 1.5 * 2^23 addition leaves n in the low
+// mantissa bits) and f in [-1/2, 1/2]; 2^f by a cubic fitted here to 2^f on
+// [-1/2, 1/2] (least squares on the relative error, reweighted towards its
+// maximum; maximum relative error 7.6e-5, far below the 2^-9 of the bf16
+// rounding every probability gets); n added to the exponent field.  x is
+// clamped at -125 (2^-125 stands in for 0: past-the-end keys meet zeroed V
+// rows, and the sum of P is at least 1).
+__device__ __forceinline__ float2 exp2_poly2(float2 x) {
+  constexpr float kRound = 12582912.f;  // 1.5 * 2^23
+  x = make_float2(fmaxf(x.x, -125.f), fmaxf(x.y, -125.f));
+  const float2 t = __fadd2_rn(x, make_float2(kRound, kRound));
+  const float2 r = __fadd2_rn(t, make_float2(-kRound, -kRound));  // n as a float
+  const float2 f = __ffma2_rn(r, make_float2(-1.f, -1.f), x);        // x - n
+  float2 q = __ffma2_rn(make_float2(0.05517030f, 0.05517030f), f,
+                        make_float2(0.24260803f, 0.24260803f));
+  q = __ffma2_rn(q, f, make_float2(0.69326091f, 0.69326091f));
+  q = __ffma2_rn(q, f, make_float2(0.99992830f, 0.99992830f));
+  // bits(t) << 23 = n << 23 (mod 2^32): the rounding constant's own bits shift out
+  return make_float2(__int_as_float(__float_as_int(q.x) + (__float_as_int(t.x) << 23)),
+                     __int_as_float(__float_as_int(q.y) + (__float_as_int(t.y) << 23)));
+}
 
 struct SaParams {
   const int32_t *seq_lens;
@@ -217,12 +241,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&s_empty[sb]);  // the score buffer may be overwritten
       const int kv_valid = L - j * kKey;           // keys of this block before the end
-      float mb = -INFINITY;
+      if (kv_valid < kKey) {                       // the last block: keys past the end
 #pragma unroll
-      for (int i = 0; i < kKey; ++i) {
-        sv[i] = i < kv_valid ? sv[i] * c : -INFINITY;
-        mb = fmaxf(mb, sv[i]);
+        for (int i = 0; i < kKey; ++i) sv[i] = i < kv_valid ? sv[i] : -INFINITY;
       }
+      float mb = -INFINITY;  // the row maximum of the raw scores, then in log2 units (c > 0)
+#pragma unroll
+      for (int i = 0; i < kKey; i += 2) mb = fmaxf(mb, fmaxf(sv[i], sv[i + 1]));
+      mb *= c;
       // The row maximum grew: rescale O and l (lazily).  TMEM loads and stores
       // are warp-wide, so the whole warp takes the O pass when any lane needs
       // it, with alpha = 1 on the other lanes.
@@ -246,14 +272,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         l_run *= alpha;
       }
       if (grow) m_run = mb;
-      // P = 2^(s - m) (at most 2^8 with the lazy maximum); the sum in fp32
-      float ls = 0.f;
+      // P = 2^(s c - m) (at most 2^8 with the lazy maximum), every kPolyEvery-th
+      // pair by the polynomial, the others by ex2; the sum in fp32
+      float2 ls2 = make_float2(0.f, 0.f);
 #pragma unroll
-      for (int i = 0; i < kKey; ++i) {
-        sv[i] = ex2_approx(sv[i] - m_run);
-        ls += sv[i];
+      for (int i = 0; i < kKey; i += 2) {
+        const float2 x = __ffma2_rn(make_float2(sv[i], sv[i + 1]), make_float2(c, c),
+                                    make_float2(-m_run, -m_run));
+        const float2 e = (i / 2) % kPolyEvery == kPolyEvery - 1
+                             ? exp2_poly2(x)
+                             : make_float2(ex2_approx(x.x), ex2_approx(x.y));
+        sv[i] = e.x;
+        sv[i + 1] = e.y;
+        ls2 = __fadd2_rn(ls2, e);
       }
-      l_run += ls;
+      l_run += ls2.x + ls2.y;
       if (j >= 2 && !mbar_wait(&p_empty[sb], ((j - 2) >> 1) & 1, &ab) && !ab.raised())
         sa_error(16, ab);  // the P buffer is free once the P V of block j - 2 is done
       // row `row` of P: two 64-key K blocks, 16-byte chunks swizzled by the row

@@ -111,6 +111,26 @@ def test_attention_table5_shape_sampled_rows():
     log_stats({"test": "attention_sampled", "shape": [B, N, H], **worst})
 
 
+def test_attention_table5_longest_sampled_rows():
+    """Table 5's longest length (batch 8, 16 heads of 64, L = 32768: 256 query
+    tiles and 256 key blocks per (b, h)), 6 query rows per (batch, head) spread
+    over the sequence, against the oracle row by row over all 32768 keys."""
+    B, N, H = 8, 32768, 16
+    q, k, v, _ = _inputs(B, N, H, seed=9)
+    y = _run(q, k, v, None)
+    rows = np.array([0, 127, 128, 16383, 30001, N - 1])
+    worst = None
+    for b in range(B):
+        kc, vc = to64(k[b]), to64(v[b])
+        qc, yc = to64(q[b, rows]), to64(y[b, rows])
+        for h in range(H):
+            ref, a = oracle.softmax_attention_rows(qc[:, h], kc[:, h], vc[:, h])
+            st = _check(yc[:, h], ref, a)
+            if worst is None or st["worst_excess"] > worst["worst_excess"]:
+                worst = st
+    log_stats({"test": "attention_sampled_32768", "shape": [B, N, H], **worst})
+
+
 def test_attention_dominant_scores_are_stable():
     """Scores far above the rest (row maxima growing block after block) are
     handled by the running maximum: the output is the dominant key's value."""
