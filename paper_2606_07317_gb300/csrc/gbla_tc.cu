@@ -490,6 +490,11 @@ __global__ void __launch_bounds__(kSThreads, 1)
     tma_prefetch_desc(&tm_v);
   }
   __syncthreads();
+  // The grid is launched with programmatic dependent launch: the set-up above
+  // overlaps the end of the kernel before it on the stream, whose results the
+  // inputs may be; nothing is read before that kernel has completed, and the
+  // dependents (the reduction) launch only after this wait.
+  grid_dep_wait();
 
   // Stage prefix over the batch (ragged lengths only; uniform lengths decode
   // by arithmetic, so the first loads go out at once).
@@ -1147,6 +1152,10 @@ __global__ void __launch_bounds__(kRThreads, 1)
   // Everything below may read what earlier work on the stream wrote, unless
   // that work is the state reduction, which only `state` depends on.
   if (!p.wait_late) grid_dep_wait();
+  // The next kernel on the stream may launch now: its CTAs take the SMs as
+  // these leave.  A dependent that reads what this grid writes waits for it
+  // to complete (the state kernel does so before its first read).
+  grid_dep_launch();
   if (warp < 4) {
     prefix_counts(pre, B, tid, 128, 1, s_tot, [&](int b) {
       const int L = clamp_len(p.seq_lens, b, N);
@@ -1725,15 +1734,24 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   if ((e = cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, kSSmemBytes)) !=
       cudaSuccess)
     return e;
-  k1<<<num_sms(), kSThreads, kSSmemBytes, st>>>(sp, tm_k, tm_v);
-  count_launch();
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-
-  constexpr int F = D * D + D;
-  cudaLaunchConfig_t cfg = {};
+  // programmatic dependent launch: the CTAs take the SMs as those of the
+  // kernel before leave, and wait for it (in the kernel) before reading
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t scfg = {};
+  scfg.gridDim = dim3(num_sms());
+  scfg.blockDim = dim3(kSThreads);
+  scfg.dynamicSmemBytes = kSSmemBytes;
+  scfg.stream = st;
+  scfg.attrs = attr;
+  scfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&scfg, k1, sp, tm_k, tm_v);
+  count_launch();
+  if (e != cudaSuccess) return e;
+
+  constexpr int F = D * D + D;
+  cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.B * p.H, (F / 4 + kReduceThreads - 1) / kReduceThreads);
   const bool lean = (long long)cfg.gridDim.x * cfg.gridDim.y <= num_sms();
   if (lean) {  // the SMs keep the state kernel's shared-memory split for the lean blocks
