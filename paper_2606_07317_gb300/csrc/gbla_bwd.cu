@@ -484,14 +484,10 @@ __device__ __forceinline__ void ld4(const __nv_bfloat16 *p, float (&f)[4]) {
   f[2] = __uint_as_float(u.y << 16); f[3] = __uint_as_float(u.y & 0xFFFF0000u);
 }
 // Four channels as loaded (raw), then widened to fp32: the Conv1D backward
-// issues a batch of raw loads before it converts any of them.
+// stages a batch of raw loads in shared memory before it converts any of them.
 template <typename T> struct Raw4;
 template <> struct Raw4<float> { using type = float4; };
 template <> struct Raw4<__nv_bfloat16> { using type = uint2; };
-__device__ __forceinline__ float4 ld4raw(const float *p) { return __ldg((const float4 *)p); }
-__device__ __forceinline__ uint2 ld4raw(const __nv_bfloat16 *p) { return __ldg((const uint2 *)p); }
-__device__ __forceinline__ void zero4raw(float4 &r) { r = make_float4(0.f, 0.f, 0.f, 0.f); }
-__device__ __forceinline__ void zero4raw(uint2 &r) { r = make_uint2(0u, 0u); }
 __device__ __forceinline__ void cvt4raw(const float4 &a, float (&f)[4]) {
   f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
 }
@@ -506,6 +502,29 @@ __device__ __forceinline__ void st4(__nv_bfloat16 *p, const float (&f)[4]) {
   const __nv_bfloat162 a = __floats2bfloat162_rn(f[0], f[1]), b = __floats2bfloat162_rn(f[2], f[3]);
   *(uint2 *)p = make_uint2(*reinterpret_cast<const uint32_t *>(&a),
                            *reinterpret_cast<const uint32_t *>(&b));
+}
+
+// Asynchronous copy of BYTES (8 or 16) global bytes into shared memory; the
+// destination is zero-filled when src_bytes is 0 (src must still be a valid
+// address, and is not read).
+template <int BYTES>
+__device__ __forceinline__ void cp_async_z(uint32_t dst, const void *src, uint32_t src_bytes) {
+  if constexpr (BYTES == 16)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(src_bytes)
+                 : "memory");
+  else
+    asm volatile("cp.async.ca.shared.global [%0], [%1], %2, %3;" ::"r"(dst), "l"(src),
+                 "n"(BYTES), "r"(src_bytes)
+                 : "memory");
+}
+// Steps of the Conv1D backward whose loads are staged together, and the
+// dynamic shared memory of the staging buffers (two batches in flight).
+template <typename T>
+constexpr int conv_batch() { return sizeof(T) == 2 ? 8 : 4; }
+template <typename T>
+constexpr size_t conv_stage_bytes() {
+  return (size_t)2 * 2 * conv_batch<T>() * kNT * sizeof(typename Raw4<T>::type);
 }
 
 template <typename T, int D>
@@ -555,25 +574,47 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
     ldx(ta - 3 + i, xm[i]);
     ldd(ta + i, dm[i]);
   }
-  // U steps at a time: their 2 U loads are issued together (zero outside
-  // [0, L)), then the steps run in order
+  // U steps at a time: their 2 U loads go to shared memory by cp.async (no
+  // registers held while they are in flight), the next batch's copies are
+  // issued before this batch is converted, and each thread reads back only
+  // its own slots (no barrier).  Rows at or past L are zero-filled.
   using Raw = typename Raw4<T>::type;
-  constexpr int U = sizeof(T) == 2 ? 8 : 4;
-  for (int t0 = ta; t0 < tb; t0 += U) {
-    Raw xr[U], dr[U];
+  constexpr int U = conv_batch<T>();
+  constexpr int RB = (int)sizeof(Raw);
+  extern __shared__ __align__(16) uint8_t conv_stage[];
+  // this thread's slot for x (arr 0) or dx~ (arr 1) of step u in batch buffer buf
+  auto slot_off = [&](int buf, int arr, int u) {
+    return (uint32_t)((((buf * 2 + arr) * U + u) * kNT + tid) * RB);
+  };
+  const uint32_t stg0 = (uint32_t)__cvta_generic_to_shared(conv_stage);
+  const int nbat = (tb - ta + U - 1) / U;
+  auto issue = [&](int bt) {
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int tx = t0 + u, td = t0 + u + 3;
-      if (tx < L) xr[u] = ld4raw(x + col + (size_t)tx * rs); else zero4raw(xr[u]);
-      if (td < L) dr[u] = ld4raw(dxs + col + (size_t)td * rs); else zero4raw(dr[u]);
+      const int tx = ta + bt * U + u, td = tx + 3;
+      const bool vx = tx < tb && tx < L, vd = tx < tb && td < L;
+      cp_async_z<RB>(stg0 + slot_off(bt & 1, 0, u), x + col + (vx ? (size_t)tx * rs : 0),
+                     vx ? RB : 0);
+      cp_async_z<RB>(stg0 + slot_off(bt & 1, 1, u), dxs + col + (vd ? (size_t)td * rs : 0),
+                     vd ? RB : 0);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  if (nbat > 0) issue(0);
+  for (int bt = 0; bt < nbat; ++bt) {
+    if (bt + 1 < nbat) {
+      issue(bt + 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-    const int t = t0 + u;
+    const int t = ta + bt * U + u;
     if (t >= tb) break;
     float xc[kConvCh], dn[kConvCh], o[kConvCh];
-    cvt4raw(xr[u], xc);  // x_t
-    cvt4raw(dr[u], dn);  // dx~_{t+3}
+    cvt4raw(*(const Raw *)(conv_stage + slot_off(bt & 1, 0, u)), xc);  // x_t
+    cvt4raw(*(const Raw *)(conv_stage + slot_off(bt & 1, 1, u)), dn);  // dx~_{t+3}
 #pragma unroll
     for (int c = 0; c < kConvCh; ++c) {
       // dx_t = w0 dx~_{t+3} + w1 dx~_{t+2} + w2 dx~_{t+1} + w3 dx~_t
@@ -713,7 +754,11 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
   constexpr int kRuns = kNT / (D / kConvCh);
   const int rl = 64;
   const int nckc = (N + kRuns * rl - 1) / (kRuns * rl);  // Conv1D backward blocks per (b, h)
-  bwd_conv<T, D><<<dim3(nckc, BH, 3), kNT, 0, st>>>(
+  // the staging buffers exceed the default 48 KB of dynamic shared memory
+  if ((e = cudaFuncSetAttribute(bwd_conv<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)conv_stage_bytes<T>())) != cudaSuccess)
+    return e;
+  bwd_conv<T, D><<<dim3(nckc, BH, 3), kNT, conv_stage_bytes<T>(), st>>>(
       (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
       (T *)a.dk, (T *)a.dv, wpart, H, N, nckc, rl);
   count_launch();
