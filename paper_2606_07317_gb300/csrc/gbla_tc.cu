@@ -149,18 +149,27 @@ constexpr int kRQRows = kRTok + 3;              // q tile rows: 3-token conv hal
 
 template <int D>
 struct ReadoutCfg {
-  static constexpr bool QT = D == 64;                     // q through TMA (else 128-bit loads)
+  static constexpr bool QT = D == 64;                     // q through TMA into its own ring
+  // D = 128: no room for a q ring beside [S | z] (N = 144, hi + lo) and the
+  // out_gate stages, so q comes by TMA straight into the A slot (3 rows of
+  // conv history in front) and the producers turn it into phi(Conv1D(q)) in
+  // place; the MMA reads the slot from row 3 on.
+  static constexpr bool QA = D == 128;
   static constexpr int NR = D + 16;                       // MMA N: D columns of S, z, zeros
   static constexpr int KB = D / 64;                       // 64-element K blocks
   static constexpr int NCH = QT ? 4 : 8;                  // channels per producer thread
   static constexpr int TPR = D / NCH;                     // producer threads per token row
   static constexpr int STREAMS = kRProd / TPR;            // producer sub-streams per tile
   static constexpr int TPS = kRTok / STREAMS;             // tokens per sub-stream
-  static constexpr int kABytes = kRTok * D * 2;           // one A tile
+  // one 64-channel block of an A slot: 128 token rows (QA: 131 with the conv
+  // history, rounded up to whole 1024-byte swizzle atoms)
+  static constexpr int kABlk = QA ? (kRQRows * 128 + 1023) / 1024 * 1024 : kRTok * 128;
+  static constexpr int kARow0 = QA ? 3 * 128 : 0;          // byte offset of A row 0 in a block
+  static constexpr int kABytes = KB * kABlk;              // one A slot
   static constexpr int kBBytes = NR * D * 2;              // one of B_hi / B_lo
   static constexpr int kOgStages = D == 128 ? 2 : 4;
   static constexpr int kOgBytes = kRTok * D * 2;
-  static constexpr int kQStages = QT ? 3 : 0;
+  static constexpr int kQStages = QT ? 3 : (QA ? kRAStages : 0);  // QA: one per A slot
   static constexpr int kQTileBytes = kRQRows * 128;                  // one 64-channel block
   static constexpr int kQBytes = (kQTileBytes + 1023) / 1024 * 1024;  // 1024-aligned stride
   static constexpr int kOffA = 0;
@@ -168,7 +177,7 @@ struct ReadoutCfg {
   static constexpr int kOffBlo = kOffBhi + kBBytes;
   static constexpr int kOffOg = kOffBlo + kBBytes;
   static constexpr int kOffQ = kOffOg + kOgStages * kOgBytes;
-  static constexpr int kOffPre = kOffQ + kQStages * kQBytes;      // int [kMaxBatch + 1]
+  static constexpr int kOffPre = kOffQ + (QT ? kQStages * kQBytes : 0);  // int [kMaxBatch + 1]
   static constexpr int kOffSs = kOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;  // float [256]
   static constexpr int kOffW = kOffSs + kREpi * 4;  // float [D]: norm weights of the head
   static constexpr int kOffBar = kOffW + D * 4;
@@ -1192,12 +1201,14 @@ __global__ void __launch_bounds__(kRThreads, 1)
     const int row0 = stream * TPS;  // first tile row of this sub-stream
     // swizzled offsets of this thread's 16-byte pieces of A rows row0 + u
     // (the TMA q path uses one 8-row atom per sub-stream and needs none)
+    // (QA: offsets of the slot rows row0 + 3 + u, which hold the raw q of this
+    // sub-stream's tokens and receive A rows row0 + u in place)
     uint32_t aoff[C::QT ? 1 : TPS];
     if constexpr (!C::QT) {
 #pragma unroll
       for (int u = 0; u < TPS; ++u) {
-        const int row = row0 + u;
-        aoff[u] = kb * (kRTok * 128) + (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
+        const int row = row0 + u + (C::QA ? 3 : 0);
+        aoff[u] = kb * C::kABlk + (row >> 3) * 1024 + (row & 7) * 128 + ((cc ^ (row & 7)) << 4);
       }
     }
     // TMA q path: q tile row j holds token r0 - 3 + j; this thread reads rows
@@ -1227,10 +1238,31 @@ __global__ void __launch_bounds__(kRThreads, 1)
         cur_h = h;
       }
       const int sa = li & 1;
-      if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab) && !ab.raised())
-        report_error(32, ab);
+      if constexpr (C::QA) {  // the raw q tile has landed in the slot (freed by the MMA before)
+        if (!mbar_wait(&q_full[sa], (li >> 1) & 1, &ab) && !ab.raised()) report_error(32, ab);
+      } else {
+        if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab) && !ab.raised())
+          report_error(32, ab);
+      }
       const uint32_t abase = smem_u32(smem + C::kOffA + sa * C::kABytes);
-      if constexpr (C::QT) {
+      if constexpr (C::QA) {
+        // slot row j holds token r0 - 3 + j; this thread reads rows row0 .. row0
+        // + 10 of its 8 channels and rewrites rows row0 + 3 .. row0 + 10 (A rows
+        // row0 .. row0 + 7).  The 3 history rows are read before the producers'
+        // barrier, since the sub-stream before rewrites them; each other row is
+        // read by its own thread just before it rewrites it.
+        float xm[3][8];
+#pragma unroll
+        for (int u = 0; u < 3; ++u) {
+          const int row = row0 + u;
+          unpack8(lds_v4(abase + kb * C::kABlk + row * 128 + ((cc ^ (row & 7)) << 4)), xm[u]);
+        }
+        named_barrier(2, kRProd);
+#pragma unroll
+        for (int g4 = 0; g4 < TPS; g4 += 4)
+          readout_rows4(wq, xm, [&](int u) { return lds_v4(abase + aoff[g4 + u]); }, abase,
+                        aoff + g4);
+      } else if constexpr (C::QT) {
         // q tile from TMA (128-byte swizzle); rows row0 .. row0 + 10 hold this
         // sub-stream's 3 history tokens and its 8 tokens
         const int sq = li % QS;
@@ -1248,26 +1280,6 @@ __global__ void __launch_bounds__(kRThreads, 1)
           const float2 p01 = phi2_log2(conv_rows_n(wq, x, u, 0));
           const float2 p23 = phi2_log2(conv_rows_n(wq, x, u, 2));
           sts_v2(at + u * 128 + ((cc ^ u) << 4), f2_to_bf2(p01.x, p01.y), f2_to_bf2(p23.x, p23.y));
-        }
-      } else {
-        float xm[3][8];
-        const size_t rs = (size_t)H * D;
-        const __nv_bfloat16 *qp = p.q + ((size_t)b * N * H + h) * D + 8 * c;
-        const int ts = r0 + row0;        // first token of this sub-stream
-        const int tmax = r0 + nrow - 1;  // last valid token of the tile
-        auto ld = [&](int t) {
-          return t < 0 ? make_uint4(0, 0, 0, 0) : ldg_nc_v4(qp + (size_t)min(t, tmax) * rs);
-        };
-        uint4 raw[4];
-#pragma unroll
-        for (int u = 0; u < 3; ++u) raw[u] = ld(ts - 3 + u);
-#pragma unroll
-        for (int u = 0; u < 3; ++u) unpack8(raw[u], xm[u]);
-#pragma unroll
-        for (int g4 = 0; g4 < TPS; g4 += 4) {
-#pragma unroll
-          for (int u = 0; u < 4; ++u) raw[u] = ld(ts + g4 + u);
-          readout_rows4(wq, xm, [&](int u) { return raw[u]; }, abase, aoff + g4);
         }
       }
       fence_proxy_async_smem();
@@ -1538,7 +1550,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         for (int kbk = 0; kbk < C::KB; ++kbk)
 #pragma unroll
           for (int k16 = 0; k16 < 4; ++k16) {
-            const uint32_t ao = kbk * (kRTok * 128) + k16 * 32;
+            const uint32_t ao = kbk * C::kABlk + C::kARow0 + k16 * 32;
             const uint32_t bo = kbk * (NR * 128) + k16 * 32;
             const uint64_t ad = sw128_desc(abase + ao, 16, 1024);
             mma_bf16(dacc, ad, sw128_desc(bhi + bo, 16, 1024), C::kIdesc, (kbk | k16) != 0);
@@ -1577,20 +1589,27 @@ __global__ void __launch_bounds__(kRThreads, 1)
         for (int kbo = 0; kbo < C::KB; ++kbo)
           tma_load_4d_hint(dst + kbo * (kRTok * 128), &tm_og, &og_full[so], kbo * 64, h, r0, b,
                            pol);
-        if constexpr (!C::QT) {  // q is read with plain loads: warm L2 two tiles ahead
-          if (ii + 2 < i1) {
-            TileCursor nx = tc0;
-            tile_next(nx, p.seq_lens, B, H, N);
-            tile_next(nx, p.seq_lens, B, H, N);
-#pragma unroll
-            for (int kbo = 0; kbo < C::KB; ++kbo)
-              tma_prefetch_l2_4d(&tm_q, kbo * 64, nx.h, nx.r0, nx.b);
-          }
-        }
       }
     }
   } else {
     // ------------------------------------------------------------ TMA: q
+    if (lane == 0 && C::QA) {  // into the A slot, once the MMA has read it
+      const uint64_t pol = l2_policy_evict_first();
+      for (long long ii = i0; ii < i1; ++ii) {
+        int b, h, r0, nrow;
+        tile_of(ii, b, h, r0, nrow);
+        const int li = (int)(ii - i0), sa = li & 1;
+        if (!mbar_wait(&a_empty[sa], ((li >> 1) & 1) ^ 1, &ab)) {
+          if (!ab.raised()) report_error(1024, ab);
+          break;
+        }
+        mbar_arrive_expect_tx(&q_full[sa], C::KB * C::kQTileBytes);
+#pragma unroll
+        for (int kbo = 0; kbo < C::KB; ++kbo)
+          tma_load_4d_hint(smem + C::kOffA + sa * C::kABytes + kbo * C::kABlk, &tm_q, &q_full[sa],
+                           kbo * 64, h, r0 - 3, b, pol);
+      }
+    }
     if (lane == 0 && C::QT) {
       const uint64_t pol = l2_policy_evict_first();  // read once (3 halo rows aside)
       for (long long ii = i0; ii < i1; ++ii) {
@@ -1784,7 +1803,7 @@ cudaError_t run_readout(const Problem &p, const void *q, const void *og, const f
   cudaError_t e = make_bnhd_map(&tm_og, og, p.B, p.N, p.H, D, kRTok);
   if (e != cudaSuccess) return e;
   if ((e = make_bnhd_map(&tm_o, o, p.B, p.N, p.H, D, 32)) != cudaSuccess) return e;  // a quarter
-  if ((e = make_bnhd_map(&tm_q, q, p.B, p.N, p.H, D, C::QT ? kRQRows : kRTok)) != cudaSuccess)
+  if ((e = make_bnhd_map(&tm_q, q, p.B, p.N, p.H, D, kRQRows)) != cudaSuccess)
     return e;
   ReadoutParams rp;
   rp.q = (const __nv_bfloat16 *)q;
