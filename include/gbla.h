@@ -143,8 +143,8 @@ gbla_status gbla_forward_f32out(const void *q, const void *k, const void *v,
                                 gbla_stream_t stream);
 
 /*
- * gbla_backward -- gradients of sum(dy * o) of the layer core (full core, no
- * ablation) with respect to every input: the chain rule through the steps of
+ * gbla_backward -- gradients of sum(dy * o) of the layer core (the full core;
+ * gbla_backward_variant below takes the ablations) with respect to every input: the chain rule through the steps of
  * Sec. 2.1 in reverse (gated RMSNorm, readout, state, key-gate softmax, phi,
  * Conv1D).  Used to train the model end to end (the paper's training-speed
  * comparison, Sec. 3).
@@ -170,6 +170,27 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
                           void *dv, void *dgate, void *dout_gate, float *dconv_w,
                           float *dnorm_w, int B, int H, int N, int D, gbla_dtype dtype,
                           gbla_stream_t stream);
+
+/*
+ * gbla_backward_variant -- gbla_backward of an ablation of Table 4 (`flags`:
+ * gbla_flags OR-ed, as gbla_forward_variant; 0 is gbla_backward): the
+ * gradients of sum(dy * o) with o the variant's output.  The parameters a
+ * variant does not use get zero gradients: dconv_w under GBLA_FLAG_NO_CONV,
+ * dgate (every row) under GBLA_FLAG_NO_GATE, dout_gate and dnorm_w under
+ * GBLA_FLAG_NO_NORM.  Variants run the token passes on CUDA cores (fp32
+ * arithmetic for every dtype and D); the identity Conv1D and the uniform gate
+ * are computed as the full core on identity taps and all-zero gate logits
+ * (scratch copies made by the call).  Flags outside GBLA_FLAG_BLA return
+ * GBLA_ERR_INVALID_ARG; arguments, limits, errors and asynchrony otherwise
+ * as gbla_backward.
+ */
+gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
+                                  const void *gate, const void *out_gate,
+                                  const float *conv_w, const float *norm_w,
+                                  const int32_t *seq_lens, const void *dy, void *dq, void *dk,
+                                  void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                  float *dnorm_w, int B, int H, int N, int D,
+                                  gbla_dtype dtype, uint32_t flags, gbla_stream_t stream);
 
 /*
  * gbla_project -- the layer front end: Sec. 2.1 item 1 (X~ = Conv1D(X), then

@@ -333,6 +333,19 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
                           void *dv, void *dgate, void *dout_gate, float *dconv_w,
                           float *dnorm_w, int B, int H, int N, int D, gbla_dtype dtype,
                           gbla_stream_t stream) {
+  return gbla_backward_variant(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, dq, dk,
+                               dv, dgate, dout_gate, dconv_w, dnorm_w, B, H, N, D, dtype, 0u,
+                               stream);
+}
+
+gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
+                                  const void *gate, const void *out_gate,
+                                  const float *conv_w, const float *norm_w,
+                                  const int32_t *seq_lens, const void *dy, void *dq, void *dk,
+                                  void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                  float *dnorm_w, int B, int H, int N, int D,
+                                  gbla_dtype dtype, uint32_t flags, gbla_stream_t stream) {
+  if (flags & ~(uint32_t)GBLA_FLAG_BLA) return GBLA_ERR_INVALID_ARG;
   bool empty = false;
   gbla_status s = check_dims(B, H, N, D, dtype, &empty);
   if (s != GBLA_OK) return s;
@@ -369,17 +382,47 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
   bool tc = use_tc(p, GBLA_ALGO_AUTO, &s);
   if (s != GBLA_OK) return s;
   const BwdLayout lay = bwd_layout(p);
+  // Ablations (Table 4): the identity Conv1D and the uniform key gate are the
+  // full core on substituted inputs -- taps (0, 0, 0, 1) on every channel,
+  // and all-zero gate logits, whose softmax over the valid positions is
+  // 1 / L_b -- so every kernel runs as is on them; the gradients of the
+  // parameters a variant does not use are zero.  Without the gated RMSNorm
+  // the query pass takes dO = dy (its CUDA-core build; the tensor-core token
+  // passes serve the full core only).
+  const size_t tap_floats = (flags & GBLA_FLAG_NO_CONV) ? (size_t)3 * H * D * kConvW : 0;
+  const size_t zgate_bytes = (flags & GBLA_FLAG_NO_GATE) ? gbytes : 0;
+  const size_t sub_off = round_up(sizeof(float) * lay.total, 256);
   Scratch scr;
-  if ((s = scr.alloc(sizeof(float) * lay.total, st)) != GBLA_OK) return s;
+  if ((s = scr.alloc(sub_off + round_up(sizeof(float) * tap_floats, 256) + zgate_bytes, st)) !=
+      GBLA_OK)
+    return s;
   float *base = (float *)scr.ptr;
+  const float *cw = conv_w;
+  const void *gt = gate;
+  if (tap_floats) {
+    float *taps = (float *)((char *)scr.ptr + sub_off);
+    if (fill_identity_taps(taps, 3 * H * D, st) != cudaSuccess) return GBLA_ERR_CUDA;
+    cw = taps;
+  }
+  if (zgate_bytes) {
+    void *zg = (char *)scr.ptr + sub_off + round_up(sizeof(float) * tap_floats, 256);
+    if (cudaMemsetAsync(zg, 0, zgate_bytes, st) != cudaSuccess) return GBLA_ERR_CUDA;
+    gt = zg;
+  }
   // the forward state S, z through the forward's own state path, which on
   // tensor cores also yields the gate statistics the backward needs
-  if ((s = run_state(p, tc, k, v, gate, conv_w, base + lay.state, st,
+  if ((s = run_state(p, tc, k, v, gt, cw, base + lay.state, st,
                      tc ? (float2 *)(base + lay.stats) : nullptr)) != GBLA_OK)
     return s;
-  BwdArgs a{q, k, v, gate, out_gate, dy, conv_w, norm_w, dq, dk, dv, dgate, dout_gate,
+  BwdArgs a{q, k, v, gt, out_gate, dy, cw, norm_w, dq, dk, dv, dgate, dout_gate,
             dconv_w, dnorm_w};
-  return from_cuda(bwd_run(p, a, base, tc, st));
+  Problem pb = p;
+  pb.flags = flags;
+  if ((s = from_cuda(bwd_run(pb, a, base, tc, st))) != GBLA_OK) return s;
+  if (((flags & GBLA_FLAG_NO_CONV) && cudaMemsetAsync(dconv_w, 0, wbytes, st) != cudaSuccess) ||
+      ((flags & GBLA_FLAG_NO_GATE) && cudaMemsetAsync(dgate, 0, gbytes, st) != cudaSuccess))
+    return from_cuda(cudaGetLastError());
+  return GBLA_OK;
 }
 
 // Validation shared by gbla_project and gbla_layer_forward.

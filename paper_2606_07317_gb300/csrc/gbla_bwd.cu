@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(kNT) bwd_query(
     const float *__restrict__ conv_w, const float *__restrict__ norm_w,
     const float *__restrict__ state, const int32_t *__restrict__ seq_lens, float eps,
     T *__restrict__ dog, T *__restrict__ dqt, float *__restrict__ part, int H, int N,
-    int nck) {
+    int nck, int no_norm) {
   constexpr int F = D * D + D;
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;
   constexpr int RB = D / 16;  // this thread's RB x RB block of dS (16 x 16 threads)
@@ -276,9 +276,9 @@ __global__ void __launch_bounds__(kNT) bwd_query(
       const float sg = 1.f / (1.f + expf(-ogv[u])), si = ogv[u] * sg;
       if (t < t1) {
         const size_t row = (((size_t)b * N + t) * H + h) * D + c;
-        stf(dog, row, dyv[u] * O[u] * r[u] * nw * sg * (1.f + ogv[u] * (1.f - sg)));
+        stf(dog, row, no_norm ? 0.f : dyv[u] * O[u] * r[u] * nw * sg * (1.f + ogv[u] * (1.f - sg)));
       }
-      dnw = fmaf(dyv[u] * O[u], r[u] * si, dnw);
+      if (!no_norm) dnw = fmaf(dyv[u] * O[u], r[u] * si, dnw);
       uu[u] = dyv[u] * nw * si;
       x[u] = uu[u] * O[u];
     }
@@ -286,7 +286,8 @@ __global__ void __launch_bounds__(kNT) bwd_query(
     float dO[TPT];
 #pragma unroll
     for (int u = 0; u < TPT; ++u) {
-      dO[u] = r[u] * uu[u] - (r[u] * r[u] * r[u] / (float)D) * O[u] * x[u];
+      // without the gated RMSNorm (ablation) o = O, so dO = dy
+      dO[u] = no_norm ? dyv[u] : r[u] * uu[u] - (r[u] * r[u] * r[u] / (float)D) * O[u] * x[u];
       x[u] = dO[u] * O[u];
     }
     chan_sum<D, TPT>(x, red);  // dO . O
@@ -726,7 +727,8 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
       return e;
     kq<<<dim3(nck, BH), kNT, smq, st>>>((const T *)a.q, (const T *)a.out_gate, (const T *)a.dy,
                                         a.conv_w, a.norm_w, state, p.seq_lens, kRmsEps,
-                                        (T *)a.dout_gate, dxt, qpart, H, N, nck);
+                                        (T *)a.dout_gate, dxt, qpart, H, N, nck,
+                                        (p.flags & GBLA_FLAG_NO_NORM) ? 1 : 0);
     count_launch();
   }
   constexpr int F = D * D + D;
@@ -787,6 +789,21 @@ BwdLayout bwd_layout(const Problem &p) {
   l.wpart = up(l.dxt + 3 * BH * (size_t)p.N * D);
   l.total = up(l.wpart + 3 * BH * nck * D * kConvW);
   return l;
+}
+
+namespace {
+// Taps (0, 0, 0, 1) on n channels: the identity Conv1D (tap 3 on the current token).
+__global__ void __launch_bounds__(256) identity_taps(float4 *__restrict__ taps, int n) {
+  const int i = blockIdx.x * 256 + threadIdx.x;
+  if (i < n) taps[i] = make_float4(0.f, 0.f, 0.f, 1.f);
+}
+}  // namespace
+
+cudaError_t fill_identity_taps(float *taps, int n, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  identity_taps<<<(n + 255) / 256, 256, 0, st>>>((float4 *)taps, n);
+  count_launch();
+  return cudaGetLastError();
 }
 
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,

@@ -87,6 +87,10 @@ struct BwdLayout {
   size_t state, stats, gpart, qpart, red, cpart, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
+// Taps (0, 0, 0, 1) for n channels (the identity Conv1D of the ablations), [n][4].
+cudaError_t fill_identity_taps(float *taps, int n, cudaStream_t st);
+// p.flags selects an ablation (the CUDA-core token passes; the caller
+// substitutes identity taps and zero gate logits, see gbla_backward_variant).
 cudaError_t bwd_run(const Problem &p, const BwdArgs &a, float *scratch, bool stats_ready,
                     cudaStream_t st);
 // Key pass on tensor cores (gbla_bwd_tc.cu): bf16, D = 64, sm_103.  Writes the

@@ -24,7 +24,7 @@ FLAG_BLA = FLAG_NO_CONV | FLAG_NO_GATE | FLAG_NO_NORM
 CONV_WIDTH = 4
 
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_forward_f32out",
-            "gbla_backward",
+            "gbla_backward", "gbla_backward_variant",
             "gbla_state",
             "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
@@ -74,6 +74,8 @@ def load(path: str | None = None):
         lib.gbla_forward_f32out.restype = _i
         lib.gbla_backward.argtypes = [_vp] * 16 + [_i] * 5 + [_vp]
         lib.gbla_backward.restype = _i
+        lib.gbla_backward_variant.argtypes = [_vp] * 16 + [_i] * 5 + [ctypes.c_uint32, _vp]
+        lib.gbla_backward_variant.restype = _i
         lib.gbla_project.argtypes = [_vp] * 9 + [_i] * 6 + [_vp]
         lib.gbla_project.restype = _i
         lib.gbla_layer_forward.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
@@ -216,20 +218,26 @@ def forward_f32out(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=N
     return out
 
 
-def backward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, stream=None) -> dict:
+def backward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, stream=None,
+             flags: int = 0) -> dict:
     """Gradients of sum(dy * o) (gbla_backward): dq, dk, dv, dout_gate like q; dgate like
-    gate; dconv_w [3, H, D, W] and dnorm_w [H, D] fp32.  Rows past seq_lens are 0."""
+    gate; dconv_w [3, H, D, W] and dnorm_w [H, D] fp32.  Rows past seq_lens are 0.
+    `flags` (FLAG_*) selects an ablation (gbla_backward_variant); 0 is the full core."""
     B, H, N, D = _bhnd(q)
     g = dict(dq=torch.empty_like(q), dk=torch.empty_like(q), dv=torch.empty_like(q),
              dgate=torch.empty_like(gate), dout_gate=torch.empty_like(q),
              dconv_w=torch.empty_like(conv_w, dtype=torch.float32),
              dnorm_w=torch.empty_like(norm_w, dtype=torch.float32))
-    st = load().gbla_backward(
-        _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w), _ptr(norm_w),
-        _ptr(seq_lens), _ptr(dy), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]),
-        _ptr(g["dgate"]), _ptr(g["dout_gate"]), _ptr(g["dconv_w"]), _ptr(g["dnorm_w"]),
-        B, H, N, D, _dtype_code(q), _stream(stream))
-    _check(st, "gbla_backward")
+    args = (_ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(out_gate), _ptr(conv_w), _ptr(norm_w),
+            _ptr(seq_lens), _ptr(dy), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]),
+            _ptr(g["dgate"]), _ptr(g["dout_gate"]), _ptr(g["dconv_w"]), _ptr(g["dnorm_w"]),
+            B, H, N, D, _dtype_code(q))
+    if flags:
+        st = load().gbla_backward_variant(*args, int(flags), _stream(stream))
+        _check(st, "gbla_backward_variant")
+    else:
+        st = load().gbla_backward(*args, _stream(stream))
+        _check(st, "gbla_backward")
     return g
 
 

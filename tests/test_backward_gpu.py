@@ -43,17 +43,17 @@ def _dy(inp, seed):
     return torch.randn(inp["q"].shape, generator=g, device="cuda").to(inp["q"].dtype)
 
 
-def _oracle(inp, dy):
+def _oracle(inp, dy, flags=0):
     sl = inp["seq_lens"].cpu().numpy() if inp["seq_lens"] is not None else None
     return oracle.gbla_backward(
         _to64(inp["q"]), _to64(inp["k"]), _to64(inp["v"]), _to64(inp["gate"]),
         _to64(inp["out_gate"]), _to64(inp["conv_w"]), _to64(inp["norm_w"]), _to64(dy),
-        seq_lens=sl, scales=True, n_threads=8)
+        seq_lens=sl, flags=flags, scales=True, n_threads=8)
 
 
-def _run(inp, dy):
+def _run(inp, dy, flags=0):
     return gbla.backward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"],
-                         inp["conv_w"], inp["norm_w"], inp["seq_lens"], dy)
+                         inp["conv_w"], inp["norm_w"], inp["seq_lens"], dy, flags=flags)
 
 
 BOUNDS = {"bf16": (2.0 ** -7, 2.0 ** -6), "fp32": (2.0 ** -11, 2.0 ** -16)}
@@ -164,3 +164,33 @@ def test_backward_rejects_aliasing():
                            p(dq), p(dq), p(others[1]), p(dgate), p(others[2]), p(dcw), p(dnw),
                            B, H, N, D, 1, None)
     assert st == 1
+
+
+@pytest.mark.parametrize("flags", [1, 2, 4, 3, 5, 6, 7])
+@pytest.mark.parametrize("dtype,D", [("bf16", 64), ("fp32", 32)])
+def test_backward_ablations(flags, dtype, D):
+    """The ablations of Table 4 through gbla_backward_variant, against the
+    oracle's backward with the same flags (pinned by finite differences and by
+    autograd for these flag sets), under the same bounds; the gradients of the
+    parameters a variant does not use are exactly zero."""
+    w = custom(B=2, H=2, N=300, D=D, dtype=dtype, seed=41, seq_lens=[300, 77])
+    inp = make_inputs(w, "cuda")
+    dy = _dy(inp, 42)
+    got = _run(inp, dy, flags)
+    if flags & gbla.FLAG_NO_CONV:
+        assert torch.all(got["dconv_w"] == 0)
+    if flags & gbla.FLAG_NO_GATE:
+        assert torch.all(got["dgate"] == 0)
+    if flags & gbla.FLAG_NO_NORM:
+        assert torch.all(got["dout_gate"] == 0) and torch.all(got["dnorm_w"] == 0)
+    for n in ("dq", "dk", "dv", "dout_gate"):
+        assert torch.all(got[n][1, 77:] == 0), n
+    _check(got, _oracle(inp, dy, flags), dtype, f"_flags{flags}_D{D}")
+
+
+def test_backward_variant_rejects_unknown_flags():
+    w = custom(B=1, H=2, N=64, D=64, dtype="bf16", seed=43)
+    inp = make_inputs(w, "cuda")
+    dy = _dy(inp, 44)
+    with pytest.raises(gbla.GblaError):
+        _run(inp, dy, 8)
