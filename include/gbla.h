@@ -273,6 +273,40 @@ gbla_status gbla_state(const void *k, const void *v, const void *gate,
                        gbla_dtype dtype, gbla_algo algo, gbla_stream_t stream);
 
 /*
+ * gbla_state_stats -- gbla_state plus the key gate's softmax statistics of
+ * each sequence (Sec. 2.1 item 2): stats [B, H, 2] fp32 receives (m, l), m the
+ * largest gate logit over the valid positions t < L_b and l = sum over them of
+ * exp(logit - m); an empty sequence gives (-inf, 0) and a zero state.  These
+ * are what combining the states of disjoint token segments of a sequence
+ * needs (gbla_combine_states).  A logit of -inf gives its token weight 0, so a
+ * segment may carry conv-history rows in front of its own tokens with -inf
+ * logits.  Arguments, limits and errors as gbla_state; `stats` must not
+ * overlap any input or `state`.
+ */
+gbla_status gbla_state_stats(const void *k, const void *v, const void *gate,
+                             const float *conv_w, const int32_t *seq_lens, float *state,
+                             float *stats, int B, int H, int N, int D, gbla_dtype dtype,
+                             gbla_algo algo, gbla_stream_t stream);
+
+/*
+ * gbla_combine_states -- the state of whole sequences from the states of P
+ * disjoint token segments of them (a sequence split across devices; Sec. 2.1
+ * item 2, the softmax-weighted sums split over the segments):
+ *   M = max_p m_p,  w_p = l_p exp(m_p - M),  S = sum_p w_p S_p / sum_p w_p,
+ * z likewise, sums in segment order p = 0 .. P-1 (deterministic); segments
+ * with l_p = 0 weigh 0.
+ *   states    [P, B, H, D*D + D] fp32: gbla_state_stats of each segment.
+ *   stats     [P, B, H, 2] fp32:       their (m, l).
+ *   state     [B, H, D*D + D] fp32:    output, as gbla_state of the whole.
+ *   out_stats [B, H, 2] fp32:          output (M, sum_p w_p).
+ * 1 <= P <= 1024, D in {32, 64, 128} (GBLA_ERR_INVALID_ARG / _UNSUPPORTED);
+ * device pointers, 16-byte aligned, outputs not overlapping the inputs or
+ * each other.  Asynchronous on `stream`; allocates nothing.
+ */
+gbla_status gbla_combine_states(const float *states, const float *stats, int P, float *state,
+                                float *out_stats, int B, int H, int D, gbla_stream_t stream);
+
+/*
  * gbla_readout -- the per-token part: Conv1D of q, phi, O_i = phi(q~_i)^T S /
  * phi(q~_i)^T z (Sec. 2.1 item 2) and the gated RMSNorm (Sec. 2.1 item 3),
  * from a state laid out as gbla_state writes it.  Any positive common scale

@@ -21,7 +21,7 @@ LIB_PATH = os.path.join(LIB_DIR, "libgbla.so")
 OBJ_DIR = os.path.join(PKG, "_build")
 
 SOURCES = ["gbla_api.cu", "gbla_simt.cu", "gbla_tc.cu", "gbla_bwd.cu", "gbla_bwd_tc.cu",
-           "gbla_project.cu", "gbla_static_scratch.cu", "gbla_sa.cu"]
+           "gbla_project.cu", "gbla_static_scratch.cu", "gbla_sa.cu", "gbla_seqsplit.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -233,6 +233,57 @@ gbla_status gbla_state(const void *k, const void *v, const void *gate,
   return run_state(p, tc, k, v, gate, conv_w, state, (cudaStream_t)stream);
 }
 
+gbla_status gbla_state_stats(const void *k, const void *v, const void *gate,
+                             const float *conv_w, const int32_t *seq_lens, float *state,
+                             float *stats, int B, int H, int N, int D, gbla_dtype dtype,
+                             gbla_algo algo, gbla_stream_t stream) {
+  bool empty = false;
+  gbla_status s = check_dims(B, H, N, D, dtype, &empty);
+  if (s != GBLA_OK || empty) return s;
+  if ((s = check_ptrs({k, v, gate, conv_w, state, stats})) != GBLA_OK) return s;
+  if ((s = check_seq_lens(seq_lens)) != GBLA_OK) return s;
+  const size_t in_bytes = (size_t)B * N * H * D * elem_bytes(dtype);
+  const Range out = range_of(state, sizeof(float) * state_floats(D) * B * H);
+  const Range outs = range_of(stats, sizeof(float) * 2 * B * H);
+  for (const Range &o : {out, outs})
+    if (overlap(o, range_of(k, in_bytes)) || overlap(o, range_of(v, in_bytes)) ||
+        overlap(o, range_of(gate, (size_t)B * N * H * elem_bytes(dtype))) ||
+        overlap(o, range_of(conv_w, sizeof(float) * 3 * H * D * kConvW)) ||
+        (seq_lens && overlap(o, range_of(seq_lens, sizeof(int32_t) * B))))
+      return GBLA_ERR_INVALID_ARG;
+  if (overlap(out, outs)) return GBLA_ERR_INVALID_ARG;
+  Problem p{B, H, N, D, dtype, seq_lens};
+  bool tc = use_tc(p, algo, &s);
+  if (s != GBLA_OK) return s;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (tc)  // the tensor-core reduction writes the statistics as it combines the records
+    return run_state(p, tc, k, v, gate, conv_w, state, st, (float2 *)stats);
+  if ((s = run_state(p, tc, k, v, gate, conv_w, state, st)) != GBLA_OK) return s;
+  Scratch part;
+  if ((s = part.alloc(sizeof(float) * gate_stats_part_floats(p), st)) != GBLA_OK) return s;
+  return from_cuda(gate_stats(p, gate, (float2 *)part.ptr, (float2 *)stats, st));
+}
+
+gbla_status gbla_combine_states(const float *states, const float *stats, int P, float *state,
+                                float *out_stats, int B, int H, int D, gbla_stream_t stream) {
+  if (P <= 0 || P > 1024 || B < 0 || H < 0) return GBLA_ERR_INVALID_ARG;
+  if (D != 32 && D != 64 && D != 128) return GBLA_ERR_UNSUPPORTED;
+  if ((long long)B * H == 0) return GBLA_OK;
+  gbla_status s = check_ptrs({states, stats, state, out_stats});
+  if (s != GBLA_OK) return s;
+  const size_t BH = (size_t)B * H;
+  const Range ins[2] = {range_of(states, sizeof(float) * state_floats(D) * BH * P),
+                        range_of(stats, sizeof(float) * 2 * BH * P)};
+  const Range outs[2] = {range_of(state, sizeof(float) * state_floats(D) * BH),
+                         range_of(out_stats, sizeof(float) * 2 * BH)};
+  for (const Range &o : outs)
+    for (const Range &i : ins)
+      if (overlap(o, i)) return GBLA_ERR_INVALID_ARG;
+  if (overlap(outs[0], outs[1])) return GBLA_ERR_INVALID_ARG;
+  return from_cuda(combine_states(states, (const float2 *)stats, P, (int)BH, D, state,
+                                  (float2 *)out_stats, (cudaStream_t)stream));
+}
+
 gbla_status gbla_readout(const void *q, const void *out_gate, const float *conv_w,
                          const float *norm_w, const int32_t *seq_lens,
                          const float *state, void *o, int B, int H, int N, int D,

@@ -791,6 +791,21 @@ BwdLayout bwd_layout(const Problem &p) {
   return l;
 }
 
+cudaError_t gate_stats(const Problem &p, const void *gate, float2 *part, float2 *stats,
+                       cudaStream_t st) {
+  const int BH = p.B * p.H;
+  if (p.dtype == GBLA_BF16)
+    bwd_gate_split<__nv_bfloat16><<<dim3(BH, kGateSplits), 256, 0, st>>>(
+        (const __nv_bfloat16 *)gate, p.seq_lens, part, p.H, p.N);
+  else
+    bwd_gate_split<float><<<dim3(BH, kGateSplits), 256, 0, st>>>((const float *)gate, p.seq_lens,
+                                                                 part, p.H, p.N);
+  bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(part, stats, BH);
+  count_launch(2);
+  return cudaGetLastError();
+}
+size_t gate_stats_part_floats(const Problem &p) { return (size_t)2 * p.B * p.H * kGateSplits; }
+
 namespace {
 // Taps (0, 0, 0, 1) on n channels: the identity Conv1D (tap 3 on the current token).
 __global__ void __launch_bounds__(256) identity_taps(float4 *__restrict__ taps, int n) {

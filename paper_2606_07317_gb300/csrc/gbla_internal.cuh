@@ -87,6 +87,15 @@ struct BwdLayout {
   size_t state, stats, gpart, qpart, red, cpart, dxt, wpart, total;
 };
 BwdLayout bwd_layout(const Problem &p);
+// The key gate's softmax statistics per (b, h) on CUDA cores: (max of the
+// logits, sum of exp(logit - max)) over the valid positions, (-inf, 0) for an
+// empty sequence.  `part` holds gate_stats_part_floats(p) floats of scratch.
+cudaError_t gate_stats(const Problem &p, const void *gate, float2 *part, float2 *stats,
+                       cudaStream_t st);
+size_t gate_stats_part_floats(const Problem &p);
+// Fixed-order max-rescaled combination of P partial states (gbla_seqsplit.cu).
+cudaError_t combine_states(const float *states, const float2 *stats, int P, int BH, int D,
+                           float *state, float2 *out_stats, cudaStream_t st);
 // Taps (0, 0, 0, 1) for n channels (the identity Conv1D of the ablations), [n][4].
 cudaError_t fill_identity_taps(float *taps, int n, cudaStream_t st);
 // p.flags selects an ablation (the CUDA-core token passes; the caller

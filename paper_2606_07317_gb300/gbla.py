@@ -25,7 +25,7 @@ CONV_WIDTH = 4
 
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_forward_f32out",
             "gbla_backward", "gbla_backward_variant",
-            "gbla_state",
+            "gbla_state", "gbla_state_stats", "gbla_combine_states",
             "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
             "gbla_status_string", "gbla_version", "gbla_release", "gbla_launch_count",
@@ -86,6 +86,10 @@ def load(path: str | None = None):
         lib.gbla_forward_host.restype = _i
         lib.gbla_state.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
         lib.gbla_state.restype = _i
+        lib.gbla_state_stats.argtypes = [_vp] * 7 + [_i] * 6 + [_vp]
+        lib.gbla_state_stats.restype = _i
+        lib.gbla_combine_states.argtypes = [_vp, _vp, _i, _vp, _vp, _i, _i, _i, _vp]
+        lib.gbla_combine_states.restype = _i
         lib.gbla_readout.argtypes = [_vp] * 7 + [_i] * 6 + [_vp]
         lib.gbla_readout.restype = _i
         lib.gbla_state_static_scratch.argtypes = [_vp] * 6 + [_i] * 5 + [_vp]
@@ -294,6 +298,35 @@ def state(k, v, gate, conv_w, seq_lens=None, out=None, algo: int = ALGO_AUTO,
                            _stream(stream))
     _check(st, "gbla_state")
     return out
+
+
+def state_stats(k, v, gate, conv_w, seq_lens=None, algo: int = ALGO_AUTO, stream=None):
+    """gbla_state_stats: (state [B, H, D*D + D], stats [B, H, 2]) fp32, stats = (max gate
+    logit, sum of exp(logit - max)) over each sequence's valid positions."""
+    B, H, N, D = _bhnd(k)
+    out = torch.empty((B, H, D * D + D), dtype=torch.float32, device=k.device)
+    stats = torch.empty((B, H, 2), dtype=torch.float32, device=k.device)
+    st = load().gbla_state_stats(_ptr(k), _ptr(v), _ptr(gate), _ptr(conv_w), _ptr(seq_lens),
+                                 _ptr(out), _ptr(stats), B, H, N, D, _dtype_code(k), int(algo),
+                                 _stream(stream))
+    _check(st, "gbla_state_stats")
+    return out, stats
+
+
+def combine_states(states, stats, stream=None):
+    """gbla_combine_states: states [P, B, H, D*D + D] and stats [P, B, H, 2] (fp32, one
+    CUDA device) of P disjoint token segments -> (state, stats) of the whole sequences."""
+    P, B, H, F = states.shape
+    D = int(round((F + 0.25) ** 0.5 - 0.5))
+    if D * D + D != F or tuple(stats.shape) != (P, B, H, 2):
+        raise ValueError("states must be [P, B, H, D*D + D] and stats [P, B, H, 2]")
+    states, stats = states.contiguous(), stats.contiguous()
+    out = torch.empty((B, H, F), dtype=torch.float32, device=states.device)
+    out_stats = torch.empty((B, H, 2), dtype=torch.float32, device=states.device)
+    st = load().gbla_combine_states(_ptr(states), _ptr(stats), P, _ptr(out), _ptr(out_stats),
+                                    B, H, D, _stream(stream))
+    _check(st, "gbla_combine_states")
+    return out, out_stats
 
 
 def readout(q, out_gate, conv_w, norm_w, state_t, seq_lens=None, out=None,
