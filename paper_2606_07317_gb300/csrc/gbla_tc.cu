@@ -64,7 +64,7 @@ constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the
 // 19 warps: two groups of 8 converter warps, each group converting one
 // 32-token half of every 64-token stage; one warp issues the MMAs; warp 17
 // loads the k tiles (one issuing lane per k ring slot) and warp 18 the v tiles
-// (two issuing lanes, lane l filling the operand slots l and l + 2: a single
+// (two issuing lanes, lane l filling the v slots l and l + 2: a single
 // issuing thread caps an SM's bulk-copy rate at about one box per 0.5 us,
 // below its share of HBM bandwidth).  Every waiter on a ring barrier waits for
 // each of its phases in turn (a parity wait can only tell the current phase
@@ -72,9 +72,9 @@ constexpr int kGroupCh = 128;  // channels of one head group: MMA M and N of the
 //
 // The k tile of a stage (one head group, 64 tokens + 3 rows of conv history)
 // lands in the k ring and is free again as soon as the converters have turned
-// it into K^ = g phi(Conv1D(k)) (bf16, the A operand).  The v tile (two
-// 64-channel blocks, 128B-swizzled) lands next to K^ in the operand ring and
-// is the B operand as it stands: the Conv1D of v is linear, so
+// it into K^ = g phi(Conv1D(k)) (bf16, the A operand), which they write into
+// the K^ ring.  The v tile (two 64-channel blocks, 128B-swizzled) lands in the
+// v ring and is the B operand as it stands: the Conv1D of v is linear, so
 // S = sum_tau w_tau (K^T v shifted by tau), the four shifted views of the v
 // tile forming one N = 256 operand per block, with the taps applied per column
 // when the accumulators are drained.  V~ is never formed or rounded.
@@ -90,13 +90,19 @@ constexpr int kSHalo = kConvW - 1;                   // conv history rows in fro
 constexpr int kSRawRows = kSTok + kSHalo;            // 67
 constexpr int kSRawRowB = kGroupCh * 2;              // bytes of one token's k group row
 constexpr int kSKBox = kSRawRows * kSRawRowB;        // 17152: one k tile
-constexpr int kSKStages = 3;                         // k ring: one issuing lane per slot
+constexpr int kSKStages = 4;                         // k ring: one issuing lane per slot
 constexpr int kSVBlock = 72 * 128;                   // 9216: v block pitch (1024-aligned)
 constexpr int kSVBoxBytes = kSRawRows * 128;         // 8576 written by one v box
 constexpr int kSMnBlock = kSTok * 128;               // 8192: one 64-channel MN block of K^
-constexpr int kSOpV = 2 * kSMnBlock;                 // v blocks after K^ in an operand slot
-constexpr int kSOpStage = kSOpV + 2 * kSVBlock;      // 34816
-constexpr int kSOpStages = 4;                        // operand ring: v lane l fills l, l + 2
+// The K^ tile only has to outlive its stage's MMAs, while the v tile is
+// fetched stages ahead, so they have rings of their own: the shared memory a
+// K^ slot per v slot would take goes to a deeper k ring (a per-stage clock64
+// trace showed the converters waiting ~600 cycles a stage for their k tile
+// with three k slots).
+constexpr int kSKhStage = 2 * kSMnBlock;             // 16384: one K^ tile (two MN blocks)
+constexpr int kSKhStages = 3;                        // K^ ring
+constexpr int kSVStage = 2 * kSVBlock;               // 18432: one v tile (two blocks)
+constexpr int kSVStages = 4;                         // v ring: v lane l fills l, l + 2
 constexpr int kSVLanes = 2;
 constexpr int kRangeStages = 32;                     // longest range (stages)
 constexpr int kRangeTok = kRangeStages * kSTok;      // 2048
@@ -105,8 +111,9 @@ constexpr uint32_t kSTmemCols = 512;                 // per v block: 4 taps x 64
 constexpr int kMaxBatch = 2048;
 
 // Shared-memory map of the state kernel (offsets from a 1024-aligned base).
-constexpr int kSOffOp = 0;
-constexpr int kSOffK = kSOffOp + kSOpStages * kSOpStage;
+constexpr int kSOffKh = 0;
+constexpr int kSOffV = kSOffKh + kSKhStages * kSKhStage;
+constexpr int kSOffK = kSOffV + kSVStages * kSVStage;
 constexpr int kSOffGate = kSOffK + kSKStages * kSKBox;              // u16 [2][kRangeTok]
 constexpr int kSOffHmax = kSOffGate + 2 * kRangeTok * 2;            // float [2][64]: half-stage max
 constexpr int kSOffSegm = kSOffHmax + 2 * 64 * 4;                   // float [2][32]: segment max
@@ -116,16 +123,16 @@ constexpr int kSOffWv = kSOffLred + 16 * 2 * 4;                     // float4 [1
 constexpr int kSOffRed = kSOffWv + kGroupCh * 16;                   // int [32]: scan scratch
 constexpr int kSOffPre = kSOffRed + 32 * 4;                         // int [kMaxBatch + 1]
 constexpr int kSOffBar = kSOffPre + ((kMaxBatch + 1) * 4 + 15) / 16 * 16;
-// k_full, k_empty, op_full (K^ written), v_full (v landed), op_empty, done, final,
-// logits_in (the first range's gate logits are in shared memory)
-constexpr int kSBarCount = 2 * kSKStages + 3 * kSOpStages + 3;
+// k_full, k_empty, kh_full (K^ written), kh_empty, v_full (v landed), v_empty,
+// done, final, logits_in (the first range's gate logits are in shared memory)
+constexpr int kSBarCount = 2 * kSKStages + 2 * kSKhStages + 2 * kSVStages + 3;
 constexpr int kSOffMisc = kSOffBar + kSBarCount * 8;                // tmem addr, abort flag
 constexpr int kSSmemBytes = kSOffMisc + 16 + 1024;                  // + alignment slack
 static_assert(kSSmemBytes <= 227 * 1024, "state shared memory");
-static_assert(kSOpStage % 1024 == 0 && kSVBlock % 1024 == 0 && kSOffK % 128 == 0 &&
-                  kSKBox % 128 == 0,
+static_assert(kSKhStage % 1024 == 0 && kSVStage % 1024 == 0 && kSVBlock % 1024 == 0 &&
+                  kSOffV % 1024 == 0 && kSOffK % 128 == 0 && kSKBox % 128 == 0,
               "TMA and swizzled operand alignment");
-static_assert(kSOpStages % kSVLanes == 0, "each operand slot has one issuing lane");
+static_assert(kSVStages % kSVLanes == 0, "each v slot has one issuing lane");
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -456,9 +463,9 @@ __global__ void __launch_bounds__(kSThreads, 1)
   int *pre = (int *)(smem + kSOffPre);
   uint64_t *bars = (uint64_t *)(smem + kSOffBar);
   uint64_t *k_full = bars, *k_empty = bars + kSKStages;
-  uint64_t *op_full = bars + 2 * kSKStages, *v_full = op_full + kSOpStages;
-  uint64_t *op_empty = v_full + kSOpStages;
-  uint64_t *done = op_empty + kSOpStages, *fin = done + 1, *logits_in = fin + 1;
+  uint64_t *kh_full = bars + 2 * kSKStages, *kh_empty = kh_full + kSKhStages;
+  uint64_t *v_full = kh_empty + kSKhStages, *v_empty = v_full + kSVStages;
+  uint64_t *done = v_empty + kSVStages, *fin = done + 1, *logits_in = fin + 1;
   uint32_t *tmem_slot = (uint32_t *)(smem + kSOffMisc);
   const AbortFlag ab{smem_u32(smem + kSOffMisc + 4)};
 
@@ -484,10 +491,13 @@ __global__ void __launch_bounds__(kSThreads, 1)
       mbar_init(&k_full[i], 1);            // the k box (expect_tx)
       mbar_init(&k_empty[i], kSCvtWarps);  // released by both converter groups
     }
-    for (int i = 0; i < kSOpStages; ++i) {
-      mbar_init(&op_full[i], kSCvtWarps);  // K^ written (and v rows past the end zeroed)
+    for (int i = 0; i < kSKhStages; ++i) {
+      mbar_init(&kh_full[i], kSCvtWarps);  // K^ written (and v rows past the end zeroed)
+      mbar_init(&kh_empty[i], 1);          // the stage's MMAs completed
+    }
+    for (int i = 0; i < kSVStages; ++i) {
       mbar_init(&v_full[i], 1);            // the v boxes (expect_tx)
-      mbar_init(&op_empty[i], 1);          // the stage's MMAs completed
+      mbar_init(&v_empty[i], 1);           // the stage's MMAs completed
     }
     mbar_init(done, 1);
     mbar_init(fin, 1);
@@ -547,9 +557,9 @@ __global__ void __launch_bounds__(kSThreads, 1)
         tma_load_4d_hint(smem + kSOffK + ks * kSKBox, &tm_k, &k_full[ks], 0, st.hg * G, tok, st.b,
                          pol);
       } else {
-        const uint32_t os = gs % kSOpStages, ph = (gs / kSOpStages) & 1;
-        if (!mbar_wait(&op_empty[os], ph ^ 1, &ab)) return false;
-        uint8_t *dst = smem + kSOffOp + os * kSOpStage + kSOpV;
+        const uint32_t os = gs % kSVStages, ph = (gs / kSVStages) & 1;
+        if (!mbar_wait(&v_empty[os], ph ^ 1, &ab)) return false;
+        uint8_t *dst = smem + kSOffV + os * kSVStage;
         // the second block is absent for a missing head (D = 64, odd H)
         const bool two = !(D == 64 && st.hg * G + 1 >= H);
         mbar_arrive_expect_tx(&v_full[os], (two ? 2 : 1) * kSVBoxBytes);
@@ -585,7 +595,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
       // phases of its slot complete in order: waiting for the last suffices)
       if (last != 0xffffffffu) {
         const bool okw = kw ? mbar_wait(&k_full[last % kSKStages], (last / kSKStages) & 1, nullptr)
-                            : mbar_wait(&v_full[last % kSOpStages], (last / kSOpStages) & 1, nullptr);
+                            : mbar_wait(&v_full[last % kSVStages], (last / kSVStages) & 1, nullptr);
         if (!okw) report_error(4096, ab);
       }
     }
@@ -607,7 +617,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
     // ------------------------------------------------------------ converters
     // K^ rows: MN block q / 16, token row 4j + u, 16-byte chunk (q % 16) / 2
     // swizzled by the row, 8-byte half q & 1
-    const uint32_t arow0 = smem_u32(smem + kSOffOp) +
+    const uint32_t arow0 = smem_u32(smem + kSOffKh) +
                            (uint32_t)((q >> 4) * kSMnBlock + 4 * j * 128 + (q & 1) * 8);
     const uint32_t cs = (uint32_t)(((q & 15) >> 1) ^ (4 * (j & 1)));
     const uint32_t raw0 = smem_u32(smem + kSOffK) + (uint32_t)(4 * j * kSRawRowB + q * 8);
@@ -708,13 +718,14 @@ __global__ void __launch_bounds__(kSThreads, 1)
         for (int it = 0; it < nst; ++it) {  // this group converts token rows 32 grp .. 32 grp + 31
           const uint32_t gs = gs0 + it;
           const uint32_t ks = gs % kSKStages, kph = (gs / kSKStages) & 1;
-          const uint32_t os = gs % kSOpStages, oph = (gs / kSOpStages) & 1;
+          const uint32_t hs = gs % kSKhStages, hph = (gs / kSKhStages) & 1;
+          const uint32_t os = gs % kSVStages, oph = (gs / kSVStages) & 1;
           if (!mbar_wait(&k_full[ks], kph, &ab) && !ab.raised()) report_error(1, ab);
-          if (!mbar_wait(&op_empty[os], oph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
+          if (!mbar_wait(&kh_empty[hs], hph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
           const int T = (st.st + it) * kSTok;
           const int nvalid = min(max(st.L - (T + 32 * grp + 4 * j), 0), 4);
           const float ls = state_convert_k(
-              raw0 + ks * kSKBox + grp * 32 * kSRawRowB, arow0 + os * kSOpStage + grp * 32 * 128, cs,
+              raw0 + ks * kSKBox + grp * 32 * kSRawRowB, arow0 + hs * kSKhStage + grp * 32 * 128, cs,
               gws + (uint32_t)((lst0 + it) * kSTok + 32 * grp) * 2, mlog, wk, z, nvalid);
           if (d0 == 0) lacc += ls;
           __syncwarp();
@@ -724,7 +735,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
             // NaN or inf: zero them (both 64-channel blocks) once they have landed
             if (!mbar_wait(&v_full[os], oph, &ab) && !ab.raised()) report_error(1, ab);
             const int r0 = max(st.L - (T - kSHalo), 0);
-            const uint32_t vb = smem_u32(smem + kSOffOp) + os * kSOpStage + kSOpV;
+            const uint32_t vb = smem_u32(smem + kSOffV) + os * kSVStage;
             for (int e = tid; e < (kSRawRows - r0) * 16; e += kSProd) {
               const int rr = r0 + e / 16, blk = (e / 8) & 1, ck = e & 7;
               sts_v4(vb + blk * kSVBlock + rr * 128 + ck * 16, make_uint4(0, 0, 0, 0));
@@ -732,7 +743,7 @@ __global__ void __launch_bounds__(kSThreads, 1)
           }
           fence_proxy_async_smem();  // K^ (and zeroed v rows) visible to the tensor cores
           __syncwarp();
-          if (lane == 0) mbar_arrive(&op_full[os]);
+          if (lane == 0) mbar_arrive(&kh_full[hs]);
         }
         gs0 += nst;
 
@@ -817,9 +828,9 @@ __global__ void __launch_bounds__(kSThreads, 1)
       // the slot offsets (a descriptor's address field is the byte address
       // >> 4, and shared addresses stay below 256 KB, so adding never carries).
       constexpr uint32_t idesc = idesc_bf16_f32(128, 256, 1, 1);
-      const uint64_t ad0 = sw128_desc(smem_u32(smem + kSOffOp), kSMnBlock, 1024);
-      const uint64_t bd0 = sw128_desc(smem_u32(smem + kSOffOp + kSOpV), 128, 1024);
-      uint32_t os = 0, oph = 0;
+      const uint64_t ad0 = sw128_desc(smem_u32(smem + kSOffKh), kSMnBlock, 1024);
+      const uint64_t bd0 = sw128_desc(smem_u32(smem + kSOffV), 128, 1024);
+      uint32_t hs = 0, hph = 0, os = 0, oph = 0;
       bool ok = true;
       for (long long r = blockIdx.x; r < R && ok; r += gridDim.x) {
         const long long se = range_begin(NS, R, r + 1);
@@ -828,22 +839,25 @@ __global__ void __launch_bounds__(kSThreads, 1)
           const long long seg_end = min(se, st.s0 + st.nst);
           const int nst = (int)(seg_end - s);
           for (int it = 0; it < nst; ++it) {
-            if (!mbar_wait(&op_full[os], oph, &ab) || !mbar_wait(&v_full[os], oph, &ab)) {
+            if (!mbar_wait(&kh_full[hs], hph, &ab) || !mbar_wait(&v_full[os], oph, &ab)) {
               if (!ab.raised()) report_error(4, ab);
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint64_t off = (uint64_t)(os * kSOpStage) >> 4;
+            const uint64_t aoff = (uint64_t)(hs * kSKhStage) >> 4;
+            const uint64_t boff = (uint64_t)(os * kSVStage) >> 4;
 #pragma unroll
             for (int blk = 0; blk < 2; ++blk)
 #pragma unroll
               for (int k16 = 0; k16 < kSTok / 16; ++k16)
-                mma_bf16(tmem + 256 * blk, ad0 + off + (k16 * 2048 >> 4),
-                         bd0 + off + ((blk * kSVBlock + 16 * k16 * 128) >> 4), idesc,
+                mma_bf16(tmem + 256 * blk, ad0 + aoff + (k16 * 2048 >> 4),
+                         bd0 + boff + ((blk * kSVBlock + 16 * k16 * 128) >> 4), idesc,
                          (it | k16) != 0);
-            mma_commit(&op_empty[os]);
-            if (++os == kSOpStages) { os = 0; oph ^= 1; }
+            mma_commit(&kh_empty[hs]);
+            mma_commit(&v_empty[os]);
+            if (++hs == kSKhStages) { hs = 0; hph ^= 1; }
+            if (++os == kSVStages) { os = 0; oph ^= 1; }
           }
           if (ok) mma_commit(done);
           s = seg_end;
