@@ -349,6 +349,9 @@ __device__ __forceinline__ float gate_log2(unsigned short a, float mlog) {
 // MN-major, 128B-swizzled A tile (one 8-byte piece per token row).  Tokens past
 // the sequence end (nvalid < 4) are zeros.  Returns the sum of 2^a' ln 2 over
 // the 4 tokens (0 for tokens past the end, whose logits are -inf).
+// FULL: all 4 tokens are valid (nvalid == 4), the case of every token quad but
+// the sequence's last, compiled without the masking.
+template <bool FULL>
 __device__ __forceinline__ float state_convert_k(uint32_t raw, uint32_t arow, uint32_t cs,
                                                  uint32_t gws, float mlog, const float (&w)[4][4],
                                                  float2 (&z)[2], int nvalid) {
@@ -365,7 +368,7 @@ __device__ __forceinline__ float state_convert_k(uint32_t raw, uint32_t arow, ui
     lsum += wl;
     float2 k01 = khat2(conv_rows(w, x, u, 0), al, wl);
     float2 k23 = khat2(conv_rows(w, x, u, 2), al, wl);
-    if (u >= nvalid) {  // rows past the sequence end may hold anything, NaN included
+    if (!FULL && u >= nvalid) {  // rows past the sequence end may hold anything, NaN included
       k01 = make_float2(0.f, 0.f);
       k23 = make_float2(0.f, 0.f);
     }
@@ -724,9 +727,12 @@ __global__ void __launch_bounds__(kSThreads, 1)
           if (!mbar_wait(&kh_empty[hs], hph ^ 1, &ab) && !ab.raised()) report_error(1, ab);
           const int T = (st.st + it) * kSTok;
           const int nvalid = min(max(st.L - (T + 32 * grp + 4 * j), 0), 4);
-          const float ls = state_convert_k(
-              raw0 + ks * kSKBox + grp * 32 * kSRawRowB, arow0 + hs * kSKhStage + grp * 32 * 128, cs,
-              gws + (uint32_t)((lst0 + it) * kSTok + 32 * grp) * 2, mlog, wk, z, nvalid);
+          const uint32_t rawp = raw0 + ks * kSKBox + grp * 32 * kSRawRowB;
+          const uint32_t arp = arow0 + hs * kSKhStage + grp * 32 * 128;
+          const uint32_t gwp = gws + (uint32_t)((lst0 + it) * kSTok + 32 * grp) * 2;
+          const float ls = nvalid == 4
+                               ? state_convert_k<true>(rawp, arp, cs, gwp, mlog, wk, z, 4)
+                               : state_convert_k<false>(rawp, arp, cs, gwp, mlog, wk, z, nvalid);
           if (d0 == 0) lacc += ls;
           __syncwarp();
           if (lane == 0) mbar_arrive(&k_empty[ks]);  // the k tile is consumed
