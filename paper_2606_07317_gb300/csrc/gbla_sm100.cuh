@@ -303,11 +303,11 @@ __device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap *m, int c0,
       "r"(c0), "r"(c1), "r"(c2), "r"(c3)
       : "memory");
 }
-// Hint: pull [p, p + bytes) into L2 (16-byte aligned, bytes a multiple of 16).
-// Prefetches the cache line holding *p into L2 (a hint; no register result).
+// Hint: pull the cache line holding *p into L2 (no register result).
 __device__ __forceinline__ void prefetch_l2_line(const void *p) {
   asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
 }
+// Hint: pull [p, p + bytes) into L2 (16-byte aligned, bytes a multiple of 16).
 __device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
