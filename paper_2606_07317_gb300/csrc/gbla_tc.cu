@@ -889,13 +889,15 @@ __global__ void __launch_bounds__(kSThreads, 1)
 // over the batch in record order, 16 loads in flight at a time, with the
 // scale factors broadcast from the lanes that computed them.
 //
-// LEAN (the grid has at most one block per SM): 32 registers a thread, 4
-// loads in flight in registers and 5 more staged through shared memory by
-// cp.async (10 KB).  The state kernel's 19 warps leave exactly one 32-register
-// warp per SM sub-partition free, and its shared memory leaves room for the
-// staging buffer, so a lean block is made resident beside the state CTA as
+// LEAN: 32 registers a thread, 4 loads in flight in registers and 5 more
+// staged through shared memory by cp.async (10 KB).  The state kernel's 19
+// warps leave exactly one 32-register warp per SM sub-partition free, and its
+// shared memory leaves room for the staging buffer, so when the grid has at
+// most one block per SM a lean block is made resident beside the state CTA as
 // soon as the state grid signals its dependents, and waits there for the
-// state grid to complete instead of being scheduled after it.
+// state grid to complete instead of being scheduled after it.  Lean blocks
+// also serve grids too large for one wave of the wide ones (16 of them fit an
+// SM, against a handful of wide blocks).
 constexpr int kReduceThreads = 128;
 template <int D, bool LEAN>
 __global__ void __launch_bounds__(kReduceThreads, LEAN ? 16 : 1)
@@ -1792,7 +1794,23 @@ cudaError_t run_state(const Problem &p, const void *k, const void *v, const void
   constexpr int F = D * D + D;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.B * p.H, (F / 4 + kReduceThreads - 1) / kReduceThreads);
-  const bool lean = (long long)cfg.gridDim.x * cfg.gridDim.y <= num_sms();
+  // Lean blocks (32 registers, up to 16 an SM) for a grid of at most one block
+  // per SM, which then waits beside the state CTAs, and for a grid that the
+  // wide blocks (16 loads in flight, 116 registers) would run in more than one
+  // wave; wide blocks when they fit one wave.  Measured at D = 128 on 32
+  // ragged sequences (8448 blocks): 562.8 -> 540.1 us per forward with lean
+  // blocks; with 288 and 576 blocks lean ones were 6.5-9.4 us slower.
+  static const int wide_per_sm = [] {
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, tc_reduce_kernel<D, false>,
+                                                      kReduceThreads, 0) != cudaSuccess) {
+      (void)cudaGetLastError();
+      n = 1;
+    }
+    return n;
+  }();
+  const long long nblk = (long long)cfg.gridDim.x * cfg.gridDim.y;
+  const bool lean = nblk <= num_sms() || nblk > (long long)wide_per_sm * num_sms();
   if (lean) {  // the SMs keep the state kernel's shared-memory split for the lean blocks
     static std::once_flag carve;
     std::call_once(carve, [] {  // a hint: if it is refused, the launch goes on without it
