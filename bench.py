@@ -291,9 +291,12 @@ def bench_ours(args, ws, rank, local):
 
 
 def bench_backward(args, ws, rank, local):
-    """--backward: gbla_backward (gradients of sum(dy * o) for every input) on the
+    """--backward: the backward (gradients of sum(dy * o) for every input) on the
     workload; tokens/s and the whole-step roofline (bf16: q, k, v, out_gate, dy, gate
-    read and dq, dk, dv, dout_gate, dgate written, 18 D + 4 bytes per token-head)."""
+    read and dq, dk, dv, dout_gate, dgate written, 18 D + 4 bytes per token-head).
+    The line's value is gbla_backward_from_state, given the state and gate statistics
+    the forward keeps (gbla_state_stats of each input set, made before the timed
+    region); `recompute` times gbla_backward, which runs the state pass again."""
     from paper_2606_07317_gb300 import gbla
 
     dev = torch.device("cuda", local)
@@ -308,36 +311,44 @@ def bench_backward(args, ws, rank, local):
     gen.manual_seed(w.seed + 1000)
     dys = [torch.randn(inp0["q"].shape, generator=gen, device=dev).to(inp0["q"].dtype)
            for _ in sets]
+    saved = [gbla.state_stats(s["k"], s["v"], s["gate"], s["conv_w"], s["seq_lens"])
+             for s in sets]
     e_el = 2 if w.dtype == "bf16" else 4
     step_bytes = w.valid_tokens * w.H * e_el * (9 * w.D + 2)
     stream = torch.cuda.current_stream(dev)
 
-    def step(i):
+    def step(i, from_state):
         s = sets[i % 2]
+        kw = dict(state=saved[i % 2][0], stats=saved[i % 2][1]) if from_state else {}
         gbla.backward(s["q"], s["k"], s["v"], s["gate"], s["out_gate"], s["conv_w"],
-                      s["norm_w"], s["seq_lens"], dys[i % 2], stream=stream)
+                      s["norm_w"], s["seq_lens"], dys[i % 2], stream=stream, **kw)
 
-    for i in range(args.warmup):
-        step(i)
-    torch.cuda.synchronize(dev)
+    def timed(from_state):
+        for i in range(args.warmup):
+            step(i, from_state)
+        torch.cuda.synchronize(dev)
+        n0 = gbla.launch_count()
+        barrier(ws)
+        torch.cuda.synchronize(dev)
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for i in range(args.steps):
+            step(i, from_state)
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier(ws)
+        return (max_over_ranks(ev0.elapsed_time(ev1) / args.steps, ws, dev),
+                gbla.launch_count() - n0)
+
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.1)
-    n0 = gbla.launch_count()
-    barrier(ws)
-    torch.cuda.synchronize(dev)
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
-    ev1.record(stream)
-    torch.cuda.synchronize(dev)
-    barrier(ws)
-    launches = gbla.launch_count() - n0
+    ms, launches = timed(True)
+    ms_re, launches_re = timed(False)
     clocks = sampler.stop()
-    ms = max_over_ranks(ev0.elapsed_time(ev1) / args.steps, ws, dev)
     peak, peak_kind = measured_peaks()
     achieved = step_bytes / (ms * 1e-3) / 1e9
+    achieved_re = step_bytes / (ms_re * 1e-3) / 1e9
     if rank == 0:
         print(json.dumps({
             "metric": "GBLA bwd tokens/sec (gradients of every input)", "value":
@@ -347,11 +358,16 @@ def bench_backward(args, ws, rank, local):
             "dtype": w.dtype, "data": "synthetic (seeded N(0,1) inputs and dy)",
             "config": {"workload": w.name, "B": w.B, "H": w.H, "N": w.N, "D": w.D,
                        "alg_bytes_per_step": step_bytes,
+                       "state": "the forward's, kept (gbla_backward_from_state)",
                        "l2": "inputs larger than L2, two sets rotated"},
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                          "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
                          "kernel": "whole backward step",
                          "peak_source": f"{peak_kind} (MEASURED_PEAKS.json hbm_gbs)"},
+            "recompute": {"entry": "gbla_backward (state pass included)",
+                          "ms_per_step": round(ms_re, 6),
+                          "value": round(tokens * ws / (ms_re * 1e-3), 1),
+                          "frac": round(achieved_re / peak, 4), "gpu_launches": launches_re},
             "gpu_launches": launches, "clocks": clocks}), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()

@@ -157,7 +157,8 @@ gbla_status gbla_forward_f32out(const void *q, const void *k, const void *v,
  *   dconv_w [3, H, D, W] fp32 (q, k, v taps);   dnorm_w [H, D] fp32.
  * Rows t >= L_b of dq, dk, dv, dout_gate and dgate are written as 0; dconv_w
  * and dnorm_w are overwritten with sums over the batch.  The forward state is
- * recomputed inside (nothing is kept from a forward call).  fp32 arithmetic
+ * recomputed inside (nothing is kept from a forward call; see
+ * gbla_backward_from_state for a backward that takes it).  fp32 arithmetic
  * (for bf16 with D = 64 the token contractions run on tensor cores with bf16
  * operands, S and dS split into bf16 hi + lo, fp32 accumulation); every sum
  * runs in a fixed order (bitwise reproducible).  Asynchronous on
@@ -191,6 +192,30 @@ gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
                                   void *dv, void *dgate, void *dout_gate, float *dconv_w,
                                   float *dnorm_w, int B, int H, int N, int D,
                                   gbla_dtype dtype, uint32_t flags, gbla_stream_t stream);
+
+/*
+ * gbla_backward_from_state -- gbla_backward given the forward's state: for
+ * training, where the forward ran as gbla_state_stats + gbla_readout and kept
+ * what the backward needs instead of recomputing it (the key-gate softmax and
+ * the state of Sec. 2.1 item 2 over the whole sequence):
+ *   state [B, H, D*D + D] fp32  S and z of each sequence, and
+ *   stats [B, H, 2] fp32        its (m, l),
+ * exactly as gbla_state_stats returned them for the same k, v, gate, conv_w
+ * and seq_lens (other values give gradients of another forward; nothing
+ * checks them).  The call skips the state pass and reads nothing else of the
+ * forward.  Both are inputs: device pointers, 16-byte aligned, not
+ * overlapping any output (GBLA_ERR_INVALID_ARG otherwise).  Every other
+ * argument, output, limit, error and the asynchrony as gbla_backward (the full
+ * core).
+ */
+gbla_status gbla_backward_from_state(const void *q, const void *k, const void *v,
+                                     const void *gate, const void *out_gate,
+                                     const float *conv_w, const float *norm_w,
+                                     const int32_t *seq_lens, const float *state,
+                                     const float *stats, const void *dy, void *dq, void *dk,
+                                     void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                     float *dnorm_w, int B, int H, int N, int D,
+                                     gbla_dtype dtype, gbla_stream_t stream);
 
 /*
  * gbla_project -- the layer front end: Sec. 2.1 item 1 (X~ = Conv1D(X), then

@@ -389,13 +389,18 @@ gbla_status gbla_backward(const void *q, const void *k, const void *v, const voi
                                stream);
 }
 
-gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
-                                  const void *gate, const void *out_gate,
-                                  const float *conv_w, const float *norm_w,
-                                  const int32_t *seq_lens, const void *dy, void *dq, void *dk,
-                                  void *dv, void *dgate, void *dout_gate, float *dconv_w,
-                                  float *dnorm_w, int B, int H, int N, int D,
-                                  gbla_dtype dtype, uint32_t flags, gbla_stream_t stream) {
+}  // extern "C"
+
+// gbla_backward_variant, and gbla_backward_from_state when `saved` (state_in and
+// stats_in are the forward's state and gate statistics; flags 0): the state
+// pass is then skipped.
+static gbla_status backward_impl(const void *q, const void *k, const void *v, const void *gate,
+                                 const void *out_gate, const float *conv_w, const float *norm_w,
+                                 const int32_t *seq_lens, const float *state_in,
+                                 const float *stats_in, const void *dy, void *dq, void *dk,
+                                 void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                 float *dnorm_w, int B, int H, int N, int D, gbla_dtype dtype,
+                                 uint32_t flags, bool saved, gbla_stream_t stream) {
   if (flags & ~(uint32_t)GBLA_FLAG_BLA) return GBLA_ERR_INVALID_ARG;
   bool empty = false;
   gbla_status s = check_dims(B, H, N, D, dtype, &empty);
@@ -412,6 +417,9 @@ gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
       return GBLA_ERR_CUDA;
     return GBLA_OK;
   }
+  if (saved && (state_in == nullptr || stats_in == nullptr || !aligned(state_in) ||
+                !aligned(stats_in)))
+    return GBLA_ERR_INVALID_ARG;
   const size_t bytes = (size_t)B * N * H * D * elem_bytes(dtype);
   const size_t gbytes = (size_t)B * N * H * elem_bytes(dtype);
   const Range outs[7] = {range_of(dq, bytes),     range_of(dk, bytes),
@@ -423,9 +431,13 @@ gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
                         range_of(dy, bytes),     range_of(gate, gbytes),
                         range_of(conv_w, wbytes), range_of(norm_w, nbytes),
                         range_of(seq_lens, seq_lens ? sizeof(int32_t) * B : 0)};
+  const Range kept[2] = {range_of(state_in, sizeof(float) * state_floats(D) * B * H),
+                          range_of(stats_in, sizeof(float) * 2 * B * H)};
   for (int i = 0; i < 7; ++i) {
     for (int j = 0; j < 9; ++j)
       if (overlap(outs[i], ins[j])) return GBLA_ERR_INVALID_ARG;
+    for (int j = 0; j < 2; ++j)
+      if (saved && overlap(outs[i], kept[j])) return GBLA_ERR_INVALID_ARG;
     for (int j = i + 1; j < 7; ++j)
       if (overlap(outs[i], outs[j])) return GBLA_ERR_INVALID_ARG;
   }
@@ -460,20 +472,53 @@ gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
     if (cudaMemsetAsync(zg, 0, zgate_bytes, st) != cudaSuccess) return GBLA_ERR_CUDA;
     gt = zg;
   }
-  // the forward state S, z through the forward's own state path, which on
-  // tensor cores also yields the gate statistics the backward needs
-  if ((s = run_state(p, tc, k, v, gt, cw, base + lay.state, st,
-                     tc ? (float2 *)(base + lay.stats) : nullptr)) != GBLA_OK)
-    return s;
   BwdArgs a{q, k, v, gt, out_gate, dy, cw, norm_w, dq, dk, dv, dgate, dout_gate,
-            dconv_w, dnorm_w};
+            dconv_w, dnorm_w, base + lay.state, (const float2 *)(base + lay.stats)};
+  bool stats_ready = tc;
+  if (saved) {  // the forward's own state and gate statistics
+    a.state = state_in;
+    a.stats = (const float2 *)stats_in;
+    stats_ready = true;
+  } else if ((s = run_state(p, tc, k, v, gt, cw, base + lay.state, st,
+                            tc ? (float2 *)(base + lay.stats) : nullptr)) != GBLA_OK) {
+    // the forward state S, z through the forward's own state path, which on
+    // tensor cores also yields the gate statistics the backward needs
+    return s;
+  }
   Problem pb = p;
   pb.flags = flags;
-  if ((s = from_cuda(bwd_run(pb, a, base, tc, st))) != GBLA_OK) return s;
+  if ((s = from_cuda(bwd_run(pb, a, base, stats_ready, st))) != GBLA_OK) return s;
   if (((flags & GBLA_FLAG_NO_CONV) && cudaMemsetAsync(dconv_w, 0, wbytes, st) != cudaSuccess) ||
       ((flags & GBLA_FLAG_NO_GATE) && cudaMemsetAsync(dgate, 0, gbytes, st) != cudaSuccess))
     return from_cuda(cudaGetLastError());
   return GBLA_OK;
+}
+
+extern "C" {
+
+gbla_status gbla_backward_variant(const void *q, const void *k, const void *v,
+                                  const void *gate, const void *out_gate,
+                                  const float *conv_w, const float *norm_w,
+                                  const int32_t *seq_lens, const void *dy, void *dq, void *dk,
+                                  void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                  float *dnorm_w, int B, int H, int N, int D,
+                                  gbla_dtype dtype, uint32_t flags, gbla_stream_t stream) {
+  return backward_impl(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, nullptr, nullptr, dy,
+                       dq, dk, dv, dgate, dout_gate, dconv_w, dnorm_w, B, H, N, D, dtype, flags,
+                       false, stream);
+}
+
+gbla_status gbla_backward_from_state(const void *q, const void *k, const void *v,
+                                     const void *gate, const void *out_gate,
+                                     const float *conv_w, const float *norm_w,
+                                     const int32_t *seq_lens, const float *state,
+                                     const float *stats, const void *dy, void *dq, void *dk,
+                                     void *dv, void *dgate, void *dout_gate, float *dconv_w,
+                                     float *dnorm_w, int B, int H, int N, int D,
+                                     gbla_dtype dtype, gbla_stream_t stream) {
+  return backward_impl(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, state, stats, dy,
+                       dq, dk, dv, dgate, dout_gate, dconv_w, dnorm_w, B, H, N, D, dtype, 0u,
+                       true, stream);
 }
 
 // Validation shared by gbla_project and gbla_layer_forward.

@@ -699,18 +699,19 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
   const int B = p.B, H = p.H, N = p.N, BH = B * H;
   const int nck = (N + kChunk - 1) / kChunk;
   const BwdLayout lay = bwd_layout(p);
-  float2 *stats = (float2 *)(scratch + lay.stats);
+  float2 *stats_w = (float2 *)(scratch + lay.stats);  // filled here unless stats_ready
+  const float2 *stats = stats_ready ? a.stats : stats_w;
   float *qpart = scratch + lay.qpart, *red = scratch + lay.red;
   T *dxt = (T *)(scratch + lay.dxt);  // dq~, dk~, dv~ planes in the storage dtype
   float *wpart = scratch + lay.wpart;
-  const float *state = scratch + lay.state;
+  const float *state = a.state;
   const size_t plane = (size_t)B * N * H * D;
   cudaError_t e;
   float2 *gpart = (float2 *)(scratch + lay.gpart);
   if (!stats_ready) {
     bwd_gate_split<T><<<dim3(BH, kGateSplits), 256, 0, st>>>((const T *)a.gate, p.seq_lens,
                                                              gpart, H, N);
-    bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(gpart, stats, BH);
+    bwd_gate_join<<<(BH + 255) / 256, 256, 0, st>>>(gpart, stats_w, BH);
     count_launch(2);
   }
   constexpr int TPT = Tok<D>::TPT, kTB = Tok<D>::TB;

@@ -77,12 +77,17 @@ struct BwdArgs {
   const float *conv_w, *norm_w;
   void *dq, *dk, *dv, *dgate, *dout_gate;
   float *dconv_w, *dnorm_w;
+  // the forward state S, z [B*H][D*D + D] and, when stats_ready, the key gate's
+  // softmax statistics [B*H] (max, sum of exp): the scratch slots of the
+  // layout below, or a forward's saved copies
+  const float *state;
+  const float2 *stats;
 };
 // Scratch of the backward, in floats from one base: the forward state (filled
-// by the caller through the forward's state path), gate statistics (filled by
-// the caller too when stats_ready, else by the backward itself), chunk
-// partials, reduced dS / dz, the per-token dq~ / dk~ / dv~ planes and the tap
-// gradient partials.
+// by the caller through the forward's state path, unless a saved state is
+// given), gate statistics (filled by the caller too when stats_ready, else by
+// the backward itself), chunk partials, reduced dS / dz, the per-token
+// dq~ / dk~ / dv~ planes and the tap gradient partials.
 struct BwdLayout {
   size_t state, stats, gpart, qpart, red, cpart, dxt, wpart, total;
 };

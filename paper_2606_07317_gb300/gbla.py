@@ -24,7 +24,7 @@ FLAG_BLA = FLAG_NO_CONV | FLAG_NO_GATE | FLAG_NO_NORM
 CONV_WIDTH = 4
 
 EXPORTED = ["gbla_forward", "gbla_forward_ex", "gbla_forward_variant", "gbla_forward_f32out",
-            "gbla_backward", "gbla_backward_variant",
+            "gbla_backward", "gbla_backward_variant", "gbla_backward_from_state",
             "gbla_state", "gbla_state_stats", "gbla_combine_states",
             "gbla_readout",
             "gbla_forward_host", "gbla_state_floats", "gbla_rms_eps",
@@ -76,6 +76,8 @@ def load(path: str | None = None):
         lib.gbla_backward.restype = _i
         lib.gbla_backward_variant.argtypes = [_vp] * 16 + [_i] * 5 + [ctypes.c_uint32, _vp]
         lib.gbla_backward_variant.restype = _i
+        lib.gbla_backward_from_state.argtypes = [_vp] * 18 + [_i] * 5 + [_vp]
+        lib.gbla_backward_from_state.restype = _i
         lib.gbla_project.argtypes = [_vp] * 9 + [_i] * 6 + [_vp]
         lib.gbla_project.restype = _i
         lib.gbla_layer_forward.argtypes = [_vp] * 6 + [_i] * 6 + [_vp]
@@ -223,11 +225,17 @@ def forward_f32out(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens=None, out=N
 
 
 def backward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, stream=None,
-             flags: int = 0) -> dict:
+             flags: int = 0, state=None, stats=None) -> dict:
     """Gradients of sum(dy * o) (gbla_backward): dq, dk, dv, dout_gate like q; dgate like
     gate; dconv_w [3, H, D, W] and dnorm_w [H, D] fp32.  Rows past seq_lens are 0.
-    `flags` (FLAG_*) selects an ablation (gbla_backward_variant); 0 is the full core."""
+    `flags` (FLAG_*) selects an ablation (gbla_backward_variant); 0 is the full core.
+    `state` and `stats`, as state_stats returned them for this forward, skip the state
+    pass (gbla_backward_from_state; full core only)."""
     B, H, N, D = _bhnd(q)
+    if (state is None) != (stats is None):
+        raise ValueError("state and stats go together")
+    if state is not None and flags:
+        raise ValueError("a saved state serves the full core only (flags 0)")
     g = dict(dq=torch.empty_like(q), dk=torch.empty_like(q), dv=torch.empty_like(q),
              dgate=torch.empty_like(gate), dout_gate=torch.empty_like(q),
              dconv_w=torch.empty_like(conv_w, dtype=torch.float32),
@@ -236,7 +244,16 @@ def backward(q, k, v, gate, out_gate, conv_w, norm_w, seq_lens, dy, stream=None,
             _ptr(seq_lens), _ptr(dy), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]),
             _ptr(g["dgate"]), _ptr(g["dout_gate"]), _ptr(g["dconv_w"]), _ptr(g["dnorm_w"]),
             B, H, N, D, _dtype_code(q))
-    if flags:
+    if state is not None:
+        if (state.dtype != torch.float32 or stats.dtype != torch.float32
+                or tuple(state.shape) != (B, H, D * D + D) or tuple(stats.shape) != (B, H, 2)
+                or not state.is_contiguous() or not stats.is_contiguous()):
+            raise ValueError("state must be [B, H, D*D + D] and stats [B, H, 2], contiguous fp32")
+        a = list(args)
+        a[8:8] = [_ptr(state), _ptr(stats)]  # after seq_lens
+        st = load().gbla_backward_from_state(*a, _stream(stream))
+        _check(st, "gbla_backward_from_state")
+    elif flags:
         st = load().gbla_backward_variant(*args, int(flags), _stream(stream))
         _check(st, "gbla_backward_variant")
     else:

@@ -115,3 +115,15 @@ def test_state_and_readout_validation(lib):
         gbla.GBLA_ERR_INVALID_ARG
     assert lib.gbla_forward_host(None, P16, P16, P16, P16, P16, P16, None, P16,
                                  1, 1, 4, 64, 1, None) == gbla.GBLA_ERR_INVALID_ARG
+
+
+def test_backward_from_state_validates_saved_state(lib):
+    # q k v gate out_gate conv_w norm_w seq_lens state stats dy dq dk dv dgate dout_gate
+    # dconv_w dnorm_w: distinct aligned fake addresses, seq_lens NULL
+    base = [P16 + i * 0x100000 for i in range(18)]
+    base[7] = None
+    for i, bad in [(8, None), (8, base[8] + 4), (9, None), (9, base[9] + 8)]:
+        ptrs = list(base)
+        ptrs[i] = bad
+        st = lib.gbla_backward_from_state(*ptrs, 1, 1, 4, 64, gbla.GBLA_BF16, None)
+        assert st == gbla.GBLA_ERR_INVALID_ARG, (i, bad)

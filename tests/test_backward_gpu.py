@@ -194,3 +194,54 @@ def test_backward_variant_rejects_unknown_flags():
     dy = _dy(inp, 44)
     with pytest.raises(gbla.GblaError):
         _run(inp, dy, 8)
+
+
+@pytest.mark.parametrize("dtype,D", [("bf16", 64), ("bf16", 128), ("fp32", 32)])
+def test_backward_from_state_matches_recompute(dtype, D):
+    """gbla_backward_from_state given what gbla_state_stats returned for the same inputs
+    (the state and gate statistics a training forward keeps) gives the recomputing
+    backward's gradients bit for bit -- both run the same state path -- and so the
+    oracle's under the bounds above."""
+    w = custom(B=2, H=2, N=300, D=D, dtype=dtype, seed=45, seq_lens=[300, 77])
+    inp = make_inputs(w, "cuda")
+    dy = _dy(inp, 46)
+    state, stats = gbla.state_stats(inp["k"], inp["v"], inp["gate"], inp["conv_w"],
+                                    inp["seq_lens"])
+    got = gbla.backward(inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"],
+                        inp["conv_w"], inp["norm_w"], inp["seq_lens"], dy, state=state,
+                        stats=stats)
+    ref = _run(inp, dy)
+    for n in NAMES:
+        assert torch.equal(got[n], ref[n]), n
+    _check(got, _oracle(inp, dy), dtype, f"_from_state_D{D}")
+
+
+def test_backward_from_state_rejects():
+    w = custom(B=1, H=2, N=64, D=64, dtype="bf16", seed=47)
+    inp = make_inputs(w, "cuda")
+    dy = _dy(inp, 48)
+    state, stats = gbla.state_stats(inp["k"], inp["v"], inp["gate"], inp["conv_w"])
+    args = (inp["q"], inp["k"], inp["v"], inp["gate"], inp["out_gate"], inp["conv_w"],
+            inp["norm_w"], None, dy)
+    with pytest.raises(ValueError):
+        gbla.backward(*args, state=state)  # stats missing
+    with pytest.raises(ValueError):
+        gbla.backward(*args, flags=gbla.FLAG_NO_CONV, state=state, stats=stats)
+    lib = gbla.load()
+    p = gbla._ptr
+    B, N, H, D = inp["q"].shape
+    outs = [torch.empty_like(inp["q"]) for _ in range(4)]
+    dgate = torch.empty_like(inp["gate"])
+    dcw = torch.empty((3, H, D, 4), device="cuda")
+
+    def call(st_ptr, dnw_ptr):
+        return lib.gbla_backward_from_state(
+            p(inp["q"]), p(inp["k"]), p(inp["v"]), p(inp["gate"]), p(inp["out_gate"]),
+            p(inp["conv_w"]), p(inp["norm_w"]), None, st_ptr, p(stats), p(dy), p(outs[0]),
+            p(outs[1]), p(outs[2]), p(dgate), p(outs[3]), p(dcw), dnw_ptr, B, H, N, D, 1, None)
+
+    dnw = torch.empty((H, D), device="cuda")
+    assert call(None, p(dnw)) == gbla.GBLA_ERR_INVALID_ARG          # no state
+    assert call(p(state), p(state)) == gbla.GBLA_ERR_INVALID_ARG    # dnorm_w over the state
+    assert call(p(state), p(dnw)) == gbla.GBLA_OK
+    torch.cuda.synchronize()
