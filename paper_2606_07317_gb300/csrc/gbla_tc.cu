@@ -637,26 +637,42 @@ __global__ void __launch_bounds__(kSThreads, 1)
       // past a sequence end or for a missing head), half-stage maxima, then
       // for every stage the maximum over its segment.
       {
-        unsigned short a[kRangeTok / kSProd][G];
+        // The 32 slots tid + i kSProd of a warp are 32 consecutive tokens of one
+        // stage: lane i decodes the warp's stage of round i, and the rounds'
+        // (b, hg, stage, L) go round by shuffles, so the decodes (a search of
+        // the stage prefix and a length load when ragged) run side by side.
+        constexpr int NSL = kRangeTok / kSProd;
+        static_assert(kSTok % 32 == 0 && kSProd % 32 == 0 && NSL <= 32,
+                      "a warp's 32 slots of a round lie in one stage");
+        int db = 0, dhg = 0, dst = 0, dL = 0;
+        if (lane < NSL && (tid & ~31) + lane * kSProd < nsr * kSTok) {
+          const StageRef st = decode_stage(p, pre, sb + ((tid & ~31) + lane * kSProd) / kSTok);
+          db = st.b;
+          dhg = st.hg;
+          dst = st.st;
+          dL = st.L;
+        }
+        unsigned short a[NSL][G];
 #pragma unroll
-        for (int i = 0; i < kRangeTok / kSProd; ++i) {
+        for (int i = 0; i < NSL; ++i) {
           const int slot = tid + i * kSProd;
+          const int sbi = __shfl_sync(0xffffffffu, db, i), shg = __shfl_sync(0xffffffffu, dhg, i);
+          const int sst = __shfl_sync(0xffffffffu, dst, i), sL = __shfl_sync(0xffffffffu, dL, i);
 #pragma unroll
           for (int g = 0; g < G; ++g) a[i][g] = 0xff80u;  // bf16 -inf
           if (slot < nsr * kSTok) {
-            const StageRef st = decode_stage(p, pre, sb + slot / kSTok);
-            const int t = st.st * kSTok + slot % kSTok;
-            if (t < st.L) {
+            const int t = sst * kSTok + slot % kSTok;
+            if (t < sL) {
               const unsigned short *gp = (const unsigned short *)p.gate +
-                                         ((size_t)st.b * p.N + t) * H + st.hg * G;
+                                         ((size_t)sbi * p.N + t) * H + shg * G;
 #pragma unroll
               for (int g = 0; g < G; ++g)
-                if (st.hg * G + g < H) a[i][g] = no_gate ? (unsigned short)0 : __ldg(gp + g);
+                if (shg * G + g < H) a[i][g] = no_gate ? (unsigned short)0 : __ldg(gp + g);
             }
           }
         }
 #pragma unroll
-        for (int i = 0; i < kRangeTok / kSProd; ++i) {
+        for (int i = 0; i < NSL; ++i) {
           const int slot = tid + i * kSProd;
 #pragma unroll
           for (int g = 0; g < G; ++g) {
