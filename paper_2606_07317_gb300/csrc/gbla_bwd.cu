@@ -35,6 +35,7 @@
 #include <math.h>
 
 #include "gbla_internal.cuh"
+#include "gbla_sm100.cuh"
 
 namespace gbla {
 namespace {
@@ -362,6 +363,8 @@ __global__ void __launch_bounds__(256) bwd_reduce_state(const float *__restrict_
                                                         float *__restrict__ dotpart, int nck) {
   constexpr int F = D * D + D;
   const int bh = blockIdx.y, i = blockIdx.x * 256 + threadIdx.x;
+  sm100::grid_dep_wait();  // the partials come from the query pass
+  sm100::grid_dep_launch();
   float a = 0.f;
   if (i < F) {
     for (int ch = 0; ch < nck; ++ch) a += part[((size_t)bh * nck + ch) * qrec<D>() + i];
@@ -554,6 +557,8 @@ __global__ void __launch_bounds__(kNT, 2) bwd_conv(
 #pragma unroll
     for (int i = 0; i < kConvW; ++i) dw[c][i] = 0.f;
   }
+  sm100::grid_dep_wait();  // the dx~ planes come from the token passes
+  sm100::grid_dep_launch();
   const size_t rs = (size_t)H * D;
   const size_t col = ((size_t)b * N * H + h) * D + kConvCh * g;
   auto ldx = [&](int t, float (&f)[kConvCh]) {  // x_t, zero outside [0, L)
@@ -666,6 +671,8 @@ __global__ void __launch_bounds__(256) bwd_reduce_w(const float *__restrict__ wp
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int idx = blockIdx.x * 32 + lane;
   __shared__ float part[8][32];
+  sm100::grid_dep_wait();  // the tap partials come from the Conv1D backward
+  sm100::grid_dep_launch();
   float a = 0.f;
   if (idx < total_w) {
     const int s = idx / (H * D * kConvW), r = idx % (H * D * kConvW);
@@ -734,8 +741,10 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
   }
   constexpr int F = D * D + D;
   // on tensor cores the key pass forms c from the reduction's partial dot products
-  bwd_reduce_state<D><<<dim3((F + 255) / 256, BH), 256, 0, st>>>(
-      qpart, red, tc ? state : nullptr, tc ? scratch + lay.cpart : nullptr, nckq);
+  if ((e = launch_pdl(bwd_reduce_state<D>, dim3((F + 255) / 256, BH), dim3(256), 0, st,
+                      (const float *)qpart, red, tc ? state : nullptr,
+                      tc ? scratch + lay.cpart : nullptr, nckq)) != cudaSuccess)
+    return e;
   count_launch();
   if (tc) {
     if ((e = bwd_tc_key(p, a, stats, red, scratch + lay.cpart, (F + 255) / 256, dxt + plane,
@@ -761,13 +770,17 @@ cudaError_t run_bwd(const Problem &p, const BwdArgs &a, float *scratch, bool sta
   if ((e = cudaFuncSetAttribute(bwd_conv<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)conv_stage_bytes<T>())) != cudaSuccess)
     return e;
-  bwd_conv<T, D><<<dim3(nckc, BH, 3), kNT, conv_stage_bytes<T>(), st>>>(
-      (const T *)a.q, (const T *)a.k, (const T *)a.v, dxt, a.conv_w, p.seq_lens, (T *)a.dq,
-      (T *)a.dk, (T *)a.dv, wpart, H, N, nckc, rl);
+  if ((e = launch_pdl(bwd_conv<T, D>, dim3(nckc, BH, 3), dim3(kNT), conv_stage_bytes<T>(), st,
+                      (const T *)a.q, (const T *)a.k, (const T *)a.v, (const T *)dxt, a.conv_w,
+                      p.seq_lens, (T *)a.dq, (T *)a.dk, (T *)a.dv, wpart, H, N, nckc, rl)) !=
+      cudaSuccess)
+    return e;
   count_launch();
   const int nw = 3 * H * D * kConvW + H * D;
-  bwd_reduce_w<D><<<(nw + 31) / 32, 256, 0, st>>>(wpart, qpart, a.dconv_w, a.dnorm_w, B, H,
-                                                     nckc, nckq);
+  if ((e = launch_pdl(bwd_reduce_w<D>, dim3((nw + 31) / 32), dim3(256), 0, st,
+                      (const float *)wpart, (const float *)qpart, a.dconv_w, a.dnorm_w, B, H,
+                      nckc, nckq)) != cudaSuccess)
+    return e;
   count_launch();
   return cudaGetLastError();
 }

@@ -198,6 +198,11 @@ __global__ void __launch_bounds__(kKThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // launched with programmatic dependent launch: dS, dz and the partials of c
+  // come from the reduction before, and nothing global is written before it
+  // has completed
+  grid_dep_wait();
+  grid_dep_launch();
 
   if (warp == kKTmaWarp) {
     // ------------------------------------------------------------ TMA: raw k, v rows
@@ -644,6 +649,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
   if (tid < kD)  // the head's q taps, read by the producers
     *(float4 *)(smem + kQOffTaps + 16 * tid) =
         __ldg((const float4 *)(p.conv_w + ((size_t)h * kD + tid) * kConvW));
+  // launched with programmatic dependent launch: the state may come from the
+  // kernel before, and nothing global is written before it has completed
+  grid_dep_wait();
+  grid_dep_launch();
   {
     // B tiles from S (every thread; contiguous 32-byte reads of S rows, all in
     // flight together): S as bf16 hi + lo with rows d, K = e (for dP), and its
@@ -1153,7 +1162,9 @@ cudaError_t bwd_tc_key(const Problem &p, const BwdArgs &a, const float2 *stats,
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const long long tiles = (long long)BH * kp.tps;
   const int grid = (int)(tiles < sms ? tiles : sms);
-  tc_bwd_key_kernel<<<grid, kKThreads, kKSmem, st>>>(kp, tm_k, tm_v);
+  if ((e = launch_pdl(tc_bwd_key_kernel, dim3(grid), dim3(kKThreads), (size_t)kKSmem, st, kp,
+                      tm_k, tm_v)) != cudaSuccess)
+    return e;
   count_launch();
   return cudaGetLastError();
 }
@@ -1206,7 +1217,9 @@ cudaError_t bwd_tc_query(const Problem &p, const BwdArgs &a, const float *state,
   if ((e = cudaFuncSetAttribute(tc_bwd_query_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kQSmem)) != cudaSuccess)
     return e;
-  tc_bwd_query_kernel<<<dim3(qp.nck, BH), kQThreads, kQSmem, st>>>(qp, tm_q, tm_og, tm_dy);
+  if ((e = launch_pdl(tc_bwd_query_kernel, dim3(qp.nck, BH), dim3(kQThreads), (size_t)kQSmem,
+                      st, qp, tm_q, tm_og, tm_dy)) != cudaSuccess)
+    return e;
   count_launch();
   return cudaGetLastError();
 }

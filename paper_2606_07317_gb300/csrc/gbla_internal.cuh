@@ -71,6 +71,25 @@ cudaError_t tc_readout(const Problem &p, const void *q, const void *og,
                        const float *conv_w, const float *norm_w,
                        const float *state, void *o, cudaStream_t st,
                        bool after_state = false, bool f32_out = false);
+// Programmatic dependent launch: the grid may start while the kernel before it
+// on the stream ends (once that kernel's blocks have all signalled, or
+// exited); the kernel itself waits (griddepcontrol.wait) before it reads
+// anything the kernel before may write, and before its first global write.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
 // ---- backward (CUDA cores, fp32 arithmetic; gbla_bwd.cu) ------------------
 struct BwdArgs {
   const void *q, *k, *v, *gate, *out_gate, *dy;
