@@ -347,8 +347,11 @@ gbla_status gbla_readout(const void *q, const void *out_gate,
  * gbla_forward_host -- gbla_forward for callers whose tensors live in HOST
  * memory (pinned for full copy speed; pageable works).  Same layouts as
  * above, all pointers host pointers.  Copies the inputs to device scratch,
- * runs the forward and copies rows t < L_b of o back, all enqueued on
- * `stream`; the call then waits for the stream, so o is ready on return.
+ * runs the forward and copies rows t < L_b of o back: k, v and the gate
+ * first, then q and out_gate in chunks of 4096 tokens whose readouts start as
+ * they land, o going back chunk by chunk (two streams of its own beside
+ * `stream`, joined to it); o is gbla_forward's bit for bit.  The call waits
+ * for `stream`, so o is ready on return.
  */
 gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
                               const void *gate, const void *out_gate,

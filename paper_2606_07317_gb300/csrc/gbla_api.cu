@@ -5,6 +5,7 @@
 
 #include <atomic>
 #include <mutex>
+#include <vector>
 
 #include "gbla_internal.cuh"
 
@@ -638,10 +639,37 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
   const size_t gbytes = (size_t)B * N * grow;
   const size_t cw = sizeof(float) * 3 * H * D * kConvW, nw = sizeof(float) * H * D;
   const size_t F = state_floats(D);
-  // Layout of the device scratch: q k v og o | gate | conv_w | norm_w | seq_lens | state
+  auto valid_rows = [&](int b) -> size_t {
+    long L = seq_lens ? seq_lens[b] : N;
+    return (size_t)(L < 0 ? 0 : (L > N ? N : L));
+  };
+  // The readout goes in chunks of up to kHostChunk tokens of one batch row.  A
+  // chunk's readout sees the h0 = min(3, t0) rows before it as Conv1D history:
+  // its view of q and out_gate starts h0 rows early, and its output view, of
+  // its own in the o region (obase: first row), holds those h0 rows' outputs
+  // (not copied out) before the chunk's own.  Per token the readout does the
+  // same arithmetic however the rows are cut, so o is that of gbla_forward.
+  constexpr int kHostChunk = 4096;
+  struct Chunk {
+    int b, t0, t1;
+    size_t obase;
+  };
+  std::vector<Chunk> chunks;
+  size_t orows = 0;
+  for (int b = 0; b < B; ++b) {
+    const int L = (int)valid_rows(b);
+    for (int t0 = 0; t0 < L; t0 += kHostChunk) {
+      const int t1 = t0 + kHostChunk < L ? t0 + kHostChunk : L;
+      chunks.push_back({b, t0, t1, orows});
+      orows += (size_t)(t1 - t0) + (size_t)(t0 < 3 ? t0 : 3);
+    }
+  }
+  // Layout of the device scratch: q k v og | o chunks | gate | conv_w | norm_w |
+  // seq_lens | state
   size_t off[10];
   size_t at = 0;
-  for (int i = 0; i < 5; ++i) { off[i] = at; at = round_up(at + tens, 256); }
+  for (int i = 0; i < 4; ++i) { off[i] = at; at = round_up(at + tens, 256); }
+  off[4] = at; at = round_up(at + orows * row, 256);
   off[5] = at; at = round_up(at + gbytes, 256);
   off[6] = at; at = round_up(at + cw, 256);
   off[7] = at; at = round_up(at + nw, 256);
@@ -653,82 +681,97 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
   Scratch dev;
   if ((s = dev.alloc(at, st)) != GBLA_OK) return s;
   char *base = (char *)dev.ptr;
-  auto valid_rows = [&](int b) -> size_t {
-    long L = seq_lens ? seq_lens[b] : N;
-    return (size_t)(L < 0 ? 0 : (L > N ? N : L));
+  // rows [t0, t1) of batch row b of a [B, N, ...] host tensor into device slot i
+  auto h2d = [&](int i, const void *src, size_t stride, int b, size_t t0, size_t t1,
+                 cudaStream_t cs) {
+    if (t1 <= t0) return cudaSuccess;
+    const size_t o0 = ((size_t)b * N + t0) * stride;
+    return cudaMemcpyAsync(base + off[i] + o0, (const char *)src + o0, (t1 - t0) * stride,
+                           cudaMemcpyHostToDevice, cs);
   };
-  auto h2d = [&](int i, const void *src, size_t stride, int b) {  // rows t < L_b of row b
-    const size_t n = valid_rows(b) * stride;
-    if (n == 0) return cudaSuccess;
-    return cudaMemcpyAsync(base + off[i] + (size_t)b * N * stride,
-                           (const char *)src + (size_t)b * N * stride, n,
-                           cudaMemcpyHostToDevice, st);
+  // Streams: `stream` takes k, v, the gate and the weights, the state and the
+  // readouts; `in_st` takes q and out_gate after k, v and the gate (the copies
+  // share the host link, so they go in that order) while the state runs;
+  // `out_st` takes o out chunk by chunk while later chunks come in.
+  cudaStream_t in_st = nullptr, out_st = nullptr;
+  cudaEvent_t ev_kvg = nullptr, ev_in = nullptr, ev_out = nullptr, ev_done = nullptr;
+  auto cleanup = [&]() {
+    if (ev_kvg) cudaEventDestroy(ev_kvg);
+    if (ev_in) cudaEventDestroy(ev_in);
+    if (ev_out) cudaEventDestroy(ev_out);
+    if (ev_done) cudaEventDestroy(ev_done);
+    if (in_st) cudaStreamDestroy(in_st);
+    if (out_st) cudaStreamDestroy(out_st);
   };
+  if (cudaStreamCreateWithFlags(&in_st, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&out_st, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev_kvg, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev_in, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&ev_done, cudaEventDisableTiming) != cudaSuccess) {
+    const cudaError_t e = cudaGetLastError();
+    cleanup();
+    dev.release();
+    return from_cuda(e);
+  }
+  cudaError_t e = cudaSuccess;
   // 1. What the state needs (k, v, gate, weights, lengths), then the state.
-  for (int b = 0; b < B; ++b)
-    if (h2d(1, k, row, b) != cudaSuccess || h2d(2, v, row, b) != cudaSuccess ||
-        h2d(5, gate, grow, b) != cudaSuccess)
-      return GBLA_ERR_CUDA;
-  if (cudaMemcpyAsync(base + off[6], conv_w, cw, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-      cudaMemcpyAsync(base + off[7], norm_w, nw, cudaMemcpyHostToDevice, st) != cudaSuccess)
-    return GBLA_ERR_CUDA;
+  for (int b = 0; b < B && e == cudaSuccess; ++b) {
+    const size_t L = valid_rows(b);
+    if ((e = h2d(1, k, row, b, 0, L, st)) == cudaSuccess &&
+        (e = h2d(2, v, row, b, 0, L, st)) == cudaSuccess)
+      e = h2d(5, gate, grow, b, 0, L, st);
+  }
+  if (e == cudaSuccess &&
+      (e = cudaMemcpyAsync(base + off[6], conv_w, cw, cudaMemcpyHostToDevice, st)) == cudaSuccess)
+    e = cudaMemcpyAsync(base + off[7], norm_w, nw, cudaMemcpyHostToDevice, st);
   const int32_t *dsl = nullptr;
-  if (seq_lens) {
-    if (cudaMemcpyAsync(base + off[8], seq_lens, sizeof(int32_t) * B, cudaMemcpyHostToDevice,
-                        st) != cudaSuccess)
-      return GBLA_ERR_CUDA;
+  if (e == cudaSuccess && seq_lens) {
+    e = cudaMemcpyAsync(base + off[8], seq_lens, sizeof(int32_t) * B, cudaMemcpyHostToDevice, st);
     dsl = (const int32_t *)(base + off[8]);
   }
+  if (e == cudaSuccess && (e = cudaEventRecord(ev_kvg, st)) == cudaSuccess)
+    e = cudaStreamWaitEvent(in_st, ev_kvg, 0);
   p.seq_lens = dsl;
   float *state = (float *)(base + off[9]);
   const float *dcw = (const float *)(base + off[6]), *dnw = (const float *)(base + off[7]);
-  if ((s = run_state(p, tc, base + off[1], base + off[2], base + off[5], dcw, state, st)) !=
-      GBLA_OK)
-    return s;
-  // 2. The readout in up to 4 slices of batch rows: q and out_gate of a slice
-  // come in on `stream`, its o goes out on a second stream, so the copy-out of
-  // one slice runs while the next slice is copied in.
-  cudaStream_t out_st = nullptr;
-  cudaEvent_t ev = nullptr, ev_out = nullptr;
-  if (cudaStreamCreateWithFlags(&out_st, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&ev_out, cudaEventDisableTiming) != cudaSuccess) {
-    if (out_st) cudaStreamDestroy(out_st);
-    if (ev) cudaEventDestroy(ev);
-    return from_cuda(cudaGetLastError());
-  }
-  const int nseg = B < 4 ? B : 4;
-  const int per = (B + nseg - 1) / nseg;
-  cudaError_t e = cudaSuccess;
-  for (int b0 = 0; b0 < B && e == cudaSuccess && s == GBLA_OK; b0 += per) {
-    const int b1 = b0 + per < B ? b0 + per : B;
-    for (int b = b0; b < b1 && e == cudaSuccess; ++b) {
-      if ((e = h2d(0, q, row, b)) == cudaSuccess) e = h2d(3, out_gate, row, b);
-    }
-    if (e != cudaSuccess) break;
-    Problem ps{b1 - b0, H, N, D, dtype, dsl ? dsl + b0 : nullptr};
-    const size_t tb = (size_t)b0 * N * row;
-    s = run_readout(ps, tc, base + off[0] + tb, base + off[3] + tb, dcw, dnw,
-                    state + (size_t)b0 * H * F, base + off[4] + tb, st);
-    if (s != GBLA_OK) break;
-    if ((e = cudaEventRecord(ev, st)) != cudaSuccess ||
-        (e = cudaStreamWaitEvent(out_st, ev, 0)) != cudaSuccess)
+  if (e == cudaSuccess)
+    s = run_state(p, tc, base + off[1], base + off[2], base + off[5], dcw, state, st);
+  // 2. The readout chunk by chunk: its q and out_gate rows in on `in_st`, its
+  // readout on `stream` (after the state), its o out on `out_st`.
+  for (size_t c = 0; c < chunks.size() && e == cudaSuccess && s == GBLA_OK; ++c) {
+    const Chunk &ch = chunks[c];
+    const int h0 = ch.t0 < 3 ? ch.t0 : 3, n = ch.t1 - ch.t0 + h0;
+    if ((e = h2d(0, q, row, ch.b, ch.t0, ch.t1, in_st)) != cudaSuccess ||
+        (e = h2d(3, out_gate, row, ch.b, ch.t0, ch.t1, in_st)) != cudaSuccess ||
+        (e = cudaEventRecord(ev_in, in_st)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(st, ev_in, 0)) != cudaSuccess)
       break;
-    for (int b = b0; b < b1 && e == cudaSuccess; ++b) {
-      const size_t n = valid_rows(b) * row;
-      if (n)
-        e = cudaMemcpyAsync((char *)o + (size_t)b * N * row, base + off[4] + (size_t)b * N * row,
-                            n, cudaMemcpyDeviceToHost, out_st);
-    }
+    const size_t v0 = ((size_t)ch.b * N + (ch.t0 - h0)) * row;  // first row of the view
+    Problem pc{1, H, n, D, dtype, nullptr};  // every row of the view is valid
+    char *ov = base + off[4] + ch.obase * row;
+    if ((s = run_readout(pc, tc, base + off[0] + v0, base + off[3] + v0, dcw, dnw,
+                         state + (size_t)ch.b * H * F, ov, st)) != GBLA_OK)
+      break;
+    if ((e = cudaEventRecord(ev_out, st)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(out_st, ev_out, 0)) != cudaSuccess)
+      break;
+    e = cudaMemcpyAsync((char *)o + ((size_t)ch.b * N + ch.t0) * row, ov + (size_t)h0 * row,
+                        (size_t)(ch.t1 - ch.t0) * row, cudaMemcpyDeviceToHost, out_st);
   }
-  // the scratch is freed on `stream` only after the copies out have finished
-  if (cudaEventRecord(ev_out, out_st) != cudaSuccess || cudaStreamWaitEvent(st, ev_out, 0) != cudaSuccess)
-    e = e == cudaSuccess ? cudaGetLastError() : e;
+  // the scratch is freed on `stream` only after both side streams are done with it
+  const cudaError_t ej = [&]() {
+    cudaError_t x;
+    if ((x = cudaEventRecord(ev_done, in_st)) != cudaSuccess ||
+        (x = cudaStreamWaitEvent(st, ev_done, 0)) != cudaSuccess ||
+        (x = cudaEventRecord(ev_done, out_st)) != cudaSuccess)
+      return x;
+    return cudaStreamWaitEvent(st, ev_done, 0);
+  }();
+  if (e == cudaSuccess) e = ej;
   dev.release();
   const cudaError_t es2 = cudaStreamSynchronize(st);
-  cudaEventDestroy(ev);
-  cudaEventDestroy(ev_out);
-  cudaStreamDestroy(out_st);
+  cleanup();
   if (s != GBLA_OK) return s;
   if (e != cudaSuccess) return from_cuda(e);
   return from_cuda(es2);

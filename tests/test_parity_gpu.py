@@ -212,6 +212,24 @@ def test_host_entry_matches_device():
     assert torch.equal(out, y_dev.cpu())
 
 
+@pytest.mark.parametrize("dtype,D", [("bf16", 64), ("bf16", 128), ("fp32", 32)])
+def test_host_entry_chunks_match_device(dtype, D):
+    """gbla_forward_host reads out in chunks of 4096 tokens, each seeing the 3 rows
+    before it as conv history: lengths at, just past and just short of chunk edges
+    give gbla_forward's o bit for bit, and padded rows keep their sentinel."""
+    w = custom(B=4, H=2, N=9000, D=D, dtype=dtype, seed=16,
+               seq_lens=[9000, 4096, 4099, 8191])
+    inp = make_inputs(w, "cuda")
+    y_dev = _run(inp)
+    host = {k_: (v_.cpu().pin_memory() if v_ is not None else None) for k_, v_ in inp.items()}
+    out = torch.full_like(host["q"], SENTINEL).pin_memory()
+    gbla.forward_host(host["q"], host["k"], host["v"], host["gate"], host["out_gate"],
+                      host["conv_w"], host["norm_w"], host["seq_lens"], out=out)
+    assert torch.equal(out, y_dev.cpu())
+    for b, L in enumerate([9000, 4096, 4099, 8191]):
+        assert torch.equal(out[b, L:], torch.full_like(out[b, L:], SENTINEL))
+
+
 def test_empty_inputs_are_noops():
     for shape in [(0, 5, 2, 64), (2, 0, 2, 64), (2, 5, 0, 64)]:
         q = torch.empty(shape, dtype=torch.bfloat16, device="cuda")
