@@ -637,13 +637,14 @@ __global__ void __launch_bounds__(kSThreads, 1)
       // past a sequence end or for a missing head), half-stage maxima, then
       // for every stage the maximum over its segment.
       {
-        // The 32 slots tid + i kSProd of a warp are 32 consecutive tokens of one
-        // stage: lane i decodes the warp's stage of round i, and the rounds'
-        // (b, hg, stage, L) go round by shuffles, so the decodes (a search of
-        // the stage prefix and a length load when ragged) run side by side.
+        // For each i, the 32 slots tid + i kSProd of a warp are 32 consecutive
+        // tokens of one stage: lane i decodes the warp's stage for that i, and
+        // each stage's (b, hg, stage, L) reaches the other lanes by shuffle, so
+        // the decodes (a search of the stage prefix and a length load when
+        // ragged) run side by side.
         constexpr int NSL = kRangeTok / kSProd;
         static_assert(kSTok % 32 == 0 && kSProd % 32 == 0 && NSL <= 32,
-                      "a warp's 32 slots of a round lie in one stage");
+                      "a warp's 32 slots for one i lie in one stage");
         int db = 0, dhg = 0, dst = 0, dL = 0;
         if (lane < NSL && (tid & ~31) + lane * kSProd < nsr * kSTok) {
           const StageRef st = decode_stage(p, pre, sb + ((tid & ~31) + lane * kSProd) / kSTok);
