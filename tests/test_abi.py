@@ -127,3 +127,21 @@ def test_backward_from_state_validates_saved_state(lib):
         ptrs[i] = bad
         st = lib.gbla_backward_from_state(*ptrs, 1, 1, 4, 64, gbla.GBLA_BF16, None)
         assert st == gbla.GBLA_ERR_INVALID_ARG, (i, bad)
+
+
+def test_backward_saved_state_arguments_checked_on_host():
+    """The binding rejects a saved state without its statistics (or the reverse),
+    with an ablation, or of the wrong shape or dtype, before calling the library."""
+    import torch
+    q = torch.zeros((1, 8, 2, 64), dtype=torch.bfloat16)
+    g = torch.zeros((1, 8, 2), dtype=torch.bfloat16)
+    cw, nw = torch.zeros((3, 2, 64, 4)), torch.zeros((2, 64))
+    state, stats = torch.zeros((1, 2, 64 * 64 + 64)), torch.zeros((1, 2, 2))
+    args = (q, q, q, g, q, cw, nw, None, q)
+    for kw in (dict(state=state), dict(stats=stats),
+               dict(flags=gbla.FLAG_NO_GATE, state=state, stats=stats),
+               dict(state=state[:, :1], stats=stats),
+               dict(state=state.double(), stats=stats),
+               dict(state=state, stats=stats[..., :1])):
+        with pytest.raises(ValueError):
+            gbla.backward(*args, **kw)
