@@ -656,13 +656,17 @@ gbla_status gbla_forward_host(const void *q, const void *k, const void *v,
   };
   std::vector<Chunk> chunks;
   size_t orows = 0;
-  for (int b = 0; b < B; ++b) {
-    const int L = (int)valid_rows(b);
-    for (int t0 = 0; t0 < L; t0 += kHostChunk) {
-      const int t1 = t0 + kHostChunk < L ? t0 + kHostChunk : L;
-      chunks.push_back({b, t0, t1, orows});
-      orows += (size_t)(t1 - t0) + (size_t)(t0 < 3 ? t0 : 3);
+  try {  // no exception may leave this C entry point
+    for (int b = 0; b < B; ++b) {
+      const int L = (int)valid_rows(b);
+      for (int t0 = 0; t0 < L; t0 += kHostChunk) {
+        const int t1 = t0 + kHostChunk < L ? t0 + kHostChunk : L;
+        chunks.push_back({b, t0, t1, orows});
+        orows += (size_t)(t1 - t0) + (size_t)(t0 < 3 ? t0 : 3);
+      }
     }
+  } catch (...) {
+    return GBLA_ERR_ALLOC;
   }
   // Layout of the device scratch: q k v og | o chunks | gate | conv_w | norm_w |
   // seq_lens | state
